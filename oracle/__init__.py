@@ -1,0 +1,25 @@
+"""fp64 CPU oracle for Curvature-Conditioned Query (arxiv 2606.01294).
+
+TEST INFRASTRUCTURE ONLY: the test-suite, the smoke check and the CPU-baseline
+leg of the benchmark are the only callers.  The GPU library never imports,
+links or executes anything here, and nothing here imports the GPU library.
+
+The arithmetic lives in ``ccq_oracle.c`` (plain C, fp64, token by token);
+this module compiles it with gcc on first use and marshals numpy arrays.
+
+Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``):
+  forward(chunk=0)   recurrent CCQ-GLA / CCQ-GDN (Algorithm 2, Eq. clean/read)
+                     -- pinned by brute force, closed forms, invariants and the
+                     finite-difference Hessian identity.
+  forward(chunk>0)   chunkwise form (Algorithm 1, App. B) -- pinned by equality
+                     with the recurrent form.
+  Absolute outputs on the benchmark-shaped random inputs are pinned only
+  through the above: the paper prints no worked numerical example.
+"""
+from .ccq_oracle import (  # noqa: F401
+    build_oracle,
+    forward,
+    decode_step,
+    GLA,
+    GDN,
+)

@@ -1,0 +1,408 @@
+/*
+ * ccq_oracle.c -- fp64 CPU oracle for Curvature-Conditioned Query (CCQ).
+ *
+ * TEST INFRASTRUCTURE ONLY. This file is the plain, slow, obviously correct
+ * statement of what the CCQ hot path computes. Only the test-suite, the smoke
+ * check and the CPU-baseline leg of the benchmark may load it. The CUDA
+ * library never links, includes or calls anything in this directory, and
+ * this file includes nothing from the CUDA library.
+ *
+ * What it computes (arxiv 2606.01294):
+ *   - running key statistics C_sum = sum_j kbar_j kbar_j^T and m_sum = sum_j kbar_j
+ *     with the length normalisation 1/t (Sec. 3.2 "Idea 1"; App. A.2, Eq. hess);
+ *   - Sigma_t = C_sum/t - (m_sum/t)(m_sum/t)^T, the centred sample covariance
+ *     (App. A.2), or C_sum/t for the uncentred variant (App. D ablation);
+ *   - the cleaned query q_clean = qbar - lambda_t Sigma_t qbar (Eq. clean,
+ *     Algorithm 2), applied to the l2-normalised query (Algorithms 1 and 2);
+ *   - the backbone write S_t = Update(S_{t-1}; kbar_t, v_t, ...) and the read
+ *     o_t = scale * S_t q_clean (Eq. read).  The paper treats the backbone as a
+ *     black box (Sec. 2.2); the two write rules are GLA's per-key-dimension
+ *     forget gate and Gated DeltaNet's gated delta rule, as those methods
+ *     define them and as Sec. 2.2 summarises them.
+ *
+ * State orientation: the paper's S is d_v x d_k.  Here every state is stored
+ * as its transpose Hs[dk][dv] (row = key dimension), i.e. Hs = S^T.
+ *
+ * Readings of the paper that this file fixes (where the paper is silent):
+ *   - zero-norm rows: l2-normalising an all-zero row yields the zero row
+ *     (the paper gives no epsilon);
+ *   - the position counter t is inclusive of the current token (sums over
+ *     j <= t, Sec. 3.2) and continues from the caller's t0;
+ *   - the read uses the state after token t has been written (Eq. read);
+ *   - scale multiplies the read only.
+ *
+ * Every routine is fp64.  Work over (batch, head) pairs is spread over
+ * POSIX threads; each pair is computed by exactly one thread in a fixed
+ * order, so results do not depend on the thread count.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define CCQ_ORACLE_GLA 0
+#define CCQ_ORACLE_GDN 1
+
+typedef struct {
+    int backbone, B, T, H, Dk, Dv, l2norm, centered, chunk;
+    double scale;
+    const double *q, *k, *v, *gate, *beta, *lam;
+    const double *S0, *C0, *m0;
+    const int64_t *t0;
+    double *o, *ST, *CT, *mT, *qc_out;
+    int64_t *tT;
+    /* work queue over (b, h) pairs */
+    int next;
+    pthread_mutex_t mu;
+} job_t;
+
+/* l2-normalise x[0..n) into y; the zero row maps to the zero row. */
+static void l2_normalise(const double *x, double *y, int n, int enabled) {
+    if (!enabled) {
+        memcpy(y, x, sizeof(double) * (size_t)n);
+        return;
+    }
+    double s = 0.0;
+    for (int i = 0; i < n; ++i) s += x[i] * x[i];
+    double r = s > 0.0 ? 1.0 / sqrt(s) : 0.0;
+    for (int i = 0; i < n; ++i) y[i] = x[i] * r;
+}
+
+static size_t row(const job_t *J, int b, int t, int h) {
+    return ((size_t)b * J->T + t) * J->H + h;
+}
+
+/* Load the initial states of pair (b, h): zero when the pointer is NULL. */
+static void load_states(const job_t *J, int b, int h, double *Hs, double *Cs,
+                        double *ms, int64_t *t) {
+    const int Dk = J->Dk, Dv = J->Dv;
+    const size_t bh = (size_t)b * J->H + h;
+    if (J->S0) memcpy(Hs, J->S0 + bh * Dk * Dv, sizeof(double) * Dk * Dv);
+    else memset(Hs, 0, sizeof(double) * Dk * Dv);
+    if (J->C0) memcpy(Cs, J->C0 + bh * Dk * Dk, sizeof(double) * Dk * Dk);
+    else memset(Cs, 0, sizeof(double) * Dk * Dk);
+    if (J->m0) memcpy(ms, J->m0 + bh * Dk, sizeof(double) * Dk);
+    else memset(ms, 0, sizeof(double) * Dk);
+    *t = J->t0 ? J->t0[b] : 0;
+}
+
+static void store_states(const job_t *J, int b, int h, const double *Hs,
+                         const double *Cs, const double *ms, int64_t t) {
+    const int Dk = J->Dk, Dv = J->Dv;
+    const size_t bh = (size_t)b * J->H + h;
+    if (J->ST) memcpy(J->ST + bh * Dk * Dv, Hs, sizeof(double) * Dk * Dv);
+    if (J->CT) memcpy(J->CT + bh * Dk * Dk, Cs, sizeof(double) * Dk * Dk);
+    if (J->mT) memcpy(J->mT + bh * Dk, ms, sizeof(double) * Dk);
+    if (J->tT && h == 0) J->tT[b] = t;
+}
+
+/*
+ * Sigma_t qbar from the running sums (App. A.2): C_sum qbar / t minus the
+ * mean term m (m^T qbar) / t^2; the mean term is dropped when uncentred.
+ */
+static void sigma_times(const double *Cs, const double *ms, const double *qb,
+                        int Dk, double t, int centered, double *out) {
+    double mq = 0.0;
+    for (int j = 0; j < Dk; ++j) mq += ms[j] * qb[j];
+    for (int i = 0; i < Dk; ++i) {
+        double acc = 0.0;
+        for (int j = 0; j < Dk; ++j) acc += Cs[(size_t)i * Dk + j] * qb[j];
+        out[i] = acc / t;
+        if (centered) out[i] -= ms[i] * mq / (t * t);
+    }
+}
+
+/*
+ * One (b, h) pair, token by token: Algorithm 2 with the statistics kept as
+ * unnormalised sums and divided by t on use (the same Sigma_t, App. A.2).
+ */
+static void recurrent_pair(const job_t *J, int b, int h) {
+    const int Dk = J->Dk, Dv = J->Dv;
+    double *Hs = malloc(sizeof(double) * Dk * Dv);
+    double *Cs = malloc(sizeof(double) * Dk * Dk);
+    double *ms = malloc(sizeof(double) * Dk);
+    double *qb = malloc(sizeof(double) * Dk), *kb = malloc(sizeof(double) * Dk);
+    double *sq = malloc(sizeof(double) * Dk), *qc = malloc(sizeof(double) * Dk);
+    double *kS = malloc(sizeof(double) * Dv);
+    int64_t t;
+    load_states(J, b, h, Hs, Cs, ms, &t);
+
+    for (int tl = 0; tl < J->T; ++tl) {
+        const size_t r = row(J, b, tl, h);
+        const double *qr = J->q + r * Dk, *kr = J->k + r * Dk, *vr = J->v + r * Dv;
+        /* Algorithm 2: normalise query and key */
+        l2_normalise(qr, qb, Dk, J->l2norm);
+        l2_normalise(kr, kb, Dk, J->l2norm);
+        /* key statistics include the current token (sums over j <= t) */
+        t += 1;
+        for (int i = 0; i < Dk; ++i) {
+            for (int j = 0; j < Dk; ++j) Cs[(size_t)i * Dk + j] += kb[i] * kb[j];
+            ms[i] += kb[i];
+        }
+        /* Eq. clean: q_clean = qbar - lambda Sigma_t qbar */
+        const double lam = J->lam[r];
+        sigma_times(Cs, ms, qb, Dk, (double)t, J->centered, sq);
+        for (int i = 0; i < Dk; ++i) qc[i] = qb[i] - lam * sq[i];
+        if (J->qc_out) memcpy(J->qc_out + r * Dk, qc, sizeof(double) * Dk);
+
+        /* backbone write with the normalised key */
+        if (J->backbone == CCQ_ORACLE_GLA) {
+            /* GLA: S_t = S_{t-1} Diag(alpha_t) + v_t kbar_t^T, alpha = exp(gk) */
+            const double *gr = J->gate + r * Dk;
+            for (int i = 0; i < Dk; ++i) {
+                const double a = exp(gr[i]);
+                for (int j = 0; j < Dv; ++j)
+                    Hs[(size_t)i * Dv + j] = a * Hs[(size_t)i * Dv + j] + kb[i] * vr[j];
+            }
+        } else {
+            /* Gated DeltaNet: S_t = alpha_t S_{t-1} (I - beta_t k k^T) + beta_t v k^T */
+            const double a = exp(J->gate[r]), be = J->beta[r];
+            for (int j = 0; j < Dv; ++j) {
+                double acc = 0.0;
+                for (int i = 0; i < Dk; ++i) acc += kb[i] * Hs[(size_t)i * Dv + j];
+                kS[j] = acc;
+            }
+            for (int i = 0; i < Dk; ++i)
+                for (int j = 0; j < Dv; ++j)
+                    Hs[(size_t)i * Dv + j] =
+                        a * (Hs[(size_t)i * Dv + j] - be * kb[i] * kS[j]) + be * kb[i] * vr[j];
+        }
+        /* Eq. read: o_t = S_t q_clean (times the read scale) */
+        double *orow = J->o + r * Dv;
+        for (int j = 0; j < Dv; ++j) {
+            double acc = 0.0;
+            for (int i = 0; i < Dk; ++i) acc += Hs[(size_t)i * Dv + j] * qc[i];
+            orow[j] = J->scale * acc;
+        }
+    }
+    store_states(J, b, h, Hs, Cs, ms, t);
+    free(Hs); free(Cs); free(ms); free(qb); free(kb); free(sq); free(qc); free(kS);
+}
+
+/*
+ * One (b, h) pair in the chunkwise form of Algorithm 1 (App. B), with the
+ * backbone's own chunk update.  This is a second statement of the same
+ * computation used to check that the chunkwise re-association is exact; it
+ * is not what the tests compare GPU results against.
+ */
+static void chunkwise_pair(const job_t *J, int b, int h) {
+    const int Dk = J->Dk, Dv = J->Dv, C = J->chunk;
+    double *Hs = malloc(sizeof(double) * Dk * Dv);
+    double *SK = malloc(sizeof(double) * Dk * Dk);
+    double *M = malloc(sizeof(double) * Dk);
+    double *Qb = malloc(sizeof(double) * C * Dk), *Kb = malloc(sizeof(double) * C * Dk);
+    double *P = malloc(sizeof(double) * C * Dk), *CumK = malloc(sizeof(double) * C * Dk);
+    double *Qc = malloc(sizeof(double) * C * Dk);
+    double *G = malloc(sizeof(double) * C * Dk); /* GLA: in-chunk cumulative log gate */
+    double *gc = malloc(sizeof(double) * C);     /* GDN: in-chunk cumulative log decay */
+    double *U = malloc(sizeof(double) * C * Dv); /* GDN: pseudo-values u_j */
+    double *Hn = malloc(sizeof(double) * Dk * Dv);
+    int64_t t;
+    load_states(J, b, h, Hs, SK, M, &t);
+
+    for (int c0 = 0; c0 < J->T; c0 += C) {
+        const int n = (J->T - c0 < C) ? J->T - c0 : C;
+        /* Algorithm 1: normalised queries and keys of the chunk */
+        for (int i = 0; i < n; ++i) {
+            const size_t r = row(J, b, c0 + i, h);
+            l2_normalise(J->q + r * Dk, Qb + (size_t)i * Dk, Dk, J->l2norm);
+            l2_normalise(J->k + r * Dk, Kb + (size_t)i * Dk, Dk, J->l2norm);
+        }
+        for (int i = 0; i < n; ++i) {
+            const double *qi = Qb + (size_t)i * Dk;
+            /* P_prev = S^K_r qbar_i (S^K symmetric) */
+            for (int a = 0; a < Dk; ++a) {
+                double acc = 0.0;
+                for (int e = 0; e < Dk; ++e) acc += SK[(size_t)a * Dk + e] * qi[e];
+                P[(size_t)i * Dk + a] = acc;
+            }
+            /* P_intra = sum_{j <= i} (qbar_i . kbar_j) kbar_j (mask includes the diagonal) */
+            for (int j = 0; j <= i; ++j) {
+                const double *kj = Kb + (size_t)j * Dk;
+                double s = 0.0;
+                for (int e = 0; e < Dk; ++e) s += qi[e] * kj[e];
+                for (int a = 0; a < Dk; ++a) P[(size_t)i * Dk + a] += s * kj[a];
+            }
+            /* CumK = M_r + cumsum(kbar) */
+            for (int a = 0; a < Dk; ++a)
+                CumK[(size_t)i * Dk + a] =
+                    (i == 0 ? M[a] : CumK[(size_t)(i - 1) * Dk + a]) + Kb[(size_t)i * Dk + a];
+            /* D = 1/(t+i); MeanCorr_i = D^2 CumK_i (CumK_i . qbar_i), read row by row */
+            const double tpos = (double)(t + i + 1);
+            double cq = 0.0;
+            for (int a = 0; a < Dk; ++a) cq += CumK[(size_t)i * Dk + a] * qi[a];
+            const double lam = J->lam[row(J, b, c0 + i, h)];
+            for (int a = 0; a < Dk; ++a) {
+                double corr = P[(size_t)i * Dk + a] / tpos;
+                if (J->centered) corr -= CumK[(size_t)i * Dk + a] * cq / (tpos * tpos);
+                Qc[(size_t)i * Dk + a] = qi[a] - lam * corr;
+            }
+            if (J->qc_out)
+                memcpy(J->qc_out + row(J, b, c0 + i, h) * Dk, Qc + (size_t)i * Dk,
+                       sizeof(double) * Dk);
+        }
+
+        if (J->backbone == CCQ_ORACLE_GLA) {
+            /* GLA chunk update: G_i = sum_{s <= i} gk_s within the chunk */
+            for (int i = 0; i < n; ++i) {
+                const double *gr = J->gate + row(J, b, c0 + i, h) * Dk;
+                for (int a = 0; a < Dk; ++a)
+                    G[(size_t)i * Dk + a] = (i ? G[(size_t)(i - 1) * Dk + a] : 0.0) + gr[a];
+            }
+            for (int i = 0; i < n; ++i) {
+                double *orow = J->o + row(J, b, c0 + i, h) * Dv;
+                const double *qi = Qc + (size_t)i * Dk, *Gi = G + (size_t)i * Dk;
+                for (int e = 0; e < Dv; ++e) {
+                    /* inter-chunk: (q_clean_i * exp(G_i)) S_r */
+                    double acc = 0.0;
+                    for (int a = 0; a < Dk; ++a)
+                        acc += qi[a] * exp(Gi[a]) * Hs[(size_t)a * Dv + e];
+                    orow[e] = acc;
+                }
+                /* intra-chunk: sum_{j <= i} (q_clean_i * exp(G_i - G_j) . kbar_j) v_j */
+                for (int j = 0; j <= i; ++j) {
+                    const double *Gj = G + (size_t)j * Dk, *kj = Kb + (size_t)j * Dk;
+                    double s = 0.0;
+                    for (int a = 0; a < Dk; ++a) s += qi[a] * exp(Gi[a] - Gj[a]) * kj[a];
+                    const double *vj = J->v + row(J, b, c0 + j, h) * Dv;
+                    for (int e = 0; e < Dv; ++e) orow[e] += s * vj[e];
+                }
+                for (int e = 0; e < Dv; ++e) orow[e] *= J->scale;
+            }
+            /* S_{r+1} = Diag(exp(G_n)) S_r + sum_j (kbar_j * exp(G_n - G_j)) v_j^T */
+            const double *Gn = G + (size_t)(n - 1) * Dk;
+            for (int a = 0; a < Dk; ++a)
+                for (int e = 0; e < Dv; ++e) {
+                    double acc = exp(Gn[a]) * Hs[(size_t)a * Dv + e];
+                    for (int j = 0; j < n; ++j)
+                        acc += Kb[(size_t)j * Dk + a] * exp(Gn[a] - G[(size_t)j * Dk + a]) *
+                               J->v[row(J, b, c0 + j, h) * Dv + e];
+                    Hn[(size_t)a * Dv + e] = acc;
+                }
+            memcpy(Hs, Hn, sizeof(double) * Dk * Dv);
+        } else {
+            /* Gated DeltaNet chunk update.  With H = S^T and gamma_i the in-chunk
+             * decay product, the per-token write is H_i = alpha_i H_{i-1} + kbar_i u_i^T
+             * with u_i = beta_i (v_i - alpha_i H_{i-1}^T kbar_i).  Unrolling gives the
+             * unit lower-triangular system
+             *   u_i + beta_i sum_{j<i} (gamma_i/gamma_j)(kbar_i . kbar_j) u_j
+             *       = beta_i v_i - beta_i gamma_i H_0^T kbar_i,
+             * solved here by forward substitution (the WY/UT form inverts the same
+             * matrix). */
+            for (int i = 0; i < n; ++i)
+                gc[i] = (i ? gc[i - 1] : 0.0) + J->gate[row(J, b, c0 + i, h)];
+            for (int i = 0; i < n; ++i) {
+                const double be = J->beta[row(J, b, c0 + i, h)];
+                const double *ki = Kb + (size_t)i * Dk;
+                const double *vi = J->v + row(J, b, c0 + i, h) * Dv;
+                double *ui = U + (size_t)i * Dv;
+                for (int e = 0; e < Dv; ++e) {
+                    double hk = 0.0;
+                    for (int a = 0; a < Dk; ++a) hk += Hs[(size_t)a * Dv + e] * ki[a];
+                    ui[e] = be * vi[e] - be * exp(gc[i]) * hk;
+                }
+                for (int j = 0; j < i; ++j) {
+                    const double *kj = Kb + (size_t)j * Dk;
+                    double s = 0.0;
+                    for (int a = 0; a < Dk; ++a) s += ki[a] * kj[a];
+                    const double Aij = be * exp(gc[i] - gc[j]) * s;
+                    for (int e = 0; e < Dv; ++e) ui[e] -= Aij * U[(size_t)j * Dv + e];
+                }
+            }
+            for (int i = 0; i < n; ++i) {
+                double *orow = J->o + row(J, b, c0 + i, h) * Dv;
+                const double *qi = Qc + (size_t)i * Dk;
+                for (int e = 0; e < Dv; ++e) {
+                    double acc = 0.0;
+                    for (int a = 0; a < Dk; ++a) acc += qi[a] * Hs[(size_t)a * Dv + e];
+                    orow[e] = exp(gc[i]) * acc;
+                }
+                for (int j = 0; j <= i; ++j) {
+                    const double *kj = Kb + (size_t)j * Dk;
+                    double s = 0.0;
+                    for (int a = 0; a < Dk; ++a) s += qi[a] * kj[a];
+                    s *= exp(gc[i] - gc[j]);
+                    for (int e = 0; e < Dv; ++e) orow[e] += s * U[(size_t)j * Dv + e];
+                }
+                for (int e = 0; e < Dv; ++e) orow[e] *= J->scale;
+            }
+            for (int a = 0; a < Dk; ++a)
+                for (int e = 0; e < Dv; ++e) {
+                    double acc = exp(gc[n - 1]) * Hs[(size_t)a * Dv + e];
+                    for (int j = 0; j < n; ++j)
+                        acc += exp(gc[n - 1] - gc[j]) * Kb[(size_t)j * Dk + a] * U[(size_t)j * Dv + e];
+                    Hn[(size_t)a * Dv + e] = acc;
+                }
+            memcpy(Hs, Hn, sizeof(double) * Dk * Dv);
+        }
+        /* S^K_{r+1} = S^K_r + Kbar^T Kbar ; M_{r+1} = M_r + sum_j kbar_j ; t += n */
+        for (int j = 0; j < n; ++j) {
+            const double *kj = Kb + (size_t)j * Dk;
+            for (int a = 0; a < Dk; ++a) {
+                for (int e = 0; e < Dk; ++e) SK[(size_t)a * Dk + e] += kj[a] * kj[e];
+                M[a] += kj[a];
+            }
+        }
+        t += n;
+    }
+    store_states(J, b, h, Hs, SK, M, t);
+    free(Hs); free(SK); free(M); free(Qb); free(Kb); free(P); free(CumK); free(Qc);
+    free(G); free(gc); free(U); free(Hn);
+}
+
+static void *worker(void *arg) {
+    job_t *J = (job_t *)arg;
+    for (;;) {
+        pthread_mutex_lock(&J->mu);
+        const int w = J->next++;
+        pthread_mutex_unlock(&J->mu);
+        if (w >= J->B * J->H) break;
+        const int b = w / J->H, h = w % J->H;
+        if (J->chunk > 0) chunkwise_pair(J, b, h);
+        else recurrent_pair(J, b, h);
+    }
+    return NULL;
+}
+
+/*
+ * Forward over a [B, T, H, D] sequence batch (D contiguous).
+ *   backbone   0 = GLA (gate: log alpha [B,T,H,Dk]), 1 = Gated DeltaNet
+ *              (gate: log alpha [B,T,H], beta [B,T,H]).
+ *   lam        lambda_t [B,T,H].
+ *   S0/C0/m0   initial S^T [B,H,Dk,Dv], C_sum [B,H,Dk,Dk], m_sum [B,H,Dk]; NULL = 0.
+ *   t0         initial position per batch row [B]; NULL = 0.
+ *   o          [B,T,H,Dv].  ST/CT/mT/tT final states (each may be NULL).
+ *   qc_out     optional [B,T,H,Dk] cleaned queries (NULL = not written).
+ *   chunk      0 = token-by-token recurrence; >0 = chunkwise form, chunk size.
+ *   nthreads   worker threads (>= 1).
+ * Returns 0, or -1 on a bad argument.
+ */
+int ccq_oracle_forward(int backbone, int B, int T, int H, int Dk, int Dv,
+                       const double *q, const double *k, const double *v,
+                       const double *gate, const double *beta, const double *lam,
+                       const double *S0, const double *C0, const double *m0,
+                       const int64_t *t0, double *o, double *ST, double *CT,
+                       double *mT, int64_t *tT, double *qc_out, int l2norm,
+                       int centered, double scale, int chunk, int nthreads) {
+    if (B < 0 || T < 0 || H < 0 || Dk <= 0 || Dv <= 0 || chunk < 0 || nthreads < 1) return -1;
+    if (!q || !k || !v || !gate || !lam || !o) return -1;
+    if (backbone == CCQ_ORACLE_GDN && !beta) return -1;
+    if (backbone != CCQ_ORACLE_GLA && backbone != CCQ_ORACLE_GDN) return -1;
+    job_t J;
+    memset(&J, 0, sizeof J);
+    J.backbone = backbone; J.B = B; J.T = T; J.H = H; J.Dk = Dk; J.Dv = Dv;
+    J.l2norm = l2norm; J.centered = centered; J.chunk = chunk; J.scale = scale;
+    J.q = q; J.k = k; J.v = v; J.gate = gate; J.beta = beta; J.lam = lam;
+    J.S0 = S0; J.C0 = C0; J.m0 = m0; J.t0 = t0;
+    J.o = o; J.ST = ST; J.CT = CT; J.mT = mT; J.tT = tT; J.qc_out = qc_out;
+    pthread_mutex_init(&J.mu, NULL);
+    if (nthreads > B * H) nthreads = B * H > 0 ? B * H : 1;
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int i = 0; i < nthreads; ++i) pthread_create(&th[i], NULL, worker, &J);
+    for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
+    free(th);
+    pthread_mutex_destroy(&J.mu);
+    /* T == 0: the per-pair loops still copy the initial states through */
+    return 0;
+}

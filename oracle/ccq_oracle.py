@@ -1,0 +1,141 @@
+"""ctypes marshalling for the fp64 C oracle (test infrastructure only).
+
+Compiles ``ccq_oracle.c`` with gcc into ``_ccq_oracle.so`` beside it the first
+time it is needed (or when the source is newer), then calls
+``ccq_oracle_forward``.  All arrays are converted to contiguous float64 (or
+int64 for positions); inputs that were rounded to bf16/fp32 are passed as
+their exactly upcast values.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+GLA = 0
+GDN = 1
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "ccq_oracle.c")
+_LIB_PATH = os.path.join(_HERE, "_ccq_oracle.so")
+_lib = None
+_lock = threading.Lock()
+
+
+def build_oracle(force: bool = False) -> str:
+    """Compile the oracle shared library with gcc; return its path."""
+    stale = (not os.path.exists(_LIB_PATH)) or (
+        os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC))
+    if force or stale:
+        tmp = _LIB_PATH + f".{os.getpid()}.tmp"
+        subprocess.check_call(
+            ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-pthread", _SRC,
+             "-o", tmp, "-lm"])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def load_library(path: str):
+    """Open a compiled oracle library at ``path`` and declare its signature."""
+    lib = ctypes.CDLL(path)
+    dp = ctypes.POINTER(ctypes.c_double)
+    ip = ctypes.POINTER(ctypes.c_int64)
+    lib.ccq_oracle_forward.argtypes = (
+        [ctypes.c_int] * 6 + [dp] * 9 + [ip] + [dp] * 4 + [ip] + [dp]
+        + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int,
+           ctypes.c_int])
+    lib.ccq_oracle_forward.restype = ctypes.c_int
+    return lib
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = load_library(build_oracle())
+    return _lib
+
+
+def _f64(x):
+    if x is None:
+        return None
+    if hasattr(x, "detach"):  # torch tensor
+        x = x.detach().to("cpu").double().numpy()
+    return np.ascontiguousarray(x, dtype=np.float64)
+
+
+def _i64(x):
+    if x is None:
+        return None
+    if hasattr(x, "detach"):
+        x = x.detach().to("cpu").numpy()
+    return np.ascontiguousarray(x, dtype=np.int64)
+
+
+def _ptr(a, kind=ctypes.c_double):
+    if a is None:
+        return None
+    return a.ctypes.data_as(ctypes.POINTER(kind))
+
+
+def forward(backbone, q, k, v, gate, lam, beta=None, S0=None, C0=None, m0=None,
+            t0=None, *, l2norm=True, centered=True, scale=None, chunk=0,
+            nthreads=None, want_qclean=False, lib=None):
+    """Oracle CCQ forward.
+
+    Shapes: q, k [B,T,H,Dk]; v [B,T,H,Dv]; gate [B,T,H,Dk] (GLA log-forget)
+    or [B,T,H] (GDN log-decay); beta [B,T,H] (GDN); lam [B,T,H];
+    S0 [B,H,Dk,Dv] (the transpose of the paper's d_v x d_k state);
+    C0 [B,H,Dk,Dk]; m0 [B,H,Dk]; t0 [B].
+    Returns dict with o [B,T,H,Dv], S [B,H,Dk,Dv], C [B,H,Dk,Dk], m [B,H,Dk],
+    t [B] and (optionally) qclean [B,T,H,Dk]; all float64 / int64.
+    """
+    lib = lib or _load()
+    q, k, v, gate, lam = map(_f64, (q, k, v, gate, lam))
+    beta, S0, C0, m0 = map(_f64, (beta, S0, C0, m0))
+    t0 = _i64(t0)
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    if scale is None:
+        scale = Dk ** -0.5
+    if nthreads is None:
+        nthreads = os.cpu_count() or 1
+    o = np.zeros((B, T, H, Dv))
+    S = np.zeros((B, H, Dk, Dv))
+    C = np.zeros((B, H, Dk, Dk))
+    m = np.zeros((B, H, Dk))
+    t = np.zeros((B,), dtype=np.int64)
+    qc = np.zeros((B, T, H, Dk)) if want_qclean else None
+    rc = lib.ccq_oracle_forward(
+        int(backbone), B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(gate),
+        _ptr(beta), _ptr(lam), _ptr(S0), _ptr(C0), _ptr(m0),
+        _ptr(t0, ctypes.c_int64), _ptr(o), _ptr(S), _ptr(C), _ptr(m),
+        _ptr(t, ctypes.c_int64), _ptr(qc), int(bool(l2norm)),
+        int(bool(centered)), float(scale), int(chunk), int(nthreads))
+    if rc != 0:
+        raise ValueError("ccq_oracle_forward rejected its arguments")
+    out = {"o": o, "S": S, "C": C, "m": m, "t": t}
+    if want_qclean:
+        out["qclean"] = qc
+    return out
+
+
+def decode_step(backbone, q, k, v, gate, lam, S, C, m, t, beta=None, *,
+                l2norm=True, centered=True, scale=None, nthreads=None):
+    """One recurrent token (Algorithm 2) for a batch of states.
+
+    q, k [B,H,Dk]; v [B,H,Dv]; gate [B,H,Dk] (GLA) or [B,H] (GDN); lam, beta
+    [B,H]; S [B,H,Dk,Dv]; C [B,H,Dk,Dk]; m [B,H,Dk]; t [B].
+    Returns o [B,H,Dv] and the updated (S, C, m, t).
+    """
+    q, k, v, gate, lam, beta = map(_f64, (q, k, v, gate, lam, beta))
+    add_t = lambda a: None if a is None else a[:, None]  # noqa: E731
+    res = forward(backbone, add_t(q), add_t(k), add_t(v), add_t(gate),
+                  add_t(lam), beta=add_t(beta), S0=S, C0=C, m0=m, t0=t,
+                  l2norm=l2norm, centered=centered, scale=scale,
+                  nthreads=nthreads)
+    return {"o": res["o"][:, 0], "S": res["S"], "C": res["C"], "m": res["m"],
+            "t": res["t"]}

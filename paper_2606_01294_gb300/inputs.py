@@ -1,0 +1,125 @@
+"""Seeded synthetic inputs shaped like the paper's CCQ workloads.
+
+This module only draws random tensors; it holds none of the CCQ arithmetic.
+Both the GPU tests / benchmark and the CPU oracle consume what it returns.
+
+Recipe (all draws fp32 from a CPU ``torch.Generator`` seeded with ``seed``, in
+the order q, k, v, gate, beta, lambda, then cast to the requested dtype):
+  q, k, v        ~ N(0, 1), layout [B, T, H, D] with D contiguous;
+                   k (and for Gated DeltaNet also q) l2-normalised per head row
+                   before the cast, as the workload description specifies.
+  GLA gate       log-forget per key dim: logsigmoid(N(0,1)) / 16, [B,T,H,Dk].
+  GDN gate       log decay per token/head: -softplus(N(0,1)) (alpha =
+                 exp(-softplus)), [B,T,H] fp32; beta = sigmoid(N(0,1)) fp32.
+  lambda         [B,T,H] fp32 in (0, 1):
+                   "init"     0.01 everywhere (W_lambda = 0, sigma(b) = 0.01, App. D);
+                   "trained"  sigmoid(N(logit(0.29), 0.5)) (App. E gate statistics);
+                   "high"     0.9 (App. A.3: stable as lambda approaches 1);
+                   a float    that constant.
+  keys           "iso" (above) or "structured": k = normalise(m0 + U z + 0.25 eps),
+                 U a fixed random orthonormal d x 16 basis, z ~ N(0, I_16),
+                 eps ~ N(0, I_d), m0 a fixed random vector of norm 0.5 -- a
+                 low-rank key spread with a non-zero mean, so Sigma_t is large and
+                 the mean term matters.
+"""
+from __future__ import annotations
+
+import math
+
+import torch
+import torch.nn.functional as F
+
+GLA = 0
+GDN = 1
+
+
+def _normalise_rows(x: torch.Tensor) -> torch.Tensor:
+    return x / x.norm(dim=-1, keepdim=True).clamp_min(1e-30)
+
+
+def _structured_keys(gen, B, T, H, Dk, rank=16):
+    basis_gen = torch.Generator().manual_seed(7919)
+    U, _ = torch.linalg.qr(torch.randn(Dk, min(rank, Dk), generator=basis_gen))
+    m0 = torch.randn(Dk, generator=basis_gen)
+    m0 = 0.5 * m0 / m0.norm()
+    z = torch.randn(B, T, H, U.shape[1], generator=gen)
+    eps = torch.randn(B, T, H, Dk, generator=gen)
+    return m0 + z @ U.T + 0.25 * eps
+
+
+def _lambda(gen, B, T, H, lam):
+    if isinstance(lam, (int, float)):
+        return torch.full((B, T, H), float(lam))
+    if lam == "init":
+        return torch.full((B, T, H), 0.01)
+    if lam == "trained":
+        logit = math.log(0.29 / 0.71)
+        return torch.sigmoid(logit + 0.5 * torch.randn(B, T, H, generator=gen))
+    if lam == "high":
+        return torch.full((B, T, H), 0.9)
+    raise ValueError(f"unknown lambda regime {lam!r}")
+
+
+def make_inputs(backbone: int, B: int, T: int, H: int, Dk: int, Dv: int, *,
+                dtype=torch.bfloat16, gate_dtype=None, seed: int = 1234,
+                lam="init", keys: str = "iso") -> dict:
+    """Draw one CCQ forward problem on the CPU.
+
+    Returns a dict of CPU tensors: q, k [B,T,H,Dk] and v [B,T,H,Dv] in
+    ``dtype``; ``gate`` ([B,T,H,Dk] in ``gate_dtype`` (default ``dtype``) for
+    GLA, [B,T,H] fp32 for GDN); ``beta`` ([B,T,H] fp32, GDN only, else None);
+    ``lam`` [B,T,H] fp32.
+    """
+    gen = torch.Generator().manual_seed(seed)
+    q = torch.randn(B, T, H, Dk, generator=gen)
+    if keys == "iso":
+        k = torch.randn(B, T, H, Dk, generator=gen)
+    elif keys == "structured":
+        k = _structured_keys(gen, B, T, H, Dk)
+    else:
+        raise ValueError(f"unknown key distribution {keys!r}")
+    k = _normalise_rows(k)
+    if backbone == GDN:
+        q = _normalise_rows(q)
+    v = torch.randn(B, T, H, Dv, generator=gen)
+    if backbone == GLA:
+        gate = F.logsigmoid(torch.randn(B, T, H, Dk, generator=gen)) / 16
+        gate = gate.to(gate_dtype or dtype)
+        beta = None
+    else:
+        gate = -F.softplus(torch.randn(B, T, H, generator=gen))
+        beta = torch.sigmoid(torch.randn(B, T, H, generator=gen))
+    lam_t = _lambda(gen, B, T, H, lam)
+    return {"q": q.to(dtype), "k": k.to(dtype), "v": v.to(dtype), "gate": gate,
+            "beta": beta, "lam": lam_t.float()}
+
+
+def make_decode_inputs(backbone: int, B: int, H: int, Dk: int, Dv: int, *,
+                       dtype=torch.bfloat16, seed: int = 4321, lam="init",
+                       prefix: int = 64) -> dict:
+    """Draw a decode problem: a ``prefix``-token history (a [B,prefix,H,*]
+    forward problem whose final states seed the decode state) plus one new
+    token per (batch, head) with the same value distributions."""
+    hist = make_inputs(backbone, B, prefix + 1, H, Dk, Dv, dtype=dtype,
+                       seed=seed, lam=lam)
+    pre = {n: (None if x is None else x[:, :prefix].contiguous())
+           for n, x in hist.items()}
+    tok = {n: (None if x is None else x[:, prefix].contiguous())
+           for n, x in hist.items()}
+    return {"prefix": pre, "token": tok}
+
+
+# The five workload shapes (name -> keyword arguments), one per benchmark line
+# or parity case.  "chunk" is the chunk length of the chunkwise kernels.
+WORKLOADS = {
+    "gla_fp32_small": dict(backbone=GLA, B=1, H=2, T=256, Dk=64, Dv=64,
+                           dtype=torch.float32, seed=1235),
+    "gla_bf16_4k": dict(backbone=GLA, B=8, H=16, T=4096, Dk=128, Dv=128,
+                        dtype=torch.bfloat16, seed=1236),
+    "gdn_bf16_4k": dict(backbone=GDN, B=8, H=16, T=4096, Dk=128, Dv=128,
+                        dtype=torch.bfloat16, seed=1237),
+    "gla_bf16_20k": dict(backbone=GLA, B=1, H=16, T=20480, Dk=128, Dv=128,
+                         dtype=torch.bfloat16, seed=1238),
+    "gdn_bf16_20k": dict(backbone=GDN, B=1, H=16, T=20480, Dk=128, Dv=128,
+                         dtype=torch.bfloat16, seed=1238),
+}
