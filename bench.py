@@ -1,0 +1,410 @@
+"""Benchmark of the CCQ hot path on GB300.
+
+One step = one CCQ chunkwise forward over the whole workload batch (one call
+of ccq_gla_fwd / ccq_gdn_fwd, or one ccq_decode_step), inputs resident in HBM.
+The default workload is CCQ-GLA forward, bf16, B=8, H=16, T=4096,
+Dk=Dv=128, chunk 64 (the metric's configuration).  Prints ONE JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   (the fp64 CPU oracle on host cores)
+
+Multi-GPU (torchrun, one rank per GPU): every rank runs its own copy of the
+workload (independent sequences, no data-path collective); value is the
+total tokens of all ranks / the max over ranks of the timed region.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "CCQ chunked fwd tokens/s at T=4K,d=128 bf16; % of roofline (tensor/HBM)"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
+
+# Workloads: name -> (backbone, B, H, T, D, kernel name, description)
+WORKLOADS = {
+    "gla_bf16_4k": ("gla", 8, 16, 4096, 128),
+    "gdn_bf16_4k": ("gdn", 8, 16, 4096, 128),
+    "gla_bf16_20k": ("gla", 1, 16, 20480, 128),
+    "gdn_bf16_20k": ("gdn", 1, 16, 20480, 128),
+    "decode_b256": ("decode", 256, 16, 1, 128),
+}
+KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_recurrent.cu", "decode": "ccq_recurrent.cu"}
+KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "recurrent_kernel", "decode": "recurrent_kernel"}
+
+
+def algorithmic_bytes(kind, B, H, T, D):
+    """Bytes one launch must move at minimum: every input read once, o written
+    once, final fp32 states written once (initial states are zero / absent
+    except for decode, whose cache is read and written)."""
+    tok = B * T * H
+    if kind == "gla":
+        return tok * D * 2 * 4 + tok * D * 2 + tok * 4 + B * H * (2 * D * D + D) * 4 + B * 8
+    if kind == "gdn":
+        return tok * D * 2 * 3 + tok * D * 2 + tok * 4 * 3 + B * H * (2 * D * D + D) * 4 + B * 8
+    # decode: q, k, v, gate (bf16) + lambda in, o out, cache (S, C, m) read and written
+    return tok * D * 2 * 4 + tok * 4 + tok * D * 2 + 2 * B * H * (2 * D * D + D) * 4 + 2 * B * 8
+
+
+def algorithmic_flops(kind, B, H, T, D, C=64):
+    """Dense tile FLOPs of the chunkwise algorithm (Algorithm 1 products)."""
+    nc = (T + C - 1) // C
+    # GLA: four C x D x D products (Qbar S^K, Qg S, Ku^T V, Kbar^T Kbar) and four
+    # C x C x D products (Qbar Kbar^T, W' Kbar, Qg Kg^T, A V), 2 FLOP per MAC.
+    per_chunk = {"gla": 8 * C * D * D + 8 * C * C * D,
+                 "gdn": 10 * C * D * D + 12 * C * C * D}.get(kind)
+    if per_chunk is None:
+        return B * H * 8 * D * D
+    return B * H * nc * per_chunk
+
+
+def kernel_sha(kind):
+    p = os.path.join(ROOT, "paper_2606_01294_gb300", "csrc", KERNEL_SOURCES[kind])
+    with open(p, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_traffic(kind, workload):
+    """dram bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source; else None."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            t = json.load(f)
+        e = t.get(workload)
+        if e and e.get("kernel_sha") == kernel_sha(kind):
+            return e.get("dram_bytes_per_launch")
+    except (OSError, ValueError):
+        pass
+    return None
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.window = None  # (start, end) wall-clock seconds of the timed region
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "20"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        rows = []
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                ts = time.mktime(time.strptime(parts[0].split(".")[0], "%Y/%m/%d %H:%M:%S"))
+                ts += float("0." + parts[0].split(".")[1]) if "." in parts[0] else 0.0
+                rows.append((ts, float(parts[1]), float(parts[2]),
+                             [n for n, v in zip(names, parts[5:9]) if v.lower() == "active"]))
+            except (ValueError, IndexError):
+                continue
+        inside = rows
+        where = "timed region"
+        if self.window:
+            inside = [r for r in rows if self.window[0] - 0.05 <= r[0] <= self.window[1] + 0.05]
+            if not inside:  # region shorter than the sampling interval
+                inside = [r for r in rows if r[0] <= self.window[1] + 0.05][-2:]
+                where = "last samples before the end of the timed region"
+        sm = [r[1] for r in inside]
+        reasons = sorted({n for r in inside for n in r[3]})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": inside[-1][2] if inside else None,
+                "reasons": reasons, "samples": len(sm), "window": where}
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), \
+        int(os.environ.get("WORLD_SIZE", 1))
+
+
+def cpu_oracle_run(kind, B, H, T, D, sample_b, seed):
+    """Time the fp64 oracle on host cores over `sample_b` batch rows of T tokens."""
+    import torch
+    import oracle
+    from paper_2606_01294_gb300 import inputs as gen
+    if kind == "decode":
+        Dd = gen.make_decode_inputs(gen.GLA, sample_b, H, D, D, seed=seed)
+        pre = oracle.forward(gen.GLA, Dd["prefix"]["q"], Dd["prefix"]["k"], Dd["prefix"]["v"],
+                             Dd["prefix"]["gate"], Dd["prefix"]["lam"])
+        tk = Dd["token"]
+        t0 = time.perf_counter()
+        oracle.decode_step(gen.GLA, tk["q"], tk["k"], tk["v"], tk["gate"], tk["lam"],
+                           pre["S"], pre["C"], pre["m"], pre["t"])
+        dt = time.perf_counter() - t0
+        return sample_b / dt, dt
+    bb = gen.GLA if kind == "gla" else gen.GDN
+    P = gen.make_inputs(bb, sample_b, T, H, D, D, dtype=torch.bfloat16, seed=seed)
+    t0 = time.perf_counter()
+    oracle.forward(bb, P["q"], P["k"], P["v"], P["gate"], P["lam"], beta=P["beta"])
+    dt = time.perf_counter() - t0
+    return sample_b * T / dt, dt
+
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    oracle.build_oracle()
+    kind, B, H, T, D = WORKLOADS[args.workload]
+    # one step = a bounded sample of the workload: one batch row (all heads)
+    # over the first Ts tokens, so that warm-up + steps stay within minutes
+    sample_b = 1 if kind != "decode" else 16
+    Ts = min(T, 1024) if kind != "decode" else 1
+    cores = os.cpu_count() or 1
+    for _ in range(args.warmup):
+        cpu_oracle_run(kind, B, H, Ts, D, sample_b, seed=99)
+    times = []
+    for _ in range(args.steps):
+        _, dt = cpu_oracle_run(kind, B, H, Ts, D, sample_b, seed=1236)
+        times.append(dt)
+    rate = sample_b * Ts * args.steps / sum(times)
+    sample = (f"batch row 0 of {B}, all {H} heads, first {Ts} of {T} tokens, per step"
+              if kind != "decode" else f"{sample_b} of {B} batch rows, all {H} heads, one token")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": rate, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload, "backbone": kind, "B": B, "H": H, "T": T,
+                   "d_k": D, "d_v": D, "chunk": 64, "global_batch": B, "seq_len": T},
+        "cpu_baseline": {"value": rate, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": rate, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    from __graft_entry__ import build
+    if rank == 0 or world == 1:
+        build()
+    if world > 1:
+        dist.barrier()
+        build()
+    from paper_2606_01294_gb300 import ccq
+    from paper_2606_01294_gb300 import inputs as gen
+
+    kind, B, H, T, D = WORKLOADS[args.workload]
+    seed = 1236 + rank
+    stream = torch.cuda.current_stream(dev)
+
+    # ---------------- inputs resident in HBM
+    if kind == "decode":
+        Dd = gen.make_decode_inputs(gen.GLA, B, H, D, D, seed=seed)
+        pre = {n: (None if x is None else x.to(dev)) for n, x in Dd["prefix"].items()}
+        tok = {n: (None if x is None else x.to(dev)) for n, x in Dd["token"].items()}
+        _, state0 = ccq.gla_fwd(pre["q"], pre["k"], pre["v"], pre["gate"], pre["lam"])
+        state = ccq.CCQState(*(x.clone() for x in (state0.S, state0.C, state0.m, state0.t)))
+        out = torch.empty(B, H, D, dtype=torch.bfloat16, device=dev)
+
+        def step():
+            ccq.decode_step(gen.GLA, tok["q"], tok["k"], tok["v"], tok["gate"], tok["lam"], state,
+                            out=out)
+        tokens_per_step = B
+        host = {n: (None if x is None else x.pin_memory()) for n, x in Dd["token"].items()}
+    else:
+        bb = gen.GLA if kind == "gla" else gen.GDN
+        P = gen.make_inputs(bb, B, T, H, D, D, dtype=torch.bfloat16, seed=seed)
+        Dv = {n: (None if x is None else x.to(dev)) for n, x in P.items()}
+        out = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
+        fstate = ccq.CCQState.empty(B, H, D, D, dev)
+
+        def step():
+            if kind == "gla":
+                ccq.gla_fwd(Dv["q"], Dv["k"], Dv["v"], Dv["gate"], Dv["lam"], out=out,
+                            final_state=fstate)
+            else:
+                ccq.gdn_fwd(Dv["q"], Dv["k"], Dv["v"], Dv["gate"], Dv["beta"], Dv["lam"], out=out,
+                            final_state=fstate)
+        tokens_per_step = B * T
+        host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    with ClockSampler(local_rank) as clocks:
+        time.sleep(0.3)  # nvidia-smi start-up
+        for _ in range(args.warmup):
+            step()
+        ccq.device_status()
+        torch.cuda.synchronize()
+        # ---------------- timed region: device-resident inputs
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+        w0 = time.time()
+        t_start = torch.cuda.Event(enable_timing=True)
+        t_end = torch.cuda.Event(enable_timing=True)
+        t_start.record(stream)
+        for i in range(args.steps):
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+        t_end.record(stream)
+        torch.cuda.synchronize()
+        clocks.window = (w0, time.time())
+        time.sleep(0.1)
+    if world > 1:
+        dist.barrier()
+    ccq.device_status()
+    total_ms = t_start.elapsed_time(t_end)
+    launch_ms = [a.elapsed_time(b) for a, b in ev]
+    if world > 1:
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    value = world * tokens_per_step * args.steps / (total_ms / 1e3)
+
+    # ---------------- e2e: host buffers, copies inside the timed region
+    def e2e_step():
+        if kind == "decode":
+            d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
+            o = ccq.decode_step(gen.GLA, d["q"], d["k"], d["v"], d["gate"], d["lam"], state, out=out)
+            res = o.to("cpu", non_blocking=True)
+            return res
+        d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
+        if kind == "gla":
+            o, st = ccq.gla_fwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out,
+                                final_state=fstate)
+        else:
+            o, st = ccq.gdn_fwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], out=out,
+                                final_state=fstate)
+        return o.to("cpu", non_blocking=True)
+
+    h2d = sum(x.numel() * x.element_size() for x in host.values() if x is not None)
+    d2h = out.numel() * out.element_size()
+    e2e_steps = max(3, min(args.steps, 10))
+    e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e_value = world * tokens_per_step / (e2e_ms / 1e3)
+
+    line = None
+    if rank == 0:
+        with open(PEAKS_FILE) as f:
+            peaks = json.load(f)
+        kern_ms = statistics.mean(launch_ms)
+        bytes_ = algorithmic_bytes(kind, B, H, T, D)
+        achieved = bytes_ / (kern_ms / 1e3) / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": achieved / peaks["hbm_gbs"],
+                "traffic": measured_traffic(kind, args.workload),
+                "kernel": KERNEL_NAMES[kind], "algorithmic_bytes": bytes_,
+                "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
+                "flops": algorithmic_flops(kind, B, H, T, D)}
+        cpu = None
+        if not args.no_cpu_baseline and world == 1:
+            import oracle
+            oracle.build_oracle()
+            sample_b = B if kind != "decode" else 32
+            rate, dt = cpu_oracle_run(kind, B, H, T, D, sample_b, seed=seed)
+            cpu = {"value": rate, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                   "sample": (f"{sample_b} of {B} batch rows, all {H} heads, {T} tokens, one pass "
+                              f"({dt:.1f} s)")}
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": args.workload, "backbone": kind, "B": B, "H": H, "T": T,
+                       "d_k": D, "d_v": D, "chunk": 64, "global_batch": B * world, "seq_len": T,
+                       "parallelism": f"replicas{world}",
+                       "l2": "inputs larger than L2 (no flush)"},
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": args.steps,
+            "clocks": clocks.summary(),
+            "kernel_ms_mean": kern_ms,
+            "kernel_ms_min": min(launch_ms),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="gla_bf16_4k", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

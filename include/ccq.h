@@ -1,0 +1,154 @@
+/*
+ * ccq.h -- C ABI of the GB300 (sm_103a) Curvature-Conditioned Query library.
+ *
+ * CCQ (arxiv 2606.01294) modifies only the read of a linear-attention layer:
+ * before the query reads the fast-weight state S, it is contracted by
+ * (I - lambda_t Sigma_t), where Sigma_t is the running, length-normalised key
+ * covariance (Sec. 3.2, Eq. clean; App. A.2):
+ *
+ *   C_t = sum_{j<=t} kbar_j kbar_j^T,   m_t = sum_{j<=t} kbar_j,
+ *   Sigma_t = C_t / t - (m_t / t)(m_t / t)^T            (centred, default)
+ *   q_clean = qbar_t - lambda_t Sigma_t qbar_t           (Eq. clean, Algorithm 2)
+ *   o_t     = scale * S_t q_clean                        (Eq. read)
+ *
+ * with qbar, kbar the per-head l2-normalised query and key (Algorithms 1, 2).
+ * The backbone write S_t = Update(S_{t-1}; kbar_t, v_t, ...) is either
+ *   GLA:            S_t = S_{t-1} Diag(alpha_t) + v_t kbar_t^T,   alpha_t = exp(gk_t) in R^{Dk}
+ *   Gated DeltaNet: S_t = alpha_t S_{t-1} (I - beta_t kbar_t kbar_t^T) + beta_t v_t kbar_t^T,
+ *                   alpha_t = exp(g_t) scalar
+ * (Sec. 2.2; the paper treats the write rule as a black box).  The chunkwise
+ * kernels follow Algorithm 1 (App. B): the key statistics are carried across
+ * chunks as a d_k x d_k second-moment sum and a d_k key-sum vector.
+ *
+ * Conventions shared by every entry point
+ *   - Pointers are DEVICE pointers owned by the caller and must be 16-byte
+ *     aligned.  Nothing is allocated and nothing is freed by the library.
+ *   - Token tensors are [B, T, H, D] with D contiguous (row-major).
+ *   - States are fp32.  S is stored as its transpose: S[B, H, Dk, Dv], element
+ *     [i][j] is the paper's S_{j,i}.  C is the second-moment SUM C_t
+ *     [B, H, Dk, Dk] (not divided by t), m the key SUM m_t [B, H, Dk], and t the
+ *     per-batch-row token count [B] (int64).  Algorithm 2's running means are
+ *     C_t / t and m_t / t; keeping sums makes chunk, prefill and decode
+ *     resumption exact.
+ *   - Initial-state pointers may be NULL (zero state, t0 = 0).  Final-state
+ *     pointers may be NULL (not written).  A final-state buffer may alias the
+ *     corresponding initial-state buffer.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream).  Argument errors are reported synchronously through the
+ *     return value; the calls never abort the process.  Every in-kernel wait is
+ *     bounded: a wait that runs out records CCQ_ERR_TIMEOUT in a device status
+ *     word that ccq_device_status() reads back.
+ */
+#ifndef CCQ_H_
+#define CCQ_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define CCQ_API __attribute__((visibility("default")))
+#else
+#define CCQ_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    CCQ_OK = 0,
+    CCQ_ERR_INVALID_ARG = 1, /* NULL or misaligned pointer, negative size, ...    */
+    CCQ_ERR_UNSUPPORTED = 2, /* a valid request this build does not implement     */
+    CCQ_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed                 */
+    CCQ_ERR_TIMEOUT = 4      /* an in-kernel bounded wait ran out (device status) */
+} ccq_status;
+
+typedef enum { CCQ_BF16 = 0, CCQ_FP32 = 1 } ccq_dtype;
+
+typedef enum {
+    CCQ_ALGO_AUTO = 0,      /* chunkwise tensor-core kernel when supported, else recurrent */
+    CCQ_ALGO_RECURRENT = 1, /* token-by-token CUDA-core kernel (fp32 arithmetic)         */
+    CCQ_ALGO_CHUNKWISE = 2  /* chunkwise tcgen05 kernel (bf16 operands, fp32 accumulate)  */
+} ccq_algo;
+
+/* Contraction and read hyper-parameters. */
+typedef struct {
+    int l2norm_qk; /* 1: l2-normalise q and k per head row in the kernel (Algorithms 1, 2);
+                      0: use q and k as given.  The norm uses rsqrt(max(|x|^2, 1e-12)),
+                      so an all-zero row stays zero.                                     */
+    float scale;   /* read scale multiplying o; <= 0 selects 1/sqrt(Dk) (paper silent)    */
+    int centered;  /* 1: Sigma_t = C_t/t - mu_t mu_t^T (App. A.2); 0: uncentred C_t/t
+                      (App. D ablation)                                                  */
+    int chunk;     /* chunk length of the chunkwise kernels; 0 or 64 (Algorithm 1)        */
+    int algo;      /* a ccq_algo value                                                   */
+} ccq_params;
+
+/* Fill *p with the defaults: l2norm_qk = 1, scale = 0 (1/sqrt(Dk)), centered = 1,
+   chunk = 64, algo = CCQ_ALGO_AUTO. */
+CCQ_API void ccq_default_params(ccq_params *p);
+
+/*
+ * CCQ-GLA chunkwise forward (Algorithm 1 with the GLA write rule).
+ *   q, k      [B,T,H,Dk] in in_dtype;  v [B,T,H,Dv] in in_dtype.
+ *   gk        log forget gate log(alpha) [B,T,H,Dk] in gate_dtype (<= 0).
+ *   lambda    [B,T,H] fp32, the CCQ gate lambda_t in (0,1) (Eq. clean; the caller
+ *             applies W_lambda and the sigmoid).
+ *   S0/C0/m0/t0  initial states (see conventions); ST/CT/mT/tT final states.
+ *   o         [B,T,H,Dv] in in_dtype.
+ * Supported: Dk = Dv in {64, 128}; T >= 0; B, H >= 1.  in_dtype BF16 runs the
+ * chunkwise tensor-core kernel for Dk = Dv = 128 and the recurrent kernel
+ * otherwise; FP32 always runs the recurrent kernel (fp32 arithmetic).
+ * The chunkwise kernel scales by exp of in-chunk cumulative gates measured from
+ * the chunk midpoint; per-chunk cumulative log-gates must stay above about -160
+ * (more negative sums underflow to an exact-zero contribution).
+ * Returns CCQ_OK or an error code; launches asynchronously on `stream`.
+ */
+CCQ_API ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
+                       const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream);
+
+/*
+ * CCQ-Gated-DeltaNet forward (the gated delta rule as the backbone).
+ *   g         log decay log(alpha) [B,T,H] fp32 (<= 0);  beta [B,T,H] fp32 in [0,1].
+ * All other arguments as ccq_gla_fwd.
+ */
+CCQ_API ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
+                       const float *beta, const float *lambda, ccq_dtype in_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream);
+
+/*
+ * One recurrent CCQ token for a batch of cached states (Algorithm 2), updating
+ * the cache (S, C, m, t) IN PLACE and writing o.
+ *   backbone  0 = GLA (gate: log alpha [B,H,Dk] in gate_dtype),
+ *             1 = Gated DeltaNet (gate: log alpha [B,H] fp32; beta [B,H] fp32).
+ *   q, k      [B,H,Dk]; v [B,H,Dv]; lambda [B,H] fp32; o [B,H,Dv] (in_dtype).
+ *   S [B,H,Dk,Dv], C [B,H,Dk,Dk], m [B,H,Dk] fp32 and t [B] int64, read and written.
+ */
+CCQ_API ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,
+                           const void *gate, const float *beta, const float *lambda,
+                           ccq_dtype in_dtype, ccq_dtype gate_dtype, float *S, float *C,
+                           float *m, int64_t *t, void *o, int B, int H, int Dk, int Dv,
+                           const ccq_params *p, void *stream);
+
+/*
+ * Synchronise `stream`, then read and clear the device status word that the
+ * kernels' bounded waits write.  Returns CCQ_OK, CCQ_ERR_TIMEOUT (a kernel gave
+ * up waiting; its outputs are not valid) or CCQ_ERR_CUDA.
+ */
+CCQ_API ccq_status ccq_device_status(void *stream);
+
+/* Static description of a status code. */
+CCQ_API const char *ccq_status_string(ccq_status s);
+
+/* Human-readable detail of the most recent error returned on this host thread. */
+CCQ_API const char *ccq_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CCQ_H_ */

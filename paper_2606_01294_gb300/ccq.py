@@ -1,0 +1,265 @@
+"""Python binding of libccq.so (include/ccq.h): argument marshalling only.
+
+Every step of the CCQ computation runs in the library's CUDA kernels; this
+module checks tensor placement/dtype/layout, allocates outputs with torch on
+the input's device, and passes raw device pointers plus the current CUDA
+stream through ctypes.  There is no CPU path: if the library is missing, or a
+tensor is not on a CUDA device, the call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from . import _build
+
+CCQ_OK, CCQ_ERR_INVALID_ARG, CCQ_ERR_UNSUPPORTED, CCQ_ERR_CUDA, CCQ_ERR_TIMEOUT = range(5)
+BF16, FP32 = 0, 1
+ALGO = {"auto": 0, "recurrent": 1, "chunkwise": 2}
+GLA, GDN = 0, 1
+
+
+class CCQError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"[ccq status {status}] {msg}")
+        self.status = status
+
+
+class _Params(ctypes.Structure):
+    _fields_ = [("l2norm_qk", ctypes.c_int), ("scale", ctypes.c_float),
+                ("centered", ctypes.c_int), ("chunk", ctypes.c_int),
+                ("algo", ctypes.c_int)]
+
+
+_lib = None
+_VP = ctypes.c_void_p
+_I = ctypes.c_int
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def load_library() -> ctypes.CDLL:
+    """Open libccq.so (it must have been built); raises if it is absent."""
+    global _lib
+    if _lib is None:
+        path = _build.LIB_PATH
+        if not os.path.exists(path):
+            raise RuntimeError(
+                f"{path} is missing: build the CUDA library first "
+                "(python -c 'import __graft_entry__ as g; g.build()')")
+        lib = ctypes.CDLL(path)
+        lib.ccq_default_params.argtypes = [ctypes.POINTER(_Params)]
+        lib.ccq_default_params.restype = None
+        lib.ccq_status_string.argtypes = [_I]
+        lib.ccq_status_string.restype = ctypes.c_char_p
+        lib.ccq_last_error.argtypes = []
+        lib.ccq_last_error.restype = ctypes.c_char_p
+        lib.ccq_device_status.argtypes = [_VP]
+        lib.ccq_device_status.restype = _I
+        lib.ccq_gla_fwd.argtypes = ([_VP] * 5 + [_I, _I] + [_VP] * 9 + [_I] * 5
+                                    + [ctypes.POINTER(_Params), _VP])
+        lib.ccq_gla_fwd.restype = _I
+        lib.ccq_gdn_fwd.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 5
+                                    + [ctypes.POINTER(_Params), _VP])
+        lib.ccq_gdn_fwd.restype = _I
+        lib.ccq_decode_step.argtypes = ([_I] + [_VP] * 6 + [_I, _I] + [_VP] * 5
+                                        + [_I] * 4 + [ctypes.POINTER(_Params), _VP])
+        lib.ccq_decode_step.restype = _I
+        _lib = lib
+    return _lib
+
+
+def header_symbols() -> list:
+    """Names of every function include/*.h declares with CCQ_API."""
+    names = []
+    for f in sorted(os.listdir(_build.INCLUDE)):
+        if f.endswith(".h"):
+            with open(os.path.join(_build.INCLUDE, f)) as fh:
+                names += re.findall(r"CCQ_API\s+[\w\s\*]*?\b(ccq_\w+)\s*\(", fh.read())
+    return names
+
+
+def _check(status: int):
+    if status != CCQ_OK:
+        lib = load_library()
+        raise CCQError(status, lib.ccq_last_error().decode())
+
+
+def params(*, l2norm: bool = True, scale: Optional[float] = None, centered: bool = True,
+           chunk: int = 64, algo: str = "auto") -> _Params:
+    p = _Params()
+    load_library().ccq_default_params(ctypes.byref(p))
+    p.l2norm_qk = int(bool(l2norm))
+    p.scale = 0.0 if scale is None else float(scale)
+    p.centered = int(bool(centered))
+    p.chunk = int(chunk)
+    p.algo = ALGO[algo]
+    return p
+
+
+def _ptr(x: Optional[torch.Tensor]):
+    return None if x is None else ctypes.c_void_p(x.data_ptr())
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return FP32
+    raise TypeError(f"unsupported dtype {t.dtype}: bf16 or fp32")
+
+
+def _req(t, name, device, dtype=None, shape=None):
+    if t is None:
+        raise ValueError(f"{name} is required")
+    if not isinstance(t, torch.Tensor) or t.device.type != "cuda":
+        raise ValueError(f"{name} must be a CUDA tensor (there is no CPU path)")
+    if t.device != device:
+        raise ValueError(f"{name} is on {t.device}, expected {device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t
+
+
+def _stream(device, stream):
+    s = stream if stream is not None else torch.cuda.current_stream(device)
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+@dataclass
+class CCQState:
+    """Recurrent cache (Algorithm 2's triple plus the position): S^T [B,H,Dk,Dv],
+    key second-moment SUM C [B,H,Dk,Dk], key SUM m [B,H,Dk] (fp32), t [B] int64."""
+    S: torch.Tensor
+    C: torch.Tensor
+    m: torch.Tensor
+    t: torch.Tensor
+
+    @staticmethod
+    def zeros(B, H, Dk, Dv, device):
+        return CCQState(torch.zeros(B, H, Dk, Dv, device=device),
+                        torch.zeros(B, H, Dk, Dk, device=device),
+                        torch.zeros(B, H, Dk, device=device),
+                        torch.zeros(B, dtype=torch.int64, device=device))
+
+    @staticmethod
+    def empty(B, H, Dk, Dv, device):
+        return CCQState(torch.empty(B, H, Dk, Dv, device=device),
+                        torch.empty(B, H, Dk, Dk, device=device),
+                        torch.empty(B, H, Dk, device=device),
+                        torch.empty(B, dtype=torch.int64, device=device))
+
+
+def _state_in(state, B, H, Dk, Dv, device):
+    if state is None:
+        return None, None, None, None
+    return (_req(state.S, "S0", device, torch.float32, (B, H, Dk, Dv)),
+            _req(state.C, "C0", device, torch.float32, (B, H, Dk, Dk)),
+            _req(state.m, "m0", device, torch.float32, (B, H, Dk)),
+            _req(state.t, "t0", device, torch.int64, (B,)))
+
+
+def gla_fwd(q, k, v, gk, lam, state: Optional[CCQState] = None, *, out=None,
+            final_state: Optional[CCQState] = None, return_state: bool = True,
+            stream=None, **kw):
+    """CCQ-GLA forward: o [B,T,H,Dv] and (optionally) the final CCQState.
+
+    q, k [B,T,H,Dk], v [B,T,H,Dv] bf16 or fp32 (same dtype); gk [B,T,H,Dk]
+    log-forget gate (bf16 or fp32); lam [B,T,H] fp32.  ``state`` is the initial
+    cache (None = zero).  Keyword arguments go to :func:`params`.
+    """
+    dev = q.device
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, T, H, Dv))
+    _req(gk, "gk", dev, None, (B, T, H, Dk))
+    _req(lam, "lam", dev, torch.float32, (B, T, H))
+    S0, C0, m0, t0 = _state_in(state, B, H, Dk, Dv, dev)
+    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
+    _req(o, "out", dev, q.dtype, (B, T, H, Dv))
+    fs = final_state
+    if fs is None and return_state:
+        fs = CCQState.empty(B, H, Dk, Dv, dev)
+    p = params(**kw)
+    st = load_library().ccq_gla_fwd(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gk), _ptr(lam), _dtype_code(q), _dtype_code(gk),
+        _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(o),
+        _ptr(fs.S if fs else None), _ptr(fs.C if fs else None), _ptr(fs.m if fs else None),
+        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, ctypes.byref(p), _stream(dev, stream))
+    _check(st)
+    return (o, fs) if return_state else o
+
+
+def gdn_fwd(q, k, v, g, beta, lam, state: Optional[CCQState] = None, *, out=None,
+            final_state: Optional[CCQState] = None, return_state: bool = True,
+            stream=None, **kw):
+    """CCQ-Gated-DeltaNet forward.  g (log decay) and beta are [B,T,H] fp32."""
+    dev = q.device
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, T, H, Dv))
+    _req(g, "g", dev, torch.float32, (B, T, H))
+    _req(beta, "beta", dev, torch.float32, (B, T, H))
+    _req(lam, "lam", dev, torch.float32, (B, T, H))
+    S0, C0, m0, t0 = _state_in(state, B, H, Dk, Dv, dev)
+    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
+    _req(o, "out", dev, q.dtype, (B, T, H, Dv))
+    fs = final_state
+    if fs is None and return_state:
+        fs = CCQState.empty(B, H, Dk, Dv, dev)
+    p = params(**kw)
+    st = load_library().ccq_gdn_fwd(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _dtype_code(q),
+        _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(o),
+        _ptr(fs.S if fs else None), _ptr(fs.C if fs else None), _ptr(fs.m if fs else None),
+        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, ctypes.byref(p), _stream(dev, stream))
+    _check(st)
+    return (o, fs) if return_state else o
+
+
+def decode_step(backbone: int, q, k, v, gate, lam, state: CCQState, beta=None, *,
+                out=None, stream=None, **kw):
+    """One recurrent token (Algorithm 2): q, k [B,H,Dk], v [B,H,Dv]; gate
+    [B,H,Dk] (GLA, bf16/fp32) or [B,H] fp32 (GDN); lam (and beta) [B,H] fp32.
+    Updates ``state`` in place and returns o [B,H,Dv]."""
+    dev = q.device
+    B, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, H, Dv))
+    _req(gate, "gate", dev, None, (B, H, Dk) if backbone == GLA else (B, H))
+    _req(lam, "lam", dev, torch.float32, (B, H))
+    if backbone == GDN:
+        _req(beta, "beta", dev, torch.float32, (B, H))
+    S, C, m, t = _state_in(state, B, H, Dk, Dv, dev)
+    o = out if out is not None else torch.empty(B, H, Dv, dtype=q.dtype, device=dev)
+    _req(o, "out", dev, q.dtype, (B, H, Dv))
+    p = params(**kw)
+    st = load_library().ccq_decode_step(
+        int(backbone), _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(beta), _ptr(lam),
+        _dtype_code(q), _dtype_code(gate), _ptr(S), _ptr(C), _ptr(m), _ptr(t), _ptr(o),
+        B, H, Dk, Dv, ctypes.byref(p), _stream(dev, stream))
+    _check(st)
+    return o
+
+
+def device_status(stream=None, device=None):
+    """Synchronise and read/clear the kernels' status word; raises on a timeout."""
+    dev = device or torch.device("cuda", torch.cuda.current_device())
+    _check(load_library().ccq_device_status(_stream(dev, stream)))

@@ -1,0 +1,286 @@
+// ccq_capi.cu -- the extern "C" boundary of the CCQ library (include/ccq.h):
+// argument validation, tensor-map encoding, kernel dispatch and the device
+// status word.  No entry point allocates memory.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdint.h>
+#include <stdio.h>
+
+#include <initializer_list>
+
+#include "../../include/ccq.h"
+#include "ccq_internal.h"
+
+namespace ccq {
+
+// Written by a kernel whose bounded wait gave up; read and cleared by
+// ccq_device_status().
+__device__ int g_status = 0;
+
+int *device_status_word() {
+    // one slot per device ordinal; filled on first use with that device current
+    static int *addr[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<int *>(p);
+    }
+    return addr[dev];
+}
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+ccq_status fail(ccq_status s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+ccq_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(CCQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+struct Common {
+    ccq_params p;
+    float scale;
+};
+
+ccq_status check_common(const ccq_params *pin, int B, int T, int H, int Dk, int Dv, Common *c) {
+    if (pin) c->p = *pin;
+    else ccq_default_params(&c->p);
+    if (B < 1 || H < 1 || T < 0) return fail(CCQ_ERR_INVALID_ARG, "bad sizes B=%d T=%d H=%d", B, T, H);
+    if (Dk != Dv || (Dk != 64 && Dk != 128))
+        return fail(CCQ_ERR_UNSUPPORTED, "head dims Dk=%d Dv=%d: supported Dk = Dv in {64, 128}", Dk, Dv);
+    if (c->p.chunk != 0 && c->p.chunk != 64)
+        return fail(CCQ_ERR_UNSUPPORTED, "chunk=%d: supported 64", c->p.chunk);
+    if (c->p.algo < CCQ_ALGO_AUTO || c->p.algo > CCQ_ALGO_CHUNKWISE)
+        return fail(CCQ_ERR_INVALID_ARG, "unknown algo %d", c->p.algo);
+    if ((static_cast<long long>(B) * H) > 0x7fffffffLL)
+        return fail(CCQ_ERR_INVALID_ARG, "B*H too large");
+    c->scale = c->p.scale > 0.f ? c->p.scale : 1.f / sqrtf(static_cast<float>(Dk));
+    return CCQ_OK;
+}
+
+ccq_status check_ptrs(const char *names, std::initializer_list<const void *> required,
+                      std::initializer_list<const void *> optional) {
+    int i = 0;
+    for (const void *p : required) {
+        if (!p) return fail(CCQ_ERR_INVALID_ARG, "required pointer #%d of (%s) is NULL", i, names);
+        if (!aligned16(p)) return fail(CCQ_ERR_INVALID_ARG, "pointer #%d of (%s) is not 16-byte aligned", i, names);
+        ++i;
+    }
+    for (const void *p : optional) {
+        if (p && !aligned16(p)) return fail(CCQ_ERR_INVALID_ARG, "an optional state pointer is not 16-byte aligned");
+    }
+    return CCQ_OK;
+}
+
+ccq_status run_recurrent(RecurrentArgs &ra, cudaStream_t s) {
+    cudaError_t e = launch_recurrent(ra, s);
+    if (e != cudaSuccess) return cuda_fail(e, "recurrent kernel launch");
+    return CCQ_OK;
+}
+
+}  // namespace
+
+bool make_token_map(CUtensorMap *map, const void *base, int elem_bytes, int B, int T, int H, int D,
+                    int box_inner, bool swizzle128) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[4] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(H),
+                                static_cast<cuuint64_t>(T), static_cast<cuuint64_t>(B)};
+    const cuuint64_t eb = static_cast<cuuint64_t>(elem_bytes);
+    const cuuint64_t strides[3] = {eb * D, eb * D * H, eb * D * H * T};
+    const cuuint32_t box[4] = {static_cast<cuuint32_t>(box_inner), 1, 64, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    const CUtensorMapDataType dt =
+        elem_bytes == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    CUresult r = fn(map, dt, 4, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+}  // namespace ccq
+
+using namespace ccq;
+
+extern "C" {
+
+void ccq_default_params(ccq_params *p) {
+    if (!p) return;
+    p->l2norm_qk = 1;
+    p->scale = 0.f;
+    p->centered = 1;
+    p->chunk = 64;
+    p->algo = CCQ_ALGO_AUTO;
+}
+
+const char *ccq_status_string(ccq_status s) {
+    switch (s) {
+        case CCQ_OK: return "ok";
+        case CCQ_ERR_INVALID_ARG: return "invalid argument";
+        case CCQ_ERR_UNSUPPORTED: return "unsupported configuration";
+        case CCQ_ERR_CUDA: return "CUDA error";
+        case CCQ_ERR_TIMEOUT: return "a kernel's bounded wait timed out";
+    }
+    return "unknown status";
+}
+
+const char *ccq_last_error(void) { return g_last_error; }
+
+ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
+                       const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if ((in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) || (gate_dtype != CCQ_BF16 && gate_dtype != CCQ_FP32))
+        return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    if (T > 0) {
+        st = check_ptrs("q,k,v,gk,lambda,o", {q, k, v, gk, lambda, o}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        if (st != CCQ_OK) return st;
+    } else {
+        st = check_ptrs("", {}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        if (st != CCQ_OK) return st;
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool chunk_ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
+    if (c.p.algo == CCQ_ALGO_CHUNKWISE && !chunk_ok)
+        return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
+    if (chunk_ok && c.p.algo != CCQ_ALGO_RECURRENT) {
+        ChunkMaps maps;
+        const int geb = gate_dtype == CCQ_BF16 ? 2 : 4;
+        if (!make_token_map(&maps.q, q, 2, B, T, H, 128, 64, true) ||
+            !make_token_map(&maps.k, k, 2, B, T, H, 128, 64, true) ||
+            !make_token_map(&maps.v, v, 2, B, T, H, 128, 64, true) ||
+            !make_token_map(&maps.g, gk, geb, B, T, H, 128, 128, false))
+            return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
+        ChunkArgs a = {};
+        a.B = B; a.T = T; a.H = H;
+        a.gate_dtype = gate_dtype == CCQ_BF16 ? 0 : 1;
+        a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
+        a.lambda = lambda;
+        a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
+        a.o = static_cast<__nv_bfloat16 *>(o);
+        a.ST = ST; a.CT = CT; a.mT = mT; a.tT = tT;
+        a.status = device_status_word();
+        if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
+        cudaError_t e = launch_gla_chunk(a, maps, s);
+        if (e != cudaSuccess) return cuda_fail(e, "chunkwise GLA kernel launch");
+        return CCQ_OK;
+    }
+    RecurrentArgs ra = {};
+    ra.backbone = 0; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
+    ra.in_dtype = in_dtype; ra.gate_dtype = gate_dtype;
+    ra.l2norm = c.p.l2norm_qk; ra.centered = c.p.centered; ra.scale = c.scale;
+    ra.q = q; ra.k = k; ra.v = v; ra.gate = gk; ra.beta = nullptr; ra.lambda = lambda;
+    ra.S0 = S0; ra.C0 = C0; ra.m0 = m0; ra.t0 = t0;
+    ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT; ra.tT = tT;
+    return run_recurrent(ra, s);
+}
+
+ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
+                       const float *beta, const float *lambda, ccq_dtype in_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    if (T > 0) {
+        st = check_ptrs("q,k,v,g,beta,lambda,o", {q, k, v, g, beta, lambda, o}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        if (st != CCQ_OK) return st;
+    } else {
+        st = check_ptrs("", {}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        if (st != CCQ_OK) return st;
+    }
+    if (c.p.algo == CCQ_ALGO_CHUNKWISE)
+        return fail(CCQ_ERR_UNSUPPORTED, "chunkwise Gated DeltaNet kernel not built yet");
+    RecurrentArgs ra = {};
+    ra.backbone = 1; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
+    ra.in_dtype = in_dtype; ra.gate_dtype = CCQ_FP32;
+    ra.l2norm = c.p.l2norm_qk; ra.centered = c.p.centered; ra.scale = c.scale;
+    ra.q = q; ra.k = k; ra.v = v; ra.gate = g; ra.beta = beta; ra.lambda = lambda;
+    ra.S0 = S0; ra.C0 = C0; ra.m0 = m0; ra.t0 = t0;
+    ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT; ra.tT = tT;
+    return run_recurrent(ra, static_cast<cudaStream_t>(stream));
+}
+
+ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,
+                           const void *gate, const float *beta, const float *lambda,
+                           ccq_dtype in_dtype, ccq_dtype gate_dtype, float *S, float *C,
+                           float *m, int64_t *t, void *o, int B, int H, int Dk, int Dv,
+                           const ccq_params *p, void *stream) {
+    Common c;
+    ccq_status st = check_common(p, B, 1, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (backbone != 0 && backbone != 1) return fail(CCQ_ERR_INVALID_ARG, "backbone must be 0 (GLA) or 1 (GDN)");
+    if ((in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) || (gate_dtype != CCQ_BF16 && gate_dtype != CCQ_FP32))
+        return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    if (backbone == 1 && gate_dtype != CCQ_FP32)
+        return fail(CCQ_ERR_INVALID_ARG, "Gated DeltaNet decay must be fp32");
+    if (backbone == 1) st = check_ptrs("q,k,v,gate,beta,lambda,S,C,m,t,o", {q, k, v, gate, beta, lambda, S, C, m, t, o}, {});
+    else st = check_ptrs("q,k,v,gate,lambda,S,C,m,t,o", {q, k, v, gate, lambda, S, C, m, t, o}, {});
+    if (st != CCQ_OK) return st;
+    RecurrentArgs ra = {};
+    ra.backbone = backbone; ra.B = B; ra.T = 1; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
+    ra.in_dtype = in_dtype; ra.gate_dtype = gate_dtype;
+    ra.l2norm = c.p.l2norm_qk; ra.centered = c.p.centered; ra.scale = c.scale;
+    ra.q = q; ra.k = k; ra.v = v; ra.gate = gate; ra.beta = beta; ra.lambda = lambda;
+    ra.S0 = S; ra.C0 = C; ra.m0 = m; ra.t0 = t;
+    ra.o = o; ra.ST = S; ra.CT = C; ra.mT = m; ra.tT = t;
+    return run_recurrent(ra, static_cast<cudaStream_t>(stream));
+}
+
+ccq_status ccq_device_status(void *stream) {
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    int v = 0;
+    e = cudaMemcpyFromSymbol(&v, ccq::g_status, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "read device status");
+    if (v != 0) {
+        const int zero = 0;
+        e = cudaMemcpyToSymbol(ccq::g_status, &zero, sizeof(int));
+        if (e != cudaSuccess) return cuda_fail(e, "clear device status");
+        return fail(CCQ_ERR_TIMEOUT, "device status %d: an in-kernel wait gave up", v);
+    }
+    return CCQ_OK;
+}
+
+}  // extern "C"

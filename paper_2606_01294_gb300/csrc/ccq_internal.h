@@ -1,0 +1,65 @@
+// ccq_internal.h -- launch descriptors shared by the C ABI and the kernels.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace ccq {
+
+// Arguments of the token-by-token kernel (ccq_recurrent.cu).  dtype codes
+// follow ccq_dtype (0 = bf16, 1 = fp32).
+struct RecurrentArgs {
+    int backbone;  // 0 GLA, 1 Gated DeltaNet
+    int B, T, H, Dk, Dv;
+    int in_dtype, gate_dtype;
+    int l2norm, centered;
+    float scale;
+    const void *q, *k, *v, *gate;
+    const float *beta, *lambda;
+    const float *S0, *C0, *m0;
+    const int64_t *t0;
+    void *o;
+    float *ST, *CT, *mT;
+    int64_t *tT;
+};
+
+cudaError_t launch_recurrent(const RecurrentArgs &a, cudaStream_t s);
+
+// Arguments of the chunkwise tensor-core kernels (Dk = Dv = 128, chunk 64,
+// bf16 q/k/v/o).
+struct ChunkArgs {
+    int B, T, H;
+    int gate_dtype;  // GLA gate: 0 bf16, 1 fp32
+    int l2norm, centered;
+    float scale;
+    const float *lambda;
+    const float *g, *beta;  // Gated DeltaNet scalar log-decay and beta
+    const float *S0, *C0, *m0;
+    const int64_t *t0;
+    __nv_bfloat16 *o;
+    float *ST, *CT, *mT;
+    int64_t *tT;
+    int *status;  // device status word (bounded-wait give-ups)
+};
+
+// Device address of the library's status word on the current device.
+int *device_status_word();
+
+// Tensor maps of q, k, v (and the GLA gate) viewed as 4-D [B][T][H][D]
+// tensors, so that rows past T load as zeros.
+struct ChunkMaps {
+    CUtensorMap q, k, v, g;
+};
+
+cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
+
+// Encode the tensor map of a [B][T][H][D] tensor with a (box_inner x 1 x 64 x 1)
+// box.  swizzle128 selects the 128-byte swizzle (bf16 MMA operands, box_inner
+// 64); otherwise the box lands as a plain row-major [64][box_inner] array.
+// Returns false when the driver entry point is missing or rejects the map.
+bool make_token_map(CUtensorMap *map, const void *base, int elem_bytes, int B, int T, int H,
+                    int D, int box_inner, bool swizzle128);
+
+}  // namespace ccq

@@ -20,7 +20,9 @@ the order q, k, v, gate, beta, lambda, then cast to the requested dtype):
                  U a fixed random orthonormal d x 16 basis, z ~ N(0, I_16),
                  eps ~ N(0, I_d), m0 a fixed random vector of norm 0.5 -- a
                  low-rank key spread with a non-zero mean, so Sigma_t is large and
-                 the mean term matters.
+                 the mean term matters; or "lowrank": k = normalise(U z + 0.1 eps)
+                 with a fixed orthonormal d x 2 basis U, so Sigma_t has two
+                 eigenvalues near 1/2 and the CCQ correction is large.
 """
 from __future__ import annotations
 
@@ -45,6 +47,14 @@ def _structured_keys(gen, B, T, H, Dk, rank=16):
     z = torch.randn(B, T, H, U.shape[1], generator=gen)
     eps = torch.randn(B, T, H, Dk, generator=gen)
     return m0 + z @ U.T + 0.25 * eps
+
+
+def _lowrank_keys(gen, B, T, H, Dk, rank=2):
+    basis_gen = torch.Generator().manual_seed(104729)
+    U, _ = torch.linalg.qr(torch.randn(Dk, rank, generator=basis_gen))
+    z = torch.randn(B, T, H, rank, generator=gen)
+    eps = torch.randn(B, T, H, Dk, generator=gen)
+    return z @ U.T + 0.1 * eps
 
 
 def _lambda(gen, B, T, H, lam):
@@ -76,6 +86,8 @@ def make_inputs(backbone: int, B: int, T: int, H: int, Dk: int, Dv: int, *,
         k = torch.randn(B, T, H, Dk, generator=gen)
     elif keys == "structured":
         k = _structured_keys(gen, B, T, H, Dk)
+    elif keys == "lowrank":
+        k = _lowrank_keys(gen, B, T, H, Dk)
     else:
         raise ValueError(f"unknown key distribution {keys!r}")
     k = _normalise_rows(k)

@@ -1,0 +1,83 @@
+"""Host-side checks of the C ABI: the library loads without a GPU, exports
+every function include/*.h declares, and rejects bad arguments before any
+CUDA call is made."""
+import ctypes
+
+import pytest
+
+from paper_2606_01294_gb300 import _build, ccq
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return ccq.load_library()
+
+
+def test_library_exports_every_header_symbol(lib):
+    names = ccq.header_symbols()
+    assert {"ccq_gla_fwd", "ccq_gdn_fwd", "ccq_decode_step", "ccq_device_status",
+            "ccq_status_string", "ccq_last_error", "ccq_default_params"} <= set(names)
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in include/ but not exported"
+
+
+def test_default_params(lib):
+    p = ccq._Params()
+    lib.ccq_default_params(ctypes.byref(p))
+    assert (p.l2norm_qk, p.scale, p.centered, p.chunk, p.algo) == (1, 0.0, 1, 64, 0)
+
+
+def test_status_strings(lib):
+    for s in range(5):
+        assert lib.ccq_status_string(s)
+    assert b"unknown" in lib.ccq_status_string(99)
+
+
+def _gla(lib, ptrs=None, sizes=(1, 4, 1, 128, 128), p=None, dtypes=(0, 0)):
+    fake = ctypes.c_void_p(0x10000)  # aligned, never dereferenced on these paths
+    args = ptrs if ptrs is not None else [fake] * 5
+    return lib.ccq_gla_fwd(*args, *dtypes, *([None] * 4), fake, *([None] * 4),
+                           *sizes, ctypes.byref(p or ccq.params()), None)
+
+
+def test_rejects_null_and_misaligned_pointers(lib):
+    fake = ctypes.c_void_p(0x10000)
+    assert _gla(lib, [None] + [fake] * 4) == ccq.CCQ_ERR_INVALID_ARG
+    assert b"NULL" in lib.ccq_last_error()
+    assert _gla(lib, [ctypes.c_void_p(0x10002)] + [fake] * 4) == ccq.CCQ_ERR_INVALID_ARG
+    assert b"aligned" in lib.ccq_last_error()
+
+
+def test_rejects_bad_sizes_and_params(lib):
+    assert _gla(lib, sizes=(0, 4, 1, 128, 128)) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gla(lib, sizes=(1, -1, 1, 128, 128)) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gla(lib, sizes=(1, 4, 1, 96, 96)) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _gla(lib, sizes=(1, 4, 1, 128, 64)) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _gla(lib, p=ccq.params(chunk=32)) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _gla(lib, dtypes=(7, 0)) == ccq.CCQ_ERR_INVALID_ARG
+    bad = ccq.params()
+    bad.algo = 9
+    assert _gla(lib, p=bad) == ccq.CCQ_ERR_INVALID_ARG
+    # the chunkwise kernel needs bf16 and Dk = 128
+    assert _gla(lib, sizes=(1, 4, 1, 64, 64), p=ccq.params(algo="chunkwise")) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _gla(lib, dtypes=(1, 1), p=ccq.params(algo="chunkwise")) == ccq.CCQ_ERR_UNSUPPORTED
+
+
+def test_decode_rejects_bad_backbone_and_gate(lib):
+    fake = ctypes.c_void_p(0x10000)
+    p = ccq.params()
+    st = lib.ccq_decode_step(5, *([fake] * 6), 0, 0, *([fake] * 5), 1, 1, 128, 128, ctypes.byref(p), None)
+    assert st == ccq.CCQ_ERR_INVALID_ARG
+    st = lib.ccq_decode_step(1, *([fake] * 6), 0, 0, *([fake] * 5), 1, 1, 128, 128, ctypes.byref(p), None)
+    assert st == ccq.CCQ_ERR_INVALID_ARG  # GDN decay must be fp32
+    st = lib.ccq_decode_step(1, fake, fake, fake, fake, None, fake, 0, 1, *([fake] * 5), 1, 1, 128, 128,
+                             ctypes.byref(p), None)
+    assert st == ccq.CCQ_ERR_INVALID_ARG  # GDN needs beta
+
+
+def test_binding_refuses_cpu_tensors():
+    import torch
+    x = torch.zeros(1, 4, 1, 128, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="CUDA"):
+        ccq.gla_fwd(x, x, x, x, torch.zeros(1, 4, 1))
