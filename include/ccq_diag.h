@@ -13,16 +13,18 @@ extern "C" {
 #endif
 
 /*
- * D = A B on one CTA through the same shared-memory tiles, descriptors and
+ * A B on one CTA through the same shared-memory tiles, descriptors and
  * tcgen05.mma sequence as the CCQ kernels.
- *   A  device bf16 [128][K] row-major;  B device bf16 [K][N] row-major;
- *   D  device fp32 [128][N] row-major (written).
- *   N in {64, 128}; K in {64, 128}; a_mn / b_mn = 1 stage that operand
- *   MN-major in shared memory, 0 = K-major.
+ *   A  device bf16 [M][K] row-major;  B device bf16 [K][N] row-major;
+ *   D  device fp32 [128][N] row-major: the raw accumulator, TMEM lane by
+ *      TMEM lane (for M = 128 lane i holds row i); lanes the MMA leaves
+ *      untouched read back as NaN.
+ *   M in {64, 128}; N in {64, 128}; K in {64, 128}; a_mn / b_mn = 1 stage that
+ *   operand MN-major in shared memory, 0 = K-major (M = 64 needs a_mn = 0).
  * Asynchronous on `stream`; CCQ_ERR_UNSUPPORTED for other shapes.
  */
-CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *D, int N, int K, int a_mn,
-                                int b_mn, void *stream);
+CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *D, int M, int N, int K,
+                                int a_mn, int b_mn, void *stream);
 
 #ifdef __cplusplus
 }

@@ -1,9 +1,10 @@
 // ccq_diag.cu -- layout self-test of the tensor-core building blocks.
 //
-// One CTA stages A (M=128 x K) and B (K x N) from global memory into the same
+// One CTA stages A (M x K, M in {64, 128}) and B (K x N) from global memory into the same
 // 128-byte-swizzled T64 tiles the CCQ kernels use -- K-major or MN-major for
 // each operand -- issues the tcgen05.mma sequence over K with the kernels'
-// descriptors, and writes D = A B (fp32) back through tcgen05.ld.  The C ABI
+// descriptors, and dumps all 128 TMEM lanes x N columns of the accumulator
+// (lanes the MMA does not write read back as NaN) through tcgen05.ld.  The C ABI
 // entry point ccq_diag_mma (include/ccq_diag.h) lets tests check every
 // descriptor form against a plain matrix product.
 #include <cuda_bf16.h>
@@ -23,8 +24,8 @@ constexpr int kM = 128;
 // (tile bytes 16K); MN-major -> tiles [K rows][64 m] for each 64-wide M block
 // (tile bytes K*128).  B likewise with N in place of M.
 __global__ void __launch_bounds__(128, 1)
-diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int N, int K, int a_mn,
-                int b_mn, int *status) {
+diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int M, int N, int K,
+                int a_mn, int b_mn, int *status) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~static_cast<uintptr_t>(1023));
@@ -42,11 +43,11 @@ diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int N
         fence_barrier_init();
     }
     if (warp == 0) tmem_alloc(slot, 128);
-    // stage A (logical [128][K] row-major in global)
-    for (int e = tid; e < kM * K; e += 128) {
+    // stage A (logical [M][K] row-major in global)
+    for (int e = tid; e < M * K; e += 128) {
         const int m = e / K, k = e % K;
         uint32_t off;
-        if (!a_mn) off = (k >> 6) * 16384 + t64_offset(m, k & 63);
+        if (!a_mn) off = (k >> 6) * (M * 128) + t64_offset(m, k & 63);
         else off = (m >> 6) * (K * 128) + t64_offset(k, m & 63);
         *reinterpret_cast<__nv_bfloat16 *>(sa + off) = A[e];
     }
@@ -59,15 +60,25 @@ diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int N
         *reinterpret_cast<__nv_bfloat16 *>(sbm + off) = Bm[e];
     }
     fence_proxy_async_smem();
-    tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *slot;
+    {
+        // mark every TMEM lane / column first, so lanes the MMA does not write show NaN
+        float nanv[32];
+        for (int i = 0; i < 32; ++i) nanv[i] = __int_as_float(0x7fc00000);
+        for (int c = 0; c < N; c += 32)
+            tmem_st32(tbase + (static_cast<uint32_t>(32 * warp) << 16) + c, nanv);
+        tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
     if (tid == 0) {
-        const uint32_t idesc = make_idesc(128, N, a_mn, b_mn);
+        const uint32_t idesc = make_idesc(M, N, a_mn, b_mn);
         for (int k16 = 0; k16 < K / 16; ++k16) {
             const uint64_t ad = a_mn ? desc_mnmajor(sb, K * 128, k16)
-                                     : desc_kmajor(sb + (k16 >> 2) * 16384, k16 & 3);
+                                     : desc_kmajor(sb + (k16 >> 2) * (M * 128), k16 & 3);
             const uint64_t bd = b_mn ? desc_mnmajor(sb + 32768, K * 128, k16)
                                      : desc_kmajor(sb + 32768 + (k16 >> 2) * (N * 128), k16 & 3);
             mma_bf16(tbase, ad, bd, idesc, k16 != 0);
@@ -93,10 +104,11 @@ diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int N
 }  // namespace
 }  // namespace ccq
 
-extern "C" CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *D, int N, int K,
-                                           int a_mn, int b_mn, void *stream) {
+extern "C" CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *D, int M, int N,
+                                           int K, int a_mn, int b_mn, void *stream) {
     if (!A || !B || !D) return CCQ_ERR_INVALID_ARG;
-    if ((N != 64 && N != 128) || (K != 64 && K != 128) || (a_mn | b_mn) > 1 || a_mn < 0 || b_mn < 0)
+    if ((M != 64 && M != 128) || (N != 64 && N != 128) || (K != 64 && K != 128) ||
+        (a_mn | b_mn) > 1 || a_mn < 0 || b_mn < 0 || (M == 64 && a_mn))
         return CCQ_ERR_UNSUPPORTED;
     int *status = ccq::device_status_word();
     if (!status) return CCQ_ERR_CUDA;
@@ -105,7 +117,7 @@ extern "C" CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *
         cudaSuccess)
         return CCQ_ERR_CUDA;
     ccq::diag_mma_kernel<<<1, 128, smem, static_cast<cudaStream_t>(stream)>>>(
-        static_cast<const __nv_bfloat16 *>(A), static_cast<const __nv_bfloat16 *>(B), D, N, K, a_mn,
-        b_mn, status);
+        static_cast<const __nv_bfloat16 *>(A), static_cast<const __nv_bfloat16 *>(B), D, M, N, K,
+        a_mn, b_mn, status);
     return cudaGetLastError() == cudaSuccess ? CCQ_OK : CCQ_ERR_CUDA;
 }

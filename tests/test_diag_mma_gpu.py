@@ -16,13 +16,13 @@ pytestmark = pytest.mark.gpu
                                            (1, 0, 128, 128)])
 def test_mma_layout(a_mn, b_mn, N, K):
     lib = ccq.load_library()
-    lib.ccq_diag_mma.argtypes = [ctypes.c_void_p] * 3 + [ctypes.c_int] * 4 + [ctypes.c_void_p]
+    lib.ccq_diag_mma.argtypes = [ctypes.c_void_p] * 3 + [ctypes.c_int] * 5 + [ctypes.c_void_p]
     lib.ccq_diag_mma.restype = ctypes.c_int
     g = torch.Generator().manual_seed(N * 7 + K + 3 * a_mn + b_mn)
     A = torch.randn(128, K, generator=g).to(torch.bfloat16).cuda()
     B = torch.randn(K, N, generator=g).to(torch.bfloat16).cuda()
     D = torch.full((128, N), float("nan"), device="cuda")
-    st = lib.ccq_diag_mma(A.data_ptr(), B.data_ptr(), D.data_ptr(), N, K, a_mn, b_mn,
+    st = lib.ccq_diag_mma(A.data_ptr(), B.data_ptr(), D.data_ptr(), 128, N, K, a_mn, b_mn,
                           torch.cuda.current_stream().cuda_stream)
     assert st == 0
     ccq.device_status()
