@@ -16,9 +16,9 @@ extern "C" {
  * A B on one CTA through the same shared-memory tiles, descriptors and
  * tcgen05.mma sequence as the CCQ kernels.
  *   A  device bf16 [M][K] row-major;  B device bf16 [K][N] row-major;
- *   D  device fp32 [128][N] row-major: the raw accumulator, TMEM lane by
- *      TMEM lane (for M = 128 lane i holds row i); lanes the MMA leaves
- *      untouched read back as NaN.
+ *   D  device fp32 [128][N] row-major.  M = 128: the accumulator, TMEM lane i
+ *      holding row i.  M = 64: rows 0..63 of D = A B read back with the
+ *      16-lane split load the kernels use (rows 64..127 are not written).
  *   M in {64, 128}; N in {64, 128}; K in {64, 128}; a_mn / b_mn = 1 stage that
  *   operand MN-major in shared memory, 0 = K-major (M = 64 needs a_mn = 0).
  * Asynchronous on `stream`; CCQ_ERR_UNSUPPORTED for other shapes.

@@ -187,7 +187,8 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
         if (!make_token_map(&maps.q, q, 2, B, T, H, 128, 64, true) ||
             !make_token_map(&maps.k, k, 2, B, T, H, 128, 64, true) ||
             !make_token_map(&maps.v, v, 2, B, T, H, 128, 64, true) ||
-            !make_token_map(&maps.g, gk, geb, B, T, H, 128, 128, false))
+            !make_token_map(&maps.g, gk, geb, B, T, H, 128, 128, false) ||
+            !make_token_map(&maps.o, o, 2, B, T, H, 128, 64, true))
             return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
         ChunkArgs a = {};
         a.B = B; a.T = T; a.H = H;

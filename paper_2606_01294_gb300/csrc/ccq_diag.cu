@@ -18,8 +18,6 @@
 namespace ccq {
 namespace {
 
-constexpr int kM = 128;
-
 // A tile set: K-major -> tiles [128 rows (m)][64 k] for each 64-wide K block
 // (tile bytes 16K); MN-major -> tiles [K rows][64 m] for each 64-wide M block
 // (tile bytes K*128).  B likewise with N in place of M.
@@ -87,11 +85,28 @@ diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int M
     }
     mbar_wait(bar, 0, abort_flag, status);
     tc_fence_after();
-    const int row = 32 * warp + lane;
-    for (int c = 0; c < N; c += 32) {
+    if (M == 128 || N == 0) {
+        const int row = 32 * warp + lane;
+        for (int c = 0; c < N; c += 32) {
+            float x[32];
+            tmem_ld32(tbase + (static_cast<uint32_t>(32 * warp) << 16) + c, x);
+            for (int i = 0; i < 32; ++i) D[row * N + c + i] = x[i];
+        }
+    } else {
+        // M = 64: rows 16w..16w+15 of warp w, read with the 16-lane split load;
+        // D rows 64..127 are left untouched
+        const int row = 16 * warp + (lane & 15), half = lane >> 4;
+        const uint32_t ta = tbase + (static_cast<uint32_t>(32 * warp) << 16);
         float x[32];
-        tmem_ld32(tbase + (static_cast<uint32_t>(32 * warp) << 16) + c, x);
-        for (int i = 0; i < 32; ++i) D[row * N + c + i] = x[i];
+        if (N == 64) {
+            tmem_ld16x2_32<32>(ta, x);
+            for (int i = 0; i < 32; ++i) D[row * N + 32 * half + i] = x[i];
+        } else {
+            tmem_ld16x2_32<64>(ta, x);
+            for (int i = 0; i < 32; ++i) D[row * N + 64 * half + i] = x[i];
+            tmem_ld16x2_32<64>(ta + 32, x);
+            for (int i = 0; i < 32; ++i) D[row * N + 64 * half + 32 + i] = x[i];
+        }
     }
     tc_fence_before();
     __syncthreads();

@@ -1,34 +1,49 @@
 // ccq_gla_chunk.cu -- chunkwise CCQ-GLA forward on sm_103a tensor cores.
 //
-// One CTA per (batch, head) walks the chunks of Algorithm 1 (chunk C = 64,
-// Dk = Dv = 128).  The two recurrent states live in tensor memory as fp32
+// One CTA per (batch, head) walks the 64-token chunks of Algorithm 1
+// (Dk = Dv = 128).  The two recurrent states stay in tensor memory as fp32
 // accumulators for the whole sequence:
-//   S   [Dk lanes][Dv cols]  the GLA state (transposed, S[a][e])
-//   SK  [Dk lanes][Dk cols]  the undecayed key second-moment sum S^K (App. B)
-// and every product of the chunk is a tcgen05.mma with bf16 operands staged
-// in 128-byte-swizzled shared-memory tiles (TMA-loaded for q, k, v):
+//   S   [Dk lanes][Dv cols]   the GLA state, transposed (S[a][e]), kept as
+//                             X = Diag(e^{Gmid - Gtot}) S between chunks
+//   SK  [Dk lanes][Dk cols]   the undecayed key second-moment sum S^K (App. B)
+// and every product of a chunk is a tcgen05.mma with bf16 operands in
+// 128-byte-swizzled shared-memory tiles (q, k, v, gates loaded by TMA):
 //
-//   G2  Sc   = Qbar Kbar^T                    (CCQ intra-chunk scores)
-//   G1  P    = Qbar S^K                       (CCQ inter-chunk read, P^prev)
-//   G8  S^K += Kbar^T Kbar                    (second-moment update)
-//   G3  P   += W' Kbar,  W'_ij = [j<=i](Sc_ij - c_i)   (P^intra with the mean fold)
-//   G4  A    = Qg Kg^T                        (gated GLA scores)
-//   G6  O    = Qg (Diag(e^{Gmid}) S)          (GLA inter-chunk read)
-//   G5  O   += [j<=i] A  V                    (GLA intra-chunk read)
-//   G7  S    = Diag(e^{Gtot}) S + Ku^T V      (GLA state update)
+//   group A  G2  Sc  = Q Kbar^T                   (CCQ intra scores, raw q)
+//            G1  P   = Q S^K                      (CCQ inter read, App. B P^prev)
+//   group B  G3  P  += W Kbar                     (CCQ intra read with the mean fold)
+//   group C  G4  A   = Qg Kg^T                    (gated GLA scores)
+//            G6  O   = Qg Ssnap                   (GLA inter read)
+//   group S  G7  X  += Kg^T V                     (GLA state update)
+//            G8  S^K += Kbar^T Kbar               (second-moment update)
+//   group D  G5  O  += [j<=i] A V                 (GLA intra read)
+// Group S is issued right after group C: it runs under the mask epilogue and
+// releases the next chunk's state snapshot early.
 //
-// The CCQ mean term is folded into the intra product: with
-// cq_i = CumK_i . qbar_i = M . qbar_i + sum_{j<=i} Sc_ij and c_i = cq_i / t_i,
-//   D (P^prev + P^intra) - MeanCorr = (P_i - c_i M) / t_i          (App. B)
-// where P_i = S^K qbar_i + sum_{j<=i} (Sc_ij - c_i) kbar_j.  Then
-//   q_clean_i = qbar_i - lambda_i (P_i - c_i M) / t_i               (Eq. clean)
-// and the GLA chunk form reads with q_clean scaled by exp(G_i - Gmid) and keys
-// scaled by exp(Gmid - G_j), Gmid the cumulative gate at the chunk midpoint
-// (halves the exponent range), the state snapshot scaled by exp(Gmid).
+// Notation (chunk r, positions t_i = t_r + i + 1, rq_i = 1/|q_i|):
+//   cq_i = CumK_i . qbar_i = M . qbar_i + rq_i sum_{j<=i} Sc_ij,   c_i = cq_i / t_i,
+//   W_ij = [j<=i] (Sc_ij - c_i |q_i|), so that rq_i P_i = S^K qbar_i
+//   + sum_{j<=i} (qbar_i . kbar_j - c_i) kbar_j and
+//   D (P^prev + P^intra) - MeanCorr = (rq_i P_i - c_i M) / t_i     (App. B, re-associated)
+//   q_clean_i = qbar_i - lambda_i (rq_i P_i - c_i M) / t_i          (Eq. clean)
+// GLA gates are measured from the chunk midpoint Gmid: Qg = q_clean * e^{G - Gmid},
+// Kg = kbar * e^{Gmid - G}, Ssnap = e^{Gmid} S_r, and S_{r+1} = e^{Gtot - Gmid} X_{r+1}
+// (that factor is applied at the next snapshot).
 //
-// Rows past T load as zeros through the tensor maps: zero keys add nothing to
-// any sum and zero gates leave the cumulative gate unchanged, so the ragged
-// tail needs no special arithmetic; only its output rows are not stored.
+// Warp specialisation (384 threads):
+//   WG0 (warps 0-3)  the dependent chain of chunk r: MMA issue (thread 0) and
+//                    the epilogues W, q_clean, mask of A, output (staged in the
+//                    chunk's Q tile and written by a TMA store).  The 64-row
+//                    products are M = 64 MMAs: rows 16q..16q+15 land in TMEM
+//                    lanes 32q..32q+15, so each warp owns 16 rows.
+//   WG1 (warps 4-7)  prep of chunk r+1 while WG0 runs chunk r: gate cumsum,
+//                    row norms, kbar, Kg, e^{G-Gmid}, M . qbar, lambda.
+//   WG2 (warps 8-11) state snapshot of chunk r+1 (bf16 copies of S^K and
+//                    e^{Gmid} S, rescaling X in TMEM) and the final states.
+// Per-chunk tiles are double-buffered (two slots); v is single-buffered and
+// reloaded as soon as the chunk's last product that reads it completes.
+// Rows past T load as zeros: zero keys add nothing to any sum, zero gates keep
+// the cumulative gate, so the ragged tail needs no special arithmetic.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -43,532 +58,543 @@ namespace {
 
 constexpr int kC = 64;         // chunk length
 constexpr int kD = 128;        // Dk = Dv
-constexpr int kThreads = 256;  // 8 warps (two warpgroups)
+constexpr int kThreads = 384;  // three warpgroups
 
 // ---- shared memory map (bytes from the 1024-aligned base)
-constexpr uint32_t OFF_Q = 0;        // 16K  q raw -> qbar -> q_clean*e^{G-Gmid} ([64][128], 2 T64 tiles of 8K)
-constexpr uint32_t OFF_K = 16384;    // 16K  k raw -> kbar
-constexpr uint32_t OFF_V = 32768;    // 16K  v
-constexpr uint32_t OFF_KG = 49152;   // 16K  kbar * e^{Gmid - G}
-constexpr uint32_t OFF_KU = 65536;   // 16K  kbar * e^{Gtot - G}
-constexpr uint32_t OFF_W = 81920;    // 8K   W' then masked A ([64][64], one T64 tile)
-constexpr uint32_t OFF_SK = 90112;   // 32K  bf16 snapshot of S^K ([128][128], 2 T64 tiles of 16K)
-constexpr uint32_t OFF_S = 122880;   // 32K  bf16 snapshot of e^{Gmid} S ([128][128], 2 T64 tiles of 16K)
-constexpr uint32_t OFF_G = 155648;   // 32K  raw gates, plain [64][128] (bf16 or fp32)
-constexpr uint32_t OFF_EG = 188416;  // 17K  e^{G - Gmid} bf16, [64][kEgStride]
-constexpr int kEgStride = 136;       // padded row (272 B) -> conflict-free row reads
-constexpr uint32_t OFF_MISC = OFF_EG + 64 * kEgStride * 2;  // 205824
-// misc (fp32 unless noted)
-constexpr uint32_t M_M = 0;           // [128] key sum M (chunk start)
-constexpr uint32_t M_DM = 512;        // [2][128] partial key sums of the chunk
-constexpr uint32_t M_GP = 1536;       // [2][128] partial gate sums
-constexpr uint32_t M_EGT = 2560;      // [128] e^{Gtot}
-constexpr uint32_t M_EGM = 3072;      // [128] e^{Gmid}
-constexpr uint32_t M_RQ = 3584;       // [64] 1/|q_i|
-constexpr uint32_t M_RK = 3840;       // [64] 1/|k_j|
-constexpr uint32_t M_MQ = 4096;       // [64] M . qbar_i
-constexpr uint32_t M_LAM = 4352;      // [64] lambda_i
-constexpr uint32_t M_CV = 4608;       // [64] c_i
-constexpr uint32_t M_PART = 4864;     // [2][64] masked row sums of Sc
-constexpr uint32_t M_BAR = 5376;      // 5 mbarriers (8 B each)
-constexpr uint32_t M_TMEM = 5424;     // u32 TMEM base
-constexpr uint32_t M_ABORT = 5428;    // int abort flag
-constexpr uint32_t kMiscBytes = 5504;
+// two slots of per-chunk tiles, each [64 rows][128 cols] bf16 as two T64 tiles of 8 KB:
+constexpr uint32_t SLOT_BYTES = 65536;
+constexpr uint32_t SO_Q = 0;       // raw q, then q_clean * e^{G - Gmid}
+constexpr uint32_t SO_K = 16384;   // raw k, then kbar
+constexpr uint32_t SO_KG = 32768;  // raw gates land here (bf16: 16 KB, fp32: KG+EG 32 KB); then Kg
+constexpr uint32_t SO_EG = 49152;  // e^{G - Gmid}
+constexpr uint32_t OFF_V = 131072;   // 16K  v
+constexpr uint32_t OFF_W = 147456;   // 8K   W, then the masked A ([64][64], one T64 tile)
+constexpr uint32_t OFF_SK = 155648;  // 32K  bf16 S^K ([128][128], two T64 tiles of 16 KB)
+constexpr uint32_t OFF_S = 188416;   // 32K  bf16 e^{Gmid} S ([128][128], two T64 tiles of 16 KB)
+constexpr uint32_t OFF_MISC = 221184;
+// misc: per-slot arrays (2560 B per slot)
+constexpr uint32_t MS_BYTES = 2560;
+constexpr uint32_t MS_RQ = 0;      // [64] 1/|q_i|
+constexpr uint32_t MS_MQ = 256;    // [64] M . qbar_i
+constexpr uint32_t MS_LAM = 512;   // [64] lambda_i
+constexpr uint32_t MS_RK = 768;    // [64] 1/|k_j|
+constexpr uint32_t MS_EGM = 1024;  // [128] e^{Gmid}
+constexpr uint32_t MS_F = 1536;    // [128] e^{Gtot - Gmid}
+constexpr uint32_t MS_MST = 2048;  // [128] key sum M at the chunk start
+constexpr uint32_t M_DMP = 5120;   // [2][128] partial key sums of the chunk (prep)
+constexpr uint32_t M_DMPREV = 6144;  // [128] key sum of the previous chunk
+constexpr uint32_t M_GT0 = 6656;   // [128] gate sum over tokens 0..31
+constexpr uint32_t M_CV = 7168;    // [64] c_i
+constexpr uint32_t M_BAR = 7424;   // 13 mbarriers
+constexpr uint32_t M_TMEM = 7528;
+constexpr uint32_t M_ABORT = 7532;
+constexpr uint32_t kMiscBytes = 7680;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;  // + alignment slack
-
-static_assert(OFF_MISC == 205824, "smem map");
 static_assert(kSmemBytes <= 232448, "exceeds the 227 KB per-CTA limit");
+
+enum {
+    BAR_IN0 = 0, BAR_IN1 = 1, BAR_V = 2, BAR_GA = 3, BAR_GB = 4, BAR_GC = 5, BAR_GD = 6,
+    BAR_PREP0 = 7, BAR_PREP1 = 8, BAR_SNAP = 9, BAR_GS = 10, BAR_GA2 = 11, BAR_GC2 = 12,
+    kNumBars = 13
+};
 
 // ---- tensor memory columns
 constexpr uint32_t TM_S = 0;     // 128 cols
 constexpr uint32_t TM_SK = 128;  // 128 cols
-constexpr uint32_t TM_PO = 256;  // 128 cols: P, then O
-constexpr uint32_t TM_SA = 384;  // 64 cols: Sc, then A
+constexpr uint32_t TM_PO = 256;  // 128 cols: P, then O (M = 64 layout)
+constexpr uint32_t TM_SA = 384;  // 64 cols: Sc, then A (M = 64 layout)
 constexpr uint32_t kTmemCols = 512;
 
-// ---- instruction descriptors
-constexpr uint32_t ID_N64_KK = make_idesc(128, 64, 0, 0);
-constexpr uint32_t ID_N128_KK = make_idesc(128, 128, 0, 0);
-constexpr uint32_t ID_N128_KM = make_idesc(128, 128, 0, 1);
-constexpr uint32_t ID_N128_MM = make_idesc(128, 128, 1, 1);
+constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
+constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
+constexpr uint32_t ID_64x128_KM = make_idesc(64, 128, 0, 1);
+constexpr uint32_t ID_128x128_MM = make_idesc(128, 128, 1, 1);
 
-enum { BAR_Q = 0, BAR_K = 1, BAR_V = 2, BAR_G = 3, BAR_MMA = 4 };
-
-__device__ __forceinline__ float bf(const uint8_t *p) {
-    return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(p));
-}
-__device__ __forceinline__ void st_bf(uint8_t *p, float x) {
-    *reinterpret_cast<__nv_bfloat16 *>(p) = __float2bfloat16_rn(x);
+__device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chunk, const float *w) {
+    uint4 u;
+    u.x = pack_bf16(w[0], w[1]);
+    u.y = pack_bf16(w[2], w[3]);
+    u.z = pack_bf16(w[4], w[5]);
+    u.w = pack_bf16(w[6], w[7]);
+    *reinterpret_cast<uint4 *>(tile + t64_chunk(row, chunk)) = u;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
 gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                  const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_g,
-                 const ChunkArgs a) {
+                 const __grid_constant__ CUtensorMap map_o, const ChunkArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                               ~static_cast<uintptr_t>(1023));
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
-    float *Mv = reinterpret_cast<float *>(misc + M_M);
-    float *dm = reinterpret_cast<float *>(misc + M_DM);
-    float *gp = reinterpret_cast<float *>(misc + M_GP);
-    float *egt = reinterpret_cast<float *>(misc + M_EGT);
-    float *egm = reinterpret_cast<float *>(misc + M_EGM);
-    float *rq = reinterpret_cast<float *>(misc + M_RQ);
-    float *rk = reinterpret_cast<float *>(misc + M_RK);
-    float *mq = reinterpret_cast<float *>(misc + M_MQ);
-    float *lam = reinterpret_cast<float *>(misc + M_LAM);
+    float *dmp = reinterpret_cast<float *>(misc + M_DMP);
+    float *dmprev = reinterpret_cast<float *>(misc + M_DMPREV);
+    float *gt0 = reinterpret_cast<float *>(misc + M_GT0);
     float *cv = reinterpret_cast<float *>(misc + M_CV);
-    float *part = reinterpret_cast<float *>(misc + M_PART);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
+    auto slot_f = [&](int s, uint32_t off) {
+        return reinterpret_cast<float *>(misc + s * MS_BYTES + off);
+    };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int wg = tid >> 7, wt = tid & 127;
     const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H;
     const int NC = (T + kC - 1) / kC;
     const bool gate_f32 = a.gate_dtype != 0;
     const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
-
-    // lane quarter (TMEM lanes 32*lq..) and column half of this warp
-    const int lq = warp & 3, ch = warp >> 2;
-    const int row = 32 * lq + lane;  // TMEM lane: state row a, or chunk row i
+    const int64_t t0 = a.t0 ? a.t0[b] : 0;
+    int *status = a.status;
 
     if (tid == 0) {
-        for (int i = 0; i < 5; ++i) mbar_init(&bar[i], 1);
+        for (int i = 0; i < kNumBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_k);
         tma_prefetch_desc(&map_v);
         tma_prefetch_desc(&map_g);
+        tma_prefetch_desc(&map_o);
     }
     if (warp == 0) tmem_alloc(tmem_slot, kTmemCols);
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
-    const uint32_t tl = tbase + (static_cast<uint32_t>(32 * lq) << 16);  // this warp's lane base
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * (warp & 3)) << 16);  // warp's lane quadrant
 
-    // ---- initial states into TMEM, M into shared memory
-    {
-        const size_t bhs = static_cast<size_t>(bh);
-        float x[32];
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            const int c0 = 64 * ch + 32 * half;
-            if (a.S0) {
-                const float4 *src = reinterpret_cast<const float4 *>(a.S0 + (bhs * kD + row) * kD + c0);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    float4 f = src[i];
-                    x[4 * i] = f.x; x[4 * i + 1] = f.y; x[4 * i + 2] = f.z; x[4 * i + 3] = f.w;
-                }
-            } else {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) x[i] = 0.f;
-            }
-            tmem_st32(tl + TM_S + c0, x);
-            if (a.C0) {
-                const float4 *src = reinterpret_cast<const float4 *>(a.C0 + (bhs * kD + row) * kD + c0);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    float4 f = src[i];
-                    x[4 * i] = f.x; x[4 * i + 1] = f.y; x[4 * i + 2] = f.z; x[4 * i + 3] = f.w;
-                }
-            } else {
-#pragma unroll
-                for (int i = 0; i < 32; ++i) x[i] = 0.f;
-            }
-            tmem_st32(tl + TM_SK + c0, x);
-        }
-        if (tid < kD) Mv[tid] = a.m0 ? a.m0[bhs * kD + tid] : 0.f;
-        tmem_wait_st();
-    }
-    int64_t tpos = a.t0 ? a.t0[b] : 0;  // tokens before the current chunk
-
-    auto issue_q = [&](int r) {
-        mbar_arrive_expect_tx(&bar[BAR_Q], 2 * 8192);
-        tma_load_4d(sm + OFF_Q, &map_q, &bar[BAR_Q], 0, h, r * kC, b);
-        tma_load_4d(sm + OFF_Q + 8192, &map_q, &bar[BAR_Q], 64, h, r * kC, b);
-    };
-    auto issue_k = [&](int r) {
-        mbar_arrive_expect_tx(&bar[BAR_K], 2 * 8192);
-        tma_load_4d(sm + OFF_K, &map_k, &bar[BAR_K], 0, h, r * kC, b);
-        tma_load_4d(sm + OFF_K + 8192, &map_k, &bar[BAR_K], 64, h, r * kC, b);
+    auto issue_in = [&](int r) {  // q, k, gates of chunk r into slot r & 1
+        const int s = r & 1;
+        uint8_t *base = sm + s * SLOT_BYTES;
+        uint64_t *bb = &bar[BAR_IN0 + s];
+        mbar_arrive_expect_tx(bb, 4 * 8192 + g_bytes);
+        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, r * kC, b);
+        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, r * kC, b);
+        tma_load_4d(base + SO_K, &map_k, bb, 0, h, r * kC, b);
+        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, r * kC, b);
+        tma_load_4d(base + SO_KG, &map_g, bb, 0, h, r * kC, b);
     };
     auto issue_v = [&](int r) {
         mbar_arrive_expect_tx(&bar[BAR_V], 2 * 8192);
         tma_load_4d(sm + OFF_V, &map_v, &bar[BAR_V], 0, h, r * kC, b);
         tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, r * kC, b);
     };
-    auto issue_g = [&](int r) {
-        mbar_arrive_expect_tx(&bar[BAR_G], g_bytes);
-        tma_load_4d(sm + OFF_G, &map_g, &bar[BAR_G], 0, h, r * kC, b);
-    };
-    if (tid == 0 && NC > 0) {
-        issue_q(0);
-        issue_k(0);
+
+    // ---- set-up: initial states into TMEM (WG2), key sum (WG1), first loads (thread 0)
+    if (wg == 2) {
+        const size_t bhs = static_cast<size_t>(bh);
+        const int row = 32 * (warp & 3) + lane;
+        for (int m = 0; m < 2; ++m) {
+            const float *src = m == 0 ? a.S0 : a.C0;
+            const uint32_t col0 = m == 0 ? TM_S : TM_SK;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                if (src) {
+                    const float4 *p4 = reinterpret_cast<const float4 *>(src + (bhs * kD + row) * kD + 32 * c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float4 f = p4[e];
+                        x[4 * e] = f.x; x[4 * e + 1] = f.y; x[4 * e + 2] = f.z; x[4 * e + 3] = f.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) x[e] = 0.f;
+                }
+                tmem_st32(tq + col0 + 32 * c, x);
+            }
+        }
+        tmem_wait_st();
+    } else if (wg == 1) {
+        slot_f(0, MS_MST)[wt] = a.m0 ? a.m0[static_cast<size_t>(bh) * kD + wt] : 0.f;
+        dmprev[wt] = 0.f;
+    } else if (tid == 0) {
+        issue_in(0);
         issue_v(0);
-        issue_g(0);
-    }
-    // lambda of the next chunk is prefetched into a register by warps 2-3
-    float lam_next = 0.f;
-    if (tid >= 64 && tid < 128) {
-        const int i = tid - 64;
-        lam_next = (i < T) ? a.lambda[(static_cast<size_t>(b) * T + i) * H + h] : 0.f;
     }
     tc_fence_before();
     __syncthreads();
 
-    uint32_t mma_par = 0;
-    for (int r = 0; r < NC; ++r) {
-        const int c0 = r * kC;
-        const int n = min(kC, T - c0);
-        const uint32_t tpar = static_cast<uint32_t>(r & 1);
-        const float tf = static_cast<float>(tpos);
-
-        // ================= P1a: row norms, M . qbar, lambda
-        mbar_wait(&bar[BAR_Q], tpar, abort_flag, a.status);
-        mbar_wait(&bar[BAR_K], tpar, abort_flag, a.status);
-        if (tid < 128) {
-            const bool isq = tid < 64;
-            const int i = tid & 63;
-            const uint8_t *base = sm + (isq ? OFF_Q : OFF_K);
-            float ss = 0.f, mdot = 0.f;
+    if (wg == 0) {
+        // =============================================================== WG0: the chain
+        const int i = 16 * warp + (lane & 15);  // chunk row owned by this thread
+        const int hf = lane >> 4;               // column half
+        // descriptor bases (start-address field advanced per K slice: +2 per 32 B)
+        const uint64_t dW = make_desc(sb + OFF_W, 16, 1024);
+        const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
+        const uint64_t dS = make_desc(sb + OFF_S, 16384, 1024);
+        const uint64_t dV = make_desc(sb + OFF_V, 8192, 1024);
+        for (int r = 0; r < NC; ++r) {
+            const int s = r & 1;
+            const uint32_t sp = (r >> 1) & 1, par = r & 1;
+            uint8_t *slot = sm + s * SLOT_BYTES;
+            const uint32_t ss = sb + s * SLOT_BYTES;
+            const int c0 = r * kC, n = min(kC, T - c0);
+            const float ti = static_cast<float>(t0 + c0 + i + 1);
+            mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
+            mbar_wait(&bar[BAR_SNAP], par, abort_flag, status);
+            const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
+            const uint64_t dK = make_desc(ss + SO_K, 16, 1024);
+            const uint64_t dKm = make_desc(ss + SO_K, 8192, 1024);
+            const uint64_t dKG = make_desc(ss + SO_KG, 16, 1024);
+            const uint64_t dKGm = make_desc(ss + SO_KG, 8192, 1024);
+            if (tid == 0 && !*abort_flag) {
+                if (r + 1 < NC) {
+                    tma_store_wait_read();  // the next slot's Q tile staged an earlier output
+                    issue_in(r + 1);
+                }
+                tc_fence_after();
+                // group A: G2 Sc = Q Kbar^T, G1 P = Q S^K
+                for (int k = 0; k < 8; ++k) {
+                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
+                }
+                mma_commit(&bar[BAR_GA]);  // Sc: the W epilogue needs only this
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
+                             dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
+                mma_commit(&bar[BAR_GA2]);
+            }
+            // ---- W epilogue: c_i and W_ij = [j<=i](Sc_ij - c_i |q_i|)
+            mbar_wait(&bar[BAR_GA], par, abort_flag, status);
+            tc_fence_after();
+            const float rqi = slot_f(s, MS_RQ)[i];
+            {
+                float sc[32];
+                tmem_ld16x2_32<32>(tq + TM_SA, sc);
+                float part = 0.f;
 #pragma unroll
-            for (int t64 = 0; t64 < 2; ++t64) {
+                for (int jj = 0; jj < 32; ++jj)
+                    if (32 * hf + jj <= i) part += sc[jj];
+                part += __shfl_xor_sync(0xffffffffu, part, 16);
+                const float cq = slot_f(s, MS_MQ)[i] + rqi * part;
+                const float c = a.centered ? cq / ti : 0.f;
+                if (hf == 0) cv[i] = c;
+                const float cn = c / rqi;  // c_i |q_i|
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    float w[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const int j = 32 * hf + 8 * q4 + e;
+                        w[e] = (j <= i) ? sc[8 * q4 + e] - cn : 0.f;
+                    }
+                    store_row_chunk(sm + OFF_W, i, 4 * hf + q4, w);
+                }
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(1, 128);
+            if (tid == 0 && !*abort_flag) {
+                tc_fence_after();
+                // group B: G3 P += W Kbar
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_PO, dW + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GB]);
+            }
+            // ---- q_clean epilogue (Eq. clean), scaled by e^{G - Gmid}, into the Q tile.
+            // q_clean e^{G-Gmid} = e^{G-Gmid} (rq q - (lambda/t)(rq P - c M)), computed as
+            // e^{G-Gmid} (rq (q - (lambda/t) P) + (lambda c / t) M).  The shared-memory
+            // operands are read while group B is still running.
+            {
+                uint8_t *qt = slot + SO_Q + hf * 8192;
+                const uint8_t *et = slot + SO_EG + hf * 8192;
+                const float *Mst = slot_f(s, MS_MST) + 64 * hf;
+                uint4 qraw[8], eraw[8];
 #pragma unroll
                 for (int cc = 0; cc < 8; ++cc) {
-                    const uint4 u = *reinterpret_cast<const uint4 *>(base + t64 * 8192 + t64_chunk(i, cc));
-                    float f[8];
-                    unpack_bf16x8(u, f);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        ss = fmaf(f[e], f[e], ss);
-                        mdot = fmaf(f[e], Mv[64 * t64 + 8 * cc + e], mdot);
-                    }
+                    qraw[cc] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, cc));
+                    eraw[cc] = *reinterpret_cast<const uint4 *>(et + t64_chunk(i, cc));
                 }
-            }
-            const float rn = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
-            if (isq) {
-                rq[i] = rn;
-                mq[i] = mdot * rn;
-            } else {
-                rk[i] = rn;
-            }
-            if (tid >= 64) lam[i] = lam_next;
-        }
-        __syncthreads();
-
-        // ================= P1b: gate cumsum (per key dim), normalised and gated operand tiles
-        mbar_wait(&bar[BAR_G], tpar, abort_flag, a.status);
-        {
-            const int d = tid & 127, th = tid >> 7;  // key dim, token half
-            float gl[32];
-            float run = 0.f;
+                const float lt = slot_f(s, MS_LAM)[i] / ti;  // lambda_i / t_i
+                mbar_wait(&bar[BAR_GA2], par, abort_flag, status);
+                mbar_wait(&bar[BAR_GB], par, abort_flag, status);
+                tc_fence_after();
+                const float cm = lt * cv[i];                  // lambda_i c_i / t_i
 #pragma unroll
-            for (int jj = 0; jj < 32; ++jj) {
-                const int j = 32 * th + jj;
-                const float g = gate_f32 ? reinterpret_cast<const float *>(sm + OFF_G)[j * kD + d]
-                                         : bf(sm + OFF_G + (j * kD + d) * 2);
-                run += g;
-                gl[jj] = run;
-            }
-            gp[th * kD + d] = run;
-            __syncthreads();  // all raw gates read; partial sums visible
-            if (tid == 0 && r + 1 < NC) issue_g(r + 1);
-            const float gmid = gp[d];               // cumulative gate after token 31
-            const float gtot = gp[d] + gp[kD + d];  // after token 63 (zero-filled past T)
-            const float off = th ? gmid : 0.f;
-            if (th == 0) {
-                egt[d] = __expf(gtot);
-                egm[d] = __expf(gmid);
-            }
-            const int tile = d >> 6, dc = d & 63;
-            float dmp = 0.f;
-#pragma unroll
-            for (int jj = 0; jj < 32; ++jj) {
-                const int j = 32 * th + jj;
-                const float G = gl[jj] + off;
-                const uint32_t o = tile * 8192 + t64_offset(j, dc);
-                const float kb = bf(sm + OFF_K + o) * rk[j];
-                const float qb = bf(sm + OFF_Q + o) * rq[j];
-                st_bf(sm + OFF_K + o, kb);
-                st_bf(sm + OFF_Q + o, qb);
-                st_bf(sm + OFF_KG + o, kb * __expf(gmid - G));
-                st_bf(sm + OFF_KU + o, kb * __expf(gtot - G));
-                st_bf(sm + OFF_EG + (j * kEgStride + d) * 2, __expf(G - gmid));
-                dmp += kb;
-            }
-            dm[th * kD + d] = dmp;
-        }
-        fence_proxy_async_smem();
-        __syncthreads();
-
-        // ================= P1c: snapshot S (scaled by e^{Gmid}) and S^K to bf16; decay S in TMEM
-        tc_fence_after();
-        {
-            const float sgm = egm[row], sgt = egt[row];
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                const uint32_t col = 64 * ch + 32 * half;
-                float x[32];
-                tmem_ld32(tl + TM_S + col, x);
-                uint8_t *dst = sm + OFF_S + ch * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    uint4 u;
-                    u.x = pack_bf16(x[8 * q4 + 0] * sgm, x[8 * q4 + 1] * sgm);
-                    u.y = pack_bf16(x[8 * q4 + 2] * sgm, x[8 * q4 + 3] * sgm);
-                    u.z = pack_bf16(x[8 * q4 + 4] * sgm, x[8 * q4 + 5] * sgm);
-                    u.w = pack_bf16(x[8 * q4 + 6] * sgm, x[8 * q4 + 7] * sgm);
-                    *reinterpret_cast<uint4 *>(dst + t64_chunk(row, 4 * half + q4)) = u;
-                }
-#pragma unroll
-                for (int i = 0; i < 32; ++i) x[i] *= sgt;
-                tmem_st32(tl + TM_S + col, x);
-                tmem_ld32(tl + TM_SK + col, x);
-                dst = sm + OFF_SK + ch * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    uint4 u;
-                    u.x = pack_bf16(x[8 * q4 + 0], x[8 * q4 + 1]);
-                    u.y = pack_bf16(x[8 * q4 + 2], x[8 * q4 + 3]);
-                    u.z = pack_bf16(x[8 * q4 + 4], x[8 * q4 + 5]);
-                    u.w = pack_bf16(x[8 * q4 + 6], x[8 * q4 + 7]);
-                    *reinterpret_cast<uint4 *>(dst + t64_chunk(row, 4 * half + q4)) = u;
-                }
-            }
-            tmem_wait_st();
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-
-        // ================= P2: G2 (Sc), G1 (P = Qbar S^K), G8 (S^K += Kbar^T Kbar)
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int kb = 0; kb < 2; ++kb)
-                for (int k16 = 0; k16 < 4; ++k16)
-                    mma_bf16(tbase + TM_SA, desc_kmajor(sb + OFF_Q + kb * 8192, k16),
-                             desc_kmajor(sb + OFF_K + kb * 8192, k16), ID_N64_KK, (kb | k16) != 0);
-            for (int kb = 0; kb < 2; ++kb)
-                for (int k16 = 0; k16 < 4; ++k16)
-                    mma_bf16(tbase + TM_PO, desc_kmajor(sb + OFF_Q + kb * 8192, k16),
-                             desc_kmajor(sb + OFF_SK + kb * 16384, k16), ID_N128_KK, (kb | k16) != 0);
-            for (int k16 = 0; k16 < 4; ++k16)
-                mma_bf16(tbase + TM_SK, desc_mnmajor(sb + OFF_K, 8192, k16),
-                         desc_mnmajor(sb + OFF_K, 8192, k16), ID_N128_MM, 1);
-            mma_commit(&bar[BAR_MMA]);
-        }
-
-        // ================= P3: masked row sums of Sc -> c_i; W'
-        mbar_wait(&bar[BAR_MMA], mma_par, abort_flag, a.status);
-        mma_par ^= 1;
-        tc_fence_after();
-        const bool rows_warp = lq < 2;  // warps 0,1,4,5 own chunk rows 0..63
-        float sc[32];
-        if (rows_warp) {
-            tmem_ld32(tl + TM_SA + 32 * ch, sc);
-            float s = 0.f;
-#pragma unroll
-            for (int jj = 0; jj < 32; ++jj)
-                if (32 * ch + jj <= row) s += sc[jj];
-            part[ch * 64 + row] = s;
-        }
-        __syncthreads();
-        if (rows_warp) {
-            const float ti = tf + static_cast<float>(row + 1);
-            const float cq = mq[row] + part[row] + part[64 + row];
-            const float c = a.centered ? cq / ti : 0.f;
-            if (ch == 0) cv[row] = c;
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-                float w[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int j = 32 * ch + 8 * q4 + e;
-                    w[e] = (j <= row) ? sc[8 * q4 + e] - c : 0.f;
-                }
-                uint4 u;
-                u.x = pack_bf16(w[0], w[1]);
-                u.y = pack_bf16(w[2], w[3]);
-                u.z = pack_bf16(w[4], w[5]);
-                u.w = pack_bf16(w[6], w[7]);
-                *reinterpret_cast<uint4 *>(sm + OFF_W + t64_chunk(row, 4 * ch + q4)) = u;
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-
-        // ================= P4: G3 (P += W' Kbar)
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int k16 = 0; k16 < 4; ++k16)
-                mma_bf16(tbase + TM_PO, desc_kmajor(sb + OFF_W, k16), desc_mnmajor(sb + OFF_K, 8192, k16),
-                         ID_N128_KM, 1);
-            mma_commit(&bar[BAR_MMA]);
-        }
-        // lambda prefetch for the next chunk (warps 2-3 are idle here)
-        if (tid >= 64 && tid < 128) {
-            const int i = tid - 64, tn = c0 + kC + i;
-            lam_next = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
-        }
-
-        // ================= P5: q_clean (Eq. clean), scaled by e^{G - Gmid}, into the Q tile
-        mbar_wait(&bar[BAR_MMA], mma_par, abort_flag, a.status);
-        mma_par ^= 1;
-        tc_fence_after();
-        if (tid == 0 && r + 1 < NC && !*abort_flag) issue_k(r + 1);  // Kbar no longer read
-        if (rows_warp) {
-            const float ti = tf + static_cast<float>(row + 1);
-            const float inv_t = 1.f / ti;
-            const float c = cv[row], lm = lam[row];
-            uint8_t *qt = sm + OFF_Q + ch * 8192;
-            const uint8_t *eg = sm + OFF_EG + (row * kEgStride + 64 * ch) * 2;
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                float p[32];
-                tmem_ld32(tl + TM_PO + 64 * ch + 32 * half, p);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const int cc = 4 * half + q4;
-                    uint4 *qp = reinterpret_cast<uint4 *>(qt + t64_chunk(row, cc));
-                    float qb[8], e8[8];
-                    unpack_bf16x8(*qp, qb);
-                    unpack_bf16x8(*reinterpret_cast<const uint4 *>(eg + 16 * cc), e8);
-                    float out[8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float corr = (p[8 * q4 + e] - c * Mv[64 * ch + 8 * cc + e]) * inv_t;
-                        out[e] = (qb[e] - lm * corr) * e8[e];
-                    }
-                    uint4 u;
-                    u.x = pack_bf16(out[0], out[1]);
-                    u.y = pack_bf16(out[2], out[3]);
-                    u.z = pack_bf16(out[4], out[5]);
-                    u.w = pack_bf16(out[6], out[7]);
-                    *qp = u;
-                }
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-
-        // ================= P6: G4 (A = Qg Kg^T), G6 (O = Qg Ssnap)
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int kb = 0; kb < 2; ++kb)
-                for (int k16 = 0; k16 < 4; ++k16)
-                    mma_bf16(tbase + TM_SA, desc_kmajor(sb + OFF_Q + kb * 8192, k16),
-                             desc_kmajor(sb + OFF_KG + kb * 8192, k16), ID_N64_KK, (kb | k16) != 0);
-            for (int k16 = 0; k16 < 8; ++k16)
-                mma_bf16(tbase + TM_PO, desc_kmajor(sb + OFF_Q + (k16 >> 2) * 8192, k16 & 3),
-                         desc_mnmajor(sb + OFF_S, 16384, k16), ID_N128_KM, k16 != 0);
-            mma_commit(&bar[BAR_MMA]);
-        }
-
-        // ================= P7: causal mask of A -> bf16 tile
-        mbar_wait(&bar[BAR_MMA], mma_par, abort_flag, a.status);
-        mma_par ^= 1;
-        tc_fence_after();
-        if (tid == 0 && r + 1 < NC && !*abort_flag) issue_q(r + 1);  // Q tile no longer read
-        if (rows_warp) {
-            tmem_ld32(tl + TM_SA + 32 * ch, sc);
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-                float w[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int j = 32 * ch + 8 * q4 + e;
-                    w[e] = (j <= row) ? sc[8 * q4 + e] : 0.f;
-                }
-                uint4 u;
-                u.x = pack_bf16(w[0], w[1]);
-                u.y = pack_bf16(w[2], w[3]);
-                u.z = pack_bf16(w[4], w[5]);
-                u.w = pack_bf16(w[6], w[7]);
-                *reinterpret_cast<uint4 *>(sm + OFF_W + t64_chunk(row, 4 * ch + q4)) = u;
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-
-        // ================= P8: G5 (O += A V), G7 (S += Ku^T V)
-        if (tid == 0 && !*abort_flag) {
-            mbar_wait(&bar[BAR_V], tpar, abort_flag, a.status);
-            tc_fence_after();
-            for (int k16 = 0; k16 < 4; ++k16)
-                mma_bf16(tbase + TM_PO, desc_kmajor(sb + OFF_W, k16), desc_mnmajor(sb + OFF_V, 8192, k16),
-                         ID_N128_KM, 1);
-            for (int k16 = 0; k16 < 4; ++k16)
-                mma_bf16(tbase + TM_S, desc_mnmajor(sb + OFF_KU, 8192, k16),
-                         desc_mnmajor(sb + OFF_V, 8192, k16), ID_N128_MM, 1);
-            mma_commit(&bar[BAR_MMA]);
-        }
-
-        // ================= P9: o = scale * O; M += chunk key sum; t += n
-        mbar_wait(&bar[BAR_MMA], mma_par, abort_flag, a.status);
-        mma_par ^= 1;
-        tc_fence_after();
-        if (tid == 0 && r + 1 < NC && !*abort_flag) issue_v(r + 1);  // V no longer read
-        if (rows_warp) {
-            const bool valid = row < n;
-            __nv_bfloat16 *dst = a.o + ((static_cast<size_t>(b) * T + c0 + row) * H + h) * kD + 64 * ch;
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                float x[32];
-                tmem_ld32(tl + TM_PO + 64 * ch + 32 * half, x);
-                if (valid) {
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    float p[32];
+                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, p);
 #pragma unroll
                     for (int q4 = 0; q4 < 4; ++q4) {
-                        uint4 u;
-                        u.x = pack_bf16(a.scale * x[8 * q4 + 0], a.scale * x[8 * q4 + 1]);
-                        u.y = pack_bf16(a.scale * x[8 * q4 + 2], a.scale * x[8 * q4 + 3]);
-                        u.z = pack_bf16(a.scale * x[8 * q4 + 4], a.scale * x[8 * q4 + 5]);
-                        u.w = pack_bf16(a.scale * x[8 * q4 + 6], a.scale * x[8 * q4 + 7]);
-                        reinterpret_cast<uint4 *>(dst)[4 * half + q4] = u;
+                        const int cc = 4 * h2 + q4;  // chunk inside the T64 tile
+                        float qr[8], eg[8], out[8];
+                        unpack_bf16x8(qraw[cc], qr);
+                        unpack_bf16x8(eraw[cc], eg);
+                        const float4 m0 = *reinterpret_cast<const float4 *>(Mst + 8 * cc);
+                        const float4 m1 = *reinterpret_cast<const float4 *>(Mst + 8 * cc + 4);
+                        const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+#pragma unroll
+                        for (int e = 0; e < 8; ++e)
+                            out[e] = eg[e] * fmaf(rqi, fmaf(-lt, p[8 * q4 + e], qr[e]), cm * mv[e]);
+                        store_row_chunk(qt, i, cc, out);
                     }
                 }
             }
-        } else {
-            const int d = 32 * (lq - 2) + 64 * ch + lane;  // warps 2,3,6,7 cover dims 0..127
-            Mv[d] += dm[d] + dm[kD + d];
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(1, 128);
+            if (tid == 0 && !*abort_flag) {
+                mbar_wait(&bar[BAR_V], par, abort_flag, status);
+                tc_fence_after();
+                // group C: G4 A = Qg Kg^T, G6 O = Qg Ssnap
+                for (int k = 0; k < 8; ++k) {
+                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                    mma_bf16(tbase + TM_SA, dQ + ko, dKG + ko, ID_64x64_KK, k != 0);
+                }
+                mma_commit(&bar[BAR_GC]);  // A: the mask epilogue needs only this
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dS + k * 128, ID_64x128_KM,
+                             k != 0);
+                mma_commit(&bar[BAR_GC2]);
+                // group S: G7 X += Kg^T V, G8 S^K += Kbar^T Kbar (needed only by the next snapshot)
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_S, dKGm + k * 128, dV + k * 128, ID_128x128_MM, 1);
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
+                mma_commit(&bar[BAR_GS]);
+            }
+            // ---- causal mask of A
+            mbar_wait(&bar[BAR_GC], par, abort_flag, status);
+            tc_fence_after();
+            {
+                float sc[32];
+                tmem_ld16x2_32<32>(tq + TM_SA, sc);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    float w[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const int j = 32 * hf + 8 * q4 + e;
+                        w[e] = (j <= i) ? sc[8 * q4 + e] : 0.f;
+                    }
+                    store_row_chunk(sm + OFF_W, i, 4 * hf + q4, w);
+                }
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(1, 128);
+            if (tid == 0 && !*abort_flag) {
+                tc_fence_after();
+                // group D: G5 O += A V
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_PO, dW + k * 2, dV + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GD]);
+            }
+            // ---- output
+            mbar_wait(&bar[BAR_GD], par, abort_flag, status);
+            tc_fence_after();
+            if (tid == 0 && r + 1 < NC && !*abort_flag) issue_v(r + 1);  // v no longer read
+            {
+                // stage o (bf16, swizzled) in the chunk's Q tile, then one TMA store;
+                // rows past T fall outside the tensor and are not written
+                uint8_t *ot = slot + SO_Q + hf * 8192;
+#pragma unroll
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    float x[32];
+                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, x);
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) x[e] *= a.scale;
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(ot, i, 4 * h2 + q4, x + 8 * q4);
+                }
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(1, 128);
+            if (tid == 0 && !*abort_flag) {
+                tma_store_4d(&map_o, slot + SO_Q, 0, h, c0, b);
+                tma_store_4d(&map_o, slot + SO_Q + 8192, 64, h, c0, b);
+                tma_store_commit();
+            }
         }
-        tpos += n;
-        tc_fence_before();
-        __syncthreads();
+        if (tid == 0) tma_store_wait_all();
+    } else if (wg == 1) {
+        // =============================================================== WG1: prep
+        const int p = wt & 63, th = wt >> 6;  // key-dim pair (2p, 2p+1), token half
+        const int d0 = 2 * p;
+        float lam_reg = 0.f;
+        if (wt < 64) lam_reg = (wt < T) ? a.lambda[(static_cast<size_t>(b) * T + wt) * H + h] : 0.f;
+        for (int r = 0; r < NC; ++r) {
+            const int s = r & 1;
+            const uint32_t sp = (r >> 1) & 1;
+            uint8_t *slot = sm + s * SLOT_BYTES;
+            float *Mst = slot_f(s, MS_MST);
+            mbar_wait(&bar[BAR_IN0 + s], sp, abort_flag, status);
+            // key sum at the chunk start and lambda of the chunk
+            if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
+            if (wt < 64) {
+                slot_f(s, MS_LAM)[wt] = lam_reg;
+                const int tn = (r + 1) * kC + wt;
+                lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+            }
+            named_bar(2, 128);
+            // row norms (thread = one row of q or k) and M . qbar
+            {
+                const int j = wt & 63;
+                const bool isq = wt < 64;
+                const uint8_t *base = slot + (isq ? SO_Q : SO_K);
+                float ss = 0.f, md = 0.f;
+#pragma unroll
+                for (int t64 = 0; t64 < 2; ++t64) {
+#pragma unroll
+                    for (int cc = 0; cc < 8; ++cc) {
+                        float f[8];
+                        unpack_bf16x8(*reinterpret_cast<const uint4 *>(base + t64 * 8192 + t64_chunk(j, cc)), f);
+                        const float4 m0 = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc);
+                        const float4 m1 = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc + 4);
+                        const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            ss = fmaf(f[e], f[e], ss);
+                            if (isq) md = fmaf(f[e], mv[e], md);
+                        }
+                    }
+                }
+                const float rn = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+                if (isq) {
+                    slot_f(s, MS_RQ)[j] = rn;
+                    slot_f(s, MS_MQ)[j] = md * rn;
+                } else {
+                    slot_f(s, MS_RK)[j] = rn;
+                }
+            }
+            // gate cumsum over this thread's 32 tokens for dims d0, d0+1
+            float g0[32], g1[32];
+            {
+                float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+                for (int jj = 0; jj < 32; ++jj) {
+                    const int j = 32 * th + jj;
+                    float x0, x1;
+                    if (gate_f32) {
+                        const float2 f2 = *reinterpret_cast<const float2 *>(slot + SO_KG + (j * kD + d0) * 4);
+                        x0 = f2.x; x1 = f2.y;
+                    } else {
+                        const __nv_bfloat162 b2 =
+                            *reinterpret_cast<const __nv_bfloat162 *>(slot + SO_KG + (j * kD + d0) * 2);
+                        const float2 f2 = __bfloat1622float2(b2);
+                        x0 = f2.x; x1 = f2.y;
+                    }
+                    r0 += x0; r1 += x1;
+                    g0[jj] = r0; g1[jj] = r1;
+                }
+                if (th == 0) {
+                    gt0[d0] = r0;
+                    gt0[d0 + 1] = r1;
+                }
+            }
+            named_bar(2, 128);  // raw gates all read, norms and gt0 visible
+            {
+                constexpr float kLog2e = 1.4426950408889634f;
+                const float gm0 = gt0[d0], gm1 = gt0[d0 + 1];   // Gmid
+                // exponents in log2 units relative to Gmid: x = (G - Gmid) log2(e)
+                const float o0 = ((th ? gm0 : 0.f) - gm0) * kLog2e, o1 = ((th ? gm1 : 0.f) - gm1) * kLog2e;
+                if (th == 1) {
+                    // f = e^{Gtot - Gmid} (gate sum of tokens 32..63), e^{Gmid}
+                    slot_f(s, MS_F)[d0] = fast_exp2(g0[31] * kLog2e);
+                    slot_f(s, MS_F)[d0 + 1] = fast_exp2(g1[31] * kLog2e);
+                    slot_f(s, MS_EGM)[d0] = fast_exp2(gm0 * kLog2e);
+                    slot_f(s, MS_EGM)[d0 + 1] = fast_exp2(gm1 * kLog2e);
+                }
+                const float *rk = slot_f(s, MS_RK);
+                const uint32_t tcol = (d0 >> 6) * 8192;
+                float dm0 = 0.f, dm1 = 0.f;
+#pragma unroll
+                for (int jj = 0; jj < 32; ++jj) {
+                    const int j = 32 * th + jj;
+                    const uint32_t off = tcol + t64_offset(j, d0 & 63);
+                    const float2 kr =
+                        __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(slot + SO_K + off));
+                    const float rkj = rk[j];
+                    const float k0 = kr.x * rkj, k1 = kr.y * rkj;
+                    const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
+                    *reinterpret_cast<uint32_t *>(slot + SO_K + off) = pack_bf16(k0, k1);
+                    *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
+                        pack_bf16(k0 * fast_exp2(-x0), k1 * fast_exp2(-x1));
+                    *reinterpret_cast<uint32_t *>(slot + SO_EG + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
+                    dm0 += k0;
+                    dm1 += k1;
+                }
+                dmp[th * kD + d0] = dm0;
+                dmp[th * kD + d0 + 1] = dm1;
+            }
+            fence_proxy_async_smem();
+            named_bar(2, 128);
+            dmprev[wt] = dmp[wt] + dmp[kD + wt];
+            named_bar(2, 128);
+            if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
+        }
+        // final key sum and position
+        if (NC > 0 && a.mT) {
+            const int sl = (NC - 1) & 1;
+            a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
+        }
+        if (a.tT && h == 0 && wt == 0) a.tT[b] = t0 + T;
+    } else {
+        // =============================================================== WG2: states
+        const int row = 32 * (warp & 3) + lane;  // state row a (key dim)
+        for (int r = 0; r < NC; ++r) {
+            const int s = r & 1;
+            const uint32_t sp = (r >> 1) & 1;
+            if (r > 0) mbar_wait(&bar[BAR_GS], (r - 1) & 1, abort_flag, status);
+            mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
+            tc_fence_after();
+            const float hs = (r > 0 ? slot_f(s ^ 1, MS_F)[row] : 1.f) * slot_f(s, MS_EGM)[row];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                tmem_ld32(tq + TM_S + 32 * c, x);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) x[e] *= hs;
+                uint8_t *tile = sm + OFF_S + (c >> 1) * 16384;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
+                tmem_st32(tq + TM_S + 32 * c, x);
+            }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                tmem_ld32(tq + TM_SK + 32 * c, x);
+                uint8_t *tile = sm + OFF_SK + (c >> 1) * 16384;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
+            }
+            tmem_wait_st();
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(3, 128);
+            if (wt == 0) mbar_arrive(&bar[BAR_SNAP]);
+        }
+        // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K
+        if (NC > 0) {
+            mbar_wait(&bar[BAR_GS], (NC - 1) & 1, abort_flag, status);
+            tc_fence_after();
+            const float fs = slot_f((NC - 1) & 1, MS_F)[row];
+            const size_t bhs = static_cast<size_t>(bh);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                tmem_ld32(tq + TM_S + 32 * c, x);
+                if (a.ST) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],
+                                             fs * x[4 * e + 3]);
+                }
+                tmem_ld32(tq + TM_SK + 32 * c, x);
+                if (a.CT) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.CT + (bhs * kD + row) * kD + 32 * c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+                }
+            }
+        }
     }
 
-    // ---- final states
-    tc_fence_after();
-    {
-        const size_t bhs = static_cast<size_t>(bh);
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            const int c0 = 64 * ch + 32 * half;
-            float x[32];
-            tmem_ld32(tl + TM_S + c0, x);
-            if (a.ST) {
-                float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + c0);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) dst[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
-            }
-            tmem_ld32(tl + TM_SK + c0, x);
-            if (a.CT) {
-                float4 *dst = reinterpret_cast<float4 *>(a.CT + (bhs * kD + row) * kD + c0);
-#pragma unroll
-                for (int i = 0; i < 8; ++i) dst[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
-            }
-        }
-        if (a.mT && tid < kD) a.mT[bhs * kD + tid] = Mv[tid];
-        if (a.tT && h == 0 && tid == 0) a.tT[b] = tpos;
-    }
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
@@ -587,7 +613,7 @@ cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gla_chunk_kernel<<<a.B * a.H, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, a);
+    gla_chunk_kernel<<<a.B * a.H, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, m.o, a);
     return cudaGetLastError();
 }
 

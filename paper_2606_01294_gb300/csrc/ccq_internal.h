@@ -50,7 +50,7 @@ int *device_status_word();
 // Tensor maps of q, k, v (and the GLA gate) viewed as 4-D [B][T][H][D]
 // tensors, so that rows past T load as zeros.
 struct ChunkMaps {
-    CUtensorMap q, k, v, g;
+    CUtensorMap q, k, v, g, o;
 };
 
 cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
