@@ -39,8 +39,9 @@ WORKLOADS = {
     "gdn_bf16_20k": ("gdn", 1, 16, 20480, 128),
     "decode_b256": ("decode", 256, 16, 1, 128),
 }
-KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_recurrent.cu", "decode": "ccq_recurrent.cu"}
-KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "recurrent_kernel", "decode": "recurrent_kernel"}
+KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode": "ccq_recurrent.cu"}
+KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_kernel",
+                "decode": "recurrent_kernel"}
 
 
 def algorithmic_bytes(kind, B, H, T, D):
@@ -259,6 +260,7 @@ def run_gpu(args):
         Dv = {n: (None if x is None else x.to(dev)) for n, x in P.items()}
         out = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
         fstate = ccq.CCQState.empty(B, H, D, D, dev)
+        ws = ccq.gdn_workspace(B, T, H, D, D, dev) if kind == "gdn" else None
 
         def step():
             if kind == "gla":
@@ -266,7 +268,7 @@ def run_gpu(args):
                             final_state=fstate)
             else:
                 ccq.gdn_fwd(Dv["q"], Dv["k"], Dv["v"], Dv["gate"], Dv["beta"], Dv["lam"], out=out,
-                            final_state=fstate)
+                            final_state=fstate, workspace=ws)
         tokens_per_step = B * T
         host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
 
@@ -319,7 +321,7 @@ def run_gpu(args):
                                 final_state=fstate)
         else:
             o, st = ccq.gdn_fwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], out=out,
-                                final_state=fstate)
+                                final_state=fstate, workspace=ws)
         return o.to("cpu", non_blocking=True)
 
     h2d = sum(x.numel() * x.element_size() for x in host.values() if x is not None)

@@ -112,13 +112,27 @@ CCQ_API ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, cons
 /*
  * CCQ-Gated-DeltaNet forward (the gated delta rule as the backbone).
  *   g         log decay log(alpha) [B,T,H] fp32 (<= 0);  beta [B,T,H] fp32 in [0,1].
- * All other arguments as ccq_gla_fwd.
+ *   workspace caller-owned device scratch of at least the size ccq_gdn_workspace_size()
+ *             reports (16-byte aligned), used by the chunkwise kernel to hold the
+ *             per-chunk WY/UT matrices; may be NULL when that size is 0.  Its contents
+ *             on entry do not matter and are undefined on return.
+ * All other arguments as ccq_gla_fwd.  bf16 inputs with Dk = Dv = 128 run the chunkwise
+ * tensor-core kernels (CCQ_ALGO_AUTO / CHUNKWISE; CCQ_ERR_INVALID_ARG if the workspace is
+ * missing or too small); other inputs run the recurrent kernel.
  */
 CCQ_API ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
                        const float *beta, const float *lambda, ccq_dtype in_dtype,
                        const float *S0, const float *C0, const float *m0, const int64_t *t0,
                        void *o, float *ST, float *CT, float *mT, int64_t *tT,
-                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream);
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream);
+
+/*
+ * Workspace bytes ccq_gdn_fwd needs for these sizes and parameters (0 when the
+ * selected kernel needs none).  Host-only; launches nothing.
+ */
+CCQ_API ccq_status ccq_gdn_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                          const ccq_params *p, size_t *bytes);
 
 /*
  * One recurrent CCQ token for a batch of cached states (Algorithm 2), updating

@@ -67,7 +67,10 @@ def load_library() -> ctypes.CDLL:
                                     + [ctypes.POINTER(_Params), _VP])
         lib.ccq_gla_fwd.restype = _I
         lib.ccq_gdn_fwd.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 5
-                                    + [ctypes.POINTER(_Params), _VP])
+                                    + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
+        lib.ccq_gdn_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
+                                                           ctypes.POINTER(ctypes.c_size_t)])
+        lib.ccq_gdn_workspace_size.restype = _I
         lib.ccq_gdn_fwd.restype = _I
         lib.ccq_decode_step.argtypes = ([_I] + [_VP] * 6 + [_I, _I] + [_VP] * 5
                                         + [_I] * 4 + [ctypes.POINTER(_Params), _VP])
@@ -205,8 +208,10 @@ def gla_fwd(q, k, v, gk, lam, state: Optional[CCQState] = None, *, out=None,
 
 def gdn_fwd(q, k, v, g, beta, lam, state: Optional[CCQState] = None, *, out=None,
             final_state: Optional[CCQState] = None, return_state: bool = True,
-            stream=None, **kw):
-    """CCQ-Gated-DeltaNet forward.  g (log decay) and beta are [B,T,H] fp32."""
+            workspace: Optional[torch.Tensor] = None, stream=None, **kw):
+    """CCQ-Gated-DeltaNet forward.  g (log decay) and beta are [B,T,H] fp32.
+    ``workspace`` (a CUDA byte tensor of at least ccq_gdn_workspace_size bytes)
+    is allocated on the fly when not given."""
     dev = q.device
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -223,13 +228,31 @@ def gdn_fwd(q, k, v, g, beta, lam, state: Optional[CCQState] = None, *, out=None
     if fs is None and return_state:
         fs = CCQState.empty(B, H, Dk, Dv, dev)
     p = params(**kw)
-    st = load_library().ccq_gdn_fwd(
+    lib = load_library()
+    need = ctypes.c_size_t(0)
+    _check(lib.ccq_gdn_workspace_size(B, T, H, Dk, Dv, _dtype_code(q), ctypes.byref(p),
+                                      ctypes.byref(need)))
+    if workspace is None and need.value:
+        workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_gdn_fwd(
         _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _dtype_code(q),
         _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(o),
         _ptr(fs.S if fs else None), _ptr(fs.C if fs else None), _ptr(fs.m if fs else None),
-        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, ctypes.byref(p), _stream(dev, stream))
+        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, _ptr(workspace), ws_bytes,
+        ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
+
+
+def gdn_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):
+    """Allocate the workspace ccq_gdn_fwd needs for these sizes (None if none)."""
+    p = params(**kw)
+    need = ctypes.c_size_t(0)
+    code = BF16 if dtype == torch.bfloat16 else FP32
+    _check(load_library().ccq_gdn_workspace_size(B, T, H, Dk, Dv, code, ctypes.byref(p),
+                                                  ctypes.byref(need)))
+    return torch.empty(need.value, dtype=torch.uint8, device=device) if need.value else None
 
 
 def decode_step(backbone: int, q, k, v, gate, lam, state: CCQState, beta=None, *,

@@ -132,6 +132,19 @@ bool make_token_map(CUtensorMap *map, const void *base, int elem_bytes, int B, i
     return r == CUDA_SUCCESS;
 }
 
+bool make_rows_map(CUtensorMap *map, const void *base, long long rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint64_t dims[2] = {128, static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {128 * 2};
+    const cuuint32_t box[2] = {64, 64};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+                    estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
 }  // namespace ccq
 
 using namespace ccq;
@@ -214,11 +227,27 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
     return run_recurrent(ra, s);
 }
 
+static bool gdn_chunk_selected(const ccq_params &p, ccq_dtype in_dtype, int Dk, int T) {
+    const bool ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
+    return ok && p.algo != CCQ_ALGO_RECURRENT;
+}
+
+ccq_status ccq_gdn_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                  const ccq_params *p, size_t *bytes) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    *bytes = gdn_chunk_selected(c.p, in_dtype, Dk, T) ? gdn_workspace_bytes(B, T, H) : 0;
+    return CCQ_OK;
+}
+
 ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
                        const float *beta, const float *lambda, ccq_dtype in_dtype,
                        const float *S0, const float *C0, const float *m0, const int64_t *t0,
                        void *o, float *ST, float *CT, float *mT, int64_t *tT,
-                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream) {
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
@@ -230,8 +259,40 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
         st = check_ptrs("", {}, {S0, C0, m0, t0, ST, CT, mT, tT});
         if (st != CCQ_OK) return st;
     }
-    if (c.p.algo == CCQ_ALGO_CHUNKWISE)
-        return fail(CCQ_ERR_UNSUPPORTED, "chunkwise Gated DeltaNet kernel not built yet");
+    const bool chunk_ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
+    if (c.p.algo == CCQ_ALGO_CHUNKWISE && !chunk_ok)
+        return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
+    if (gdn_chunk_selected(c.p, in_dtype, Dk, T)) {
+        const size_t need = gdn_workspace_bytes(B, T, H);
+        if (!workspace || workspace_bytes < need)
+            return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
+                        workspace ? workspace_bytes : static_cast<size_t>(0));
+        if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+        const int nc = (T + 63) / 64;
+        const long long rows = static_cast<long long>(B) * H * nc * 64;
+        const __nv_bfloat16 *ut = static_cast<const __nv_bfloat16 *>(workspace);
+        const __nv_bfloat16 *w = ut + static_cast<size_t>(rows) * 128;
+        GdnMaps maps;
+        if (!make_token_map(&maps.q, q, 2, B, T, H, 128, 64, true) ||
+            !make_token_map(&maps.k, k, 2, B, T, H, 128, 64, true) ||
+            !make_token_map(&maps.v, v, 2, B, T, H, 128, 64, true) ||
+            !make_token_map(&maps.o, o, 2, B, T, H, 128, 64, true) ||
+            !make_rows_map(&maps.ut, ut, rows) || !make_rows_map(&maps.w, w, rows))
+            return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
+        ChunkArgs a = {};
+        a.B = B; a.T = T; a.H = H;
+        a.gate_dtype = 1;
+        a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
+        a.lambda = lambda; a.g = g; a.beta = beta;
+        a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
+        a.o = static_cast<__nv_bfloat16 *>(o);
+        a.ST = ST; a.CT = CT; a.mT = mT; a.tT = tT;
+        a.status = device_status_word();
+        if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
+        cudaError_t e = launch_gdn_chunk(a, maps, static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return cuda_fail(e, "chunkwise Gated DeltaNet kernel launch");
+        return CCQ_OK;
+    }
     RecurrentArgs ra = {};
     ra.backbone = 1; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
     ra.in_dtype = in_dtype; ra.gate_dtype = CCQ_FP32;

@@ -55,6 +55,23 @@ struct ChunkMaps {
 
 cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
 
+// Chunkwise Gated DeltaNet: tensor maps of q, k, v, o ([B][T][H][128], 64 x 64
+// boxes) and of the two workspace matrices Ut and W ([B*H*NC*64][128] bf16).
+struct GdnMaps {
+    CUtensorMap q, k, v, o, ut, w;
+};
+
+// Launches the per-chunk WY kernel then the sequential chunk kernel.
+cudaError_t launch_gdn_chunk(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
+cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
+
+// Workspace bytes of the chunkwise Gated DeltaNet path (Ut and W of every chunk).
+size_t gdn_workspace_bytes(int B, int T, int H);
+
+// Encode the tensor map of a row-major [rows][128] bf16 matrix with 64 x 64 boxes
+// (128-byte swizzle).
+bool make_rows_map(CUtensorMap *map, const void *base, long long rows);
+
 // Encode the tensor map of a [B][T][H][D] tensor with a (box_inner x 1 x 64 x 1)
 // box.  swizzle128 selects the 128-byte swizzle (bf16 MMA operands, box_inner
 // 64); otherwise the box lands as a plain row-major [64][box_inner] array.

@@ -68,3 +68,11 @@ def compare(o, fs, ref, tol, what=""):
 def slice_bh(P, b, h):
     """Inputs of one (batch row, head) pair, kept 4-D."""
     return {n: (None if x is None else x[b:b + 1, :, h:h + 1].contiguous()) for n, x in P.items()}
+
+
+def correction_bound(o1_ref, d_ref, dtype) -> float:
+    """Bound for the isolated CCQ term o(lambda) - o(0): the stated output
+    tolerance plus the floor of differencing two outputs rounded to the output
+    dtype (each carries up to half an ulp, 2^-9 of its magnitude for bf16)."""
+    half_ulp = {torch.float32: 2.0 ** -24, torch.bfloat16: 2.0 ** -9}[dtype]
+    return TOL[dtype] + 2 * half_ulp * float(np.abs(o1_ref).max()) / float(np.abs(d_ref).max())

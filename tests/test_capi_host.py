@@ -16,7 +16,7 @@ def lib():
 
 def test_library_exports_every_header_symbol(lib):
     names = ccq.header_symbols()
-    assert {"ccq_gla_fwd", "ccq_gdn_fwd", "ccq_decode_step", "ccq_device_status",
+    assert {"ccq_gla_fwd", "ccq_gdn_fwd", "ccq_gdn_workspace_size", "ccq_decode_step", "ccq_device_status",
             "ccq_status_string", "ccq_last_error", "ccq_default_params"} <= set(names)
     for n in names:
         assert hasattr(lib, n), f"{n} declared in include/ but not exported"
@@ -81,3 +81,18 @@ def test_binding_refuses_cpu_tensors():
     x = torch.zeros(1, 4, 1, 128, dtype=torch.bfloat16)
     with pytest.raises(ValueError, match="CUDA"):
         ccq.gla_fwd(x, x, x, x, torch.zeros(1, 4, 1))
+
+
+def test_gdn_workspace_size(lib):
+    n = ctypes.c_size_t(7)
+    assert lib.ccq_gdn_workspace_size(8, 4096, 16, 128, 128, 0, ctypes.byref(ccq.params()), ctypes.byref(n)) == 0
+    assert n.value == 2 * 8 * 16 * 64 * 64 * 128 * 2
+    assert lib.ccq_gdn_workspace_size(1, 100, 2, 128, 128, 1, ctypes.byref(ccq.params()), ctypes.byref(n)) == 0
+    assert n.value == 0  # fp32 inputs run the recurrent kernel
+    assert lib.ccq_gdn_workspace_size(1, 100, 2, 128, 128, 0, ctypes.byref(ccq.params(algo="recurrent")),
+                                      ctypes.byref(n)) == 0
+    assert n.value == 0
+    fake = ctypes.c_void_p(0x10000)
+    st = lib.ccq_gdn_fwd(*([fake] * 6), 0, *([None] * 4), fake, *([None] * 4), 1, 64, 1, 128, 128,
+                         None, 0, ctypes.byref(ccq.params()), None)
+    assert st == ccq.CCQ_ERR_INVALID_ARG and b"workspace" in lib.ccq_last_error()

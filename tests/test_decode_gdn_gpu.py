@@ -7,7 +7,7 @@ import torch
 import oracle
 from paper_2606_01294_gb300 import ccq
 from paper_2606_01294_gb300 import inputs as gen
-from tests.helpers import (GDN, GLA, TOL, compare, gpu_forward, oracle_forward, rel_err, slice_bh,
+from tests.helpers import (correction_bound, GDN, GLA, TOL, compare, gpu_forward, oracle_forward, rel_err, slice_bh,
                            state_f32, state_to_dev)
 
 pytestmark = pytest.mark.gpu
@@ -84,13 +84,58 @@ def test_gdn_forward_matches_oracle(lam, dtype, d):
     compare(o, fs, oracle_forward(GDN, P), TOL[dtype], f"gdn {lam}")
 
 
+@pytest.mark.parametrize("lam", ["init", "trained", "high"])
+@pytest.mark.parametrize("keys", ["iso", "structured", "lowrank"])
+def test_gdn_chunkwise_ragged(lam, keys):
+    """Chunkwise tensor-core GDN (WY/UT kernel + sequential kernel), T = 200."""
+    P = gen.make_inputs(GDN, 2, 200, 3, 128, 128, dtype=torch.bfloat16, seed=31, lam=lam, keys=keys)
+    o, fs = gpu_forward(GDN, P, algo="chunkwise")
+    compare(o, fs, oracle_forward(GDN, P), TOL[torch.bfloat16], f"gdn chunkwise {lam} {keys}")
+
+
+@pytest.mark.parametrize("T", [1, 63, 64, 65, 129])
+def test_gdn_chunk_boundaries(T):
+    P = gen.make_inputs(GDN, 1, T, 2, 128, 128, dtype=torch.bfloat16, seed=200 + T, lam="trained",
+                        keys="structured")
+    o, fs = gpu_forward(GDN, P, algo="chunkwise")
+    compare(o, fs, oracle_forward(GDN, P), TOL[torch.bfloat16], f"gdn T={T}")
+
+
+def test_gdn_chunkwise_correction_isolated():
+    P = gen.make_inputs(GDN, 1, 192, 2, 128, 128, dtype=torch.bfloat16, seed=32, lam="high", keys="lowrank")
+    P0 = dict(P, lam=torch.zeros_like(P["lam"]))
+    o1, _ = gpu_forward(GDN, P, algo="chunkwise")
+    o0, _ = gpu_forward(GDN, P0, algo="chunkwise")
+    ref1 = oracle_forward(GDN, P)["o"]
+    d_ref = ref1 - oracle_forward(GDN, P0)["o"]
+    d = o1.double().cpu().numpy() - o0.double().cpu().numpy()
+    assert np.abs(d_ref).max() > 0.1 * np.abs(ref1).max()
+    assert rel_err(d, d_ref) <= correction_bound(ref1, d_ref, torch.bfloat16)
+
+
+def test_gdn_chunkwise_resume_and_matches_recurrent():
+    P = gen.make_inputs(GDN, 2, 230, 2, 128, 128, dtype=torch.bfloat16, seed=33, lam="trained",
+                        keys="structured")
+    head = {n: (None if x is None else x[:, :100].contiguous()) for n, x in P.items()}
+    tail = {n: (None if x is None else x[:, 100:].contiguous()) for n, x in P.items()}
+    o1, fs1 = gpu_forward(GDN, head, algo="chunkwise")
+    o2, fs2 = gpu_forward(GDN, tail, fs1, algo="chunkwise")
+    full = oracle_forward(GDN, P)
+    assert rel_err(torch.cat([o1, o2], dim=1), full["o"]) <= TOL[torch.bfloat16]
+    assert rel_err(fs2.S, full["S"]) <= TOL[torch.bfloat16]
+    orr, _ = gpu_forward(GDN, P, algo="recurrent")
+    oc, _ = gpu_forward(GDN, P, algo="chunkwise")
+    assert rel_err(oc, orr.double().cpu().numpy()) <= TOL[torch.bfloat16]
+
+
 def test_gdn_full_size_sampled():
+    """B=8, H=16, T=4096 (the benchmark's launch); sampled pairs against the oracle."""
     w = dict(gen.WORKLOADS["gdn_bf16_4k"])
     backbone = w.pop("backbone")
-    w["B"] = 2  # the recurrent GDN kernel is a CUDA-core path; keep the runtime short
     P = gen.make_inputs(backbone, **w)
     o, fs = gpu_forward(GDN, P)
-    for b, h in [(0, 0), (1, 11)]:
+    for b, h in [(0, 0), (5, 11), (7, 15)]:
         ref = oracle_forward(GDN, slice_bh(P, b, h))
         assert rel_err(o[b:b + 1, :, h:h + 1], ref["o"]) <= TOL[torch.bfloat16]
         assert rel_err(fs.S[b:b + 1, h:h + 1], ref["S"]) <= TOL[torch.bfloat16]
+        assert rel_err(fs.C[b:b + 1, h:h + 1], ref["C"]) <= TOL[torch.bfloat16]
