@@ -260,12 +260,12 @@ def run_gpu(args):
         Dv = {n: (None if x is None else x.to(dev)) for n, x in P.items()}
         out = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
         fstate = ccq.CCQState.empty(B, H, D, D, dev)
-        ws = ccq.gdn_workspace(B, T, H, D, D, dev) if kind == "gdn" else None
+        ws = (ccq.gdn_workspace if kind == "gdn" else ccq.gla_workspace)(B, T, H, D, D, dev)
 
         def step():
             if kind == "gla":
                 ccq.gla_fwd(Dv["q"], Dv["k"], Dv["v"], Dv["gate"], Dv["lam"], out=out,
-                            final_state=fstate)
+                            final_state=fstate, workspace=ws)
             else:
                 ccq.gdn_fwd(Dv["q"], Dv["k"], Dv["v"], Dv["gate"], Dv["beta"], Dv["lam"], out=out,
                             final_state=fstate, workspace=ws)
@@ -318,7 +318,7 @@ def run_gpu(args):
         d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
         if kind == "gla":
             o, st = ccq.gla_fwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out,
-                                final_state=fstate)
+                                final_state=fstate, workspace=ws)
         else:
             o, st = ccq.gdn_fwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], out=out,
                                 final_state=fstate, workspace=ws)

@@ -81,10 +81,13 @@ typedef struct {
                       (App. D ablation)                                                  */
     int chunk;     /* chunk length of the chunkwise kernels; 0 or 64 (Algorithm 1)        */
     int algo;      /* a ccq_algo value                                                   */
+    int seq_split; /* chunkwise GLA only: segments each sequence is cut into so that few
+                      long sequences still fill the GPU (states compose exactly across
+                      segments); 0 = choose from B*H and the SM count, 1 = never split */
 } ccq_params;
 
 /* Fill *p with the defaults: l2norm_qk = 1, scale = 0 (1/sqrt(Dk)), centered = 1,
-   chunk = 64, algo = CCQ_ALGO_AUTO. */
+   chunk = 64, algo = CCQ_ALGO_AUTO, seq_split = 0. */
 CCQ_API void ccq_default_params(ccq_params *p);
 
 /*
@@ -101,13 +104,26 @@ CCQ_API void ccq_default_params(ccq_params *p);
  * The chunkwise kernel scales by exp of in-chunk cumulative gates measured from
  * the chunk midpoint; per-chunk cumulative log-gates must stay above about -160
  * (more negative sums underflow to an exact-zero contribution).
+ *   workspace  caller-owned device scratch of at least ccq_gla_workspace_size()
+ *              bytes (16-byte aligned) when that size is non-zero (long sequences
+ *              split into segments); may be NULL otherwise.  Contents undefined on
+ *              return.
  * Returns CCQ_OK or an error code; launches asynchronously on `stream`.
  */
 CCQ_API ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
                        const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
                        const float *S0, const float *C0, const float *m0, const int64_t *t0,
                        void *o, float *ST, float *CT, float *mT, int64_t *tT,
-                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream);
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream);
+
+/*
+ * Workspace bytes ccq_gla_fwd needs (the per-segment states of a split sequence;
+ * 0 when sequences are not split).  The split depends on B*H, T and the current
+ * device's SM count.  Queries the device but launches nothing.
+ */
+CCQ_API ccq_status ccq_gla_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                          const ccq_params *p, size_t *bytes);
 
 /*
  * CCQ-Gated-DeltaNet forward (the gated delta rule as the backbone).

@@ -33,7 +33,7 @@ class CCQError(RuntimeError):
 class _Params(ctypes.Structure):
     _fields_ = [("l2norm_qk", ctypes.c_int), ("scale", ctypes.c_float),
                 ("centered", ctypes.c_int), ("chunk", ctypes.c_int),
-                ("algo", ctypes.c_int)]
+                ("algo", ctypes.c_int), ("seq_split", ctypes.c_int)]
 
 
 _lib = None
@@ -64,8 +64,11 @@ def load_library() -> ctypes.CDLL:
         lib.ccq_device_status.argtypes = [_VP]
         lib.ccq_device_status.restype = _I
         lib.ccq_gla_fwd.argtypes = ([_VP] * 5 + [_I, _I] + [_VP] * 9 + [_I] * 5
-                                    + [ctypes.POINTER(_Params), _VP])
+                                    + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
         lib.ccq_gla_fwd.restype = _I
+        lib.ccq_gla_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
+                                                           ctypes.POINTER(ctypes.c_size_t)])
+        lib.ccq_gla_workspace_size.restype = _I
         lib.ccq_gdn_fwd.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 5
                                     + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
         lib.ccq_gdn_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
@@ -96,7 +99,7 @@ def _check(status: int):
 
 
 def params(*, l2norm: bool = True, scale: Optional[float] = None, centered: bool = True,
-           chunk: int = 64, algo: str = "auto") -> _Params:
+           chunk: int = 64, algo: str = "auto", seq_split: int = 0) -> _Params:
     p = _Params()
     load_library().ccq_default_params(ctypes.byref(p))
     p.l2norm_qk = int(bool(l2norm))
@@ -104,6 +107,7 @@ def params(*, l2norm: bool = True, scale: Optional[float] = None, centered: bool
     p.centered = int(bool(centered))
     p.chunk = int(chunk)
     p.algo = ALGO[algo]
+    p.seq_split = int(seq_split)
     return p
 
 
@@ -175,12 +179,14 @@ def _state_in(state, B, H, Dk, Dv, device):
 
 def gla_fwd(q, k, v, gk, lam, state: Optional[CCQState] = None, *, out=None,
             final_state: Optional[CCQState] = None, return_state: bool = True,
-            stream=None, **kw):
+            workspace: Optional[torch.Tensor] = None, stream=None, **kw):
     """CCQ-GLA forward: o [B,T,H,Dv] and (optionally) the final CCQState.
 
     q, k [B,T,H,Dk], v [B,T,H,Dv] bf16 or fp32 (same dtype); gk [B,T,H,Dk]
     log-forget gate (bf16 or fp32); lam [B,T,H] fp32.  ``state`` is the initial
-    cache (None = zero).  Keyword arguments go to :func:`params`.
+    cache (None = zero).  ``workspace`` (CUDA bytes, ccq_gla_workspace_size)
+    is allocated on the fly when needed and not given.  Keyword arguments go to
+    :func:`params`.
     """
     dev = q.device
     B, T, H, Dk = q.shape
@@ -197,11 +203,20 @@ def gla_fwd(q, k, v, gk, lam, state: Optional[CCQState] = None, *, out=None,
     if fs is None and return_state:
         fs = CCQState.empty(B, H, Dk, Dv, dev)
     p = params(**kw)
-    st = load_library().ccq_gla_fwd(
+    lib = load_library()
+    if workspace is None:
+        need = ctypes.c_size_t(0)
+        _check(lib.ccq_gla_workspace_size(B, T, H, Dk, Dv, _dtype_code(q), ctypes.byref(p),
+                                          ctypes.byref(need)))
+        if need.value:
+            workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_gla_fwd(
         _ptr(q), _ptr(k), _ptr(v), _ptr(gk), _ptr(lam), _dtype_code(q), _dtype_code(gk),
         _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(o),
         _ptr(fs.S if fs else None), _ptr(fs.C if fs else None), _ptr(fs.m if fs else None),
-        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, ctypes.byref(p), _stream(dev, stream))
+        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, _ptr(workspace), ws_bytes,
+        ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
 
@@ -243,6 +258,16 @@ def gdn_fwd(q, k, v, g, beta, lam, state: Optional[CCQState] = None, *, out=None
         ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
+
+
+def gla_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):
+    """Allocate the workspace ccq_gla_fwd needs for these sizes (None if none)."""
+    p = params(**kw)
+    need = ctypes.c_size_t(0)
+    code = BF16 if dtype == torch.bfloat16 else FP32
+    _check(load_library().ccq_gla_workspace_size(B, T, H, Dk, Dv, code, ctypes.byref(p),
+                                                  ctypes.byref(need)))
+    return torch.empty(need.value, dtype=torch.uint8, device=device) if need.value else None
 
 
 def gdn_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):

@@ -8,6 +8,7 @@
 #include <stdint.h>
 #include <stdio.h>
 
+#include <algorithm>
 #include <initializer_list>
 
 #include "../../include/ccq.h"
@@ -85,6 +86,7 @@ ccq_status check_common(const ccq_params *pin, int B, int T, int H, int Dk, int 
         return fail(CCQ_ERR_UNSUPPORTED, "chunk=%d: supported 64", c->p.chunk);
     if (c->p.algo < CCQ_ALGO_AUTO || c->p.algo > CCQ_ALGO_CHUNKWISE)
         return fail(CCQ_ERR_INVALID_ARG, "unknown algo %d", c->p.algo);
+    if (c->p.seq_split < 0) return fail(CCQ_ERR_INVALID_ARG, "seq_split must be >= 0");
     if ((static_cast<long long>(B) * H) > 0x7fffffffLL)
         return fail(CCQ_ERR_INVALID_ARG, "B*H too large");
     c->scale = c->p.scale > 0.f ? c->p.scale : 1.f / sqrtf(static_cast<float>(Dk));
@@ -158,6 +160,7 @@ void ccq_default_params(ccq_params *p) {
     p->centered = 1;
     p->chunk = 64;
     p->algo = CCQ_ALGO_AUTO;
+    p->seq_split = 0;
 }
 
 const char *ccq_status_string(ccq_status s) {
@@ -173,11 +176,57 @@ const char *ccq_status_string(ccq_status s) {
 
 const char *ccq_last_error(void) { return g_last_error; }
 
+static int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+        n = 148;
+    return n;
+}
+
+// Segments per sequence for the chunkwise GLA path, and chunks per segment.
+static void gla_split(const ccq_params &p, int B, int T, int H, int *nseg, int *seg_chunks) {
+    const int nc = (T + 63) / 64;
+    int ns = 1;
+    if (p.seq_split > 0) {
+        ns = p.seq_split;
+    } else if (p.seq_split == 0) {
+        const long long seqs = static_cast<long long>(B) * H;
+        const int sms = sm_count();
+        if (seqs * 2 <= sms) ns = static_cast<int>(sms / seqs);
+        ns = std::min(ns, nc / 8);  // keep at least 8 chunks per segment
+    }
+    ns = std::max(1, std::min(ns, nc));
+    const int per = (nc + ns - 1) / ns;
+    *seg_chunks = per;
+    *nseg = (nc + per - 1) / per;  // no empty segment
+}
+
+static bool gla_chunk_selected(const ccq_params &p, ccq_dtype in_dtype, int Dk, int T) {
+    return in_dtype == CCQ_BF16 && Dk == 128 && T > 0 && p.algo != CCQ_ALGO_RECURRENT;
+}
+
+ccq_status ccq_gla_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                  const ccq_params *p, size_t *bytes) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    *bytes = 0;
+    if (gla_chunk_selected(c.p, in_dtype, Dk, T)) {
+        int ns, per;
+        gla_split(c.p, B, T, H, &ns, &per);
+        if (ns > 1) *bytes = static_cast<size_t>(B) * H * ns * kSegFloats * sizeof(float);
+    }
+    return CCQ_OK;
+}
+
 ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
                        const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
                        const float *S0, const float *C0, const float *m0, const int64_t *t0,
                        void *o, float *ST, float *CT, float *mT, int64_t *tT,
-                       int B, int T, int H, int Dk, int Dv, const ccq_params *p, void *stream) {
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
@@ -195,6 +244,15 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
     if (c.p.algo == CCQ_ALGO_CHUNKWISE && !chunk_ok)
         return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
     if (chunk_ok && c.p.algo != CCQ_ALGO_RECURRENT) {
+        int nseg = 1, seg_chunks = 0;
+        gla_split(c.p, B, T, H, &nseg, &seg_chunks);
+        if (nseg > 1) {
+            const size_t need = static_cast<size_t>(B) * H * nseg * kSegFloats * sizeof(float);
+            if (!workspace || workspace_bytes < need)
+                return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
+                            workspace ? workspace_bytes : static_cast<size_t>(0));
+            if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+        }
         ChunkMaps maps;
         const int geb = gate_dtype == CCQ_BF16 ? 2 : 4;
         if (!make_token_map(&maps.q, q, 2, B, T, H, 128, 64, true) ||
@@ -213,6 +271,14 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
         a.ST = ST; a.CT = CT; a.mT = mT; a.tT = tT;
         a.status = device_status_word();
         if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
+        a.nseg = nseg;
+        a.seg_chunks = seg_chunks;
+        if (a.nseg > 1) {
+            a.seg_ws = static_cast<float *>(workspace);
+            cudaError_t e = launch_gla_segments(a, maps, s);
+            if (e != cudaSuccess) return cuda_fail(e, "segmented chunkwise GLA launch");
+            return CCQ_OK;
+        }
         cudaError_t e = launch_gla_chunk(a, maps, s);
         if (e != cudaSuccess) return cuda_fail(e, "chunkwise GLA kernel launch");
         return CCQ_OK;

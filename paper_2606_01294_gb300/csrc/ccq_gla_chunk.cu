@@ -44,6 +44,9 @@
 // reloaded as soon as the chunk's last product that reads it completes.
 // Rows past T load as zeros: zero keys add nothing to any sum, zero gates keep
 // the cumulative gate, so the ragged tail needs no special arithmetic.
+// With a.nseg > 1 every CTA walks one segment (a range of whole chunks) of one
+// sequence, starting from the segment's initial states in a.seg_ws
+// (ccq_gla_segment.cu); only the last segment writes the final states.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -141,12 +144,19 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int wg = tid >> 7, wt = tid & 127;
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int bh = blockIdx.x / a.nseg, seg = blockIdx.x % a.nseg, b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H;
-    const int NC = (T + kC - 1) / kC;
+    const int NCt = (T + kC - 1) / kC;
+    const int cb = a.nseg > 1 ? seg * a.seg_chunks : 0;  // first chunk of this CTA
+    const int NC = a.nseg > 1 ? min(NCt, cb + a.seg_chunks) - cb : NCt;
+    const bool last_seg = seg == a.nseg - 1;
+    const float *segst = a.nseg > 1 ? a.seg_ws + static_cast<size_t>(blockIdx.x) * kSegFloats : nullptr;
+    const float *S0 = segst ? segst : a.S0;
+    const float *C0 = segst ? segst + kD * kD : a.C0;
+    const float *m0 = segst ? segst + 2 * kD * kD : a.m0;
     const bool gate_f32 = a.gate_dtype != 0;
     const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
-    const int64_t t0 = a.t0 ? a.t0[b] : 0;
+    const int64_t tseq0 = a.t0 ? a.t0[b] : 0;  // position before the sequence
     int *status = a.status;
 
     if (tid == 0) {
@@ -165,21 +175,22 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     const uint32_t tbase = *tmem_slot;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * (warp & 3)) << 16);  // warp's lane quadrant
 
-    auto issue_in = [&](int r) {  // q, k, gates of chunk r into slot r & 1
-        const int s = r & 1;
+    auto issue_in = [&](int r) {  // q, k, gates of local chunk r into slot r & 1
+        const int s = r & 1, tg = (cb + r) * kC;
         uint8_t *base = sm + s * SLOT_BYTES;
         uint64_t *bb = &bar[BAR_IN0 + s];
         mbar_arrive_expect_tx(bb, 4 * 8192 + g_bytes);
-        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, r * kC, b);
-        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, r * kC, b);
-        tma_load_4d(base + SO_K, &map_k, bb, 0, h, r * kC, b);
-        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, r * kC, b);
-        tma_load_4d(base + SO_KG, &map_g, bb, 0, h, r * kC, b);
+        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tg, b);
+        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tg, b);
+        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tg, b);
+        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tg, b);
+        tma_load_4d(base + SO_KG, &map_g, bb, 0, h, tg, b);
     };
     auto issue_v = [&](int r) {
+        const int tg = (cb + r) * kC;
         mbar_arrive_expect_tx(&bar[BAR_V], 2 * 8192);
-        tma_load_4d(sm + OFF_V, &map_v, &bar[BAR_V], 0, h, r * kC, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, r * kC, b);
+        tma_load_4d(sm + OFF_V, &map_v, &bar[BAR_V], 0, h, tg, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, tg, b);
     };
 
     // ---- set-up: initial states into TMEM (WG2), key sum (WG1), first loads (thread 0)
@@ -187,13 +198,14 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const size_t bhs = static_cast<size_t>(bh);
         const int row = 32 * (warp & 3) + lane;
         for (int m = 0; m < 2; ++m) {
-            const float *src = m == 0 ? a.S0 : a.C0;
+            const float *src = m == 0 ? S0 : C0;
             const uint32_t col0 = m == 0 ? TM_S : TM_SK;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 float x[32];
                 if (src) {
-                    const float4 *p4 = reinterpret_cast<const float4 *>(src + (bhs * kD + row) * kD + 32 * c);
+                    const float4 *p4 = reinterpret_cast<const float4 *>(
+                        src + (segst ? static_cast<size_t>(row) * kD : (bhs * kD + row) * kD) + 32 * c);
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
                         const float4 f = p4[e];
@@ -208,7 +220,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         }
         tmem_wait_st();
     } else if (wg == 1) {
-        slot_f(0, MS_MST)[wt] = a.m0 ? a.m0[static_cast<size_t>(bh) * kD + wt] : 0.f;
+        slot_f(0, MS_MST)[wt] = m0 ? m0[(segst ? 0 : static_cast<size_t>(bh) * kD) + wt] : 0.f;
         dmprev[wt] = 0.f;
     } else if (tid == 0) {
         issue_in(0);
@@ -231,8 +243,8 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const uint32_t sp = (r >> 1) & 1, par = r & 1;
             uint8_t *slot = sm + s * SLOT_BYTES;
             const uint32_t ss = sb + s * SLOT_BYTES;
-            const int c0 = r * kC, n = min(kC, T - c0);
-            const float ti = static_cast<float>(t0 + c0 + i + 1);
+            const int c0 = (cb + r) * kC;  // first token of the chunk (sequence position)
+            const float ti = static_cast<float>(tseq0 + c0 + i + 1);
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
             mbar_wait(&bar[BAR_SNAP], par, abort_flag, status);
             const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
@@ -416,7 +428,10 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const int p = wt & 63, th = wt >> 6;  // key-dim pair (2p, 2p+1), token half
         const int d0 = 2 * p;
         float lam_reg = 0.f;
-        if (wt < 64) lam_reg = (wt < T) ? a.lambda[(static_cast<size_t>(b) * T + wt) * H + h] : 0.f;
+        if (wt < 64) {
+            const int tn = cb * kC + wt;
+            lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+        }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1;
@@ -427,7 +442,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
             if (wt < 64) {
                 slot_f(s, MS_LAM)[wt] = lam_reg;
-                const int tn = (r + 1) * kC + wt;
+                const int tn = (cb + r + 1) * kC + wt;
                 lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
             }
             named_bar(2, 128);
@@ -528,11 +543,11 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
         }
         // final key sum and position
-        if (NC > 0 && a.mT) {
+        if (NC > 0 && a.mT && last_seg) {
             const int sl = (NC - 1) & 1;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
-        if (a.tT && h == 0 && wt == 0) a.tT[b] = t0 + T;
+        if (a.tT && h == 0 && wt == 0 && last_seg) a.tT[b] = tseq0 + T;
     } else {
         // =============================================================== WG2: states
         const int row = 32 * (warp & 3) + lane;  // state row a (key dim)
@@ -569,7 +584,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (wt == 0) mbar_arrive(&bar[BAR_SNAP]);
         }
         // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K
-        if (NC > 0) {
+        if (NC > 0 && last_seg) {
             mbar_wait(&bar[BAR_GS], (NC - 1) & 1, abort_flag, status);
             tc_fence_after();
             const float fs = slot_f((NC - 1) & 1, MS_F)[row];
@@ -613,7 +628,7 @@ cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gla_chunk_kernel<<<a.B * a.H, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, m.o, a);
+    gla_chunk_kernel<<<a.B * a.H * a.nseg, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, m.o, a);
     return cudaGetLastError();
 }
 

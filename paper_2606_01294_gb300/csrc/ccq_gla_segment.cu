@@ -1,0 +1,270 @@
+// ccq_gla_segment.cu -- sequence-segment parallelism for long CCQ-GLA sequences.
+//
+// With few (batch, head) sequences (B*H well below the SM count), each sequence
+// is cut into `nseg` segments of whole chunks.  Every recurrent state of the
+// layer composes across a segment boundary in closed form:
+//   GLA state   S_out = Diag(D) S_in + dS,     D = e^{sum of the segment's log gates}
+//   second moment  C_out = C_in + dC,  key sum  m_out = m_in + dm  (undecayed, App. B)
+// so three launches replace one long sequential walk:
+//   1. gla_segment_state_kernel: per segment, from a zero state, the deltas
+//      (dS, dC, dm, D) -- no read, no output.  Chunks are visited last to first so
+//      each chunk's write is scaled by the decay of the chunks after it and
+//      accumulates straight into TMEM: dS = sum_r (kbar e^{Gtot_r - G} * Dsuf_r)^T V.
+//   2. gla_segment_combine_kernel: per sequence, an exclusive scan over its
+//      segments that replaces each delta with that segment's initial state.
+//   3. gla_chunk_kernel with one CTA per (sequence, segment), started from those
+//      states (ccq_gla_chunk.cu).
+// Workspace per (sequence, segment): S [128][128], C [128][128], m [128], D [128] fp32.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ccq_internal.h"
+#include "sm100_ptx.cuh"
+
+namespace ccq {
+
+namespace {
+
+constexpr int kC = 64;
+constexpr int kD = 128;
+constexpr int kThreads = 256;
+constexpr float kLog2e = 1.4426950408889634f;
+
+// shared memory: two slots of {k 16K, v 16K, gates 32K, Ku 16K}
+constexpr uint32_t SL_BYTES = 81920;
+constexpr uint32_t SL_K = 0, SL_V = 16384, SL_G = 32768, SL_KU = 65536;
+constexpr uint32_t OFF_MISC = 2 * SL_BYTES;  // 163840
+constexpr uint32_t M_DSUF = 0;     // [128] decay of the chunks already visited (later ones)
+constexpr uint32_t M_MSUM = 512;   // [128] key sum
+constexpr uint32_t M_GP = 1024;    // [2][128] gate partial sums
+constexpr uint32_t M_DM = 2048;    // [2][128] key partial sums
+constexpr uint32_t M_RK = 3072;    // [64]
+constexpr uint32_t M_BAR = 3328;   // 4 mbarriers: in[2], mma[2]
+constexpr uint32_t M_TMEM = 3360, M_ABORT = 3364;
+constexpr uint32_t kSmem = OFF_MISC + 4096 + 1024;
+static_assert(kSmem <= 232448, "smem");
+
+__global__ void __launch_bounds__(kThreads, 1)
+gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
+                         const __grid_constant__ CUtensorMap map_g, const ChunkArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                              ~static_cast<uintptr_t>(1023));
+    const uint32_t sb = smem_addr(sm);
+    uint8_t *misc = sm + OFF_MISC;
+    float *dsuf = reinterpret_cast<float *>(misc + M_DSUF);
+    float *msum = reinterpret_cast<float *>(misc + M_MSUM);
+    float *gp = reinterpret_cast<float *>(misc + M_GP);
+    float *dm = reinterpret_cast<float *>(misc + M_DM);
+    float *rk = reinterpret_cast<float *>(misc + M_RK);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int seq = blockIdx.x / a.nseg, seg = blockIdx.x % a.nseg;
+    const int b = seq / a.H, h = seq % a.H;
+    const int NCt = (a.T + kC - 1) / kC;
+    const int cb = seg * a.seg_chunks, ce = min(NCt, cb + a.seg_chunks);
+    const int n = ce - cb;  // chunks of this segment (>= 1)
+    const bool gate_f32 = a.gate_dtype != 0;
+    const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
+    int *status = a.status;
+
+    if (tid == 0) {
+        for (int i = 0; i < 4; ++i) mbar_init(&bar[i], 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+    }
+    if (warp == 0) tmem_alloc(tslot, 256);
+    if (tid < kD) {
+        dsuf[tid] = 1.f;
+        msum[tid] = 0.f;
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tslot;
+    // visit chunks last to first: local step i handles global chunk ce - 1 - i
+    auto issue = [&](int i) {
+        const int s = i & 1, cg = ce - 1 - i;
+        uint8_t *base = sm + s * SL_BYTES;
+        mbar_arrive_expect_tx(&bar[s], 4 * 8192 + g_bytes);
+        tma_load_4d(base + SL_K, &map_k, &bar[s], 0, h, cg * kC, b);
+        tma_load_4d(base + SL_K + 8192, &map_k, &bar[s], 64, h, cg * kC, b);
+        tma_load_4d(base + SL_V, &map_v, &bar[s], 0, h, cg * kC, b);
+        tma_load_4d(base + SL_V + 8192, &map_v, &bar[s], 64, h, cg * kC, b);
+        tma_load_4d(base + SL_G, &map_g, &bar[s], 0, h, cg * kC, b);
+    };
+    if (tid == 0) {
+        issue(0);
+        if (n > 1) issue(1);
+    }
+    for (int i = 0; i < n; ++i) {
+        const int s = i & 1;
+        const uint32_t par = (i >> 1) & 1;
+        uint8_t *slot = sm + s * SL_BYTES;
+        mbar_wait(&bar[s], par, abort_flag, status);
+        // k row norms
+        if (tid < 64) {
+            float ss = 0.f;
+#pragma unroll
+            for (int t64 = 0; t64 < 2; ++t64)
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc) {
+                    float f[8];
+                    unpack_bf16x8(*reinterpret_cast<const uint4 *>(slot + SL_K + t64 * 8192 + t64_chunk(tid, cc)), f);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) ss = fmaf(f[e], f[e], ss);
+                }
+            rk[tid] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+        }
+        // gate cumsum per key dim over this thread's 32 tokens
+        const int d = tid & 127, th = tid >> 7;
+        float gl[32];
+        {
+            float run = 0.f;
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {
+                const int j = 32 * th + jj;
+                const float g = gate_f32 ? reinterpret_cast<const float *>(slot + SL_G)[j * kD + d]
+                                         : __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(slot + SL_G)[j * kD + d]);
+                run += g;
+                gl[jj] = run;
+            }
+            gp[th * kD + d] = run;
+        }
+        __syncthreads();
+        {
+            const float g0 = gp[d], gtot = gp[d] + gp[kD + d];
+            const float off = th ? g0 : 0.f;
+            const float ds = dsuf[d];
+            const uint32_t tcol = (d >> 6) * 8192;
+            float dmp = 0.f;
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) {
+                const int j = 32 * th + jj;
+                const uint32_t o = tcol + t64_offset(j, d & 63);
+                const float kb = __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(slot + SL_K + o)) * rk[j];
+                *reinterpret_cast<__nv_bfloat16 *>(slot + SL_K + o) = __float2bfloat16_rn(kb);
+                const float ku = kb * ds * fast_exp2((gtot - (gl[jj] + off)) * kLog2e);
+                *reinterpret_cast<__nv_bfloat16 *>(slot + SL_KU + o) = __float2bfloat16_rn(ku);
+                dmp += kb;
+            }
+            dm[th * kD + d] = dmp;
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tc_fence_after();
+            const uint32_t ss = sb + s * SL_BYTES;
+            const uint64_t dku = make_desc(ss + SL_KU, 8192, 1024);
+            const uint64_t dv = make_desc(ss + SL_V, 8192, 1024);
+            const uint64_t dk = make_desc(ss + SL_K, 8192, 1024);
+            const uint32_t id = make_idesc(128, 128, 1, 1);
+            for (int k = 0; k < 4; ++k) mma_bf16(tbase, dku + k * 128, dv + k * 128, id, (i | k) != 0);
+            for (int k = 0; k < 4; ++k) mma_bf16(tbase + 128, dk + k * 128, dk + k * 128, id, (i | k) != 0);
+            mma_commit(&bar[2 + s]);
+        }
+        if (tid < kD) {
+            dsuf[tid] *= fast_exp2((gp[tid] + gp[kD + tid]) * kLog2e);
+            msum[tid] += dm[tid] + dm[kD + tid];
+        }
+        // refill this slot with chunk step i + 2 once its products are done
+        if (tid == 0 && i + 2 < n && !*abort_flag) {
+            mbar_wait(&bar[2 + s], par, abort_flag, status);
+            issue(i + 2);
+        }
+        __syncthreads();
+    }
+    // wait for the last products of both slots
+    if (n >= 1) mbar_wait(&bar[2 + ((n - 1) & 1)], ((n - 1) >> 1) & 1, abort_flag, status);
+    if (n >= 2) mbar_wait(&bar[2 + ((n - 2) & 1)], ((n - 2) >> 1) & 1, abort_flag, status);
+    tc_fence_after();
+    float *out = a.seg_ws + static_cast<size_t>(blockIdx.x) * kSegFloats;
+    {
+        const int lq = warp & 3, ch = warp >> 2;  // 8 warps: lane quadrant, column half
+        const int row = 32 * lq + lane;
+        const uint32_t tl = tbase + (static_cast<uint32_t>(32 * lq) << 16);
+#pragma unroll
+        for (int m = 0; m < 2; ++m) {
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                const int col = 64 * ch + 32 * c;
+                float x[32];
+                tmem_ld32(tl + 128 * m + col, x);
+                float4 *dst = reinterpret_cast<float4 *>(out + m * kD * kD + row * kD + col);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+            }
+        }
+    }
+    if (tid < kD) {
+        out[2 * kD * kD + tid] = msum[tid];
+        out[2 * kD * kD + kD + tid] = dsuf[tid];
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tbase, 256);
+    }
+}
+
+// Exclusive scan over the segments of each sequence: the delta stored in slot s
+// is replaced by the state entering segment s.
+__global__ void __launch_bounds__(256)
+gla_segment_combine_kernel(const ChunkArgs a) {
+    const int seq = blockIdx.x, tid = threadIdx.x;
+    const size_t sq = static_cast<size_t>(seq);
+    float cs[64], cc[64];
+#pragma unroll
+    for (int k = 0; k < 64; ++k) {
+        const int e = tid + 256 * k;
+        cs[k] = a.S0 ? a.S0[sq * kD * kD + e] : 0.f;
+        cc[k] = a.C0 ? a.C0[sq * kD * kD + e] : 0.f;
+    }
+    float cm = (tid < kD && a.m0) ? a.m0[sq * kD + tid] : 0.f;
+    for (int s = 0; s < a.nseg; ++s) {
+        float *slot = a.seg_ws + (sq * a.nseg + s) * kSegFloats;
+        const float *D = slot + 2 * kD * kD + kD;
+#pragma unroll
+        for (int k = 0; k < 64; ++k) {
+            const int e = tid + 256 * k;
+            const float dS = slot[e], dC = slot[kD * kD + e];
+            slot[e] = cs[k];
+            slot[kD * kD + e] = cc[k];
+            cs[k] = fmaf(D[e >> 7], cs[k], dS);
+            cc[k] += dC;
+        }
+        if (tid < kD) {
+            const float dmv = slot[2 * kD * kD + tid];
+            slot[2 * kD * kD + tid] = cm;
+            cm += dmv;
+        }
+        __syncthreads();  // D of this slot read by every thread before the next slot
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_gla_segments(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(gla_segment_state_kernel,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmem));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    gla_segment_state_kernel<<<a.B * a.H * a.nseg, kThreads, kSmem, s>>>(m.k, m.v, m.g, a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    gla_segment_combine_kernel<<<a.B * a.H, 256, 0, s>>>(a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return launch_gla_chunk(a, m, s);
+}
+
+}  // namespace ccq

@@ -42,7 +42,16 @@ struct ChunkArgs {
     float *ST, *CT, *mT;
     int64_t *tT;
     int *status;  // device status word (bounded-wait give-ups)
+    // sequence segments (long sequences): nseg segments of seg_chunks chunks each
+    // (the last one shorter); seg_ws holds kSegFloats floats per (sequence, segment).
+    int nseg = 1;
+    int seg_chunks = 0;
+    float *seg_ws = nullptr;
 };
+
+// Per (sequence, segment) workspace: S [128][128], C [128][128], m [128], D [128].
+constexpr int kSegFloats = 2 * 128 * 128 + 2 * 128;
+
 
 // Device address of the library's status word on the current device.
 int *device_status_word();
@@ -54,6 +63,10 @@ struct ChunkMaps {
 };
 
 cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
+
+// Segment-parallel CCQ-GLA (ccq_gla_segment.cu): state deltas per segment, an
+// exclusive combine, then gla_chunk_kernel on every (sequence, segment).
+cudaError_t launch_gla_segments(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
 
 // Chunkwise Gated DeltaNet: tensor maps of q, k, v, o ([B][T][H][128], 64 x 64
 // boxes) and of the two workspace matrices Ut and W ([B*H*NC*64][128] bf16).

@@ -25,7 +25,7 @@ def test_library_exports_every_header_symbol(lib):
 def test_default_params(lib):
     p = ccq._Params()
     lib.ccq_default_params(ctypes.byref(p))
-    assert (p.l2norm_qk, p.scale, p.centered, p.chunk, p.algo) == (1, 0.0, 1, 64, 0)
+    assert (p.l2norm_qk, p.scale, p.centered, p.chunk, p.algo, p.seq_split) == (1, 0.0, 1, 64, 0, 0)
 
 
 def test_status_strings(lib):
@@ -38,7 +38,7 @@ def _gla(lib, ptrs=None, sizes=(1, 4, 1, 128, 128), p=None, dtypes=(0, 0)):
     fake = ctypes.c_void_p(0x10000)  # aligned, never dereferenced on these paths
     args = ptrs if ptrs is not None else [fake] * 5
     return lib.ccq_gla_fwd(*args, *dtypes, *([None] * 4), fake, *([None] * 4),
-                           *sizes, ctypes.byref(p or ccq.params()), None)
+                           *sizes, None, 0, ctypes.byref(p or ccq.params()), None)
 
 
 def test_rejects_null_and_misaligned_pointers(lib):
@@ -96,3 +96,26 @@ def test_gdn_workspace_size(lib):
     st = lib.ccq_gdn_fwd(*([fake] * 6), 0, *([None] * 4), fake, *([None] * 4), 1, 64, 1, 128, 128,
                          None, 0, ctypes.byref(ccq.params()), None)
     assert st == ccq.CCQ_ERR_INVALID_ARG and b"workspace" in lib.ccq_last_error()
+
+
+def test_gla_workspace_size_and_split(lib):
+    n = ctypes.c_size_t(7)
+    seg_bytes = (2 * 128 * 128 + 2 * 128) * 4
+    # many sequences: never split
+    assert lib.ccq_gla_workspace_size(8, 4096, 16, 128, 128, 0, ctypes.byref(ccq.params()), ctypes.byref(n)) == 0
+    assert n.value == 0
+    # forced split: 4 segments of a 300-token (5-chunk) sequence -> 3 segments of 2 chunks
+    assert lib.ccq_gla_workspace_size(1, 300, 2, 128, 128, 0, ctypes.byref(ccq.params(seq_split=4)),
+                                      ctypes.byref(n)) == 0
+    assert n.value == 1 * 2 * 3 * seg_bytes
+    # split never applies to the recurrent kernel
+    assert lib.ccq_gla_workspace_size(1, 300, 2, 128, 128, 1, ctypes.byref(ccq.params(seq_split=4)),
+                                      ctypes.byref(n)) == 0
+    assert n.value == 0
+    fake = ctypes.c_void_p(0x10000)
+    st = lib.ccq_gla_fwd(*([fake] * 5), 0, 0, *([None] * 4), fake, *([None] * 4), 1, 300, 2, 128, 128,
+                         None, 0, ctypes.byref(ccq.params(seq_split=4)), None)
+    assert st == ccq.CCQ_ERR_INVALID_ARG and b"workspace" in lib.ccq_last_error()
+    bad = ccq.params()
+    bad.seq_split = -1
+    assert _gla(lib, p=bad) == ccq.CCQ_ERR_INVALID_ARG

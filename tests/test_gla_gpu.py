@@ -135,3 +135,15 @@ def test_full_size_sampled(name, pairs):
                 "m": rel_err(fs.m[b:b + 1, h:h + 1], ref["m"])}
         assert max(errs.values()) <= TOL[torch.bfloat16], (b, h, errs)
         assert int(fs.t[b]) == P["q"].shape[1]
+
+
+@pytest.mark.parametrize("split", [2, 3, 5])
+def test_segmented_sequences(split):
+    """Sequences cut into segments (state deltas, exclusive combine, recompute)
+    equal one sequential walk: T = 700 (11 chunks, ragged tail), resumed state."""
+    P = gen.make_inputs(GLA, 2, 700, 2, 128, 128, dtype=torch.bfloat16, seed=40 + split, lam="trained",
+                        keys="structured")
+    prev = gen.make_inputs(GLA, 2, 90, 2, 128, 128, dtype=torch.bfloat16, seed=50, lam="trained")
+    st = state_f32(oracle_forward(GLA, prev))
+    o, fs = gpu_forward(GLA, P, state_to_dev(st), algo="chunkwise", seq_split=split)
+    compare(o, fs, oracle_forward(GLA, P, st), TOL[torch.bfloat16], f"split={split}")
