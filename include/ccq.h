@@ -165,6 +165,30 @@ CCQ_API ccq_status ccq_decode_step(int backbone, const void *q, const void *k, c
                            const ccq_params *p, void *stream);
 
 /*
+ * ccq_gla_fwd for callers that cannot supply any device memory of their own --
+ * for instance an engine that gave all device memory to its own caches at
+ * start-up, or code on a path where allocating is not allowed or would stall
+ * the device.  The paper has no counterpart; this is a deployment convenience.
+ * Same arguments as ccq_gla_fwd minus the workspace: the per-segment states of
+ * split sequences live in a fixed 24 MiB array inside the library (190
+ * (sequence, segment) states), which every GPU that loads the library keeps
+ * until the process exits.  Nothing is allocated.
+ *   - Requests needing more scratch than that (ccq_gla_workspace_size) fail with
+ *     CCQ_ERR_INVALID_ARG and a message naming both sizes.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - All calls share the one array and it keeps the last call's contents: two
+ *     calls whose work overlaps on the GPU (other streams, other host threads)
+ *     race and corrupt each other's results; serialise them.
+ */
+CCQ_API ccq_status ccq_gla_fwd_fixed_scratch(const void *q, const void *k, const void *v, const void *gk,
+                                             const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                                             const float *S0, const float *C0, const float *m0,
+                                             const int64_t *t0, void *o, float *ST, float *CT, float *mT,
+                                             int64_t *tT, int B, int T, int H, int Dk, int Dv,
+                                             const ccq_params *p, void *stream);
+
+/*
  * Synchronise `stream`, then read and clear the device status word that the
  * kernels' bounded waits write.  Returns CCQ_OK, CCQ_ERR_TIMEOUT (a kernel gave
  * up waiting; its outputs are not valid) or CCQ_ERR_CUDA.

@@ -115,6 +115,11 @@ ccq_status run_recurrent(RecurrentArgs &ra, cudaStream_t s) {
 
 }  // namespace
 
+int record_error_code(int st, const char *msg) {
+    snprintf(g_last_error, sizeof g_last_error, "%s", msg);
+    return st;
+}
+
 bool make_token_map(CUtensorMap *map, const void *base, int elem_bytes, int B, int T, int H, int D,
                     int box_inner, bool swizzle128) {
     EncodeTiledFn fn = encode_fn();

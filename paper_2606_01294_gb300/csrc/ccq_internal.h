@@ -56,6 +56,10 @@ constexpr int kSegFloats = 2 * 128 * 128 + 2 * 128;
 // Device address of the library's status word on the current device.
 int *device_status_word();
 
+// Store `msg` as this host thread's ccq_last_error() text and return `st`.
+// (ccq_status is an int-valued enum of include/ccq.h.)
+int record_error_code(int st, const char *msg);
+
 // Tensor maps of q, k, v (and the GLA gate) viewed as 4-D [B][T][H][D]
 // tensors, so that rows past T load as zeros.
 struct ChunkMaps {
