@@ -56,16 +56,16 @@ __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chun
 
 constexpr uint32_t WY_K = 0;        // 16K  k raw -> kbar; later staging of W
 constexpr uint32_t WY_V = 16384;    // 16K  v; later staging of Ut
-constexpr uint32_t WY_A = 32768;    // 64 x 68 fp32: A
+constexpr uint32_t WY_A = 32768;    // 64 x 68 fp32: A; after the inversion the two bf16 tiles:
+constexpr uint32_t WY_TB = 32768;   //   8K  bf16 Tt diag(beta)               ([64][64] T64 tile)
+constexpr uint32_t WY_TG = 40960;   //   8K  bf16 Tt diag(beta e^{gc - gc_m})
 constexpr uint32_t WY_T = 50176;    // 64 x 68 fp32: Tt
 constexpr uint32_t WY_Y = 67584;    // 3 x 256 fp32: block products
-constexpr uint32_t WY_TB = 71680;   // 8K  bf16 Tt diag(beta)               ([64][64] T64 tile)
-constexpr uint32_t WY_TG = 79872;   // 8K  bf16 Tt diag(beta e^{gc - gc_m})
-constexpr uint32_t WY_MISC = 88064; // gc, beta, factors, rk, barrier
-constexpr uint32_t WY_SMEM = WY_MISC + 2048 + 1024;
+constexpr uint32_t WY_MISC = 70656; // gc, beta, factors, rk, barrier
+constexpr uint32_t WY_SMEM = WY_MISC + 2048 + 1024;  // 73.7 KB: three CTAs per SM
 constexpr int kAS = 68;             // padded fp32 row stride of A and Tt
 
-__global__ void __launch_bounds__(128, 2)
+__global__ void __launch_bounds__(128, 3)
 gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
               const __grid_constant__ CUtensorMap map_ut, const __grid_constant__ CUtensorMap map_w,
               const ChunkArgs a, int NC) {
@@ -102,7 +102,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         tma_load_4d(sm + WY_V, &map_v, &bar[0], 0, h, c0, b);
         tma_load_4d(sm + WY_V + 8192, &map_v, &bar[0], 64, h, c0, b);
     }
-    if (warp == 0) tmem_alloc(tslot, 256);
+    if (warp == 0) tmem_alloc(tslot, 128);
     if (tid < 64) {
         const int t = c0 + tid;
         const size_t row = (static_cast<size_t>(b) * T + t) * H + h;
@@ -114,13 +114,17 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     const uint32_t tb = *tslot;
     const uint32_t tq = tb + (static_cast<uint32_t>(32 * warp) << 16);
 
-    // ---- cumulative decay (one thread; 64 adds) and the k row norms
-    if (tid == 64) {
-        float run = 0.f;
-        for (int i = 0; i < 64; ++i) {
-            run += gcs[i];
-            gcs[i] = run;
+    // ---- cumulative decay (warp 2: two values per lane, shuffle scan) and the k row norms
+    if (warp == 2) {
+        const float x0 = gcs[2 * lane], x1 = gcs[2 * lane + 1];
+        float p = x0 + x1;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const float y = __shfl_up_sync(0xffffffffu, p, o);
+            if (lane >= o) p += y;
         }
+        gcs[2 * lane] = p - x1;
+        gcs[2 * lane + 1] = p;
     }
     mbar_wait(&bar[0], 0, abort_flag, status);
     if (tid < 64) {
@@ -233,7 +237,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int j = 32 * hf + 8 * q4 + e;
-                const float t = (j <= i) ? Tt[i * kAS + j] : 0.f;
+                const float t = (j <= i) ? Tt[i * kAS + j] : 0.f;  // A is dead: its space takes the tiles
                 wb[e] = t * bet[j];
                 wg[e] = wb[e] * epos[j];
             }
@@ -252,7 +256,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
             const uint64_t da = make_desc(sb + (pass == 0 ? WY_TB : WY_TG), 16, 1024);
             const uint64_t dbm = make_desc(sb + (pass == 0 ? WY_V : WY_K), 8192, 1024);
             for (int k = 0; k < 4; ++k)
-                mma_bf16(tb + 128, da + k * 2, dbm + k * 128, make_idesc(64, 128, 0, 1), k != 0);
+                mma_bf16(tb, da + k * 2, dbm + k * 128, make_idesc(64, 128, 0, 1), k != 0);
             mma_commit(&bar[2]);
         }
         mbar_wait(&bar[2], pass, abort_flag, status);
@@ -263,7 +267,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 #pragma unroll
             for (int h2 = 0; h2 < 2; ++h2) {
                 float x[32];
-                tmem_ld16x2_32<64>(tq + 128 + 32 * h2, x);
+                tmem_ld16x2_32<64>(tq + 32 * h2, x);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(stage, i, 4 * h2 + q4, x + 8 * q4);
             }
@@ -287,12 +291,12 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
             tma_store_commit();
         }
     }
-    if (tid == 0) tma_store_wait_all();
+    if (tid == 0) tma_store_wait_read();  // shared memory must outlive the stores' reads
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tb, 256);
+        tmem_dealloc(tb, 128);
     }
 }
 

@@ -214,37 +214,39 @@ gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
 }
 
 // Exclusive scan over the segments of each sequence: the delta stored in slot s
-// is replaced by the state entering segment s.
+// is replaced by the state entering segment s.  Elementwise, so the grid spans
+// (sequence, 1024-element block) and every thread walks the segments of 4 elements.
+constexpr int kCombineBlock = 1024;
+
 __global__ void __launch_bounds__(256)
 gla_segment_combine_kernel(const ChunkArgs a) {
-    const int seq = blockIdx.x, tid = threadIdx.x;
+    const int nblk = (kSegFloats - kD + kCombineBlock - 1) / kCombineBlock;  // D is not scanned
+    const int seq = blockIdx.x / nblk, blk = blockIdx.x % nblk;
     const size_t sq = static_cast<size_t>(seq);
-    float cs[64], cc[64];
+    constexpr int kSS = kD * kD;  // S block, then C block, then m
+    float cur[4];
+    int el[4];
 #pragma unroll
-    for (int k = 0; k < 64; ++k) {
-        const int e = tid + 256 * k;
-        cs[k] = a.S0 ? a.S0[sq * kD * kD + e] : 0.f;
-        cc[k] = a.C0 ? a.C0[sq * kD * kD + e] : 0.f;
+    for (int u = 0; u < 4; ++u) {
+        const int e = blk * kCombineBlock + u * 256 + threadIdx.x;
+        el[u] = e;
+        float x = 0.f;
+        if (e < kSS) x = a.S0 ? a.S0[sq * kSS + e] : 0.f;
+        else if (e < 2 * kSS) x = a.C0 ? a.C0[sq * kSS + e - kSS] : 0.f;
+        else if (e < 2 * kSS + kD) x = a.m0 ? a.m0[sq * kD + e - 2 * kSS] : 0.f;
+        cur[u] = x;
     }
-    float cm = (tid < kD && a.m0) ? a.m0[sq * kD + tid] : 0.f;
     for (int s = 0; s < a.nseg; ++s) {
         float *slot = a.seg_ws + (sq * a.nseg + s) * kSegFloats;
-        const float *D = slot + 2 * kD * kD + kD;
+        const float *D = slot + 2 * kSS + kD;
 #pragma unroll
-        for (int k = 0; k < 64; ++k) {
-            const int e = tid + 256 * k;
-            const float dS = slot[e], dC = slot[kD * kD + e];
-            slot[e] = cs[k];
-            slot[kD * kD + e] = cc[k];
-            cs[k] = fmaf(D[e >> 7], cs[k], dS);
-            cc[k] += dC;
+        for (int u = 0; u < 4; ++u) {
+            const int e = el[u];
+            if (e >= 2 * kSS + kD) continue;
+            const float d = slot[e];
+            slot[e] = cur[u];
+            cur[u] = (e < kSS ? D[e >> 7] * cur[u] : cur[u]) + d;
         }
-        if (tid < kD) {
-            const float dmv = slot[2 * kD * kD + tid];
-            slot[2 * kD * kD + tid] = cm;
-            cm += dmv;
-        }
-        __syncthreads();  // D of this slot read by every thread before the next slot
     }
 }
 
@@ -261,7 +263,8 @@ cudaError_t launch_gla_segments(const ChunkArgs &a, const ChunkMaps &m, cudaStre
     gla_segment_state_kernel<<<a.B * a.H * a.nseg, kThreads, kSmem, s>>>(m.k, m.v, m.g, a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    gla_segment_combine_kernel<<<a.B * a.H, 256, 0, s>>>(a);
+    const int nblk = (kSegFloats - kD + kCombineBlock - 1) / kCombineBlock;
+    gla_segment_combine_kernel<<<a.B * a.H * nblk, 256, 0, s>>>(a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     return launch_gla_chunk(a, m, s);
