@@ -13,6 +13,8 @@ Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``)
                      finite-difference Hessian identity.
   forward(chunk>0)   chunkwise form (Algorithm 1, App. B) -- pinned by equality
                      with the recurrent form.
+  gla_backward       reverse mode of the CCQ-GLA forward -- pinned by central
+                     finite differences of the forward (fp64).
   Absolute outputs on the benchmark-shaped random inputs are pinned only
   through the above: the paper prints no worked numerical example.
 """
@@ -20,6 +22,7 @@ from .ccq_oracle import (  # noqa: F401
     build_oracle,
     forward,
     decode_step,
+    gla_backward,
     GLA,
     GDN,
 )

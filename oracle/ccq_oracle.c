@@ -406,3 +406,262 @@ int ccq_oracle_forward(int backbone, int B, int T, int H, int Dk, int Dv,
     /* T == 0: the per-pair loops still copy the initial states through */
     return 0;
 }
+
+/* ====================================================================== reverse mode
+ *
+ * Gradients of the CCQ-GLA forward (recurrent form above) with respect to every
+ * input, by hand-written reverse mode.  Per (b, h): the forward states are
+ * checkpointed at every 64-token boundary; the tokens of each block are
+ * recomputed from its checkpoint (keeping every per-token state of the block),
+ * then walked backwards.  For token t (all sums and products of Algorithm 2):
+ *   o = scale S_t q_clean,  q_clean = qbar - lambda z,  z = Sigma_t qbar
+ *   Sigma_t qbar = C_t qbar / t - m_t (m_t . qbar) / t^2,  C_t = C_{t-1} + kbar kbar^T,
+ *   m_t = m_{t-1} + kbar,  S_t = Diag(e^{gk_t}) S_{t-1} + kbar v^T  (S stored [Dk][Dv]),
+ * the adjoints are
+ *   dq_clean = scale S_t do,  dS_t += scale q_clean do^T,  dz = -lambda dq_clean,
+ *   dlambda = -z . dq_clean,  dqbar = dq_clean + Sigma_t dz,
+ *   dC += dz qbar^T / t,  dm -= ((m . qbar) dz + (dz . m) qbar) / t^2,
+ *   dkbar = dS v + (dC + dC^T) kbar + dm,  dv = dS^T kbar,
+ *   dgk = e^{gk} * rowsum(dS * S_{t-1}),  dS <- Diag(e^{gk}) dS,
+ *   dx = (dxbar - xbar (xbar . dxbar)) / |x| for x = q, k (l2 normalisation).
+ */
+
+typedef struct {
+    int B, T, H, Dk, Dv, l2norm, centered;
+    double scale;
+    const double *q, *k, *v, *gk, *lam, *S0, *C0, *m0, *dout, *dST, *dCT, *dmT;
+    const int64_t *t0;
+    double *dq, *dk, *dv, *dgk, *dlam, *dS0, *dC0, *dm0;
+    int next;
+    pthread_mutex_t mu;
+} bjob_t;
+
+static size_t brow(const bjob_t *J, int b, int t, int h) { return ((size_t)b * J->T + t) * J->H + h; }
+
+static void normalise_with_norm(const double *x, double *y, double *nrm, int n, int enabled) {
+    if (!enabled) {
+        memcpy(y, x, sizeof(double) * (size_t)n);
+        *nrm = 1.0;
+        return;
+    }
+    double s = 0.0;
+    for (int i = 0; i < n; ++i) s += x[i] * x[i];
+    *nrm = sqrt(s);
+    const double r = s > 0.0 ? 1.0 / *nrm : 0.0;
+    for (int i = 0; i < n; ++i) y[i] = x[i] * r;
+}
+
+/* dx = (dxbar - xbar (xbar . dxbar)) / |x|; the zero row maps to zero */
+static void normalise_backward(const double *xbar, double nrm, const double *dxbar, double *dx, int n,
+                               int enabled) {
+    if (!enabled) {
+        memcpy(dx, dxbar, sizeof(double) * (size_t)n);
+        return;
+    }
+    if (nrm == 0.0) {
+        for (int i = 0; i < n; ++i) dx[i] = 0.0;
+        return;
+    }
+    double d = 0.0;
+    for (int i = 0; i < n; ++i) d += xbar[i] * dxbar[i];
+    for (int i = 0; i < n; ++i) dx[i] = (dxbar[i] - xbar[i] * d) / nrm;
+}
+
+static void backward_pair(const bjob_t *J, int b, int h) {
+    const int Dk = J->Dk, Dv = J->Dv, T = J->T, BL = 64;
+    const int NB = (T + BL - 1) / BL;
+    const size_t bh = (size_t)b * J->H + h;
+    const size_t SS = (size_t)Dk * Dv, CC = (size_t)Dk * Dk;
+    /* checkpoints at block starts */
+    double *ckS = malloc(sizeof(double) * SS * (NB + 1));
+    double *ckC = malloc(sizeof(double) * CC * (NB + 1));
+    double *ckm = malloc(sizeof(double) * Dk * (NB + 1));
+    /* per-token states of one block: S after each token (BL + 1 incl. the block start), C, m */
+    double *bS = malloc(sizeof(double) * SS * (BL + 1));
+    double *bC = malloc(sizeof(double) * CC * (BL + 1));
+    double *bm = malloc(sizeof(double) * Dk * (BL + 1));
+    double *qb = malloc(sizeof(double) * Dk), *kb = malloc(sizeof(double) * Dk);
+    double *z = malloc(sizeof(double) * Dk), *qc = malloc(sizeof(double) * Dk);
+    double *dqc = malloc(sizeof(double) * Dk), *dz = malloc(sizeof(double) * Dk);
+    double *dqb = malloc(sizeof(double) * Dk), *dkb = malloc(sizeof(double) * Dk);
+    double *dS = malloc(sizeof(double) * SS), *dC = malloc(sizeof(double) * CC);
+    double *dm = malloc(sizeof(double) * Dk);
+    const int64_t tstart = J->t0 ? J->t0[b] : 0;
+
+    if (J->S0) memcpy(ckS, J->S0 + bh * SS, sizeof(double) * SS); else memset(ckS, 0, sizeof(double) * SS);
+    if (J->C0) memcpy(ckC, J->C0 + bh * CC, sizeof(double) * CC); else memset(ckC, 0, sizeof(double) * CC);
+    if (J->m0) memcpy(ckm, J->m0 + bh * Dk, sizeof(double) * Dk); else memset(ckm, 0, sizeof(double) * Dk);
+
+    /* forward over the blocks, keeping only the block-start checkpoints */
+    for (int blk = 0; blk < NB; ++blk) {
+        double *S = ckS + SS * (blk + 1), *C = ckC + CC * (blk + 1), *m = ckm + (size_t)Dk * (blk + 1);
+        memcpy(S, ckS + SS * blk, sizeof(double) * SS);
+        memcpy(C, ckC + CC * blk, sizeof(double) * CC);
+        memcpy(m, ckm + (size_t)Dk * blk, sizeof(double) * Dk);
+        for (int tl = blk * BL; tl < T && tl < (blk + 1) * BL; ++tl) {
+            const size_t r = brow(J, b, tl, h);
+            double nk;
+            normalise_with_norm(J->k + r * Dk, kb, &nk, Dk, J->l2norm);
+            for (int i = 0; i < Dk; ++i) {
+                for (int j = 0; j < Dk; ++j) C[(size_t)i * Dk + j] += kb[i] * kb[j];
+                m[i] += kb[i];
+            }
+            for (int i = 0; i < Dk; ++i) {
+                const double a = exp(J->gk[r * Dk + i]);
+                for (int e = 0; e < Dv; ++e)
+                    S[(size_t)i * Dv + e] = a * S[(size_t)i * Dv + e] + kb[i] * J->v[r * Dv + e];
+            }
+        }
+    }
+
+    /* adjoints of the final states */
+    if (J->dST) memcpy(dS, J->dST + bh * SS, sizeof(double) * SS); else memset(dS, 0, sizeof(double) * SS);
+    if (J->dCT) memcpy(dC, J->dCT + bh * CC, sizeof(double) * CC); else memset(dC, 0, sizeof(double) * CC);
+    if (J->dmT) memcpy(dm, J->dmT + bh * Dk, sizeof(double) * Dk); else memset(dm, 0, sizeof(double) * Dk);
+
+    for (int blk = NB - 1; blk >= 0; --blk) {
+        const int t_lo = blk * BL, t_hi = (T < (blk + 1) * BL) ? T : (blk + 1) * BL;
+        /* recompute the block's per-token states: index 0 = block start, i + 1 = after token t_lo + i */
+        memcpy(bS, ckS + SS * blk, sizeof(double) * SS);
+        memcpy(bC, ckC + CC * blk, sizeof(double) * CC);
+        memcpy(bm, ckm + (size_t)Dk * blk, sizeof(double) * Dk);
+        for (int tl = t_lo; tl < t_hi; ++tl) {
+            const int ix = tl - t_lo;
+            const size_t r = brow(J, b, tl, h);
+            double nk;
+            normalise_with_norm(J->k + r * Dk, kb, &nk, Dk, J->l2norm);
+            const double *Sp = bS + SS * ix, *Cp = bC + CC * ix, *mp = bm + (size_t)Dk * ix;
+            double *Sn = bS + SS * (ix + 1), *Cn = bC + CC * (ix + 1), *mn = bm + (size_t)Dk * (ix + 1);
+            for (int i = 0; i < Dk; ++i) {
+                for (int j = 0; j < Dk; ++j) Cn[(size_t)i * Dk + j] = Cp[(size_t)i * Dk + j] + kb[i] * kb[j];
+                mn[i] = mp[i] + kb[i];
+                const double a = exp(J->gk[r * Dk + i]);
+                for (int e = 0; e < Dv; ++e)
+                    Sn[(size_t)i * Dv + e] = a * Sp[(size_t)i * Dv + e] + kb[i] * J->v[r * Dv + e];
+            }
+        }
+        for (int tl = t_hi - 1; tl >= t_lo; --tl) {
+            const int ix = tl - t_lo;
+            const size_t r = brow(J, b, tl, h);
+            const double tf = (double)(tstart + tl + 1);
+            const double *St = bS + SS * (ix + 1), *Sp = bS + SS * ix;
+            const double *Ct = bC + CC * (ix + 1), *mt = bm + (size_t)Dk * (ix + 1);
+            const double lam = J->lam[r];
+            const double *dor = J->dout + r * Dv, *vr = J->v + r * Dv, *gr = J->gk + r * Dk;
+            double nq, nk;
+            normalise_with_norm(J->q + r * Dk, qb, &nq, Dk, J->l2norm);
+            normalise_with_norm(J->k + r * Dk, kb, &nk, Dk, J->l2norm);
+            /* forward quantities of token t */
+            double mq = 0.0;
+            for (int j = 0; j < Dk; ++j) mq += mt[j] * qb[j];
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int j = 0; j < Dk; ++j) acc += Ct[(size_t)i * Dk + j] * qb[j];
+                z[i] = acc / tf - (J->centered ? mt[i] * mq / (tf * tf) : 0.0);
+                qc[i] = qb[i] - lam * z[i];
+            }
+            /* read: o = scale S_t q_clean */
+            double dl = 0.0;
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int e = 0; e < Dv; ++e) {
+                    acc += St[(size_t)i * Dv + e] * dor[e];
+                    dS[(size_t)i * Dv + e] += J->scale * qc[i] * dor[e];
+                }
+                dqc[i] = J->scale * acc;
+                dz[i] = -lam * dqc[i];
+                dl -= z[i] * dqc[i];
+            }
+            J->dlam[r] = dl;
+            /* clean: dqbar = dq_clean + Sigma_t dz; statistics adjoints */
+            double mdz = 0.0;
+            for (int j = 0; j < Dk; ++j) mdz += mt[j] * dz[j];
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int j = 0; j < Dk; ++j) acc += Ct[(size_t)i * Dk + j] * dz[j];
+                dqb[i] = dqc[i] + acc / tf - (J->centered ? mt[i] * mdz / (tf * tf) : 0.0);
+            }
+            for (int i = 0; i < Dk; ++i) {
+                for (int j = 0; j < Dk; ++j) dC[(size_t)i * Dk + j] += dz[i] * qb[j] / tf;
+                if (J->centered) dm[i] -= (mq * dz[i] + mdz * qb[i]) / (tf * tf);
+            }
+            /* write: S_t = Diag(alpha) S_{t-1} + kbar v^T */
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0, gs = 0.0;
+                for (int e = 0; e < Dv; ++e) {
+                    acc += dS[(size_t)i * Dv + e] * vr[e];
+                    gs += dS[(size_t)i * Dv + e] * Sp[(size_t)i * Dv + e];
+                }
+                dkb[i] = acc;
+                const double a = exp(gr[i]);
+                J->dgk[r * Dk + i] = a * gs;
+            }
+            for (int e = 0; e < Dv; ++e) {
+                double acc = 0.0;
+                for (int i = 0; i < Dk; ++i) acc += dS[(size_t)i * Dv + e] * kb[i];
+                J->dv[r * Dv + e] = acc;
+            }
+            for (int i = 0; i < Dk; ++i) {
+                const double a = exp(gr[i]);
+                for (int e = 0; e < Dv; ++e) dS[(size_t)i * Dv + e] *= a;
+            }
+            /* statistics: C_t = C_{t-1} + kbar kbar^T, m_t = m_{t-1} + kbar */
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int j = 0; j < Dk; ++j) acc += (dC[(size_t)i * Dk + j] + dC[(size_t)j * Dk + i]) * kb[j];
+                dkb[i] += acc + dm[i];
+            }
+            normalise_backward(qb, nq, dqb, J->dq + r * Dk, Dk, J->l2norm);
+            normalise_backward(kb, nk, dkb, J->dk + r * Dk, Dk, J->l2norm);
+        }
+    }
+    if (J->dS0) memcpy(J->dS0 + bh * SS, dS, sizeof(double) * SS);
+    if (J->dC0) memcpy(J->dC0 + bh * CC, dC, sizeof(double) * CC);
+    if (J->dm0) memcpy(J->dm0 + bh * Dk, dm, sizeof(double) * Dk);
+    free(ckS); free(ckC); free(ckm); free(bS); free(bC); free(bm); free(qb); free(kb); free(z); free(qc);
+    free(dqc); free(dz); free(dqb); free(dkb); free(dS); free(dC); free(dm);
+}
+
+static void *bworker(void *arg) {
+    bjob_t *J = (bjob_t *)arg;
+    for (;;) {
+        pthread_mutex_lock(&J->mu);
+        const int w = J->next++;
+        pthread_mutex_unlock(&J->mu);
+        if (w >= J->B * J->H) break;
+        backward_pair(J, w / J->H, w % J->H);
+    }
+    return NULL;
+}
+
+/*
+ * CCQ-GLA backward.  Inputs as ccq_oracle_forward (GLA) plus dout [B,T,H,Dv] and
+ * optional adjoints of the final states dST [B,H,Dk,Dv], dCT [B,H,Dk,Dk],
+ * dmT [B,H,Dk] (NULL = 0).  Outputs dq, dk [B,T,H,Dk], dv [B,T,H,Dv],
+ * dgk [B,T,H,Dk], dlam [B,T,H], dS0, dC0, dm0 (each may be NULL only for the
+ * initial-state gradients).  Returns 0, or -1 on a bad argument.
+ */
+int ccq_oracle_gla_backward(int B, int T, int H, int Dk, int Dv, const double *q, const double *k,
+                            const double *v, const double *gk, const double *lam, const double *S0,
+                            const double *C0, const double *m0, const int64_t *t0, const double *dout,
+                            const double *dST, const double *dCT, const double *dmT, double *dq,
+                            double *dk, double *dv, double *dgk, double *dlam, double *dS0, double *dC0,
+                            double *dm0, int l2norm, int centered, double scale, int nthreads) {
+    if (B < 0 || T < 0 || H < 0 || Dk <= 0 || Dv <= 0 || nthreads < 1) return -1;
+    if (!q || !k || !v || !gk || !lam || !dout || !dq || !dk || !dv || !dgk || !dlam) return -1;
+    bjob_t J;
+    memset(&J, 0, sizeof J);
+    J.B = B; J.T = T; J.H = H; J.Dk = Dk; J.Dv = Dv; J.l2norm = l2norm; J.centered = centered;
+    J.scale = scale;
+    J.q = q; J.k = k; J.v = v; J.gk = gk; J.lam = lam; J.S0 = S0; J.C0 = C0; J.m0 = m0; J.t0 = t0;
+    J.dout = dout; J.dST = dST; J.dCT = dCT; J.dmT = dmT;
+    J.dq = dq; J.dk = dk; J.dv = dv; J.dgk = dgk; J.dlam = dlam; J.dS0 = dS0; J.dC0 = dC0; J.dm0 = dm0;
+    pthread_mutex_init(&J.mu, NULL);
+    if (nthreads > B * H) nthreads = B * H > 0 ? B * H : 1;
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int i = 0; i < nthreads; ++i) pthread_create(&th[i], NULL, bworker, &J);
+    for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
+    free(th);
+    pthread_mutex_destroy(&J.mu);
+    return 0;
+}

@@ -48,6 +48,10 @@ def load_library(path: str):
         + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int,
            ctypes.c_int])
     lib.ccq_oracle_forward.restype = ctypes.c_int
+    lib.ccq_oracle_gla_backward.argtypes = (
+        [ctypes.c_int] * 5 + [dp] * 8 + [ip] + [dp] * 4 + [dp] * 8
+        + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int])
+    lib.ccq_oracle_gla_backward.restype = ctypes.c_int
     return lib
 
 
@@ -139,3 +143,34 @@ def decode_step(backbone, q, k, v, gate, lam, S, C, m, t, beta=None, *,
                   nthreads=nthreads)
     return {"o": res["o"][:, 0], "S": res["S"], "C": res["C"], "m": res["m"],
             "t": res["t"]}
+
+
+def gla_backward(q, k, v, gk, lam, dout, S0=None, C0=None, m0=None, t0=None, dST=None,
+                 dCT=None, dmT=None, *, l2norm=True, centered=True, scale=None,
+                 nthreads=None, lib=None):
+    """Reverse mode of the CCQ-GLA forward: gradients of sum(dout * o)
+    + sum(dST * S_T) + sum(dCT * C_T) + sum(dmT * m_T) with respect to
+    q, k, v, gk, lam, S0, C0, m0 (shapes as in :func:`forward`)."""
+    lib = lib or _load()
+    q, k, v, gk, lam, dout = map(_f64, (q, k, v, gk, lam, dout))
+    S0, C0, m0, dST, dCT, dmT = map(_f64, (S0, C0, m0, dST, dCT, dmT))
+    t0 = _i64(t0)
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    if scale is None:
+        scale = Dk ** -0.5
+    if nthreads is None:
+        nthreads = os.cpu_count() or 1
+    g = {"dq": np.zeros_like(q), "dk": np.zeros_like(k), "dv": np.zeros_like(v),
+         "dgk": np.zeros_like(gk), "dlam": np.zeros_like(lam),
+         "dS0": np.zeros((B, H, Dk, Dv)), "dC0": np.zeros((B, H, Dk, Dk)),
+         "dm0": np.zeros((B, H, Dk))}
+    rc = lib.ccq_oracle_gla_backward(
+        B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(gk), _ptr(lam), _ptr(S0), _ptr(C0),
+        _ptr(m0), _ptr(t0, ctypes.c_int64), _ptr(dout), _ptr(dST), _ptr(dCT), _ptr(dmT),
+        _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]), _ptr(g["dgk"]), _ptr(g["dlam"]),
+        _ptr(g["dS0"]), _ptr(g["dC0"]), _ptr(g["dm0"]), int(bool(l2norm)), int(bool(centered)),
+        float(scale), int(nthreads))
+    if rc != 0:
+        raise ValueError("ccq_oracle_gla_backward rejected its arguments")
+    return g
