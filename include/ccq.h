@@ -165,6 +165,71 @@ CCQ_API ccq_status ccq_decode_step(int backbone, const void *q, const void *k, c
                            const ccq_params *p, void *stream);
 
 /*
+ * Bytes of the checkpoint buffer ccq_gla_fwd_save writes for these sizes: per
+ * (sequence, head), 66048 bytes per 64-token chunk (the bf16 S^K and
+ * e^{Gmid} S of the chunk start, the fp32 key sum) plus 65536 bytes (fp32 S_T).
+ * Host-only.
+ */
+CCQ_API ccq_status ccq_gla_ckpt_size(int B, int T, int H, int Dk, int Dv, size_t *bytes);
+
+/*
+ * ccq_gla_fwd that also saves, into `ckpt` (device memory, at least
+ * ccq_gla_ckpt_size() bytes, 16-byte aligned), the chunk-start states the
+ * backward needs, so that ccq_gla_bwd does not recompute them (a training
+ * step's forward).  Only the chunkwise tensor-core path saves checkpoints:
+ * bf16 inputs, Dk = Dv = 128, T >= 1, algo AUTO or CHUNKWISE; anything else
+ * returns CCQ_ERR_UNSUPPORTED.  All other arguments as ccq_gla_fwd.
+ */
+CCQ_API ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v, const void *gk,
+                                    const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                                    const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                                    void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                                    int B, int T, int H, int Dk, int Dv, void *workspace,
+                                    size_t workspace_bytes, void *ckpt, size_t ckpt_bytes,
+                                    const ccq_params *p, void *stream);
+
+/*
+ * CCQ-GLA backward: the gradients of a scalar loss L through ccq_gla_fwd, given
+ * dL/do and (optionally) dL/d(final states).  The paper times a backward pass
+ * but does not write it out; it is the reverse mode of Eqs. clean/read, the
+ * running sums of Sec. 3.2 and the GLA write, chunked like Algorithm 1.
+ *   q, k, v, gk, lambda, in/gate dtypes, S0/C0/m0/t0   the forward's inputs.
+ *   dout      dL/do [B,T,H,Dv] in in_dtype.
+ *   dST [B,H,Dk,Dv], dCT [B,H,Dk,Dk], dmT [B,H,Dk] fp32: dL/d(ST, CT, mT); NULL = 0.
+ *   ckpt      checkpoints written by ccq_gla_fwd_save on the same inputs, or
+ *             NULL: the call then recomputes them (one forward pass without
+ *             the output) into the workspace.
+ *   dq, dk    [B,T,H,Dk], dv [B,T,H,Dv] in in_dtype; dgk [B,T,H,Dk] in
+ *             gate_dtype: gradients of q, k, v and gk (the raw, un-normalised
+ *             q and k when l2norm_qk = 1).
+ *   dlambda   [B,T,H] fp32 (may be NULL);  dS0 [B,H,Dk,Dv], dC0 [B,H,Dk,Dk],
+ *             dm0 [B,H,Dk] fp32 (each may be NULL): gradients of lambda and of
+ *             the initial states.
+ *   workspace at least ccq_gla_bwd_workspace_size() bytes (16-byte aligned):
+ *             three bf16 [B,T,H,128] tensors the two backward kernels exchange,
+ *             plus the checkpoints and forward scratch when ckpt is NULL.
+ * Supported: bf16 inputs with Dk = Dv = 128 (the chunkwise tensor-core path),
+ * algo AUTO or CHUNKWISE; otherwise CCQ_ERR_UNSUPPORTED.  T = 0 copies the
+ * final-state gradients to the initial-state ones.
+ */
+CCQ_API ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *gk,
+                               const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                               const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                               const void *dout, const float *dST, const float *dCT, const float *dmT,
+                               const void *ckpt, void *dq, void *dk, void *dv, void *dgk,
+                               float *dlambda, float *dS0, float *dC0, float *dm0,
+                               int B, int T, int H, int Dk, int Dv, void *workspace,
+                               size_t workspace_bytes, const ccq_params *p, void *stream);
+
+/*
+ * Workspace bytes ccq_gla_bwd needs; with_ckpt = 1 when the caller passes
+ * checkpoints (then only the exchange tensors), 0 otherwise.  Queries the
+ * device (the forward's segment split) but launches nothing.
+ */
+CCQ_API ccq_status ccq_gla_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                              int with_ckpt, const ccq_params *p, size_t *bytes);
+
+/*
  * ccq_gla_fwd for callers that cannot supply any device memory of their own --
  * for instance an engine that gave all device memory to its own caches at
  * start-up, or code on a path where allocating is not allowed or would stall

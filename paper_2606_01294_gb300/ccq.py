@@ -78,6 +78,18 @@ def load_library() -> ctypes.CDLL:
         lib.ccq_decode_step.argtypes = ([_I] + [_VP] * 6 + [_I, _I] + [_VP] * 5
                                         + [_I] * 4 + [ctypes.POINTER(_Params), _VP])
         lib.ccq_decode_step.restype = _I
+        lib.ccq_gla_ckpt_size.argtypes = [_I] * 5 + [ctypes.POINTER(ctypes.c_size_t)]
+        lib.ccq_gla_ckpt_size.restype = _I
+        lib.ccq_gla_fwd_save.argtypes = ([_VP] * 5 + [_I, _I] + [_VP] * 9 + [_I] * 5
+                                         + [_VP, ctypes.c_size_t, _VP, ctypes.c_size_t,
+                                            ctypes.POINTER(_Params), _VP])
+        lib.ccq_gla_fwd_save.restype = _I
+        lib.ccq_gla_bwd.argtypes = ([_VP] * 5 + [_I, _I] + [_VP] * 17 + [_I] * 5
+                                    + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
+        lib.ccq_gla_bwd.restype = _I
+        lib.ccq_gla_bwd_workspace_size.argtypes = ([_I] * 7 + [ctypes.POINTER(_Params),
+                                                               ctypes.POINTER(ctypes.c_size_t)])
+        lib.ccq_gla_bwd_workspace_size.restype = _I
         _lib = lib
     return _lib
 
@@ -219,6 +231,115 @@ def gla_fwd(q, k, v, gk, lam, state: Optional[CCQState] = None, *, out=None,
         ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
+
+
+def gla_ckpt_size(B, T, H, Dk=128, Dv=128) -> int:
+    """Bytes of the checkpoint buffer :func:`gla_fwd_save` writes."""
+    need = ctypes.c_size_t(0)
+    _check(load_library().ccq_gla_ckpt_size(B, T, H, Dk, Dv, ctypes.byref(need)))
+    return need.value
+
+
+def gla_fwd_save(q, k, v, gk, lam, state: Optional[CCQState] = None, *, ckpt=None, out=None,
+                 final_state: Optional[CCQState] = None, return_state: bool = True,
+                 workspace: Optional[torch.Tensor] = None, stream=None, **kw):
+    """:func:`gla_fwd` that also writes the chunk-start states the backward
+    needs into ``ckpt`` (a CUDA uint8 tensor of :func:`gla_ckpt_size` bytes,
+    allocated when not given).  Returns (o, final_state, ckpt)."""
+    dev = q.device
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, T, H, Dv))
+    _req(gk, "gk", dev, None, (B, T, H, Dk))
+    _req(lam, "lam", dev, torch.float32, (B, T, H))
+    S0, C0, m0, t0 = _state_in(state, B, H, Dk, Dv, dev)
+    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
+    _req(o, "out", dev, q.dtype, (B, T, H, Dv))
+    fs = final_state
+    if fs is None and return_state:
+        fs = CCQState.empty(B, H, Dk, Dv, dev)
+    if ckpt is None:
+        ckpt = torch.empty(gla_ckpt_size(B, T, H, Dk, Dv), dtype=torch.uint8, device=dev)
+    _req(ckpt, "ckpt", dev, torch.uint8)
+    p = params(**kw)
+    lib = load_library()
+    if workspace is None:
+        need = ctypes.c_size_t(0)
+        _check(lib.ccq_gla_workspace_size(B, T, H, Dk, Dv, _dtype_code(q), ctypes.byref(p),
+                                          ctypes.byref(need)))
+        if need.value:
+            workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_gla_fwd_save(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gk), _ptr(lam), _dtype_code(q), _dtype_code(gk),
+        _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(o),
+        _ptr(fs.S if fs else None), _ptr(fs.C if fs else None), _ptr(fs.m if fs else None),
+        _ptr(fs.t if fs else None), B, T, H, Dk, Dv, _ptr(workspace), ws_bytes,
+        _ptr(ckpt), ckpt.numel(), ctypes.byref(p), _stream(dev, stream))
+    _check(st)
+    return o, fs, ckpt
+
+
+def gla_bwd_workspace(B, T, H, Dk, Dv, device, *, with_ckpt: bool, dtype=torch.bfloat16, **kw):
+    """Allocate the workspace ccq_gla_bwd needs (None if none)."""
+    p = params(**kw)
+    need = ctypes.c_size_t(0)
+    code = BF16 if dtype == torch.bfloat16 else FP32
+    _check(load_library().ccq_gla_bwd_workspace_size(B, T, H, Dk, Dv, code, int(bool(with_ckpt)),
+                                                      ctypes.byref(p), ctypes.byref(need)))
+    return torch.empty(need.value, dtype=torch.uint8, device=device) if need.value else None
+
+
+def gla_bwd(q, k, v, gk, lam, dout, state: Optional[CCQState] = None, *, dST=None, dCT=None,
+            dmT=None, ckpt=None, out: Optional[dict] = None, workspace=None, stream=None, **kw):
+    """CCQ-GLA backward.  Returns a dict of gradients dq, dk, dv (q's dtype),
+    dgk (gk's dtype), dlambda, dS0, dC0, dm0 (fp32).  ``dST``/``dCT``/``dmT`` are
+    the gradients of the final states (None = 0); ``ckpt`` the checkpoints of
+    :func:`gla_fwd_save` on the same inputs (None = recompute them).  ``out``
+    may hold preallocated tensors under those names."""
+    dev = q.device
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, T, H, Dv))
+    _req(gk, "gk", dev, None, (B, T, H, Dk))
+    _req(lam, "lam", dev, torch.float32, (B, T, H))
+    _req(dout, "dout", dev, q.dtype, (B, T, H, Dv))
+    S0, C0, m0, t0 = _state_in(state, B, H, Dk, Dv, dev)
+    if dST is not None:
+        _req(dST, "dST", dev, torch.float32, (B, H, Dk, Dv))
+    if dCT is not None:
+        _req(dCT, "dCT", dev, torch.float32, (B, H, Dk, Dk))
+    if dmT is not None:
+        _req(dmT, "dmT", dev, torch.float32, (B, H, Dk))
+    if ckpt is not None:
+        _req(ckpt, "ckpt", dev, torch.uint8)
+    g = dict(out or {})
+    shapes = {"dq": ((B, T, H, Dk), q.dtype), "dk": ((B, T, H, Dk), q.dtype),
+              "dv": ((B, T, H, Dv), q.dtype), "dgk": ((B, T, H, Dk), gk.dtype),
+              "dlambda": ((B, T, H), torch.float32), "dS0": ((B, H, Dk, Dv), torch.float32),
+              "dC0": ((B, H, Dk, Dk), torch.float32), "dm0": ((B, H, Dk), torch.float32)}
+    for name, (shape, dt) in shapes.items():
+        if g.get(name) is None:
+            g[name] = torch.empty(shape, dtype=dt, device=dev)
+        _req(g[name], name, dev, dt, shape)
+    p = params(**kw)
+    lib = load_library()
+    if workspace is None:
+        workspace = gla_bwd_workspace(B, T, H, Dk, Dv, dev, with_ckpt=ckpt is not None,
+                                      dtype=q.dtype, **kw)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_gla_bwd(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(gk), _ptr(lam), _dtype_code(q), _dtype_code(gk),
+        _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(dout), _ptr(dST), _ptr(dCT), _ptr(dmT),
+        _ptr(ckpt), _ptr(g["dq"]), _ptr(g["dk"]), _ptr(g["dv"]), _ptr(g["dgk"]),
+        _ptr(g["dlambda"]), _ptr(g["dS0"]), _ptr(g["dC0"]), _ptr(g["dm0"]),
+        B, T, H, Dk, Dv, _ptr(workspace), ws_bytes, ctypes.byref(p), _stream(dev, stream))
+    _check(st)
+    return g
 
 
 def gdn_fwd(q, k, v, g, beta, lam, state: Optional[CCQState] = None, *, out=None,

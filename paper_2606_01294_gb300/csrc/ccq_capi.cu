@@ -226,12 +226,16 @@ ccq_status ccq_gla_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype
     return CCQ_OK;
 }
 
-ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
-                       const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
-                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
-                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
-                       int B, int T, int H, int Dk, int Dv, void *workspace,
-                       size_t workspace_bytes, const ccq_params *p, void *stream) {
+// The GLA forward behind ccq_gla_fwd, ccq_gla_fwd_save and the backward's
+// checkpoint recompute: ckpt (nullable) receives the chunk-start states,
+// skip_o suppresses the output.
+static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, const void *gk,
+                               const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                               const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                               void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                               int B, int T, int H, int Dk, int Dv, void *workspace,
+                               size_t workspace_bytes, uint8_t *ckpt, int skip_o, const ccq_params *p,
+                               void *stream) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
@@ -246,8 +250,10 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
     }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bool chunk_ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
-    if (c.p.algo == CCQ_ALGO_CHUNKWISE && !chunk_ok)
+    if ((c.p.algo == CCQ_ALGO_CHUNKWISE || ckpt) && !chunk_ok)
         return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
+    if (ckpt && c.p.algo == CCQ_ALGO_RECURRENT)
+        return fail(CCQ_ERR_UNSUPPORTED, "checkpoints come from the chunkwise kernel (algo recurrent given)");
     if (chunk_ok && c.p.algo != CCQ_ALGO_RECURRENT) {
         int nseg = 1, seg_chunks = 0;
         gla_split(c.p, B, T, H, &nseg, &seg_chunks);
@@ -278,6 +284,8 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
         if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
         a.nseg = nseg;
         a.seg_chunks = seg_chunks;
+        a.ckpt = ckpt;
+        a.skip_o = skip_o;
         if (a.nseg > 1) {
             a.seg_ws = static_cast<float *>(workspace);
             cudaError_t e = launch_gla_segments(a, maps, s);
@@ -296,6 +304,154 @@ ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *
     ra.S0 = S0; ra.C0 = C0; ra.m0 = m0; ra.t0 = t0;
     ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT; ra.tT = tT;
     return run_recurrent(ra, s);
+}
+
+ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
+                       const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream) {
+    return gla_fwd_impl(q, k, v, gk, lambda, in_dtype, gate_dtype, S0, C0, m0, t0, o, ST, CT, mT, tT, B, T,
+                        H, Dk, Dv, workspace, workspace_bytes, nullptr, 0, p, stream);
+}
+
+ccq_status ccq_gla_ckpt_size(int B, int T, int H, int Dk, int Dv, size_t *bytes) {
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    if (B < 1 || H < 1 || T < 0) return fail(CCQ_ERR_INVALID_ARG, "bad sizes B=%d T=%d H=%d", B, T, H);
+    if (Dk != 128 || Dv != 128) return fail(CCQ_ERR_UNSUPPORTED, "checkpoints need Dk = Dv = 128");
+    *bytes = static_cast<size_t>(B) * H * ckpt_head_bytes(T);
+    return CCQ_OK;
+}
+
+ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v, const void *gk,
+                            const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                            const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                            void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                            int B, int T, int H, int Dk, int Dv, void *workspace,
+                            size_t workspace_bytes, void *ckpt, size_t ckpt_bytes,
+                            const ccq_params *p, void *stream) {
+    size_t need = 0;
+    ccq_status st = ccq_gla_ckpt_size(B, T, H, Dk, Dv, &need);
+    if (st != CCQ_OK) return st;
+    if (!ckpt || ckpt_bytes < need)
+        return fail(CCQ_ERR_INVALID_ARG, "checkpoint buffer of %zu bytes required (got %zu)", need,
+                    ckpt ? ckpt_bytes : static_cast<size_t>(0));
+    if (!aligned16(ckpt)) return fail(CCQ_ERR_INVALID_ARG, "ckpt is not 16-byte aligned");
+    return gla_fwd_impl(q, k, v, gk, lambda, in_dtype, gate_dtype, S0, C0, m0, t0, o, ST, CT, mT, tT, B, T,
+                        H, Dk, Dv, workspace, workspace_bytes, static_cast<uint8_t *>(ckpt), 0, p, stream);
+}
+
+// Workspace layout of ccq_gla_bwd: three bf16 [B,T,H,128] exchange tensors,
+// then (without caller checkpoints) the checkpoints and the forward's scratch.
+static size_t gla_bwd_exchange_bytes(int B, int T, int H) {
+    return 3 * static_cast<size_t>(B) * T * H * 128 * 2;
+}
+
+static size_t gla_fwd_scratch_bytes(const ccq_params &p, int B, int T, int H) {
+    int ns, per;
+    gla_split(p, B, T, H, &ns, &per);
+    return ns > 1 ? static_cast<size_t>(B) * H * ns * kSegFloats * sizeof(float) : 0;
+}
+
+ccq_status ccq_gla_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                      int with_ckpt, const ccq_params *p, size_t *bytes) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    if (in_dtype != CCQ_BF16 || Dk != 128)
+        return fail(CCQ_ERR_UNSUPPORTED, "the backward needs bf16 inputs and Dk = Dv = 128");
+    *bytes = 0;
+    if (T == 0) return CCQ_OK;
+    *bytes = gla_bwd_exchange_bytes(B, T, H);
+    if (!with_ckpt) *bytes += static_cast<size_t>(B) * H * ckpt_head_bytes(T) + gla_fwd_scratch_bytes(c.p, B, T, H);
+    return CCQ_OK;
+}
+
+ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *gk,
+                       const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       const void *dout, const float *dST, const float *dCT, const float *dmT,
+                       const void *ckpt, void *dq, void *dk, void *dv, void *dgk,
+                       float *dlambda, float *dS0, float *dC0, float *dm0,
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if ((in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) || (gate_dtype != CCQ_BF16 && gate_dtype != CCQ_FP32))
+        return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    if (in_dtype != CCQ_BF16 || Dk != 128)
+        return fail(CCQ_ERR_UNSUPPORTED, "the backward needs bf16 inputs and Dk = Dv = 128");
+    if (c.p.algo == CCQ_ALGO_RECURRENT)
+        return fail(CCQ_ERR_UNSUPPORTED, "the backward is chunkwise only (algo recurrent given)");
+    st = check_ptrs("", {}, {S0, C0, m0, t0, dST, dCT, dmT, ckpt, dlambda, dS0, dC0, dm0});
+    if (st != CCQ_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) {
+        // no tokens: the initial states are the final states
+        const size_t n[3] = {static_cast<size_t>(B) * H * Dk * Dv * 4, static_cast<size_t>(B) * H * Dk * Dk * 4,
+                             static_cast<size_t>(B) * H * Dk * 4};
+        float *dst[3] = {dS0, dC0, dm0};
+        const float *src[3] = {dST, dCT, dmT};
+        for (int i = 0; i < 3; ++i) {
+            if (!dst[i]) continue;
+            cudaError_t e = src[i] ? cudaMemcpyAsync(dst[i], src[i], n[i], cudaMemcpyDeviceToDevice, s)
+                                   : cudaMemsetAsync(dst[i], 0, n[i], s);
+            if (e != cudaSuccess) return cuda_fail(e, "state gradient copy");
+        }
+        return CCQ_OK;
+    }
+    st = check_ptrs("q,k,v,gk,lambda,dout,dq,dk,dv,dgk", {q, k, v, gk, lambda, dout, dq, dk, dv, dgk}, {});
+    if (st != CCQ_OK) return st;
+    size_t need = gla_bwd_exchange_bytes(B, T, H);
+    const size_t ck_bytes = static_cast<size_t>(B) * H * ckpt_head_bytes(T);
+    const size_t fwd_bytes = ckpt ? 0 : gla_fwd_scratch_bytes(c.p, B, T, H);
+    if (!ckpt) need += ck_bytes + fwd_bytes;
+    if (!workspace || workspace_bytes < need)
+        return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
+                    workspace ? workspace_bytes : static_cast<size_t>(0));
+    if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    const size_t xbytes = static_cast<size_t>(B) * T * H * 128 * 2;
+    uint8_t *qg = ws, *dkc = ws + xbytes, *gq = ws + 2 * xbytes;
+    const uint8_t *ck = static_cast<const uint8_t *>(ckpt);
+    if (!ckpt) {
+        uint8_t *own = ws + 3 * xbytes;
+        // forward without output: dq stands in for the unused output tensor
+        st = gla_fwd_impl(q, k, v, gk, lambda, in_dtype, gate_dtype, S0, C0, m0, t0, dq, nullptr, nullptr,
+                          nullptr, nullptr, B, T, H, Dk, Dv, fwd_bytes ? own + ck_bytes : nullptr, fwd_bytes,
+                          own, 1, &c.p, stream);
+        if (st != CCQ_OK) return st;
+        ck = own;
+    }
+    BwdMaps maps;
+    const int geb = gate_dtype == CCQ_BF16 ? 2 : 4;
+    if (!make_token_map(&maps.q, q, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.k, k, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.v, v, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.dO, dout, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.g, gk, geb, B, T, H, 128, 128, false) ||
+        !make_token_map(&maps.dq, dq, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.dk, dk, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.dv, dv, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.qg, qg, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.dkc, dkc, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.gq, gq, 2, B, T, H, 128, 64, true))
+        return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
+    BwdArgs a = {};
+    a.B = B; a.T = T; a.H = H;
+    a.gate_dtype = gate_dtype == CCQ_BF16 ? 0 : 1;
+    a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
+    a.lambda = lambda; a.t0 = t0; a.ckpt = ck;
+    a.dST = dST; a.dCT = dCT; a.dmT = dmT;
+    a.dlambda = dlambda; a.dgk = dgk; a.dS0 = dS0; a.dC0 = dC0; a.dm0 = dm0;
+    a.status = device_status_word();
+    if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
+    cudaError_t e = launch_gla_bwd(a, maps, s);
+    if (e != cudaSuccess) return cuda_fail(e, "GLA backward kernel launch");
+    return CCQ_OK;
 }
 
 static bool gdn_chunk_selected(const ccq_params &p, ccq_dtype in_dtype, int Dk, int T) {

@@ -123,7 +123,7 @@ extern "C" CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *
                                            int K, int a_mn, int b_mn, void *stream) {
     if (!A || !B || !D) return CCQ_ERR_INVALID_ARG;
     if ((M != 64 && M != 128) || (N != 64 && N != 128) || (K != 64 && K != 128) ||
-        (a_mn | b_mn) > 1 || a_mn < 0 || b_mn < 0 || (M == 64 && a_mn))
+        (a_mn | b_mn) > 1 || a_mn < 0 || b_mn < 0)
         return CCQ_ERR_UNSUPPORTED;
     int *status = ccq::device_status_word();
     if (!status) return CCQ_ERR_CUDA;

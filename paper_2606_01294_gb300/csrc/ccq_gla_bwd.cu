@@ -1,0 +1,983 @@
+// ccq_gla_bwd.cu -- chunkwise CCQ-GLA backward on sm_103a tensor cores.
+//
+// Reverse mode of the chunkwise forward (Algorithm 1 with the GLA write,
+// Eqs. clean/read, the undecayed running sums of Section 3.2).  The paper
+// times a backward but gives none; the adjoint below is derived from those
+// definitions and checked against the oracle's reverse mode, which is itself
+// pinned by finite differences.
+//
+// Per chunk r (tokens i, positions t_i, qbar/kbar the unit rows, G the
+// in-chunk cumulative log gate, Gmid its value after token 31, Gc after token
+// 63, S_r / S^K_r / M_r the forward states at the chunk start, EG = e^{G-Gmid},
+// Kd = kbar e^{Gmid-G}, Sx_r = e^{Gmid} S_r):
+//   z_i    = Sigma_{t_i} qbar_i = (Zi_i - c1_i M_r) / t_i,  Zi = Qbar S^K + W2 Kbar,
+//            c1_i = m_i . qbar_i / t_i,  W2_ij = [j<=i](qbar_i . kbar_j - c1_i)
+//   qc_i   = qbar_i - lambda_i z_i                             (Eq. clean)
+//   dqc_i  = scale S_{t_i} do_i = scale EG_i (dO Sx_r^T + P1 Kd)_i,  P1_ij = [j<=i] do_i . v_j
+//   dlambda_i = -z_i . dqc_i
+//   dz'_i  = -lambda_i dqc_i / t_i   (adjoint of z_i, divided by t_i)
+//   dqbar_i = dqc_i + C_{t_i} dz'_i - m_i (m_i . dz'_i) / t_i = dqc_i + u_i - cz_i M_r,
+//            u = DZ S^K + W3 Kbar,  cz_i = m_i . dz'_i / t_i,  W3_ij = [j<=i](dz'_i . kbar_j - cz_i)
+//   carried backwards over chunks (no decay):
+//            DC = dC_T + sum dz'_t qbar_t^T      (adjoint of the second-moment sum)
+//            Dm = dm_T - sum (c1_t dz'_t + cz_t qbar_t)   (adjoint of the key sum)
+//   dkbar_j (CCQ part) = (DC_{r+1} + DC_{r+1}^T) kbar_j + Dm_{r+1} + (W2^T DZ + W3^T Qbar)_j
+//   GLA adjoint with q_clean as the query (QG = scale qc EG):
+//            dS_r  = Diag(e^{Gc}) dS_{r+1} + Diag(e^{Gmid}) QG^T dO
+//            dkbar_j (write part) = e^{Gmid-G_j} (V dSs^T + P1^T QG)_j,  dSs = Diag(e^{Gc-Gmid}) dS_{r+1}
+//            dv_j  = (Kd dSs + SA dO)_j,  SA_jt = [t>=j] Kd_j . QG_t
+//            dG_t  = qc_t dqc_t - kbar_t dkbar_t(write);  dgk_t = sum_{s>=t} dG_s + rowsum(dS_T S_T),
+//            evaluated per chunk as sum_{s>=t in chunk r} dG_s + rowsum(dS_{r+1} S_{r+1})
+//   l2 normalisation: dq = (dqbar - qbar (qbar . dqbar)) / |q|, likewise dk.
+//
+// Two kernels, one CTA per (batch, head), chunks in reverse order; each keeps
+// its carried state in tensor memory as an fp32 accumulator:
+//   gla_bwd_q_kernel   DC (TMEM) and Dm: recomputes z and qc, forms dqc, dq,
+//                      dlambda and the CCQ part of dkbar; writes QG, qc*dqc
+//                      and that dkbar part to bf16 scratch tensors.
+//   gla_bwd_kv_kernel  dS (TMEM, kept as e^{-Gmid} dS like the forward's
+//                      deferred state scaling): dk, dv and dgk.
+// The forward states of each chunk come from the checkpoints the forward
+// kernel writes (ccq_internal.h); 64-row products are M = 64 MMAs whose rows
+// 16q..16q+15 sit in TMEM lanes 32q..32q+15, so thread (warp w, lane l) owns
+// row 16w + l % 16 and column half l / 16 in every epilogue.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ccq_internal.h"
+#include "sm100_ptx.cuh"
+
+namespace ccq {
+
+namespace {
+
+constexpr int kC = 64;
+constexpr int kD = 128;
+constexpr int kThreads = 128;
+constexpr float kLog2e = 1.4426950408889634f;
+
+constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
+constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
+constexpr uint32_t ID_64x128_KM = make_idesc(64, 128, 0, 1);
+constexpr uint32_t ID_64x128_MM = make_idesc(64, 128, 1, 1);
+constexpr uint32_t ID_128x128_MM = make_idesc(128, 128, 1, 1);
+constexpr uint32_t ID_128x64_MK = make_idesc(128, 64, 1, 0);
+
+__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
+    return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
+}
+
+__device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chunk, const float *w) {
+    uint4 u;
+    u.x = pack_bf16(w[0], w[1]);
+    u.y = pack_bf16(w[2], w[3]);
+    u.z = pack_bf16(w[4], w[5]);
+    u.w = pack_bf16(w[6], w[7]);
+    *reinterpret_cast<uint4 *>(tile + t64_chunk(row, chunk)) = u;
+}
+
+__device__ __forceinline__ void load_row_chunk(const uint8_t *tile, int row, int chunk, float (&f)[8]) {
+    unpack_bf16x8(*reinterpret_cast<const uint4 *>(tile + t64_chunk(row, chunk)), f);
+}
+
+// Chunk preparation shared by both kernels (all 128 threads).  Normalises the
+// k rows (and the q rows when q_tile is set) of the chunk in place and turns
+// the raw gates landed at kd_tile (a plain [64][128] array, bf16 or fp32; the
+// fp32 one also covers eg_tile) into the tiles Kd = kbar e^{Gmid-G} and
+// EG = e^{G-Gmid}.  Outputs per row: rq (1/|q|), mq (M_r . qbar), rk (1/|k|);
+// per key dim (when non-null): f = e^{Gc-Gmid}, emid = e^{Gmid}.
+__device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, uint8_t *eg_tile,
+                           bool gate_f32, bool l2norm, const float *Mr, float *rq, float *mq, float *rk,
+                           float *gmid, float *f, float *emid, int wt) {
+    {
+        const bool isq = q_tile != nullptr && wt < 64;
+        const bool active = q_tile != nullptr || wt < 64;
+        const int row = wt & 63;
+        uint8_t *base = isq ? q_tile : k_tile;
+        if (active) {
+            float ss = 0.f, md = 0.f;
+#pragma unroll
+            for (int t64 = 0; t64 < 2; ++t64) {
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc) {
+                    float x[8];
+                    load_row_chunk(base + t64 * 8192, row, cc, x);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        ss = fmaf(x[e], x[e], ss);
+                        if (isq) md = fmaf(x[e], Mr[64 * t64 + 8 * cc + e], md);
+                    }
+                }
+            }
+            const float rn = l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+            if (l2norm) {
+#pragma unroll
+                for (int t64 = 0; t64 < 2; ++t64) {
+#pragma unroll
+                    for (int cc = 0; cc < 8; ++cc) {
+                        float x[8];
+                        load_row_chunk(base + t64 * 8192, row, cc, x);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) x[e] *= rn;
+                        store_row_chunk(base + t64 * 8192, row, cc, x);
+                    }
+                }
+            }
+            if (isq) {
+                rq[row] = rn;
+                mq[row] = md * rn;
+            } else {
+                rk[row] = rn;
+            }
+        }
+    }
+    __syncthreads();
+    const int p = wt & 63, th = wt >> 6, d0 = 2 * p;
+    float g0[32], g1[32];
+    float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+        const int j = 32 * th + jj;
+        float x0, x1;
+        if (gate_f32) {
+            const float2 f2 = *reinterpret_cast<const float2 *>(kd_tile + (j * kD + d0) * 4);
+            x0 = f2.x; x1 = f2.y;
+        } else {
+            const float2 f2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(kd_tile + (j * kD + d0) * 2));
+            x0 = f2.x; x1 = f2.y;
+        }
+        r0 += x0; r1 += x1;
+        g0[jj] = r0; g1[jj] = r1;
+    }
+    if (th == 0) {
+        gmid[d0] = r0;
+        gmid[d0 + 1] = r1;
+    }
+    __syncthreads();  // every raw gate read, Gmid visible
+    const float gm0 = gmid[d0], gm1 = gmid[d0 + 1];
+    const float o0 = th ? 0.f : -gm0 * kLog2e, o1 = th ? 0.f : -gm1 * kLog2e;
+    if (th == 1) {
+        if (f) {
+            f[d0] = fast_exp2(r0 * kLog2e);
+            f[d0 + 1] = fast_exp2(r1 * kLog2e);
+        }
+        if (emid) {
+            emid[d0] = fast_exp2(gm0 * kLog2e);
+            emid[d0 + 1] = fast_exp2(gm1 * kLog2e);
+        }
+    }
+    const uint32_t tcol = (d0 >> 6) * 8192;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj) {
+        const int j = 32 * th + jj;
+        const uint32_t off = tcol + t64_offset(j, d0 & 63);
+        const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(k_tile + off));
+        const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
+        *reinterpret_cast<uint32_t *>(kd_tile + off) = pack_bf16(kr.x * fast_exp2(-x0), kr.y * fast_exp2(-x1));
+        *reinterpret_cast<uint32_t *>(eg_tile + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
+    }
+    fence_proxy_async_smem();
+    __syncthreads();
+}
+
+// Masked row of a 64 x 64 score tile: w_j = [j <= i] (sc_j - c) for the 32
+// columns [32 hf, 32 hf + 32) this thread holds; also returns the masked sum.
+__device__ __forceinline__ void masked_row(uint8_t *tile, int i, int hf, const float (&sc)[32], float c) {
+#pragma unroll
+    for (int q4 = 0; q4 < 4; ++q4) {
+        float w[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int j = 32 * hf + 8 * q4 + e;
+            w[e] = (j <= i) ? sc[8 * q4 + e] - c : 0.f;
+        }
+        store_row_chunk(tile, i, 4 * hf + q4, w);
+    }
+}
+
+__device__ __forceinline__ float masked_sum(int i, int hf, const float (&sc)[32]) {
+    float part = 0.f;
+#pragma unroll
+    for (int jj = 0; jj < 32; ++jj)
+        if (32 * hf + jj <= i) part += sc[jj];
+    return part + __shfl_xor_sync(0xffffffffu, part, 16);
+}
+
+// =====================================================================================
+// gla_bwd_q_kernel
+// =====================================================================================
+namespace qk {
+constexpr uint32_t OFF_Q = 0;        // qbar; then dq (staged for the store)
+constexpr uint32_t OFF_K = 16384;    // kbar; then the CCQ part of dkbar (staged)
+constexpr uint32_t OFF_V = 32768;    // v; then QG (staged)
+constexpr uint32_t OFF_DO = 49152;   // do; then DZ
+constexpr uint32_t OFF_KD = 65536;   // raw gates land here (fp32: KD + EG); then Kd
+constexpr uint32_t OFF_EG = 81920;   // EG
+constexpr uint32_t OFF_SK = 98304;   // S^K_r      } one checkpoint record,
+constexpr uint32_t OFF_SX = 131072;  // Sx_r       } one bulk copy; then dqc (16K) + qc*dqc (16K)
+constexpr uint32_t OFF_DC = 163840;  // bf16 DC_{r+1}
+constexpr uint32_t OFF_W2 = 196608;  // W2
+constexpr uint32_t OFF_P1 = 204800;  // P1, then W3
+constexpr uint32_t OFF_BC = 212992;  // [64][64] K-major B operand of the Dm update: row 0 = -c1, then -cz
+constexpr uint32_t OFF_MISC = 221184;
+constexpr uint32_t M_MR = 0, M_DM = 512, M_RQ = 1024, M_LAM = 1280, M_ITAU = 1536, M_MQ = 1792,
+                   M_C1 = 2048, M_MDZ = 2304, M_CZ = 2560, M_RK = 2816, M_GP = 3072, M_BAR = 3584,
+                   M_TMEM = 3632, M_ABORT = 3636;
+constexpr uint32_t kMisc = 3712;
+constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
+static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
+static_assert(OFF_SX == OFF_SK + 32768, "a checkpoint record lands as one block");
+enum { BAR_IN = 0, BAR_R1, BAR_R2, BAR_R3, BAR_R4, kBars };
+constexpr uint32_t TM_DC = 0, TM_SC = 128, TM_T1 = 192, TM_Z = 256, TM_DQ = 384;
+}  // namespace qk
+
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
+                 const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
+                 const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
+                 const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
+                 const __grid_constant__ CUtensorMap map_gq, const BwdArgs a) {
+    using namespace qk;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    const uint32_t sb = smem_addr(sm);
+    uint8_t *misc = sm + OFF_MISC;
+    float *Mr = reinterpret_cast<float *>(misc + M_MR);
+    float *Dm = reinterpret_cast<float *>(misc + M_DM);
+    float *rqv = reinterpret_cast<float *>(misc + M_RQ);
+    float *lamv = reinterpret_cast<float *>(misc + M_LAM);
+    float *itauv = reinterpret_cast<float *>(misc + M_ITAU);
+    float *mqv = reinterpret_cast<float *>(misc + M_MQ);
+    float *c1v = reinterpret_cast<float *>(misc + M_C1);
+    float *mdzv = reinterpret_cast<float *>(misc + M_MDZ);
+    float *czv = reinterpret_cast<float *>(misc + M_CZ);
+    float *rkv = reinterpret_cast<float *>(misc + M_RK);
+    float *gp = reinterpret_cast<float *>(misc + M_GP);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
+    const bool gate_f32 = a.gate_dtype != 0;
+    const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
+    const int64_t tseq0 = a.t0 ? a.t0[b] : 0;
+    const uint8_t *ck = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T);
+    int *status = a.status;
+
+    if (tid == 0) {
+        for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+        tma_prefetch_desc(&map_do);
+        tma_prefetch_desc(&map_g);
+    }
+    if (warp == 0) tmem_alloc(tmem_slot, 512);
+    for (int e = tid; e < 8192 / 16; e += kThreads)
+        reinterpret_cast<uint4 *>(sm + OFF_BC)[e] = make_uint4(0u, 0u, 0u, 0u);
+    Dm[tid] = a.dmT ? a.dmT[static_cast<size_t>(bh) * kD + tid] : 0.f;
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tmem_slot;
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
+    {
+        // DC <- dC_T (row a = tid)
+        const float *src = a.dCT ? a.dCT + (static_cast<size_t>(bh) * kD + tid) * kD : nullptr;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[32];
+#pragma unroll
+            for (int e = 0; e < 32; ++e) x[e] = src ? src[32 * c + e] : 0.f;
+            tmem_st32(tq + TM_DC + 32 * c, x);
+        }
+        tmem_wait_st();
+    }
+    auto issue = [&](int r) {
+        const int tg = r * kC;
+        uint64_t *bb = &bar[BAR_IN];
+        mbar_arrive_expect_tx(bb, 4 * 16384 + g_bytes + 65536 + 512);
+        tma_load_4d(sm + OFF_Q, &map_q, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_Q + 8192, &map_q, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, tg, b);
+        const uint8_t *rec = ck + static_cast<size_t>(r) * kCkptChunkBytes;
+        bulk_load(sm + OFF_SK, rec, 65536, bb);
+        bulk_load(misc + M_MR, rec + 65536, 512, bb);
+    };
+    if (tid == 0 && NC > 0) issue(NC - 1);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    const int i = 16 * warp + (lane & 15);  // chunk row of this thread in the M = 64 products
+    const int hf = lane >> 4;               // column half
+    // descriptors (K-major: advance 32 B per K16 slice, 8 KB / 16 KB per 64-wide K block;
+    // MN-major: advance 2 KB per 16 K rows)
+    const uint64_t dQ = make_desc(sb + OFF_Q, 16, 1024), dQm = make_desc(sb + OFF_Q, 8192, 1024);
+    const uint64_t dK = make_desc(sb + OFF_K, 16, 1024), dKm = make_desc(sb + OFF_K, 8192, 1024);
+    const uint64_t dV = make_desc(sb + OFF_V, 16, 1024);
+    const uint64_t dDO = make_desc(sb + OFF_DO, 16, 1024), dDOm = make_desc(sb + OFF_DO, 8192, 1024);
+    const uint64_t dKDm = make_desc(sb + OFF_KD, 8192, 1024);
+    const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024), dSX = make_desc(sb + OFF_SX, 16, 1024);
+    const uint64_t dDC = make_desc(sb + OFF_DC, 16, 1024), dDCm = make_desc(sb + OFF_DC, 16384, 1024);
+    const uint64_t dW2 = make_desc(sb + OFF_W2, 16, 1024), dW2m = make_desc(sb + OFF_W2, 8192, 1024);
+    const uint64_t dP1 = make_desc(sb + OFF_P1, 16, 1024), dP1m = make_desc(sb + OFF_P1, 8192, 1024);
+    const uint64_t dBC = make_desc(sb + OFF_BC, 16, 1024);
+
+    for (int it = 0; it < NC; ++it) {
+        const int r = NC - 1 - it;
+        const uint32_t par = it & 1;
+        const int c0 = r * kC;
+        mbar_wait(&bar[BAR_IN], par, abort_flag, status);
+        if (tid < kC) {
+            const int n = c0 + tid;
+            lamv[tid] = n < T ? a.lambda[(static_cast<size_t>(b) * T + n) * H + h] : 0.f;
+            itauv[tid] = 1.f / static_cast<float>(tseq0 + n + 1);
+        }
+        prep_chunk(sm + OFF_Q, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, Mr, rqv, mqv, rkv,
+                   gp, nullptr, nullptr, tid);
+        {
+            // DC_{r+1} -> bf16 operand tile (row a = tid)
+            tc_fence_after();
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                tmem_ld32(tq + TM_DC + 32 * c, x);
+                uint8_t *tile = sm + OFF_DC + (c >> 1) * 16384;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tc_fence_after();
+            for (int k = 0; k < 8; ++k) {  // Sc = Qbar Kbar^T, T1 = dO V^T
+                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                mma_bf16(tbase + TM_SC, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {
+                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                mma_bf16(tbase + TM_T1, dDO + ko, dV + ko, ID_64x64_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {  // Zi = Qbar S^K, Dq = dO Sx^T
+                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+                mma_bf16(tbase + TM_Z, dQ + ka, dSK + kb, ID_64x128_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {
+                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+                mma_bf16(tbase + TM_DQ, dDO + ka, dSX + kb, ID_64x128_KK, k != 0);
+            }
+            mma_commit(&bar[BAR_R1]);
+        }
+        // ---- E1: c1, W2, P1
+        mbar_wait(&bar[BAR_R1], par, abort_flag, status);
+        tc_fence_after();
+        {
+            float sc[32];
+            tmem_ld16x2_32<32>(tq + TM_SC, sc);
+            const float part = masked_sum(i, hf, sc);
+            const float c1 = a.centered ? (mqv[i] + part) * itauv[i] : 0.f;
+            if (hf == 0) {
+                c1v[i] = c1;
+                *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-c1);
+            }
+            masked_row(sm + OFF_W2, i, hf, sc, c1);
+            float t1[32];
+            tmem_ld16x2_32<32>(tq + TM_T1, t1);
+            masked_row(sm + OFF_P1, i, hf, t1, 0.f);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tc_fence_after();
+            for (int k = 0; k < 4; ++k)  // Zi += W2 Kbar, Dq += P1 Kd
+                mma_bf16(tbase + TM_Z, dW2 + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+            for (int k = 0; k < 4; ++k)
+                mma_bf16(tbase + TM_DQ, dP1 + k * 2, dKDm + k * 128, ID_64x128_KM, 1);
+            mma_commit(&bar[BAR_R2]);
+        }
+        // ---- E2: z, q_clean, dqc, dlambda; tiles QG, DZ, dqc, qc*dqc
+        mbar_wait(&bar[BAR_R2], par, abort_flag, status);
+        tc_fence_after();
+        {
+            const float lam = lamv[i], itau = itauv[i], c1 = c1v[i];
+            const float nl = -lam * itau;
+            const float *Mh = Mr + 64 * hf;
+            const uint8_t *qbt = sm + OFF_Q + hf * 8192;
+            const uint8_t *egt = sm + OFF_EG + hf * 8192;
+            float dl = 0.f, mdz = 0.f;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                float zi[32], dqa[32];
+                tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, zi);
+                tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, dqa);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const int cc = 4 * h2 + q4;
+                    float qb[8], eg[8], qg[8], dz[8], dqv[8], gq[8];
+                    load_row_chunk(qbt, i, cc, qb);
+                    load_row_chunk(egt, i, cc, eg);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float m = Mh[8 * cc + e];
+                        const float z = (zi[8 * q4 + e] - c1 * m) * itau;
+                        const float qc = qb[e] - lam * z;
+                        const float dqc = a.scale * eg[e] * dqa[8 * q4 + e];
+                        const float d = nl * dqc;
+                        dl = fmaf(-z, dqc, dl);
+                        mdz = fmaf(m, d, mdz);
+                        qg[e] = a.scale * qc * eg[e];
+                        dz[e] = d;
+                        dqv[e] = dqc;
+                        gq[e] = qc * dqc;
+                    }
+                    store_row_chunk(sm + OFF_V + hf * 8192, i, cc, qg);
+                    store_row_chunk(sm + OFF_DO + hf * 8192, i, cc, dz);
+                    store_row_chunk(sm + OFF_SX + hf * 8192, i, cc, dqv);
+                    store_row_chunk(sm + OFF_SX + 16384 + hf * 8192, i, cc, gq);
+                }
+            }
+            dl += __shfl_xor_sync(0xffffffffu, dl, 16);
+            mdz += __shfl_xor_sync(0xffffffffu, mdz, 16);
+            if (hf == 0) {
+                mdzv[i] = mdz;
+                const int n = c0 + i;
+                if (n < T && a.dlambda) a.dlambda[(static_cast<size_t>(b) * T + n) * H + h] = dl;
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tma_store_4d(&map_qg, sm + OFF_V, 0, h, c0, b);
+            tma_store_4d(&map_qg, sm + OFF_V + 8192, 64, h, c0, b);
+            tma_store_4d(&map_gq, sm + OFF_SX + 16384, 0, h, c0, b);
+            tma_store_4d(&map_gq, sm + OFF_SX + 16384 + 8192, 64, h, c0, b);
+            tma_store_commit();
+            tc_fence_after();
+            for (int k = 0; k < 8; ++k) {  // T3 = DZ Kbar^T
+                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                mma_bf16(tbase + TM_SC, dDO + ko, dK + ko, ID_64x64_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {  // u = DZ S^K
+                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+                mma_bf16(tbase + TM_Z, dDO + ka, dSK + kb, ID_64x128_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {  // dkc = Kbar DC + Kbar DC^T
+                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+                mma_bf16(tbase + TM_DQ, dK + ka, dDCm + k * 128, ID_64x128_KM, k != 0);
+                mma_bf16(tbase + TM_DQ, dK + ka, dDC + kb, ID_64x128_KK, 1);
+            }
+            for (int k = 0; k < 4; ++k)  // dkc += W2^T DZ
+                mma_bf16(tbase + TM_DQ, dW2m + k * 128, dDOm + k * 128, ID_64x128_MM, 1);
+            for (int k = 0; k < 4; ++k)  // DC += DZ^T Qbar
+                mma_bf16(tbase + TM_DC, dDOm + k * 128, dQm + k * 128, ID_128x128_MM, 1);
+            for (int k = 0; k < 4; ++k)  // Dm increment, first half: DZ^T (-c1)
+                mma_bf16(tbase + TM_T1, dDOm + k * 128, dBC + k * 2, ID_128x64_MK, k != 0);
+            mma_commit(&bar[BAR_R3]);
+        }
+        // ---- E3: cz, W3
+        mbar_wait(&bar[BAR_R3], par, abort_flag, status);
+        tc_fence_after();
+        {
+            float t3[32];
+            tmem_ld16x2_32<32>(tq + TM_SC, t3);
+            const float part = masked_sum(i, hf, t3);
+            const float cz = a.centered ? (mdzv[i] + part) * itauv[i] : 0.f;
+            if (hf == 0) {
+                czv[i] = cz;
+                *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-cz);
+            }
+            masked_row(sm + OFF_P1, i, hf, t3, cz);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tc_fence_after();
+            for (int k = 0; k < 4; ++k)  // u += W3 Kbar
+                mma_bf16(tbase + TM_Z, dP1 + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+            for (int k = 0; k < 4; ++k)  // dkc += W3^T Qbar
+                mma_bf16(tbase + TM_DQ, dP1m + k * 128, dQm + k * 128, ID_64x128_MM, 1);
+            for (int k = 0; k < 4; ++k)  // Dm increment, second half: Qbar^T (-cz)
+                mma_bf16(tbase + TM_T1, dQm + k * 128, dBC + k * 2, ID_128x64_MK, 1);
+            mma_commit(&bar[BAR_R4]);
+        }
+        // ---- E4: dq, the CCQ part of dkbar, Dm
+        mbar_wait(&bar[BAR_R4], par, abort_flag, status);
+        tc_fence_after();
+        float dm_inc;
+        {
+            float x[32];
+            tmem_ld32(tq + TM_T1, x);  // lane tid, column 0
+            dm_inc = x[0];
+        }
+        {
+            const float cz = czv[i], rq = rqv[i];
+            const float *Mh = Mr + 64 * hf;
+            uint8_t *qbt = sm + OFF_Q + hf * 8192;
+            const uint8_t *dqt = sm + OFF_SX + hf * 8192;
+            float dqb[64];
+            float dot = 0.f;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                float u[32];
+                tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, u);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const int cc = 4 * h2 + q4;
+                    float dqc[8], qb[8];
+                    load_row_chunk(dqt, i, cc, dqc);
+                    load_row_chunk(qbt, i, cc, qb);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float v = dqc[e] + u[8 * q4 + e] - cz * Mh[8 * cc + e];
+                        dqb[8 * cc + e] = v;
+                        dot = fmaf(qb[e], v, dot);
+                    }
+                }
+            }
+            dot += __shfl_xor_sync(0xffffffffu, dot, 16);
+#pragma unroll
+            for (int cc = 0; cc < 8; ++cc) {
+                float qb[8], out[8];
+                load_row_chunk(qbt, i, cc, qb);
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    out[e] = a.l2norm ? rq * fmaf(-qb[e], dot, dqb[8 * cc + e]) : dqb[8 * cc + e];
+                store_row_chunk(qbt, i, cc, out);
+            }
+        }
+        {
+            const float *Dh = Dm + 64 * hf;
+            uint8_t *kt = sm + OFF_K + hf * 8192;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                float x[32];
+                tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, x);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const int cc = 4 * h2 + q4;
+                    float out[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) out[e] = x[8 * q4 + e] + Dh[8 * cc + e];
+                    store_row_chunk(kt, i, cc, out);
+                }
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        Dm[tid] += dm_inc;  // Dm_r, read again only after the next chunk's barriers
+        if (tid == 0 && !*abort_flag) {
+            tma_store_4d(&map_dq, sm + OFF_Q, 0, h, c0, b);
+            tma_store_4d(&map_dq, sm + OFF_Q + 8192, 64, h, c0, b);
+            tma_store_4d(&map_dkc, sm + OFF_K, 0, h, c0, b);
+            tma_store_4d(&map_dkc, sm + OFF_K + 8192, 64, h, c0, b);
+            tma_store_commit();
+            if (it + 1 < NC) {
+                tma_store_wait_read();  // staged tiles read before the next chunk lands on them
+                issue(r - 1);
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (a.dC0) {
+        float *dst = a.dC0 + (static_cast<size_t>(bh) * kD + tid) * kD;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[32];
+            tmem_ld32(tq + TM_DC + 32 * c, x);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                reinterpret_cast<float4 *>(dst + 32 * c)[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+        }
+    }
+    if (a.dm0) a.dm0[static_cast<size_t>(bh) * kD + tid] = Dm[tid];
+    if (tid == 0) tma_store_wait_all();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tbase, 512);
+    }
+}
+
+// =====================================================================================
+// gla_bwd_kv_kernel
+// =====================================================================================
+namespace kv {
+constexpr uint32_t OFF_K = 0;        // kbar; then dk (staged)
+constexpr uint32_t OFF_V = 16384;    // v; then dv (staged)
+constexpr uint32_t OFF_DO = 32768;   // do
+constexpr uint32_t OFF_KD = 49152;   // raw gates (fp32: KD + EG); then Kd
+constexpr uint32_t OFF_EG = 65536;   // EG
+constexpr uint32_t OFF_QG = 81920;   // QG      (scratch from gla_bwd_q_kernel)
+constexpr uint32_t OFF_DKC = 98304;  // CCQ part of dkbar (scratch)
+constexpr uint32_t OFF_GQ = 114688;  // qc * dqc (scratch)
+constexpr uint32_t OFF_DS = 131072;  // bf16 dSs = Diag(e^{Gc-Gmid}) dS_{r+1}
+constexpr uint32_t OFF_P1 = 163840;  // P1
+constexpr uint32_t OFF_SA = 172032;  // SA
+constexpr uint32_t OFF_DG = 131072;  // fp32 dG [64][kDgStride], over dSs and P1 once both are dead
+constexpr int kDgStride = 129;
+constexpr uint32_t OFF_SXC = 180224; // Sx_r = e^{Gmid} S_r (checkpoint tile, for the gate carry)
+constexpr uint32_t OFF_MISC = 214016;
+constexpr uint32_t M_RK = 0, M_F = 256, M_EM = 768, M_EMP = 1280, M_CARRY = 1792, M_GP = 2304,
+                   M_CNEXT = 2816, M_BAR = 3328, M_TMEM = 3360, M_ABORT = 3364;
+constexpr uint32_t kMisc = 3456;
+constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
+static_assert(OFF_DG + 64 * kDgStride * 4 <= OFF_SA, "dG scratch reaches SA");
+static_assert(OFF_SXC + 32768 <= OFF_MISC, "Sx tile overlaps misc");
+static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
+enum { BAR_IN = 0, BAR_R1, BAR_R2, kBars };
+constexpr uint32_t TM_X = 0, TM_T1 = 128, TM_SA = 192, TM_DK = 256, TM_DV = 384;
+}  // namespace kv
+
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
+                  const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
+                  const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
+                  const __grid_constant__ CUtensorMap map_gq, const __grid_constant__ CUtensorMap map_dk,
+                  const __grid_constant__ CUtensorMap map_dv, const BwdArgs a) {
+    using namespace kv;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    const uint32_t sb = smem_addr(sm);
+    uint8_t *misc = sm + OFF_MISC;
+    float *rkv = reinterpret_cast<float *>(misc + M_RK);
+    float *fv = reinterpret_cast<float *>(misc + M_F);
+    float *emv = reinterpret_cast<float *>(misc + M_EM);
+    float *emp = reinterpret_cast<float *>(misc + M_EMP);
+    float *carry = reinterpret_cast<float *>(misc + M_CARRY);
+    float *cnext = reinterpret_cast<float *>(misc + M_CNEXT);
+    float *gp = reinterpret_cast<float *>(misc + M_GP);
+    float *dG = reinterpret_cast<float *>(sm + OFF_DG);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
+    const bool gate_f32 = a.gate_dtype != 0;
+    const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
+    const uint8_t *ck = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T);
+    int *status = a.status;
+
+    if (tid == 0) {
+        for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+        tma_prefetch_desc(&map_do);
+        tma_prefetch_desc(&map_g);
+        tma_prefetch_desc(&map_qg);
+        tma_prefetch_desc(&map_dkc);
+        tma_prefetch_desc(&map_gq);
+    }
+    if (warp == 0) tmem_alloc(tmem_slot, 512);
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tmem_slot;
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
+    {
+        // X <- dS_T; the gate-gradient carry starts at rowsum(dS_T * S_T)
+        const float *dst_row = a.dST ? a.dST + (static_cast<size_t>(bh) * kD + tid) * kD : nullptr;
+        const float *st_row = reinterpret_cast<const float *>(ck + static_cast<size_t>(NC) * kCkptChunkBytes) + tid * kD;
+        float cs = 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[32];
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+                x[e] = dst_row ? dst_row[32 * c + e] : 0.f;
+                if (dst_row) cs = fmaf(x[e], st_row[32 * c + e], cs);
+            }
+            tmem_st32(tq + TM_X + 32 * c, x);
+        }
+        tmem_wait_st();
+        carry[tid] = cs;
+        emp[tid] = 1.f;
+    }
+    auto issue = [&](int r) {
+        const int tg = r * kC;
+        uint64_t *bb = &bar[BAR_IN];
+        mbar_arrive_expect_tx(bb, 6 * 16384 + g_bytes + 32768);
+        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_QG, &map_qg, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_QG + 8192, &map_qg, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_DKC, &map_dkc, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_DKC + 8192, &map_dkc, bb, 64, h, tg, b);
+        tma_load_4d(sm + OFF_GQ, &map_gq, bb, 0, h, tg, b);
+        tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, tg, b);
+        bulk_load(sm + OFF_SXC, ck + static_cast<size_t>(r) * kCkptChunkBytes + 32768, 32768, bb);
+    };
+    if (tid == 0 && NC > 0) issue(NC - 1);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    const int i = 16 * warp + (lane & 15), hf = lane >> 4;
+    const uint64_t dV = make_desc(sb + OFF_V, 16, 1024);
+    const uint64_t dDO = make_desc(sb + OFF_DO, 16, 1024), dDOm = make_desc(sb + OFF_DO, 8192, 1024);
+    const uint64_t dKD = make_desc(sb + OFF_KD, 16, 1024);
+    const uint64_t dQG = make_desc(sb + OFF_QG, 16, 1024), dQGm = make_desc(sb + OFF_QG, 8192, 1024);
+    const uint64_t dDS = make_desc(sb + OFF_DS, 16, 1024), dDSm = make_desc(sb + OFF_DS, 16384, 1024);
+    const uint64_t dP1m = make_desc(sb + OFF_P1, 8192, 1024);
+    const uint64_t dSA = make_desc(sb + OFF_SA, 16, 1024);
+
+    for (int it = 0; it < NC; ++it) {
+        const int r = NC - 1 - it;
+        const uint32_t par = it & 1;
+        const int c0 = r * kC;
+        mbar_wait(&bar[BAR_IN], par, abort_flag, status);
+        prep_chunk(nullptr, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, nullptr, nullptr, nullptr,
+                   rkv, gp, fv, emv, tid);
+        {
+            // dSs = Diag(e^{Gc - Gmid}) dS_{r+1}: X holds e^{-Gmid_{r+1}} dS_{r+1}
+            tc_fence_after();
+            const float hs = fv[tid] * emp[tid];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                tmem_ld32(tq + TM_X + 32 * c, x);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) x[e] *= hs;
+                uint8_t *tile = sm + OFF_DS + (c >> 1) * 16384;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
+                tmem_st32(tq + TM_X + 32 * c, x);
+            }
+            emp[tid] = emv[tid];
+            tmem_wait_st();
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tc_fence_after();
+            for (int k = 0; k < 8; ++k) {  // T1 = dO V^T, SA = Kd QG^T
+                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                mma_bf16(tbase + TM_T1, dDO + ko, dV + ko, ID_64x64_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {
+                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                mma_bf16(tbase + TM_SA, dKD + ko, dQG + ko, ID_64x64_KK, k != 0);
+            }
+            for (int k = 0; k < 8; ++k) {  // dkw = V dSs^T, dv = Kd dSs
+                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+                mma_bf16(tbase + TM_DK, dV + ka, dDS + kb, ID_64x128_KK, k != 0);
+                mma_bf16(tbase + TM_DV, dKD + ka, dDSm + k * 128, ID_64x128_KM, k != 0);
+            }
+            for (int k = 0; k < 4; ++k)  // X += QG^T dO
+                mma_bf16(tbase + TM_X, dQGm + k * 128, dDOm + k * 128, ID_128x128_MM, 1);
+            mma_commit(&bar[BAR_R1]);
+        }
+        mbar_wait(&bar[BAR_R1], par, abort_flag, status);
+        tc_fence_after();
+        {
+            // gate carry of the chunk before: rowsum(dS_r * S_r) = rowsum(X * Sx_r) (the
+            // e^{-Gmid} of X and the e^{Gmid} of Sx cancel); a boundary value, so rounding
+            // does not accumulate across chunks
+            float cs = 0.f;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float x[32];
+                tmem_ld32(tq + TM_X + 32 * c, x);
+                const uint8_t *tile = sm + OFF_SXC + (c >> 1) * 16384;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    float sx[8];
+                    load_row_chunk(tile, tid, 4 * (c & 1) + q4, sx);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) cs = fmaf(x[8 * q4 + e], sx[e], cs);
+                }
+            }
+            cnext[tid] = cs;
+        }
+        {
+            float t1[32];
+            tmem_ld16x2_32<32>(tq + TM_T1, t1);
+            masked_row(sm + OFF_P1, i, hf, t1, 0.f);  // P1[t][j] = [j <= t] do_t . v_j
+            float sa[32];
+            tmem_ld16x2_32<32>(tq + TM_SA, sa);
+            // SA[j][t] = [t >= j] Kd_j . QG_t (row i is key j)
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                float w[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const int t = 32 * hf + 8 * q4 + e;
+                    w[e] = (t >= i) ? sa[8 * q4 + e] : 0.f;
+                }
+                store_row_chunk(sm + OFF_SA, i, 4 * hf + q4, w);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tc_fence_after();
+            for (int k = 0; k < 4; ++k)  // dkw += P1^T QG, dv += SA dO
+                mma_bf16(tbase + TM_DK, dP1m + k * 128, dQGm + k * 128, ID_64x128_MM, 1);
+            for (int k = 0; k < 4; ++k)
+                mma_bf16(tbase + TM_DV, dSA + k * 2, dDOm + k * 128, ID_64x128_KM, 1);
+            mma_commit(&bar[BAR_R2]);
+        }
+        mbar_wait(&bar[BAR_R2], par, abort_flag, status);
+        tc_fence_after();
+        {
+            // dk: dkbar = e^{Gmid-G} dkw + (CCQ part); normalisation backward; dG
+            const float rk = rkv[i];
+            uint8_t *kt = sm + OFF_K + hf * 8192;
+            const uint8_t *egt = sm + OFF_EG + hf * 8192;
+            const uint8_t *dkct = sm + OFF_DKC + hf * 8192;
+            const uint8_t *gqt = sm + OFF_GQ + hf * 8192;
+            float *dgrow = dG + i * kDgStride + 64 * hf;
+            float dkb[64];
+            float dot = 0.f;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                float x[32];
+                tmem_ld16x2_32<64>(tq + TM_DK + 32 * h2, x);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const int cc = 4 * h2 + q4;
+                    float eg[8], kb[8], kc[8], gq[8];
+                    load_row_chunk(egt, i, cc, eg);
+                    load_row_chunk(kt, i, cc, kb);
+                    load_row_chunk(dkct, i, cc, kc);
+                    load_row_chunk(gqt, i, cc, gq);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float dkw = x[8 * q4 + e] * __frcp_rn(eg[e]);
+                        const float v = dkw + kc[e];
+                        dkb[8 * cc + e] = v;
+                        dot = fmaf(kb[e], v, dot);
+                        dgrow[8 * cc + e] = fmaf(-kb[e], dkw, gq[e]);
+                    }
+                }
+            }
+            dot += __shfl_xor_sync(0xffffffffu, dot, 16);
+#pragma unroll
+            for (int cc = 0; cc < 8; ++cc) {
+                float kb[8], out[8];
+                load_row_chunk(kt, i, cc, kb);
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    out[e] = a.l2norm ? rk * fmaf(-kb[e], dot, dkb[8 * cc + e]) : dkb[8 * cc + e];
+                store_row_chunk(kt, i, cc, out);
+            }
+            uint8_t *vt = sm + OFF_V + hf * 8192;
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                float x[32];
+                tmem_ld16x2_32<64>(tq + TM_DV + 32 * h2, x);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(vt, i, 4 * h2 + q4, x + 8 * q4);
+            }
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0 && !*abort_flag) {
+            tma_store_4d(&map_dk, sm + OFF_K, 0, h, c0, b);
+            tma_store_4d(&map_dk, sm + OFF_K + 8192, 64, h, c0, b);
+            tma_store_4d(&map_dv, sm + OFF_V, 0, h, c0, b);
+            tma_store_4d(&map_dv, sm + OFF_V + 8192, 64, h, c0, b);
+            tma_store_commit();
+        }
+        {
+            // dgk_t = sum_{s >= t in the chunk} dG_s + rowsum(dS_{r+1} * S_{r+1}),
+            // column d = tid, tokens in reverse
+            float acc = carry[tid];
+            const int nvalid = min(kC, T - c0);
+            for (int t = kC - 1; t >= 0; --t) {
+                acc += dG[t * kDgStride + tid];
+                if (t < nvalid) {
+                    const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + tid;
+                    if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
+                    else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
+                }
+            }
+            carry[tid] = cnext[tid];
+        }
+        __syncthreads();
+        if (tid == 0 && !*abort_flag && it + 1 < NC) {
+            tma_store_wait_read();
+            issue(r - 1);
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (a.dS0) {
+        // dS_0 = e^{Gmid_0} X
+        const float em = emp[tid];
+        float *dst = a.dS0 + (static_cast<size_t>(bh) * kD + tid) * kD;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[32];
+            tmem_ld32(tq + TM_X + 32 * c, x);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                reinterpret_cast<float4 *>(dst + 32 * c)[e] =
+                    make_float4(em * x[4 * e], em * x[4 * e + 1], em * x[4 * e + 2], em * x[4 * e + 3]);
+        }
+    }
+    if (tid == 0) tma_store_wait_all();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tbase, 512);
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
+        cudaError_t e = cudaFuncSetAttribute(gla_bwd_q_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(qk::kSmem));
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(gla_bwd_kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kv::kSmem));
+        if (e != cudaSuccess) return e;
+        attr_set = true;
+    }
+    const int grid = a.B * a.H;
+    gla_bwd_q_kernel<<<grid, kThreads, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq, a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    gla_bwd_kv_kernel<<<grid, kThreads, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
+    return cudaGetLastError();
+}
+
+}  // namespace ccq

@@ -44,6 +44,9 @@
 // reloaded as soon as the chunk's last product that reads it completes.
 // Rows past T load as zeros: zero keys add nothing to any sum, zero gates keep
 // the cumulative gate, so the ragged tail needs no special arithmetic.
+// With a.ckpt set, WG2 also copies each chunk's two state tiles and key sum to
+// the checkpoint buffer (one bulk copy per chunk) and the last segment writes
+// S_T there; the backward (ccq_gla_bwd.cu) reads them.
 // With a.nseg > 1 every CTA walks one segment (a range of whole chunks) of one
 // sequence, starting from the segment's initial states in a.seg_ws
 // (ccq_gla_segment.cu); only the last segment writes the final states.
@@ -94,6 +97,7 @@ constexpr uint32_t M_ABORT = 7532;
 constexpr uint32_t kMiscBytes = 7680;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;  // + alignment slack
 static_assert(kSmemBytes <= 232448, "exceeds the 227 KB per-CTA limit");
+static_assert(OFF_S == OFF_SK + 32768, "a checkpoint copies the S^K and S tiles as one block");
 
 enum {
     BAR_IN0 = 0, BAR_IN1 = 1, BAR_V = 2, BAR_GA = 3, BAR_GB = 4, BAR_GC = 5, BAR_GD = 6,
@@ -399,6 +403,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             if (tid == 0 && r + 1 < NC && !*abort_flag) issue_v(r + 1);  // v no longer read
+            if (a.skip_o) continue;  // checkpoint-only pass: no output
             {
                 // stage o (bf16, swizzled) in the chunk's Q tile, then one TMA store;
                 // rows past T fall outside the tensor and are not written
@@ -551,11 +556,17 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     } else {
         // =============================================================== WG2: states
         const int row = 32 * (warp & 3) + lane;  // state row a (key dim)
+        uint8_t *ck_head = a.ckpt ? a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T) : nullptr;
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1;
             if (r > 0) mbar_wait(&bar[BAR_GS], (r - 1) & 1, abort_flag, status);
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
+            if (ck_head && r > 0) {
+                // the previous checkpoint copy must have read the tiles before they change
+                if (wt == 0) tma_store_wait_read();
+                named_bar(3, 128);
+            }
             tc_fence_after();
             const float hs = (r > 0 ? slot_f(s ^ 1, MS_F)[row] : 1.f) * slot_f(s, MS_EGM)[row];
 #pragma unroll
@@ -581,8 +592,18 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar(3, 128);
+            if (ck_head) {
+                // checkpoint of chunk cb + r: the S^K and e^{Gmid} S tiles, then M_r
+                uint8_t *rec = ck_head + static_cast<size_t>(cb + r) * kCkptChunkBytes;
+                reinterpret_cast<float *>(rec + 65536)[row] = slot_f(s, MS_MST)[row];
+                if (wt == 0) {
+                    bulk_store(rec, sm + OFF_SK, 65536);
+                    tma_store_commit();
+                }
+            }
             if (wt == 0) mbar_arrive(&bar[BAR_SNAP]);
         }
+        if (ck_head && wt == 0) tma_store_wait_all();
         // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K
         if (NC > 0 && last_seg) {
             mbar_wait(&bar[BAR_GS], (NC - 1) & 1, abort_flag, status);
@@ -595,6 +616,14 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 tmem_ld32(tq + TM_S + 32 * c, x);
                 if (a.ST) {
                     float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],
+                                             fs * x[4 * e + 3]);
+                }
+                if (ck_head) {
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        ck_head + static_cast<size_t>(NCt) * kCkptChunkBytes + (static_cast<size_t>(row) * kD + 32 * c) * 4);
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
                         dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],

@@ -47,10 +47,25 @@ struct ChunkArgs {
     int nseg = 1;
     int seg_chunks = 0;
     float *seg_ws = nullptr;
+    // GLA only: when set, the chunk-start states of every chunk are saved for the
+    // backward (layout below); skip_o suppresses the output write.
+    uint8_t *ckpt = nullptr;
+    int skip_o = 0;
 };
 
 // Per (sequence, segment) workspace: S [128][128], C [128][128], m [128], D [128].
 constexpr int kSegFloats = 2 * 128 * 128 + 2 * 128;
+
+// GLA checkpoints, per (sequence, head): one record per chunk r, then the final
+// state.  A chunk record is the byte image of the forward kernel's bf16 operand
+// tiles -- S^K_r ([128][128] as two T64 tiles) then e^{Gmid_r} S_r (same) --
+// followed by the key sum M_r (128 fp32).  The final record is S_T (fp32
+// [128][128], row-major, key dim first).
+constexpr size_t kCkptChunkBytes = 65536 + 512;
+constexpr size_t kCkptFinalBytes = 65536;
+__host__ __device__ inline size_t ckpt_head_bytes(int T) {
+    return static_cast<size_t>((T + 63) / 64) * kCkptChunkBytes + kCkptFinalBytes;
+}
 
 
 // Device address of the library's status word on the current device.
@@ -84,6 +99,33 @@ cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
 
 // Workspace bytes of the chunkwise Gated DeltaNet path (Ut and W of every chunk).
 size_t gdn_workspace_bytes(int B, int T, int H);
+
+// Arguments of the chunkwise CCQ-GLA backward (ccq_gla_bwd.cu).  ckpt holds
+// the forward checkpoints (layout above); dgk is written in the gate dtype.
+struct BwdArgs {
+    int B, T, H;
+    int gate_dtype;
+    int l2norm, centered;
+    float scale;
+    const float *lambda;
+    const int64_t *t0;
+    const uint8_t *ckpt;
+    const float *dST, *dCT, *dmT;
+    float *dlambda;
+    void *dgk;
+    float *dS0, *dC0, *dm0;
+    int *status;
+};
+
+// Tensor maps ([B][T][H][128], 64 x 64 swizzled boxes; g as in ChunkMaps) of
+// the inputs, the outputs dq, dk, dv and the three bf16 scratch tensors the
+// two backward kernels exchange (QG, the CCQ part of dkbar, qc * dqc).
+struct BwdMaps {
+    CUtensorMap q, k, v, dO, g, dq, dk, dv, qg, dkc, gq;
+};
+
+// Launches gla_bwd_q_kernel then gla_bwd_kv_kernel (one CTA per sequence and head).
+cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s);
 
 // Encode the tensor map of a row-major [rows][128] bf16 matrix with 64 x 64 boxes
 // (128-byte swizzle).

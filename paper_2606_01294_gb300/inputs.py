@@ -121,7 +121,32 @@ def make_decode_inputs(backbone: int, B: int, H: int, Dk: int, Dv: int, *,
     return {"prefix": pre, "token": tok}
 
 
-# The five workload shapes (name -> keyword arguments), one per benchmark line
+def make_backward_inputs(B: int, T: int, H: int, Dk: int, Dv: int, *, dtype=torch.bfloat16,
+                         seed: int = 5678, prefix: int = 0, state_grads: bool = True) -> dict:
+    """Draw the extra inputs of a backward problem on the CPU: the output
+    gradient ``dout`` [B,T,H,Dv] (N(0,1) in ``dtype``); final-state gradients
+    ``dST`` [B,H,Dk,Dv], ``dCT`` [B,H,Dk,Dk], ``dmT`` [B,H,Dk] (fp32, N(0,1)
+    scaled by 1/Dk so that each weighs about as much as the output's; None
+    unless ``state_grads``); and, when ``prefix`` > 0, a consistent initial
+    state from a ``prefix``-token history of unit keys (S0 ~ N(0,1)/sqrt(Dk),
+    C0 = sum k k^T, m0 = sum k, t0 = prefix), else None."""
+    gen = torch.Generator().manual_seed(seed)
+    out = {"dout": torch.randn(B, T, H, Dv, generator=gen).to(dtype),
+           "dST": None, "dCT": None, "dmT": None, "state": None}
+    if state_grads:
+        out["dST"] = torch.randn(B, H, Dk, Dv, generator=gen) / Dk
+        out["dCT"] = torch.randn(B, H, Dk, Dk, generator=gen) / Dk
+        out["dmT"] = torch.randn(B, H, Dk, generator=gen) / Dk
+    if prefix > 0:
+        kp = _normalise_rows(torch.randn(B, prefix, H, Dk, generator=gen)).double()
+        out["state"] = {"S": torch.randn(B, H, Dk, Dv, generator=gen).double() / Dk ** 0.5,
+                        "C": torch.einsum("bthd,bthe->bhde", kp, kp),
+                        "m": kp.sum(dim=1),
+                        "t": torch.full((B,), prefix, dtype=torch.int64)}
+    return out
+
+
+# The workload shapes (name -> keyword arguments), one per benchmark line
 # or parity case.  "chunk" is the chunk length of the chunkwise kernels.
 WORKLOADS = {
     "gla_fp32_small": dict(backbone=GLA, B=1, H=2, T=256, Dk=64, Dv=64,
@@ -134,4 +159,6 @@ WORKLOADS = {
                          dtype=torch.bfloat16, seed=1238),
     "gdn_bf16_20k": dict(backbone=GDN, B=1, H=16, T=20480, Dk=128, Dv=128,
                          dtype=torch.bfloat16, seed=1238),
+    "gla_bf16_4k_fwdbwd": dict(backbone=GLA, B=4, H=16, T=4096, Dk=128, Dv=128,
+                               dtype=torch.bfloat16, seed=1239),
 }

@@ -119,3 +119,54 @@ def test_gla_workspace_size_and_split(lib):
     bad = ccq.params()
     bad.seq_split = -1
     assert _gla(lib, p=bad) == ccq.CCQ_ERR_INVALID_ARG
+
+
+def test_gla_ckpt_and_bwd_workspace_sizes(lib):
+    n = ctypes.c_size_t(7)
+    assert lib.ccq_gla_ckpt_size(4, 4096, 16, 128, 128, ctypes.byref(n)) == 0
+    assert n.value == 4 * 16 * (64 * (65536 + 512) + 65536)
+    assert lib.ccq_gla_ckpt_size(1, 65, 1, 128, 128, ctypes.byref(n)) == 0
+    assert n.value == 2 * (65536 + 512) + 65536  # ragged tail: two chunks
+    assert lib.ccq_gla_ckpt_size(1, 64, 1, 64, 64, ctypes.byref(n)) == ccq.CCQ_ERR_UNSUPPORTED
+    p = ctypes.byref(ccq.params(seq_split=1))
+    x = 3 * 4 * 4096 * 16 * 128 * 2
+    assert lib.ccq_gla_bwd_workspace_size(4, 4096, 16, 128, 128, 0, 1, p, ctypes.byref(n)) == 0
+    assert n.value == x
+    assert lib.ccq_gla_bwd_workspace_size(4, 4096, 16, 128, 128, 0, 0, p, ctypes.byref(n)) == 0
+    assert n.value == x + 4 * 16 * (64 * (65536 + 512) + 65536)
+    assert lib.ccq_gla_bwd_workspace_size(1, 64, 1, 128, 128, 1, 1, p, ctypes.byref(n)) == ccq.CCQ_ERR_UNSUPPORTED
+    assert lib.ccq_gla_bwd_workspace_size(1, 0, 1, 128, 128, 0, 0, p, ctypes.byref(n)) == 0
+    assert n.value == 0
+
+
+def _bwd(lib, ptrs=None, sizes=(1, 64, 1, 128, 128), p=None, dtypes=(0, 0), ws=None, ws_bytes=0, ckpt=None):
+    fake = ctypes.c_void_p(0x10000)
+    req = ptrs if ptrs is not None else [fake] * 10  # q k v gk lambda dout dq dk dv dgk
+    return lib.ccq_gla_bwd(*req[:5], *dtypes, *([None] * 4), req[5], None, None, None, ckpt,
+                           *req[6:10], None, None, None, None, *sizes, ws, ws_bytes,
+                           ctypes.byref(p or ccq.params(seq_split=1)), None)
+
+
+def test_gla_bwd_rejects_bad_arguments(lib):
+    fake = ctypes.c_void_p(0x10000)
+    assert _bwd(lib, dtypes=(1, 1)) == ccq.CCQ_ERR_UNSUPPORTED  # fp32 inputs
+    assert _bwd(lib, sizes=(1, 64, 1, 64, 64)) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _bwd(lib, p=ccq.params(algo="recurrent")) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _bwd(lib, ptrs=[fake] * 5 + [None] + [fake] * 4) == ccq.CCQ_ERR_INVALID_ARG  # no dout
+    assert b"NULL" in lib.ccq_last_error()
+    assert _bwd(lib) == ccq.CCQ_ERR_INVALID_ARG and b"workspace" in lib.ccq_last_error()
+    assert _bwd(lib, ws=ctypes.c_void_p(0x10008), ws_bytes=1 << 30, ckpt=fake) == ccq.CCQ_ERR_INVALID_ARG
+    assert b"aligned" in lib.ccq_last_error()
+    # no tokens and no state gradients requested: nothing to do
+    assert _bwd(lib, sizes=(1, 0, 1, 128, 128)) == ccq.CCQ_OK
+
+
+def test_gla_fwd_save_rejects_bad_checkpoint_buffer(lib):
+    fake = ctypes.c_void_p(0x10000)
+    p = ctypes.byref(ccq.params(seq_split=1))
+    st = lib.ccq_gla_fwd_save(*([fake] * 5), 0, 0, *([None] * 4), fake, *([None] * 4), 1, 64, 1, 128, 128,
+                              None, 0, fake, 1024, p, None)
+    assert st == ccq.CCQ_ERR_INVALID_ARG and b"checkpoint" in lib.ccq_last_error()
+    st = lib.ccq_gla_fwd_save(*([fake] * 5), 1, 1, *([None] * 4), fake, *([None] * 4), 1, 64, 1, 128, 128,
+                              None, 0, fake, 1 << 20, p, None)
+    assert st == ccq.CCQ_ERR_UNSUPPORTED  # fp32 inputs have no checkpointing path
