@@ -1,7 +1,9 @@
 """Benchmark of the CCQ hot path on GB300.
 
 One step = one CCQ chunkwise forward over the whole workload batch (one call
-of ccq_gla_fwd / ccq_gdn_fwd, or one ccq_decode_step), inputs resident in HBM.
+of ccq_gla_fwd / ccq_gdn_fwd, or one ccq_decode_step), inputs resident in HBM;
+for the fwd+bwd workload one step is a training step of the layer: the
+forward that saves checkpoints (ccq_gla_fwd_save) then ccq_gla_bwd.
 The default workload is CCQ-GLA forward, bf16, B=8, H=16, T=4096,
 Dk=Dv=128, chunk 64 (the metric's configuration).  Prints ONE JSON line.
 
@@ -28,6 +30,7 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
 METRIC = "CCQ chunked fwd tokens/s at T=4K,d=128 bf16; % of roofline (tensor/HBM)"
+METRIC_FWDBWD = "CCQ-GLA chunked fwd+bwd tokens/s at T=4K,d=128 bf16; % of roofline (HBM)"
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 
@@ -38,10 +41,28 @@ WORKLOADS = {
     "gla_bf16_20k": ("gla", 1, 16, 20480, 128),
     "gdn_bf16_20k": ("gdn", 1, 16, 20480, 128),
     "decode_b256": ("decode", 256, 16, 1, 128),
+    "gla_bf16_4k_fwdbwd": ("glabwd", 4, 16, 4096, 128),
 }
-KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode": "ccq_recurrent.cu"}
+KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode": "ccq_recurrent.cu",
+                  "glabwd": "ccq_gla_bwd.cu"}
 KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_kernel",
-                "decode": "recurrent_kernel"}
+                "decode": "recurrent_kernel",
+                "glabwd": "whole step: forward (saving checkpoints) + gla_bwd_q_kernel + gla_bwd_kv_kernel"}
+
+
+def gla_segments(B, H, T, sms):
+    """Segments per sequence the library's default split picks (ccq_capi.cu)."""
+    nc = (T + 63) // 64
+    ns = sms // (B * H) if B * H * 2 <= sms else 1
+    ns = max(1, min(ns, nc // 8, nc))
+    per = (nc + ns - 1) // ns
+    return (nc + per - 1) // per
+
+
+def launches_per_step(kind, B, H, T, sms):
+    """Kernel launches of one step (the segmented GLA forward is three kernels)."""
+    fwd = 1 if gla_segments(B, H, T, sms) == 1 else 3
+    return {"gla": fwd, "gdn": 2, "decode": 1, "glabwd": fwd + 2}[kind]
 
 
 def algorithmic_bytes(kind, B, H, T, D):
@@ -49,6 +70,13 @@ def algorithmic_bytes(kind, B, H, T, D):
     once, final fp32 states written once (initial states are zero / absent
     except for decode, whose cache is read and written)."""
     tok = B * T * H
+    if kind == "glabwd":
+        # forward: q, k, v, gk, lambda in, o out, final states out; backward:
+        # q, k, v, gk, lambda, dout in, dq, dk, dv, dgk, dlambda and the three
+        # initial-state gradients out (each pass reads its own inputs once)
+        fwd = algorithmic_bytes("gla", B, H, T, D)
+        bwd = tok * D * 2 * 5 + tok * 4 + tok * D * 2 * 4 + tok * 4 + B * H * (2 * D * D + D) * 4
+        return fwd + bwd
     if kind == "gla":
         return tok * D * 2 * 4 + tok * D * 2 + tok * 4 + B * H * (2 * D * D + D) * 4 + B * 8
     if kind == "gdn":
@@ -62,8 +90,16 @@ def algorithmic_flops(kind, B, H, T, D, C=64):
     nc = (T + C - 1) // C
     # GLA: four C x D x D products (Qbar S^K, Qg S, Ku^T V, Kbar^T Kbar) and four
     # C x C x D products (Qbar Kbar^T, W' Kbar, Qg Kg^T, A V), 2 FLOP per MAC.
+    # GLA backward (ccq_gla_bwd.cu), its tcgen05 products per chunk (M x N x K):
+    # q kernel: C x C x D (Sc, T1, T3), C x D x D (Zi, Dq, u, two for dkc),
+    # C x D x C (W2 Kbar, P1 Kd, W2^T DZ, W3 Kbar, W3^T Qbar), D x D x C (DC),
+    # D x C x C twice (Dm); kv kernel: C x C x D (T1, SA), C x D x D (dkw, dv),
+    # D x D x C (dS), C x D x C (P1^T QG, SA dO).
+    bwd = 2 * (3 * C * C * D + 5 * C * D * D + 5 * C * D * C + D * D * C + 2 * D * C * C
+               + 2 * C * C * D + 2 * C * D * D + D * D * C + 2 * C * D * C)
     per_chunk = {"gla": 8 * C * D * D + 8 * C * C * D,
-                 "gdn": 10 * C * D * D + 12 * C * C * D}.get(kind)
+                 "gdn": 10 * C * D * D + 12 * C * C * D,
+                 "glabwd": 8 * C * D * D + 8 * C * C * D + bwd}.get(kind)
     if per_chunk is None:
         return B * H * 8 * D * D
     return B * H * nc * per_chunk
@@ -174,10 +210,14 @@ def cpu_oracle_run(kind, B, H, T, D, sample_b, seed):
                            pre["S"], pre["C"], pre["m"], pre["t"])
         dt = time.perf_counter() - t0
         return sample_b / dt, dt
-    bb = gen.GLA if kind == "gla" else gen.GDN
+    bb = gen.GDN if kind == "gdn" else gen.GLA
     P = gen.make_inputs(bb, sample_b, T, H, D, D, dtype=torch.bfloat16, seed=seed)
+    G = gen.make_backward_inputs(sample_b, T, H, D, D, seed=seed + 1, state_grads=False) \
+        if kind == "glabwd" else None
     t0 = time.perf_counter()
     oracle.forward(bb, P["q"], P["k"], P["v"], P["gate"], P["lam"], beta=P["beta"])
+    if kind == "glabwd":
+        oracle.gla_backward(P["q"], P["k"], P["v"], P["gate"], P["lam"], G["dout"])
     dt = time.perf_counter() - t0
     return sample_b * T / dt, dt
 
@@ -204,7 +244,8 @@ def run_reference(args):
     sample = (f"batch row 0 of {B}, all {H} heads, first {Ts} of {T} tokens, per step"
               if kind != "decode" else f"{sample_b} of {B} batch rows, all {H} heads, one token")
     line = {
-        "impl": "reference", "metric": METRIC, "value": rate, "unit": "tokens/s",
+        "impl": "reference", "metric": METRIC_FWDBWD if kind == "glabwd" else METRIC,
+        "value": rate, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
@@ -254,6 +295,33 @@ def run_gpu(args):
                             out=out)
         tokens_per_step = B
         host = {n: (None if x is None else x.pin_memory()) for n, x in Dd["token"].items()}
+    elif kind == "glabwd":
+        P = gen.make_inputs(gen.GLA, B, T, H, D, D, dtype=torch.bfloat16, seed=seed, lam="trained")
+        P["dout"] = gen.make_backward_inputs(B, T, H, D, D, seed=seed + 1, state_grads=False)["dout"]
+        Dv = {n: (None if x is None else x.to(dev)) for n, x in P.items()}
+        out = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
+        fstate = ccq.CCQState.empty(B, H, D, D, dev)
+        ws = ccq.gla_workspace(B, T, H, D, D, dev)
+        ck = torch.empty(ccq.gla_ckpt_size(B, T, H, D, D), dtype=torch.uint8, device=dev)
+        bws = ccq.gla_bwd_workspace(B, T, H, D, D, dev, with_ckpt=True)
+        grads = {"dq": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dk": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dv": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dgk": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dlambda": torch.empty(B, T, H, device=dev),
+                 "dS0": torch.empty(B, H, D, D, device=dev), "dC0": torch.empty(B, H, D, D, device=dev),
+                 "dm0": torch.empty(B, H, D, device=dev)}
+
+        def train_step(d):
+            ccq.gla_fwd_save(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out, final_state=fstate,
+                             workspace=ws, ckpt=ck)
+            ccq.gla_bwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], d["dout"], ckpt=ck, out=grads,
+                        workspace=bws)
+
+        def step():
+            train_step(Dv)
+        tokens_per_step = B * T
+        host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
     else:
         bb = gen.GLA if kind == "gla" else gen.GDN
         P = gen.make_inputs(bb, B, T, H, D, D, dtype=torch.bfloat16, seed=seed)
@@ -316,6 +384,9 @@ def run_gpu(args):
             res = o.to("cpu", non_blocking=True)
             return res
         d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
+        if kind == "glabwd":
+            train_step(d)
+            return [grads[n].to("cpu", non_blocking=True) for n in ("dq", "dk", "dv", "dgk")]
         if kind == "gla":
             o, st = ccq.gla_fwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out,
                                 final_state=fstate, workspace=ws)
@@ -325,7 +396,7 @@ def run_gpu(args):
         return o.to("cpu", non_blocking=True)
 
     h2d = sum(x.numel() * x.element_size() for x in host.values() if x is not None)
-    d2h = out.numel() * out.element_size()
+    d2h = out.numel() * out.element_size() * (4 if kind == "glabwd" else 1)
     e2e_steps = max(3, min(args.steps, 10))
     e2e_step()
     torch.cuda.synchronize()
@@ -363,19 +434,22 @@ def run_gpu(args):
             import oracle
             oracle.build_oracle()
             # repeat passes over a bounded sample until about 10 s of CPU work
-            sample_b = B if kind != "decode" else 32
+            sample_b = {"decode": 32, "glabwd": 1}.get(kind, B)
+            Tc = min(T, 1024) if kind == "glabwd" else T
             toks, secs, passes = 0.0, 0.0, 0
             while secs < 10.0 and passes < 20:
-                rate, dt = cpu_oracle_run(kind, B, H, T, D, sample_b, seed=seed)
+                rate, dt = cpu_oracle_run(kind, B, H, Tc, D, sample_b, seed=seed)
                 toks += rate * dt
                 secs += dt
                 passes += 1
             cpu = {"value": toks / secs, "unit": "tokens/s", "cores": os.cpu_count(),
                    "kind": "oracle",
-                   "sample": (f"{sample_b} of {B} batch rows, all {H} heads, {T} tokens, "
+                   "sample": (f"{sample_b} of {B} batch rows, all {H} heads, {Tc} of {T} tokens, "
                               f"{passes} passes ({secs:.1f} s)")}
+        sms = torch.cuda.get_device_properties(dev).multi_processor_count
         line = {
-            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "metric": METRIC_FWDBWD if kind == "glabwd" else METRIC, "value": value,
+            "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
@@ -387,7 +461,7 @@ def run_gpu(args):
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
-            "gpu_launches": args.steps,
+            "gpu_launches": args.steps * launches_per_step(kind, B, H, T, sms),
             "clocks": clocks.summary(),
             "kernel_ms_mean": kern_ms,
             "kernel_ms_min": min(launch_ms),
