@@ -105,24 +105,48 @@ def algorithmic_flops(kind, B, H, T, D, C=64):
     return B * H * nc * per_chunk
 
 
-def kernel_sha(kind):
-    p = os.path.join(ROOT, "paper_2606_01294_gb300", "csrc", KERNEL_SOURCES[kind])
+# The kernels of one step of each workload and the source file of each kernel.
+STEP_KERNELS = {
+    "gla_bf16_4k": ["gla_chunk_kernel"],
+    "gdn_bf16_4k": ["gdn_wy_kernel", "gdn_chunk_kernel"],
+    "gla_bf16_20k": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel"],
+    "gdn_bf16_20k": ["gdn_wy_kernel", "gdn_chunk_kernel"],
+    "decode_b256": ["recurrent"],
+    "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
+                           "gla_bwd_q_kernel", "gla_bwd_kv_kernel"],
+}
+KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kernel": "ccq_gla_segment.cu",
+                "gla_segment_combine_kernel": "ccq_gla_segment.cu", "gdn_wy_kernel": "ccq_gdn_chunk.cu",
+                "gdn_chunk_kernel": "ccq_gdn_chunk.cu", "recurrent": "ccq_recurrent.cu",
+                "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu"}
+
+
+def source_sha(fname):
+    p = os.path.join(ROOT, "paper_2606_01294_gb300", "csrc", fname)
     with open(p, "rb") as f:
         return hashlib.sha256(f.read()).hexdigest()[:16]
 
 
+def kernel_sha(kind):
+    return source_sha(KERNEL_SOURCES[kind])
+
+
 def measured_traffic(kind, workload):
-    """dram bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source; else None."""
+    """DRAM bytes of one step (summed over its kernels) from the committed ncu
+    captures, if every kernel of the step was captured on its current source;
+    else None."""
     try:
         with open(TRAFFIC_FILE) as f:
-            t = json.load(f)
-        e = t.get(workload)
-        if e and e.get("kernel_sha") == kernel_sha(kind):
-            return e.get("dram_bytes_per_launch")
-    except (OSError, ValueError):
-        pass
-    return None
+            t = json.load(f).get(workload, {})
+        total = 0
+        for k in STEP_KERNELS[workload]:
+            e = t.get(k)
+            if not e or e.get("source_sha") != source_sha(KERNEL_FILES[k]):
+                return None
+            total += e["dram_bytes_per_launch"]
+        return total
+    except (OSError, ValueError, KeyError):
+        return None
 
 
 class ClockSampler:
@@ -426,7 +450,8 @@ def run_gpu(args):
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / peaks["hbm_gbs"],
                 "traffic": measured_traffic(kind, args.workload),
-                "kernel": KERNEL_NAMES[kind], "algorithmic_bytes": bytes_,
+                "kernel": KERNEL_NAMES[kind] if args.workload != "gla_bf16_20k"
+                else "whole step: gla_segment_state_kernel + gla_segment_combine_kernel + gla_chunk_kernel", "algorithmic_bytes": bytes_,
                 "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
                 "flops": algorithmic_flops(kind, B, H, T, D)}
         cpu = None
