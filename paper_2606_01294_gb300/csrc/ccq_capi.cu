@@ -342,10 +342,15 @@ ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v, const v
                         H, Dk, Dv, workspace, workspace_bytes, static_cast<uint8_t *>(ckpt), 0, p, stream);
 }
 
-// Workspace layout of ccq_gla_bwd: three bf16 [B,T,H,128] exchange tensors,
+// Workspace layout of ccq_gla_bwd: three bf16 [B,T,H,128] exchange tensors and
+// the B*H progress counters of the concurrent walks (rounded to 256 bytes),
 // then (without caller checkpoints) the checkpoints and the forward's scratch.
+static size_t gla_bwd_counter_bytes(int B, int H) {
+    return (static_cast<size_t>(B) * H * sizeof(int) + 255) / 256 * 256;
+}
+
 static size_t gla_bwd_exchange_bytes(int B, int T, int H) {
-    return 3 * static_cast<size_t>(B) * T * H * 128 * 2;
+    return 3 * static_cast<size_t>(B) * T * H * 128 * 2 + gla_bwd_counter_bytes(B, H);
 }
 
 static size_t gla_fwd_scratch_bytes(const ccq_params &p, int B, int T, int H) {
@@ -416,9 +421,10 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     const size_t xbytes = static_cast<size_t>(B) * T * H * 128 * 2;
     uint8_t *qg = ws, *dkc = ws + xbytes, *gq = ws + 2 * xbytes;
+    int *ready = reinterpret_cast<int *>(ws + 3 * xbytes);
     const uint8_t *ck = static_cast<const uint8_t *>(ckpt);
     if (!ckpt) {
-        uint8_t *own = ws + 3 * xbytes;
+        uint8_t *own = ws + gla_bwd_exchange_bytes(B, T, H);
         // forward without output: dq stands in for the unused output tensor
         st = gla_fwd_impl(q, k, v, gk, lambda, in_dtype, gate_dtype, S0, C0, m0, t0, dq, nullptr, nullptr,
                           nullptr, nullptr, B, T, H, Dk, Dv, fwd_bytes ? own + ck_bytes : nullptr, fwd_bytes,
@@ -449,7 +455,7 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
     a.dlambda = dlambda; a.dgk = dgk; a.dS0 = dS0; a.dC0 = dC0; a.dm0 = dm0;
     a.status = device_status_word();
     if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
-    cudaError_t e = launch_gla_bwd(a, maps, s);
+    cudaError_t e = launch_gla_bwd(a, maps, ready, s);
     if (e != cudaSuccess) return cuda_fail(e, "GLA backward kernel launch");
     return CCQ_OK;
 }

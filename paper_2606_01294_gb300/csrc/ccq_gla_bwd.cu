@@ -233,12 +233,16 @@ enum { BAR_IN = 0, BAR_R1, BAR_R2, BAR_R3, BAR_R4, kBars };
 constexpr uint32_t TM_DC = 0, TM_SC = 128, TM_T1 = 192, TM_Z = 256, TM_DQ = 384;
 }  // namespace qk
 
-__global__ void __launch_bounds__(kThreads, 1)
-gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                 const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
-                 const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
-                 const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
-                 const __grid_constant__ CUtensorMap map_gq, const BwdArgs a) {
+// The q-side walk of one (sequence, head) pair bh.  With `ready` set, once a
+// chunk's exchange tensors are complete in global memory ready[bh] is raised to
+// the number of chunks done (release), for a kv-side CTA that trails this one;
+// chunk r is published while chunk r - 1 runs, so the q side never waits for a
+// store to complete.
+__device__ __forceinline__ void q_body(const CUtensorMap &map_q, const CUtensorMap &map_k, const CUtensorMap &map_v,
+                                       const CUtensorMap &map_do, const CUtensorMap &map_g,
+                                       const CUtensorMap &map_dq, const CUtensorMap &map_qg,
+                                       const CUtensorMap &map_dkc, const CUtensorMap &map_gq, const BwdArgs &a,
+                                       int bh, int *ready) {
     using namespace qk;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
@@ -260,7 +264,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
     const bool gate_f32 = a.gate_dtype != 0;
     const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
@@ -468,6 +472,13 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tma_store_4d(&map_gq, sm + OFF_SX + 16384, 0, h, c0, b);
             tma_store_4d(&map_gq, sm + OFF_SX + 16384 + 8192, 64, h, c0, b);
             tma_store_commit();
+            if (ready && it > 0) {
+                // every store of the previous chunk is older than the group just
+                // committed: once they are complete, publish that chunk
+                tma_store_wait_group<1>();
+                fence_proxy_async_global();
+                st_release_gpu(ready + bh, it);
+            }
             tc_fence_after();
             for (int k = 0; k < 8; ++k) {  // T3 = DZ Kbar^T
                 const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
@@ -589,6 +600,12 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tma_store_4d(&map_dkc, sm + OFF_K, 0, h, c0, b);
             tma_store_4d(&map_dkc, sm + OFF_K + 8192, 64, h, c0, b);
             tma_store_commit();
+            if (ready && it + 1 == NC) {
+                // the last chunk: publish as soon as its stores are complete
+                tma_store_wait_all();
+                fence_proxy_async_global();
+                st_release_gpu(ready + bh, NC);
+            }
             if (it + 1 < NC) {
                 tma_store_wait_read();  // staged tiles read before the next chunk lands on them
                 issue(r - 1);
@@ -650,12 +667,14 @@ enum { BAR_IN = 0, BAR_R1, BAR_R2, kBars };
 constexpr uint32_t TM_X = 0, TM_T1 = 128, TM_SA = 192, TM_DK = 256, TM_DV = 384;
 }  // namespace kv
 
-__global__ void __launch_bounds__(kThreads, 1)
-gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-                  const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
-                  const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
-                  const __grid_constant__ CUtensorMap map_gq, const __grid_constant__ CUtensorMap map_dk,
-                  const __grid_constant__ CUtensorMap map_dv, const BwdArgs a) {
+// The kv-side walk of (sequence, head) pair bh.  With `ready` set, each chunk's
+// exchange tensors are loaded only once ready[bh] shows the q side is past that
+// chunk (acquire; bounded wait, CCQ_ERR_TIMEOUT on give-up).
+__device__ __forceinline__ void kv_body(const CUtensorMap &map_k, const CUtensorMap &map_v, const CUtensorMap &map_do,
+                                        const CUtensorMap &map_g, const CUtensorMap &map_qg,
+                                        const CUtensorMap &map_dkc, const CUtensorMap &map_gq,
+                                        const CUtensorMap &map_dk, const CUtensorMap &map_dv, const BwdArgs &a,
+                                        int bh, const int *ready) {
     using namespace kv;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
@@ -674,7 +693,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
     const bool gate_f32 = a.gate_dtype != 0;
     const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
@@ -719,6 +738,21 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     }
     auto issue = [&](int r) {
         const int tg = r * kC;
+        if (ready) {
+            // wait (bounded) until the q side has published chunk r
+            const int need = NC - r;
+            if (ld_acquire_gpu(ready + bh) < need) {
+                const long long start = clock64();
+                while (ld_acquire_gpu(ready + bh) < need) {
+                    if (clock64() - start > kWaitLimitCycles) {
+                        *abort_flag = 1;
+                        atomicExch(status, kStatusTimeout);
+                        return;
+                    }
+                }
+            }
+            fence_proxy_async_global();
+        }
         uint64_t *bb = &bar[BAR_IN];
         mbar_arrive_expect_tx(bb, 6 * 16384 + g_bytes + 32768);
         tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, tg, b);
@@ -959,18 +993,90 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     }
 }
 
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
+                 const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
+                 const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
+                 const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
+                 const __grid_constant__ CUtensorMap map_gq, const BwdArgs a) {
+    q_body(map_q, map_k, map_v, map_do, map_g, map_dq, map_qg, map_dkc, map_gq, a, blockIdx.x, nullptr);
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
+                  const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
+                  const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
+                  const __grid_constant__ CUtensorMap map_gq, const __grid_constant__ CUtensorMap map_dk,
+                  const __grid_constant__ CUtensorMap map_dv, const BwdArgs a) {
+    kv_body(map_k, map_v, map_do, map_g, map_qg, map_dkc, map_gq, map_dk, map_dv, a, blockIdx.x, nullptr);
+}
+
+// Both walks at once: clusters of four CTAs for two (sequence, head) pairs --
+// ranks 0 and 1 the q sides, ranks 2 and 3 the kv sides.  The CTAs of a cluster
+// are co-scheduled, so a kv side can wait on its q side's progress counter;
+// neighbouring ranks run the same code, which keeps the two roles' instruction
+// streams from competing for the instruction cache they share.
+constexpr int kPairCluster = 4;
+
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_pair_kernel(const __grid_constant__ BwdMaps m, const BwdArgs a, int *ready) {
+    const int rank = blockIdx.x % kPairCluster;
+    const int bh = 2 * (blockIdx.x / kPairCluster) + (rank & 1);
+    if (rank < 2)
+        q_body(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq, a, bh, ready);
+    else
+        kv_body(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a, bh, ready);
+}
+
+constexpr uint32_t kPairSmem = qk::kSmem > kv::kSmem ? qk::kSmem : kv::kSmem;
+
 }  // namespace
 
-cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s) {
-    static bool attr_set = false;
-    if (!attr_set) {
+cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, int *ready, cudaStream_t s) {
+    static int pair_ok = -1;  // -1 unknown, 0 no, 1 yes (per process; one device type)
+    if (pair_ok < 0) {
         cudaError_t e = cudaFuncSetAttribute(gla_bwd_q_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(qk::kSmem));
         if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(gla_bwd_kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(kv::kSmem));
         if (e != cudaSuccess) return e;
-        attr_set = true;
+        e = cudaFuncSetAttribute(gla_bwd_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kPairSmem));
+        if (e != cudaSuccess) return e;
+        pair_ok = 0;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = kPairCluster;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(kPairCluster);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = kPairSmem;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int clusters = 0;
+        if (cudaOccupancyMaxActiveClusters(&clusters, gla_bwd_pair_kernel, &cfg) == cudaSuccess && clusters > 0)
+            pair_ok = 1;
+        (void)cudaGetLastError();
+    }
+    if (pair_ok == 1 && ready && (a.B * a.H) % 2 == 0) {
+        cudaError_t e = cudaMemsetAsync(ready, 0, sizeof(int) * static_cast<size_t>(a.B) * a.H, s);
+        if (e != cudaSuccess) return e;
+        cudaLaunchConfig_t cfg = {};
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = kPairCluster;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.gridDim = dim3(2 * a.B * a.H);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = kPairSmem;
+        cfg.stream = s;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        return cudaLaunchKernelEx(&cfg, gla_bwd_pair_kernel, m, a, ready);
     }
     const int grid = a.B * a.H;
     gla_bwd_q_kernel<<<grid, kThreads, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq, a);

@@ -124,8 +124,12 @@ struct BwdMaps {
     CUtensorMap q, k, v, dO, g, dq, dk, dv, qg, dkc, gq;
 };
 
-// Launches gla_bwd_q_kernel then gla_bwd_kv_kernel (one CTA per sequence and head).
-cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s);
+// Runs the q-side and kv-side walks of the backward: as clusters of two CTAs per
+// (sequence, head) that run concurrently, the kv side trailing the q side through
+// the progress counters `ready` (B*H ints of workspace, zeroed here), or -- when
+// the device cannot hold such a cluster, or `ready` is NULL -- as
+// gla_bwd_q_kernel then gla_bwd_kv_kernel.
+cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, int *ready, cudaStream_t s);
 
 // Encode the tensor map of a row-major [rows][128] bf16 matrix with 64 x 64 boxes
 // (128-byte swizzle).

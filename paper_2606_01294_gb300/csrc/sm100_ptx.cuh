@@ -138,6 +138,12 @@ __device__ __forceinline__ void tma_store_wait_all() {
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
+// Wait until at most the N most recently committed store groups are pending.
+template <int N>
+__device__ __forceinline__ void tma_store_wait_group() {
+    asm volatile("cp.async.bulk.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // Plain (untiled) bulk copy global -> shared completing on `bar`.  Both
 // addresses 16-byte aligned, `bytes` a multiple of 16.
 __device__ __forceinline__ void bulk_load(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
@@ -154,6 +160,22 @@ __device__ __forceinline__ void bulk_store(void *dst, const void *src, uint32_t 
                      reinterpret_cast<uint64_t>(dst)),
                  "r"(smem_addr(src)), "r"(bytes)
                  : "memory");
+}
+
+// Make async-proxy global writes (completed bulk stores) and generic accesses
+// mutually ordered; used around a release/acquire hand-off of TMA-written data.
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+__device__ __forceinline__ void st_release_gpu(int *p, int v) {
+    asm volatile("st.release.gpu.global.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ int ld_acquire_gpu(const int *p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
 }
 
 // 2^x on the SFU (ex2.approx.ftz.f32: relative error about 2^-22).
