@@ -182,9 +182,14 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         tmem_ld16x2_32<32>(tq, kk);
         const float ri = bet[i] * epos[i];
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-            const int j = 32 * hf + jj;
-            A[i * kAS + j] = (j < i) ? ri * eneg[j] * kk[jj] : 0.f;
+        for (int q4 = 0; q4 < 8; ++q4) {
+            float w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int j = 32 * hf + 4 * q4 + e;
+                w[e] = (j < i) ? ri * eneg[j] * kk[4 * q4 + e] : 0.f;
+            }
+            *reinterpret_cast<float4 *>(A + i * kAS + 32 * hf + 4 * q4) = make_float4(w[0], w[1], w[2], w[3]);
         }
     }
     __syncthreads();
@@ -205,26 +210,67 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     __syncthreads();
     // off-diagonal blocks, by distance from the diagonal:
     //   Tt_IJ = -Tt_II sum_{K=J}^{I-1} A_IK Tt_KJ
+    // 16 threads per 16 x 16 block, each a 4 x 4 sub-tile with float4 shared loads
     for (int dist = 1; dist < 4; ++dist) {
         const int nblk = 4 - dist;
-        for (int e = tid; e < nblk * 256; e += 128) {
-            const int blk = e >> 8, rr = (e >> 4) & 15, cc = e & 15;
-            const int J = blk, I = blk + dist;
-            float s = 0.f;
-            for (int K = J; K < I; ++K)
+        const int blk = tid >> 4, t = tid & 15, r0 = 4 * (t >> 2), c0 = 4 * (t & 3);
+        const int J = blk, I = blk + dist;
+        if (blk < nblk) {
+            float acc[4][4] = {};
+            for (int K = J; K < I; ++K) {
 #pragma unroll
-                for (int m = 0; m < 16; ++m)
-                    s = fmaf(A[(16 * I + rr) * kAS + 16 * K + m], Tt[(16 * K + m) * kAS + 16 * J + cc], s);
-            Y[e] = s;
+                for (int m = 0; m < 16; m += 4) {
+                    float4 av[4], tv[4];
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        av[u] = *reinterpret_cast<const float4 *>(A + (16 * I + r0 + u) * kAS + 16 * K + m);
+                        tv[u] = *reinterpret_cast<const float4 *>(Tt + (16 * K + m + u) * kAS + 16 * J + c0);
+                    }
+#pragma unroll
+                    for (int u = 0; u < 4; ++u) {
+                        const float a4[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
+#pragma unroll
+                        for (int mm = 0; mm < 4; ++mm) {
+                            acc[u][0] = fmaf(a4[mm], tv[mm].x, acc[u][0]);
+                            acc[u][1] = fmaf(a4[mm], tv[mm].y, acc[u][1]);
+                            acc[u][2] = fmaf(a4[mm], tv[mm].z, acc[u][2]);
+                            acc[u][3] = fmaf(a4[mm], tv[mm].w, acc[u][3]);
+                        }
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                *reinterpret_cast<float4 *>(Y + blk * 256 + (r0 + u) * 16 + c0) =
+                    make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
         }
         __syncthreads();
-        for (int e = tid; e < nblk * 256; e += 128) {
-            const int blk = e >> 8, rr = (e >> 4) & 15, cc = e & 15;
-            const int J = blk, I = blk + dist;
-            float s = 0.f;
+        if (blk < nblk) {
+            float acc[4][4] = {};
 #pragma unroll
-            for (int m = 0; m < 16; ++m) s = fmaf(Tt[(16 * I + rr) * kAS + 16 * I + m], Y[blk * 256 + m * 16 + cc], s);
-            Tt[(16 * I + rr) * kAS + 16 * J + cc] = -s;
+            for (int m = 0; m < 16; m += 4) {
+                float4 av[4], yv[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    av[u] = *reinterpret_cast<const float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * I + m);
+                    yv[u] = *reinterpret_cast<const float4 *>(Y + blk * 256 + (m + u) * 16 + c0);
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const float a4[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
+#pragma unroll
+                    for (int mm = 0; mm < 4; ++mm) {
+                        acc[u][0] = fmaf(a4[mm], yv[mm].x, acc[u][0]);
+                        acc[u][1] = fmaf(a4[mm], yv[mm].y, acc[u][1]);
+                        acc[u][2] = fmaf(a4[mm], yv[mm].z, acc[u][2]);
+                        acc[u][3] = fmaf(a4[mm], yv[mm].w, acc[u][3]);
+                    }
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                *reinterpret_cast<float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * J + c0) =
+                    make_float4(-acc[u][0], -acc[u][1], -acc[u][2], -acc[u][3]);
         }
         __syncthreads();
     }
@@ -234,10 +280,13 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 #pragma unroll
         for (int q4 = 0; q4 < 4; ++q4) {
             float wb[8], wg[8];
+            const float4 t0 = *reinterpret_cast<const float4 *>(Tt + i * kAS + 32 * hf + 8 * q4);
+            const float4 t1 = *reinterpret_cast<const float4 *>(Tt + i * kAS + 32 * hf + 8 * q4 + 4);
+            const float tr[8] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int j = 32 * hf + 8 * q4 + e;
-                const float t = (j <= i) ? Tt[i * kAS + j] : 0.f;  // A is dead: its space takes the tiles
+                const float t = (j <= i) ? tr[e] : 0.f;  // A is dead: its space takes the tiles
                 wb[e] = t * bet[j];
                 wg[e] = wb[e] * epos[j];
             }
