@@ -107,6 +107,13 @@ ccq_status check_ptrs(const char *names, std::initializer_list<const void *> req
     return CCQ_OK;
 }
 
+// Final position count, after the kernels that read t0 (tT may alias it).
+ccq_status finish_t(const int64_t *t0, int64_t *tT, int B, int T, cudaStream_t s) {
+    cudaError_t e = launch_t_update(t0, tT, B, T, s);
+    if (e != cudaSuccess) return cuda_fail(e, "position update launch");
+    return CCQ_OK;
+}
+
 ccq_status run_recurrent(RecurrentArgs &ra, cudaStream_t s) {
     cudaError_t e = launch_recurrent(ra, s);
     if (e != cudaSuccess) return cuda_fail(e, "recurrent kernel launch");
@@ -279,7 +286,7 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
         a.lambda = lambda;
         a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
         a.o = static_cast<__nv_bfloat16 *>(o);
-        a.ST = ST; a.CT = CT; a.mT = mT; a.tT = tT;
+        a.ST = ST; a.CT = CT; a.mT = mT;
         a.status = device_status_word();
         if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
         a.nseg = nseg;
@@ -290,11 +297,11 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
             a.seg_ws = static_cast<float *>(workspace);
             cudaError_t e = launch_gla_segments(a, maps, s);
             if (e != cudaSuccess) return cuda_fail(e, "segmented chunkwise GLA launch");
-            return CCQ_OK;
+            return finish_t(t0, tT, B, T, s);
         }
         cudaError_t e = launch_gla_chunk(a, maps, s);
         if (e != cudaSuccess) return cuda_fail(e, "chunkwise GLA kernel launch");
-        return CCQ_OK;
+        return finish_t(t0, tT, B, T, s);
     }
     RecurrentArgs ra = {};
     ra.backbone = 0; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
@@ -302,8 +309,9 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
     ra.l2norm = c.p.l2norm_qk; ra.centered = c.p.centered; ra.scale = c.scale;
     ra.q = q; ra.k = k; ra.v = v; ra.gate = gk; ra.beta = nullptr; ra.lambda = lambda;
     ra.S0 = S0; ra.C0 = C0; ra.m0 = m0; ra.t0 = t0;
-    ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT; ra.tT = tT;
-    return run_recurrent(ra, s);
+    ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT;
+    st = run_recurrent(ra, s);
+    return st != CCQ_OK ? st : finish_t(t0, tT, B, T, s);
 }
 
 ccq_status ccq_gla_fwd(const void *q, const void *k, const void *v, const void *gk,
@@ -519,12 +527,12 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
         a.lambda = lambda; a.g = g; a.beta = beta;
         a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
         a.o = static_cast<__nv_bfloat16 *>(o);
-        a.ST = ST; a.CT = CT; a.mT = mT; a.tT = tT;
+        a.ST = ST; a.CT = CT; a.mT = mT;
         a.status = device_status_word();
         if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
         cudaError_t e = launch_gdn_chunk(a, maps, static_cast<cudaStream_t>(stream));
         if (e != cudaSuccess) return cuda_fail(e, "chunkwise Gated DeltaNet kernel launch");
-        return CCQ_OK;
+        return finish_t(t0, tT, B, T, static_cast<cudaStream_t>(stream));
     }
     RecurrentArgs ra = {};
     ra.backbone = 1; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
@@ -532,8 +540,9 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
     ra.l2norm = c.p.l2norm_qk; ra.centered = c.p.centered; ra.scale = c.scale;
     ra.q = q; ra.k = k; ra.v = v; ra.gate = g; ra.beta = beta; ra.lambda = lambda;
     ra.S0 = S0; ra.C0 = C0; ra.m0 = m0; ra.t0 = t0;
-    ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT; ra.tT = tT;
-    return run_recurrent(ra, static_cast<cudaStream_t>(stream));
+    ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT;
+    st = run_recurrent(ra, static_cast<cudaStream_t>(stream));
+    return st != CCQ_OK ? st : finish_t(t0, tT, B, T, static_cast<cudaStream_t>(stream));
 }
 
 ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,
@@ -558,8 +567,9 @@ ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const voi
     ra.l2norm = c.p.l2norm_qk; ra.centered = c.p.centered; ra.scale = c.scale;
     ra.q = q; ra.k = k; ra.v = v; ra.gate = gate; ra.beta = beta; ra.lambda = lambda;
     ra.S0 = S; ra.C0 = C; ra.m0 = m; ra.t0 = t;
-    ra.o = o; ra.ST = S; ra.CT = C; ra.mT = m; ra.tT = t;
-    return run_recurrent(ra, static_cast<cudaStream_t>(stream));
+    ra.o = o; ra.ST = S; ra.CT = C; ra.mT = m;
+    st = run_recurrent(ra, static_cast<cudaStream_t>(stream));
+    return st != CCQ_OK ? st : finish_t(t, t, B, 1, static_cast<cudaStream_t>(stream));
 }
 
 ccq_status ccq_device_status(void *stream) {

@@ -552,7 +552,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const int sl = (NC - 1) & 1;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
-        if (a.tT && h == 0 && wt == 0 && last_seg) a.tT[b] = tseq0 + T;
     } else {
         // =============================================================== WG2: states
         const int row = 32 * (warp & 3) + lane;  // state row a (key dim)

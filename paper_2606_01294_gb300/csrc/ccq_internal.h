@@ -22,10 +22,14 @@ struct RecurrentArgs {
     const int64_t *t0;
     void *o;
     float *ST, *CT, *mT;
-    int64_t *tT;
 };
 
 cudaError_t launch_recurrent(const RecurrentArgs &a, cudaStream_t s);
+
+// tT[b] = t0[b] + T (t0 NULL: T), one thread per batch row.  The kernels leave
+// the final count to this launch, enqueued after them: tT may alias t0, and
+// every (batch, head) CTA reads t0[b] while it runs.
+cudaError_t launch_t_update(const int64_t *t0, int64_t *tT, int B, int T, cudaStream_t s);
 
 // Arguments of the chunkwise tensor-core kernels (Dk = Dv = 128, chunk 64,
 // bf16 q/k/v/o).
@@ -40,7 +44,6 @@ struct ChunkArgs {
     const int64_t *t0;
     __nv_bfloat16 *o;
     float *ST, *CT, *mT;
-    int64_t *tT;
     int *status;  // device status word (bounded-wait give-ups)
     // sequence segments (long sequences): nseg segments of seg_chunks chunks each
     // (the last one shorter); seg_ws holds kSegFloats floats per (sequence, segment).

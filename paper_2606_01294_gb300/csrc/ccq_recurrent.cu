@@ -289,12 +289,214 @@ recurrent_kernel(RecurrentArgs a) {
         if (a.CT) stv<CK>(a.CT + (sbase * DK + r) * DK + lane * CK, C[rr]);
     }
     if (a.mT && tid < DK) a.mT[sbase * DK + tid] = ms[tid];
-    if (a.tT && h == 0 && tid == 0) a.tT[b] = t;
+}
+
+// The decode step (T = 1) as a streaming pass: the cache of one (batch, head)
+// is read and written once, C first (rank-one update, row dots C qbar, stored
+// back at once), then S (update, read with q_clean, stored back), so only one
+// of the two 64 KB states is live in registers at a time.  At about half the
+// registers of recurrent_kernel two CTAs share an SM and one CTA's loads overlap
+// the other's arithmetic and stores.  Same arithmetic as recurrent_kernel with
+// T = 1 (Algorithm 2, Eq. clean, Eq. read).
+template <int DK, int DV, int BACKBONE, typename IT, typename GT>
+__global__ void __launch_bounds__(kThreads, 2)
+decode_kernel(RecurrentArgs a) {
+    constexpr int RS = DK / kWarps;  // state rows per warp
+    constexpr int CS = DV / 32;      // S columns per lane
+    constexpr int CK = DK / 32;      // C columns per lane
+
+    __shared__ float qs[DK], ks[DK], vs[DV], gs[DK], qcs[DK], ms[DK], cqs[DK];
+    __shared__ float red0[kWarps][DV], red1[kWarps][DV];
+    __shared__ float scal[8];  // 0 rq, 1 rk, 2 lambda, 3 alpha, 4 beta, 5 m.q, 6 qc.k
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const size_t sbase = static_cast<size_t>(bh);
+    const size_t row = static_cast<size_t>(b) * a.H + h;  // T = 1
+
+    // ---- C rows first: their loads are in flight while the token is prepared
+    float C[RS][CK];
+#pragma unroll
+    for (int rr = 0; rr < RS; ++rr) {
+        const int r = warp * RS + rr;
+        if (a.C0) ldv<CK>(a.C0 + (sbase * DK + r) * DK + lane * CK, C[rr]);
+        else
+#pragma unroll
+            for (int c = 0; c < CK; ++c) C[rr][c] = 0.f;
+    }
+    const IT *q = static_cast<const IT *>(a.q);
+    const IT *k = static_cast<const IT *>(a.k);
+    const IT *v = static_cast<const IT *>(a.v);
+    IT *o = static_cast<IT *>(a.o);
+    if (tid < DK) {
+        qs[tid] = to_f(q[row * DK + tid]);
+        ks[tid] = to_f(k[row * DK + tid]);
+        if (BACKBONE == 0) gs[tid] = __expf(to_f(static_cast<const GT *>(a.gate)[row * DK + tid]));
+        ms[tid] = a.m0 ? a.m0[sbase * DK + tid] : 0.f;
+    }
+    if (tid < DV) vs[tid] = to_f(v[row * DV + tid]);
+    if (tid == 0) {
+        scal[2] = a.lambda[row];
+        if (BACKBONE == 1) {
+            scal[3] = __expf(static_cast<const float *>(a.gate)[row]);
+            scal[4] = a.beta[row];
+        }
+    }
+    const int64_t t = (a.t0 ? a.t0[b] : 0) + 1;
+    __syncthreads();
+    if (warp < 2) {
+        const float *x = warp == 0 ? qs : ks;
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < CK; ++c) s += x[lane * CK + c] * x[lane * CK + c];
+        s = warp_sum(s);
+        if (lane == 0) scal[warp] = a.l2norm ? rsqrtf(fmaxf(s, 1e-12f)) : 1.f;
+    }
+    __syncthreads();
+    if (tid < DK) {
+        qs[tid] *= scal[0];
+        ks[tid] *= scal[1];
+        ms[tid] += ks[tid];  // m_t = m_{t-1} + kbar_t
+    }
+    __syncthreads();
+    // ---- C_t = C_{t-1} + kbar kbar^T, its row dots with qbar, and C_t written back
+    float kc[CK], qv[CK];
+#pragma unroll
+    for (int c = 0; c < CK; ++c) {
+        kc[c] = ks[lane * CK + c];
+        qv[c] = qs[lane * CK + c];
+    }
+    if (warp == 0) {
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < CK; ++c) s += ms[lane * CK + c] * qv[c];
+        s = warp_sum(s);
+        if (lane == 0) scal[5] = s;
+    }
+#pragma unroll
+    for (int rr = 0; rr < RS; ++rr) {
+        const int r = warp * RS + rr;
+        const float kr = ks[r];
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < CK; ++c) {
+            C[rr][c] = fmaf(kr, kc[c], C[rr][c]);
+            s = fmaf(C[rr][c], qv[c], s);
+        }
+        if (a.CT) stv<CK>(a.CT + (sbase * DK + r) * DK + lane * CK, C[rr]);
+        s = warp_sum(s);
+        if (lane == 0) cqs[r] = s;
+    }
+    // ---- S rows: loads issued before q_clean is formed
+    float S[RS][CS];
+#pragma unroll
+    for (int rr = 0; rr < RS; ++rr) {
+        const int r = warp * RS + rr;
+        if (a.S0) ldv<CS>(a.S0 + (sbase * DK + r) * DV + lane * CS, S[rr]);
+        else
+#pragma unroll
+            for (int c = 0; c < CS; ++c) S[rr][c] = 0.f;
+    }
+    __syncthreads();
+    // ---- Eq. clean: q_clean = qbar - lambda (C qbar / t - m (m.qbar) / t^2)
+    if (tid < DK) {
+        const float inv_t = 1.f / static_cast<float>(t);
+        float sig = cqs[tid] * inv_t;
+        if (a.centered) sig -= ms[tid] * scal[5] * inv_t * inv_t;
+        qcs[tid] = qs[tid] - scal[2] * sig;
+    }
+    __syncthreads();
+    if (BACKBONE == 1 && warp == 0) {
+        float s = 0.f;
+#pragma unroll
+        for (int c = 0; c < CK; ++c) s += qcs[lane * CK + c] * kc[c];
+        s = warp_sum(s);
+        if (lane == 0) scal[6] = s;
+    }
+    float vv[CS];
+#pragma unroll
+    for (int c = 0; c < CS; ++c) vv[c] = vs[lane * CS + c];
+    if (BACKBONE == 0) {
+        float po[CS];
+#pragma unroll
+        for (int c = 0; c < CS; ++c) po[c] = 0.f;
+#pragma unroll
+        for (int rr = 0; rr < RS; ++rr) {
+            const int r = warp * RS + rr;
+            const float al = gs[r], kr = ks[r], qr = qcs[r];
+#pragma unroll
+            for (int c = 0; c < CS; ++c) {
+                S[rr][c] = fmaf(al, S[rr][c], kr * vv[c]);
+                po[c] = fmaf(S[rr][c], qr, po[c]);
+            }
+            if (a.ST) stv<CS>(a.ST + (sbase * DK + r) * DV + lane * CS, S[rr]);
+        }
+#pragma unroll
+        for (int c = 0; c < CS; ++c) red0[warp][lane * CS + c] = po[c];
+        __syncthreads();
+        if (tid < DV) {
+            float s = 0.f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) s += red0[w][tid];
+            o[row * DV + tid] = from_f<IT>(a.scale * s);
+        }
+    } else {
+        float pk[CS], pq[CS];
+#pragma unroll
+        for (int c = 0; c < CS; ++c) pk[c] = pq[c] = 0.f;
+#pragma unroll
+        for (int rr = 0; rr < RS; ++rr) {
+            const int r = warp * RS + rr;
+            const float kr = ks[r], qr = qcs[r];
+#pragma unroll
+            for (int c = 0; c < CS; ++c) {
+                pk[c] = fmaf(kr, S[rr][c], pk[c]);
+                pq[c] = fmaf(qr, S[rr][c], pq[c]);
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < CS; ++c) {
+            red0[warp][lane * CS + c] = pk[c];
+            red1[warp][lane * CS + c] = pq[c];
+        }
+        __syncthreads();
+        if (tid < DV) {
+            float sk = 0.f, sq = 0.f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) {
+                sk += red0[w][tid];
+                sq += red1[w][tid];
+            }
+            red0[0][tid] = sk;  // kbar^T S (old state)
+            const float al = scal[3], be = scal[4], qk = scal[6];
+            o[row * DV + tid] = from_f<IT>(a.scale * (al * sq - al * be * qk * sk + be * qk * vs[tid]));
+        }
+        __syncthreads();
+        const float al = scal[3], be = scal[4];
+        float ksv[CS];
+#pragma unroll
+        for (int c = 0; c < CS; ++c) ksv[c] = red0[0][lane * CS + c];
+#pragma unroll
+        for (int rr = 0; rr < RS; ++rr) {
+            const int r = warp * RS + rr;
+            const float kr = ks[r];
+#pragma unroll
+            for (int c = 0; c < CS; ++c) S[rr][c] = al * (S[rr][c] - be * kr * ksv[c]) + be * kr * vv[c];
+            if (a.ST) stv<CS>(a.ST + (sbase * DK + r) * DV + lane * CS, S[rr]);
+        }
+    }
+    if (a.mT && tid < DK) a.mT[sbase * DK + tid] = ms[tid];
 }
 
 template <int DK, int DV, int BB, typename IT>
 cudaError_t launch_gate(const RecurrentArgs &a, cudaStream_t s) {
-    if (BB == 0 && a.gate_dtype == 0)
+    const bool gbf = BB == 0 && a.gate_dtype == 0;
+    if (a.T == 1) {
+        if (gbf) decode_kernel<DK, DV, BB, IT, __nv_bfloat16><<<a.B * a.H, kThreads, 0, s>>>(a);
+        else decode_kernel<DK, DV, BB, IT, float><<<a.B * a.H, kThreads, 0, s>>>(a);
+        return cudaGetLastError();
+    }
+    if (gbf)
         recurrent_kernel<DK, DV, BB, IT, __nv_bfloat16><<<a.B * a.H, kThreads, 0, s>>>(a);
     else
         recurrent_kernel<DK, DV, BB, IT, float><<<a.B * a.H, kThreads, 0, s>>>(a);
@@ -313,7 +515,18 @@ cudaError_t launch_bb(const RecurrentArgs &a, cudaStream_t s) {
     return launch_in<DK, DV, 1>(a, s);
 }
 
+__global__ void t_update_kernel(const int64_t *t0, int64_t *tT, int B, int T) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < B) tT[i] = (t0 ? t0[i] : 0) + T;
+}
+
 }  // namespace
+
+cudaError_t launch_t_update(const int64_t *t0, int64_t *tT, int B, int T, cudaStream_t s) {
+    if (!tT || B == 0) return cudaSuccess;
+    t_update_kernel<<<(B + 255) / 256, 256, 0, s>>>(t0, tT, B, T);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_recurrent(const RecurrentArgs &a, cudaStream_t s) {
     if (a.B * a.H == 0) return cudaSuccess;

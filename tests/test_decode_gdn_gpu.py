@@ -58,6 +58,29 @@ def test_prefill_then_decode_equals_longer_prefill(backbone):
     assert int(st.t[0]) == 97
 
 
+@pytest.mark.parametrize("backbone", [GLA, GDN])
+def test_repeated_in_place_decode_every_head(backbone):
+    """Five decode steps in place on 64 batch rows x 16 heads (1024 CTAs, so the
+    heads of one row run in different waves): the shared position count t must
+    advance by exactly one per step for every head, whatever the CTA order."""
+    B, H, d = 64, 16, 128
+    steps = 5
+    P = gen.make_inputs(backbone, B, 40 + steps, H, d, d, dtype=torch.bfloat16, seed=31, lam="high",
+                        keys="structured")
+    pre = {n: (None if x is None else x[:, :40].contiguous()) for n, x in P.items()}
+    _, st = gpu_forward(backbone, pre)
+    for s in range(steps):
+        tok = {n: (None if x is None else x[:, 40 + s].contiguous().cuda()) for n, x in P.items()}
+        o = ccq.decode_step(backbone, tok["q"], tok["k"], tok["v"], tok["gate"], tok["lam"], st,
+                            beta=tok["beta"])
+        torch.cuda.synchronize()
+        assert (st.t.cpu() == 41 + s).all()
+    full = oracle_forward(backbone, P)
+    assert rel_err(o, full["o"][:, -1]) <= TOL[torch.bfloat16]
+    for n in ("S", "C", "m"):
+        assert rel_err(getattr(st, n), full[n]) <= TOL[torch.bfloat16], n
+
+
 def test_decode_full_size_sampled():
     """B=256, H=16, Dk=Dv=128 (the decode benchmark's launch), sampled pairs."""
     B, H, d = 256, 16, 128
