@@ -117,6 +117,7 @@ STEP_KERNELS = {
     "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
                            "gla_bwd_pair_kernel"],
 }
+# (each step also runs the one-thread-per-row position update: 8 bytes per batch row, not counted)
 KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kernel": "ccq_gla_segment.cu",
                 "gla_segment_combine_kernel": "ccq_gla_segment.cu", "gdn_wy_kernel": "ccq_gdn_chunk.cu",
                 "gdn_chunk_kernel": "ccq_gdn_chunk.cu", "recurrent": "ccq_recurrent.cu",

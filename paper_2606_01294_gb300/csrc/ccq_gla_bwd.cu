@@ -950,12 +950,19 @@ __device__ __forceinline__ void kv_body(const CUtensorMap &map_k, const CUtensor
             // column d = tid, tokens in reverse
             float acc = carry[tid];
             const int nvalid = min(kC, T - c0);
-            for (int t = kC - 1; t >= 0; --t) {
-                acc += dG[t * kDgStride + tid];
-                if (t < nvalid) {
-                    const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + tid;
-                    if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
-                    else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
+            for (int t8 = kC - 8; t8 >= 0; t8 -= 8) {
+                float x[8];
+#pragma unroll
+                for (int u = 0; u < 8; ++u) x[u] = dG[(t8 + u) * kDgStride + tid];  // loads in flight together
+#pragma unroll
+                for (int u = 7; u >= 0; --u) {
+                    acc += x[u];
+                    const int t = t8 + u;
+                    if (t < nvalid) {
+                        const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + tid;
+                        if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
+                        else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
+                    }
                 }
             }
             carry[tid] = cnext[tid];
