@@ -223,6 +223,23 @@ def dist_env():
         int(os.environ.get("WORLD_SIZE", 1))
 
 
+def max_over_ranks(value, device=None):
+    """The largest of every rank's `value` (the identity without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(value)
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device or "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(world, units_per_step, steps, max_ms):
+    """Units all ranks processed per second, timed by the slowest rank (weak
+    scaling: every rank runs its own replica of the workload)."""
+    return world * units_per_step * steps / (max_ms / 1e3)
+
+
 def cpu_oracle_run(kind, B, H, T, D, sample_b, seed):
     """Time the fp64 oracle on host cores over `sample_b` batch rows of T tokens."""
     import torch
@@ -395,14 +412,10 @@ def run_gpu(args):
     if world > 1:
         dist.barrier()
     ccq.device_status()
-    total_ms = t_start.elapsed_time(t_end)
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), dev)
     launch_ms = [a.elapsed_time(b) for a, b in ev]
-    if world > 1:
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
     ms_per_step = total_ms / args.steps
-    value = world * tokens_per_step * args.steps / (total_ms / 1e3)
+    value = whole_job_rate(world, tokens_per_step, args.steps, total_ms)
 
     # ---------------- e2e: host buffers, copies inside the timed region
     def e2e_step():
@@ -437,12 +450,8 @@ def run_gpu(args):
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e_value = world * tokens_per_step / (e2e_ms / 1e3)
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dev)
+    e2e_value = whole_job_rate(world, tokens_per_step, 1, e2e_ms)
 
     line = None
     if rank == 0:

@@ -20,11 +20,21 @@ extern "C" {
  *      holding row i.  M = 64: rows 0..63 of D = A B read back with the
  *      16-lane split load the kernels use (rows 64..127 are not written).
  *   M in {64, 128}; N in {64, 128}; K in {64, 128}; a_mn / b_mn = 1 stage that
- *   operand MN-major in shared memory, 0 = K-major (M = 64 needs a_mn = 0).
+ *   operand MN-major in shared memory, 0 = K-major.
  * Asynchronous on `stream`; CCQ_ERR_UNSUPPORTED for other shapes.
  */
 CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *D, int M, int N, int K,
                                 int a_mn, int b_mn, void *stream);
+
+/*
+ * Exercises the kernels' failure path without a fault: one CTA waits on an
+ * mbarrier that nothing arrives on, with the same bounded wait every CCQ kernel
+ * uses (about one second of SM clock).  The wait gives up, records
+ * CCQ_ERR_TIMEOUT in the device status word and the kernel returns normally,
+ * so the context stays usable; ccq_device_status() then reports (and clears)
+ * the timeout.  Asynchronous on `stream`.
+ */
+CCQ_API ccq_status ccq_diag_wait_timeout(void *stream);
 
 #ifdef __cplusplus
 }

@@ -116,8 +116,28 @@ diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int M
     }
 }
 
+// Waits (bounded) on a barrier that no thread or copy ever completes.
+__global__ void diag_wait_kernel(int *status) {
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        fence_barrier_init();
+    }
+    __syncthreads();
+    mbar_wait(&bar, 0, &abort_flag, status);
+}
+
 }  // namespace
 }  // namespace ccq
+
+extern "C" CCQ_API ccq_status ccq_diag_wait_timeout(void *stream) {
+    int *status = ccq::device_status_word();
+    if (!status) return CCQ_ERR_CUDA;
+    ccq::diag_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(status);
+    return cudaGetLastError() == cudaSuccess ? CCQ_OK : CCQ_ERR_CUDA;
+}
 
 extern "C" CCQ_API ccq_status ccq_diag_mma(const void *A, const void *B, float *D, int M, int N,
                                            int K, int a_mn, int b_mn, void *stream) {
