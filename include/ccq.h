@@ -206,8 +206,9 @@ CCQ_API ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v,
  *             dm0 [B,H,Dk] fp32 (each may be NULL): gradients of lambda and of
  *             the initial states.
  *   workspace at least ccq_gla_bwd_workspace_size() bytes (16-byte aligned):
- *             three bf16 [B,T,H,128] tensors the two backward kernels exchange,
- *             plus the checkpoints and forward scratch when ckpt is NULL.
+ *             four bf16 [B,T,H,128] tensors and 67 KB per 64-token chunk that
+ *             the backward kernels exchange, plus the checkpoints and forward
+ *             scratch when ckpt is NULL.
  * Supported: bf16 inputs with Dk = Dv = 128 (the chunkwise tensor-core path),
  * algo AUTO or CHUNKWISE; otherwise CCQ_ERR_UNSUPPORTED.  T = 0 copies the
  * final-state gradients to the initial-state ones.

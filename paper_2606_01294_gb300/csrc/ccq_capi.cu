@@ -350,15 +350,13 @@ ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v, const v
                         H, Dk, Dv, workspace, workspace_bytes, static_cast<uint8_t *>(ckpt), 0, p, stream);
 }
 
-// Workspace layout of ccq_gla_bwd: three bf16 [B,T,H,128] exchange tensors and
-// the B*H progress counters of the concurrent walks (rounded to 256 bytes),
-// then (without caller checkpoints) the checkpoints and the forward's scratch.
-static size_t gla_bwd_counter_bytes(int B, int H) {
-    return (static_cast<size_t>(B) * H * sizeof(int) + 255) / 256 * 256;
-}
-
+// Workspace layout of ccq_gla_bwd: four bf16 [B,T,H,128] exchange tensors, then
+// per chunk the q kernel's vectors (3 x 128 fp32), the state pass's images (64 KB)
+// and vectors (2 x 128 fp32); then (without caller checkpoints) the checkpoints
+// and the forward's scratch.
 static size_t gla_bwd_exchange_bytes(int B, int T, int H) {
-    return 3 * static_cast<size_t>(B) * T * H * 128 * 2 + gla_bwd_counter_bytes(B, H);
+    const size_t chunks = static_cast<size_t>(B) * H * ((T + 63) / 64);
+    return 4 * static_cast<size_t>(B) * T * H * 128 * 2 + chunks * (3 * 128 * 4 + 65536 + 2 * 128 * 4);
 }
 
 static size_t gla_fwd_scratch_bytes(const ccq_params &p, int B, int T, int H) {
@@ -428,8 +426,11 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
     if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
     uint8_t *ws = static_cast<uint8_t *>(workspace);
     const size_t xbytes = static_cast<size_t>(B) * T * H * 128 * 2;
-    uint8_t *qg = ws, *dkc = ws + xbytes, *gq = ws + 2 * xbytes;
-    int *ready = reinterpret_cast<int *>(ws + 3 * xbytes);
+    const size_t chunks = static_cast<size_t>(B) * H * ((T + 63) / 64);
+    uint8_t *qg = ws, *dkc = ws + xbytes, *gq = ws + 2 * xbytes, *dzr = ws + 3 * xbytes;
+    float *chunk_vec = reinterpret_cast<float *>(ws + 4 * xbytes);
+    uint8_t *state_img = ws + 4 * xbytes + chunks * 3 * 128 * 4;
+    float *state_vec = reinterpret_cast<float *>(state_img + chunks * 65536);
     const uint8_t *ck = static_cast<const uint8_t *>(ckpt);
     if (!ckpt) {
         uint8_t *own = ws + gla_bwd_exchange_bytes(B, T, H);
@@ -452,7 +453,8 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
         !make_token_map(&maps.dv, dv, 2, B, T, H, 128, 64, true) ||
         !make_token_map(&maps.qg, qg, 2, B, T, H, 128, 64, true) ||
         !make_token_map(&maps.dkc, dkc, 2, B, T, H, 128, 64, true) ||
-        !make_token_map(&maps.gq, gq, 2, B, T, H, 128, 64, true))
+        !make_token_map(&maps.gq, gq, 2, B, T, H, 128, 64, true) ||
+        !make_token_map(&maps.dzr, dzr, 2, B, T, H, 128, 64, true))
         return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
     BwdArgs a = {};
     a.B = B; a.T = T; a.H = H;
@@ -461,9 +463,10 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
     a.lambda = lambda; a.t0 = t0; a.ckpt = ck;
     a.dST = dST; a.dCT = dCT; a.dmT = dmT;
     a.dlambda = dlambda; a.dgk = dgk; a.dS0 = dS0; a.dC0 = dC0; a.dm0 = dm0;
+    a.chunk_vec = chunk_vec; a.state_img = state_img; a.state_vec = state_vec;
     a.status = device_status_word();
     if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
-    cudaError_t e = launch_gla_bwd(a, maps, ready, s);
+    cudaError_t e = launch_gla_bwd(a, maps, s);
     if (e != cudaSuccess) return cuda_fail(e, "GLA backward kernel launch");
     return CCQ_OK;
 }

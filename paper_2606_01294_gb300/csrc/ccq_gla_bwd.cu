@@ -30,17 +30,25 @@
 //            evaluated per chunk as sum_{s>=t in chunk r} dG_s + rowsum(dS_{r+1} S_{r+1})
 //   l2 normalisation: dq = (dqbar - qbar (qbar . dqbar)) / |q|, likewise dk.
 //
-// Two kernels, one CTA per (batch, head), chunks in reverse order; each keeps
-// its carried state in tensor memory as an fp32 accumulator:
-//   gla_bwd_q_kernel   DC (TMEM) and Dm: recomputes z and qc, forms dqc, dq,
-//                      dlambda and the CCQ part of dkbar; writes QG, qc*dqc
-//                      and that dkbar part to bf16 scratch tensors.
-//   gla_bwd_kv_kernel  dS (TMEM, kept as e^{-Gmid} dS like the forward's
-//                      deferred state scaling): dk, dv and dgk.
-// The forward states of each chunk come from the checkpoints the forward
-// kernel writes (ccq_internal.h); 64-row products are M = 64 MMAs whose rows
-// 16q..16q+15 sit in TMEM lanes 32q..32q+15, so thread (warp w, lane l) owns
-// row 16w + l % 16 and column half l / 16 in every epilogue.
+// Everything per chunk depends only on the forward's chunk-start states (the
+// checkpoints ccq_gla_chunk.cu writes) and on the three carried adjoints
+// (dS, DC, Dm) at the chunk's end, so the backward is three launches:
+//   gla_bwd_q_kernel     one CTA per chunk (parallel): z, qc, dqc, dq, dlambda,
+//                        the chunk-local CCQ part of dkbar (W2^T DZ + W3^T Qbar),
+//                        and the chunk's inputs to the carried sums (QG, DZ
+//                        scaled by 1/|q|, the Dm increment, the gate factors).
+//   gla_bwd_state_kernel one CTA per sequence and head, chunks last to first:
+//                        carries dS (kept as e^{-Gmid} dS, like the forward's
+//                        deferred state scaling) and DC in TMEM and Dm, and
+//                        writes, per chunk, the states carried into it (bf16
+//                        tile images of Diag(e^{Gc-Gmid}) dS_{r+1} and DC_{r+1},
+//                        Dm_{r+1}) and the gate carry rowsum(dS_{r+1} S_{r+1}).
+//   gla_bwd_kv_kernel    one CTA per chunk (parallel): dk (write part, the
+//                        CCQ inter term K (DC + DC^T), Dm), dv, dgk.
+// 64-row products are M = 64 MMAs whose rows 16q..16q+15 sit in TMEM lanes
+// 32q..32q+15, so thread (warp w, lane l) owns row 16w + l % 16 and column
+// half l / 16 in every 64-row epilogue; 128-row products (the carried states)
+// give thread t row t.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -206,50 +214,45 @@ __device__ __forceinline__ float masked_sum(int i, int hf, const float (&sc)[32]
 }
 
 // =====================================================================================
-// gla_bwd_q_kernel
+// gla_bwd_q_kernel: one CTA per (sequence, head, chunk)
 // =====================================================================================
 namespace qk {
 constexpr uint32_t OFF_Q = 0;        // qbar; then dq (staged for the store)
-constexpr uint32_t OFF_K = 16384;    // kbar; then the CCQ part of dkbar (staged)
+constexpr uint32_t OFF_K = 16384;    // kbar; then the chunk-local CCQ part of dkbar (staged)
 constexpr uint32_t OFF_V = 32768;    // v; then QG (staged)
 constexpr uint32_t OFF_DO = 49152;   // do; then DZ
-constexpr uint32_t OFF_KD = 65536;   // raw gates land here (fp32: KD + EG); then Kd
+constexpr uint32_t OFF_KD = 65536;   // raw gates land here (fp32: KD + EG); then Kd; then DZ / |q| (staged)
 constexpr uint32_t OFF_EG = 81920;   // EG
 constexpr uint32_t OFF_SK = 98304;   // S^K_r      } one checkpoint record,
 constexpr uint32_t OFF_SX = 131072;  // Sx_r       } one bulk copy; then dqc (16K) + qc*dqc (16K)
-constexpr uint32_t OFF_DC = 163840;  // bf16 DC_{r+1}
-constexpr uint32_t OFF_W2 = 196608;  // W2
-constexpr uint32_t OFF_P1 = 204800;  // P1, then W3
-constexpr uint32_t OFF_BC = 212992;  // [64][64] K-major B operand of the Dm update: row 0 = -c1, then -cz
-constexpr uint32_t OFF_MISC = 221184;
-constexpr uint32_t M_MR = 0, M_DM = 512, M_RQ = 1024, M_LAM = 1280, M_ITAU = 1536, M_MQ = 1792,
-                   M_C1 = 2048, M_MDZ = 2304, M_CZ = 2560, M_RK = 2816, M_GP = 3072, M_BAR = 3584,
-                   M_TMEM = 3632, M_ABORT = 3636;
-constexpr uint32_t kMisc = 3712;
+constexpr uint32_t OFF_W2 = 163840;  // W2
+constexpr uint32_t OFF_P1 = 172032;  // P1, then W3
+constexpr uint32_t OFF_BC = 180224;  // [64][64] K-major B operand of the Dm increment: row 0 = -c1, then -cz
+constexpr uint32_t OFF_MISC = 188416;
+constexpr uint32_t M_MR = 0, M_RQ = 512, M_LAM = 768, M_ITAU = 1024, M_MQ = 1280, M_C1 = 1536, M_MDZ = 1792,
+                   M_CZ = 2048, M_RK = 2304, M_GP = 2560, M_F = 3072, M_EM = 3584, M_BAR = 4096,
+                   M_TMEM = 4144, M_ABORT = 4148;
+constexpr uint32_t kMisc = 4224;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
 static_assert(OFF_SX == OFF_SK + 32768, "a checkpoint record lands as one block");
 enum { BAR_IN = 0, BAR_R1, BAR_R2, BAR_R3, BAR_R4, kBars };
-constexpr uint32_t TM_DC = 0, TM_SC = 128, TM_T1 = 192, TM_Z = 256, TM_DQ = 384;
+constexpr uint32_t TM_SC = 0, TM_T1 = 64, TM_Z = 128, TM_DQ = 256;
 }  // namespace qk
 
-// The q-side walk of one (sequence, head) pair bh.  With `ready` set, once a
-// chunk's exchange tensors are complete in global memory ready[bh] is raised to
-// the number of chunks done (release), for a kv-side CTA that trails this one;
-// chunk r is published while chunk r - 1 runs, so the q side never waits for a
-// store to complete.
-__device__ __forceinline__ void q_body(const CUtensorMap &map_q, const CUtensorMap &map_k, const CUtensorMap &map_v,
-                                       const CUtensorMap &map_do, const CUtensorMap &map_g,
-                                       const CUtensorMap &map_dq, const CUtensorMap &map_qg,
-                                       const CUtensorMap &map_dkc, const CUtensorMap &map_gq, const BwdArgs &a,
-                                       int bh, int *ready) {
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
+                 const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
+                 const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
+                 const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
+                 const __grid_constant__ CUtensorMap map_gq, const __grid_constant__ CUtensorMap map_dzr,
+                 const BwdArgs a) {
     using namespace qk;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *Mr = reinterpret_cast<float *>(misc + M_MR);
-    float *Dm = reinterpret_cast<float *>(misc + M_DM);
     float *rqv = reinterpret_cast<float *>(misc + M_RQ);
     float *lamv = reinterpret_cast<float *>(misc + M_LAM);
     float *itauv = reinterpret_cast<float *>(misc + M_ITAU);
@@ -259,70 +262,53 @@ __device__ __forceinline__ void q_body(const CUtensorMap &map_q, const CUtensorM
     float *czv = reinterpret_cast<float *>(misc + M_CZ);
     float *rkv = reinterpret_cast<float *>(misc + M_RK);
     float *gp = reinterpret_cast<float *>(misc + M_GP);
+    float *fv = reinterpret_cast<float *>(misc + M_F);
+    float *emv = reinterpret_cast<float *>(misc + M_EM);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
+    const int bh = blockIdx.x / NC, r = blockIdx.x % NC, b = bh / H, h = bh % H;
+    const int c0 = r * kC;
     const bool gate_f32 = a.gate_dtype != 0;
     const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
     const int64_t tseq0 = a.t0 ? a.t0[b] : 0;
-    const uint8_t *ck = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T);
+    const uint8_t *rec = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T) + static_cast<size_t>(r) * kCkptChunkBytes;
+    float *cvec = a.chunk_vec + static_cast<size_t>(blockIdx.x) * 3 * kD;  // f, e^{Gmid}, Dm increment
     int *status = a.status;
 
     if (tid == 0) {
         for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        tma_prefetch_desc(&map_q);
-        tma_prefetch_desc(&map_k);
-        tma_prefetch_desc(&map_v);
-        tma_prefetch_desc(&map_do);
-        tma_prefetch_desc(&map_g);
+        uint64_t *bb = &bar[BAR_IN];
+        mbar_arrive_expect_tx(bb, 4 * 16384 + g_bytes + 65536 + 512);
+        tma_load_4d(sm + OFF_Q, &map_q, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_Q + 8192, &map_q, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, c0, b);
+        bulk_load(sm + OFF_SK, rec, 65536, bb);
+        bulk_load(misc + M_MR, rec + 65536, 512, bb);
     }
     if (warp == 0) tmem_alloc(tmem_slot, 512);
     for (int e = tid; e < 8192 / 16; e += kThreads)
         reinterpret_cast<uint4 *>(sm + OFF_BC)[e] = make_uint4(0u, 0u, 0u, 0u);
-    Dm[tid] = a.dmT ? a.dmT[static_cast<size_t>(bh) * kD + tid] : 0.f;
+    if (tid < kC) {
+        const int n = c0 + tid;
+        lamv[tid] = n < T ? a.lambda[(static_cast<size_t>(b) * T + n) * H + h] : 0.f;
+        itauv[tid] = 1.f / static_cast<float>(tseq0 + n + 1);
+    }
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
-    {
-        // DC <- dC_T (row a = tid)
-        const float *src = a.dCT ? a.dCT + (static_cast<size_t>(bh) * kD + tid) * kD : nullptr;
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            float x[32];
-#pragma unroll
-            for (int e = 0; e < 32; ++e) x[e] = src ? src[32 * c + e] : 0.f;
-            tmem_st32(tq + TM_DC + 32 * c, x);
-        }
-        tmem_wait_st();
-    }
-    auto issue = [&](int r) {
-        const int tg = r * kC;
-        uint64_t *bb = &bar[BAR_IN];
-        mbar_arrive_expect_tx(bb, 4 * 16384 + g_bytes + 65536 + 512);
-        tma_load_4d(sm + OFF_Q, &map_q, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_Q + 8192, &map_q, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, tg, b);
-        const uint8_t *rec = ck + static_cast<size_t>(r) * kCkptChunkBytes;
-        bulk_load(sm + OFF_SK, rec, 65536, bb);
-        bulk_load(misc + M_MR, rec + 65536, 512, bb);
-    };
-    if (tid == 0 && NC > 0) issue(NC - 1);
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
 
     const int i = 16 * warp + (lane & 15);  // chunk row of this thread in the M = 64 products
     const int hf = lane >> 4;               // column half
@@ -334,301 +320,233 @@ __device__ __forceinline__ void q_body(const CUtensorMap &map_q, const CUtensorM
     const uint64_t dDO = make_desc(sb + OFF_DO, 16, 1024), dDOm = make_desc(sb + OFF_DO, 8192, 1024);
     const uint64_t dKDm = make_desc(sb + OFF_KD, 8192, 1024);
     const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024), dSX = make_desc(sb + OFF_SX, 16, 1024);
-    const uint64_t dDC = make_desc(sb + OFF_DC, 16, 1024), dDCm = make_desc(sb + OFF_DC, 16384, 1024);
     const uint64_t dW2 = make_desc(sb + OFF_W2, 16, 1024), dW2m = make_desc(sb + OFF_W2, 8192, 1024);
     const uint64_t dP1 = make_desc(sb + OFF_P1, 16, 1024), dP1m = make_desc(sb + OFF_P1, 8192, 1024);
     const uint64_t dBC = make_desc(sb + OFF_BC, 16, 1024);
 
-    for (int it = 0; it < NC; ++it) {
-        const int r = NC - 1 - it;
-        const uint32_t par = it & 1;
-        const int c0 = r * kC;
-        mbar_wait(&bar[BAR_IN], par, abort_flag, status);
-        if (tid < kC) {
-            const int n = c0 + tid;
-            lamv[tid] = n < T ? a.lambda[(static_cast<size_t>(b) * T + n) * H + h] : 0.f;
-            itauv[tid] = 1.f / static_cast<float>(tseq0 + n + 1);
-        }
-        prep_chunk(sm + OFF_Q, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, Mr, rqv, mqv, rkv,
-                   gp, nullptr, nullptr, tid);
-        {
-            // DC_{r+1} -> bf16 operand tile (row a = tid)
-            tc_fence_after();
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_DC + 32 * c, x);
-                uint8_t *tile = sm + OFF_DC + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int k = 0; k < 8; ++k) {  // Sc = Qbar Kbar^T, T1 = dO V^T
-                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                mma_bf16(tbase + TM_SC, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {
-                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                mma_bf16(tbase + TM_T1, dDO + ko, dV + ko, ID_64x64_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {  // Zi = Qbar S^K, Dq = dO Sx^T
-                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
-                mma_bf16(tbase + TM_Z, dQ + ka, dSK + kb, ID_64x128_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {
-                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
-                mma_bf16(tbase + TM_DQ, dDO + ka, dSX + kb, ID_64x128_KK, k != 0);
-            }
-            mma_commit(&bar[BAR_R1]);
-        }
-        // ---- E1: c1, W2, P1
-        mbar_wait(&bar[BAR_R1], par, abort_flag, status);
+    mbar_wait(&bar[BAR_IN], 0, abort_flag, status);
+    prep_chunk(sm + OFF_Q, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, Mr, rqv, mqv, rkv, gp, fv,
+               emv, tid);
+    tc_fence_before();
+    if (tid == 0 && !*abort_flag) {
         tc_fence_after();
-        {
-            float sc[32];
-            tmem_ld16x2_32<32>(tq + TM_SC, sc);
-            const float part = masked_sum(i, hf, sc);
-            const float c1 = a.centered ? (mqv[i] + part) * itauv[i] : 0.f;
-            if (hf == 0) {
-                c1v[i] = c1;
-                *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-c1);
-            }
-            masked_row(sm + OFF_W2, i, hf, sc, c1);
-            float t1[32];
-            tmem_ld16x2_32<32>(tq + TM_T1, t1);
-            masked_row(sm + OFF_P1, i, hf, t1, 0.f);
+        for (int k = 0; k < 8; ++k) {  // Sc = Qbar Kbar^T, T1 = dO V^T
+            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+            mma_bf16(tbase + TM_SC, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
         }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int k = 0; k < 4; ++k)  // Zi += W2 Kbar, Dq += P1 Kd
-                mma_bf16(tbase + TM_Z, dW2 + k * 2, dKm + k * 128, ID_64x128_KM, 1);
-            for (int k = 0; k < 4; ++k)
-                mma_bf16(tbase + TM_DQ, dP1 + k * 2, dKDm + k * 128, ID_64x128_KM, 1);
-            mma_commit(&bar[BAR_R2]);
+        for (int k = 0; k < 8; ++k) {
+            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+            mma_bf16(tbase + TM_T1, dDO + ko, dV + ko, ID_64x64_KK, k != 0);
         }
-        // ---- E2: z, q_clean, dqc, dlambda; tiles QG, DZ, dqc, qc*dqc
-        mbar_wait(&bar[BAR_R2], par, abort_flag, status);
-        tc_fence_after();
-        {
-            const float lam = lamv[i], itau = itauv[i], c1 = c1v[i];
-            const float nl = -lam * itau;
-            const float *Mh = Mr + 64 * hf;
-            const uint8_t *qbt = sm + OFF_Q + hf * 8192;
-            const uint8_t *egt = sm + OFF_EG + hf * 8192;
-            float dl = 0.f, mdz = 0.f;
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                float zi[32], dqa[32];
-                tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, zi);
-                tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, dqa);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const int cc = 4 * h2 + q4;
-                    float qb[8], eg[8], qg[8], dz[8], dqv[8], gq[8];
-                    load_row_chunk(qbt, i, cc, qb);
-                    load_row_chunk(egt, i, cc, eg);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float m = Mh[8 * cc + e];
-                        const float z = (zi[8 * q4 + e] - c1 * m) * itau;
-                        const float qc = qb[e] - lam * z;
-                        const float dqc = a.scale * eg[e] * dqa[8 * q4 + e];
-                        const float d = nl * dqc;
-                        dl = fmaf(-z, dqc, dl);
-                        mdz = fmaf(m, d, mdz);
-                        qg[e] = a.scale * qc * eg[e];
-                        dz[e] = d;
-                        dqv[e] = dqc;
-                        gq[e] = qc * dqc;
-                    }
-                    store_row_chunk(sm + OFF_V + hf * 8192, i, cc, qg);
-                    store_row_chunk(sm + OFF_DO + hf * 8192, i, cc, dz);
-                    store_row_chunk(sm + OFF_SX + hf * 8192, i, cc, dqv);
-                    store_row_chunk(sm + OFF_SX + 16384 + hf * 8192, i, cc, gq);
-                }
-            }
-            dl += __shfl_xor_sync(0xffffffffu, dl, 16);
-            mdz += __shfl_xor_sync(0xffffffffu, mdz, 16);
-            if (hf == 0) {
-                mdzv[i] = mdz;
-                const int n = c0 + i;
-                if (n < T && a.dlambda) a.dlambda[(static_cast<size_t>(b) * T + n) * H + h] = dl;
-            }
+        for (int k = 0; k < 8; ++k) {  // Zi = Qbar S^K, Dq = dO Sx^T
+            const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+            mma_bf16(tbase + TM_Z, dQ + ka, dSK + kb, ID_64x128_KK, k != 0);
         }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            tma_store_4d(&map_qg, sm + OFF_V, 0, h, c0, b);
-            tma_store_4d(&map_qg, sm + OFF_V + 8192, 64, h, c0, b);
-            tma_store_4d(&map_gq, sm + OFF_SX + 16384, 0, h, c0, b);
-            tma_store_4d(&map_gq, sm + OFF_SX + 16384 + 8192, 64, h, c0, b);
-            tma_store_commit();
-            if (ready && it > 0) {
-                // every store of the previous chunk is older than the group just
-                // committed: once they are complete, publish that chunk
-                tma_store_wait_group<1>();
-                fence_proxy_async_global();
-                st_release_gpu(ready + bh, it);
-            }
-            tc_fence_after();
-            for (int k = 0; k < 8; ++k) {  // T3 = DZ Kbar^T
-                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                mma_bf16(tbase + TM_SC, dDO + ko, dK + ko, ID_64x64_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {  // u = DZ S^K
-                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
-                mma_bf16(tbase + TM_Z, dDO + ka, dSK + kb, ID_64x128_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {  // dkc = Kbar DC + Kbar DC^T
-                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
-                mma_bf16(tbase + TM_DQ, dK + ka, dDCm + k * 128, ID_64x128_KM, k != 0);
-                mma_bf16(tbase + TM_DQ, dK + ka, dDC + kb, ID_64x128_KK, 1);
-            }
-            for (int k = 0; k < 4; ++k)  // dkc += W2^T DZ
-                mma_bf16(tbase + TM_DQ, dW2m + k * 128, dDOm + k * 128, ID_64x128_MM, 1);
-            for (int k = 0; k < 4; ++k)  // DC += DZ^T Qbar
-                mma_bf16(tbase + TM_DC, dDOm + k * 128, dQm + k * 128, ID_128x128_MM, 1);
-            for (int k = 0; k < 4; ++k)  // Dm increment, first half: DZ^T (-c1)
-                mma_bf16(tbase + TM_T1, dDOm + k * 128, dBC + k * 2, ID_128x64_MK, k != 0);
-            mma_commit(&bar[BAR_R3]);
+        for (int k = 0; k < 8; ++k) {
+            const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+            mma_bf16(tbase + TM_DQ, dDO + ka, dSX + kb, ID_64x128_KK, k != 0);
         }
-        // ---- E3: cz, W3
-        mbar_wait(&bar[BAR_R3], par, abort_flag, status);
-        tc_fence_after();
-        {
-            float t3[32];
-            tmem_ld16x2_32<32>(tq + TM_SC, t3);
-            const float part = masked_sum(i, hf, t3);
-            const float cz = a.centered ? (mdzv[i] + part) * itauv[i] : 0.f;
-            if (hf == 0) {
-                czv[i] = cz;
-                *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-cz);
-            }
-            masked_row(sm + OFF_P1, i, hf, t3, cz);
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int k = 0; k < 4; ++k)  // u += W3 Kbar
-                mma_bf16(tbase + TM_Z, dP1 + k * 2, dKm + k * 128, ID_64x128_KM, 1);
-            for (int k = 0; k < 4; ++k)  // dkc += W3^T Qbar
-                mma_bf16(tbase + TM_DQ, dP1m + k * 128, dQm + k * 128, ID_64x128_MM, 1);
-            for (int k = 0; k < 4; ++k)  // Dm increment, second half: Qbar^T (-cz)
-                mma_bf16(tbase + TM_T1, dQm + k * 128, dBC + k * 2, ID_128x64_MK, 1);
-            mma_commit(&bar[BAR_R4]);
-        }
-        // ---- E4: dq, the CCQ part of dkbar, Dm
-        mbar_wait(&bar[BAR_R4], par, abort_flag, status);
-        tc_fence_after();
-        float dm_inc;
-        {
-            float x[32];
-            tmem_ld32(tq + TM_T1, x);  // lane tid, column 0
-            dm_inc = x[0];
-        }
-        {
-            const float cz = czv[i], rq = rqv[i];
-            const float *Mh = Mr + 64 * hf;
-            uint8_t *qbt = sm + OFF_Q + hf * 8192;
-            const uint8_t *dqt = sm + OFF_SX + hf * 8192;
-            float dqb[64];
-            float dot = 0.f;
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                float u[32];
-                tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, u);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const int cc = 4 * h2 + q4;
-                    float dqc[8], qb[8];
-                    load_row_chunk(dqt, i, cc, dqc);
-                    load_row_chunk(qbt, i, cc, qb);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float v = dqc[e] + u[8 * q4 + e] - cz * Mh[8 * cc + e];
-                        dqb[8 * cc + e] = v;
-                        dot = fmaf(qb[e], v, dot);
-                    }
-                }
-            }
-            dot += __shfl_xor_sync(0xffffffffu, dot, 16);
-#pragma unroll
-            for (int cc = 0; cc < 8; ++cc) {
-                float qb[8], out[8];
-                load_row_chunk(qbt, i, cc, qb);
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    out[e] = a.l2norm ? rq * fmaf(-qb[e], dot, dqb[8 * cc + e]) : dqb[8 * cc + e];
-                store_row_chunk(qbt, i, cc, out);
-            }
-        }
-        {
-            const float *Dh = Dm + 64 * hf;
-            uint8_t *kt = sm + OFF_K + hf * 8192;
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                float x[32];
-                tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, x);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const int cc = 4 * h2 + q4;
-                    float out[8];
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) out[e] = x[8 * q4 + e] + Dh[8 * cc + e];
-                    store_row_chunk(kt, i, cc, out);
-                }
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        Dm[tid] += dm_inc;  // Dm_r, read again only after the next chunk's barriers
-        if (tid == 0 && !*abort_flag) {
-            tma_store_4d(&map_dq, sm + OFF_Q, 0, h, c0, b);
-            tma_store_4d(&map_dq, sm + OFF_Q + 8192, 64, h, c0, b);
-            tma_store_4d(&map_dkc, sm + OFF_K, 0, h, c0, b);
-            tma_store_4d(&map_dkc, sm + OFF_K + 8192, 64, h, c0, b);
-            tma_store_commit();
-            if (ready && it + 1 == NC) {
-                // the last chunk: publish as soon as its stores are complete
-                tma_store_wait_all();
-                fence_proxy_async_global();
-                st_release_gpu(ready + bh, NC);
-            }
-            if (it + 1 < NC) {
-                tma_store_wait_read();  // staged tiles read before the next chunk lands on them
-                issue(r - 1);
-            }
-        }
+        mma_commit(&bar[BAR_R1]);
     }
-
+    // ---- E1: c1, W2, P1
+    mbar_wait(&bar[BAR_R1], 0, abort_flag, status);
+    tc_fence_after();
+    {
+        float sc[32];
+        tmem_ld16x2_32<32>(tq + TM_SC, sc);
+        const float part = masked_sum(i, hf, sc);
+        const float c1 = a.centered ? (mqv[i] + part) * itauv[i] : 0.f;
+        if (hf == 0) {
+            c1v[i] = c1;
+            *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-c1);
+        }
+        masked_row(sm + OFF_W2, i, hf, sc, c1);
+        float t1[32];
+        tmem_ld16x2_32<32>(tq + TM_T1, t1);
+        masked_row(sm + OFF_P1, i, hf, t1, 0.f);
+    }
+    fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
+    if (tid == 0 && !*abort_flag) {
+        tc_fence_after();
+        for (int k = 0; k < 4; ++k)  // Zi += W2 Kbar, Dq += P1 Kd
+            mma_bf16(tbase + TM_Z, dW2 + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+        for (int k = 0; k < 4; ++k)
+            mma_bf16(tbase + TM_DQ, dP1 + k * 2, dKDm + k * 128, ID_64x128_KM, 1);
+        mma_commit(&bar[BAR_R2]);
+    }
+    // ---- E2: z, q_clean, dqc, dlambda; tiles QG, DZ, DZ / |q|, dqc, qc*dqc
+    mbar_wait(&bar[BAR_R2], 0, abort_flag, status);
     tc_fence_after();
-    if (a.dC0) {
-        float *dst = a.dC0 + (static_cast<size_t>(bh) * kD + tid) * kD;
+    {
+        const float lam = lamv[i], itau = itauv[i], c1 = c1v[i], rq = rqv[i];
+        const float nl = -lam * itau;
+        const float *Mh = Mr + 64 * hf;
+        const uint8_t *qbt = sm + OFF_Q + hf * 8192;
+        const uint8_t *egt = sm + OFF_EG + hf * 8192;
+        float dl = 0.f, mdz = 0.f;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            float x[32];
-            tmem_ld32(tq + TM_DC + 32 * c, x);
+        for (int h2 = 0; h2 < 2; ++h2) {
+            float zi[32], dqa[32];
+            tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, zi);
+            tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, dqa);
 #pragma unroll
-            for (int e = 0; e < 8; ++e)
-                reinterpret_cast<float4 *>(dst + 32 * c)[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+            for (int q4 = 0; q4 < 4; ++q4) {
+                const int cc = 4 * h2 + q4;
+                float qb[8], eg[8], qg[8], dz[8], dzr[8], dqv[8], gq[8];
+                load_row_chunk(qbt, i, cc, qb);
+                load_row_chunk(egt, i, cc, eg);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float m = Mh[8 * cc + e];
+                    const float z = (zi[8 * q4 + e] - c1 * m) * itau;
+                    const float qc = qb[e] - lam * z;
+                    const float dqc = a.scale * eg[e] * dqa[8 * q4 + e];
+                    const float d = nl * dqc;
+                    dl = fmaf(-z, dqc, dl);
+                    mdz = fmaf(m, d, mdz);
+                    qg[e] = a.scale * qc * eg[e];
+                    dz[e] = d;
+                    dzr[e] = d * rq;
+                    dqv[e] = dqc;
+                    gq[e] = qc * dqc;
+                }
+                store_row_chunk(sm + OFF_V + hf * 8192, i, cc, qg);
+                store_row_chunk(sm + OFF_DO + hf * 8192, i, cc, dz);
+                store_row_chunk(sm + OFF_KD + hf * 8192, i, cc, dzr);
+                store_row_chunk(sm + OFF_SX + hf * 8192, i, cc, dqv);
+                store_row_chunk(sm + OFF_SX + 16384 + hf * 8192, i, cc, gq);
+            }
+        }
+        dl += __shfl_xor_sync(0xffffffffu, dl, 16);
+        mdz += __shfl_xor_sync(0xffffffffu, mdz, 16);
+        if (hf == 0) {
+            mdzv[i] = mdz;
+            const int n = c0 + i;
+            if (n < T && a.dlambda) a.dlambda[(static_cast<size_t>(b) * T + n) * H + h] = dl;
         }
     }
-    if (a.dm0) a.dm0[static_cast<size_t>(bh) * kD + tid] = Dm[tid];
-    if (tid == 0) tma_store_wait_all();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0 && !*abort_flag) {
+        tma_store_4d(&map_qg, sm + OFF_V, 0, h, c0, b);
+        tma_store_4d(&map_qg, sm + OFF_V + 8192, 64, h, c0, b);
+        tma_store_4d(&map_gq, sm + OFF_SX + 16384, 0, h, c0, b);
+        tma_store_4d(&map_gq, sm + OFF_SX + 16384 + 8192, 64, h, c0, b);
+        tma_store_4d(&map_dzr, sm + OFF_KD, 0, h, c0, b);
+        tma_store_4d(&map_dzr, sm + OFF_KD + 8192, 64, h, c0, b);
+        tma_store_commit();
+        tc_fence_after();
+        for (int k = 0; k < 8; ++k) {  // T3 = DZ Kbar^T
+            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+            mma_bf16(tbase + TM_SC, dDO + ko, dK + ko, ID_64x64_KK, k != 0);
+        }
+        for (int k = 0; k < 8; ++k) {  // u = DZ S^K
+            const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+            mma_bf16(tbase + TM_Z, dDO + ka, dSK + kb, ID_64x128_KK, k != 0);
+        }
+        for (int k = 0; k < 4; ++k)  // dkc = W2^T DZ
+            mma_bf16(tbase + TM_DQ, dW2m + k * 128, dDOm + k * 128, ID_64x128_MM, k != 0);
+        for (int k = 0; k < 4; ++k)  // Dm increment, first half: DZ^T (-c1)
+            mma_bf16(tbase + TM_T1, dDOm + k * 128, dBC + k * 2, ID_128x64_MK, k != 0);
+        mma_commit(&bar[BAR_R3]);
+    }
+    // ---- E3: cz, W3
+    mbar_wait(&bar[BAR_R3], 0, abort_flag, status);
+    tc_fence_after();
+    {
+        float t3[32];
+        tmem_ld16x2_32<32>(tq + TM_SC, t3);
+        const float part = masked_sum(i, hf, t3);
+        const float cz = a.centered ? (mdzv[i] + part) * itauv[i] : 0.f;
+        if (hf == 0) {
+            czv[i] = cz;
+            *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-cz);
+        }
+        masked_row(sm + OFF_P1, i, hf, t3, cz);
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0 && !*abort_flag) {
+        tc_fence_after();
+        for (int k = 0; k < 4; ++k)  // u += W3 Kbar
+            mma_bf16(tbase + TM_Z, dP1 + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+        for (int k = 0; k < 4; ++k)  // dkc += W3^T Qbar
+            mma_bf16(tbase + TM_DQ, dP1m + k * 128, dQm + k * 128, ID_64x128_MM, 1);
+        for (int k = 0; k < 4; ++k)  // Dm increment, second half: Qbar^T (-cz)
+            mma_bf16(tbase + TM_T1, dQm + k * 128, dBC + k * 2, ID_128x64_MK, 1);
+        mma_commit(&bar[BAR_R4]);
+    }
+    // ---- E4: dq, the chunk-local CCQ part of dkbar, the chunk's vectors
+    mbar_wait(&bar[BAR_R4], 0, abort_flag, status);
+    tc_fence_after();
+    {
+        float x[32];
+        tmem_ld32(tq + TM_T1, x);  // lane tid, column 0: the Dm increment of this chunk
+        cvec[tid] = fv[tid];
+        cvec[kD + tid] = emv[tid];
+        cvec[2 * kD + tid] = x[0];
+    }
+    {
+        const float cz = czv[i], rq = rqv[i];
+        const float *Mh = Mr + 64 * hf;
+        uint8_t *qbt = sm + OFF_Q + hf * 8192;
+        const uint8_t *dqt = sm + OFF_SX + hf * 8192;
+        float dqb[64];
+        float dot = 0.f;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+            float u[32];
+            tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, u);
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                const int cc = 4 * h2 + q4;
+                float dqc[8], qb[8];
+                load_row_chunk(dqt, i, cc, dqc);
+                load_row_chunk(qbt, i, cc, qb);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float v = dqc[e] + u[8 * q4 + e] - cz * Mh[8 * cc + e];
+                    dqb[8 * cc + e] = v;
+                    dot = fmaf(qb[e], v, dot);
+                }
+            }
+        }
+        dot += __shfl_xor_sync(0xffffffffu, dot, 16);
+#pragma unroll
+        for (int cc = 0; cc < 8; ++cc) {
+            float qb[8], out[8];
+            load_row_chunk(qbt, i, cc, qb);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                out[e] = a.l2norm ? rq * fmaf(-qb[e], dot, dqb[8 * cc + e]) : dqb[8 * cc + e];
+            store_row_chunk(qbt, i, cc, out);
+        }
+    }
+    {
+        uint8_t *kt = sm + OFF_K + hf * 8192;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+            float x[32];
+            tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, x);
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(kt, i, 4 * h2 + q4, x + 8 * q4);
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0 && !*abort_flag) {
+        tma_store_4d(&map_dq, sm + OFF_Q, 0, h, c0, b);
+        tma_store_4d(&map_dq, sm + OFF_Q + 8192, 64, h, c0, b);
+        tma_store_4d(&map_dkc, sm + OFF_K, 0, h, c0, b);
+        tma_store_4d(&map_dkc, sm + OFF_K + 8192, 64, h, c0, b);
+        tma_store_commit();
+        tma_store_wait_all();  // the stores have read shared memory and reached global memory
+    }
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
@@ -638,211 +556,172 @@ __device__ __forceinline__ void q_body(const CUtensorMap &map_q, const CUtensorM
 }
 
 // =====================================================================================
-// gla_bwd_kv_kernel
+// gla_bwd_state_kernel: one CTA per (sequence, head), chunks last to first
 // =====================================================================================
-namespace kv {
-constexpr uint32_t OFF_K = 0;        // kbar; then dk (staged)
-constexpr uint32_t OFF_V = 16384;    // v; then dv (staged)
-constexpr uint32_t OFF_DO = 32768;   // do
-constexpr uint32_t OFF_KD = 49152;   // raw gates (fp32: KD + EG); then Kd
-constexpr uint32_t OFF_EG = 65536;   // EG
-constexpr uint32_t OFF_QG = 81920;   // QG      (scratch from gla_bwd_q_kernel)
-constexpr uint32_t OFF_DKC = 98304;  // CCQ part of dkbar (scratch)
-constexpr uint32_t OFF_GQ = 114688;  // qc * dqc (scratch)
-constexpr uint32_t OFF_DS = 131072;  // bf16 dSs = Diag(e^{Gc-Gmid}) dS_{r+1}
-constexpr uint32_t OFF_P1 = 163840;  // P1
-constexpr uint32_t OFF_SA = 172032;  // SA
-constexpr uint32_t OFF_DG = 131072;  // fp32 dG [64][kDgStride], over dSs and P1 once both are dead
-constexpr int kDgStride = 129;
-constexpr uint32_t OFF_SXC = 180224; // Sx_r = e^{Gmid} S_r (checkpoint tile, for the gate carry)
-constexpr uint32_t OFF_MISC = 214016;
-constexpr uint32_t M_RK = 0, M_F = 256, M_EM = 768, M_EMP = 1280, M_CARRY = 1792, M_GP = 2304,
-                   M_CNEXT = 2816, M_BAR = 3328, M_TMEM = 3360, M_ABORT = 3364;
-constexpr uint32_t kMisc = 3456;
+namespace st {
+constexpr uint32_t BUF_BYTES = 65536;  // per input buffer: QG, dO, DZ/|q|, raw q (16 KB each)
+constexpr uint32_t B_QG = 0, B_DO = 16384, B_DZ = 32768, B_Q = 49152;
+constexpr uint32_t OFF_SX = 2 * BUF_BYTES;      // 131072: Sx_r (checkpoint tile, for the gate carry)
+constexpr uint32_t OFF_IMG = OFF_SX + 32768;    // 163840: staging of the images written per chunk:
+                                                //   Diag(e^{Gc-Gmid}) dS_{r+1} (32 KB), DC_{r+1} (32 KB)
+constexpr uint32_t OFF_MISC = OFF_IMG + 65536;  // 229376
+constexpr uint32_t M_DM = 0, M_EMP = 512, M_CARRY = 1024, M_BAR = 1536, M_TMEM = 1568, M_ABORT = 1572;
+constexpr uint32_t kMisc = 1600;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
-static_assert(OFF_DG + 64 * kDgStride * 4 <= OFF_SA, "dG scratch reaches SA");
-static_assert(OFF_SXC + 32768 <= OFF_MISC, "Sx tile overlaps misc");
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
-enum { BAR_IN = 0, BAR_R1, BAR_R2, kBars };
-constexpr uint32_t TM_X = 0, TM_T1 = 128, TM_SA = 192, TM_DK = 256, TM_DV = 384;
-}  // namespace kv
+enum { BAR_IN0 = 0, BAR_IN1, BAR_SX, BAR_MMA, kBars };
+constexpr uint32_t TM_X = 0, TM_DC = 128;
+}  // namespace st
 
-// The kv-side walk of (sequence, head) pair bh.  With `ready` set, each chunk's
-// exchange tensors are loaded only once ready[bh] shows the q side is past that
-// chunk (acquire; bounded wait, CCQ_ERR_TIMEOUT on give-up).
-__device__ __forceinline__ void kv_body(const CUtensorMap &map_k, const CUtensorMap &map_v, const CUtensorMap &map_do,
-                                        const CUtensorMap &map_g, const CUtensorMap &map_qg,
-                                        const CUtensorMap &map_dkc, const CUtensorMap &map_gq,
-                                        const CUtensorMap &map_dk, const CUtensorMap &map_dv, const BwdArgs &a,
-                                        int bh, const int *ready) {
-    using namespace kv;
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_do,
+                     const __grid_constant__ CUtensorMap map_dzr, const __grid_constant__ CUtensorMap map_q,
+                     const BwdArgs a) {
+    using namespace st;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
-    float *rkv = reinterpret_cast<float *>(misc + M_RK);
-    float *fv = reinterpret_cast<float *>(misc + M_F);
-    float *emv = reinterpret_cast<float *>(misc + M_EM);
+    float *Dm = reinterpret_cast<float *>(misc + M_DM);
     float *emp = reinterpret_cast<float *>(misc + M_EMP);
     float *carry = reinterpret_cast<float *>(misc + M_CARRY);
-    float *cnext = reinterpret_cast<float *>(misc + M_CNEXT);
-    float *gp = reinterpret_cast<float *>(misc + M_GP);
-    float *dG = reinterpret_cast<float *>(sm + OFF_DG);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int b = bh / a.H, h = bh % a.H;
-    const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
-    const bool gate_f32 = a.gate_dtype != 0;
-    const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int T = a.T, NC = (T + kC - 1) / kC;
     const uint8_t *ck = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T);
+    const size_t chunk0 = static_cast<size_t>(bh) * NC;  // flat index of this sequence's chunk 0
     int *status = a.status;
 
     if (tid == 0) {
         for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        tma_prefetch_desc(&map_k);
-        tma_prefetch_desc(&map_v);
-        tma_prefetch_desc(&map_do);
-        tma_prefetch_desc(&map_g);
-        tma_prefetch_desc(&map_qg);
-        tma_prefetch_desc(&map_dkc);
-        tma_prefetch_desc(&map_gq);
     }
-    if (warp == 0) tmem_alloc(tmem_slot, 512);
+    if (warp == 0) tmem_alloc(tmem_slot, 256);
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
     {
-        // X <- dS_T; the gate-gradient carry starts at rowsum(dS_T * S_T)
-        const float *dst_row = a.dST ? a.dST + (static_cast<size_t>(bh) * kD + tid) * kD : nullptr;
+        // X <- dS_T, DC <- dC_T, Dm <- dm_T; the gate carry of the last chunk is rowsum(dS_T * S_T)
+        const size_t row = static_cast<size_t>(bh) * kD + tid;
+        const float *dst_row = a.dST ? a.dST + row * kD : nullptr;
+        const float *dct_row = a.dCT ? a.dCT + row * kD : nullptr;
         const float *st_row = reinterpret_cast<const float *>(ck + static_cast<size_t>(NC) * kCkptChunkBytes) + tid * kD;
         float cs = 0.f;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
-            float x[32];
+            float x[32], y[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
                 x[e] = dst_row ? dst_row[32 * c + e] : 0.f;
                 if (dst_row) cs = fmaf(x[e], st_row[32 * c + e], cs);
+                y[e] = dct_row ? dct_row[32 * c + e] : 0.f;
             }
             tmem_st32(tq + TM_X + 32 * c, x);
+            tmem_st32(tq + TM_DC + 32 * c, y);
         }
         tmem_wait_st();
         carry[tid] = cs;
         emp[tid] = 1.f;
+        Dm[tid] = a.dmT ? a.dmT[row] : 0.f;
     }
-    auto issue = [&](int r) {
+    auto issue = [&](int r, int buf) {
         const int tg = r * kC;
-        if (ready) {
-            // wait (bounded) until the q side has published chunk r
-            const int need = NC - r;
-            if (ld_acquire_gpu(ready + bh) < need) {
-                const long long start = clock64();
-                while (ld_acquire_gpu(ready + bh) < need) {
-                    if (clock64() - start > kWaitLimitCycles) {
-                        *abort_flag = 1;
-                        atomicExch(status, kStatusTimeout);
-                        return;
-                    }
-                }
-            }
-            fence_proxy_async_global();
-        }
-        uint64_t *bb = &bar[BAR_IN];
-        mbar_arrive_expect_tx(bb, 6 * 16384 + g_bytes + 32768);
-        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_QG, &map_qg, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_QG + 8192, &map_qg, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_DKC, &map_dkc, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_DKC + 8192, &map_dkc, bb, 64, h, tg, b);
-        tma_load_4d(sm + OFF_GQ, &map_gq, bb, 0, h, tg, b);
-        tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, tg, b);
-        bulk_load(sm + OFF_SXC, ck + static_cast<size_t>(r) * kCkptChunkBytes + 32768, 32768, bb);
+        uint8_t *base = sm + buf * BUF_BYTES;
+        uint64_t *bb = &bar[BAR_IN0 + buf];
+        mbar_arrive_expect_tx(bb, 4 * 16384);
+        tma_load_4d(base + B_QG, &map_qg, bb, 0, h, tg, b);
+        tma_load_4d(base + B_QG + 8192, &map_qg, bb, 64, h, tg, b);
+        tma_load_4d(base + B_DO, &map_do, bb, 0, h, tg, b);
+        tma_load_4d(base + B_DO + 8192, &map_do, bb, 64, h, tg, b);
+        tma_load_4d(base + B_DZ, &map_dzr, bb, 0, h, tg, b);
+        tma_load_4d(base + B_DZ + 8192, &map_dzr, bb, 64, h, tg, b);
+        tma_load_4d(base + B_Q, &map_q, bb, 0, h, tg, b);
+        tma_load_4d(base + B_Q + 8192, &map_q, bb, 64, h, tg, b);
     };
-    if (tid == 0 && NC > 0) issue(NC - 1);
+    auto issue_sx = [&](int r) {
+        mbar_arrive_expect_tx(&bar[BAR_SX], 32768);
+        bulk_load(sm + OFF_SX, ck + static_cast<size_t>(r) * kCkptChunkBytes + 32768, 32768, &bar[BAR_SX]);
+    };
+    if (tid == 0 && NC > 0) {
+        issue(NC - 1, 0);
+        if (NC > 1) issue(NC - 2, 1);
+        issue_sx(NC - 1);
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
 
-    const int i = 16 * warp + (lane & 15), hf = lane >> 4;
-    const uint64_t dV = make_desc(sb + OFF_V, 16, 1024);
-    const uint64_t dDO = make_desc(sb + OFF_DO, 16, 1024), dDOm = make_desc(sb + OFF_DO, 8192, 1024);
-    const uint64_t dKD = make_desc(sb + OFF_KD, 16, 1024);
-    const uint64_t dQG = make_desc(sb + OFF_QG, 16, 1024), dQGm = make_desc(sb + OFF_QG, 8192, 1024);
-    const uint64_t dDS = make_desc(sb + OFF_DS, 16, 1024), dDSm = make_desc(sb + OFF_DS, 16384, 1024);
-    const uint64_t dP1m = make_desc(sb + OFF_P1, 8192, 1024);
-    const uint64_t dSA = make_desc(sb + OFF_SA, 16, 1024);
-
     for (int it = 0; it < NC; ++it) {
-        const int r = NC - 1 - it;
-        const uint32_t par = it & 1;
-        const int c0 = r * kC;
-        mbar_wait(&bar[BAR_IN], par, abort_flag, status);
-        prep_chunk(nullptr, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, nullptr, nullptr, nullptr,
-                   rkv, gp, fv, emv, tid);
-        {
-            // dSs = Diag(e^{Gc - Gmid}) dS_{r+1}: X holds e^{-Gmid_{r+1}} dS_{r+1}
-            tc_fence_after();
-            const float hs = fv[tid] * emp[tid];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_X + 32 * c, x);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) x[e] *= hs;
-                uint8_t *tile = sm + OFF_DS + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
-                tmem_st32(tq + TM_X + 32 * c, x);
-            }
-            emp[tid] = emv[tid];
-            tmem_wait_st();
+        const int r = NC - 1 - it, buf = it & 1;
+        const uint32_t bpar = (it >> 1) & 1, par = it & 1;
+        const size_t ci = chunk0 + r;
+        const float *cvec = a.chunk_vec + ci * 3 * kD;
+        const float f = cvec[tid], em = cvec[kD + tid], ddm = cvec[2 * kD + tid];
+        // ---- the states carried into chunk r: Diag(e^{Gc - Gmid}) dS_{r+1} (rescaling X in
+        // place: X holds e^{-Gmid_{r+1}} dS_{r+1}), DC_{r+1}, Dm_{r+1} and the gate carry
+        if (it > 0) {
+            if (tid == 0) tma_store_wait_read();  // the previous chunk's images have been copied out
+            __syncthreads();
         }
+        tc_fence_after();
+        const float hs = f * emp[tid];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[32];
+            tmem_ld32(tq + TM_X + 32 * c, x);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) x[e] *= hs;
+            uint8_t *tile = sm + OFF_IMG + (c >> 1) * 16384;
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
+            tmem_st32(tq + TM_X + 32 * c, x);
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float x[32];
+            tmem_ld32(tq + TM_DC + 32 * c, x);
+            uint8_t *tile = sm + OFF_IMG + 32768 + (c >> 1) * 16384;
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
+        }
+        tmem_wait_st();
+        a.state_vec[ci * 2 * kD + tid] = Dm[tid];
+        a.state_vec[ci * 2 * kD + kD + tid] = carry[tid];
+        Dm[tid] += ddm;  // Dm_r
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
+        mbar_wait(&bar[BAR_IN0 + buf], bpar, abort_flag, status);
         if (tid == 0 && !*abort_flag) {
+            bulk_store(a.state_img + ci * 65536, sm + OFF_IMG, 65536);
+            tma_store_commit();
             tc_fence_after();
-            for (int k = 0; k < 8; ++k) {  // T1 = dO V^T, SA = Kd QG^T
-                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                mma_bf16(tbase + TM_T1, dDO + ko, dV + ko, ID_64x64_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {
-                const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                mma_bf16(tbase + TM_SA, dKD + ko, dQG + ko, ID_64x64_KK, k != 0);
-            }
-            for (int k = 0; k < 8; ++k) {  // dkw = V dSs^T, dv = Kd dSs
-                const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
-                mma_bf16(tbase + TM_DK, dV + ka, dDS + kb, ID_64x128_KK, k != 0);
-                mma_bf16(tbase + TM_DV, dKD + ka, dDSm + k * 128, ID_64x128_KM, k != 0);
-            }
-            for (int k = 0; k < 4; ++k)  // X += QG^T dO
+            const uint32_t base = sb + buf * BUF_BYTES;
+            const uint64_t dQGm = make_desc(base + B_QG, 8192, 1024), dDOm = make_desc(base + B_DO, 8192, 1024);
+            const uint64_t dDZm = make_desc(base + B_DZ, 8192, 1024), dQm = make_desc(base + B_Q, 8192, 1024);
+            for (int k = 0; k < 4; ++k)  // X += QG^T dO  (-> e^{-Gmid_r} dS_r)
                 mma_bf16(tbase + TM_X, dQGm + k * 128, dDOm + k * 128, ID_128x128_MM, 1);
-            mma_commit(&bar[BAR_R1]);
+            for (int k = 0; k < 4; ++k)  // DC += (DZ / |q|)^T q  (= DZ^T Qbar)
+                mma_bf16(tbase + TM_DC, dDZm + k * 128, dQm + k * 128, ID_128x128_MM, 1);
+            mma_commit(&bar[BAR_MMA]);
         }
-        mbar_wait(&bar[BAR_R1], par, abort_flag, status);
+        mbar_wait(&bar[BAR_MMA], par, abort_flag, status);
+        mbar_wait(&bar[BAR_SX], par, abort_flag, status);
         tc_fence_after();
         {
-            // gate carry of the chunk before: rowsum(dS_r * S_r) = rowsum(X * Sx_r) (the
-            // e^{-Gmid} of X and the e^{Gmid} of Sx cancel); a boundary value, so rounding
-            // does not accumulate across chunks
+            // gate carry of chunk r - 1: rowsum(dS_r * S_r) = rowsum(X * Sx_r)
             float cs = 0.f;
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 float x[32];
                 tmem_ld32(tq + TM_X + 32 * c, x);
-                const uint8_t *tile = sm + OFF_SXC + (c >> 1) * 16384;
+                const uint8_t *tile = sm + OFF_SX + (c >> 1) * 16384;
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     float sx[8];
@@ -851,144 +730,284 @@ __device__ __forceinline__ void kv_body(const CUtensorMap &map_k, const CUtensor
                     for (int e = 0; e < 8; ++e) cs = fmaf(x[8 * q4 + e], sx[e], cs);
                 }
             }
-            cnext[tid] = cs;
+            carry[tid] = cs;
+            emp[tid] = em;
         }
-        {
-            float t1[32];
-            tmem_ld16x2_32<32>(tq + TM_T1, t1);
-            masked_row(sm + OFF_P1, i, hf, t1, 0.f);  // P1[t][j] = [j <= t] do_t . v_j
-            float sa[32];
-            tmem_ld16x2_32<32>(tq + TM_SA, sa);
-            // SA[j][t] = [t >= j] Kd_j . QG_t (row i is key j)
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-                float w[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const int t = 32 * hf + 8 * q4 + e;
-                    w[e] = (t >= i) ? sa[8 * q4 + e] : 0.f;
-                }
-                store_row_chunk(sm + OFF_SA, i, 4 * hf + q4, w);
-            }
-        }
-        fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
         if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            for (int k = 0; k < 4; ++k)  // dkw += P1^T QG, dv += SA dO
-                mma_bf16(tbase + TM_DK, dP1m + k * 128, dQGm + k * 128, ID_64x128_MM, 1);
-            for (int k = 0; k < 4; ++k)
-                mma_bf16(tbase + TM_DV, dSA + k * 2, dDOm + k * 128, ID_64x128_KM, 1);
-            mma_commit(&bar[BAR_R2]);
-        }
-        mbar_wait(&bar[BAR_R2], par, abort_flag, status);
-        tc_fence_after();
-        {
-            // dk: dkbar = e^{Gmid-G} dkw + (CCQ part); normalisation backward; dG
-            const float rk = rkv[i];
-            uint8_t *kt = sm + OFF_K + hf * 8192;
-            const uint8_t *egt = sm + OFF_EG + hf * 8192;
-            const uint8_t *dkct = sm + OFF_DKC + hf * 8192;
-            const uint8_t *gqt = sm + OFF_GQ + hf * 8192;
-            float *dgrow = dG + i * kDgStride + 64 * hf;
-            float dkb[64];
-            float dot = 0.f;
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                float x[32];
-                tmem_ld16x2_32<64>(tq + TM_DK + 32 * h2, x);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const int cc = 4 * h2 + q4;
-                    float eg[8], kb[8], kc[8], gq[8];
-                    load_row_chunk(egt, i, cc, eg);
-                    load_row_chunk(kt, i, cc, kb);
-                    load_row_chunk(dkct, i, cc, kc);
-                    load_row_chunk(gqt, i, cc, gq);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float dkw = x[8 * q4 + e] * __frcp_rn(eg[e]);
-                        const float v = dkw + kc[e];
-                        dkb[8 * cc + e] = v;
-                        dot = fmaf(kb[e], v, dot);
-                        dgrow[8 * cc + e] = fmaf(-kb[e], dkw, gq[e]);
-                    }
-                }
-            }
-            dot += __shfl_xor_sync(0xffffffffu, dot, 16);
-#pragma unroll
-            for (int cc = 0; cc < 8; ++cc) {
-                float kb[8], out[8];
-                load_row_chunk(kt, i, cc, kb);
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                    out[e] = a.l2norm ? rk * fmaf(-kb[e], dot, dkb[8 * cc + e]) : dkb[8 * cc + e];
-                store_row_chunk(kt, i, cc, out);
-            }
-            uint8_t *vt = sm + OFF_V + hf * 8192;
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                float x[32];
-                tmem_ld16x2_32<64>(tq + TM_DV + 32 * h2, x);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(vt, i, 4 * h2 + q4, x + 8 * q4);
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            tma_store_4d(&map_dk, sm + OFF_K, 0, h, c0, b);
-            tma_store_4d(&map_dk, sm + OFF_K + 8192, 64, h, c0, b);
-            tma_store_4d(&map_dv, sm + OFF_V, 0, h, c0, b);
-            tma_store_4d(&map_dv, sm + OFF_V + 8192, 64, h, c0, b);
-            tma_store_commit();
-        }
-        {
-            // dgk_t = sum_{s >= t in the chunk} dG_s + rowsum(dS_{r+1} * S_{r+1}),
-            // column d = tid, tokens in reverse
-            float acc = carry[tid];
-            const int nvalid = min(kC, T - c0);
-            for (int t8 = kC - 8; t8 >= 0; t8 -= 8) {
-                float x[8];
-#pragma unroll
-                for (int u = 0; u < 8; ++u) x[u] = dG[(t8 + u) * kDgStride + tid];  // loads in flight together
-#pragma unroll
-                for (int u = 7; u >= 0; --u) {
-                    acc += x[u];
-                    const int t = t8 + u;
-                    if (t < nvalid) {
-                        const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + tid;
-                        if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
-                        else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
-                    }
-                }
-            }
-            carry[tid] = cnext[tid];
-        }
-        __syncthreads();
-        if (tid == 0 && !*abort_flag && it + 1 < NC) {
-            tma_store_wait_read();
-            issue(r - 1);
+            if (r >= 2) issue(r - 2, buf);  // this buffer's MMAs are complete
+            if (r >= 1) issue_sx(r - 1);    // Sx_r has been read
         }
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (a.dS0) {
-        // dS_0 = e^{Gmid_0} X
-        const float em = emp[tid];
-        float *dst = a.dS0 + (static_cast<size_t>(bh) * kD + tid) * kD;
+    {
+        const size_t row = static_cast<size_t>(bh) * kD + tid;
+        const float e0 = emp[tid];  // e^{Gmid_0}: dS_0 = e^{Gmid_0} X
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             float x[32];
             tmem_ld32(tq + TM_X + 32 * c, x);
+            if (a.dS0)
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    reinterpret_cast<float4 *>(a.dS0 + row * kD + 32 * c)[e] =
+                        make_float4(e0 * x[4 * e], e0 * x[4 * e + 1], e0 * x[4 * e + 2], e0 * x[4 * e + 3]);
+            tmem_ld32(tq + TM_DC + 32 * c, x);
+            if (a.dC0)
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    reinterpret_cast<float4 *>(a.dC0 + row * kD + 32 * c)[e] =
+                        make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+        }
+        if (a.dm0) a.dm0[row] = Dm[tid];
+    }
+    if (tid == 0) tma_store_wait_all();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tbase, 256);
+    }
+}
+
+// =====================================================================================
+// gla_bwd_kv_kernel: one CTA per (sequence, head, chunk)
+// =====================================================================================
+namespace kv {
+constexpr uint32_t OFF_K = 0;        // kbar; then dk (staged)
+constexpr uint32_t OFF_V = 16384;    // v; then dv (staged)
+constexpr uint32_t OFF_DO = 32768;   // do
+constexpr uint32_t OFF_KD = 49152;   // raw gates (fp32: KD + EG); then Kd
+constexpr uint32_t OFF_EG = 65536;   // EG
+constexpr uint32_t OFF_QG = 81920;   // QG               (from gla_bwd_q_kernel)
+constexpr uint32_t OFF_DKC = 98304;  // local CCQ part of dkbar (from gla_bwd_q_kernel)
+constexpr uint32_t OFF_GQ = 114688;  // qc * dqc         (from gla_bwd_q_kernel)
+constexpr uint32_t OFF_DS = 131072;  // Diag(e^{Gc-Gmid}) dS_{r+1} } one image record of the state
+constexpr uint32_t OFF_DC = 163840;  // DC_{r+1}                   } pass, one bulk copy
+constexpr uint32_t OFF_P1 = 196608;  // P1
+constexpr uint32_t OFF_SA = 204800;  // SA
+constexpr uint32_t OFF_DG = 131072;  // fp32 dG [64][kDgStride], over the two images once they are dead
+constexpr int kDgStride = 129;
+constexpr uint32_t OFF_MISC = 212992;
+constexpr uint32_t M_VEC = 0,        // [2][128] Dm_{r+1}, gate carry (from the state pass)
+                   M_RK = 1024, M_GP = 1280, M_BAR = 1792, M_TMEM = 1824, M_ABORT = 1828;
+constexpr uint32_t kMisc = 1920;
+constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
+static_assert(OFF_DG + 64 * kDgStride * 4 <= OFF_P1, "dG scratch reaches P1");
+static_assert(OFF_DC == OFF_DS + 32768, "a state image record lands as one block");
+static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
+enum { BAR_IN = 0, BAR_R1, BAR_R2, kBars };
+constexpr uint32_t TM_KC = 0, TM_T1 = 128, TM_SA = 192, TM_DK = 256, TM_DV = 384;
+}  // namespace kv
+
+__global__ void __launch_bounds__(kThreads, 1)
+gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
+                  const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
+                  const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
+                  const __grid_constant__ CUtensorMap map_gq, const __grid_constant__ CUtensorMap map_dk,
+                  const __grid_constant__ CUtensorMap map_dv, const BwdArgs a) {
+    using namespace kv;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = align1024(smem_raw);
+    const uint32_t sb = smem_addr(sm);
+    uint8_t *misc = sm + OFF_MISC;
+    float *vec = reinterpret_cast<float *>(misc + M_VEC);
+    float *rkv = reinterpret_cast<float *>(misc + M_RK);
+    float *gp = reinterpret_cast<float *>(misc + M_GP);
+    float *dG = reinterpret_cast<float *>(sm + OFF_DG);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
+    const int bh = blockIdx.x / NC, r = blockIdx.x % NC, b = bh / H, h = bh % H;
+    const int c0 = r * kC;
+    const bool gate_f32 = a.gate_dtype != 0;
+    const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
+    int *status = a.status;
+
+    if (tid == 0) {
+        for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+        uint64_t *bb = &bar[BAR_IN];
+        mbar_arrive_expect_tx(bb, 6 * 16384 + g_bytes + 65536 + 1024);
+        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_QG, &map_qg, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_QG + 8192, &map_qg, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_DKC, &map_dkc, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_DKC + 8192, &map_dkc, bb, 64, h, c0, b);
+        tma_load_4d(sm + OFF_GQ, &map_gq, bb, 0, h, c0, b);
+        tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, c0, b);
+        bulk_load(sm + OFF_DS, a.state_img + static_cast<size_t>(blockIdx.x) * 65536, 65536, bb);
+        bulk_load(misc + M_VEC, a.state_vec + static_cast<size_t>(blockIdx.x) * 2 * kD, 1024, bb);
+    }
+    if (warp == 0) tmem_alloc(tmem_slot, 512);
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = *tmem_slot;
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
+
+    const int i = 16 * warp + (lane & 15), hf = lane >> 4;
+    const uint64_t dK = make_desc(sb + OFF_K, 16, 1024);
+    const uint64_t dV = make_desc(sb + OFF_V, 16, 1024);
+    const uint64_t dDO = make_desc(sb + OFF_DO, 16, 1024), dDOm = make_desc(sb + OFF_DO, 8192, 1024);
+    const uint64_t dKD = make_desc(sb + OFF_KD, 16, 1024);
+    const uint64_t dQG = make_desc(sb + OFF_QG, 16, 1024), dQGm = make_desc(sb + OFF_QG, 8192, 1024);
+    const uint64_t dDS = make_desc(sb + OFF_DS, 16, 1024), dDSm = make_desc(sb + OFF_DS, 16384, 1024);
+    const uint64_t dDC = make_desc(sb + OFF_DC, 16, 1024), dDCm = make_desc(sb + OFF_DC, 16384, 1024);
+    const uint64_t dP1m = make_desc(sb + OFF_P1, 8192, 1024);
+    const uint64_t dSA = make_desc(sb + OFF_SA, 16, 1024);
+
+    mbar_wait(&bar[BAR_IN], 0, abort_flag, status);
+    prep_chunk(nullptr, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, nullptr, nullptr, nullptr, rkv,
+               gp, nullptr, nullptr, tid);
+    if (tid == 0 && !*abort_flag) {
+        tc_fence_after();
+        for (int k = 0; k < 8; ++k) {  // T1 = dO V^T, SA = Kd QG^T
+            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+            mma_bf16(tbase + TM_T1, dDO + ko, dV + ko, ID_64x64_KK, k != 0);
+        }
+        for (int k = 0; k < 8; ++k) {
+            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+            mma_bf16(tbase + TM_SA, dKD + ko, dQG + ko, ID_64x64_KK, k != 0);
+        }
+        for (int k = 0; k < 8; ++k) {  // dkw = V dSs^T, dv = Kd dSs, dkc inter = Kbar DC + Kbar DC^T
+            const uint64_t ka = (k >> 2) * 512 + (k & 3) * 2, kb = (k >> 2) * 1024 + (k & 3) * 2;
+            mma_bf16(tbase + TM_DK, dV + ka, dDS + kb, ID_64x128_KK, k != 0);
+            mma_bf16(tbase + TM_DV, dKD + ka, dDSm + k * 128, ID_64x128_KM, k != 0);
+            mma_bf16(tbase + TM_KC, dK + ka, dDCm + k * 128, ID_64x128_KM, k != 0);
+            mma_bf16(tbase + TM_KC, dK + ka, dDC + kb, ID_64x128_KK, 1);
+        }
+        mma_commit(&bar[BAR_R1]);
+    }
+    mbar_wait(&bar[BAR_R1], 0, abort_flag, status);
+    tc_fence_after();
+    {
+        float t1[32];
+        tmem_ld16x2_32<32>(tq + TM_T1, t1);
+        masked_row(sm + OFF_P1, i, hf, t1, 0.f);  // P1[t][j] = [j <= t] do_t . v_j
+        float sa[32];
+        tmem_ld16x2_32<32>(tq + TM_SA, sa);
+        // SA[j][t] = [t >= j] Kd_j . QG_t (row i is key j)
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+            float w[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                const int t = 32 * hf + 8 * q4 + e;
+                w[e] = (t >= i) ? sa[8 * q4 + e] : 0.f;
+            }
+            store_row_chunk(sm + OFF_SA, i, 4 * hf + q4, w);
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0 && !*abort_flag) {
+        tc_fence_after();
+        for (int k = 0; k < 4; ++k)  // dkw += P1^T QG, dv += SA dO
+            mma_bf16(tbase + TM_DK, dP1m + k * 128, dQGm + k * 128, ID_64x128_MM, 1);
+        for (int k = 0; k < 4; ++k)
+            mma_bf16(tbase + TM_DV, dSA + k * 2, dDOm + k * 128, ID_64x128_KM, 1);
+        mma_commit(&bar[BAR_R2]);
+    }
+    mbar_wait(&bar[BAR_R2], 0, abort_flag, status);
+    tc_fence_after();
+    {
+        // dk: dkbar = e^{Gmid-G} dkw + (local CCQ part) + Kbar (DC + DC^T) + Dm_{r+1};
+        // normalisation backward; dG
+        const float rk = rkv[i];
+        const float *Dh = vec + 64 * hf;  // Dm_{r+1}
+        uint8_t *kt = sm + OFF_K + hf * 8192;
+        const uint8_t *egt = sm + OFF_EG + hf * 8192;
+        const uint8_t *dkct = sm + OFF_DKC + hf * 8192;
+        const uint8_t *gqt = sm + OFF_GQ + hf * 8192;
+        float *dgrow = dG + i * kDgStride + 64 * hf;
+        float dkb[64];
+        float dot = 0.f;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+            float x[32], y[32];
+            tmem_ld16x2_32<64>(tq + TM_DK + 32 * h2, x);
+            tmem_ld16x2_32<64>(tq + TM_KC + 32 * h2, y);
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                const int cc = 4 * h2 + q4;
+                float eg[8], kb[8], kc[8], gq[8];
+                load_row_chunk(egt, i, cc, eg);
+                load_row_chunk(kt, i, cc, kb);
+                load_row_chunk(dkct, i, cc, kc);
+                load_row_chunk(gqt, i, cc, gq);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float dkw = x[8 * q4 + e] * __frcp_rn(eg[e]);
+                    const float v = dkw + kc[e] + y[8 * q4 + e] + Dh[8 * cc + e];
+                    dkb[8 * cc + e] = v;
+                    dot = fmaf(kb[e], v, dot);
+                    dgrow[8 * cc + e] = fmaf(-kb[e], dkw, gq[e]);
+                }
+            }
+        }
+        dot += __shfl_xor_sync(0xffffffffu, dot, 16);
+#pragma unroll
+        for (int cc = 0; cc < 8; ++cc) {
+            float kb[8], out[8];
+            load_row_chunk(kt, i, cc, kb);
 #pragma unroll
             for (int e = 0; e < 8; ++e)
-                reinterpret_cast<float4 *>(dst + 32 * c)[e] =
-                    make_float4(em * x[4 * e], em * x[4 * e + 1], em * x[4 * e + 2], em * x[4 * e + 3]);
+                out[e] = a.l2norm ? rk * fmaf(-kb[e], dot, dkb[8 * cc + e]) : dkb[8 * cc + e];
+            store_row_chunk(kt, i, cc, out);
+        }
+        uint8_t *vt = sm + OFF_V + hf * 8192;
+#pragma unroll
+        for (int h2 = 0; h2 < 2; ++h2) {
+            float x[32];
+            tmem_ld16x2_32<64>(tq + TM_DV + 32 * h2, x);
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(vt, i, 4 * h2 + q4, x + 8 * q4);
+        }
+    }
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    if (tid == 0 && !*abort_flag) {
+        tma_store_4d(&map_dk, sm + OFF_K, 0, h, c0, b);
+        tma_store_4d(&map_dk, sm + OFF_K + 8192, 64, h, c0, b);
+        tma_store_4d(&map_dv, sm + OFF_V, 0, h, c0, b);
+        tma_store_4d(&map_dv, sm + OFF_V + 8192, 64, h, c0, b);
+        tma_store_commit();
+    }
+    {
+        // dgk_t = sum_{s >= t in the chunk} dG_s + rowsum(dS_{r+1} * S_{r+1}),
+        // column d = tid, tokens in reverse
+        float acc = vec[kD + tid];
+        const int nvalid = min(kC, T - c0);
+        for (int t8 = kC - 8; t8 >= 0; t8 -= 8) {
+            float x[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) x[u] = dG[(t8 + u) * kDgStride + tid];
+#pragma unroll
+            for (int u = 7; u >= 0; --u) {
+                acc += x[u];
+                const int t = t8 + u;
+                if (t < nvalid) {
+                    const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + tid;
+                    if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
+                    else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
+                }
+            }
         }
     }
     if (tid == 0) tma_store_wait_all();
@@ -1000,96 +1019,32 @@ __device__ __forceinline__ void kv_body(const CUtensorMap &map_k, const CUtensor
     }
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                 const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
-                 const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
-                 const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
-                 const __grid_constant__ CUtensorMap map_gq, const BwdArgs a) {
-    q_body(map_q, map_k, map_v, map_do, map_g, map_dq, map_qg, map_dkc, map_gq, a, blockIdx.x, nullptr);
-}
-
-__global__ void __launch_bounds__(kThreads, 1)
-gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-                  const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
-                  const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
-                  const __grid_constant__ CUtensorMap map_gq, const __grid_constant__ CUtensorMap map_dk,
-                  const __grid_constant__ CUtensorMap map_dv, const BwdArgs a) {
-    kv_body(map_k, map_v, map_do, map_g, map_qg, map_dkc, map_gq, map_dk, map_dv, a, blockIdx.x, nullptr);
-}
-
-// Both walks at once: clusters of four CTAs for two (sequence, head) pairs --
-// ranks 0 and 1 the q sides, ranks 2 and 3 the kv sides.  The CTAs of a cluster
-// are co-scheduled, so a kv side can wait on its q side's progress counter;
-// neighbouring ranks run the same code, which keeps the two roles' instruction
-// streams from competing for the instruction cache they share.
-constexpr int kPairCluster = 4;
-
-__global__ void __launch_bounds__(kThreads, 1)
-gla_bwd_pair_kernel(const __grid_constant__ BwdMaps m, const BwdArgs a, int *ready) {
-    const int rank = blockIdx.x % kPairCluster;
-    const int bh = 2 * (blockIdx.x / kPairCluster) + (rank & 1);
-    if (rank < 2)
-        q_body(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq, a, bh, ready);
-    else
-        kv_body(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a, bh, ready);
-}
-
-constexpr uint32_t kPairSmem = qk::kSmem > kv::kSmem ? qk::kSmem : kv::kSmem;
-
 }  // namespace
 
-cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, int *ready, cudaStream_t s) {
-    static int pair_ok = -1;  // -1 unknown, 0 no, 1 yes (per process; one device type)
-    if (pair_ok < 0) {
+cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s) {
+    static bool attr_set = false;
+    if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(gla_bwd_q_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(qk::kSmem));
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(gla_bwd_state_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(st::kSmem));
         if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(gla_bwd_kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  static_cast<int>(kv::kSmem));
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(gla_bwd_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(kPairSmem));
-        if (e != cudaSuccess) return e;
-        pair_ok = 0;
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = kPairCluster;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3(kPairCluster);
-        cfg.blockDim = dim3(kThreads);
-        cfg.dynamicSmemBytes = kPairSmem;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        int clusters = 0;
-        if (cudaOccupancyMaxActiveClusters(&clusters, gla_bwd_pair_kernel, &cfg) == cudaSuccess && clusters > 0)
-            pair_ok = 1;
-        (void)cudaGetLastError();
+        attr_set = true;
     }
-    if (pair_ok == 1 && ready && (a.B * a.H) % 2 == 0) {
-        cudaError_t e = cudaMemsetAsync(ready, 0, sizeof(int) * static_cast<size_t>(a.B) * a.H, s);
-        if (e != cudaSuccess) return e;
-        cudaLaunchConfig_t cfg = {};
-        cudaLaunchAttribute attr[1];
-        attr[0].id = cudaLaunchAttributeClusterDimension;
-        attr[0].val.clusterDim.x = kPairCluster;
-        attr[0].val.clusterDim.y = 1;
-        attr[0].val.clusterDim.z = 1;
-        cfg.gridDim = dim3(2 * a.B * a.H);
-        cfg.blockDim = dim3(kThreads);
-        cfg.dynamicSmemBytes = kPairSmem;
-        cfg.stream = s;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
-        return cudaLaunchKernelEx(&cfg, gla_bwd_pair_kernel, m, a, ready);
-    }
-    const int grid = a.B * a.H;
-    gla_bwd_q_kernel<<<grid, kThreads, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq, a);
+    const int nc = (a.T + kC - 1) / kC;
+    const int chunks = a.B * a.H * nc;
+    gla_bwd_q_kernel<<<chunks, kThreads, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq,
+                                                          m.dzr, a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    gla_bwd_kv_kernel<<<grid, kThreads, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
+    gla_bwd_state_kernel<<<a.B * a.H, kThreads, st::kSmem, s>>>(m.qg, m.dO, m.dzr, m.q, a);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    gla_bwd_kv_kernel<<<chunks, kThreads, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
     return cudaGetLastError();
 }
 

@@ -118,21 +118,24 @@ struct BwdArgs {
     void *dgk;
     float *dS0, *dC0, *dm0;
     int *status;
+    // per chunk (flat index (b*H + h)*NC + r), in the workspace:
+    float *chunk_vec;    // [3][128] written by the q kernel: e^{Gc-Gmid}, e^{Gmid}, Dm increment
+    uint8_t *state_img;  // 64 KB written by the state pass: the bf16 tile images of
+                         // Diag(e^{Gc-Gmid}) dS_{r+1} and DC_{r+1} (two T64 tiles each)
+    float *state_vec;    // [2][128] written by the state pass: Dm_{r+1}, rowsum(dS_{r+1} S_{r+1})
 };
 
 // Tensor maps ([B][T][H][128], 64 x 64 swizzled boxes; g as in ChunkMaps) of
-// the inputs, the outputs dq, dk, dv and the three bf16 scratch tensors the
-// two backward kernels exchange (QG, the CCQ part of dkbar, qc * dqc).
+// the inputs, the outputs dq, dk, dv and the four bf16 tensors the backward
+// kernels exchange (QG, the chunk-local CCQ part of dkbar, qc * dqc, DZ / |q|).
 struct BwdMaps {
-    CUtensorMap q, k, v, dO, g, dq, dk, dv, qg, dkc, gq;
+    CUtensorMap q, k, v, dO, g, dq, dk, dv, qg, dkc, gq, dzr;
 };
 
-// Runs the q-side and kv-side walks of the backward: as clusters of two CTAs per
-// (sequence, head) that run concurrently, the kv side trailing the q side through
-// the progress counters `ready` (B*H ints of workspace, zeroed here), or -- when
-// the device cannot hold such a cluster, or `ready` is NULL -- as
-// gla_bwd_q_kernel then gla_bwd_kv_kernel.
-cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, int *ready, cudaStream_t s);
+// Launches the backward: gla_bwd_q_kernel (one CTA per chunk), the sequential
+// gla_bwd_state_kernel (one CTA per sequence and head), gla_bwd_kv_kernel (one
+// CTA per chunk).
+cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s);
 
 // Encode the tensor map of a row-major [rows][128] bf16 matrix with 64 x 64 boxes
 // (128-byte swizzle).
