@@ -47,7 +47,8 @@ KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode"
                   "glabwd": "ccq_gla_bwd.cu"}
 KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_kernel",
                 "decode": "decode_kernel",
-                "glabwd": "whole step: forward (saving checkpoints) + gla_bwd_q_kernel + gla_bwd_kv_kernel"}
+                "glabwd": "whole step: forward (saving checkpoints) + gla_bwd_q_kernel + gla_bwd_state_kernel"
+                          " + gla_bwd_kv_kernel"}
 
 
 def gla_segments(B, H, T, sms):
@@ -61,10 +62,10 @@ def gla_segments(B, H, T, sms):
 
 def launches_per_step(kind, B, H, T, sms):
     """Kernel launches of one step: the segmented GLA forward is three kernels,
-    the backward one (its two walks run concurrently), and every call that
+    the backward three, and every call that
     returns the position count adds the one-thread-per-row count update."""
     fwd = 1 if gla_segments(B, H, T, sms) == 1 else 3
-    return {"gla": fwd + 1, "gdn": 2 + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 1}[kind]
+    return {"gla": fwd + 1, "gdn": 2 + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3}[kind]
 
 
 def algorithmic_bytes(kind, B, H, T, D):
@@ -115,13 +116,13 @@ STEP_KERNELS = {
     "gdn_bf16_20k": ["gdn_wy_kernel", "gdn_chunk_kernel"],
     "decode_b256": ["decode_kernel"],
     "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
-                           "gla_bwd_pair_kernel"],
+                           "gla_bwd_q_kernel", "gla_bwd_state_kernel", "gla_bwd_kv_kernel"],
 }
 # (each step also runs the one-thread-per-row position update: 8 bytes per batch row, not counted)
 KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kernel": "ccq_gla_segment.cu",
                 "gla_segment_combine_kernel": "ccq_gla_segment.cu", "gdn_wy_kernel": "ccq_gdn_chunk.cu",
                 "gdn_chunk_kernel": "ccq_gdn_chunk.cu", "recurrent": "ccq_recurrent.cu",
-                "decode_kernel": "ccq_recurrent.cu", "gla_bwd_pair_kernel": "ccq_gla_bwd.cu",
+                "decode_kernel": "ccq_recurrent.cu", "gla_bwd_state_kernel": "ccq_gla_bwd.cu",
                 "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu"}
 
 
