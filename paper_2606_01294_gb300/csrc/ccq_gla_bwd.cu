@@ -46,8 +46,10 @@
 //   gla_bwd_kv_kernel    one CTA per chunk (parallel): dk (write part, the
 //                        CCQ inter term K (DC + DC^T), Dm), dv, dgk.
 // 64-row products are M = 64 MMAs whose rows 16q..16q+15 sit in TMEM lanes
-// 32q..32q+15, so thread (warp w, lane l) owns row 16w + l % 16 and column
-// half l / 16 in every 64-row epilogue; 128-row products (the carried states)
+// 32q..32q+15, so in the chunk-parallel kernels (256 threads, two warps per lane
+// quadrant) thread (warp w, lane l) owns row 16 (w % 4) + l % 16, column half
+// l / 16 of a 64-column load, and -- for 128-column products -- the 32-column
+// slice w / 4 of each half; 128-row products (the carried states, 128 threads)
 // give thread t row t.
 #include <cuda.h>
 #include <cuda_bf16.h>
@@ -63,7 +65,8 @@ namespace {
 
 constexpr int kC = 64;
 constexpr int kD = 128;
-constexpr int kThreads = 128;
+constexpr int kThreads = 128;     // the state pass
+constexpr int kThreadsPar = 256;  // the chunk-parallel kernels: two warps per TMEM lane quadrant
 constexpr float kLog2e = 1.4426950408889634f;
 
 constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
@@ -90,64 +93,74 @@ __device__ __forceinline__ void load_row_chunk(const uint8_t *tile, int row, int
     unpack_bf16x8(*reinterpret_cast<const uint4 *>(tile + t64_chunk(row, chunk)), f);
 }
 
-// Chunk preparation shared by both kernels (all 128 threads).  Normalises the
-// k rows (and the q rows when q_tile is set) of the chunk in place and turns
-// the raw gates landed at kd_tile (a plain [64][128] array, bf16 or fp32; the
-// fp32 one also covers eg_tile) into the tiles Kd = kbar e^{Gmid-G} and
-// EG = e^{G-Gmid}.  Outputs per row: rq (1/|q|), mq (M_r . qbar), rk (1/|k|);
-// per key dim (when non-null): f = e^{Gc-Gmid}, emid = e^{Gmid}.
+// Chunk preparation of the chunk-parallel kernels (all 256 threads).  Normalises
+// the k rows (and the q rows when q_tile is set) of the chunk in place -- two
+// threads per row for q and k, four for k alone -- and turns the raw gates
+// landed at kd_tile (a plain [64][128] array, bf16 or fp32; the fp32 one also
+// covers eg_tile) into the tiles Kd = kbar e^{Gmid-G} and EG = e^{G-Gmid} (G the
+// in-chunk cumulative log gate over token quarters, gq4 a [4][128] scratch; Gmid
+// its value after token 31).  Outputs per row: rq (1/|q|), mq (M_r . qbar),
+// rk (1/|k|); per key dim (when non-null): f = e^{Gc-Gmid}, emid = e^{Gmid}.
 __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, uint8_t *eg_tile,
-                           bool gate_f32, bool l2norm, const float *Mr, float *rq, float *mq, float *rk,
-                           float *gmid, float *f, float *emid, int wt) {
+                              bool gate_f32, bool l2norm, const float *Mr, float *rq, float *mq, float *rk,
+                              float *gq4, float *f, float *emid, int pt) {
     {
-        const bool isq = q_tile != nullptr && wt < 64;
-        const bool active = q_tile != nullptr || wt < 64;
-        const int row = wt & 63;
+        const int tpr = q_tile ? 2 : 4;  // threads per row
+        const int rr = pt / tpr, part = pt % tpr;
+        const bool isq = q_tile != nullptr && rr < 64;
+        const int j = rr & 63;
         uint8_t *base = isq ? q_tile : k_tile;
-        if (active) {
-            float ss = 0.f, md = 0.f;
+        const int cpp = 16 / tpr;  // 16-byte chunks of the row per thread
+        float ss = 0.f, md = 0.f;
 #pragma unroll
-            for (int t64 = 0; t64 < 2; ++t64) {
+        for (int u = 0; u < 8; ++u) {
+            if (u < cpp) {
+                const int cidx = part * cpp + u, t64 = cidx >> 3, cc = cidx & 7;
+                float x[8];
+                load_row_chunk(base + t64 * 8192, j, cc, x);
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
+                for (int e = 0; e < 8; ++e) {
+                    ss = fmaf(x[e], x[e], ss);
+                    if (isq) md = fmaf(x[e], Mr[64 * t64 + 8 * cc + e], md);
+                }
+            }
+        }
+        ss += __shfl_xor_sync(0xffffffffu, ss, 1);
+        md += __shfl_xor_sync(0xffffffffu, md, 1);
+        if (tpr == 4) {
+            ss += __shfl_xor_sync(0xffffffffu, ss, 2);
+            md += __shfl_xor_sync(0xffffffffu, md, 2);
+        }
+        const float rn = l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+        if (l2norm) {
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                if (u < cpp) {
+                    const int cidx = part * cpp + u, t64 = cidx >> 3, cc = cidx & 7;
                     float x[8];
-                    load_row_chunk(base + t64 * 8192, row, cc, x);
+                    load_row_chunk(base + t64 * 8192, j, cc, x);
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        ss = fmaf(x[e], x[e], ss);
-                        if (isq) md = fmaf(x[e], Mr[64 * t64 + 8 * cc + e], md);
-                    }
+                    for (int e = 0; e < 8; ++e) x[e] *= rn;
+                    store_row_chunk(base + t64 * 8192, j, cc, x);
                 }
             }
-            const float rn = l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
-            if (l2norm) {
-#pragma unroll
-                for (int t64 = 0; t64 < 2; ++t64) {
-#pragma unroll
-                    for (int cc = 0; cc < 8; ++cc) {
-                        float x[8];
-                        load_row_chunk(base + t64 * 8192, row, cc, x);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) x[e] *= rn;
-                        store_row_chunk(base + t64 * 8192, row, cc, x);
-                    }
-                }
-            }
+        }
+        if (part == 0) {
             if (isq) {
-                rq[row] = rn;
-                mq[row] = md * rn;
+                rq[j] = rn;
+                mq[j] = md * rn;
             } else {
-                rk[row] = rn;
+                rk[j] = rn;
             }
         }
     }
     __syncthreads();
-    const int p = wt & 63, th = wt >> 6, d0 = 2 * p;
-    float g0[32], g1[32];
+    const int p = pt & 63, qt = pt >> 6, d0 = 2 * p;
+    float g0[16], g1[16];
     float r0 = 0.f, r1 = 0.f;
 #pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        const int j = 32 * th + jj;
+    for (int jj = 0; jj < 16; ++jj) {
+        const int j = 16 * qt + jj;
         float x0, x1;
         if (gate_f32) {
             const float2 f2 = *reinterpret_cast<const float2 *>(kd_tile + (j * kD + d0) * 4);
@@ -159,17 +172,22 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
         r0 += x0; r1 += x1;
         g0[jj] = r0; g1[jj] = r1;
     }
-    if (th == 0) {
-        gmid[d0] = r0;
-        gmid[d0 + 1] = r1;
-    }
-    __syncthreads();  // every raw gate read, Gmid visible
-    const float gm0 = gmid[d0], gm1 = gmid[d0 + 1];
-    const float o0 = th ? 0.f : -gm0 * kLog2e, o1 = th ? 0.f : -gm1 * kLog2e;
-    if (th == 1) {
+    gq4[qt * kD + d0] = r0;
+    gq4[qt * kD + d0 + 1] = r1;
+    __syncthreads();  // every raw gate read, quarter sums visible
+    float off0 = 0.f, off1 = 0.f;
+#pragma unroll
+    for (int q = 0; q < 3; ++q)
+        if (q < qt) {
+            off0 += gq4[q * kD + d0];
+            off1 += gq4[q * kD + d0 + 1];
+        }
+    const float gm0 = gq4[d0] + gq4[kD + d0], gm1 = gq4[d0 + 1] + gq4[kD + d0 + 1];  // Gmid
+    const float o0 = (off0 - gm0) * kLog2e, o1 = (off1 - gm1) * kLog2e;
+    if (qt == 3) {
         if (f) {
-            f[d0] = fast_exp2(r0 * kLog2e);
-            f[d0 + 1] = fast_exp2(r1 * kLog2e);
+            f[d0] = fast_exp2((off0 + r0 - gm0) * kLog2e);
+            f[d0 + 1] = fast_exp2((off1 + r1 - gm1) * kLog2e);
         }
         if (emid) {
             emid[d0] = fast_exp2(gm0 * kLog2e);
@@ -178,8 +196,8 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
     }
     const uint32_t tcol = (d0 >> 6) * 8192;
 #pragma unroll
-    for (int jj = 0; jj < 32; ++jj) {
-        const int j = 32 * th + jj;
+    for (int jj = 0; jj < 16; ++jj) {
+        const int j = 16 * qt + jj;
         const uint32_t off = tcol + t64_offset(j, d0 & 63);
         const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(k_tile + off));
         const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
@@ -230,9 +248,9 @@ constexpr uint32_t OFF_P1 = 172032;  // P1, then W3
 constexpr uint32_t OFF_BC = 180224;  // [64][64] K-major B operand of the Dm increment: row 0 = -c1, then -cz
 constexpr uint32_t OFF_MISC = 188416;
 constexpr uint32_t M_MR = 0, M_RQ = 512, M_LAM = 768, M_ITAU = 1024, M_MQ = 1280, M_C1 = 1536, M_MDZ = 1792,
-                   M_CZ = 2048, M_RK = 2304, M_GP = 2560, M_F = 3072, M_EM = 3584, M_BAR = 4096,
-                   M_TMEM = 4144, M_ABORT = 4148;
-constexpr uint32_t kMisc = 4224;
+                   M_CZ = 2048, M_RK = 2304, M_F = 2560, M_EM = 3072, M_GQ4 = 3584, M_RED = 5632,
+                   M_BAR = 6656, M_TMEM = 6704, M_ABORT = 6708;
+constexpr uint32_t kMisc = 6784;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
 static_assert(OFF_SX == OFF_SK + 32768, "a checkpoint record lands as one block");
@@ -240,7 +258,7 @@ enum { BAR_IN = 0, BAR_R1, BAR_R2, BAR_R3, BAR_R4, kBars };
 constexpr uint32_t TM_SC = 0, TM_T1 = 64, TM_Z = 128, TM_DQ = 256;
 }  // namespace qk
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreadsPar, 1)
 gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                  const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
                  const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
@@ -261,14 +279,16 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     float *mdzv = reinterpret_cast<float *>(misc + M_MDZ);
     float *czv = reinterpret_cast<float *>(misc + M_CZ);
     float *rkv = reinterpret_cast<float *>(misc + M_RK);
-    float *gp = reinterpret_cast<float *>(misc + M_GP);
     float *fv = reinterpret_cast<float *>(misc + M_F);
     float *emv = reinterpret_cast<float *>(misc + M_EM);
+    float *gq4 = reinterpret_cast<float *>(misc + M_GQ4);
+    float *red = reinterpret_cast<float *>(misc + M_RED);  // [2 groups][2][64] row partial sums
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int qd = warp & 3, grp = warp >> 2;  // TMEM lane quadrant, warp group
     const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
     const int bh = blockIdx.x / NC, r = blockIdx.x % NC, b = bh / H, h = bh % H;
     const int c0 = r * kC;
@@ -298,7 +318,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         bulk_load(misc + M_MR, rec + 65536, 512, bb);
     }
     if (warp == 0) tmem_alloc(tmem_slot, 512);
-    for (int e = tid; e < 8192 / 16; e += kThreads)
+    for (int e = tid; e < 8192 / 16; e += kThreadsPar)
         reinterpret_cast<uint4 *>(sm + OFF_BC)[e] = make_uint4(0u, 0u, 0u, 0u);
     if (tid < kC) {
         const int n = c0 + tid;
@@ -308,10 +328,11 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
-    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * qd) << 16);
 
-    const int i = 16 * warp + (lane & 15);  // chunk row of this thread in the M = 64 products
-    const int hf = lane >> 4;               // column half
+    const int i = 16 * qd + (lane & 15);  // chunk row of this thread in the M = 64 products
+    const int hf = lane >> 4;             // column half of a 64-column load; group grp takes the
+                                          // 32-column slice h2 = grp of each 128-column product
     // descriptors (K-major: advance 32 B per K16 slice, 8 KB / 16 KB per 64-wide K block;
     // MN-major: advance 2 KB per 16 K rows)
     const uint64_t dQ = make_desc(sb + OFF_Q, 16, 1024), dQm = make_desc(sb + OFF_Q, 8192, 1024);
@@ -325,8 +346,8 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     const uint64_t dBC = make_desc(sb + OFF_BC, 16, 1024);
 
     mbar_wait(&bar[BAR_IN], 0, abort_flag, status);
-    prep_chunk(sm + OFF_Q, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, Mr, rqv, mqv, rkv, gp, fv,
-               emv, tid);
+    prep_chunk(sm + OFF_Q, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, Mr, rqv, mqv, rkv, gq4,
+               fv, emv, tid);
     tc_fence_before();
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
@@ -351,7 +372,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     // ---- E1: c1, W2, P1
     mbar_wait(&bar[BAR_R1], 0, abort_flag, status);
     tc_fence_after();
-    {
+    if (grp == 0) {
         float sc[32];
         tmem_ld16x2_32<32>(tq + TM_SC, sc);
         const float part = masked_sum(i, hf, sc);
@@ -361,6 +382,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             *reinterpret_cast<__nv_bfloat16 *>(sm + OFF_BC + t64_offset(0, i)) = __float2bfloat16_rn(-c1);
         }
         masked_row(sm + OFF_W2, i, hf, sc, c1);
+    } else {
         float t1[32];
         tmem_ld16x2_32<32>(tq + TM_T1, t1);
         masked_row(sm + OFF_P1, i, hf, t1, 0.f);
@@ -386,8 +408,8 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const uint8_t *qbt = sm + OFF_Q + hf * 8192;
         const uint8_t *egt = sm + OFF_EG + hf * 8192;
         float dl = 0.f, mdz = 0.f;
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
+        {
+            const int h2 = grp;
             float zi[32], dqa[32];
             tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, zi);
             tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, dqa);
@@ -422,7 +444,13 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         dl += __shfl_xor_sync(0xffffffffu, dl, 16);
         mdz += __shfl_xor_sync(0xffffffffu, mdz, 16);
         if (hf == 0) {
-            mdzv[i] = mdz;
+            red[grp * 128 + i] = dl;
+            red[grp * 128 + 64 + i] = mdz;
+        }
+        __syncthreads();
+        if (grp == 0 && hf == 0) {
+            dl = red[i] + red[128 + i];
+            mdzv[i] = red[64 + i] + red[192 + i];
             const int n = c0 + i;
             if (n < T && a.dlambda) a.dlambda[(static_cast<size_t>(b) * T + n) * H + h] = dl;
         }
@@ -456,7 +484,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     // ---- E3: cz, W3
     mbar_wait(&bar[BAR_R3], 0, abort_flag, status);
     tc_fence_after();
-    {
+    if (grp == 0) {
         float t3[32];
         tmem_ld16x2_32<32>(tq + TM_SC, t3);
         const float part = masked_sum(i, hf, t3);
@@ -483,7 +511,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     // ---- E4: dq, the chunk-local CCQ part of dkbar, the chunk's vectors
     mbar_wait(&bar[BAR_R4], 0, abort_flag, status);
     tc_fence_after();
-    {
+    if (grp == 0) {
         float x[32];
         tmem_ld32(tq + TM_T1, x);  // lane tid, column 0: the Dm increment of this chunk
         cvec[tid] = fv[tid];
@@ -495,10 +523,10 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const float *Mh = Mr + 64 * hf;
         uint8_t *qbt = sm + OFF_Q + hf * 8192;
         const uint8_t *dqt = sm + OFF_SX + hf * 8192;
-        float dqb[64];
+        const int h2 = grp;
+        float dqb[32];
         float dot = 0.f;
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
+        {
             float u[32];
             tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, u);
 #pragma unroll
@@ -510,30 +538,32 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
                     const float v = dqc[e] + u[8 * q4 + e] - cz * Mh[8 * cc + e];
-                    dqb[8 * cc + e] = v;
+                    dqb[8 * q4 + e] = v;
                     dot = fmaf(qb[e], v, dot);
                 }
             }
         }
         dot += __shfl_xor_sync(0xffffffffu, dot, 16);
-#pragma unroll
-        for (int cc = 0; cc < 8; ++cc) {
-            float qb[8], out[8];
-            load_row_chunk(qbt, i, cc, qb);
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-                out[e] = a.l2norm ? rq * fmaf(-qb[e], dot, dqb[8 * cc + e]) : dqb[8 * cc + e];
-            store_row_chunk(qbt, i, cc, out);
-        }
-    }
-    {
+        if (hf == 0) red[grp * 128 + i] = dot;
+        // the dkc tile: this group's 32-column slice
         uint8_t *kt = sm + OFF_K + hf * 8192;
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
+        {
             float x[32];
             tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, x);
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(kt, i, 4 * h2 + q4, x + 8 * q4);
+        }
+        __syncthreads();
+        dot = red[i] + red[128 + i];
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+            const int cc = 4 * h2 + q4;
+            float qb[8], out[8];
+            load_row_chunk(qbt, i, cc, qb);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                out[e] = a.l2norm ? rq * fmaf(-qb[e], dot, dqb[8 * q4 + e]) : dqb[8 * q4 + e];
+            store_row_chunk(qbt, i, cc, out);
         }
     }
     fence_proxy_async_smem();
@@ -794,8 +824,8 @@ constexpr uint32_t OFF_DG = 131072;  // fp32 dG [64][kDgStride], over the two im
 constexpr int kDgStride = 129;
 constexpr uint32_t OFF_MISC = 212992;
 constexpr uint32_t M_VEC = 0,        // [2][128] Dm_{r+1}, gate carry (from the state pass)
-                   M_RK = 1024, M_GP = 1280, M_BAR = 1792, M_TMEM = 1824, M_ABORT = 1828;
-constexpr uint32_t kMisc = 1920;
+                   M_RK = 1024, M_GQ4 = 1280, M_RED = 3328, M_BAR = 4352, M_TMEM = 4384, M_ABORT = 4388;
+constexpr uint32_t kMisc = 4480;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(OFF_DG + 64 * kDgStride * 4 <= OFF_P1, "dG scratch reaches P1");
 static_assert(OFF_DC == OFF_DS + 32768, "a state image record lands as one block");
@@ -804,7 +834,7 @@ enum { BAR_IN = 0, BAR_R1, BAR_R2, kBars };
 constexpr uint32_t TM_KC = 0, TM_T1 = 128, TM_SA = 192, TM_DK = 256, TM_DV = 384;
 }  // namespace kv
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreadsPar, 1)
 gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
                   const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
                   const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
@@ -817,13 +847,15 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     uint8_t *misc = sm + OFF_MISC;
     float *vec = reinterpret_cast<float *>(misc + M_VEC);
     float *rkv = reinterpret_cast<float *>(misc + M_RK);
-    float *gp = reinterpret_cast<float *>(misc + M_GP);
+    float *gq4 = reinterpret_cast<float *>(misc + M_GQ4);
+    float *red = reinterpret_cast<float *>(misc + M_RED);  // [2 groups][128] partial sums
     float *dG = reinterpret_cast<float *>(sm + OFF_DG);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int qd = warp & 3, grp = warp >> 2;  // TMEM lane quadrant, warp group
     const int T = a.T, H = a.H, NC = (T + kC - 1) / kC;
     const int bh = blockIdx.x / NC, r = blockIdx.x % NC, b = bh / H, h = bh % H;
     const int c0 = r * kC;
@@ -857,9 +889,9 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
-    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * qd) << 16);
 
-    const int i = 16 * warp + (lane & 15), hf = lane >> 4;
+    const int i = 16 * qd + (lane & 15), hf = lane >> 4;
     const uint64_t dK = make_desc(sb + OFF_K, 16, 1024);
     const uint64_t dV = make_desc(sb + OFF_V, 16, 1024);
     const uint64_t dDO = make_desc(sb + OFF_DO, 16, 1024), dDOm = make_desc(sb + OFF_DO, 8192, 1024);
@@ -871,8 +903,8 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     const uint64_t dSA = make_desc(sb + OFF_SA, 16, 1024);
 
     mbar_wait(&bar[BAR_IN], 0, abort_flag, status);
-    prep_chunk(nullptr, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, nullptr, nullptr, nullptr, rkv,
-               gp, nullptr, nullptr, tid);
+    prep_chunk(nullptr, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, nullptr, nullptr, nullptr,
+               rkv, gq4, nullptr, nullptr, tid);
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
         for (int k = 0; k < 8; ++k) {  // T1 = dO V^T, SA = Kd QG^T
@@ -894,10 +926,11 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     }
     mbar_wait(&bar[BAR_R1], 0, abort_flag, status);
     tc_fence_after();
-    {
+    if (grp == 0) {
         float t1[32];
         tmem_ld16x2_32<32>(tq + TM_T1, t1);
         masked_row(sm + OFF_P1, i, hf, t1, 0.f);  // P1[t][j] = [j <= t] do_t . v_j
+    } else {
         float sa[32];
         tmem_ld16x2_32<32>(tq + TM_SA, sa);
         // SA[j][t] = [t >= j] Kd_j . QG_t (row i is key j)
@@ -935,10 +968,10 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         const uint8_t *dkct = sm + OFF_DKC + hf * 8192;
         const uint8_t *gqt = sm + OFF_GQ + hf * 8192;
         float *dgrow = dG + i * kDgStride + 64 * hf;
-        float dkb[64];
+        const int h2 = grp;  // this group's 32-column slice of each 128-column product
+        float dkb[32];
         float dot = 0.f;
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
+        {
             float x[32], y[32];
             tmem_ld16x2_32<64>(tq + TM_DK + 32 * h2, x);
             tmem_ld16x2_32<64>(tq + TM_KC + 32 * h2, y);
@@ -954,29 +987,32 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
                 for (int e = 0; e < 8; ++e) {
                     const float dkw = x[8 * q4 + e] * __frcp_rn(eg[e]);
                     const float v = dkw + kc[e] + y[8 * q4 + e] + Dh[8 * cc + e];
-                    dkb[8 * cc + e] = v;
+                    dkb[8 * q4 + e] = v;
                     dot = fmaf(kb[e], v, dot);
                     dgrow[8 * cc + e] = fmaf(-kb[e], dkw, gq[e]);
                 }
             }
         }
         dot += __shfl_xor_sync(0xffffffffu, dot, 16);
-#pragma unroll
-        for (int cc = 0; cc < 8; ++cc) {
-            float kb[8], out[8];
-            load_row_chunk(kt, i, cc, kb);
-#pragma unroll
-            for (int e = 0; e < 8; ++e)
-                out[e] = a.l2norm ? rk * fmaf(-kb[e], dot, dkb[8 * cc + e]) : dkb[8 * cc + e];
-            store_row_chunk(kt, i, cc, out);
-        }
+        if (hf == 0) red[grp * 128 + i] = dot;
         uint8_t *vt = sm + OFF_V + hf * 8192;
-#pragma unroll
-        for (int h2 = 0; h2 < 2; ++h2) {
+        {
             float x[32];
             tmem_ld16x2_32<64>(tq + TM_DV + 32 * h2, x);
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(vt, i, 4 * h2 + q4, x + 8 * q4);
+        }
+        __syncthreads();
+        dot = red[i] + red[128 + i];
+#pragma unroll
+        for (int q4 = 0; q4 < 4; ++q4) {
+            const int cc = 4 * h2 + q4;
+            float kb[8], out[8];
+            load_row_chunk(kt, i, cc, kb);
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                out[e] = a.l2norm ? rk * fmaf(-kb[e], dot, dkb[8 * q4 + e]) : dkb[8 * q4 + e];
+            store_row_chunk(kt, i, cc, out);
         }
     }
     fence_proxy_async_smem();
@@ -990,23 +1026,27 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         tma_store_commit();
     }
     {
-        // dgk_t = sum_{s >= t in the chunk} dG_s + rowsum(dS_{r+1} * S_{r+1}),
-        // column d = tid, tokens in reverse
-        float acc = vec[kD + tid];
+        // dgk_t = sum_{s >= t in the chunk} dG_s + rowsum(dS_{r+1} * S_{r+1}): column
+        // d, tokens in reverse, in two 32-row halves (half hh = rows [32 hh, 32 hh + 32))
+        const int d = tid & 127, hh = tid >> 7;
+        float x[32], tot = 0.f;
+#pragma unroll
+        for (int u = 0; u < 32; ++u) {
+            x[u] = dG[(32 * hh + u) * kDgStride + d];
+            tot += x[u];
+        }
+        red[hh * 128 + d] = tot;
+        __syncthreads();
+        float acc = vec[kD + d] + (hh == 0 ? red[128 + d] : 0.f);
         const int nvalid = min(kC, T - c0);
-        for (int t8 = kC - 8; t8 >= 0; t8 -= 8) {
-            float x[8];
 #pragma unroll
-            for (int u = 0; u < 8; ++u) x[u] = dG[(t8 + u) * kDgStride + tid];
-#pragma unroll
-            for (int u = 7; u >= 0; --u) {
-                acc += x[u];
-                const int t = t8 + u;
-                if (t < nvalid) {
-                    const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + tid;
-                    if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
-                    else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
-                }
+        for (int u = 31; u >= 0; --u) {
+            acc += x[u];
+            const int t = 32 * hh + u;
+            if (t < nvalid) {
+                const size_t o = ((static_cast<size_t>(b) * T + c0 + t) * H + h) * kD + d;
+                if (gate_f32) static_cast<float *>(a.dgk)[o] = acc;
+                else static_cast<__nv_bfloat16 *>(a.dgk)[o] = __float2bfloat16_rn(acc);
             }
         }
     }
@@ -1037,14 +1077,14 @@ cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s) {
     }
     const int nc = (a.T + kC - 1) / kC;
     const int chunks = a.B * a.H * nc;
-    gla_bwd_q_kernel<<<chunks, kThreads, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq,
+    gla_bwd_q_kernel<<<chunks, kThreadsPar, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq,
                                                           m.dzr, a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     gla_bwd_state_kernel<<<a.B * a.H, kThreads, st::kSmem, s>>>(m.qg, m.dO, m.dzr, m.q, a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    gla_bwd_kv_kernel<<<chunks, kThreads, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
+    gla_bwd_kv_kernel<<<chunks, kThreadsPar, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
     return cudaGetLastError();
 }
 
