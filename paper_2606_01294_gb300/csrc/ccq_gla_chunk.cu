@@ -30,21 +30,29 @@
 // Kg = kbar * e^{Gmid - G}, Ssnap = e^{Gmid} S_r, and S_{r+1} = e^{Gtot - Gmid} X_{r+1}
 // (that factor is applied at the next snapshot).
 //
-// Warp specialisation (384 threads):
-//   WG0 (warps 0-3)  the dependent chain of chunk r: MMA issue (thread 0) and
-//                    the epilogues W, q_clean, mask of A, output (staged in the
-//                    chunk's Q tile and written by a TMA store).  The 64-row
-//                    products are M = 64 MMAs: rows 16q..16q+15 land in TMEM
-//                    lanes 32q..32q+15, so each warp owns 16 rows.
-//   WG1 (warps 4-7)  prep of chunk r+1 while WG0 runs chunk r: gate cumsum,
-//                    row norms, kbar, Kg, e^{G-Gmid}, M . qbar, lambda.
-//   WG2 (warps 8-11) state snapshot of chunk r+1 (bf16 copies of S^K and
-//                    e^{Gmid} S, rescaling X in TMEM) and the final states.
-// Per-chunk tiles are double-buffered (two slots); v is single-buffered and
-// reloaded as soon as the chunk's last product that reads it completes.
+// Warp specialisation (13 warps):
+//   EPI   (warps 0-7)   the epilogues of chunk r -- W, q_clean, mask of A, output --
+//                       and the bf16 operand copies of the states, placed where EPI
+//                       would otherwise wait on an MMA: S^K_{r+1} while G4 runs,
+//                       e^{Gmid} S_{r+1} (rescaling X in TMEM) while G2 of chunk r+1
+//                       runs.  The 64-row products are M = 64 MMAs (rows 16q..16q+15
+//                       in TMEM lanes 32q..32q+15); warps w and w+4 share lane
+//                       quadrant q = w % 4 and split its columns.  The output goes
+//                       from registers straight to global memory.
+//   PREP  (warps 8-11)  prep of chunk r+1 while the chain runs chunk r: gate
+//                       cumsum, row norms, kbar, Kg, e^{G-Gmid}, M . qbar, lambda.
+//   ISSUE (warp 12)     one thread issues every tcgen05.mma and TMA load, in the
+//                       order G2 | G1 | G3 G8 | G7 | G4 G6 | G5, so that G1, G7 and G6
+//                       run under the epilogues.  An MMA instruction holds its issuing
+//                       thread for its whole execution, which is why no epilogue
+//                       thread issues.  EPI signals the issuer with named-barrier
+//                       arrives; the issuer signals EPI with MMA commits.
+// Per-chunk tiles are double-buffered (two slots); the loads of chunk r+2 start as
+// soon as chunk r's last MMA reader of the slot (G6) completes.  v is single-buffered
+// and reloaded once G5 of the previous chunk completes.
 // Rows past T load as zeros: zero keys add nothing to any sum, zero gates keep
 // the cumulative gate, so the ragged tail needs no special arithmetic.
-// With a.ckpt set, WG2 also copies each chunk's two state tiles and key sum to
+// With a.ckpt set, EPI also copies each chunk's two state tiles and key sum to
 // the checkpoint buffer (one bulk copy per chunk) and the last segment writes
 // S_T there; the backward (ccq_gla_bwd.cu) reads them.
 // With a.nseg > 1 every CTA walks one segment (a range of whole chunks) of one
@@ -64,7 +72,10 @@ namespace {
 
 constexpr int kC = 64;         // chunk length
 constexpr int kD = 128;        // Dk = Dv
-constexpr int kThreads = 384;  // three warpgroups
+constexpr int kEpiThreads = 256;
+constexpr int kPrepWarp0 = 8, kIssueWarp = 12;
+constexpr int kThreads = 32 * (kIssueWarp + 1);  // 416
+constexpr int kSyncCount = kEpiThreads + 32;     // EPI + the issuing warp
 
 // ---- shared memory map (bytes from the 1024-aligned base)
 // two slots of per-chunk tiles, each [64 rows][128 cols] bf16 as two T64 tiles of 8 KB:
@@ -73,37 +84,41 @@ constexpr uint32_t SO_Q = 0;       // raw q, then q_clean * e^{G - Gmid}
 constexpr uint32_t SO_K = 16384;   // raw k, then kbar
 constexpr uint32_t SO_KG = 32768;  // raw gates land here (bf16: 16 KB, fp32: KG+EG 32 KB); then Kg
 constexpr uint32_t SO_EG = 49152;  // e^{G - Gmid}
-constexpr uint32_t OFF_V = 131072;   // 16K  v
+constexpr uint32_t OFF_V = 131072;   // 16K  v; after G5 the output staging of the TMA store
 constexpr uint32_t OFF_W = 147456;   // 8K   W, then the masked A ([64][64], one T64 tile)
 constexpr uint32_t OFF_SK = 155648;  // 32K  bf16 S^K ([128][128], two T64 tiles of 16 KB)
 constexpr uint32_t OFF_S = 188416;   // 32K  bf16 e^{Gmid} S ([128][128], two T64 tiles of 16 KB)
 constexpr uint32_t OFF_MISC = 221184;
-// misc: per-slot arrays (2560 B per slot)
-constexpr uint32_t MS_BYTES = 2560;
+// misc: per-slot arrays (3072 B per slot)
+constexpr uint32_t MS_BYTES = 3072;
 constexpr uint32_t MS_RQ = 0;      // [64] 1/|q_i|
 constexpr uint32_t MS_MQ = 256;    // [64] M . qbar_i
-constexpr uint32_t MS_LAM = 512;   // [64] lambda_i
+constexpr uint32_t MS_LT = 512;    // [64] lambda_i / t_i
 constexpr uint32_t MS_RK = 768;    // [64] 1/|k_j|
 constexpr uint32_t MS_EGM = 1024;  // [128] e^{Gmid}
 constexpr uint32_t MS_F = 1536;    // [128] e^{Gtot - Gmid}
 constexpr uint32_t MS_MST = 2048;  // [128] key sum M at the chunk start
-constexpr uint32_t M_DMP = 5120;   // [2][128] partial key sums of the chunk (prep)
-constexpr uint32_t M_DMPREV = 6144;  // [128] key sum of the previous chunk
-constexpr uint32_t M_GT0 = 6656;   // [128] gate sum over tokens 0..31
-constexpr uint32_t M_CV = 7168;    // [64] c_i
-constexpr uint32_t M_BAR = 7424;   // 13 mbarriers
-constexpr uint32_t M_TMEM = 7528;
-constexpr uint32_t M_ABORT = 7532;
-constexpr uint32_t kMiscBytes = 7680;
+constexpr uint32_t MS_ITI = 2560;  // [64] 1 / t_i
+constexpr uint32_t MS_QN = 2816;   // [64] |q_i| (1 without the l2 norm)
+constexpr uint32_t M_DMP = 6144;   // [2][128] partial key sums of the chunk (prep)
+constexpr uint32_t M_DMPREV = 7168;  // [128] key sum of the previous chunk
+constexpr uint32_t M_GT0 = 7680;   // [128] gate sum over tokens 0..31
+constexpr uint32_t M_BAR = 8192;   // mbarriers
+constexpr uint32_t M_TMEM = 8304;
+constexpr uint32_t M_ABORT = 8308;
+constexpr uint32_t kMiscBytes = 8320;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;  // + alignment slack
 static_assert(kSmemBytes <= 232448, "exceeds the 227 KB per-CTA limit");
 static_assert(OFF_S == OFF_SK + 32768, "a checkpoint copies the S^K and S tiles as one block");
 
 enum {
-    BAR_IN0 = 0, BAR_IN1 = 1, BAR_V = 2, BAR_GA = 3, BAR_GB = 4, BAR_GC = 5, BAR_GD = 6,
-    BAR_PREP0 = 7, BAR_PREP1 = 8, BAR_SNAP = 9, BAR_GS = 10, BAR_GA2 = 11, BAR_GC2 = 12,
+    BAR_IN0 = 0, BAR_IN1 = 1, BAR_V = 2, BAR_GA = 3, BAR_GB = 4, BAR_GK = 5, BAR_GC = 6,
+    BAR_GC2 = 7, BAR_GD = 8, BAR_PREP0 = 9, BAR_PREP1 = 10, BAR_SNAPK = 11, BAR_SNAPS = 12,
     kNumBars = 13
 };
+static_assert(M_BAR + 8 * kNumBars <= M_TMEM, "barrier area");
+// named barriers (0 is __syncthreads)
+enum { NB_W = 1, NB_QC = 2, NB_MASK = 3, NB_OUT = 4, NB_PREP = 5, NB_EPI = 6 };
 
 // ---- tensor memory columns
 constexpr uint32_t TM_S = 0;     // 128 cols
@@ -138,7 +153,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     float *dmp = reinterpret_cast<float *>(misc + M_DMP);
     float *dmprev = reinterpret_cast<float *>(misc + M_DMPREV);
     float *gt0 = reinterpret_cast<float *>(misc + M_GT0);
-    float *cv = reinterpret_cast<float *>(misc + M_CV);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
@@ -147,7 +161,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int wg = tid >> 7, wt = tid & 127;
     const int bh = blockIdx.x / a.nseg, seg = blockIdx.x % a.nseg, b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H;
     const int NCt = (T + kC - 1) / kC;
@@ -167,11 +180,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         for (int i = 0; i < kNumBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        tma_prefetch_desc(&map_q);
-        tma_prefetch_desc(&map_k);
-        tma_prefetch_desc(&map_v);
-        tma_prefetch_desc(&map_g);
-        tma_prefetch_desc(&map_o);
     }
     if (warp == 0) tmem_alloc(tmem_slot, kTmemCols);
     __syncthreads();
@@ -197,15 +205,16 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, tg, b);
     };
 
-    // ---- set-up: initial states into TMEM (WG2), key sum (WG1), first loads (thread 0)
-    if (wg == 2) {
+    // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
+    if (warp < kPrepWarp0) {
         const size_t bhs = static_cast<size_t>(bh);
-        const int row = 32 * (warp & 3) + lane;
+        const int row = 32 * (warp & 3) + lane, grp = warp >> 2;
         for (int m = 0; m < 2; ++m) {
             const float *src = m == 0 ? S0 : C0;
             const uint32_t col0 = m == 0 ? TM_S : TM_SK;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int cc = 0; cc < 2; ++cc) {
+                const int c = 2 * grp + cc;
                 float x[32];
                 if (src) {
                     const float4 *p4 = reinterpret_cast<const float4 *>(
@@ -223,154 +232,169 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
         }
         tmem_wait_st();
-    } else if (wg == 1) {
+    } else if (warp < kIssueWarp) {
+        const int wt = tid - 32 * kPrepWarp0;
         slot_f(0, MS_MST)[wt] = m0 ? m0[(segst ? 0 : static_cast<size_t>(bh) * kD) + wt] : 0.f;
         dmprev[wt] = 0.f;
-    } else if (tid == 0) {
-        issue_in(0);
-        issue_v(0);
+    } else if (warp == kIssueWarp && lane == 0) {
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_v);
+        tma_prefetch_desc(&map_g);
+        tma_prefetch_desc(&map_o);
+        if (NC > 0) {
+            issue_in(0);
+            issue_v(0);
+        }
+        if (NC > 1) issue_in(1);
     }
     tc_fence_before();
     __syncthreads();
 
-    if (wg == 0) {
-        // =============================================================== WG0: the chain
-        const int i = 16 * warp + (lane & 15);  // chunk row owned by this thread
+    if (warp < kPrepWarp0) {
+        // =============================================================== EPI
+        const int grp = warp >> 2;              // column group
+        const int i = 16 * (warp & 3) + (lane & 15);  // chunk row owned by this thread
         const int hf = lane >> 4;               // column half
-        // descriptor bases (start-address field advanced per K slice: +2 per 32 B)
-        const uint64_t dW = make_desc(sb + OFF_W, 16, 1024);
-        const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
-        const uint64_t dS = make_desc(sb + OFF_S, 16384, 1024);
-        const uint64_t dV = make_desc(sb + OFF_V, 8192, 1024);
+        const int row = 32 * (warp & 3) + lane;  // state row a (key dim) of the M = 128 layout
+        uint8_t *ck_head = a.ckpt ? a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T) : nullptr;
+        // bf16 copy of S^K (this thread: row a, columns 64 grp .. 64 grp + 63)
+        auto snap_sk = [&]() {
+            if (ck_head) {
+                // the previous checkpoint copy must have read the tiles before they change
+                if (tid == 0) tma_store_wait_read();
+                named_bar(NB_EPI, kEpiThreads);
+            }
+            tc_fence_after();
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                float x[32];
+                tmem_ld32(tq + TM_SK + 64 * grp + 32 * cc, x);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                    store_row_chunk(sm + OFF_SK + grp * 16384, row, 4 * cc + q4, x + 8 * q4);
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(NB_EPI, kEpiThreads);
+            if (tid == 0) mbar_arrive(&bar[BAR_SNAPK]);
+        };
+        // bf16 copy of e^{Gmid_r} S_r = hs X, with X rescaled in TMEM; then the checkpoint record
+        auto snap_s = [&](int r, float hs) {
+            tc_fence_after();
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                float x[32];
+                tmem_ld32(tq + TM_S + 64 * grp + 32 * cc, x);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) x[e] *= hs;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                    store_row_chunk(sm + OFF_S + grp * 16384, row, 4 * cc + q4, x + 8 * q4);
+                tmem_st32(tq + TM_S + 64 * grp + 32 * cc, x);
+            }
+            tmem_wait_st();
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(NB_EPI, kEpiThreads);
+            if (tid == 0) mbar_arrive(&bar[BAR_SNAPS]);
+            if (ck_head) {
+                // checkpoint of chunk cb + r: the S^K and e^{Gmid} S tiles, then M_r
+                uint8_t *rec = ck_head + static_cast<size_t>(cb + r) * kCkptChunkBytes;
+                if (grp == 0) reinterpret_cast<float *>(rec + 65536)[row] = slot_f(r & 1, MS_MST)[row];
+                if (tid == 0) {
+                    bulk_store(rec, sm + OFF_SK, 65536);
+                    tma_store_commit();
+                }
+            }
+        };
+        float f_cur = 1.f;  // e^{Gtot - Gmid} of the chunk in flight, state row `row`
+        if (NC > 0) {
+            mbar_wait(&bar[BAR_PREP0], 0, abort_flag, status);
+            snap_sk();
+            snap_s(0, slot_f(0, MS_EGM)[row]);
+        }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1, par = r & 1;
             uint8_t *slot = sm + s * SLOT_BYTES;
-            const uint32_t ss = sb + s * SLOT_BYTES;
-            const int c0 = (cb + r) * kC;  // first token of the chunk (sequence position)
-            const float ti = static_cast<float>(tseq0 + c0 + i + 1);
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
-            mbar_wait(&bar[BAR_SNAP], par, abort_flag, status);
-            const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
-            const uint64_t dK = make_desc(ss + SO_K, 16, 1024);
-            const uint64_t dKm = make_desc(ss + SO_K, 8192, 1024);
-            const uint64_t dKG = make_desc(ss + SO_KG, 16, 1024);
-            const uint64_t dKGm = make_desc(ss + SO_KG, 8192, 1024);
-            if (tid == 0 && !*abort_flag) {
-                if (r + 1 < NC) {
-                    tma_store_wait_read();  // the next slot's Q tile staged an earlier output
-                    issue_in(r + 1);
-                }
-                tc_fence_after();
-                // group A: G2 Sc = Q Kbar^T, G1 P = Q S^K
-                for (int k = 0; k < 8; ++k) {
-                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
-                }
-                mma_commit(&bar[BAR_GA]);  // Sc: the W epilogue needs only this
-                for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
-                             dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
-                mma_commit(&bar[BAR_GA2]);
-            }
+            f_cur = slot_f(s, MS_F)[row];
+            const float rqi = slot_f(s, MS_RQ)[i];
+            const float mqi = slot_f(s, MS_MQ)[i];
+            const float iti = slot_f(s, MS_ITI)[i];  // 1 / t_i
+            const float qni = slot_f(s, MS_QN)[i];   // |q_i|
+            const float lt = slot_f(s, MS_LT)[i];    // lambda_i / t_i
             // ---- W epilogue: c_i and W_ij = [j<=i](Sc_ij - c_i |q_i|)
             mbar_wait(&bar[BAR_GA], par, abort_flag, status);
             tc_fence_after();
-            const float rqi = slot_f(s, MS_RQ)[i];
+            float c;
             {
                 float sc[32];
-                tmem_ld16x2_32<32>(tq + TM_SA, sc);
-                float part = 0.f;
+                tmem_ld16x2_32<32>(tq + TM_SA, sc);  // row i, columns 32 hf .. 32 hf + 31
+                float pa[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int jj = 0; jj < 32; ++jj)
-                    if (32 * hf + jj <= i) part += sc[jj];
+                    if (32 * hf + jj <= i) pa[jj & 3] += sc[jj];
+                float part = (pa[0] + pa[1]) + (pa[2] + pa[3]);
                 part += __shfl_xor_sync(0xffffffffu, part, 16);
-                const float cq = slot_f(s, MS_MQ)[i] + rqi * part;
-                const float c = a.centered ? cq / ti : 0.f;
-                if (hf == 0) cv[i] = c;
-                const float cn = c / rqi;  // c_i |q_i|
+                const float cq = mqi + rqi * part;
+                c = a.centered ? cq * iti : 0.f;
+                const float cn = c * qni;  // c_i |q_i|
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
+                for (int q2 = 0; q2 < 2; ++q2) {
                     float w[8];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                        const int j = 32 * hf + 8 * q4 + e;
-                        w[e] = (j <= i) ? sc[8 * q4 + e] - cn : 0.f;
+                        const int jj = 8 * q2 + e;
+                        const float v = grp ? sc[16 + jj] : sc[jj];
+                        w[e] = (32 * hf + 16 * grp + jj <= i) ? v - cn : 0.f;
                     }
-                    store_row_chunk(sm + OFF_W, i, 4 * hf + q4, w);
+                    store_row_chunk(sm + OFF_W, i, 4 * hf + 2 * grp + q2, w);
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                tc_fence_after();
-                // group B: G3 P += W Kbar
-                for (int k = 0; k < 4; ++k)
-                    mma_bf16(tbase + TM_PO, dW + k * 2, dKm + k * 128, ID_64x128_KM, 1);
-                mma_commit(&bar[BAR_GB]);
-            }
+            named_bar_arrive(NB_W, kSyncCount);
             // ---- q_clean epilogue (Eq. clean), scaled by e^{G - Gmid}, into the Q tile.
-            // q_clean e^{G-Gmid} = e^{G-Gmid} (rq q - (lambda/t)(rq P - c M)), computed as
-            // e^{G-Gmid} (rq (q - (lambda/t) P) + (lambda c / t) M).  The shared-memory
-            // operands are read while group B is still running.
+            // q_clean e^{G-Gmid} = e^{G-Gmid} (rq (q - (lambda/t) P) + (lambda c / t) M);
+            // this thread: row i, columns 64 grp + 32 hf .. +31 (T64 tile grp, chunks 4 hf ..)
             {
-                uint8_t *qt = slot + SO_Q + hf * 8192;
-                const uint8_t *et = slot + SO_EG + hf * 8192;
-                const float *Mst = slot_f(s, MS_MST) + 64 * hf;
-                uint4 qraw[8], eraw[8];
+                uint8_t *qt = slot + SO_Q + grp * 8192;
+                const uint8_t *et = slot + SO_EG + grp * 8192;
+                const float *Mst = slot_f(s, MS_MST) + 64 * grp + 32 * hf;
+                uint4 qraw[4], eraw[4];
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
-                    qraw[cc] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, cc));
-                    eraw[cc] = *reinterpret_cast<const uint4 *>(et + t64_chunk(i, cc));
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    qraw[q4] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, 4 * hf + q4));
+                    eraw[q4] = *reinterpret_cast<const uint4 *>(et + t64_chunk(i, 4 * hf + q4));
                 }
-                const float lt = slot_f(s, MS_LAM)[i] / ti;  // lambda_i / t_i
-                mbar_wait(&bar[BAR_GA2], par, abort_flag, status);
                 mbar_wait(&bar[BAR_GB], par, abort_flag, status);
                 tc_fence_after();
-                const float cm = lt * cv[i];                  // lambda_i c_i / t_i
+                const float cm = lt * c;  // lambda_i c_i / t_i
+                float p[32];
+                tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
 #pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    float p[32];
-                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, p);
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    float qr[8], eg[8], out[8];
+                    unpack_bf16x8(qraw[q4], qr);
+                    unpack_bf16x8(eraw[q4], eg);
+                    const float4 m0v = *reinterpret_cast<const float4 *>(Mst + 8 * q4);
+                    const float4 m1v = *reinterpret_cast<const float4 *>(Mst + 8 * q4 + 4);
+                    const float mv[8] = {m0v.x, m0v.y, m0v.z, m0v.w, m1v.x, m1v.y, m1v.z, m1v.w};
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        const int cc = 4 * h2 + q4;  // chunk inside the T64 tile
-                        float qr[8], eg[8], out[8];
-                        unpack_bf16x8(qraw[cc], qr);
-                        unpack_bf16x8(eraw[cc], eg);
-                        const float4 m0 = *reinterpret_cast<const float4 *>(Mst + 8 * cc);
-                        const float4 m1 = *reinterpret_cast<const float4 *>(Mst + 8 * cc + 4);
-                        const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
-#pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            out[e] = eg[e] * fmaf(rqi, fmaf(-lt, p[8 * q4 + e], qr[e]), cm * mv[e]);
-                        store_row_chunk(qt, i, cc, out);
-                    }
+                    for (int e = 0; e < 8; ++e)
+                        out[e] = eg[e] * fmaf(rqi, fmaf(-lt, p[8 * q4 + e], qr[e]), cm * mv[e]);
+                    store_row_chunk(qt, i, 4 * hf + q4, out);
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                mbar_wait(&bar[BAR_V], par, abort_flag, status);
-                tc_fence_after();
-                // group C: G4 A = Qg Kg^T, G6 O = Qg Ssnap
-                for (int k = 0; k < 8; ++k) {
-                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                    mma_bf16(tbase + TM_SA, dQ + ko, dKG + ko, ID_64x64_KK, k != 0);
-                }
-                mma_commit(&bar[BAR_GC]);  // A: the mask epilogue needs only this
-                for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dS + k * 128, ID_64x128_KM,
-                             k != 0);
-                mma_commit(&bar[BAR_GC2]);
-                // group S: G7 X += Kg^T V, G8 S^K += Kbar^T Kbar (needed only by the next snapshot)
-                for (int k = 0; k < 4; ++k)
-                    mma_bf16(tbase + TM_S, dKGm + k * 128, dV + k * 128, ID_128x128_MM, 1);
-                for (int k = 0; k < 4; ++k)
-                    mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
-                mma_commit(&bar[BAR_GS]);
+            named_bar_arrive(NB_QC, kSyncCount);
+            // ---- S^K_{r+1} while G4 runs (G8 of chunk r has run, after its G1 read)
+            if (r + 1 < NC) {
+                mbar_wait(&bar[BAR_GK], par, abort_flag, status);
+                snap_sk();
             }
             // ---- causal mask of A
             mbar_wait(&bar[BAR_GC], par, abort_flag, status);
@@ -379,57 +403,80 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 float sc[32];
                 tmem_ld16x2_32<32>(tq + TM_SA, sc);
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
+                for (int q2 = 0; q2 < 2; ++q2) {
                     float w[8];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                        const int j = 32 * hf + 8 * q4 + e;
-                        w[e] = (j <= i) ? sc[8 * q4 + e] : 0.f;
+                        const int jj = 8 * q2 + e;
+                        const float v = grp ? sc[16 + jj] : sc[jj];
+                        w[e] = (32 * hf + 16 * grp + jj <= i) ? v : 0.f;
                     }
-                    store_row_chunk(sm + OFF_W, i, 4 * hf + q4, w);
+                    store_row_chunk(sm + OFF_W, i, 4 * hf + 2 * grp + q2, w);
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                tc_fence_after();
-                // group D: G5 O += A V
-                for (int k = 0; k < 4; ++k)
-                    mma_bf16(tbase + TM_PO, dW + k * 2, dV + k * 128, ID_64x128_KM, 1);
-                mma_commit(&bar[BAR_GD]);
-            }
-            // ---- output
+            named_bar_arrive(NB_MASK, kSyncCount);
+            // ---- output: o = scale O staged (bf16, swizzled) in the v tile, which G5 has
+            // finished reading; the issuing thread stores it with one TMA copy (rows past T
+            // fall outside the tensor and are not written)
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
-            if (tid == 0 && r + 1 < NC && !*abort_flag) issue_v(r + 1);  // v no longer read
-            if (a.skip_o) continue;  // checkpoint-only pass: no output
-            {
-                // stage o (bf16, swizzled) in the chunk's Q tile, then one TMA store;
-                // rows past T fall outside the tensor and are not written
-                uint8_t *ot = slot + SO_Q + hf * 8192;
+            if (!a.skip_o) {
+                float x[32];
+                tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
 #pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    float x[32];
-                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, x);
+                for (int e = 0; e < 32; ++e) x[e] *= a.scale;
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) x[e] *= a.scale;
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(ot, i, 4 * h2 + q4, x + 8 * q4);
-                }
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_V + grp * 8192, i, 4 * hf + q4, x + 8 * q4);
+                fence_proxy_async_smem();
             }
-            fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                tma_store_4d(&map_o, slot + SO_Q, 0, h, c0, b);
-                tma_store_4d(&map_o, slot + SO_Q + 8192, 64, h, c0, b);
-                tma_store_commit();
+            named_bar_arrive(NB_OUT, kSyncCount);
+            // ---- e^{Gmid_{r+1}} S_{r+1} while G2 of chunk r+1 runs (G6 and G7 of chunk r
+            // have run: GD follows them)
+            if (r + 1 < NC) {
+                mbar_wait(&bar[BAR_PREP0 + (s ^ 1)], ((r + 1) >> 1) & 1, abort_flag, status);
+                snap_s(r + 1, f_cur * slot_f(s ^ 1, MS_EGM)[row]);
             }
         }
-        if (tid == 0) tma_store_wait_all();
-    } else if (wg == 1) {
-        // =============================================================== WG1: prep
+        if (ck_head && tid == 0) tma_store_wait_all();
+        // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K
+        if (NC > 0 && last_seg) {
+            tc_fence_after();
+            const float fs = f_cur;
+            const size_t bhs = static_cast<size_t>(bh);
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                const int c = 2 * grp + cc;
+                float x[32];
+                tmem_ld32(tq + TM_S + 32 * c, x);
+                if (a.ST) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],
+                                             fs * x[4 * e + 3]);
+                }
+                if (ck_head) {
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        ck_head + static_cast<size_t>(NCt) * kCkptChunkBytes + (static_cast<size_t>(row) * kD + 32 * c) * 4);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],
+                                             fs * x[4 * e + 3]);
+                }
+                tmem_ld32(tq + TM_SK + 32 * c, x);
+                if (a.CT) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.CT + (bhs * kD + row) * kD + 32 * c);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+                }
+            }
+        }
+    } else if (warp < kIssueWarp) {
+        // =============================================================== PREP
+        const int wt = tid - 32 * kPrepWarp0;
         const int p = wt & 63, th = wt >> 6;  // key-dim pair (2p, 2p+1), token half
         const int d0 = 2 * p;
         float lam_reg = 0.f;
@@ -445,38 +492,44 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             mbar_wait(&bar[BAR_IN0 + s], sp, abort_flag, status);
             // key sum at the chunk start and lambda of the chunk
             if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
+            const float lam_cur = lam_reg;
             if (wt < 64) {
-                slot_f(s, MS_LAM)[wt] = lam_reg;
                 const int tn = (cb + r + 1) * kC + wt;
                 lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
             }
-            named_bar(2, 128);
-            // row norms (thread = one row of q or k) and M . qbar
+            named_bar(NB_PREP, 128);
+            // row norms (thread = one row of q or k) and M . qbar, four partial sums each
             {
                 const int j = wt & 63;
-                const bool isq = wt < 64;
+                const bool isq = wt < 64;  // warp-uniform
                 const uint8_t *base = slot + (isq ? SO_Q : SO_K);
-                float ss = 0.f, md = 0.f;
+                float ss[4] = {0.f, 0.f, 0.f, 0.f}, md[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int t64 = 0; t64 < 2; ++t64) {
 #pragma unroll
                     for (int cc = 0; cc < 8; ++cc) {
                         float f[8];
                         unpack_bf16x8(*reinterpret_cast<const uint4 *>(base + t64 * 8192 + t64_chunk(j, cc)), f);
-                        const float4 m0 = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc);
-                        const float4 m1 = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc + 4);
-                        const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            ss = fmaf(f[e], f[e], ss);
-                            if (isq) md = fmaf(f[e], mv[e], md);
+                        for (int e = 0; e < 8; ++e) ss[e & 3] = fmaf(f[e], f[e], ss[e & 3]);
+                        if (isq) {
+                            const float4 m0v = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc);
+                            const float4 m1v = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc + 4);
+                            const float mv[8] = {m0v.x, m0v.y, m0v.z, m0v.w, m1v.x, m1v.y, m1v.z, m1v.w};
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) md[e & 3] = fmaf(f[e], mv[e], md[e & 3]);
                         }
                     }
                 }
-                const float rn = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+                const float sst = (ss[0] + ss[1]) + (ss[2] + ss[3]);
+                const float rn = a.l2norm ? rsqrtf(fmaxf(sst, 1e-12f)) : 1.f;
                 if (isq) {
+                    const float iti = 1.f / static_cast<float>(tseq0 + (cb + r) * kC + j + 1);
                     slot_f(s, MS_RQ)[j] = rn;
-                    slot_f(s, MS_MQ)[j] = md * rn;
+                    slot_f(s, MS_MQ)[j] = ((md[0] + md[1]) + (md[2] + md[3])) * rn;
+                    slot_f(s, MS_ITI)[j] = iti;
+                    slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(sst, 1e-12f) * rn : 1.f;
+                    slot_f(s, MS_LT)[j] = lam_cur * iti;
                 } else {
                     slot_f(s, MS_RK)[j] = rn;
                 }
@@ -506,7 +559,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     gt0[d0 + 1] = r1;
                 }
             }
-            named_bar(2, 128);  // raw gates all read, norms and gt0 visible
+            named_bar(NB_PREP, 128);  // raw gates all read, norms and gt0 visible
             {
                 constexpr float kLog2e = 1.4426950408889634f;
                 const float gm0 = gt0[d0], gm1 = gt0[d0 + 1];   // Gmid
@@ -522,118 +575,164 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 const float *rk = slot_f(s, MS_RK);
                 const uint32_t tcol = (d0 >> 6) * 8192;
                 float dm0 = 0.f, dm1 = 0.f;
+                // four batches of eight tokens: every load of a batch is issued before its
+                // stores (the in-place kbar store may alias a later load)
 #pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {
-                    const int j = 32 * th + jj;
-                    const uint32_t off = tcol + t64_offset(j, d0 & 63);
-                    const float2 kr =
-                        __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(slot + SO_K + off));
-                    const float rkj = rk[j];
-                    const float k0 = kr.x * rkj, k1 = kr.y * rkj;
-                    const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
-                    *reinterpret_cast<uint32_t *>(slot + SO_K + off) = pack_bf16(k0, k1);
-                    *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
-                        pack_bf16(k0 * fast_exp2(-x0), k1 * fast_exp2(-x1));
-                    *reinterpret_cast<uint32_t *>(slot + SO_EG + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
-                    dm0 += k0;
-                    dm1 += k1;
+                for (int bt = 0; bt < 4; ++bt) {
+                    uint32_t kraw[8];
+                    float rkv[8];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const int j = 32 * th + 8 * bt + u;
+                        kraw[u] = *reinterpret_cast<const uint32_t *>(slot + SO_K + tcol + t64_offset(j, d0 & 63));
+                        rkv[u] = rk[j];
+                    }
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) {
+                        const int jj = 8 * bt + u, j = 32 * th + jj;
+                        const uint32_t off = tcol + t64_offset(j, d0 & 63);
+                        const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&kraw[u]));
+                        const float k0 = kr.x * rkv[u], k1 = kr.y * rkv[u];
+                        const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
+                        *reinterpret_cast<uint32_t *>(slot + SO_K + off) = pack_bf16(k0, k1);
+                        *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
+                            pack_bf16(k0 * fast_exp2(-x0), k1 * fast_exp2(-x1));
+                        *reinterpret_cast<uint32_t *>(slot + SO_EG + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
+                        dm0 += k0;
+                        dm1 += k1;
+                    }
                 }
                 dmp[th * kD + d0] = dm0;
                 dmp[th * kD + d0 + 1] = dm1;
             }
             fence_proxy_async_smem();
-            named_bar(2, 128);
+            named_bar(NB_PREP, 128);
             dmprev[wt] = dmp[wt] + dmp[kD + wt];
-            named_bar(2, 128);
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
         }
-        // final key sum and position
+        // final key sum
         if (NC > 0 && a.mT && last_seg) {
             const int sl = (NC - 1) & 1;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
     } else {
-        // =============================================================== WG2: states
-        const int row = 32 * (warp & 3) + lane;  // state row a (key dim)
-        uint8_t *ck_head = a.ckpt ? a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T) : nullptr;
+        // =============================================================== ISSUE
+        const bool lead = lane == 0;
+        // descriptor bases (start-address field advanced per K slice: +2 per 32 B)
+        const uint64_t dW = make_desc(sb + OFF_W, 16, 1024);
+        const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
+        const uint64_t dS = make_desc(sb + OFF_S, 16384, 1024);
+        const uint64_t dV = make_desc(sb + OFF_V, 8192, 1024);
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
-            const uint32_t sp = (r >> 1) & 1;
-            if (r > 0) mbar_wait(&bar[BAR_GS], (r - 1) & 1, abort_flag, status);
+            const uint32_t sp = (r >> 1) & 1, par = r & 1;
+            const uint32_t ss = sb + s * SLOT_BYTES;
+            const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
+            const uint64_t dK = make_desc(ss + SO_K, 16, 1024);
+            const uint64_t dKm = make_desc(ss + SO_K, 8192, 1024);
+            const uint64_t dKG = make_desc(ss + SO_KG, 16, 1024);
+            const uint64_t dKGm = make_desc(ss + SO_KG, 8192, 1024);
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
-            if (ck_head && r > 0) {
-                // the previous checkpoint copy must have read the tiles before they change
-                if (wt == 0) tma_store_wait_read();
-                named_bar(3, 128);
-            }
             tc_fence_after();
-            const float hs = (r > 0 ? slot_f(s ^ 1, MS_F)[row] : 1.f) * slot_f(s, MS_EGM)[row];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_S + 32 * c, x);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) x[e] *= hs;
-                uint8_t *tile = sm + OFF_S + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
-                tmem_st32(tq + TM_S + 32 * c, x);
+            // G2 Sc = Q Kbar^T (SA is free: the mask epilogue of chunk r-1 has read A)
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 8; ++k) {
+                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
+                }
+                mma_commit(&bar[BAR_GA]);
             }
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_SK + 32 * c, x);
-                uint8_t *tile = sm + OFF_SK + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
-            }
-            tmem_wait_st();
-            fence_proxy_async_smem();
-            tc_fence_before();
-            named_bar(3, 128);
-            if (ck_head) {
-                // checkpoint of chunk cb + r: the S^K and e^{Gmid} S tiles, then M_r
-                uint8_t *rec = ck_head + static_cast<size_t>(cb + r) * kCkptChunkBytes;
-                reinterpret_cast<float *>(rec + 65536)[row] = slot_f(s, MS_MST)[row];
-                if (wt == 0) {
-                    bulk_store(rec, sm + OFF_SK, 65536);
+            __syncwarp();
+            if (r > 0) {
+                // O of chunk r-1 is staged in the v tile: store it
+                mbar_wait(&bar[BAR_GD], (r - 1) & 1, abort_flag, status);
+                named_bar(NB_OUT, kSyncCount);  // O of chunk r-1 read out of PO and staged
+                if (lead && !a.skip_o) {
+                    const int cp = (cb + r - 1) * kC;
+                    tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
+                    tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
                     tma_store_commit();
                 }
+                __syncwarp();
             }
-            if (wt == 0) mbar_arrive(&bar[BAR_SNAP]);
-        }
-        if (ck_head && wt == 0) tma_store_wait_all();
-        // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K
-        if (NC > 0 && last_seg) {
-            mbar_wait(&bar[BAR_GS], (NC - 1) & 1, abort_flag, status);
+            // G1 P = Q S^K
+            mbar_wait(&bar[BAR_SNAPK], par, abort_flag, status);
             tc_fence_after();
-            const float fs = slot_f((NC - 1) & 1, MS_F)[row];
-            const size_t bhs = static_cast<size_t>(bh);
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_S + 32 * c, x);
-                if (a.ST) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * c);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],
-                                             fs * x[4 * e + 3]);
+            if (lead && !*abort_flag)
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
+                             dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
+            // v of chunk r replaces the staged output once the store has read it
+            if (r > 0 && lead) {
+                tma_store_wait_read();
+                if (!*abort_flag) issue_v(r);
+            }
+            __syncwarp();
+            // G3 P += W Kbar, then G8 S^K += Kbar^T Kbar
+            named_bar(NB_W, kSyncCount);
+            tc_fence_after();
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_PO, dW + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GB]);
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
+                mma_commit(&bar[BAR_GK]);
+            }
+            __syncwarp();
+            // G7 X += Kg^T V (X rescaled by the snapshot of chunk r; v landed)
+            mbar_wait(&bar[BAR_SNAPS], par, abort_flag, status);
+            mbar_wait(&bar[BAR_V], par, abort_flag, status);
+            tc_fence_after();
+            if (lead && !*abort_flag)
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_S, dKGm + k * 128, dV + k * 128, ID_128x128_MM, 1);
+            __syncwarp();
+            // G4 A = Qg Kg^T, G6 O = Qg Ssnap
+            named_bar(NB_QC, kSyncCount);
+            tc_fence_after();
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 8; ++k) {
+                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                    mma_bf16(tbase + TM_SA, dQ + ko, dKG + ko, ID_64x64_KK, k != 0);
                 }
-                if (ck_head) {
-                    float4 *dst = reinterpret_cast<float4 *>(
-                        ck_head + static_cast<size_t>(NCt) * kCkptChunkBytes + (static_cast<size_t>(row) * kD + 32 * c) * 4);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2],
-                                             fs * x[4 * e + 3]);
-                }
-                tmem_ld32(tq + TM_SK + 32 * c, x);
-                if (a.CT) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.CT + (bhs * kD + row) * kD + 32 * c);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
-                }
+                mma_commit(&bar[BAR_GC]);
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dS + k * 128, ID_64x128_KM,
+                             k != 0);
+                mma_commit(&bar[BAR_GC2]);
+            }
+            __syncwarp();
+            // G5 O += A V
+            named_bar(NB_MASK, kSyncCount);
+            tc_fence_after();
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 4; ++k)
+                    mma_bf16(tbase + TM_PO, dW + k * 2, dV + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GD]);
+            }
+            __syncwarp();
+            // the slot's last MMA reader (G6) is done: load chunk r + 2 into it
+            if (r + 2 < NC) {
+                mbar_wait(&bar[BAR_GC2], par, abort_flag, status);
+                if (lead && !*abort_flag) issue_in(r + 2);
+                __syncwarp();
+            }
+        }
+        if (NC > 0) {
+            mbar_wait(&bar[BAR_GD], (NC - 1) & 1, abort_flag, status);
+            named_bar(NB_OUT, kSyncCount);
+            if (lead && !a.skip_o) {
+                const int cp = (cb + NC - 1) * kC;
+                tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
+                tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
+                tma_store_commit();
+            }
+            if (lead) tma_store_wait_all();
+            // after a give-up, wait (bounded) for the copies still in flight
+            if (lead && *abort_flag) {
+                mbar_drain(&bar[BAR_V], (NC - 1) & 1);
+                for (int r = (NC > 2 ? NC - 2 : 0); r < NC; ++r) mbar_drain(&bar[BAR_IN0 + (r & 1)], (r >> 1) & 1);
             }
         }
     }

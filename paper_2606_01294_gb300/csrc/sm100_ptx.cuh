@@ -42,14 +42,16 @@ __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
+// One bounded try: the thread may be suspended (up to about a millisecond)
+// until the phase completes, so a waiting warp does not spin on the barrier.
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(bar), "r"(parity)
+        : "r"(bar), "r"(parity), "r"(1000000u)
         : "memory");
     return ok != 0;
 }
@@ -75,6 +77,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
     return true;
 }
 
+// Bounded wait that ignores the abort flag: a thread that issued asynchronous
+// copies waits for them to land before the CTA exits, even after a give-up.
+__device__ __forceinline__ void mbar_drain(uint64_t *bar, uint32_t parity) {
+    const uint32_t a = smem_addr(bar);
+    const long long start = clock64();
+    while (!mbar_try_wait(a, parity))
+        if (clock64() - start > kWaitLimitCycles) return;
+}
+
 // ---------------------------------------------------------------- fences
 
 // Make generic-proxy shared-memory writes visible to the async proxy (TMA,
@@ -94,6 +105,12 @@ __device__ __forceinline__ void tc_fence_after() {
 // Named barrier over `count` threads (a subset of the CTA, whole warps).
 __device__ __forceinline__ void named_bar(int id, int count) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// Arrive on named barrier `id` without waiting (the waiting side uses named_bar
+// with the same count): a one-way signal from producer warps to a consumer warp.
+__device__ __forceinline__ void named_bar_arrive(int id, int count) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 // ---------------------------------------------------------------- TMA
