@@ -25,8 +25,7 @@ __global__ void __launch_bounds__(128, 1)
 diag_mma_kernel(const __nv_bfloat16 *A, const __nv_bfloat16 *Bm, float *D, int M, int N, int K,
                 int a_mn, int b_mn, int *status) {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                              ~static_cast<uintptr_t>(1023));
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *sa = sm;               // up to 32K
     uint8_t *sbm = sm + 32768;      // up to 32K

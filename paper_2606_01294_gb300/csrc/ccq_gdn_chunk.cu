@@ -70,8 +70,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
               const __grid_constant__ CUtensorMap map_ut, const __grid_constant__ CUtensorMap map_w,
               const ChunkArgs a, int NC) {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                              ~static_cast<uintptr_t>(1023));
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     float *A = reinterpret_cast<float *>(sm + WY_A);
     float *Tt = reinterpret_cast<float *>(sm + WY_T);
@@ -401,8 +400,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                  const __grid_constant__ CUtensorMap map_ut, const __grid_constant__ CUtensorMap map_w,
                  const __grid_constant__ CUtensorMap map_o, const ChunkArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                              ~static_cast<uintptr_t>(1023));
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *dmprev = reinterpret_cast<float *>(misc + M_DMPREV);

@@ -76,10 +76,6 @@ constexpr uint32_t ID_64x128_MM = make_idesc(64, 128, 1, 1);
 constexpr uint32_t ID_128x128_MM = make_idesc(128, 128, 1, 1);
 constexpr uint32_t ID_128x64_MK = make_idesc(128, 64, 1, 0);
 
-__device__ __forceinline__ uint8_t *align1024(uint8_t *p) {
-    return reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
-}
-
 __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chunk, const float *w) {
     uint4 u;
     u.x = pack_bf16(w[0], w[1]);
@@ -267,7 +263,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                  const BwdArgs a) {
     using namespace qk;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = align1024(smem_raw);
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *Mr = reinterpret_cast<float *>(misc + M_MR);
@@ -609,7 +605,7 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
                      const BwdArgs a) {
     using namespace st;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = align1024(smem_raw);
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *Dm = reinterpret_cast<float *>(misc + M_DM);
@@ -842,7 +838,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
                   const __grid_constant__ CUtensorMap map_dv, const BwdArgs a) {
     using namespace kv;
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = align1024(smem_raw);
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *vec = reinterpret_cast<float *>(misc + M_VEC);

@@ -50,8 +50,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
                          const __grid_constant__ CUtensorMap map_g, const ChunkArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                              ~static_cast<uintptr_t>(1023));
+    uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *dsuf = reinterpret_cast<float *>(misc + M_DSUF);

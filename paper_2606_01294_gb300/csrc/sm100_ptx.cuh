@@ -202,6 +202,13 @@ __device__ __forceinline__ float fast_exp2(float x) {
     return y;
 }
 
+// The first 1024-byte boundary at or after the dynamic shared-memory base,
+// reached by pointer arithmetic on the __shared__ array so that the compiler
+// keeps the shared address space (and emits shared, not generic, accesses).
+__device__ __forceinline__ uint8_t *smem_align1024(uint8_t *smem_base) {
+    return smem_base + ((1024u - (smem_addr(smem_base) & 1023u)) & 1023u);
+}
+
 // ---------------------------------------------------------------- tcgen05
 
 __device__ __forceinline__ void tmem_alloc(uint32_t *dst_smem, uint32_t ncols) {
