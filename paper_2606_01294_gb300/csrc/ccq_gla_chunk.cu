@@ -285,11 +285,19 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             for (int cc = 0; cc < 2; ++cc) {
                 float x[32];
                 tmem_ld32(tq + TM_S + 64 * grp + 32 * cc, x);
+                const uint64_t hs2 = f2_make(hs, hs);
+                uint32_t w[16];
 #pragma unroll
-                for (int e = 0; e < 32; ++e) x[e] *= hs;
+                for (int e = 0; e < 16; ++e) {
+                    const float2 y = f2_split(f2_mul(f2_make(x[2 * e], x[2 * e + 1]), hs2));
+                    x[2 * e] = y.x;
+                    x[2 * e + 1] = y.y;
+                    w[e] = pack_bf16(y.x, y.y);
+                }
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4)
-                    store_row_chunk(sm + OFF_S + grp * 16384, row, 4 * cc + q4, x + 8 * q4);
+                    *reinterpret_cast<uint4 *>(sm + OFF_S + grp * 16384 + t64_chunk(row, 4 * cc + q4)) =
+                        make_uint4(w[4 * q4], w[4 * q4 + 1], w[4 * q4 + 2], w[4 * q4 + 3]);
                 tmem_st32(tq + TM_S + 64 * grp + 32 * cc, x);
             }
             tmem_wait_st();
@@ -373,18 +381,23 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 const float cm = lt * c;  // lambda_i c_i / t_i
                 float p[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
+                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqi, rqi), cm2 = f2_make(cm, cm);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
-                    float qr[8], eg[8], out[8];
-                    unpack_bf16x8(qraw[q4], qr);
-                    unpack_bf16x8(eraw[q4], eg);
-                    const float4 m0v = *reinterpret_cast<const float4 *>(Mst + 8 * q4);
-                    const float4 m1v = *reinterpret_cast<const float4 *>(Mst + 8 * q4 + 4);
-                    const float mv[8] = {m0v.x, m0v.y, m0v.z, m0v.w, m1v.x, m1v.y, m1v.z, m1v.w};
+                    const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4);
+                    const ulonglong2 m23 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4 + 4);
+                    const uint64_t mp[4] = {m01.x, m01.y, m23.x, m23.y};
+                    const uint32_t qw[4] = {qraw[q4].x, qraw[q4].y, qraw[q4].z, qraw[q4].w};
+                    const uint32_t ew[4] = {eraw[q4].x, eraw[q4].y, eraw[q4].z, eraw[q4].w};
+                    uint32_t ow[4];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        out[e] = eg[e] * fmaf(rqi, fmaf(-lt, p[8 * q4 + e], qr[e]), cm * mv[e]);
-                    store_row_chunk(qt, i, 4 * hf + q4, out);
+                    for (int w = 0; w < 4; ++w) {
+                        const uint64_t p2 = f2_make(p[8 * q4 + 2 * w], p[8 * q4 + 2 * w + 1]);
+                        const uint64_t t = f2_fma(nlt, p2, f2_from_bf16x2(qw[w]));     // q - (lambda/t) P
+                        const uint64_t u = f2_fma(rq2, t, f2_mul(cm2, mp[w]));          // rq (.) + (lambda c/t) M
+                        ow[w] = bf16x2_from_f2(f2_mul(f2_from_bf16x2(ew[w]), u));      // * e^{G - Gmid}
+                    }
+                    *reinterpret_cast<uint4 *>(qt + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
                 }
             }
             fence_proxy_async_smem();

@@ -387,4 +387,51 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4 &u, float (&f)[8]) {
     }
 }
 
+// ---------------------------------------------------------------- packed fp32 pairs
+//
+// Two fp32 values in one 64-bit register pair, operated on by the f32x2
+// arithmetic of sm_100-family GPUs (one instruction per pair, IEEE rounding
+// of each lane as in the scalar instruction).  The low half is the first value.
+
+__device__ __forceinline__ uint64_t f2_make(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ float2 f2_split(uint64_t v) {
+    float2 r;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+    uint64_t d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+    return d;
+}
+
+// A bf16 pair (first element in the low 16 bits) as an fp32 pair.
+__device__ __forceinline__ uint64_t f2_from_bf16x2(uint32_t w) {
+    return f2_make(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+
+// An fp32 pair rounded to a bf16 pair (first element in the low 16 bits).
+__device__ __forceinline__ uint32_t bf16x2_from_f2(uint64_t v) {
+    const float2 x = f2_split(v);
+    return pack_bf16(x.x, x.y);
+}
+
 }  // namespace ccq
