@@ -350,36 +350,54 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 
 
 // ============================================================================ main kernel
+//
+// Warp specialisation (13 warps), as in the GLA kernel:
+//   EPI   (warps 0-7)   the epilogues of chunk r -- W' and U = Ut - W Hm, q_clean, Pm,
+//                       output -- and the bf16 copies of S^K_{r+1} (while D4 runs) and
+//                       Hm_{r+1} (while G2 of chunk r+1 runs).  Warps w and w+4 share
+//                       TMEM lane quadrant w % 4 and split its columns.
+//   PREP  (warps 8-11)  prep of chunk r+1: row norms, cumulative decay, kbar, Kd.
+//   ISSUE (warp 12)     every tcgen05.mma and TMA copy, in the order
+//                       G2 D2 | G1 | G3 G8 D6 | D4 D3 | D5.  D2 (W Hm) lands in the P/O
+//                       accumulator, so EPI reads it out first and frees the accumulator
+//                       for G1 before it builds U.
+// The output is staged in the U tile (dead once D5 and D6 have run) and stored by TMA.
 
-constexpr int kThreads = 384;
+constexpr int kThreads = 416;
+constexpr int kEpiThreads = 256;
+constexpr int kPrepWarp0 = 8, kIssueWarp = 12;
+constexpr int kSyncCount = kEpiThreads + 32;
 constexpr uint32_t SLOT_BYTES = 49152;
-constexpr uint32_t SO_Q = 0;        // raw q, then q_clean e^{gc - gc_m}; finally the output staging
+constexpr uint32_t SO_Q = 0;        // raw q, then q_clean e^{gc - gc_m}
 constexpr uint32_t SO_K = 16384;    // raw k, then kbar
 constexpr uint32_t SO_KD = 32768;   // kbar e^{gc_m - gc}
 constexpr uint32_t OFF_UT = 98304;  // 16K  Ut of the chunk (workspace)
 constexpr uint32_t OFF_WW = 114688; // 16K  W of the chunk (workspace)
-constexpr uint32_t OFF_UB = 131072; // 16K  U (bf16, rows j)
+constexpr uint32_t OFF_UB = 131072; // 16K  U (bf16, rows j); after D5 the output staging
 constexpr uint32_t OFF_WM = 147456; // 8K   W' of the CCQ fold, then Pm
 constexpr uint32_t OFF_SK = 155648; // 32K  bf16 S^K
 constexpr uint32_t OFF_HB = 188416; // 32K  bf16 Hm = e^{gc_m} H
 constexpr uint32_t OFF_MISC = 221184;
-constexpr uint32_t MS_BYTES = 2560;
-constexpr uint32_t MS_RQ = 0, MS_MQ = 256, MS_LAM = 512, MS_RK = 768, MS_EP = 1024, MS_EN = 1280,
-                   MS_SCAL = 1536, MS_MST = 2048;  // SCAL: [0] e^{gc_m}, [1] e^{gc_C - gc_m}, [2..65] gc
-constexpr uint32_t M_DMPREV = 5120;  // [128]
-constexpr uint32_t M_CV = 5632;      // [64]
-constexpr uint32_t M_BAR = 5888;     // 14 mbarriers
-constexpr uint32_t M_TMEM = 6016;
-constexpr uint32_t M_ABORT = 6020;
-constexpr uint32_t kMiscBytes = 6144;
+constexpr uint32_t MS_BYTES = 3072;
+constexpr uint32_t MS_RQ = 0, MS_MQ = 256, MS_LT = 512, MS_RK = 768, MS_EP = 1024, MS_EN = 1280,
+                   MS_SCAL = 1536, MS_MST = 2048, MS_ITI = 2560, MS_QN = 2816;
+// SCAL: [0] e^{gc_m}, [1] e^{gc_C - gc_m}, [2..65] gc;  LT = lambda / t, ITI = 1 / t, QN = |q|
+constexpr uint32_t M_DMP = 6144;     // [2][128] key-sum halves of the chunk
+constexpr uint32_t M_DMPREV = 7168;  // [128]
+constexpr uint32_t M_BAR = 7680;     // mbarriers
+constexpr uint32_t M_TMEM = 7808;
+constexpr uint32_t M_ABORT = 7812;
+constexpr uint32_t kMiscBytes = 7936;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;
 static_assert(kSmemBytes <= 232448, "exceeds the 227 KB per-CTA limit");
 static_assert(MS_SCAL + 66 * 4 <= MS_MST, "scalar area overlaps");
 
 enum {
-    BAR_IN0 = 0, BAR_IN1 = 1, BAR_WU = 2, BAR_GA = 3, BAR_GB = 4, BAR_GC = 5, BAR_GD = 6,
-    BAR_PREP0 = 7, BAR_PREP1 = 8, BAR_SNAP = 9, BAR_GS = 10, BAR_GC2 = 11, kNumBars = 12
+    BAR_IN0 = 0, BAR_IN1 = 1, BAR_WU = 2, BAR_GA1 = 3, BAR_GA2 = 4, BAR_GB = 5, BAR_GK = 6, BAR_GC = 7,
+    BAR_GC2 = 8, BAR_GD = 9, BAR_PREP0 = 10, BAR_PREP1 = 11, BAR_SNAPK = 12, BAR_SNAPS = 13, kNumBars = 14
 };
+static_assert(M_BAR + 8 * kNumBars <= M_TMEM, "barrier area");
+enum { NB_PO = 1, NB_W = 2, NB_QC = 3, NB_MASK = 4, NB_OUT = 5, NB_PREP = 6, NB_EPI = 7 };
 
 constexpr uint32_t TM_S = 0, TM_SK = 128, TM_PO = 256, TM_SA = 384, kTmemCols = 512;
 constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
@@ -403,8 +421,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
+    float *dmp = reinterpret_cast<float *>(misc + M_DMP);
     float *dmprev = reinterpret_cast<float *>(misc + M_DMPREV);
-    float *cv = reinterpret_cast<float *>(misc + M_CV);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
@@ -413,7 +431,6 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int wg = tid >> 7, wt = tid & 127;
     const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H;
     const int NC = (T + kC - 1) / kC;
@@ -425,11 +442,6 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         for (int i = 0; i < kNumBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        tma_prefetch_desc(&map_q);
-        tma_prefetch_desc(&map_k);
-        tma_prefetch_desc(&map_ut);
-        tma_prefetch_desc(&map_w);
-        tma_prefetch_desc(&map_o);
     }
     if (warp == 0) tmem_alloc(tmem_slot, kTmemCols);
     __syncthreads();
@@ -457,14 +469,16 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_2d(sm + OFF_WW + 8192, &map_w, bb, 64, row);
     };
 
-    if (wg == 2) {
+    // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
+    if (warp < kPrepWarp0) {
         const size_t bhs = static_cast<size_t>(bh);
-        const int row = 32 * (warp & 3) + lane;
+        const int row = 32 * (warp & 3) + lane, grp = warp >> 2;
         for (int m = 0; m < 2; ++m) {
             const float *src = m == 0 ? a.S0 : a.C0;
             const uint32_t col0 = m == 0 ? TM_S : TM_SK;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int cc = 0; cc < 2; ++cc) {
+                const int c = 2 * grp + cc;
                 float x[32];
                 if (src) {
                     const float4 *p4 = reinterpret_cast<const float4 *>(src + (bhs * kD + row) * kD + 32 * c);
@@ -481,222 +495,267 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
         }
         tmem_wait_st();
-    } else if (wg == 1) {
+    } else if (warp < kIssueWarp) {
+        const int wt = tid - 32 * kPrepWarp0;
         slot_f(0, MS_MST)[wt] = a.m0 ? a.m0[static_cast<size_t>(bh) * kD + wt] : 0.f;
         dmprev[wt] = 0.f;
-    } else if (tid == 0) {
-        issue_in(0);
-        issue_wu(0);
+    } else if (lane == 0) {
+        tma_prefetch_desc(&map_q);
+        tma_prefetch_desc(&map_k);
+        tma_prefetch_desc(&map_ut);
+        tma_prefetch_desc(&map_w);
+        tma_prefetch_desc(&map_o);
+        if (NC > 0) {
+            issue_in(0);
+            issue_wu(0);
+        }
+        if (NC > 1) issue_in(1);
     }
     tc_fence_before();
     __syncthreads();
 
-    if (wg == 0) {
-        // =============================================================== WG0: the chain
-        const int i = 16 * warp + (lane & 15);
+    if (warp < kPrepWarp0) {
+        // =============================================================== EPI
+        const int grp = warp >> 2;
+        const int i = 16 * (warp & 3) + (lane & 15);
         const int hf = lane >> 4;
-        const uint64_t dWm = make_desc(sb + OFF_WM, 16, 1024);
-        const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
-        const uint64_t dHB = make_desc(sb + OFF_HB, 16384, 1024);
-        const uint64_t dWW = make_desc(sb + OFF_WW, 16, 1024);
-        const uint64_t dUBm = make_desc(sb + OFF_UB, 8192, 1024);
+        const int row = 32 * (warp & 3) + lane;  // state row of the M = 128 layout
+        auto snap_sk = [&]() {
+            tc_fence_after();
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                float x[32];
+                tmem_ld32(tq + TM_SK + 64 * grp + 32 * cc, x);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                    store_row_chunk(sm + OFF_SK + grp * 16384, row, 4 * cc + q4, x + 8 * q4);
+            }
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(NB_EPI, kEpiThreads);
+            if (tid == 0) mbar_arrive(&bar[BAR_SNAPK]);
+        };
+        // Hm = e^{gc_m} H = hs X, X rescaled in TMEM
+        auto snap_s = [&](float hs) {
+            tc_fence_after();
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                float x[32];
+                tmem_ld32(tq + TM_S + 64 * grp + 32 * cc, x);
+                const uint64_t hs2 = f2_make(hs, hs);
+                uint32_t w[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const float2 y = f2_split(f2_mul(f2_make(x[2 * e], x[2 * e + 1]), hs2));
+                    x[2 * e] = y.x;
+                    x[2 * e + 1] = y.y;
+                    w[e] = pack_bf16(y.x, y.y);
+                }
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                    *reinterpret_cast<uint4 *>(sm + OFF_HB + grp * 16384 + t64_chunk(row, 4 * cc + q4)) =
+                        make_uint4(w[4 * q4], w[4 * q4 + 1], w[4 * q4 + 2], w[4 * q4 + 3]);
+                tmem_st32(tq + TM_S + 64 * grp + 32 * cc, x);
+            }
+            tmem_wait_st();
+            fence_proxy_async_smem();
+            tc_fence_before();
+            named_bar(NB_EPI, kEpiThreads);
+            if (tid == 0) mbar_arrive(&bar[BAR_SNAPS]);
+        };
+        float fc = 1.f;  // e^{gc_C - gc_m} of the chunk in flight
+        if (NC > 0) {
+            mbar_wait(&bar[BAR_PREP0], 0, abort_flag, status);
+            snap_sk();
+            snap_s(slot_f(0, MS_SCAL)[0]);
+        }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1, par = r & 1;
             uint8_t *slot = sm + s * SLOT_BYTES;
-            const uint32_t ss = sb + s * SLOT_BYTES;
-            const int c0 = r * kC;
-            const float ti = static_cast<float>(t0 + c0 + i + 1);
-            const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
-            const uint64_t dK = make_desc(ss + SO_K, 16, 1024);
-            const uint64_t dKm = make_desc(ss + SO_K, 8192, 1024);
-            const uint64_t dKDm = make_desc(ss + SO_KD, 8192, 1024);
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
-            mbar_wait(&bar[BAR_SNAP], par, abort_flag, status);
-            if (tid == 0 && !*abort_flag) {
-                if (r + 1 < NC) {
-                    tma_store_wait_read();
-                    issue_in(r + 1);
-                }
-                mbar_wait(&bar[BAR_WU], par, abort_flag, status);
-                tc_fence_after();
-                // group A: G2 Sc = Q Kbar^T; D2 WH = W Hm
-                for (int k = 0; k < 8; ++k) {
-                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
-                }
-                for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dWW + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM,
-                             k != 0);
-                mma_commit(&bar[BAR_GA]);
-            }
-            mbar_wait(&bar[BAR_GA], par, abort_flag, status);
-            tc_fence_after();
+            fc = slot_f(s, MS_SCAL)[1];
             const float rqi = slot_f(s, MS_RQ)[i];
+            const float mqi = slot_f(s, MS_MQ)[i];
+            const float iti = slot_f(s, MS_ITI)[i];
+            const float qni = slot_f(s, MS_QN)[i];
+            const float lt = slot_f(s, MS_LT)[i];
+            const float ep = slot_f(s, MS_EP)[i];
+            // ---- W' of the CCQ mean fold
+            mbar_wait(&bar[BAR_GA1], par, abort_flag, status);
+            tc_fence_after();
+            float c = 0.f;
             {
-                // W' of the CCQ mean fold (as in the GLA kernel)
                 float sc[32];
                 tmem_ld16x2_32<32>(tq + TM_SA, sc);
-                float part = 0.f;
+                float pa[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int jj = 0; jj < 32; ++jj)
-                    if (32 * hf + jj <= i) part += sc[jj];
+                    if (32 * hf + jj <= i) pa[jj & 3] += sc[jj];
+                float part = (pa[0] + pa[1]) + (pa[2] + pa[3]);
                 part += __shfl_xor_sync(0xffffffffu, part, 16);
-                const float cq = slot_f(s, MS_MQ)[i] + rqi * part;
-                const float c = a.centered ? cq / ti : 0.f;
-                if (hf == 0) cv[i] = c;
-                const float cn = c / rqi;
+                const float cq = mqi + rqi * part;
+                c = a.centered ? cq * iti : 0.f;
+                const float cn = c * qni;
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
+                for (int q2 = 0; q2 < 2; ++q2) {
                     float w[8];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                        const int j = 32 * hf + 8 * q4 + e;
-                        w[e] = (j <= i) ? sc[8 * q4 + e] - cn : 0.f;
+                        const int jj = 8 * q2 + e;
+                        const float v = grp ? sc[16 + jj] : sc[jj];
+                        w[e] = (32 * hf + 16 * grp + jj <= i) ? v - cn : 0.f;
                     }
-                    store_row_chunk(sm + OFF_WM, i, 4 * hf + q4, w);
+                    store_row_chunk(sm + OFF_WM, i, 4 * hf + 2 * grp + q2, w);
                 }
-                // U = Ut - W Hm  -> bf16 U tile (row i)
-                uint8_t *ut = sm + OFF_UT + hf * 8192;
-                uint8_t *ub = sm + OFF_UB + hf * 8192;
+            }
+            // ---- U = Ut - W Hm: read W Hm out of the P/O accumulator first, freeing it for G1
+            mbar_wait(&bar[BAR_GA2], par, abort_flag, status);
+            tc_fence_after();
+            {
+                float x[32];
+                tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);  // columns 64 grp + 32 hf ..
+                tc_fence_before();
+                named_bar_arrive(NB_PO, kSyncCount);
+                const uint8_t *ut = sm + OFF_UT + grp * 8192;
+                uint8_t *ub = sm + OFF_UB + grp * 8192;
 #pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    float x[32];
-                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, x);
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const uint4 u4 = *reinterpret_cast<const uint4 *>(ut + t64_chunk(i, 4 * hf + q4));
+                    const uint32_t uw[4] = {u4.x, u4.y, u4.z, u4.w};
+                    uint32_t ow[4];
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        const int cc = 4 * h2 + q4;
-                        float u8[8];
-                        unpack_bf16x8(*reinterpret_cast<const uint4 *>(ut + t64_chunk(i, cc)), u8);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) u8[e] -= x[8 * q4 + e];
-                        store_row_chunk(ub, i, cc, u8);
-                    }
+                    for (int w = 0; w < 4; ++w)
+                        ow[w] = bf16x2_from_f2(f2_add(f2_from_bf16x2(uw[w]),
+                                                      f2_make(-x[8 * q4 + 2 * w], -x[8 * q4 + 2 * w + 1])));
+                    *reinterpret_cast<uint4 *>(ub + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                if (r + 1 < NC) issue_wu(r + 1);  // Ut and W of this chunk are consumed
-                tc_fence_after();
-                // group B: G1 P = Q S^K; G3 P += W' Kbar
-                for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
-                             dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dKm + k * 128, ID_64x128_KM, 1);
-                mma_commit(&bar[BAR_GB]);
-            }
+            named_bar_arrive(NB_W, kSyncCount);
             // ---- q_clean (Eq. clean) scaled by e^{gc_i - gc_m}, into the Q tile
             {
-                uint8_t *qt = slot + SO_Q + hf * 8192;
-                const float *Mst = slot_f(s, MS_MST) + 64 * hf;
-                uint4 qraw[8];
+                uint8_t *qt = slot + SO_Q + grp * 8192;
+                const float *Mst = slot_f(s, MS_MST) + 64 * grp + 32 * hf;
+                uint4 qraw[4];
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc) qraw[cc] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, cc));
-                const float lt = slot_f(s, MS_LAM)[i] / ti;
-                const float ep = slot_f(s, MS_EP)[i];
+                for (int q4 = 0; q4 < 4; ++q4) qraw[q4] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, 4 * hf + q4));
                 mbar_wait(&bar[BAR_GB], par, abort_flag, status);
                 tc_fence_after();
-                const float cm = lt * cv[i];
+                const float cm = lt * c;
+                float p[32];
+                tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
+                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqi, rqi), cm2 = f2_make(cm, cm),
+                               ep2 = f2_make(ep, ep);
 #pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    float p[32];
-                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, p);
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4);
+                    const ulonglong2 m23 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4 + 4);
+                    const uint64_t mp[4] = {m01.x, m01.y, m23.x, m23.y};
+                    const uint32_t qw[4] = {qraw[q4].x, qraw[q4].y, qraw[q4].z, qraw[q4].w};
+                    uint32_t ow[4];
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        const int cc = 4 * h2 + q4;
-                        float qr[8], out[8];
-                        unpack_bf16x8(qraw[cc], qr);
-                        const float4 m0 = *reinterpret_cast<const float4 *>(Mst + 8 * cc);
-                        const float4 m1 = *reinterpret_cast<const float4 *>(Mst + 8 * cc + 4);
-                        const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
-#pragma unroll
-                        for (int e = 0; e < 8; ++e)
-                            out[e] = ep * fmaf(rqi, fmaf(-lt, p[8 * q4 + e], qr[e]), cm * mv[e]);
-                        store_row_chunk(qt, i, cc, out);
+                    for (int w = 0; w < 4; ++w) {
+                        const uint64_t p2 = f2_make(p[8 * q4 + 2 * w], p[8 * q4 + 2 * w + 1]);
+                        const uint64_t t = f2_fma(nlt, p2, f2_from_bf16x2(qw[w]));
+                        const uint64_t u = f2_fma(rq2, t, f2_mul(cm2, mp[w]));
+                        ow[w] = bf16x2_from_f2(f2_mul(ep2, u));
                     }
+                    *reinterpret_cast<uint4 *>(qt + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+                }
+            }
+            // e^{gc_m - gc_j} of this thread's 16 key columns, read before the slot is released
+            float ev[16];
+            {
+                const float4 *en4 = reinterpret_cast<const float4 *>(slot_f(s, MS_EN) + 32 * hf + 16 * grp);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 e4 = en4[q];
+                    ev[4 * q] = e4.x; ev[4 * q + 1] = e4.y; ev[4 * q + 2] = e4.z; ev[4 * q + 3] = e4.w;
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                tc_fence_after();
-                // group C: D4 QK = Qc Kbar^T; D3 O = Qc Hm
-                for (int k = 0; k < 8; ++k) {
-                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
-                }
-                mma_commit(&bar[BAR_GC]);
-                for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM,
-                             k != 0);
-                mma_commit(&bar[BAR_GC2]);
-                // group S: D6 X += Kd^T U; G8 S^K += Kbar^T Kbar
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_S, dKDm + k * 128, dUBm + k * 128, ID_128x128_MM, 1);
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
-                mma_commit(&bar[BAR_GS]);
+            named_bar_arrive(NB_QC, kSyncCount);
+            // ---- S^K_{r+1} while D4 runs
+            if (r + 1 < NC) {
+                mbar_wait(&bar[BAR_GK], par, abort_flag, status);
+                snap_sk();
             }
             // ---- Pm_ij = [j<=i] QK_ij e^{gc_m - gc_j}
             mbar_wait(&bar[BAR_GC], par, abort_flag, status);
             tc_fence_after();
             {
-                const float *en = slot_f(s, MS_EN) + 32 * hf;
                 float sc[32];
                 tmem_ld16x2_32<32>(tq + TM_SA, sc);
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    const float4 e0 = *reinterpret_cast<const float4 *>(en + 8 * q4);
-                    const float4 e1 = *reinterpret_cast<const float4 *>(en + 8 * q4 + 4);
-                    const float ev[8] = {e0.x, e0.y, e0.z, e0.w, e1.x, e1.y, e1.z, e1.w};
+                for (int q2 = 0; q2 < 2; ++q2) {
                     float w[8];
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
-                        const int j = 32 * hf + 8 * q4 + e;
-                        w[e] = (j <= i) ? sc[8 * q4 + e] * ev[e] : 0.f;
+                        const int jj = 8 * q2 + e;
+                        const float v = grp ? sc[16 + jj] : sc[jj];
+                        w[e] = (32 * hf + 16 * grp + jj <= i) ? v * ev[jj] : 0.f;
                     }
-                    store_row_chunk(sm + OFF_WM, i, 4 * hf + q4, w);
+                    store_row_chunk(sm + OFF_WM, i, 4 * hf + 2 * grp + q2, w);
                 }
             }
             fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                tc_fence_after();
-                // group D: D5 O += Pm U
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dUBm + k * 128, ID_64x128_KM, 1);
-                mma_commit(&bar[BAR_GD]);
-            }
+            named_bar_arrive(NB_MASK, kSyncCount);
+            // ---- output o = scale O, staged in the U tile for the TMA store
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             {
-                uint8_t *ot = slot + SO_Q + hf * 8192;
+                float x[32];
+                tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
 #pragma unroll
-                for (int h2 = 0; h2 < 2; ++h2) {
-                    float x[32];
-                    tmem_ld16x2_32<64>(tq + TM_PO + 32 * h2, x);
+                for (int e = 0; e < 32; ++e) x[e] *= a.scale;
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) x[e] *= a.scale;
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(ot, i, 4 * h2 + q4, x + 8 * q4);
-                }
+                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_UB + grp * 8192, i, 4 * hf + q4, x + 8 * q4);
+                fence_proxy_async_smem();
             }
-            fence_proxy_async_smem();
             tc_fence_before();
-            named_bar(1, 128);
-            if (tid == 0 && !*abort_flag) {
-                tma_store_4d(&map_o, slot + SO_Q, 0, h, c0, b);
-                tma_store_4d(&map_o, slot + SO_Q + 8192, 64, h, c0, b);
-                tma_store_commit();
+            named_bar_arrive(NB_OUT, kSyncCount);
+            // ---- Hm_{r+1} while G2 of chunk r+1 runs (D3, D6 of chunk r have run: GD follows them)
+            if (r + 1 < NC) {
+                mbar_wait(&bar[BAR_PREP0 + (s ^ 1)], ((r + 1) >> 1) & 1, abort_flag, status);
+                snap_s(fc * slot_f(s ^ 1, MS_SCAL)[0]);
             }
         }
-        if (tid == 0) tma_store_wait_all();
-    } else if (wg == 1) {
-        // =============================================================== WG1: prep
-        float lam_reg = 0.f, g_reg = 0.f;
-        if (wt < 64) lam_reg = (wt < T) ? a.lambda[(static_cast<size_t>(b) * T + wt) * H + h] : 0.f;
-        else g_reg = (wt - 64 < T) ? a.g[(static_cast<size_t>(b) * T + (wt - 64)) * H + h] : 0.f;
+        // final states: H_T = e^{gc_C - gc_m} X (last chunk), S^K
+        if (NC > 0) {
+            tc_fence_after();
+            const size_t bhs = static_cast<size_t>(bh);
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc) {
+                const int cl = 2 * grp + cc;
+                float x[32];
+                tmem_ld32(tq + TM_S + 32 * cl, x);
+                if (a.ST) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * cl);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        dst[e] = make_float4(fc * x[4 * e], fc * x[4 * e + 1], fc * x[4 * e + 2], fc * x[4 * e + 3]);
+                }
+                tmem_ld32(tq + TM_SK + 32 * cl, x);
+                if (a.CT) {
+                    float4 *dst = reinterpret_cast<float4 *>(a.CT + (bhs * kD + row) * kD + 32 * cl);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+                }
+            }
+        }
+    } else if (warp < kIssueWarp) {
+        // =============================================================== PREP
+        const int wt = tid - 32 * kPrepWarp0;
+        float lam_reg, g_reg;
+        {
+            const int tn = wt >> 1;
+            lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+            g_reg = (wt < 64 && wt < T) ? a.g[(static_cast<size_t>(b) * T + wt) * H + h] : 0.f;
+        }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1;
@@ -705,54 +764,74 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             float *scal = slot_f(s, MS_SCAL);
             mbar_wait(&bar[BAR_IN0 + s], sp, abort_flag, status);
             if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
-            if (wt < 64) {
-                slot_f(s, MS_LAM)[wt] = lam_reg;
-                const int tn = (r + 1) * kC + wt;
-                lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
-            } else {
-                scal[2 + wt - 64] = g_reg;
-                const int tn = (r + 1) * kC + wt - 64;
-                g_reg = (tn < T) ? a.g[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
-            }
-            named_bar(2, 128);
-            // row norms and M . qbar; in-chunk cumulative decay (one thread)
+            const float lam_cur = lam_reg;
+            if (wt < 64) scal[2 + wt] = g_reg;
             {
-                const int j = wt & 63;
-                const bool isq = wt < 64;
-                const uint8_t *base = slot + (isq ? SO_Q : SO_K);
-                float ss = 0.f, md = 0.f;
+                const int tn = (r + 1) * kC + (wt >> 1);
+                lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+                const int tg = (r + 1) * kC + wt;
+                g_reg = (wt < 64 && tg < T) ? a.g[(static_cast<size_t>(b) * T + tg) * H + h] : 0.f;
+            }
+            named_bar(NB_PREP, 128);  // key sum and raw decays visible
+            // in-chunk cumulative log decay gc: one warp, a shuffle scan over two tokens a lane
+            if (wt < 32) {
+                const float x0 = scal[2 + 2 * lane], x1 = scal[2 + 2 * lane + 1];
+                float pv = x0 + x1;
 #pragma unroll
-                for (int t64 = 0; t64 < 2; ++t64) {
+                for (int o = 1; o < 32; o <<= 1) {
+                    const float y = __shfl_up_sync(0xffffffffu, pv, o);
+                    if (lane >= o) pv += y;
+                }
+                scal[2 + 2 * lane] = pv - x1;
+                scal[2 + 2 * lane + 1] = pv;
+            }
+            // row norms of q and k and M . q (thread pair per row, one T64 tile each)
+            {
+                const int j = wt >> 1, hh = wt & 1;
+                uint4 qv[8], kv[8];
 #pragma unroll
-                    for (int cc = 0; cc < 8; ++cc) {
-                        float f[8];
-                        unpack_bf16x8(*reinterpret_cast<const uint4 *>(base + t64 * 8192 + t64_chunk(j, cc)), f);
-                        const float4 m0 = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc);
-                        const float4 m1 = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc + 4);
-                        const float mv[8] = {m0.x, m0.y, m0.z, m0.w, m1.x, m1.y, m1.z, m1.w};
+                for (int cc = 0; cc < 8; ++cc) {
+                    qv[cc] = *reinterpret_cast<const uint4 *>(slot + SO_Q + hh * 8192 + t64_chunk(j, cc));
+                    kv[cc] = *reinterpret_cast<const uint4 *>(slot + SO_K + hh * 8192 + t64_chunk(j, cc));
+                }
+                const float *Mh = Mst + 64 * hh;
+                uint64_t sq0 = 0, sq1 = 0, sk0 = 0, sk1 = 0, md0 = 0, md1 = 0;
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            ss = fmaf(f[e], f[e], ss);
-                            if (isq) md = fmaf(f[e], mv[e], md);
+                for (int cc = 0; cc < 8; ++cc) {
+                    const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc);
+                    const ulonglong2 m23 = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc + 4);
+                    const uint32_t qw[4] = {qv[cc].x, qv[cc].y, qv[cc].z, qv[cc].w};
+                    const uint32_t kw[4] = {kv[cc].x, kv[cc].y, kv[cc].z, kv[cc].w};
+                    const uint64_t mp[4] = {m01.x, m01.y, m23.x, m23.y};
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        const uint64_t q2 = f2_from_bf16x2(qw[w]), k2 = f2_from_bf16x2(kw[w]);
+                        if (w & 1) {
+                            sq1 = f2_fma(q2, q2, sq1); sk1 = f2_fma(k2, k2, sk1); md1 = f2_fma(q2, mp[w], md1);
+                        } else {
+                            sq0 = f2_fma(q2, q2, sq0); sk0 = f2_fma(k2, k2, sk0); md0 = f2_fma(q2, mp[w], md0);
                         }
                     }
                 }
-                const float rn = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
-                if (isq) {
-                    slot_f(s, MS_RQ)[j] = rn;
-                    slot_f(s, MS_MQ)[j] = md * rn;
+                const float2 a0 = f2_split(f2_add(sq0, sq1)), b0 = f2_split(f2_add(sk0, sk1)),
+                             c0v = f2_split(f2_add(md0, md1));
+                float ssq = a0.x + a0.y, ssk = b0.x + b0.y, mdt = c0v.x + c0v.y;
+                ssq += __shfl_xor_sync(0xffffffffu, ssq, 1);
+                ssk += __shfl_xor_sync(0xffffffffu, ssk, 1);
+                mdt += __shfl_xor_sync(0xffffffffu, mdt, 1);
+                if (hh == 0) {
+                    const float rq = a.l2norm ? rsqrtf(fmaxf(ssq, 1e-12f)) : 1.f;
+                    const float iti = 1.f / static_cast<float>(t0 + r * kC + j + 1);
+                    slot_f(s, MS_RQ)[j] = rq;
+                    slot_f(s, MS_MQ)[j] = mdt * rq;
+                    slot_f(s, MS_ITI)[j] = iti;
+                    slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(ssq, 1e-12f) * rq : 1.f;
+                    slot_f(s, MS_LT)[j] = lam_cur * iti;
                 } else {
-                    slot_f(s, MS_RK)[j] = rn;
-                }
-                if (wt == 127) {
-                    float run = 0.f;
-                    for (int t = 0; t < 64; ++t) {
-                        run += scal[2 + t];
-                        scal[2 + t] = run;
-                    }
+                    slot_f(s, MS_RK)[j] = a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
                 }
             }
-            named_bar(2, 128);
+            named_bar(NB_PREP, 128);  // gc, rk visible
             if (wt < 64) {
                 const float gm = scal[2 + 31];
                 slot_f(s, MS_EP)[wt] = fast_exp2((scal[2 + wt] - gm) * kLog2e);
@@ -762,38 +841,50 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     scal[1] = fast_exp2((scal[2 + 63] - gm) * kLog2e);
                 }
             }
-            named_bar(2, 128);
-            // kbar (in place) and Kd = kbar e^{gc_m - gc}: thread = (row, column half)
+            named_bar(NB_PREP, 128);  // e^{gc_m - gc} visible
+            // kbar (in place) and Kd = kbar e^{gc_m - gc}: thread = (row, T64 tile)
             {
-                const int j = wt >> 1, hf = wt & 1;
+                const int j = wt >> 1, hh = wt & 1;
                 const float rkj = slot_f(s, MS_RK)[j], enj = slot_f(s, MS_EN)[j];
-                uint8_t *kt = slot + SO_K + hf * 8192;
-                uint8_t *kd = slot + SO_KD + hf * 8192;
+                const uint64_t rk2 = f2_make(rkj, rkj), en2 = f2_make(enj, enj);
+                uint8_t *kt = slot + SO_K + hh * 8192;
+                uint8_t *kd = slot + SO_KD + hh * 8192;
+                uint4 kv[8];
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc) kv[cc] = *reinterpret_cast<const uint4 *>(kt + t64_chunk(j, cc));
 #pragma unroll
                 for (int cc = 0; cc < 8; ++cc) {
-                    float f[8], g8[8];
-                    unpack_bf16x8(*reinterpret_cast<const uint4 *>(kt + t64_chunk(j, cc)), f);
+                    const uint32_t kw[4] = {kv[cc].x, kv[cc].y, kv[cc].z, kv[cc].w};
+                    uint32_t ob[4], od[4];
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        f[e] *= rkj;
-                        g8[e] = f[e] * enj;
+                    for (int w = 0; w < 4; ++w) {
+                        const uint64_t kb2 = f2_mul(f2_from_bf16x2(kw[w]), rk2);
+                        ob[w] = bf16x2_from_f2(kb2);
+                        od[w] = bf16x2_from_f2(f2_mul(kb2, en2));
                     }
-                    store_row_chunk(kt, j, cc, f);
-                    store_row_chunk(kd, j, cc, g8);
+                    *reinterpret_cast<uint4 *>(kt + t64_chunk(j, cc)) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+                    *reinterpret_cast<uint4 *>(kd + t64_chunk(j, cc)) = make_uint4(od[0], od[1], od[2], od[3]);
                 }
             }
             fence_proxy_async_smem();
-            named_bar(2, 128);
-            // key sum of the chunk, per key dim (from the bf16 kbar tile)
+            named_bar(NB_PREP, 128);
+            // key sum of the chunk (from the bf16 kbar tile): thread = (dim pair, token half)
             {
-                const int d = wt;
-                const uint8_t *kt = slot + SO_K + (d >> 6) * 8192;
-                float sum = 0.f;
-                for (int j = 0; j < 64; ++j)
-                    sum += __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(kt + t64_offset(j, d & 63)));
-                dmprev[d] = sum;
+                const int p = wt & 63, th = wt >> 6, d0 = 2 * p;
+                const uint8_t *kt = slot + SO_K + (d0 >> 6) * 8192;
+                uint64_t acc0 = 0, acc1 = 0;
+#pragma unroll
+                for (int jj = 0; jj < 32; jj += 2) {
+                    const int j = 32 * th + jj;
+                    acc0 = f2_add(acc0, f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(kt + t64_offset(j, d0 & 63))));
+                    acc1 = f2_add(acc1, f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(kt + t64_offset(j + 1, d0 & 63))));
+                }
+                const float2 sv = f2_split(f2_add(acc0, acc1));
+                dmp[th * kD + d0] = sv.x;
+                dmp[th * kD + d0 + 1] = sv.y;
             }
-            named_bar(2, 128);
+            named_bar(NB_PREP, 128);
+            dmprev[wt] = dmp[wt] + dmp[kD + wt];
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
         }
         if (NC > 0 && a.mT) {
@@ -801,60 +892,118 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
     } else {
-        // =============================================================== WG2: states
-        const int row = 32 * (warp & 3) + lane;
+        // =============================================================== ISSUE
+        const bool lead = lane == 0;
+        const uint64_t dWm = make_desc(sb + OFF_WM, 16, 1024);
+        const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
+        const uint64_t dHB = make_desc(sb + OFF_HB, 16384, 1024);
+        const uint64_t dWW = make_desc(sb + OFF_WW, 16, 1024);
+        const uint64_t dUBm = make_desc(sb + OFF_UB, 8192, 1024);
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
-            const uint32_t sp = (r >> 1) & 1;
-            if (r > 0) mbar_wait(&bar[BAR_GS], (r - 1) & 1, abort_flag, status);
+            const uint32_t sp = (r >> 1) & 1, par = r & 1;
+            const uint32_t ss = sb + s * SLOT_BYTES;
+            const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
+            const uint64_t dK = make_desc(ss + SO_K, 16, 1024);
+            const uint64_t dKm = make_desc(ss + SO_K, 8192, 1024);
+            const uint64_t dKDm = make_desc(ss + SO_KD, 8192, 1024);
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
             tc_fence_after();
-            const float hs = (r > 0 ? slot_f(s ^ 1, MS_SCAL)[1] : 1.f) * slot_f(s, MS_SCAL)[0];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_S + 32 * c, x);
-#pragma unroll
-                for (int e = 0; e < 32; ++e) x[e] *= hs;
-                uint8_t *tile = sm + OFF_HB + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
-                tmem_st32(tq + TM_S + 32 * c, x);
+            // G2 Sc = Q Kbar^T (SA is free: the Pm epilogue of chunk r-1 has read it)
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 8; ++k) {
+                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
+                }
+                mma_commit(&bar[BAR_GA1]);
             }
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_SK + 32 * c, x);
-                uint8_t *tile = sm + OFF_SK + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
+            __syncwarp();
+            if (r > 0) {
+                // O of chunk r-1 is staged in the U tile: store it
+                mbar_wait(&bar[BAR_GD], (r - 1) & 1, abort_flag, status);
+                named_bar(NB_OUT, kSyncCount);
+                if (lead) {
+                    tma_store_4d(&map_o, sm + OFF_UB, 0, h, (r - 1) * kC, b);
+                    tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (r - 1) * kC, b);
+                    tma_store_commit();
+                }
+                __syncwarp();
             }
-            tmem_wait_st();
-            fence_proxy_async_smem();
-            tc_fence_before();
-            named_bar(3, 128);
-            if (wt == 0) mbar_arrive(&bar[BAR_SNAP]);
+            // D2 WH = W Hm (needs Ut/W of the chunk and the Hm copy)
+            mbar_wait(&bar[BAR_WU], par, abort_flag, status);
+            mbar_wait(&bar[BAR_SNAPS], par, abort_flag, status);
+            tc_fence_after();
+            if (lead && !*abort_flag)
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dWW + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
+            // the U tile is rewritten once GA2 lets EPI in: the output store must have read it
+            if (lead) {
+                tma_store_wait_read();
+                if (!*abort_flag) mma_commit(&bar[BAR_GA2]);
+            }
+            __syncwarp();
+            // G1 P = Q S^K once WH is out of the accumulator
+            named_bar(NB_PO, kSyncCount);
+            mbar_wait(&bar[BAR_SNAPK], par, abort_flag, status);
+            tc_fence_after();
+            if (lead && !*abort_flag)
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
+                             dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
+            __syncwarp();
+            // G3 P += W' Kbar, G8 S^K += Kbar^T Kbar, D6 X += Kd^T U
+            named_bar(NB_W, kSyncCount);
+            tc_fence_after();
+            if (lead && !*abort_flag) {
+                if (r + 1 < NC) issue_wu(r + 1);  // Ut and W of this chunk are consumed
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GB]);
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
+                mma_commit(&bar[BAR_GK]);
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_S, dKDm + k * 128, dUBm + k * 128, ID_128x128_MM, 1);
+            }
+            __syncwarp();
+            // D4 QK = Qc Kbar^T, D3 O = Qc Hm
+            named_bar(NB_QC, kSyncCount);
+            tc_fence_after();
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 8; ++k) {
+                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
+                }
+                mma_commit(&bar[BAR_GC]);
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
+                mma_commit(&bar[BAR_GC2]);
+            }
+            __syncwarp();
+            // D5 O += Pm U
+            named_bar(NB_MASK, kSyncCount);
+            tc_fence_after();
+            if (lead && !*abort_flag) {
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dUBm + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GD]);
+            }
+            __syncwarp();
+            // the slot's last MMA reader (D3) is done: load chunk r + 2 into it
+            if (r + 2 < NC) {
+                mbar_wait(&bar[BAR_GC2], par, abort_flag, status);
+                if (lead && !*abort_flag) issue_in(r + 2);
+                __syncwarp();
+            }
         }
         if (NC > 0) {
-            mbar_wait(&bar[BAR_GS], (NC - 1) & 1, abort_flag, status);
-            tc_fence_after();
-            const float fs = slot_f((NC - 1) & 1, MS_SCAL)[1];
-            const size_t bhs = static_cast<size_t>(bh);
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_S + 32 * c, x);
-                if (a.ST) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * c);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        dst[e] = make_float4(fs * x[4 * e], fs * x[4 * e + 1], fs * x[4 * e + 2], fs * x[4 * e + 3]);
-                }
-                tmem_ld32(tq + TM_SK + 32 * c, x);
-                if (a.CT) {
-                    float4 *dst = reinterpret_cast<float4 *>(a.CT + (bhs * kD + row) * kD + 32 * c);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+            mbar_wait(&bar[BAR_GD], (NC - 1) & 1, abort_flag, status);
+            named_bar(NB_OUT, kSyncCount);
+            if (lead) {
+                tma_store_4d(&map_o, sm + OFF_UB, 0, h, (NC - 1) * kC, b);
+                tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (NC - 1) * kC, b);
+                tma_store_commit();
+                tma_store_wait_all();
+                if (*abort_flag) {
+                    // after a give-up, wait (bounded) for the copies still in flight
+                    mbar_drain(&bar[BAR_WU], (NC - 1) & 1);
+                    for (int r = (NC > 2 ? NC - 2 : 0); r < NC; ++r) mbar_drain(&bar[BAR_IN0 + (r & 1)], (r >> 1) & 1);
                 }
             }
         }
