@@ -130,8 +130,9 @@ CCQ_API ccq_status ccq_gla_workspace_size(int B, int T, int H, int Dk, int Dv, c
  *   g         log decay log(alpha) [B,T,H] fp32 (<= 0);  beta [B,T,H] fp32 in [0,1].
  *   workspace caller-owned device scratch of at least the size ccq_gdn_workspace_size()
  *             reports (16-byte aligned), used by the chunkwise kernel to hold the
- *             per-chunk WY/UT matrices; may be NULL when that size is 0.  Its contents
- *             on entry do not matter and are undefined on return.
+ *             per-chunk UT factor Tt diag(beta) (64 x 64 bf16 per chunk); may be NULL
+ *             when that size is 0.  Its contents on entry do not matter and are
+ *             undefined on return.
  * All other arguments as ccq_gla_fwd.  bf16 inputs with Dk = Dv = 128 run the chunkwise
  * tensor-core kernels (CCQ_ALGO_AUTO / CHUNKWISE; CCQ_ERR_INVALID_ARG if the workspace is
  * missing or too small); other inputs run the recurrent kernel.

@@ -146,11 +146,11 @@ bool make_token_map(CUtensorMap *map, const void *base, int elem_bytes, int B, i
     return r == CUDA_SUCCESS;
 }
 
-bool make_rows_map(CUtensorMap *map, const void *base, long long rows) {
+bool make_rows_map(CUtensorMap *map, const void *base, long long rows, int cols) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
-    const cuuint64_t dims[2] = {128, static_cast<cuuint64_t>(rows)};
-    const cuuint64_t strides[1] = {128 * 2};
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
     const cuuint32_t box[2] = {64, 64};
     const cuuint32_t estr[2] = {1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box,
@@ -514,14 +514,12 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
         if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
         const int nc = (T + 63) / 64;
         const long long rows = static_cast<long long>(B) * H * nc * 64;
-        const __nv_bfloat16 *ut = static_cast<const __nv_bfloat16 *>(workspace);
-        const __nv_bfloat16 *w = ut + static_cast<size_t>(rows) * 128;
         GdnMaps maps;
         if (!make_token_map(&maps.q, q, 2, B, T, H, 128, 64, true) ||
             !make_token_map(&maps.k, k, 2, B, T, H, 128, 64, true) ||
             !make_token_map(&maps.v, v, 2, B, T, H, 128, 64, true) ||
             !make_token_map(&maps.o, o, 2, B, T, H, 128, 64, true) ||
-            !make_rows_map(&maps.ut, ut, rows) || !make_rows_map(&maps.w, w, rows))
+            !make_rows_map(&maps.tb, workspace, rows, 64))
             return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
         ChunkArgs a = {};
         a.B = B; a.T = T; a.H = H;

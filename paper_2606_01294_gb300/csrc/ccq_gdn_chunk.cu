@@ -5,22 +5,24 @@
 // chunk with start state H0, gc_i the in-chunk cumulative log-decay and gc_m its value at
 // the chunk midpoint (token 31), unrolling the recurrence gives (chunkwise form):
 //   A_ij = beta_i e^{gc_i - gc_j} kbar_i . kbar_j   (j < i),   Tt = (I + A)^{-1}
-//   U    = Tt diag(beta) V - Tt diag(beta e^{gc - gc_m}) Kbar (e^{gc_m} H0)  =  Ut - W Hm
+//   U    = Tt diag(beta) V - Tt diag(beta e^{gc - gc_m}) Kbar (e^{gc_m} H0)
+//        = Tb (V - Diag(e^{gc - gc_m}) Kbar Hm),   Tb = Tt diag(beta)
 //   o_i  = scale [ e^{gc_i - gc_m} q_clean_i Hm + sum_{j<=i} e^{gc_i - gc_j}(q_clean_i . kbar_j) U_j ]
 //   H_C  = e^{gc_C - gc_m} [ Hm + sum_j e^{gc_m - gc_j} kbar_j U_j^T ]
-// with Hm = e^{gc_m} H0.  Ut and W depend only on the chunk's own inputs, so they are
-// computed for every chunk in parallel by gdn_wy_kernel (into a caller workspace);
-// gdn_chunk_kernel then walks the chunks of each (batch, head) sequentially with the
-// same warp-specialised structure as the GLA kernel and the same CCQ read (App. B):
+// with Hm = e^{gc_m} H0.  Tb depends only on the chunk's own keys, gates and betas, so it
+// is computed for every chunk in parallel by gdn_wy_kernel (64 x 64 bf16 per chunk, into a
+// caller workspace); gdn_chunk_kernel then walks the chunks of each (batch, head)
+// sequentially with the same warp-specialised structure as the GLA kernel and the same CCQ
+// read (App. B):
 //
-//   group A  G2  Sc  = Q Kbar^T          D2  WH = W Hm
-//   (epilogue: W' of the CCQ mean fold;  U = Ut - WH -> bf16 U tile)
-//   group B  G1  P   = Q S^K             G3  P += W' Kbar
-//   (epilogue: q_clean e^{gc - gc_m} into the Q tile)
-//   group C  D4  QK  = Qc Kbar^T         D3  O  = Qc Hm
-//   group S  D6  X  += Kd^T U            G8  S^K += Kbar^T Kbar      (Kd = kbar e^{gc_m - gc})
+//   G2  Sc  = Q Kbar^T           D2  KH = Kbar Hm
+//   (epilogue: W' of the CCQ mean fold;  R = V - Diag(e^{gc - gc_m}) KH -> bf16 R tile)
+//   G1  P   = Q S^K              DU  U = Tb R            G3  P += W' Kbar
+//   (epilogue: U -> bf16 U tile; q_clean e^{gc - gc_m} into the Q tile)
+//   D6  X  += Kd^T U             G8  S^K += Kbar^T Kbar      (Kd = kbar e^{gc_m - gc})
+//   D4  QK  = Qc Kbar^T          D3  O  = Qc Hm
 //   (epilogue: Pm_ij = [j<=i] QK_ij e^{gc_m - gc_j})
-//   group D  D5  O  += Pm U
+//   D5  O  += Pm U
 //   (epilogue: o = scale O, TMA store)
 // X = e^{gc_m - gc_C} H_{r+1} stays in TMEM; the scalar e^{gc_C - gc_m} is applied at the
 // next snapshot.
@@ -51,30 +53,25 @@ __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chun
 
 // ============================================================================ WY kernel
 //
-// One CTA (128 threads) per (batch, head, chunk).  Writes Ut and W as bf16 rows
-// [((b*H + h)*NC + r)*64 + i][0..127] of the workspace.
+// One CTA (128 threads, four per SM) per (batch, head, chunk).  Writes Tb = Tt diag(beta)
+// as the bf16 rows [((b*H + h)*NC + r)*64 + i][0..63] of the workspace.
 
-constexpr uint32_t WY_K = 0;        // 16K  k raw -> kbar; later staging of W
-constexpr uint32_t WY_V = 16384;    // 16K  v; later staging of Ut
-constexpr uint32_t WY_A = 32768;    // 64 x 68 fp32: A; after the inversion the two bf16 tiles:
-constexpr uint32_t WY_TB = 32768;   //   8K  bf16 Tt diag(beta)               ([64][64] T64 tile)
-constexpr uint32_t WY_TG = 40960;   //   8K  bf16 Tt diag(beta e^{gc - gc_m})
-constexpr uint32_t WY_T = 50176;    // 64 x 68 fp32: Tt
-constexpr uint32_t WY_Y = 67584;    // 3 x 256 fp32: block products
-constexpr uint32_t WY_MISC = 70656; // gc, beta, factors, rk, barrier
-constexpr uint32_t WY_SMEM = WY_MISC + 2048 + 1024;  // 73.7 KB: three CTAs per SM
+constexpr uint32_t WY_K = 0;        // 16K  k raw -> kbar; after the KK product the block scratch Y
+constexpr uint32_t WY_A = 16384;    // 64 x 68 fp32: A; after the inversion the bf16 Tb tile (8K)
+constexpr uint32_t WY_T = 33792;    // 64 x 68 fp32: Tt
+constexpr uint32_t WY_MISC = 51200; // gc, beta, factors, rk, barriers
+constexpr uint32_t WY_SMEM = WY_MISC + 2048 + 1024;  // 54.3 KB: four CTAs per SM
 constexpr int kAS = 68;             // padded fp32 row stride of A and Tt
 
-__global__ void __launch_bounds__(128, 3)
-gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
-              const __grid_constant__ CUtensorMap map_ut, const __grid_constant__ CUtensorMap map_w,
+__global__ void __launch_bounds__(128, 4)
+gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_tb,
               const ChunkArgs a, int NC) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
     float *A = reinterpret_cast<float *>(sm + WY_A);
     float *Tt = reinterpret_cast<float *>(sm + WY_T);
-    float *Y = reinterpret_cast<float *>(sm + WY_Y);
+    float *Y = reinterpret_cast<float *>(sm + WY_K);               // 3 x 256 fp32, once kbar is dead
     float *gcs = reinterpret_cast<float *>(sm + WY_MISC);        // [64] cumulative log decay
     float *bet = gcs + 64;                                        // [64] beta
     float *epos = gcs + 128;                                      // [64] e^{gc - gc_m}
@@ -92,16 +89,14 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     int *status = a.status;
 
     if (tid == 0) {
-        for (int i = 0; i < 3; ++i) mbar_init(&bar[i], 1);
+        for (int i = 0; i < 2; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        mbar_arrive_expect_tx(&bar[0], 4 * 8192);
+        mbar_arrive_expect_tx(&bar[0], 2 * 8192);
         tma_load_4d(sm + WY_K, &map_k, &bar[0], 0, h, c0, b);
         tma_load_4d(sm + WY_K + 8192, &map_k, &bar[0], 64, h, c0, b);
-        tma_load_4d(sm + WY_V, &map_v, &bar[0], 0, h, c0, b);
-        tma_load_4d(sm + WY_V + 8192, &map_v, &bar[0], 64, h, c0, b);
     }
-    if (warp == 0) tmem_alloc(tslot, 128);
+    if (warp == 0) tmem_alloc(tslot, 64);
     if (tid < 64) {
         const int t = c0 + tid;
         const size_t row = (static_cast<size_t>(b) * T + t) * H + h;
@@ -126,18 +121,22 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         gcs[2 * lane + 1] = p;
     }
     mbar_wait(&bar[0], 0, abort_flag, status);
-    if (tid < 64) {
-        float ss = 0.f;
+    {
+        // row j = tid >> 1, one T64 tile (column half) per thread
+        const int j = tid >> 1, hh = tid & 1;
+        uint64_t s0 = 0, s1 = 0;
 #pragma unroll
-        for (int t64 = 0; t64 < 2; ++t64)
-#pragma unroll
-            for (int cc = 0; cc < 8; ++cc) {
-                float f[8];
-                unpack_bf16x8(*reinterpret_cast<const uint4 *>(sm + WY_K + t64 * 8192 + t64_chunk(tid, cc)), f);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) ss = fmaf(f[e], f[e], ss);
-            }
-        rk[tid] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+        for (int cc = 0; cc < 8; ++cc) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(sm + WY_K + hh * 8192 + t64_chunk(j, cc));
+            const uint64_t p0 = f2_from_bf16x2(v.x), p1 = f2_from_bf16x2(v.y), p2 = f2_from_bf16x2(v.z),
+                           p3 = f2_from_bf16x2(v.w);
+            s0 = f2_fma(p0, p0, s0); s1 = f2_fma(p1, p1, s1);
+            s0 = f2_fma(p2, p2, s0); s1 = f2_fma(p3, p3, s1);
+        }
+        const float2 sv = f2_split(f2_add(s0, s1));
+        float ss = sv.x + sv.y;
+        ss += __shfl_xor_sync(0xffffffffu, ss, 1);
+        if (hh == 0) rk[j] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
     }
     __syncthreads();
     if (tid < 64) {
@@ -149,14 +148,14 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     {
         const int j = tid >> 1, hf = tid & 1;
         const float s = rk[j];
+        const uint64_t s2 = f2_make(s, s);
         uint8_t *tile = sm + WY_K + hf * 8192;
 #pragma unroll
         for (int cc = 0; cc < 8; ++cc) {
-            float f[8];
-            unpack_bf16x8(*reinterpret_cast<const uint4 *>(tile + t64_chunk(j, cc)), f);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) f[e] *= s;
-            store_row_chunk(tile, j, cc, f);
+            const uint4 v = *reinterpret_cast<const uint4 *>(tile + t64_chunk(j, cc));
+            *reinterpret_cast<uint4 *>(tile + t64_chunk(j, cc)) =
+                make_uint4(bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.x), s2)), bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.y), s2)),
+                           bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.z), s2)), bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.w), s2)));
         }
     }
     fence_proxy_async_smem();
@@ -212,7 +211,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     // 16 threads per 16 x 16 block, each a 4 x 4 sub-tile with float4 shared loads
     for (int dist = 1; dist < 4; ++dist) {
         const int nblk = 4 - dist;
-        const int blk = tid >> 4, t = tid & 15, r0 = 4 * (t >> 2), c0 = 4 * (t & 3);
+        const int blk = tid >> 4, t = tid & 15, r0 = 4 * (t >> 2), cq = 4 * (t & 3);
         const int J = blk, I = blk + dist;
         if (blk < nblk) {
             float acc[4][4] = {};
@@ -223,7 +222,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
                         av[u] = *reinterpret_cast<const float4 *>(A + (16 * I + r0 + u) * kAS + 16 * K + m);
-                        tv[u] = *reinterpret_cast<const float4 *>(Tt + (16 * K + m + u) * kAS + 16 * J + c0);
+                        tv[u] = *reinterpret_cast<const float4 *>(Tt + (16 * K + m + u) * kAS + 16 * J + cq);
                     }
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
@@ -240,7 +239,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u)
-                *reinterpret_cast<float4 *>(Y + blk * 256 + (r0 + u) * 16 + c0) =
+                *reinterpret_cast<float4 *>(Y + blk * 256 + (r0 + u) * 16 + cq) =
                     make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
         }
         __syncthreads();
@@ -252,7 +251,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     av[u] = *reinterpret_cast<const float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * I + m);
-                    yv[u] = *reinterpret_cast<const float4 *>(Y + blk * 256 + (m + u) * 16 + c0);
+                    yv[u] = *reinterpret_cast<const float4 *>(Y + blk * 256 + (m + u) * 16 + cq);
                 }
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
@@ -268,83 +267,45 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u)
-                *reinterpret_cast<float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * J + c0) =
+                *reinterpret_cast<float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * J + cq) =
                     make_float4(-acc[u][0], -acc[u][1], -acc[u][2], -acc[u][3]);
         }
         __syncthreads();
     }
-    // zero the blocks above the diagonal, then the two scaled bf16 copies
+    // ---- Tb = Tt diag(beta) (zero above the diagonal) as the bf16 T64 tile in A's place
     {
         const int i = tid >> 1, hf = tid & 1;
 #pragma unroll
         for (int q4 = 0; q4 < 4; ++q4) {
-            float wb[8], wg[8];
+            float wb[8];
             const float4 t0 = *reinterpret_cast<const float4 *>(Tt + i * kAS + 32 * hf + 8 * q4);
             const float4 t1 = *reinterpret_cast<const float4 *>(Tt + i * kAS + 32 * hf + 8 * q4 + 4);
             const float tr[8] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int j = 32 * hf + 8 * q4 + e;
-                const float t = (j <= i) ? tr[e] : 0.f;  // A is dead: its space takes the tiles
-                wb[e] = t * bet[j];
-                wg[e] = wb[e] * epos[j];
+                wb[e] = (j <= i) ? tr[e] * bet[j] : 0.f;
             }
-            store_row_chunk(sm + WY_TB, i, 4 * hf + q4, wb);
-            store_row_chunk(sm + WY_TG, i, 4 * hf + q4, wg);
+            store_row_chunk(sm + WY_A, i, 4 * hf + q4, wb);
         }
     }
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
-    // ---- Ut = Tt diag(beta) V, then W = Tt diag(beta e^{gc-gc_m}) Kbar  (M = 64, N = 128, K = 64)
-    const size_t out_row = static_cast<size_t>(item) * kC;
-    for (int pass = 0; pass < 2; ++pass) {
-        if (tid == 0 && !*abort_flag) {
-            tc_fence_after();
-            const uint64_t da = make_desc(sb + (pass == 0 ? WY_TB : WY_TG), 16, 1024);
-            const uint64_t dbm = make_desc(sb + (pass == 0 ? WY_V : WY_K), 8192, 1024);
-            for (int k = 0; k < 4; ++k)
-                mma_bf16(tb, da + k * 2, dbm + k * 128, make_idesc(64, 128, 0, 1), k != 0);
-            mma_commit(&bar[2]);
-        }
-        mbar_wait(&bar[2], pass, abort_flag, status);
-        tc_fence_after();
-        {
-            const int i = 16 * warp + (lane & 15), hf = lane >> 4;
-            uint8_t *stage = sm + (pass == 0 ? WY_V : WY_K) + hf * 8192;  // operand no longer read
-#pragma unroll
-            for (int h2 = 0; h2 < 2; ++h2) {
-                float x[32];
-                tmem_ld16x2_32<64>(tq + 32 * h2, x);
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(stage, i, 4 * h2 + q4, x + 8 * q4);
-            }
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            const CUtensorMap *m = pass == 0 ? &map_ut : &map_w;
-            uint8_t *stage = sm + (pass == 0 ? WY_V : WY_K);
-            asm volatile(
-                "cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-                    reinterpret_cast<uint64_t>(m)),
-                "r"(smem_addr(stage)), "r"(0), "r"(static_cast<int>(out_row))
-                : "memory");
-            asm volatile(
-                "cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
-                    reinterpret_cast<uint64_t>(m)),
-                "r"(smem_addr(stage + 8192)), "r"(64), "r"(static_cast<int>(out_row))
-                : "memory");
-            tma_store_commit();
-        }
+    if (tid == 0 && !*abort_flag) {
+        asm volatile(
+            "cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                reinterpret_cast<uint64_t>(&map_tb)),
+            "r"(smem_addr(sm + WY_A)), "r"(0), "r"(item * kC)
+            : "memory");
+        tma_store_commit();
+        tma_store_wait_read();  // shared memory must outlive the store's read
     }
-    if (tid == 0) tma_store_wait_read();  // shared memory must outlive the stores' reads
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tb, 128);
+        tmem_dealloc(tb, 64);
     }
 }
 
@@ -358,10 +319,11 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 //                       TMEM lane quadrant w % 4 and split its columns.
 //   PREP  (warps 8-11)  prep of chunk r+1: row norms, cumulative decay, kbar, Kd.
 //   ISSUE (warp 12)     every tcgen05.mma and TMA copy, in the order
-//                       G2 D2 | G1 | G3 G8 D6 | D4 D3 | D5.  D2 (W Hm) lands in the P/O
-//                       accumulator, so EPI reads it out first and frees the accumulator
-//                       for G1 before it builds U.
-// The output is staged in the U tile (dead once D5 and D6 have run) and stored by TMA.
+//                       G2 D2 | G1 | DU G3 G8 | D4 D6 D3 | D5.  D2 (Kbar Hm) lands in the
+//                       P/O accumulator, so EPI reads it out first and frees the accumulator
+//                       for G1 before it builds R; U = Tb R lands in TMEM columns 384-511
+//                       (Sc has been read, QK comes later).
+// R, then U, then the output staging share one 16 KB tile.
 
 constexpr int kThreads = 416;
 constexpr int kEpiThreads = 256;
@@ -371,13 +333,13 @@ constexpr uint32_t SLOT_BYTES = 49152;
 constexpr uint32_t SO_Q = 0;        // raw q, then q_clean e^{gc - gc_m}
 constexpr uint32_t SO_K = 16384;    // raw k, then kbar
 constexpr uint32_t SO_KD = 32768;   // kbar e^{gc_m - gc}
-constexpr uint32_t OFF_UT = 98304;  // 16K  Ut of the chunk (workspace)
-constexpr uint32_t OFF_WW = 114688; // 16K  W of the chunk (workspace)
-constexpr uint32_t OFF_UB = 131072; // 16K  U (bf16, rows j); after D5 the output staging
-constexpr uint32_t OFF_WM = 147456; // 8K   W' of the CCQ fold, then Pm
-constexpr uint32_t OFF_SK = 155648; // 32K  bf16 S^K
-constexpr uint32_t OFF_HB = 188416; // 32K  bf16 Hm = e^{gc_m} H
-constexpr uint32_t OFF_MISC = 221184;
+constexpr uint32_t OFF_V = 98304;   // 16K  v of the chunk
+constexpr uint32_t OFF_TB = 114688; // 8K   Tb of the chunk (workspace), [64][64]
+constexpr uint32_t OFF_UB = 122880; // 16K  R, then U (bf16, rows j), after D5 the output staging
+constexpr uint32_t OFF_WM = 139264; // 8K   W' of the CCQ fold, then Pm
+constexpr uint32_t OFF_SK = 147456; // 32K  bf16 S^K
+constexpr uint32_t OFF_HB = 180224; // 32K  bf16 Hm = e^{gc_m} H
+constexpr uint32_t OFF_MISC = 212992;
 constexpr uint32_t MS_BYTES = 3072;
 constexpr uint32_t MS_RQ = 0, MS_MQ = 256, MS_LT = 512, MS_RK = 768, MS_EP = 1024, MS_EN = 1280,
                    MS_SCAL = 1536, MS_MST = 2048, MS_ITI = 2560, MS_QN = 2816;
@@ -399,7 +361,7 @@ enum {
 static_assert(M_BAR + 8 * kNumBars <= M_TMEM, "barrier area");
 enum { NB_PO = 1, NB_W = 2, NB_QC = 3, NB_MASK = 4, NB_OUT = 5, NB_PREP = 6, NB_EPI = 7 };
 
-constexpr uint32_t TM_S = 0, TM_SK = 128, TM_PO = 256, TM_SA = 384, kTmemCols = 512;
+constexpr uint32_t TM_S = 0, TM_SK = 128, TM_PO = 256, TM_SA = 384, TM_U = 384, kTmemCols = 512;
 constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
 constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
 constexpr uint32_t ID_64x128_KM = make_idesc(64, 128, 0, 1);
@@ -415,7 +377,7 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *m, uin
 
 __global__ void __launch_bounds__(kThreads, 1)
 gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
-                 const __grid_constant__ CUtensorMap map_ut, const __grid_constant__ CUtensorMap map_w,
+                 const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_tb,
                  const __grid_constant__ CUtensorMap map_o, const ChunkArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = smem_align1024(smem_raw);
@@ -459,14 +421,12 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_4d(base + SO_K, &map_k, bb, 0, h, r * kC, b);
         tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, r * kC, b);
     };
-    auto issue_wu = [&](int r) {
+    auto issue_wu = [&](int r) {  // v and Tb of chunk r
         uint64_t *bb = &bar[BAR_WU];
-        const int row = wrow0 + r * kC;
-        mbar_arrive_expect_tx(bb, 4 * 8192);
-        tma_load_2d(sm + OFF_UT, &map_ut, bb, 0, row);
-        tma_load_2d(sm + OFF_UT + 8192, &map_ut, bb, 64, row);
-        tma_load_2d(sm + OFF_WW, &map_w, bb, 0, row);
-        tma_load_2d(sm + OFF_WW + 8192, &map_w, bb, 64, row);
+        mbar_arrive_expect_tx(bb, 3 * 8192);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, r * kC, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, r * kC, b);
+        tma_load_2d(sm + OFF_TB, &map_tb, bb, 0, wrow0 + r * kC);
     };
 
     // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
@@ -502,8 +462,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     } else if (lane == 0) {
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_k);
-        tma_prefetch_desc(&map_ut);
-        tma_prefetch_desc(&map_w);
+        tma_prefetch_desc(&map_v);
+        tma_prefetch_desc(&map_tb);
         tma_prefetch_desc(&map_o);
         if (NC > 0) {
             issue_in(0);
@@ -609,7 +569,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     store_row_chunk(sm + OFF_WM, i, 4 * hf + 2 * grp + q2, w);
                 }
             }
-            // ---- U = Ut - W Hm: read W Hm out of the P/O accumulator first, freeing it for G1
+            // ---- R = V - e^{gc - gc_m} Kbar Hm: read Kbar Hm out of the P/O accumulator
+            // first, freeing it for G1
             mbar_wait(&bar[BAR_GA2], par, abort_flag, status);
             tc_fence_after();
             {
@@ -617,18 +578,20 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);  // columns 64 grp + 32 hf ..
                 tc_fence_before();
                 named_bar_arrive(NB_PO, kSyncCount);
-                const uint8_t *ut = sm + OFF_UT + grp * 8192;
-                uint8_t *ub = sm + OFF_UB + grp * 8192;
+                mbar_wait(&bar[BAR_WU], par, abort_flag, status);  // v of the chunk
+                const uint8_t *vt = sm + OFF_V + grp * 8192;
+                uint8_t *rt = sm + OFF_UB + grp * 8192;
+                const uint64_t nep = f2_make(-ep, -ep);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
-                    const uint4 u4 = *reinterpret_cast<const uint4 *>(ut + t64_chunk(i, 4 * hf + q4));
-                    const uint32_t uw[4] = {u4.x, u4.y, u4.z, u4.w};
+                    const uint4 v4 = *reinterpret_cast<const uint4 *>(vt + t64_chunk(i, 4 * hf + q4));
+                    const uint32_t vw[4] = {v4.x, v4.y, v4.z, v4.w};
                     uint32_t ow[4];
 #pragma unroll
                     for (int w = 0; w < 4; ++w)
-                        ow[w] = bf16x2_from_f2(f2_add(f2_from_bf16x2(uw[w]),
-                                                      f2_make(-x[8 * q4 + 2 * w], -x[8 * q4 + 2 * w + 1])));
-                    *reinterpret_cast<uint4 *>(ub + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+                        ow[w] = bf16x2_from_f2(f2_fma(nep, f2_make(x[8 * q4 + 2 * w], x[8 * q4 + 2 * w + 1]),
+                                                      f2_from_bf16x2(vw[w])));
+                    *reinterpret_cast<uint4 *>(rt + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
                 }
             }
             fence_proxy_async_smem();
@@ -643,6 +606,14 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 for (int q4 = 0; q4 < 4; ++q4) qraw[q4] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, 4 * hf + q4));
                 mbar_wait(&bar[BAR_GB], par, abort_flag, status);
                 tc_fence_after();
+                {
+                    // U = Tb R (the MMA has read R) -> bf16 U tile in R's place
+                    float u[32];
+                    tmem_ld16x2_32<32>(tq + TM_U + 64 * grp, u);
+#pragma unroll
+                    for (int q4 = 0; q4 < 4; ++q4)
+                        store_row_chunk(sm + OFF_UB + grp * 8192, i, 4 * hf + q4, u + 8 * q4);
+                }
                 const float cm = lt * c;
                 float p[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
@@ -897,7 +868,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const uint64_t dWm = make_desc(sb + OFF_WM, 16, 1024);
         const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
         const uint64_t dHB = make_desc(sb + OFF_HB, 16384, 1024);
-        const uint64_t dWW = make_desc(sb + OFF_WW, 16, 1024);
+        const uint64_t dTB = make_desc(sb + OFF_TB, 16, 1024);
         const uint64_t dUBm = make_desc(sb + OFF_UB, 8192, 1024);
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
@@ -929,14 +900,13 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 }
                 __syncwarp();
             }
-            // D2 WH = W Hm (needs Ut/W of the chunk and the Hm copy)
-            mbar_wait(&bar[BAR_WU], par, abort_flag, status);
+            // D2 KH = Kbar Hm (needs the Hm copy)
             mbar_wait(&bar[BAR_SNAPS], par, abort_flag, status);
             tc_fence_after();
             if (lead && !*abort_flag)
                 for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dWW + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
-            // the U tile is rewritten once GA2 lets EPI in: the output store must have read it
+                    mma_bf16(tbase + TM_PO, dK + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
+            // the R/U tile is rewritten once GA2 lets EPI in: the output store must have read it
             if (lead) {
                 tma_store_wait_read();
                 if (!*abort_flag) mma_commit(&bar[BAR_GA2]);
@@ -951,27 +921,29 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
                              dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
             __syncwarp();
-            // G3 P += W' Kbar, G8 S^K += Kbar^T Kbar, D6 X += Kd^T U
+            // DU U = Tb R, G3 P += W' Kbar, G8 S^K += Kbar^T Kbar
+            mbar_wait(&bar[BAR_WU], par, abort_flag, status);  // Tb of the chunk
             named_bar(NB_W, kSyncCount);
             tc_fence_after();
             if (lead && !*abort_flag) {
-                if (r + 1 < NC) issue_wu(r + 1);  // Ut and W of this chunk are consumed
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_U, dTB + k * 2, dUBm + k * 128, ID_64x128_KM, k != 0);
                 for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dKm + k * 128, ID_64x128_KM, 1);
                 mma_commit(&bar[BAR_GB]);
                 for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
                 mma_commit(&bar[BAR_GK]);
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_S, dKDm + k * 128, dUBm + k * 128, ID_128x128_MM, 1);
             }
             __syncwarp();
-            // D4 QK = Qc Kbar^T, D3 O = Qc Hm
+            // D4 QK = Qc Kbar^T, D6 X += Kd^T U, D3 O = Qc Hm
             named_bar(NB_QC, kSyncCount);
             tc_fence_after();
             if (lead && !*abort_flag) {
+                if (r + 1 < NC) issue_wu(r + 1);  // v and Tb of this chunk are consumed
                 for (int k = 0; k < 8; ++k) {
                     const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
                     mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
                 }
                 mma_commit(&bar[BAR_GC]);
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_S, dKDm + k * 128, dUBm + k * 128, ID_128x128_MM, 1);
                 for (int k = 0; k < 8; ++k)
                     mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
                 mma_commit(&bar[BAR_GC2]);
@@ -1028,7 +1000,7 @@ cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s) 
         attr_set = true;
     }
     const int NC = (a.T + kC - 1) / kC;
-    gdn_wy_kernel<<<a.B * a.H * NC, 128, WY_SMEM, s>>>(m.k, m.v, m.ut, m.w, a, NC);
+    gdn_wy_kernel<<<a.B * a.H * NC, 128, WY_SMEM, s>>>(m.k, m.tb, a, NC);
     return cudaGetLastError();
 }
 
@@ -1046,13 +1018,13 @@ cudaError_t launch_gdn_chunk(const ChunkArgs &a, const GdnMaps &m, cudaStream_t 
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gdn_chunk_kernel<<<a.B * a.H, kThreads, kSmemBytes, s>>>(m.q, m.k, m.ut, m.w, m.o, a);
+    gdn_chunk_kernel<<<a.B * a.H, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.tb, m.o, a);
     return cudaGetLastError();
 }
 
 size_t gdn_workspace_bytes(int B, int T, int H) {
     const size_t nc = static_cast<size_t>((T + kC - 1) / kC);
-    return 2 * static_cast<size_t>(B) * H * nc * kC * kD * sizeof(__nv_bfloat16);
+    return static_cast<size_t>(B) * H * nc * kC * kC * sizeof(__nv_bfloat16);
 }
 
 }  // namespace ccq

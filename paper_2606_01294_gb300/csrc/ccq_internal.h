@@ -91,16 +91,17 @@ cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_
 cudaError_t launch_gla_segments(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
 
 // Chunkwise Gated DeltaNet: tensor maps of q, k, v, o ([B][T][H][128], 64 x 64
-// boxes) and of the two workspace matrices Ut and W ([B*H*NC*64][128] bf16).
+// boxes) and of the workspace matrix Tb = Tt diag(beta) of every chunk
+// ([B*H*NC*64][64] bf16).
 struct GdnMaps {
-    CUtensorMap q, k, v, o, ut, w;
+    CUtensorMap q, k, v, o, tb;
 };
 
 // Launches the per-chunk WY kernel then the sequential chunk kernel.
 cudaError_t launch_gdn_chunk(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
 cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
 
-// Workspace bytes of the chunkwise Gated DeltaNet path (Ut and W of every chunk).
+// Workspace bytes of the chunkwise Gated DeltaNet path (Tb of every chunk).
 size_t gdn_workspace_bytes(int B, int T, int H);
 
 // Arguments of the chunkwise CCQ-GLA backward (ccq_gla_bwd.cu).  ckpt holds
@@ -139,7 +140,7 @@ cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s);
 
 // Encode the tensor map of a row-major [rows][128] bf16 matrix with 64 x 64 boxes
 // (128-byte swizzle).
-bool make_rows_map(CUtensorMap *map, const void *base, long long rows);
+bool make_rows_map(CUtensorMap *map, const void *base, long long rows, int cols = 128);
 
 // Encode the tensor map of a [B][T][H][D] tensor with a (box_inner x 1 x 64 x 1)
 // box.  swizzle128 selects the 128-byte swizzle (bf16 MMA operands, box_inner
