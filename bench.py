@@ -61,11 +61,14 @@ def gla_segments(B, H, T, sms):
 
 
 def launches_per_step(kind, B, H, T, sms):
-    """Kernel launches of one step: the segmented GLA forward is three kernels,
-    the backward three, and every call that
-    returns the position count adds the one-thread-per-row count update."""
-    fwd = 1 if gla_segments(B, H, T, sms) == 1 else 3
-    return {"gla": fwd + 1, "gdn": 2 + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3}[kind]
+    """Kernel launches of one step: the segmented GLA forward is three kernels, the
+    Gated DeltaNet forward two (WY, chunk) or four when segmented, the backward three,
+    and every call that returns the position count adds the one-thread-per-row count
+    update."""
+    split = gla_segments(B, H, T, sms) > 1
+    fwd = 3 if split else 1
+    gdn = 4 if split else 2
+    return {"gla": fwd + 1, "gdn": gdn + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3}[kind]
 
 
 def algorithmic_bytes(kind, B, H, T, D):
@@ -113,7 +116,8 @@ STEP_KERNELS = {
     "gla_bf16_4k": ["gla_chunk_kernel"],
     "gdn_bf16_4k": ["gdn_wy_kernel", "gdn_chunk_kernel"],
     "gla_bf16_20k": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel"],
-    "gdn_bf16_20k": ["gdn_wy_kernel", "gdn_chunk_kernel"],
+    "gdn_bf16_20k": ["gdn_wy_kernel", "gdn_segment_state_kernel", "gdn_segment_combine_kernel",
+                     "gdn_chunk_kernel"],
     "decode_b256": ["decode_kernel"],
     "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
                            "gla_bwd_q_kernel", "gla_bwd_state_kernel", "gla_bwd_kv_kernel"],
@@ -121,7 +125,8 @@ STEP_KERNELS = {
 # (each step also runs the one-thread-per-row position update: 8 bytes per batch row, not counted)
 KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kernel": "ccq_gla_segment.cu",
                 "gla_segment_combine_kernel": "ccq_gla_segment.cu", "gdn_wy_kernel": "ccq_gdn_chunk.cu",
-                "gdn_chunk_kernel": "ccq_gdn_chunk.cu", "recurrent": "ccq_recurrent.cu",
+                "gdn_chunk_kernel": "ccq_gdn_chunk.cu",
+                "gdn_segment_state_kernel": "ccq_gdn_segment.cu", "gdn_segment_combine_kernel": "ccq_gdn_segment.cu", "recurrent": "ccq_recurrent.cu",
                 "decode_kernel": "ccq_recurrent.cu", "gla_bwd_state_kernel": "ccq_gla_bwd.cu",
                 "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu"}
 
@@ -464,8 +469,11 @@ def run_gpu(args):
         roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": achieved / peaks["hbm_gbs"],
                 "traffic": measured_traffic(kind, args.workload),
-                "kernel": KERNEL_NAMES[kind] if args.workload != "gla_bf16_20k"
-                else "whole step: gla_segment_state_kernel + gla_segment_combine_kernel + gla_chunk_kernel", "algorithmic_bytes": bytes_,
+                "kernel": {"gla_bf16_20k": "whole step: gla_segment_state_kernel + gla_segment_combine_kernel"
+                                           " + gla_chunk_kernel",
+                           "gdn_bf16_20k": "whole step: gdn_wy_kernel + gdn_segment_state_kernel"
+                                           " + gdn_segment_combine_kernel + gdn_chunk_kernel"}.get(
+                               args.workload, KERNEL_NAMES[kind]), "algorithmic_bytes": bytes_,
                 "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
                 "flops": algorithmic_flops(kind, B, H, T, D)}
         cpu = None

@@ -197,7 +197,7 @@ static int sm_count() {
 }
 
 // Segments per sequence for the chunkwise GLA path, and chunks per segment.
-static void gla_split(const ccq_params &p, int B, int T, int H, int *nseg, int *seg_chunks) {
+static void split_sequences(const ccq_params &p, int B, int T, int H, int *nseg, int *seg_chunks) {
     const int nc = (T + 63) / 64;
     int ns = 1;
     if (p.seq_split > 0) {
@@ -227,7 +227,7 @@ ccq_status ccq_gla_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype
     *bytes = 0;
     if (gla_chunk_selected(c.p, in_dtype, Dk, T)) {
         int ns, per;
-        gla_split(c.p, B, T, H, &ns, &per);
+        split_sequences(c.p, B, T, H, &ns, &per);
         if (ns > 1) *bytes = static_cast<size_t>(B) * H * ns * kSegFloats * sizeof(float);
     }
     return CCQ_OK;
@@ -263,7 +263,7 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
         return fail(CCQ_ERR_UNSUPPORTED, "checkpoints come from the chunkwise kernel (algo recurrent given)");
     if (chunk_ok && c.p.algo != CCQ_ALGO_RECURRENT) {
         int nseg = 1, seg_chunks = 0;
-        gla_split(c.p, B, T, H, &nseg, &seg_chunks);
+        split_sequences(c.p, B, T, H, &nseg, &seg_chunks);
         if (nseg > 1) {
             const size_t need = static_cast<size_t>(B) * H * nseg * kSegFloats * sizeof(float);
             if (!workspace || workspace_bytes < need)
@@ -361,7 +361,7 @@ static size_t gla_bwd_exchange_bytes(int B, int T, int H) {
 
 static size_t gla_fwd_scratch_bytes(const ccq_params &p, int B, int T, int H) {
     int ns, per;
-    gla_split(p, B, T, H, &ns, &per);
+    split_sequences(p, B, T, H, &ns, &per);
     return ns > 1 ? static_cast<size_t>(B) * H * ns * kSegFloats * sizeof(float) : 0;
 }
 
@@ -476,13 +476,23 @@ static bool gdn_chunk_selected(const ccq_params &p, ccq_dtype in_dtype, int Dk, 
     return ok && p.algo != CCQ_ALGO_RECURRENT;
 }
 
+// Workspace of the chunkwise Gated DeltaNet path: Tb of every chunk, then (split
+// sequences) the per-segment states.
+static size_t gdn_total_workspace(const ccq_params &p, int B, int T, int H) {
+    int nseg = 1, per = 0;
+    split_sequences(p, B, T, H, &nseg, &per);
+    size_t bytes = gdn_workspace_bytes(B, T, H);
+    if (nseg > 1) bytes += static_cast<size_t>(B) * H * nseg * kGdnSegFloats * sizeof(float);
+    return bytes;
+}
+
 ccq_status ccq_gdn_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
                                   const ccq_params *p, size_t *bytes) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
     if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
-    *bytes = gdn_chunk_selected(c.p, in_dtype, Dk, T) ? gdn_workspace_bytes(B, T, H) : 0;
+    *bytes = gdn_chunk_selected(c.p, in_dtype, Dk, T) ? gdn_total_workspace(c.p, B, T, H) : 0;
     return CCQ_OK;
 }
 
@@ -507,7 +517,7 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
     if (c.p.algo == CCQ_ALGO_CHUNKWISE && !chunk_ok)
         return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
     if (gdn_chunk_selected(c.p, in_dtype, Dk, T)) {
-        const size_t need = gdn_workspace_bytes(B, T, H);
+        const size_t need = gdn_total_workspace(c.p, B, T, H);
         if (!workspace || workspace_bytes < need)
             return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
                         workspace ? workspace_bytes : static_cast<size_t>(0));
@@ -531,7 +541,17 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
         a.ST = ST; a.CT = CT; a.mT = mT;
         a.status = device_status_word();
         if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
-        cudaError_t e = launch_gdn_chunk(a, maps, static_cast<cudaStream_t>(stream));
+        int nseg = 1, seg_chunks = 0;
+        split_sequences(c.p, B, T, H, &nseg, &seg_chunks);
+        a.nseg = nseg;
+        a.seg_chunks = seg_chunks;
+        cudaError_t e;
+        if (nseg > 1) {
+            a.seg_ws = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + gdn_workspace_bytes(B, T, H));
+            e = launch_gdn_segments(a, maps, static_cast<cudaStream_t>(stream));
+        } else {
+            e = launch_gdn_chunk(a, maps, static_cast<cudaStream_t>(stream));
+        }
         if (e != cudaSuccess) return cuda_fail(e, "chunkwise Gated DeltaNet kernel launch");
         return finish_t(t0, tT, B, T, static_cast<cudaStream_t>(stream));
     }

@@ -367,14 +367,6 @@ constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
 constexpr uint32_t ID_64x128_KM = make_idesc(64, 128, 0, 1);
 constexpr uint32_t ID_128x128_MM = make_idesc(128, 128, 1, 1);
 
-__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *m, uint64_t *bar, int c0, int c1) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3}], [%4];" ::"r"(smem_addr(dst)),
-        "l"(reinterpret_cast<uint64_t>(m)), "r"(c0), "r"(c1), "r"(smem_addr(bar))
-        : "memory");
-}
-
 __global__ void __launch_bounds__(kThreads, 1)
 gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                  const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_tb,
@@ -393,12 +385,20 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     };
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int bh = blockIdx.x / a.nseg, seg = blockIdx.x % a.nseg, b = bh / a.H, h = bh % a.H;
     const int T = a.T, H = a.H;
-    const int NC = (T + kC - 1) / kC;
-    const int64_t t0 = a.t0 ? a.t0[b] : 0;
+    const int NCt = (T + kC - 1) / kC;
+    const int cb = a.nseg > 1 ? seg * a.seg_chunks : 0;  // first chunk of this CTA
+    const int NC = a.nseg > 1 ? min(NCt, cb + a.seg_chunks) - cb : NCt;
+    const bool last_seg = seg == a.nseg - 1;
+    // a segment starts from the states its slot of the workspace holds (ccq_gdn_segment.cu)
+    const float *segst = a.nseg > 1 ? a.seg_ws + static_cast<size_t>(blockIdx.x) * kGdnSegFloats : nullptr;
+    const float *S0 = segst ? segst : a.S0;
+    const float *C0 = segst ? segst + 2 * kD * kD : a.C0;
+    const float *m0 = segst ? segst + 3 * kD * kD : a.m0;
+    const int64_t t0 = (a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(cb) * kC;  // position before the CTA's first token
     int *status = a.status;
-    const int wrow0 = bh * NC * kC;  // first workspace row of this (b, h)
+    const int wrow0 = (bh * NCt + cb) * kC;  // first workspace row of this CTA's chunks
 
     if (tid == 0) {
         for (int i = 0; i < kNumBars; ++i) mbar_init(&bar[i], 1);
@@ -416,16 +416,17 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         uint8_t *base = sm + s * SLOT_BYTES;
         uint64_t *bb = &bar[BAR_IN0 + s];
         mbar_arrive_expect_tx(bb, 4 * 8192);
-        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, r * kC, b);
-        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, r * kC, b);
-        tma_load_4d(base + SO_K, &map_k, bb, 0, h, r * kC, b);
-        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, r * kC, b);
+        const int tg = (cb + r) * kC;
+        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tg, b);
+        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tg, b);
+        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tg, b);
+        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tg, b);
     };
     auto issue_wu = [&](int r) {  // v and Tb of chunk r
         uint64_t *bb = &bar[BAR_WU];
         mbar_arrive_expect_tx(bb, 3 * 8192);
-        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, r * kC, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, r * kC, b);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, (cb + r) * kC, b);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, (cb + r) * kC, b);
         tma_load_2d(sm + OFF_TB, &map_tb, bb, 0, wrow0 + r * kC);
     };
 
@@ -434,14 +435,15 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const size_t bhs = static_cast<size_t>(bh);
         const int row = 32 * (warp & 3) + lane, grp = warp >> 2;
         for (int m = 0; m < 2; ++m) {
-            const float *src = m == 0 ? a.S0 : a.C0;
+            const float *src = m == 0 ? S0 : C0;
             const uint32_t col0 = m == 0 ? TM_S : TM_SK;
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 const int c = 2 * grp + cc;
                 float x[32];
                 if (src) {
-                    const float4 *p4 = reinterpret_cast<const float4 *>(src + (bhs * kD + row) * kD + 32 * c);
+                    const float4 *p4 = reinterpret_cast<const float4 *>(
+                        src + (segst ? static_cast<size_t>(row) * kD : (bhs * kD + row) * kD) + 32 * c);
 #pragma unroll
                     for (int e = 0; e < 8; ++e) {
                         const float4 f = p4[e];
@@ -457,7 +459,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tmem_wait_st();
     } else if (warp < kIssueWarp) {
         const int wt = tid - 32 * kPrepWarp0;
-        slot_f(0, MS_MST)[wt] = a.m0 ? a.m0[static_cast<size_t>(bh) * kD + wt] : 0.f;
+        slot_f(0, MS_MST)[wt] = m0 ? m0[(segst ? 0 : static_cast<size_t>(bh) * kD) + wt] : 0.f;
         dmprev[wt] = 0.f;
     } else if (lane == 0) {
         tma_prefetch_desc(&map_q);
@@ -696,7 +698,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
         }
         // final states: H_T = e^{gc_C - gc_m} X (last chunk), S^K
-        if (NC > 0) {
+        if (NC > 0 && last_seg) {
             tc_fence_after();
             const size_t bhs = static_cast<size_t>(bh);
 #pragma unroll
@@ -723,9 +725,9 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const int wt = tid - 32 * kPrepWarp0;
         float lam_reg, g_reg;
         {
-            const int tn = wt >> 1;
+            const int tn = cb * kC + (wt >> 1), tg = cb * kC + wt;
             lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
-            g_reg = (wt < 64 && wt < T) ? a.g[(static_cast<size_t>(b) * T + wt) * H + h] : 0.f;
+            g_reg = (wt < 64 && tg < T) ? a.g[(static_cast<size_t>(b) * T + tg) * H + h] : 0.f;
         }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
@@ -738,9 +740,9 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const float lam_cur = lam_reg;
             if (wt < 64) scal[2 + wt] = g_reg;
             {
-                const int tn = (r + 1) * kC + (wt >> 1);
+                const int tn = (cb + r + 1) * kC + (wt >> 1);
                 lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
-                const int tg = (r + 1) * kC + wt;
+                const int tg = (cb + r + 1) * kC + wt;
                 g_reg = (wt < 64 && tg < T) ? a.g[(static_cast<size_t>(b) * T + tg) * H + h] : 0.f;
             }
             named_bar(NB_PREP, 128);  // key sum and raw decays visible
@@ -858,7 +860,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             dmprev[wt] = dmp[wt] + dmp[kD + wt];
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
         }
-        if (NC > 0 && a.mT) {
+        if (NC > 0 && a.mT && last_seg) {
             const int sl = (NC - 1) & 1;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
@@ -894,8 +896,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 mbar_wait(&bar[BAR_GD], (r - 1) & 1, abort_flag, status);
                 named_bar(NB_OUT, kSyncCount);
                 if (lead) {
-                    tma_store_4d(&map_o, sm + OFF_UB, 0, h, (r - 1) * kC, b);
-                    tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (r - 1) * kC, b);
+                    tma_store_4d(&map_o, sm + OFF_UB, 0, h, (cb + r - 1) * kC, b);
+                    tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (cb + r - 1) * kC, b);
                     tma_store_commit();
                 }
                 __syncwarp();
@@ -968,8 +970,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             mbar_wait(&bar[BAR_GD], (NC - 1) & 1, abort_flag, status);
             named_bar(NB_OUT, kSyncCount);
             if (lead) {
-                tma_store_4d(&map_o, sm + OFF_UB, 0, h, (NC - 1) * kC, b);
-                tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (NC - 1) * kC, b);
+                tma_store_4d(&map_o, sm + OFF_UB, 0, h, (cb + NC - 1) * kC, b);
+                tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (cb + NC - 1) * kC, b);
                 tma_store_commit();
                 tma_store_wait_all();
                 if (*abort_flag) {
@@ -1008,18 +1010,22 @@ cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s) 
 
 namespace ccq {
 
-cudaError_t launch_gdn_chunk(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s) {
-    cudaError_t e = launch_gdn_wy(a, m, s);
-    if (e != cudaSuccess) return e;
+cudaError_t launch_gdn_chunk_only(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s) {
     static bool attr_set = false;
     if (!attr_set) {
-        e = cudaFuncSetAttribute(gdn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 static_cast<int>(kSmemBytes));
+        cudaError_t e = cudaFuncSetAttribute(gdn_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(kSmemBytes));
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gdn_chunk_kernel<<<a.B * a.H, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.tb, m.o, a);
+    gdn_chunk_kernel<<<a.B * a.H * a.nseg, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.tb, m.o, a);
     return cudaGetLastError();
+}
+
+cudaError_t launch_gdn_chunk(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s) {
+    cudaError_t e = launch_gdn_wy(a, m, s);
+    if (e != cudaSuccess) return e;
+    return launch_gdn_chunk_only(a, m, s);
 }
 
 size_t gdn_workspace_bytes(int B, int T, int H) {

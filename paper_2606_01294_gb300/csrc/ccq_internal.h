@@ -46,7 +46,8 @@ struct ChunkArgs {
     float *ST, *CT, *mT;
     int *status;  // device status word (bounded-wait give-ups)
     // sequence segments (long sequences): nseg segments of seg_chunks chunks each
-    // (the last one shorter); seg_ws holds kSegFloats floats per (sequence, segment).
+    // (the last one shorter); seg_ws holds kSegFloats (GLA) or kGdnSegFloats (Gated
+    // DeltaNet) floats per (sequence, segment).
     int nseg = 1;
     int seg_chunks = 0;
     float *seg_ws = nullptr;
@@ -97,9 +98,19 @@ struct GdnMaps {
     CUtensorMap q, k, v, o, tb;
 };
 
-// Launches the per-chunk WY kernel then the sequential chunk kernel.
+// Launches the per-chunk WY kernel then the sequential chunk kernel (launch_gdn_chunk),
+// either one alone, or -- for a.nseg > 1 -- WY, the segment states, their combine and
+// the chunk kernel on every (sequence, segment) (launch_gdn_segments).
 cudaError_t launch_gdn_chunk(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
 cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
+cudaError_t launch_gdn_chunk_only(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
+cudaError_t launch_gdn_segments(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s);
+
+// Per (sequence, segment) workspace of the segmented Gated DeltaNet forward:
+// S [128][128] (the segment's state from zero, then its entering state), P [128][128]
+// (the segment's transition), C [128][128] (its covariance sum, then the entering C),
+// m [128] (its key sum, then the entering m), 128 spare.
+constexpr int kGdnSegFloats = 3 * 128 * 128 + 2 * 128;
 
 // Workspace bytes of the chunkwise Gated DeltaNet path (Tb of every chunk).
 size_t gdn_workspace_bytes(int B, int T, int H);

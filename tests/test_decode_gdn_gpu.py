@@ -162,3 +162,36 @@ def test_gdn_full_size_sampled():
         assert rel_err(o[b:b + 1, :, h:h + 1], ref["o"]) <= TOL[torch.bfloat16]
         assert rel_err(fs.S[b:b + 1, h:h + 1], ref["S"]) <= TOL[torch.bfloat16]
         assert rel_err(fs.C[b:b + 1, h:h + 1], ref["C"]) <= TOL[torch.bfloat16]
+
+
+@pytest.mark.parametrize("split", [2, 3, 5])
+@pytest.mark.parametrize("decay", ["drawn", "slow"])
+def test_gdn_segmented_sequences(split, decay):
+    """Sequences cut into segments (segment state and transition from zero, fp32
+    combine, chunk kernel per segment) equal one sequential walk: T = 700 (11 chunks,
+    ragged tail), resumed state.  "slow" divides the log decays by 100 so the segment
+    transition P stays far from zero and every term of P H + Q is exercised."""
+    P = gen.make_inputs(GDN, 2, 700, 2, 128, 128, dtype=torch.bfloat16, seed=60 + split, lam="trained",
+                        keys="structured")
+    prev = gen.make_inputs(GDN, 2, 90, 2, 128, 128, dtype=torch.bfloat16, seed=70, lam="trained")
+    if decay == "slow":
+        P["gate"] = P["gate"] / 100
+        prev["gate"] = prev["gate"] / 100
+    st = state_f32(oracle_forward(GDN, prev))
+    o, fs = gpu_forward(GDN, P, state_to_dev(st), algo="chunkwise", seq_split=split)
+    compare(o, fs, oracle_forward(GDN, P, st), TOL[torch.bfloat16], f"gdn split={split} {decay}")
+
+
+def test_gdn_20k_sampled():
+    """B=1, H=16, T=20480 (the long-context benchmark's launch, split into segments);
+    sampled heads against the oracle."""
+    w = dict(gen.WORKLOADS["gdn_bf16_20k"])
+    backbone = w.pop("backbone")
+    P = gen.make_inputs(backbone, **w)
+    o, fs = gpu_forward(GDN, P)
+    for b, h in [(0, 0), (0, 9)]:
+        ref = oracle_forward(GDN, slice_bh(P, b, h))
+        assert rel_err(o[b:b + 1, :, h:h + 1], ref["o"]) <= TOL[torch.bfloat16]
+        assert rel_err(fs.S[b:b + 1, h:h + 1], ref["S"]) <= TOL[torch.bfloat16]
+        assert rel_err(fs.C[b:b + 1, h:h + 1], ref["C"]) <= TOL[torch.bfloat16]
+        assert rel_err(fs.m[b:b + 1, h:h + 1], ref["m"]) <= TOL[torch.bfloat16]
