@@ -377,16 +377,20 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
 // Per (sequence, block of 16 state columns): walks the segments, replacing each slot's
 // S (Q), C (dC) and m (dm) with the states entering that segment:
 //   H_{s+1} = P_s H_s + Q_s,  C_{s+1} = C_s + dC_s,  m_{s+1} = m_s + dm_s.
+// P_s is staged in shared memory with coalesced loads (64 KB); the product runs there.
 constexpr int kCols = 16;
+constexpr int kCombineSmem = (kSS + kD * kCols) * 4;
 
 __global__ void __launch_bounds__(256)
 gdn_segment_combine_kernel(const ChunkArgs a) {
-    __shared__ float hcur[kD * kCols];
+    extern __shared__ float csm[];
+    float *Ps = csm;               // [128][128]
+    float *hcur = csm + kSS;       // [128][16]
     const int nblk = kD / kCols;
     const int seq = blockIdx.x / nblk, cblk = blockIdx.x % nblk;
     const size_t sq = static_cast<size_t>(seq);
     const int tid = threadIdx.x;
-    const int arow = tid >> 1, c0 = kCols * cblk + 8 * (tid & 1);  // this thread: row arow, 8 columns
+    const int arow = tid >> 1, cl = 8 * (tid & 1), c0 = kCols * cblk + cl;  // row arow, 8 columns
     float hreg[8], creg[8];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
@@ -396,28 +400,39 @@ gdn_segment_combine_kernel(const ChunkArgs a) {
     float mreg = (cblk == 0 && tid < kD) ? (a.m0 ? a.m0[sq * kD + tid] : 0.f) : 0.f;
     for (int s = 0; s < a.nseg; ++s) {
         float *slot = a.seg_ws + (sq * a.nseg + s) * kGdnSegFloats;
+        // stage P_s (16 float4 per thread, all in flight) and this block's H_s columns
+        {
+            const float4 *src = reinterpret_cast<const float4 *>(slot + kSS);
+            float4 *dst = reinterpret_cast<float4 *>(Ps);
+            float4 v[16];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) hcur[arow * kCols + (c0 - kCols * cblk) + u] = hreg[u];
+            for (int u = 0; u < 16; ++u) v[u] = src[u * 256 + tid];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) dst[u * 256 + tid] = v[u];
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) hcur[arow * kCols + cl + u] = hreg[u];
+        float acc[8], dcv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            acc[u] = slot[arow * kD + c0 + u];            // Q_s
+            dcv[u] = slot[2 * kSS + arow * kD + c0 + u];  // dC_s
+        }
         __syncthreads();
-        // next H = P H + Q (rows arow, columns c0..c0+7); read Q and dC before replacing them
-        float acc[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) acc[u] = slot[arow * kD + c0 + u];
-        const float *P = slot + kSS + arow * kD;
+        const float *P = Ps + arow * kD;
+#pragma unroll 4
         for (int bb = 0; bb < kD; bb += 4) {
             const float4 p4 = *reinterpret_cast<const float4 *>(P + bb);
             const float pv[4] = {p4.x, p4.y, p4.z, p4.w};
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
-                const float *hr = hcur + (bb + t) * kCols + (c0 - kCols * cblk);
+                const float4 h0 = *reinterpret_cast<const float4 *>(hcur + (bb + t) * kCols + cl);
+                const float4 h1 = *reinterpret_cast<const float4 *>(hcur + (bb + t) * kCols + cl + 4);
+                const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
 #pragma unroll
-                for (int u = 0; u < 8; ++u) acc[u] = fmaf(pv[t], hr[u], acc[u]);
+                for (int u = 0; u < 8; ++u) acc[u] = fmaf(pv[t], hv[u], acc[u]);
             }
         }
-        float dcv[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) dcv[u] = slot[2 * kSS + arow * kD + c0 + u];
-        __syncthreads();  // every thread has read this slot's Q rows it needs... and hcur
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
             slot[arow * kD + c0 + u] = hreg[u];
@@ -430,6 +445,7 @@ gdn_segment_combine_kernel(const ChunkArgs a) {
             slot[3 * kSS + tid] = mreg;
             mreg += dm;
         }
+        __syncthreads();  // Ps and hcur are rewritten by the next segment
     }
 }
 
@@ -448,7 +464,14 @@ cudaError_t launch_gdn_segments(const ChunkArgs &a, const GdnMaps &m, cudaStream
     gdn_segment_state_kernel<<<a.B * a.H * a.nseg, kThreads, kSmem, s>>>(m.k, m.v, m.tb, a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    gdn_segment_combine_kernel<<<a.B * a.H * (kD / kCols), 256, 0, s>>>(a);
+    static bool attr_combine = false;
+    if (!attr_combine) {
+        e = cudaFuncSetAttribute(gdn_segment_combine_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kCombineSmem);
+        if (e != cudaSuccess) return e;
+        attr_combine = true;
+    }
+    gdn_segment_combine_kernel<<<a.B * a.H * (kD / kCols), 256, kCombineSmem, s>>>(a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     return launch_gdn_chunk_only(a, m, s);
