@@ -464,6 +464,7 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
     a.dST = dST; a.dCT = dCT; a.dmT = dmT;
     a.dlambda = dlambda; a.dgk = dgk; a.dS0 = dS0; a.dC0 = dC0; a.dm0 = dm0;
     a.chunk_vec = chunk_vec; a.state_img = state_img; a.state_vec = state_vec;
+    a.wave = sm_count();
     a.status = device_status_word();
     if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
     cudaError_t e = launch_gla_bwd(a, maps, s);

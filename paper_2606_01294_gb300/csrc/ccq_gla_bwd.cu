@@ -312,6 +312,22 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, c0, b);
         bulk_load(sm + OFF_SK, rec, 65536, bb);
         bulk_load(misc + M_MR, rec + 65536, 512, bb);
+        // the chunk one wave later finds its inputs in L2
+        const int nx = blockIdx.x + a.wave;
+        if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
+            const int bh2 = nx / NC, r2 = nx % NC, b2 = bh2 / H, h2 = bh2 % H, c2 = r2 * kC;
+            tma_prefetch_l2_4d(&map_q, 0, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_q, 64, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_k, 0, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_k, 64, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_v, 0, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_v, 64, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_do, 0, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_do, 64, h2, c2, b2);
+            tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
+            bulk_prefetch_l2(a.ckpt + static_cast<size_t>(bh2) * ckpt_head_bytes(T) + static_cast<size_t>(r2) * kCkptChunkBytes,
+                             static_cast<uint32_t>(kCkptChunkBytes));
+        }
     }
     if (warp == 0) tmem_alloc(tmem_slot, 512);
     for (int e = tid; e < 8192 / 16; e += kThreadsPar)
@@ -880,6 +896,20 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, c0, b);
         bulk_load(sm + OFF_DS, a.state_img + static_cast<size_t>(blockIdx.x) * 65536, 65536, bb);
         bulk_load(misc + M_VEC, a.state_vec + static_cast<size_t>(blockIdx.x) * 2 * kD, 1024, bb);
+        // the chunk one wave later finds its inputs in L2
+        const int nx = blockIdx.x + a.wave;
+        if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
+            const int bh2 = nx / NC, r2 = nx % NC, b2 = bh2 / H, h2 = bh2 % H, c2 = r2 * kC;
+            const CUtensorMap *maps[6] = {&map_k, &map_v, &map_do, &map_qg, &map_dkc, &map_gq};
+#pragma unroll
+            for (int u = 0; u < 6; ++u) {
+                tma_prefetch_l2_4d(maps[u], 0, h2, c2, b2);
+                tma_prefetch_l2_4d(maps[u], 64, h2, c2, b2);
+            }
+            tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
+            bulk_prefetch_l2(a.state_img + static_cast<size_t>(nx) * 65536, 65536);
+            bulk_prefetch_l2(a.state_vec + static_cast<size_t>(nx) * 2 * kD, 1024);
+        }
     }
     if (warp == 0) tmem_alloc(tmem_slot, 512);
     __syncthreads();

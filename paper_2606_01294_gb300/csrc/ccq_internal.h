@@ -135,6 +135,8 @@ struct BwdArgs {
     uint8_t *state_img;  // 64 KB written by the state pass: the bf16 tile images of
                          // Diag(e^{Gc-Gmid}) dS_{r+1} and DC_{r+1} (two T64 tiles each)
     float *state_vec;    // [2][128] written by the state pass: Dm_{r+1}, rowsum(dS_{r+1} S_{r+1})
+    int wave = 0;        // chunk CTAs resident at once (one per SM): each prefetches into L2 the
+                         // inputs of the chunk one wave after its own
 };
 
 // Tensor maps ([B][T][H][128], 64 x 64 swizzled boxes; g as in ChunkMaps) of

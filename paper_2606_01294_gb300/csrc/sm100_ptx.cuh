@@ -132,6 +132,21 @@ __device__ __forceinline__ void tma_load_4d(void *dst, const CUtensorMap *m, uin
 
 // 4-D tiled store of one box from shared memory (bulk-group completion).
 // Rows outside the tensor are not written.
+// L2 prefetch of one 4-D tile of a tensor map (no shared memory, no barrier; coordinates
+// past the tensor are ignored like a load's).
+__device__ __forceinline__ void tma_prefetch_l2_4d(const CUtensorMap *m, int c0, int c1, int c2, int c3) {
+    asm volatile("cp.async.bulk.prefetch.tensor.4d.L2.global.tile [%0, {%1, %2, %3, %4}];" ::"l"(
+                     reinterpret_cast<uint64_t>(m)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+
+// L2 prefetch of a contiguous global range (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_prefetch_l2(const void *src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
+                 : "memory");
+}
+
 // 2-D tiled TMA load (rows map) completing on `bar`.
 __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *m, uint64_t *bar, int c0, int c1) {
     asm volatile(
