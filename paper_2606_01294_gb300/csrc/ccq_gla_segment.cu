@@ -96,28 +96,35 @@ gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
         tma_load_4d(base + SL_V + 8192, &map_v, &bar[s], 64, h, cg * kC, b);
         tma_load_4d(base + SL_G, &map_g, &bar[s], 0, h, cg * kC, b);
     };
-    if (tid == 0) {
-        issue(0);
-        if (n > 1) issue(1);
-    }
+    if (tid == 0) issue(0);
+    if (tid == 0 && n > 1) issue(1);
     for (int i = 0; i < n; ++i) {
         const int s = i & 1;
         const uint32_t par = (i >> 1) & 1;
         uint8_t *slot = sm + s * SL_BYTES;
+        // refill the other slot with chunk step i + 1 once the products of step i - 1 (which
+        // read it) are done; they ran under that step's tail, so this rarely waits
+        if (tid == 0 && i >= 1 && i + 1 < n && !*abort_flag) {
+            mbar_wait(&bar[2 + (s ^ 1)], ((i - 1) >> 1) & 1, abort_flag, status);
+            issue(i + 1);
+        }
         mbar_wait(&bar[s], par, abort_flag, status);
-        // k row norms
-        if (tid < 64) {
-            float ss = 0.f;
+        // k row norms: two threads per row (one T64 tile each), eight partial sums in pairs
+        if (tid < 128) {
+            const int j = tid >> 1, hh = tid & 1;
+            uint64_t s0 = 0, s1 = 0;
 #pragma unroll
-            for (int t64 = 0; t64 < 2; ++t64)
-#pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
-                    float f[8];
-                    unpack_bf16x8(*reinterpret_cast<const uint4 *>(slot + SL_K + t64 * 8192 + t64_chunk(tid, cc)), f);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) ss = fmaf(f[e], f[e], ss);
-                }
-            rk[tid] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+            for (int cc = 0; cc < 8; ++cc) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(slot + SL_K + hh * 8192 + t64_chunk(j, cc));
+                const uint64_t p0 = f2_from_bf16x2(v.x), p1 = f2_from_bf16x2(v.y), p2 = f2_from_bf16x2(v.z),
+                               p3 = f2_from_bf16x2(v.w);
+                s0 = f2_fma(p0, p0, s0); s1 = f2_fma(p1, p1, s1);
+                s0 = f2_fma(p2, p2, s0); s1 = f2_fma(p3, p3, s1);
+            }
+            const float2 sv = f2_split(f2_add(s0, s1));
+            float ss = sv.x + sv.y;
+            ss += __shfl_xor_sync(0xffffffffu, ss, 1);
+            if (hh == 0) rk[j] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
         }
         // gate cumsum per key dim over this thread's 32 tokens
         const int d = tid & 127, th = tid >> 7;
@@ -170,11 +177,6 @@ gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
         if (tid < kD) {
             dsuf[tid] *= fast_exp2((gp[tid] + gp[kD + tid]) * kLog2e);
             msum[tid] += dm[tid] + dm[kD + tid];
-        }
-        // refill this slot with chunk step i + 2 once its products are done
-        if (tid == 0 && i + 2 < n && !*abort_flag) {
-            mbar_wait(&bar[2 + s], par, abort_flag, status);
-            issue(i + 2);
         }
         __syncthreads();
     }
