@@ -38,12 +38,12 @@ constexpr uint32_t SL_K = 0, SL_V = 16384, SL_G = 32768, SL_KU = 65536;
 constexpr uint32_t OFF_MISC = 2 * SL_BYTES;  // 163840
 constexpr uint32_t M_DSUF = 0;     // [128] decay of the chunks already visited (later ones)
 constexpr uint32_t M_MSUM = 512;   // [128] key sum
-constexpr uint32_t M_GP = 1024;    // [2][128] gate partial sums
-constexpr uint32_t M_DM = 2048;    // [2][128] key partial sums
-constexpr uint32_t M_RK = 3072;    // [64]
-constexpr uint32_t M_BAR = 3328;   // 4 mbarriers: in[2], mma[2]
-constexpr uint32_t M_TMEM = 3360, M_ABORT = 3364;
-constexpr uint32_t kSmem = OFF_MISC + 4096 + 1024;
+constexpr uint32_t M_GP = 1024;    // [4][128] gate sums of the four token quarters
+constexpr uint32_t M_DM = 3072;    // [4][128] key sums of the four token quarters
+constexpr uint32_t M_RK = 5120;    // [64]
+constexpr uint32_t M_BAR = 5376;   // 4 mbarriers: in[2], mma[2]
+constexpr uint32_t M_TMEM = 5408, M_ABORT = 5412;
+constexpr uint32_t kSmem = OFF_MISC + 6144 + 1024;
 static_assert(kSmem <= 232448, "smem");
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -126,39 +126,65 @@ gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
             ss += __shfl_xor_sync(0xffffffffu, ss, 1);
             if (hh == 0) rk[j] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
         }
-        // gate cumsum per key dim over this thread's 32 tokens
-        const int d = tid & 127, th = tid >> 7;
-        float gl[32];
+        // thread = (key-dim pair (d0, d0 + 1), token quarter): gate prefix over its 16 tokens
+        const int p = tid & 63, qq = tid >> 6, d0 = 2 * p;
+        uint64_t gl[16];
         {
-            float run = 0.f;
+            uint64_t run = 0;
 #pragma unroll
-            for (int jj = 0; jj < 32; ++jj) {
-                const int j = 32 * th + jj;
-                const float g = gate_f32 ? reinterpret_cast<const float *>(slot + SL_G)[j * kD + d]
-                                         : __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(slot + SL_G)[j * kD + d]);
-                run += g;
-                gl[jj] = run;
+            for (int u = 0; u < 16; ++u) {
+                const int j = 16 * qq + u;
+                uint64_t g2;
+                if (gate_f32) {
+                    const float2 f = *reinterpret_cast<const float2 *>(slot + SL_G + (j * kD + d0) * 4);
+                    g2 = f2_make(f.x, f.y);
+                } else {
+                    g2 = f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(slot + SL_G + (j * kD + d0) * 2));
+                }
+                run = f2_add(run, g2);
+                gl[u] = run;
             }
-            gp[th * kD + d] = run;
+            const float2 rv = f2_split(run);
+            gp[qq * kD + d0] = rv.x;
+            gp[qq * kD + d0 + 1] = rv.y;
         }
         __syncthreads();
         {
-            const float g0 = gp[d], gtot = gp[d] + gp[kD + d];
-            const float off = th ? g0 : 0.f;
-            const float ds = dsuf[d];
-            const uint32_t tcol = (d >> 6) * 8192;
-            float dmp = 0.f;
+            // Ku_j = kbar_j Dsuf e^{Gtot - G_j}: the exponent is (Gtot - quarter offset) - prefix
+            float offx = 0.f, offy = 0.f, totx = 0.f, toty = 0.f;
 #pragma unroll
-            for (int jj = 0; jj < 32; ++jj) {
-                const int j = 32 * th + jj;
-                const uint32_t o = tcol + t64_offset(j, d & 63);
-                const float kb = __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(slot + SL_K + o)) * rk[j];
-                *reinterpret_cast<__nv_bfloat16 *>(slot + SL_K + o) = __float2bfloat16_rn(kb);
-                const float ku = kb * ds * fast_exp2((gtot - (gl[jj] + off)) * kLog2e);
-                *reinterpret_cast<__nv_bfloat16 *>(slot + SL_KU + o) = __float2bfloat16_rn(ku);
-                dmp += kb;
+            for (int q2 = 0; q2 < 4; ++q2) {
+                const float gx = gp[q2 * kD + d0], gy = gp[q2 * kD + d0 + 1];
+                totx += gx; toty += gy;
+                if (q2 < qq) { offx += gx; offy += gy; }
             }
-            dm[th * kD + d] = dmp;
+            const uint64_t base2 = f2_make(totx - offx, toty - offy);
+            const uint64_t l2 = f2_make(kLog2e, kLog2e);
+            const uint64_t ds2 = f2_make(dsuf[d0], dsuf[d0 + 1]);
+            const uint32_t tcol = (d0 >> 6) * 8192;
+            uint32_t kraw[16];
+            float rkv[16];
+#pragma unroll
+            for (int u = 0; u < 16; ++u) kraw[u] = *reinterpret_cast<const uint32_t *>(slot + SL_K + tcol + t64_offset(16 * qq + u, d0 & 63));
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const float4 r4 = *reinterpret_cast<const float4 *>(rk + 16 * qq + 4 * u);
+                rkv[4 * u] = r4.x; rkv[4 * u + 1] = r4.y; rkv[4 * u + 2] = r4.z; rkv[4 * u + 3] = r4.w;
+            }
+            uint64_t dm2 = 0;
+#pragma unroll
+            for (int u = 0; u < 16; ++u) {
+                const uint32_t o = tcol + t64_offset(16 * qq + u, d0 & 63);
+                const uint64_t kb2 = f2_mul(f2_from_bf16x2(kraw[u]), f2_make(rkv[u], rkv[u]));
+                const float2 x = f2_split(f2_mul(f2_add(base2, f2_make(-f2_split(gl[u]).x, -f2_split(gl[u]).y)), l2));
+                const uint64_t ku2 = f2_mul(f2_mul(kb2, ds2), f2_make(fast_exp2(x.x), fast_exp2(x.y)));
+                *reinterpret_cast<uint32_t *>(slot + SL_K + o) = bf16x2_from_f2(kb2);
+                *reinterpret_cast<uint32_t *>(slot + SL_KU + o) = bf16x2_from_f2(ku2);
+                dm2 = f2_add(dm2, kb2);
+            }
+            const float2 dv = f2_split(dm2);
+            dm[qq * kD + d0] = dv.x;
+            dm[qq * kD + d0 + 1] = dv.y;
         }
         fence_proxy_async_smem();
         tc_fence_before();
@@ -175,8 +201,8 @@ gla_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
             mma_commit(&bar[2 + s]);
         }
         if (tid < kD) {
-            dsuf[tid] *= fast_exp2((gp[tid] + gp[kD + tid]) * kLog2e);
-            msum[tid] += dm[tid] + dm[kD + tid];
+            dsuf[tid] *= fast_exp2(((gp[tid] + gp[kD + tid]) + (gp[2 * kD + tid] + gp[3 * kD + tid])) * kLog2e);
+            msum[tid] += (dm[tid] + dm[kD + tid]) + (dm[2 * kD + tid] + dm[3 * kD + tid]);
         }
         __syncthreads();
     }
