@@ -107,20 +107,30 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
         const int j = rr & 63;
         uint8_t *base = isq ? q_tile : k_tile;
         const int cpp = 16 / tpr;  // 16-byte chunks of the row per thread
-        float ss = 0.f, md = 0.f;
+        uint4 raw[8];              // the row's chunks, loaded once
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
             if (u < cpp) {
                 const int cidx = part * cpp + u, t64 = cidx >> 3, cc = cidx & 7;
-                float x[8];
-                load_row_chunk(base + t64 * 8192, j, cc, x);
+                raw[u] = *reinterpret_cast<const uint4 *>(base + t64 * 8192 + t64_chunk(j, cc));
+            }
+        }
+        uint64_t s2 = 0, m2 = 0;
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    ss = fmaf(x[e], x[e], ss);
-                    if (isq) md = fmaf(x[e], Mr[64 * t64 + 8 * cc + e], md);
+        for (int u = 0; u < 8; ++u) {
+            if (u < cpp) {
+                const int cidx = part * cpp + u, t64 = cidx >> 3, cc = cidx & 7;
+                const uint32_t w[4] = {raw[u].x, raw[u].y, raw[u].z, raw[u].w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const uint64_t x2 = f2_from_bf16x2(w[e]);
+                    s2 = f2_fma(x2, x2, s2);
+                    if (isq) m2 = f2_fma(x2, f2_make(Mr[64 * t64 + 8 * cc + 2 * e], Mr[64 * t64 + 8 * cc + 2 * e + 1]), m2);
                 }
             }
         }
+        const float2 sv = f2_split(s2), mv = f2_split(m2);
+        float ss = sv.x + sv.y, md = mv.x + mv.y;
         ss += __shfl_xor_sync(0xffffffffu, ss, 1);
         md += __shfl_xor_sync(0xffffffffu, md, 1);
         if (tpr == 4) {
@@ -129,15 +139,16 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
         }
         const float rn = l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
         if (l2norm) {
+            const uint64_t rn2 = f2_make(rn, rn);
 #pragma unroll
             for (int u = 0; u < 8; ++u) {
                 if (u < cpp) {
                     const int cidx = part * cpp + u, t64 = cidx >> 3, cc = cidx & 7;
-                    float x[8];
-                    load_row_chunk(base + t64 * 8192, j, cc, x);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) x[e] *= rn;
-                    store_row_chunk(base + t64 * 8192, j, cc, x);
+                    *reinterpret_cast<uint4 *>(base + t64 * 8192 + t64_chunk(j, cc)) =
+                        make_uint4(bf16x2_from_f2(f2_mul(f2_from_bf16x2(raw[u].x), rn2)),
+                                   bf16x2_from_f2(f2_mul(f2_from_bf16x2(raw[u].y), rn2)),
+                                   bf16x2_from_f2(f2_mul(f2_from_bf16x2(raw[u].z), rn2)),
+                                   bf16x2_from_f2(f2_mul(f2_from_bf16x2(raw[u].w), rn2)));
                 }
             }
         }
@@ -191,11 +202,15 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
         }
     }
     const uint32_t tcol = (d0 >> 6) * 8192;
+    uint32_t kraw[16];  // every k pair before any tile store
+#pragma unroll
+    for (int jj = 0; jj < 16; ++jj)
+        kraw[jj] = *reinterpret_cast<const uint32_t *>(k_tile + tcol + t64_offset(16 * qt + jj, d0 & 63));
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
         const int j = 16 * qt + jj;
         const uint32_t off = tcol + t64_offset(j, d0 & 63);
-        const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(k_tile + off));
+        const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&kraw[jj]));
         const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
         *reinterpret_cast<uint32_t *>(kd_tile + off) = pack_bf16(kr.x * fast_exp2(-x0), kr.y * fast_exp2(-x1));
         *reinterpret_cast<uint32_t *>(eg_tile + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
