@@ -491,9 +491,9 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const int wt = tid - 32 * kPrepWarp0;
         const int p = wt & 63, th = wt >> 6;  // key-dim pair (2p, 2p+1), token half
         const int d0 = 2 * p;
-        float lam_reg = 0.f;
-        if (wt < 64) {
-            const int tn = cb * kC + wt;
+        float lam_reg = 0.f;  // lambda of row wt >> 1
+        {
+            const int tn = cb * kC + (wt >> 1);
             lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
         }
         for (int r = 0; r < NC; ++r) {
@@ -505,45 +505,56 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             // key sum at the chunk start and lambda of the chunk
             if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
             const float lam_cur = lam_reg;
-            if (wt < 64) {
-                const int tn = (cb + r + 1) * kC + wt;
+            {
+                const int tn = (cb + r + 1) * kC + (wt >> 1);
                 lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
             }
             named_bar(NB_PREP, 128);
-            // row norms (thread = one row of q or k) and M . qbar, four partial sums each
+            // row norms of q and k and M . q: thread pair (2j, 2j+1) takes row j, each
+            // thread one 64-column half (one T64 tile) of both q and k, in fp32 pairs
             {
-                const int j = wt & 63;
-                const bool isq = wt < 64;  // warp-uniform
-                const uint8_t *base = slot + (isq ? SO_Q : SO_K);
-                float ss[4] = {0.f, 0.f, 0.f, 0.f}, md[4] = {0.f, 0.f, 0.f, 0.f};
+                const int j = wt >> 1, hh = wt & 1;
+                uint4 qv[8], kv[8];
 #pragma unroll
-                for (int t64 = 0; t64 < 2; ++t64) {
+                for (int cc = 0; cc < 8; ++cc) {
+                    qv[cc] = *reinterpret_cast<const uint4 *>(slot + SO_Q + hh * 8192 + t64_chunk(j, cc));
+                    kv[cc] = *reinterpret_cast<const uint4 *>(slot + SO_K + hh * 8192 + t64_chunk(j, cc));
+                }
+                const float *Mh = Mst + 64 * hh;
+                uint64_t sq0 = 0, sq1 = 0, sk0 = 0, sk1 = 0, md0 = 0, md1 = 0;
 #pragma unroll
-                    for (int cc = 0; cc < 8; ++cc) {
-                        float f[8];
-                        unpack_bf16x8(*reinterpret_cast<const uint4 *>(base + t64 * 8192 + t64_chunk(j, cc)), f);
+                for (int cc = 0; cc < 8; ++cc) {
+                    const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc);
+                    const ulonglong2 m23 = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc + 4);
+                    const uint32_t qw[4] = {qv[cc].x, qv[cc].y, qv[cc].z, qv[cc].w};
+                    const uint32_t kw[4] = {kv[cc].x, kv[cc].y, kv[cc].z, kv[cc].w};
+                    const uint64_t mp[4] = {m01.x, m01.y, m23.x, m23.y};
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) ss[e & 3] = fmaf(f[e], f[e], ss[e & 3]);
-                        if (isq) {
-                            const float4 m0v = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc);
-                            const float4 m1v = *reinterpret_cast<const float4 *>(Mst + 64 * t64 + 8 * cc + 4);
-                            const float mv[8] = {m0v.x, m0v.y, m0v.z, m0v.w, m1v.x, m1v.y, m1v.z, m1v.w};
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) md[e & 3] = fmaf(f[e], mv[e], md[e & 3]);
+                    for (int w = 0; w < 4; ++w) {
+                        const uint64_t q2 = f2_from_bf16x2(qw[w]), k2 = f2_from_bf16x2(kw[w]);
+                        if (w & 1) {
+                            sq1 = f2_fma(q2, q2, sq1); sk1 = f2_fma(k2, k2, sk1); md1 = f2_fma(q2, mp[w], md1);
+                        } else {
+                            sq0 = f2_fma(q2, q2, sq0); sk0 = f2_fma(k2, k2, sk0); md0 = f2_fma(q2, mp[w], md0);
                         }
                     }
                 }
-                const float sst = (ss[0] + ss[1]) + (ss[2] + ss[3]);
-                const float rn = a.l2norm ? rsqrtf(fmaxf(sst, 1e-12f)) : 1.f;
-                if (isq) {
+                const float2 a0 = f2_split(f2_add(sq0, sq1)), b0 = f2_split(f2_add(sk0, sk1)),
+                             c0v = f2_split(f2_add(md0, md1));
+                float ssq = a0.x + a0.y, ssk = b0.x + b0.y, mdt = c0v.x + c0v.y;
+                ssq += __shfl_xor_sync(0xffffffffu, ssq, 1);
+                ssk += __shfl_xor_sync(0xffffffffu, ssk, 1);
+                mdt += __shfl_xor_sync(0xffffffffu, mdt, 1);
+                if (hh == 0) {
+                    const float rq = a.l2norm ? rsqrtf(fmaxf(ssq, 1e-12f)) : 1.f;
                     const float iti = 1.f / static_cast<float>(tseq0 + (cb + r) * kC + j + 1);
-                    slot_f(s, MS_RQ)[j] = rn;
-                    slot_f(s, MS_MQ)[j] = ((md[0] + md[1]) + (md[2] + md[3])) * rn;
+                    slot_f(s, MS_RQ)[j] = rq;
+                    slot_f(s, MS_MQ)[j] = mdt * rq;
                     slot_f(s, MS_ITI)[j] = iti;
-                    slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(sst, 1e-12f) * rn : 1.f;
+                    slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(ssq, 1e-12f) * rq : 1.f;
                     slot_f(s, MS_LT)[j] = lam_cur * iti;
                 } else {
-                    slot_f(s, MS_RK)[j] = rn;
+                    slot_f(s, MS_RK)[j] = a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
                 }
             }
             // gate cumsum over this thread's 32 tokens for dims d0, d0+1
