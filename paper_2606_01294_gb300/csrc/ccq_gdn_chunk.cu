@@ -53,17 +53,18 @@ __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chun
 
 // ============================================================================ WY kernel
 //
-// One CTA (128 threads, four per SM) per (batch, head, chunk).  Writes Tb = Tt diag(beta)
+// One CTA (128 threads, five per SM) per (batch, head, chunk).  Writes Tb = Tt diag(beta)
 // as the bf16 rows [((b*H + h)*NC + r)*64 + i][0..63] of the workspace.
 
-constexpr uint32_t WY_K = 0;        // 16K  k raw -> kbar; after the KK product the block scratch Y
-constexpr uint32_t WY_A = 16384;    // 64 x 68 fp32: A; after the inversion the bf16 Tb tile (8K)
-constexpr uint32_t WY_T = 33792;    // 64 x 68 fp32: Tt
-constexpr uint32_t WY_MISC = 51200; // gc, beta, factors, rk, barriers
-constexpr uint32_t WY_SMEM = WY_MISC + 2048 + 1024;  // 54.3 KB: four CTAs per SM
+constexpr uint32_t WY_K = 0;        // 16K  k raw -> kbar (dead once the KK product has run)
+constexpr uint32_t WY_A = 0;        // 64 x 68 fp32 A over kbar; after the inversion the bf16 Tb tile
+constexpr uint32_t WY_T = 17408;    // 64 x 68 fp32: Tt
+constexpr uint32_t WY_Y = 34816;    // 3 x 256 fp32 block products of the inversion
+constexpr uint32_t WY_MISC = 37888; // gc, beta, factors, rk, barriers
+constexpr uint32_t WY_SMEM = WY_MISC + 2048 + 1024;  // 40 KB: five CTAs per SM
 constexpr int kAS = 68;             // padded fp32 row stride of A and Tt
 
-__global__ void __launch_bounds__(128, 4)
+__global__ void __launch_bounds__(128, 5)
 gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_tb,
               const ChunkArgs a, int NC) {
     extern __shared__ uint8_t smem_raw[];
@@ -71,7 +72,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     const uint32_t sb = smem_addr(sm);
     float *A = reinterpret_cast<float *>(sm + WY_A);
     float *Tt = reinterpret_cast<float *>(sm + WY_T);
-    float *Y = reinterpret_cast<float *>(sm + WY_K);               // 3 x 256 fp32, once kbar is dead
+    float *Y = reinterpret_cast<float *>(sm + WY_Y);
     float *gcs = reinterpret_cast<float *>(sm + WY_MISC);        // [64] cumulative log decay
     float *bet = gcs + 64;                                        // [64] beta
     float *epos = gcs + 128;                                      // [64] e^{gc - gc_m}
