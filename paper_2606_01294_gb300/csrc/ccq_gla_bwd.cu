@@ -66,7 +66,11 @@ namespace {
 constexpr int kC = 64;
 constexpr int kD = 128;
 constexpr int kThreads = 128;     // the state pass
-constexpr int kThreadsPar = 256;  // the chunk-parallel kernels: two warps per TMEM lane quadrant
+constexpr int kThreadsPar = 256;  // the chunk-parallel kernels: two warps per TMEM lane quadrant,
+constexpr int kLoadWarp = kThreadsPar / 32;       // then one warp that issues the input copies
+constexpr int kThreadsLoad = kThreadsPar + 32;
+// Barrier of the kThreadsPar compute threads (the load warp leaves once its copies are issued).
+__device__ __forceinline__ void compute_sync() { named_bar(1, kThreadsPar); }
 constexpr float kLog2e = 1.4426950408889634f;
 
 constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
@@ -161,7 +165,7 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
             }
         }
     }
-    __syncthreads();
+    compute_sync();
     const int p = pt & 63, qt = pt >> 6, d0 = 2 * p;
     float g0[16], g1[16];
     float r0 = 0.f, r1 = 0.f;
@@ -181,7 +185,7 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
     }
     gq4[qt * kD + d0] = r0;
     gq4[qt * kD + d0 + 1] = r1;
-    __syncthreads();  // every raw gate read, quarter sums visible
+    compute_sync();  // every raw gate read, quarter sums visible
     float off0 = 0.f, off1 = 0.f;
 #pragma unroll
     for (int q = 0; q < 3; ++q)
@@ -216,7 +220,7 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
         *reinterpret_cast<uint32_t *>(eg_tile + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
     }
     fence_proxy_async_smem();
-    __syncthreads();
+    compute_sync();
 }
 
 // Masked row of a 64 x 64 score tile: w_j = [j <= i] (sc_j - c) for the 32
@@ -265,11 +269,12 @@ constexpr uint32_t kMisc = 6784;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
 static_assert(OFF_SX == OFF_SK + 32768, "a checkpoint record lands as one block");
-enum { BAR_IN = 0, BAR_R1, BAR_R2, BAR_R3, BAR_R4, kBars };
+enum { BAR_IN = 0, BAR_INB, BAR_R1, BAR_R2, BAR_R3, BAR_R4, kBars };
+static_assert(M_BAR + 8 * kBars <= M_TMEM, "barriers reach the TMEM slot");
 constexpr uint32_t TM_SC = 0, TM_T1 = 64, TM_Z = 128, TM_DQ = 256;
 }  // namespace qk
 
-__global__ void __launch_bounds__(kThreadsPar, 1)
+__global__ void __launch_bounds__(kThreadsLoad, 1)
 gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                  const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_do,
                  const __grid_constant__ CUtensorMap map_g, const __grid_constant__ CUtensorMap map_dq,
@@ -310,49 +315,61 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     float *cvec = a.chunk_vec + static_cast<size_t>(blockIdx.x) * 3 * kD;  // f, e^{Gmid}, Dm increment
     int *status = a.status;
 
-    if (tid == 0) {
+    // The load warp issues the copies: first what the row norms and the gate prefix need
+    // (q, k, gates, M_r), then, once the compute threads are released, the rest, which
+    // lands while that preparation runs.  Issuing stalls as the copy engine fills, so no
+    // compute thread waits for it.
+    if (warp == kLoadWarp && lane == 0) {
         for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        uint64_t *bb = &bar[BAR_IN];
-        mbar_arrive_expect_tx(bb, 4 * 16384 + g_bytes + 65536 + 512);
-        tma_load_4d(sm + OFF_Q, &map_q, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_Q + 8192, &map_q, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, c0, b);
-        bulk_load(sm + OFF_SK, rec, 65536, bb);
-        bulk_load(misc + M_MR, rec + 65536, 512, bb);
-        // the chunk one wave later finds its inputs in L2
-        const int nx = blockIdx.x + a.wave;
-        if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
-            const int bh2 = nx / NC, r2 = nx % NC, b2 = bh2 / H, h2 = bh2 % H, c2 = r2 * kC;
-            tma_prefetch_l2_4d(&map_q, 0, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_q, 64, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_k, 0, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_k, 64, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_v, 0, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_v, 64, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_do, 0, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_do, 64, h2, c2, b2);
-            tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
-            bulk_prefetch_l2(a.ckpt + static_cast<size_t>(bh2) * ckpt_head_bytes(T) + static_cast<size_t>(r2) * kCkptChunkBytes,
-                             static_cast<uint32_t>(kCkptChunkBytes));
-        }
+        uint64_t *ba = &bar[BAR_IN], *bb = &bar[BAR_INB];
+        mbar_arrive_expect_tx(ba, 2 * 16384 + g_bytes + 512);
+        mbar_arrive_expect_tx(bb, 2 * 16384 + 65536);
+        tma_load_4d(sm + OFF_Q, &map_q, ba, 0, h, c0, b);
+        tma_load_4d(sm + OFF_Q + 8192, &map_q, ba, 64, h, c0, b);
+        tma_load_4d(sm + OFF_K, &map_k, ba, 0, h, c0, b);
+        tma_load_4d(sm + OFF_K + 8192, &map_k, ba, 64, h, c0, b);
+        tma_load_4d(sm + OFF_KD, &map_g, ba, 0, h, c0, b);
+        bulk_load(misc + M_MR, rec + 65536, 512, ba);
     }
     if (warp == 0) tmem_alloc(tmem_slot, 512);
-    for (int e = tid; e < 8192 / 16; e += kThreadsPar)
-        reinterpret_cast<uint4 *>(sm + OFF_BC)[e] = make_uint4(0u, 0u, 0u, 0u);
+    if (tid < kThreadsPar)
+        for (int e = tid; e < 8192 / 16; e += kThreadsPar)
+            reinterpret_cast<uint4 *>(sm + OFF_BC)[e] = make_uint4(0u, 0u, 0u, 0u);
     if (tid < kC) {
         const int n = c0 + tid;
         lamv[tid] = n < T ? a.lambda[(static_cast<size_t>(b) * T + n) * H + h] : 0.f;
         itauv[tid] = 1.f / static_cast<float>(tseq0 + n + 1);
     }
     __syncthreads();
+    if (warp == kLoadWarp) {
+        if (lane == 0) {
+            uint64_t *bb = &bar[BAR_INB];
+            tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, c0, b);
+            tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, c0, b);
+            bulk_load(sm + OFF_SK, rec, 65536, bb);
+            // the chunk one wave later finds its inputs in L2
+            const int nx = blockIdx.x + a.wave;
+            if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
+                const int bh2 = nx / NC, r2 = nx % NC, b2 = bh2 / H, h2 = bh2 % H, c2 = r2 * kC;
+                tma_prefetch_l2_4d(&map_q, 0, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_q, 64, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_k, 0, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_k, 64, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_v, 0, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_v, 64, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_do, 0, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_do, 64, h2, c2, b2);
+                tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
+                bulk_prefetch_l2(a.ckpt + static_cast<size_t>(bh2) * ckpt_head_bytes(T) + static_cast<size_t>(r2) * kCkptChunkBytes,
+                                 static_cast<uint32_t>(kCkptChunkBytes));
+            }
+        }
+        return;
+    }
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * qd) << 16);
@@ -375,6 +392,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     mbar_wait(&bar[BAR_IN], 0, abort_flag, status);
     prep_chunk(sm + OFF_Q, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, Mr, rqv, mqv, rkv, gq4,
                fv, emv, tid);
+    mbar_wait(&bar[BAR_INB], 0, abort_flag, status);
     tc_fence_before();
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
@@ -416,7 +434,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
         for (int k = 0; k < 4; ++k)  // Zi += W2 Kbar, Dq += P1 Kd
@@ -474,7 +492,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             red[grp * 128 + i] = dl;
             red[grp * 128 + 64 + i] = mdz;
         }
-        __syncthreads();
+        compute_sync();
         if (grp == 0 && hf == 0) {
             dl = red[i] + red[128 + i];
             mdzv[i] = red[64 + i] + red[192 + i];
@@ -484,7 +502,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (tid == 0 && !*abort_flag) {
         tma_store_4d(&map_qg, sm + OFF_V, 0, h, c0, b);
         tma_store_4d(&map_qg, sm + OFF_V + 8192, 64, h, c0, b);
@@ -524,7 +542,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
         for (int k = 0; k < 4; ++k)  // u += W3 Kbar
@@ -580,7 +598,7 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(kt, i, 4 * h2 + q4, x + 8 * q4);
         }
-        __syncthreads();
+        compute_sync();
         dot = red[i] + red[128 + i];
 #pragma unroll
         for (int q4 = 0; q4 < 4; ++q4) {
@@ -595,17 +613,17 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (tid == 0 && !*abort_flag) {
         tma_store_4d(&map_dq, sm + OFF_Q, 0, h, c0, b);
         tma_store_4d(&map_dq, sm + OFF_Q + 8192, 64, h, c0, b);
         tma_store_4d(&map_dkc, sm + OFF_K, 0, h, c0, b);
         tma_store_4d(&map_dkc, sm + OFF_K + 8192, 64, h, c0, b);
         tma_store_commit();
-        tma_store_wait_all();  // the stores have read shared memory and reached global memory
+        tma_store_wait_read();  // shared memory outlives the stores' reads
     }
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tbase, 512);
@@ -857,11 +875,12 @@ constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(OFF_DG + 64 * kDgStride * 4 <= OFF_P1, "dG scratch reaches P1");
 static_assert(OFF_DC == OFF_DS + 32768, "a state image record lands as one block");
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
-enum { BAR_IN = 0, BAR_R1, BAR_R2, kBars };
+enum { BAR_IN = 0, BAR_INB, BAR_R1, BAR_R2, kBars };
+static_assert(M_BAR + 8 * kBars <= M_TMEM, "barriers reach the TMEM slot");
 constexpr uint32_t TM_KC = 0, TM_T1 = 128, TM_SA = 192, TM_DK = 256, TM_DV = 384;
 }  // namespace kv
 
-__global__ void __launch_bounds__(kThreadsPar, 1)
+__global__ void __launch_bounds__(kThreadsLoad, 1)
 gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__ CUtensorMap map_v,
                   const __grid_constant__ CUtensorMap map_do, const __grid_constant__ CUtensorMap map_g,
                   const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_dkc,
@@ -890,44 +909,53 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     const uint32_t g_bytes = gate_f32 ? kC * kD * 4 : kC * kD * 2;
     int *status = a.status;
 
-    if (tid == 0) {
+    // The load warp issues k and the gates (the row norms and the gate prefix) first, then,
+    // once the compute threads are released, the rest.
+    if (warp == kLoadWarp && lane == 0) {
         for (int i = 0; i < kBars; ++i) mbar_init(&bar[i], 1);
         *abort_flag = 0;
         fence_barrier_init();
-        uint64_t *bb = &bar[BAR_IN];
-        mbar_arrive_expect_tx(bb, 6 * 16384 + g_bytes + 65536 + 1024);
-        tma_load_4d(sm + OFF_K, &map_k, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_K + 8192, &map_k, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_KD, &map_g, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_QG, &map_qg, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_QG + 8192, &map_qg, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_DKC, &map_dkc, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_DKC + 8192, &map_dkc, bb, 64, h, c0, b);
-        tma_load_4d(sm + OFF_GQ, &map_gq, bb, 0, h, c0, b);
-        tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, c0, b);
-        bulk_load(sm + OFF_DS, a.state_img + static_cast<size_t>(blockIdx.x) * 65536, 65536, bb);
-        bulk_load(misc + M_VEC, a.state_vec + static_cast<size_t>(blockIdx.x) * 2 * kD, 1024, bb);
-        // the chunk one wave later finds its inputs in L2
-        const int nx = blockIdx.x + a.wave;
-        if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
-            const int bh2 = nx / NC, r2 = nx % NC, b2 = bh2 / H, h2 = bh2 % H, c2 = r2 * kC;
-            const CUtensorMap *maps[6] = {&map_k, &map_v, &map_do, &map_qg, &map_dkc, &map_gq};
-#pragma unroll
-            for (int u = 0; u < 6; ++u) {
-                tma_prefetch_l2_4d(maps[u], 0, h2, c2, b2);
-                tma_prefetch_l2_4d(maps[u], 64, h2, c2, b2);
-            }
-            tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
-            bulk_prefetch_l2(a.state_img + static_cast<size_t>(nx) * 65536, 65536);
-            bulk_prefetch_l2(a.state_vec + static_cast<size_t>(nx) * 2 * kD, 1024);
-        }
+        uint64_t *ba = &bar[BAR_IN], *bb = &bar[BAR_INB];
+        mbar_arrive_expect_tx(ba, 16384 + g_bytes);
+        mbar_arrive_expect_tx(bb, 5 * 16384 + 65536 + 1024);
+        tma_load_4d(sm + OFF_K, &map_k, ba, 0, h, c0, b);
+        tma_load_4d(sm + OFF_K + 8192, &map_k, ba, 64, h, c0, b);
+        tma_load_4d(sm + OFF_KD, &map_g, ba, 0, h, c0, b);
     }
     if (warp == 0) tmem_alloc(tmem_slot, 512);
     __syncthreads();
+    if (warp == kLoadWarp) {
+        if (lane == 0) {
+            uint64_t *bb = &bar[BAR_INB];
+            tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, c0, b);
+            tma_load_4d(sm + OFF_DO, &map_do, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_DO + 8192, &map_do, bb, 64, h, c0, b);
+            tma_load_4d(sm + OFF_QG, &map_qg, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_QG + 8192, &map_qg, bb, 64, h, c0, b);
+            tma_load_4d(sm + OFF_DKC, &map_dkc, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_DKC + 8192, &map_dkc, bb, 64, h, c0, b);
+            tma_load_4d(sm + OFF_GQ, &map_gq, bb, 0, h, c0, b);
+            tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, c0, b);
+            bulk_load(sm + OFF_DS, a.state_img + static_cast<size_t>(blockIdx.x) * 65536, 65536, bb);
+            bulk_load(misc + M_VEC, a.state_vec + static_cast<size_t>(blockIdx.x) * 2 * kD, 1024, bb);
+            // the chunk one wave later finds its inputs in L2
+            const int nx = blockIdx.x + a.wave;
+            if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
+                const int bh2 = nx / NC, r2 = nx % NC, b2 = bh2 / H, h2 = bh2 % H, c2 = r2 * kC;
+                const CUtensorMap *maps[6] = {&map_k, &map_v, &map_do, &map_qg, &map_dkc, &map_gq};
+#pragma unroll
+                for (int u = 0; u < 6; ++u) {
+                    tma_prefetch_l2_4d(maps[u], 0, h2, c2, b2);
+                    tma_prefetch_l2_4d(maps[u], 64, h2, c2, b2);
+                }
+                tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
+                bulk_prefetch_l2(a.state_img + static_cast<size_t>(nx) * 65536, 65536);
+                bulk_prefetch_l2(a.state_vec + static_cast<size_t>(nx) * 2 * kD, 1024);
+            }
+        }
+        return;
+    }
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
     const uint32_t tq = tbase + (static_cast<uint32_t>(32 * qd) << 16);
@@ -946,6 +974,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     mbar_wait(&bar[BAR_IN], 0, abort_flag, status);
     prep_chunk(nullptr, sm + OFF_K, sm + OFF_KD, sm + OFF_EG, gate_f32, a.l2norm, nullptr, nullptr, nullptr,
                rkv, gq4, nullptr, nullptr, tid);
+    mbar_wait(&bar[BAR_INB], 0, abort_flag, status);
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
         for (int k = 0; k < 8; ++k) {  // T1 = dO V^T, SA = Kd QG^T
@@ -988,7 +1017,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
         for (int k = 0; k < 4; ++k)  // dkw += P1^T QG, dv += SA dO
@@ -1043,7 +1072,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(vt, i, 4 * h2 + q4, x + 8 * q4);
         }
-        __syncthreads();
+        compute_sync();
         dot = red[i] + red[128 + i];
 #pragma unroll
         for (int q4 = 0; q4 < 4; ++q4) {
@@ -1058,7 +1087,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
     }
     fence_proxy_async_smem();
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (tid == 0 && !*abort_flag) {
         tma_store_4d(&map_dk, sm + OFF_K, 0, h, c0, b);
         tma_store_4d(&map_dk, sm + OFF_K + 8192, 64, h, c0, b);
@@ -1077,7 +1106,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
             tot += x[u];
         }
         red[hh * 128 + d] = tot;
-        __syncthreads();
+        compute_sync();
         float acc = vec[kD + d] + (hh == 0 ? red[128 + d] : 0.f);
         const int nvalid = min(kC, T - c0);
 #pragma unroll
@@ -1091,9 +1120,9 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
             }
         }
     }
-    if (tid == 0) tma_store_wait_all();
+    if (tid == 0) tma_store_wait_read();  // shared memory outlives the stores' reads
     tc_fence_before();
-    __syncthreads();
+    compute_sync();
     if (warp == 0) {
         tc_fence_after();
         tmem_dealloc(tbase, 512);
@@ -1118,14 +1147,14 @@ cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s) {
     }
     const int nc = (a.T + kC - 1) / kC;
     const int chunks = a.B * a.H * nc;
-    gla_bwd_q_kernel<<<chunks, kThreadsPar, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq,
+    gla_bwd_q_kernel<<<chunks, kThreadsLoad, qk::kSmem, s>>>(m.q, m.k, m.v, m.dO, m.g, m.dq, m.qg, m.dkc, m.gq,
                                                           m.dzr, a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     gla_bwd_state_kernel<<<a.B * a.H, kThreads, st::kSmem, s>>>(m.qg, m.dO, m.dzr, m.q, a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    gla_bwd_kv_kernel<<<chunks, kThreadsPar, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
+    gla_bwd_kv_kernel<<<chunks, kThreadsLoad, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);
     return cudaGetLastError();
 }
 
