@@ -56,8 +56,8 @@ __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chun
 // One CTA (128 threads, five per SM) per (batch, head, chunk).  Writes Tb = Tt diag(beta)
 // as the bf16 rows [((b*H + h)*NC + r)*64 + i][0..63] of the workspace.
 
-constexpr uint32_t WY_K = 0;        // 16K  k raw -> kbar (dead once the KK product has run)
-constexpr uint32_t WY_A = 0;        // 64 x 68 fp32 A over kbar; after the inversion the bf16 Tb tile
+constexpr uint32_t WY_K = 0;        // 16K  raw k (dead once the KK product and the norms have read it)
+constexpr uint32_t WY_A = 0;        // 64 x 68 fp32 A over k; after the inversion the bf16 Tb tile
 constexpr uint32_t WY_T = 17408;    // 64 x 68 fp32: Tt
 constexpr uint32_t WY_Y = 34816;    // 3 x 256 fp32 block products of the inversion
 constexpr uint32_t WY_MISC = 37888; // gc, beta, factors, rk, barriers
@@ -75,8 +75,8 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     float *Y = reinterpret_cast<float *>(sm + WY_Y);
     float *gcs = reinterpret_cast<float *>(sm + WY_MISC);        // [64] cumulative log decay
     float *bet = gcs + 64;                                        // [64] beta
-    float *epos = gcs + 128;                                      // [64] e^{gc - gc_m}
-    float *eneg = gcs + 192;                                      // [64] e^{gc_m - gc}
+    float *epos = gcs + 128;                                      // [64] beta e^{gc - gc_m} / |k|
+    float *eneg = gcs + 192;                                      // [64] e^{gc_m - gc} / |k|
     float *rk = gcs + 256;                                        // [64] 1/|k|
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + WY_MISC + 1536);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(sm + WY_MISC + 1560);
@@ -122,6 +122,17 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         gcs[2 * lane + 1] = p;
     }
     mbar_wait(&bar[0], 0, abort_flag, status);
+    // ---- KK = K K^T on the raw keys (M = 64: rows 16w..16w+15 in lanes 32w..32w+15), issued
+    // as soon as k lands; the norms run under it and scale A instead of the keys
+    if (tid == 0 && !*abort_flag) {
+        tc_fence_after();
+        const uint64_t dk = make_desc(sb + WY_K, 16, 1024);
+        for (int k = 0; k < 8; ++k) {
+            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
+            mma_bf16(tb, dk + ko, dk + ko, make_idesc(64, 64, 0, 0), k != 0);
+        }
+        mma_commit(&bar[1]);
+    }
     {
         // row j = tid >> 1, one T64 tile (column half) per thread
         const int j = tid >> 1, hh = tid & 1;
@@ -140,59 +151,37 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         if (hh == 0) rk[j] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
     }
     __syncthreads();
+    // row and column factors of A: A_ij = (beta_i e^{gc_i - gc_m} rk_i) (e^{gc_m - gc_j} rk_j) KK_ij
     if (tid < 64) {
         const float gm = gcs[31];
-        epos[tid] = fast_exp2((gcs[tid] - gm) * kLog2e);
-        eneg[tid] = fast_exp2((gm - gcs[tid]) * kLog2e);
+        epos[tid] = bet[tid] * fast_exp2((gcs[tid] - gm) * kLog2e) * rk[tid];
+        eneg[tid] = fast_exp2((gm - gcs[tid]) * kLog2e) * rk[tid];
     }
-    // ---- kbar in place (row j = tid/2, column half tid%2)
-    {
-        const int j = tid >> 1, hf = tid & 1;
-        const float s = rk[j];
-        const uint64_t s2 = f2_make(s, s);
-        uint8_t *tile = sm + WY_K + hf * 8192;
-#pragma unroll
-        for (int cc = 0; cc < 8; ++cc) {
-            const uint4 v = *reinterpret_cast<const uint4 *>(tile + t64_chunk(j, cc));
-            *reinterpret_cast<uint4 *>(tile + t64_chunk(j, cc)) =
-                make_uint4(bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.x), s2)), bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.y), s2)),
-                           bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.z), s2)), bf16x2_from_f2(f2_mul(f2_from_bf16x2(v.w), s2)));
-        }
-    }
-    fence_proxy_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    // ---- KK = Kbar Kbar^T (M = 64: rows 16w..16w+15 in lanes 32w..32w+15)
-    if (tid == 0 && !*abort_flag) {
-        tc_fence_after();
-        const uint64_t dk = make_desc(sb + WY_K, 16, 1024);
-        for (int k = 0; k < 8; ++k) {
-            const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-            mma_bf16(tb, dk + ko, dk + ko, make_idesc(64, 64, 0, 0), k != 0);
-        }
-        mma_commit(&bar[1]);
-    }
+    __syncthreads();  // factors visible; every read of the k tile done
     mbar_wait(&bar[1], 0, abort_flag, status);
     tc_fence_after();
     {
-        // A_ij = beta_i e^{gc_i - gc_j} KK_ij for j < i
+        // A_ij for j < i, written over the k tile (the product has read it)
         const int i = 16 * warp + (lane & 15), hf = lane >> 4;
         float kk[32];
         tmem_ld16x2_32<32>(tq, kk);
-        const float ri = bet[i] * epos[i];
+        const float ri = epos[i];
 #pragma unroll
         for (int q4 = 0; q4 < 8; ++q4) {
+            const float4 cf = *reinterpret_cast<const float4 *>(eneg + 32 * hf + 4 * q4);
+            const float cfa[4] = {cf.x, cf.y, cf.z, cf.w};
             float w[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int j = 32 * hf + 4 * q4 + e;
-                w[e] = (j < i) ? ri * eneg[j] * kk[4 * q4 + e] : 0.f;
+                w[e] = (j < i) ? ri * cfa[e] * kk[4 * q4 + e] : 0.f;
             }
             *reinterpret_cast<float4 *>(A + i * kAS + 32 * hf + 4 * q4) = make_float4(w[0], w[1], w[2], w[3]);
         }
     }
     __syncthreads();
     // ---- Tt = (I + A)^{-1}: the four 16 x 16 diagonal blocks by forward substitution
+    // (thread = one column c of block bb; the row's A entries as float4 loads)
     if (tid < 64) {
         const int bb = tid >> 4, c = tid & 15, o = 16 * bb;
         float x[16];
@@ -200,7 +189,15 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         for (int rr = 0; rr < 16; ++rr) {
             float s = 0.f;
 #pragma unroll
-            for (int j = 0; j < rr; ++j) s = fmaf(A[(o + rr) * kAS + o + j], x[j], s);
+            for (int j4 = 0; j4 < 4; ++j4) {
+                if (4 * j4 < rr) {
+                    const float4 av = *reinterpret_cast<const float4 *>(A + (o + rr) * kAS + o + 4 * j4);
+                    s = fmaf(av.x, x[4 * j4], s);
+                    if (4 * j4 + 1 < rr) s = fmaf(av.y, x[4 * j4 + 1], s);
+                    if (4 * j4 + 2 < rr) s = fmaf(av.z, x[4 * j4 + 2], s);
+                    if (4 * j4 + 3 < rr) s = fmaf(av.w, x[4 * j4 + 3], s);
+                }
+            }
             x[rr] = (rr < c) ? 0.f : ((rr == c) ? 1.f : -s);
         }
 #pragma unroll
@@ -209,67 +206,61 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     __syncthreads();
     // off-diagonal blocks, by distance from the diagonal:
     //   Tt_IJ = -Tt_II sum_{K=J}^{I-1} A_IK Tt_KJ
-    // 16 threads per 16 x 16 block, each a 4 x 4 sub-tile with float4 shared loads
+    // one warp per 16 x 16 block, each thread a 4-row x 2-column sub-tile in fp32 pairs
     for (int dist = 1; dist < 4; ++dist) {
         const int nblk = 4 - dist;
-        const int blk = tid >> 4, t = tid & 15, r0 = 4 * (t >> 2), cq = 4 * (t & 3);
+        const int blk = warp, r0 = 4 * (lane >> 3), cq = 2 * (lane & 7);
         const int J = blk, I = blk + dist;
         if (blk < nblk) {
-            float acc[4][4] = {};
+            uint64_t acc[4] = {0, 0, 0, 0};
             for (int K = J; K < I; ++K) {
 #pragma unroll
                 for (int m = 0; m < 16; m += 4) {
-                    float4 av[4], tv[4];
+                    float4 av[4];
+                    uint64_t tv[4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
                         av[u] = *reinterpret_cast<const float4 *>(A + (16 * I + r0 + u) * kAS + 16 * K + m);
-                        tv[u] = *reinterpret_cast<const float4 *>(Tt + (16 * K + m + u) * kAS + 16 * J + cq);
+                        tv[u] = *reinterpret_cast<const uint64_t *>(Tt + (16 * K + m + u) * kAS + 16 * J + cq);
                     }
 #pragma unroll
                     for (int u = 0; u < 4; ++u) {
-                        const float a4[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
-#pragma unroll
-                        for (int mm = 0; mm < 4; ++mm) {
-                            acc[u][0] = fmaf(a4[mm], tv[mm].x, acc[u][0]);
-                            acc[u][1] = fmaf(a4[mm], tv[mm].y, acc[u][1]);
-                            acc[u][2] = fmaf(a4[mm], tv[mm].z, acc[u][2]);
-                            acc[u][3] = fmaf(a4[mm], tv[mm].w, acc[u][3]);
-                        }
+                        acc[u] = f2_fma(f2_make(av[u].x, av[u].x), tv[0], acc[u]);
+                        acc[u] = f2_fma(f2_make(av[u].y, av[u].y), tv[1], acc[u]);
+                        acc[u] = f2_fma(f2_make(av[u].z, av[u].z), tv[2], acc[u]);
+                        acc[u] = f2_fma(f2_make(av[u].w, av[u].w), tv[3], acc[u]);
                     }
                 }
             }
 #pragma unroll
             for (int u = 0; u < 4; ++u)
-                *reinterpret_cast<float4 *>(Y + blk * 256 + (r0 + u) * 16 + cq) =
-                    make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
+                *reinterpret_cast<uint64_t *>(Y + blk * 256 + (r0 + u) * 16 + cq) = acc[u];
         }
         __syncthreads();
         if (blk < nblk) {
-            float acc[4][4] = {};
+            uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
             for (int m = 0; m < 16; m += 4) {
-                float4 av[4], yv[4];
+                float4 av[4];
+                uint64_t yv[4];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     av[u] = *reinterpret_cast<const float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * I + m);
-                    yv[u] = *reinterpret_cast<const float4 *>(Y + blk * 256 + (m + u) * 16 + cq);
+                    yv[u] = *reinterpret_cast<const uint64_t *>(Y + blk * 256 + (m + u) * 16 + cq);
                 }
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
-                    const float a4[4] = {av[u].x, av[u].y, av[u].z, av[u].w};
-#pragma unroll
-                    for (int mm = 0; mm < 4; ++mm) {
-                        acc[u][0] = fmaf(a4[mm], yv[mm].x, acc[u][0]);
-                        acc[u][1] = fmaf(a4[mm], yv[mm].y, acc[u][1]);
-                        acc[u][2] = fmaf(a4[mm], yv[mm].z, acc[u][2]);
-                        acc[u][3] = fmaf(a4[mm], yv[mm].w, acc[u][3]);
-                    }
+                    acc[u] = f2_fma(f2_make(av[u].x, av[u].x), yv[0], acc[u]);
+                    acc[u] = f2_fma(f2_make(av[u].y, av[u].y), yv[1], acc[u]);
+                    acc[u] = f2_fma(f2_make(av[u].z, av[u].z), yv[2], acc[u]);
+                    acc[u] = f2_fma(f2_make(av[u].w, av[u].w), yv[3], acc[u]);
                 }
             }
 #pragma unroll
-            for (int u = 0; u < 4; ++u)
-                *reinterpret_cast<float4 *>(Tt + (16 * I + r0 + u) * kAS + 16 * J + cq) =
-                    make_float4(-acc[u][0], -acc[u][1], -acc[u][2], -acc[u][3]);
+            for (int u = 0; u < 4; ++u) {
+                const float2 v = f2_split(acc[u]);
+                *reinterpret_cast<float2 *>(Tt + (16 * I + r0 + u) * kAS + 16 * J + cq) = make_float2(-v.x, -v.y);
+            }
         }
         __syncthreads();
     }
@@ -281,11 +272,14 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
             float wb[8];
             const float4 t0 = *reinterpret_cast<const float4 *>(Tt + i * kAS + 32 * hf + 8 * q4);
             const float4 t1 = *reinterpret_cast<const float4 *>(Tt + i * kAS + 32 * hf + 8 * q4 + 4);
+            const float4 b0 = *reinterpret_cast<const float4 *>(bet + 32 * hf + 8 * q4);
+            const float4 b1 = *reinterpret_cast<const float4 *>(bet + 32 * hf + 8 * q4 + 4);
             const float tr[8] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
+            const float br[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
                 const int j = 32 * hf + 8 * q4 + e;
-                wb[e] = (j <= i) ? tr[e] * bet[j] : 0.f;
+                wb[e] = (j <= i) ? tr[e] * br[e] : 0.f;
             }
             store_row_chunk(sm + WY_A, i, 4 * hf + q4, wb);
         }
