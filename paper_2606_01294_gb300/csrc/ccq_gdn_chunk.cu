@@ -109,7 +109,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     const uint32_t tb = *tslot;
     const uint32_t tq = tb + (static_cast<uint32_t>(32 * warp) << 16);
 
-    // ---- cumulative decay (warp 2: two values per lane, shuffle scan) and the k row norms
+    // ---- cumulative decay (warp 2: two values per lane, shuffle scan)
     if (warp == 2) {
         const float x0 = gcs[2 * lane], x1 = gcs[2 * lane + 1];
         float p = x0 + x1;
@@ -122,8 +122,8 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         gcs[2 * lane + 1] = p;
     }
     mbar_wait(&bar[0], 0, abort_flag, status);
-    // ---- KK = K K^T on the raw keys (M = 64: rows 16w..16w+15 in lanes 32w..32w+15), issued
-    // as soon as k lands; the norms run under it and scale A instead of the keys
+    // ---- KK = K K^T on the raw keys (M = 64: rows 16w..16w+15 in lanes 32w..32w+15); the
+    // key norms are its diagonal, and they scale A instead of the keys
     if (tid == 0 && !*abort_flag) {
         tc_fence_after();
         const uint64_t dk = make_desc(sb + WY_K, 16, 1024);
@@ -133,22 +133,24 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         }
         mma_commit(&bar[1]);
     }
-    {
-        // row j = tid >> 1, one T64 tile (column half) per thread
-        const int j = tid >> 1, hh = tid & 1;
-        uint64_t s0 = 0, s1 = 0;
+    mbar_wait(&bar[1], 0, abort_flag, status);
+    tc_fence_after();
+    const int i = 16 * warp + (lane & 15), hf = lane >> 4;  // row i, columns 32 hf .. 32 hf + 31
+    float kk[32];
+    tmem_ld16x2_32<32>(tq, kk);
+    if ((i >> 5) == hf) {  // this thread holds KK_ii = |k_i|^2
+        // column i & 31 = 16 (warp & 1) + (lane & 15): a select tree on those bits, which keeps
+        // kk in registers
+        const int e = i & 31;
+        float v[16];
 #pragma unroll
-        for (int cc = 0; cc < 8; ++cc) {
-            const uint4 v = *reinterpret_cast<const uint4 *>(sm + WY_K + hh * 8192 + t64_chunk(j, cc));
-            const uint64_t p0 = f2_from_bf16x2(v.x), p1 = f2_from_bf16x2(v.y), p2 = f2_from_bf16x2(v.z),
-                           p3 = f2_from_bf16x2(v.w);
-            s0 = f2_fma(p0, p0, s0); s1 = f2_fma(p1, p1, s1);
-            s0 = f2_fma(p2, p2, s0); s1 = f2_fma(p3, p3, s1);
-        }
-        const float2 sv = f2_split(f2_add(s0, s1));
-        float ss = sv.x + sv.y;
-        ss += __shfl_xor_sync(0xffffffffu, ss, 1);
-        if (hh == 0) rk[j] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
+        for (int u = 0; u < 16; ++u) v[u] = (e & 16) ? kk[16 + u] : kk[u];
+#pragma unroll
+        for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+            for (int u = 0; u < w; ++u) v[u] = (e & w) ? v[w + u] : v[u];
+        const float d = v[0];
+        rk[i] = a.l2norm ? rsqrtf(fmaxf(d, 1e-12f)) : 1.f;
     }
     __syncthreads();
     // row and column factors of A: A_ij = (beta_i e^{gc_i - gc_m} rk_i) (e^{gc_m - gc_j} rk_j) KK_ij
@@ -157,14 +159,9 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         epos[tid] = bet[tid] * fast_exp2((gcs[tid] - gm) * kLog2e) * rk[tid];
         eneg[tid] = fast_exp2((gm - gcs[tid]) * kLog2e) * rk[tid];
     }
-    __syncthreads();  // factors visible; every read of the k tile done
-    mbar_wait(&bar[1], 0, abort_flag, status);
-    tc_fence_after();
+    __syncthreads();
     {
         // A_ij for j < i, written over the k tile (the product has read it)
-        const int i = 16 * warp + (lane & 15), hf = lane >> 4;
-        float kk[32];
-        tmem_ld16x2_32<32>(tq, kk);
         const float ri = epos[i];
 #pragma unroll
         for (int q4 = 0; q4 < 8; ++q4) {
