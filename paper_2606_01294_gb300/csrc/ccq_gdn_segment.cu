@@ -377,66 +377,89 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
 // Per (sequence, block of 16 state columns): walks the segments, replacing each slot's
 // S (Q), C (dC) and m (dm) with the states entering that segment:
 //   H_{s+1} = P_s H_s + Q_s,  C_{s+1} = C_s + dC_s,  m_{s+1} = m_s + dm_s.
-// P_s is staged in shared memory with coalesced loads (64 KB); the product runs there.
+// P_s is staged in shared memory with coalesced loads into rows padded to kPS floats (the
+// row-per-lane reads of the product then spread over the banks); the loads of segment s+1
+// (P, Q, dC) are in flight while segment s computes.
 constexpr int kCols = 16;
-constexpr int kCombineSmem = (kSS + kD * kCols) * 4;
+constexpr int kPS = kD + 4;
+constexpr int kCombineSmem = (kD * kPS + kD * kCols) * 4;
 
 __global__ void __launch_bounds__(256)
 gdn_segment_combine_kernel(const ChunkArgs a) {
     extern __shared__ float csm[];
-    float *Ps = csm;               // [128][128]
-    float *hcur = csm + kSS;       // [128][16]
+    float *Ps = csm;               // [128][kPS]
+    float *hcur = csm + kD * kPS;  // [128][16]
     const int nblk = kD / kCols;
     const int seq = blockIdx.x / nblk, cblk = blockIdx.x % nblk;
     const size_t sq = static_cast<size_t>(seq);
     const int tid = threadIdx.x;
     const int arow = tid >> 1, cl = 8 * (tid & 1), c0 = kCols * cblk + cl;  // row arow, 8 columns
     float hreg[8], creg[8];
+    {
+        const float4 *h4 = a.S0 ? reinterpret_cast<const float4 *>(a.S0 + sq * kSS + arow * kD + c0) : nullptr;
+        const float4 *c4 = a.C0 ? reinterpret_cast<const float4 *>(a.C0 + sq * kSS + arow * kD + c0) : nullptr;
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-        hreg[u] = a.S0 ? a.S0[sq * kSS + arow * kD + c0 + u] : 0.f;
-        creg[u] = a.C0 ? a.C0[sq * kSS + arow * kD + c0 + u] : 0.f;
+        for (int u = 0; u < 2; ++u) {
+            const float4 hv = h4 ? h4[u] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 cv = c4 ? c4[u] : make_float4(0.f, 0.f, 0.f, 0.f);
+            hreg[4 * u] = hv.x; hreg[4 * u + 1] = hv.y; hreg[4 * u + 2] = hv.z; hreg[4 * u + 3] = hv.w;
+            creg[4 * u] = cv.x; creg[4 * u + 1] = cv.y; creg[4 * u + 2] = cv.z; creg[4 * u + 3] = cv.w;
+        }
     }
     float mreg = (cblk == 0 && tid < kD) ? (a.m0 ? a.m0[sq * kD + tid] : 0.f) : 0.f;
+    // segment s+1's operands in registers while segment s computes
+    float4 pv[16], qv[2], dv[2];
+    auto load_next = [&](int s) {
+        const float *slot = a.seg_ws + (sq * a.nseg + s) * kGdnSegFloats;
+        const float4 *src = reinterpret_cast<const float4 *>(slot + kSS);
+#pragma unroll
+        for (int u = 0; u < 16; ++u) pv[u] = src[u * 256 + tid];
+        const float4 *q4 = reinterpret_cast<const float4 *>(slot + arow * kD + c0);
+        const float4 *d4 = reinterpret_cast<const float4 *>(slot + 2 * kSS + arow * kD + c0);
+        qv[0] = q4[0]; qv[1] = q4[1];
+        dv[0] = d4[0]; dv[1] = d4[1];
+    };
+    if (a.nseg > 0) load_next(0);
     for (int s = 0; s < a.nseg; ++s) {
         float *slot = a.seg_ws + (sq * a.nseg + s) * kGdnSegFloats;
-        // stage P_s (16 float4 per thread, all in flight) and this block's H_s columns
-        {
-            const float4 *src = reinterpret_cast<const float4 *>(slot + kSS);
-            float4 *dst = reinterpret_cast<float4 *>(Ps);
-            float4 v[16];
+        // stage P_s (element e = 4 (256 u + tid): row e / 128, column e % 128) and H_s
 #pragma unroll
-            for (int u = 0; u < 16; ++u) v[u] = src[u * 256 + tid];
-#pragma unroll
-            for (int u = 0; u < 16; ++u) dst[u * 256 + tid] = v[u];
+        for (int u = 0; u < 16; ++u) {
+            const int e = 4 * (u * 256 + tid);
+            *reinterpret_cast<float4 *>(Ps + (e >> 7) * kPS + (e & 127)) = pv[u];
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) hcur[arow * kCols + cl + u] = hreg[u];
-        float acc[8], dcv[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            acc[u] = slot[arow * kD + c0 + u];            // Q_s
-            dcv[u] = slot[2 * kSS + arow * kD + c0 + u];  // dC_s
-        }
+        for (int u = 0; u < 2; ++u)
+            *reinterpret_cast<float4 *>(hcur + arow * kCols + cl + 4 * u) =
+                make_float4(hreg[4 * u], hreg[4 * u + 1], hreg[4 * u + 2], hreg[4 * u + 3]);
+        float acc[8] = {qv[0].x, qv[0].y, qv[0].z, qv[0].w, qv[1].x, qv[1].y, qv[1].z, qv[1].w};  // Q_s
+        const float dcv[8] = {dv[0].x, dv[0].y, dv[0].z, dv[0].w, dv[1].x, dv[1].y, dv[1].z, dv[1].w};
         __syncthreads();
-        const float *P = Ps + arow * kD;
+        if (s + 1 < a.nseg) load_next(s + 1);
+        const float *P = Ps + arow * kPS;
 #pragma unroll 4
         for (int bb = 0; bb < kD; bb += 4) {
             const float4 p4 = *reinterpret_cast<const float4 *>(P + bb);
-            const float pv[4] = {p4.x, p4.y, p4.z, p4.w};
+            const float pw[4] = {p4.x, p4.y, p4.z, p4.w};
 #pragma unroll
             for (int t = 0; t < 4; ++t) {
                 const float4 h0 = *reinterpret_cast<const float4 *>(hcur + (bb + t) * kCols + cl);
                 const float4 h1 = *reinterpret_cast<const float4 *>(hcur + (bb + t) * kCols + cl + 4);
                 const float hv[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
 #pragma unroll
-                for (int u = 0; u < 8; ++u) acc[u] = fmaf(pv[t], hv[u], acc[u]);
+                for (int u = 0; u < 8; ++u) acc[u] = fmaf(pw[t], hv[u], acc[u]);
             }
+        }
+        // this slot now holds the states entering segment s
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            *reinterpret_cast<float4 *>(slot + arow * kD + c0 + 4 * u) =
+                make_float4(hreg[4 * u], hreg[4 * u + 1], hreg[4 * u + 2], hreg[4 * u + 3]);
+            *reinterpret_cast<float4 *>(slot + 2 * kSS + arow * kD + c0 + 4 * u) =
+                make_float4(creg[4 * u], creg[4 * u + 1], creg[4 * u + 2], creg[4 * u + 3]);
         }
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
-            slot[arow * kD + c0 + u] = hreg[u];
-            slot[2 * kSS + arow * kD + c0 + u] = creg[u];
             hreg[u] = acc[u];
             creg[u] += dcv[u];
         }
