@@ -65,7 +65,7 @@ namespace {
 
 constexpr int kC = 64;
 constexpr int kD = 128;
-constexpr int kThreads = 128;     // the state pass
+constexpr int kThreads = 256;     // the state pass: two warps per TMEM lane quadrant
 constexpr int kThreadsPar = 256;  // the chunk-parallel kernels: two warps per TMEM lane quadrant,
 constexpr int kLoadWarp = kThreadsPar / 32;       // then one warp that issues the input copies
 constexpr int kThreadsLoad = kThreadsPar + 32;
@@ -640,7 +640,7 @@ constexpr uint32_t OFF_SX = 2 * BUF_BYTES;      // 131072: Sx_r (checkpoint tile
 constexpr uint32_t OFF_IMG = OFF_SX + 32768;    // 163840: staging of the images written per chunk:
                                                 //   Diag(e^{Gc-Gmid}) dS_{r+1} (32 KB), DC_{r+1} (32 KB)
 constexpr uint32_t OFF_MISC = OFF_IMG + 65536;  // 229376
-constexpr uint32_t M_DM = 0, M_EMP = 512, M_CARRY = 1024, M_BAR = 1536, M_TMEM = 1568, M_ABORT = 1572;
+constexpr uint32_t M_DM = 0, M_CARRY = 512, M_BAR = 1536, M_TMEM = 1568, M_ABORT = 1572;
 constexpr uint32_t kMisc = 1600;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
@@ -648,6 +648,10 @@ enum { BAR_IN0 = 0, BAR_IN1, BAR_SX, BAR_MMA, kBars };
 constexpr uint32_t TM_X = 0, TM_DC = 128;
 }  // namespace st
 
+// Two warps per TMEM lane quadrant: thread (row, half) holds state row `row`, columns
+// [64 half, 64 half + 64).  Per chunk r (last to first) the chain is: read X (the state
+// after chunk r+1's update), its gate carry against Sx_{r+1}, rescale to Diag(e^{Gc-Gmid})
+// dS_{r+1} (the image, and X in place), the DC image, then the two updates of chunk r.
 __global__ void __launch_bounds__(kThreads, 1)
 gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_do,
                      const __grid_constant__ CUtensorMap map_dzr, const __grid_constant__ CUtensorMap map_q,
@@ -658,13 +662,13 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *Dm = reinterpret_cast<float *>(misc + M_DM);
-    float *emp = reinterpret_cast<float *>(misc + M_EMP);
-    float *carry = reinterpret_cast<float *>(misc + M_CARRY);
+    float *carry = reinterpret_cast<float *>(misc + M_CARRY);  // [2 halves][128] partial row sums
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5;
+    const int row = tid & (kD - 1), half = tid >> 7;
     const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
     const int T = a.T, NC = (T + kC - 1) / kC;
     const uint8_t *ck = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T);
@@ -680,16 +684,17 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
-    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * warp) << 16);
+    const uint32_t tq = tbase + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
     {
         // X <- dS_T, DC <- dC_T, Dm <- dm_T; the gate carry of the last chunk is rowsum(dS_T * S_T)
-        const size_t row = static_cast<size_t>(bh) * kD + tid;
-        const float *dst_row = a.dST ? a.dST + row * kD : nullptr;
-        const float *dct_row = a.dCT ? a.dCT + row * kD : nullptr;
-        const float *st_row = reinterpret_cast<const float *>(ck + static_cast<size_t>(NC) * kCkptChunkBytes) + tid * kD;
+        const size_t grow = static_cast<size_t>(bh) * kD + row;
+        const float *dst_row = a.dST ? a.dST + grow * kD : nullptr;
+        const float *dct_row = a.dCT ? a.dCT + grow * kD : nullptr;
+        const float *st_row = reinterpret_cast<const float *>(ck + static_cast<size_t>(NC) * kCkptChunkBytes) + row * kD;
         float cs = 0.f;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int cc = 0; cc < 2; ++cc) {
+            const int c = 2 * half + cc;
             float x[32], y[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
@@ -701,9 +706,8 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
             tmem_st32(tq + TM_DC + 32 * c, y);
         }
         tmem_wait_st();
-        carry[tid] = cs;
-        emp[tid] = 1.f;
-        Dm[tid] = a.dmT ? a.dmT[row] : 0.f;
+        carry[half * kD + row] = cs;
+        if (half == 0) Dm[row] = a.dmT ? a.dmT[grow] : 0.f;
     }
     auto issue = [&](int r, int buf) {
         const int tg = r * kC;
@@ -726,52 +730,74 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
     if (tid == 0 && NC > 0) {
         issue(NC - 1, 0);
         if (NC > 1) issue(NC - 2, 1);
-        issue_sx(NC - 1);
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
 
+    float em_next = 1.f;  // e^{Gmid_{r+1}} (1 past the last chunk)
     for (int it = 0; it < NC; ++it) {
         const int r = NC - 1 - it, buf = it & 1;
-        const uint32_t bpar = (it >> 1) & 1, par = it & 1;
+        const uint32_t bpar = (it >> 1) & 1;
         const size_t ci = chunk0 + r;
         const float *cvec = a.chunk_vec + ci * 3 * kD;
-        const float f = cvec[tid], em = cvec[kD + tid], ddm = cvec[2 * kD + tid];
-        // ---- the states carried into chunk r: Diag(e^{Gc - Gmid}) dS_{r+1} (rescaling X in
-        // place: X holds e^{-Gmid_{r+1}} dS_{r+1}), DC_{r+1}, Dm_{r+1} and the gate carry
+        const float f = cvec[row], em = cvec[kD + row], ddm = cvec[2 * kD + row];
         if (it > 0) {
-            if (tid == 0) tma_store_wait_read();  // the previous chunk's images have been copied out
+            // the update of chunk r+1 and Sx_{r+1} have landed; the previous images are out
+            mbar_wait(&bar[BAR_MMA], (it - 1) & 1, abort_flag, status);
+            mbar_wait(&bar[BAR_SX], (it - 1) & 1, abort_flag, status);
+            if (tid == 0) tma_store_wait_read();
             __syncthreads();
+            tc_fence_after();
+            if (tid == 0 && !*abort_flag && r + 1 >= 2) issue(r - 1, buf ^ 1);  // chunk r+1's buffer is free
         }
-        tc_fence_after();
-        const float hs = f * emp[tid];
+        // X holds e^{-Gmid_{r+1}} dS_{r+1}: its gate carry rowsum(X * Sx_{r+1}) (chunk r's), then
+        // Diag(e^{Gc_r - Gmid_r}) dS_{r+1} = (f_r e^{Gmid_{r+1}}) X as the image and in place
+        const float hs = f * em_next;
+        float cs = 0.f;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int cc = 0; cc < 2; ++cc) {
+            const int c = 2 * half + cc;
             float x[32];
             tmem_ld32(tq + TM_X + 32 * c, x);
+            if (it > 0) {
+                const uint8_t *tile = sm + OFF_SX + half * 16384;
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    float sx[8];
+                    load_row_chunk(tile, row, 4 * cc + q4, sx);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) cs = fmaf(x[8 * q4 + e], sx[e], cs);
+                }
+            }
 #pragma unroll
             for (int e = 0; e < 32; ++e) x[e] *= hs;
-            uint8_t *tile = sm + OFF_IMG + (c >> 1) * 16384;
+            uint8_t *tile = sm + OFF_IMG + half * 16384;
 #pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * cc + q4, x + 8 * q4);
             tmem_st32(tq + TM_X + 32 * c, x);
         }
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int cc = 0; cc < 2; ++cc) {
+            const int c = 2 * half + cc;
             float x[32];
             tmem_ld32(tq + TM_DC + 32 * c, x);
-            uint8_t *tile = sm + OFF_IMG + 32768 + (c >> 1) * 16384;
+            uint8_t *tile = sm + OFF_IMG + 32768 + half * 16384;
 #pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, tid, 4 * (c & 1) + q4, x + 8 * q4);
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * cc + q4, x + 8 * q4);
         }
+        if (it > 0) carry[half * kD + row] = cs;
+        em_next = em;
         tmem_wait_st();
-        a.state_vec[ci * 2 * kD + tid] = Dm[tid];
-        a.state_vec[ci * 2 * kD + kD + tid] = carry[tid];
-        Dm[tid] += ddm;  // Dm_r
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
+        if (half == 0) {
+            a.state_vec[ci * 2 * kD + row] = Dm[row];
+            a.state_vec[ci * 2 * kD + kD + row] = carry[row] + carry[kD + row];
+            Dm[row] += ddm;  // Dm_r
+        }
+        if (tid == 0 && !*abort_flag && r >= 1) issue_sx(r);  // Sx_{r+1} has been read
         mbar_wait(&bar[BAR_IN0 + buf], bpar, abort_flag, status);
         if (tid == 0 && !*abort_flag) {
             bulk_store(a.state_img + ci * 65536, sm + OFF_IMG, 65536);
@@ -786,59 +812,33 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
                 mma_bf16(tbase + TM_DC, dDZm + k * 128, dQm + k * 128, ID_128x128_MM, 1);
             mma_commit(&bar[BAR_MMA]);
         }
-        mbar_wait(&bar[BAR_MMA], par, abort_flag, status);
-        mbar_wait(&bar[BAR_SX], par, abort_flag, status);
-        tc_fence_after();
-        {
-            // gate carry of chunk r - 1: rowsum(dS_r * S_r) = rowsum(X * Sx_r)
-            float cs = 0.f;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float x[32];
-                tmem_ld32(tq + TM_X + 32 * c, x);
-                const uint8_t *tile = sm + OFF_SX + (c >> 1) * 16384;
-#pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    float sx[8];
-                    load_row_chunk(tile, tid, 4 * (c & 1) + q4, sx);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) cs = fmaf(x[8 * q4 + e], sx[e], cs);
-                }
-            }
-            carry[tid] = cs;
-            emp[tid] = em;
-        }
-        tc_fence_before();
-        __syncthreads();
-        if (tid == 0 && !*abort_flag) {
-            if (r >= 2) issue(r - 2, buf);  // this buffer's MMAs are complete
-            if (r >= 1) issue_sx(r - 1);    // Sx_r has been read
-        }
     }
 
+    if (NC > 0) mbar_wait(&bar[BAR_MMA], (NC - 1) & 1, abort_flag, status);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     {
-        const size_t row = static_cast<size_t>(bh) * kD + tid;
-        const float e0 = emp[tid];  // e^{Gmid_0}: dS_0 = e^{Gmid_0} X
+        const size_t grow = static_cast<size_t>(bh) * kD + row;
+        const float e0 = em_next;  // e^{Gmid_0}: dS_0 = e^{Gmid_0} X
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int cc = 0; cc < 2; ++cc) {
+            const int c = 2 * half + cc;
             float x[32];
             tmem_ld32(tq + TM_X + 32 * c, x);
             if (a.dS0)
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
-                    reinterpret_cast<float4 *>(a.dS0 + row * kD + 32 * c)[e] =
+                    reinterpret_cast<float4 *>(a.dS0 + grow * kD + 32 * c)[e] =
                         make_float4(e0 * x[4 * e], e0 * x[4 * e + 1], e0 * x[4 * e + 2], e0 * x[4 * e + 3]);
             tmem_ld32(tq + TM_DC + 32 * c, x);
             if (a.dC0)
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
-                    reinterpret_cast<float4 *>(a.dC0 + row * kD + 32 * c)[e] =
+                    reinterpret_cast<float4 *>(a.dC0 + grow * kD + 32 * c)[e] =
                         make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
         }
-        if (a.dm0) a.dm0[row] = Dm[tid];
+        if (a.dm0 && half == 0) a.dm0[grow] = Dm[row];
     }
     if (tid == 0) tma_store_wait_all();
     tc_fence_before();
