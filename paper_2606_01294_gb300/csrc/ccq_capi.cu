@@ -356,7 +356,7 @@ ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v, const v
 // and the forward's scratch.
 static size_t gla_bwd_exchange_bytes(int B, int T, int H) {
     const size_t chunks = static_cast<size_t>(B) * H * ((T + 63) / 64);
-    return 4 * static_cast<size_t>(B) * T * H * 128 * 2 + chunks * (3 * 128 * 4 + 65536 + 2 * 128 * 4);
+    return 4 * static_cast<size_t>(B) * T * H * 128 * 2 + chunks * (3 * 128 * 4 + 65536 + 3 * 128 * 4);
 }
 
 static size_t gla_fwd_scratch_bytes(const ccq_params &p, int B, int T, int H) {

@@ -631,27 +631,31 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 }
 
 // =====================================================================================
-// gla_bwd_state_kernel: one CTA per (sequence, head), chunks last to first
+// gla_bwd_state_kernel: two CTAs per (sequence, head) (column halves), chunks last to first
 // =====================================================================================
 namespace st {
-constexpr uint32_t BUF_BYTES = 65536;  // per input buffer: QG, dO, DZ/|q|, raw q (16 KB each)
-constexpr uint32_t B_QG = 0, B_DO = 16384, B_DZ = 32768, B_Q = 49152;
-constexpr uint32_t OFF_SX = 2 * BUF_BYTES;      // 131072: Sx_r (checkpoint tile, for the gate carry)
-constexpr uint32_t OFF_IMG = OFF_SX + 32768;    // 163840: staging of the images written per chunk:
-                                                //   Diag(e^{Gc-Gmid}) dS_{r+1} (32 KB), DC_{r+1} (32 KB)
-constexpr uint32_t OFF_MISC = OFF_IMG + 65536;  // 229376
+// per input buffer: QG, DZ/|q| (16 KB each), this CTA's column half of dO and raw q (8 KB each)
+constexpr uint32_t BUF_BYTES = 49152;
+constexpr uint32_t B_QG = 0, B_DZ = 16384, B_DO = 32768, B_Q = 40960;
+constexpr uint32_t OFF_SX = 2 * BUF_BYTES;      // 98304: column half of Sx_r (checkpoint, for the gate carry)
+constexpr uint32_t OFF_IMG = OFF_SX + 16384;    // 114688: column halves of the images written per chunk:
+                                                //   Diag(e^{Gc-Gmid}) dS_{r+1} (16 KB), DC_{r+1} (16 KB)
+constexpr uint32_t OFF_MISC = OFF_IMG + 32768;  // 147456
 constexpr uint32_t M_DM = 0, M_CARRY = 512, M_BAR = 1536, M_TMEM = 1568, M_ABORT = 1572;
 constexpr uint32_t kMisc = 1600;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(kSmem <= 232448, "exceeds the 227 KB per-CTA limit");
 enum { BAR_IN0 = 0, BAR_IN1, BAR_SX, BAR_MMA, kBars };
-constexpr uint32_t TM_X = 0, TM_DC = 128;
+constexpr uint32_t TM_X = 0, TM_DC = 64;
+constexpr uint32_t ID_128x64_MM = make_idesc(128, 64, 1, 1);
 }  // namespace st
 
-// Two warps per TMEM lane quadrant: thread (row, half) holds state row `row`, columns
-// [64 half, 64 half + 64).  Per chunk r (last to first) the chain is: read X (the state
-// after chunk r+1's update), its gate carry against Sx_{r+1}, rescale to Diag(e^{Gc-Gmid})
-// dS_{r+1} (the image, and X in place), the DC image, then the two updates of chunk r.
+// Two CTAs per (sequence, head), one per column half ch of dS and DC (both updates split
+// by columns), two warps per TMEM lane quadrant: thread (row, th) holds state row `row`,
+// columns 64 ch + 32 th .. + 31.  Per chunk r (last to first) the chain is: read X (the
+// state after chunk r+1's update), its gate carry against Sx_{r+1} (a partial row sum over
+// this CTA's columns; the consumer adds the two), rescale to Diag(e^{Gc-Gmid}) dS_{r+1} (the
+// image, and X in place), the DC image, then the two updates of chunk r.
 __global__ void __launch_bounds__(kThreads, 1)
 gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_constant__ CUtensorMap map_do,
                      const __grid_constant__ CUtensorMap map_dzr, const __grid_constant__ CUtensorMap map_q,
@@ -662,14 +666,15 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
     const uint32_t sb = smem_addr(sm);
     uint8_t *misc = sm + OFF_MISC;
     float *Dm = reinterpret_cast<float *>(misc + M_DM);
-    float *carry = reinterpret_cast<float *>(misc + M_CARRY);  // [2 halves][128] partial row sums
+    float *carry = reinterpret_cast<float *>(misc + M_CARRY);  // [2 thread halves][128] partial row sums
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
 
     const int tid = threadIdx.x, warp = tid >> 5;
-    const int row = tid & (kD - 1), half = tid >> 7;
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    const int row = tid & (kD - 1), th = tid >> 7;
+    const int ch = blockIdx.x & 1, c = 2 * ch + th;  // column half of the state; 32-column unit
+    const int bh = blockIdx.x >> 1, b = bh / a.H, h = bh % a.H;
     const int T = a.T, NC = (T + kC - 1) / kC;
     const uint8_t *ck = a.ckpt + static_cast<size_t>(bh) * ckpt_head_bytes(T);
     const size_t chunk0 = static_cast<size_t>(bh) * NC;  // flat index of this sequence's chunk 0
@@ -680,7 +685,7 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
         *abort_flag = 0;
         fence_barrier_init();
     }
-    if (warp == 0) tmem_alloc(tmem_slot, 256);
+    if (warp == 0) tmem_alloc(tmem_slot, 128);
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = *tmem_slot;
@@ -692,9 +697,7 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
         const float *dct_row = a.dCT ? a.dCT + grow * kD : nullptr;
         const float *st_row = reinterpret_cast<const float *>(ck + static_cast<size_t>(NC) * kCkptChunkBytes) + row * kD;
         float cs = 0.f;
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-            const int c = 2 * half + cc;
+        {
             float x[32], y[32];
 #pragma unroll
             for (int e = 0; e < 32; ++e) {
@@ -702,30 +705,28 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
                 if (dst_row) cs = fmaf(x[e], st_row[32 * c + e], cs);
                 y[e] = dct_row ? dct_row[32 * c + e] : 0.f;
             }
-            tmem_st32(tq + TM_X + 32 * c, x);
-            tmem_st32(tq + TM_DC + 32 * c, y);
+            tmem_st32(tq + TM_X + 32 * th, x);
+            tmem_st32(tq + TM_DC + 32 * th, y);
         }
         tmem_wait_st();
-        carry[half * kD + row] = cs;
-        if (half == 0) Dm[row] = a.dmT ? a.dmT[grow] : 0.f;
+        carry[th * kD + row] = cs;
+        if (th == 0) Dm[row] = a.dmT ? a.dmT[grow] : 0.f;
     }
     auto issue = [&](int r, int buf) {
         const int tg = r * kC;
         uint8_t *base = sm + buf * BUF_BYTES;
         uint64_t *bb = &bar[BAR_IN0 + buf];
-        mbar_arrive_expect_tx(bb, 4 * 16384);
+        mbar_arrive_expect_tx(bb, BUF_BYTES);
         tma_load_4d(base + B_QG, &map_qg, bb, 0, h, tg, b);
         tma_load_4d(base + B_QG + 8192, &map_qg, bb, 64, h, tg, b);
-        tma_load_4d(base + B_DO, &map_do, bb, 0, h, tg, b);
-        tma_load_4d(base + B_DO + 8192, &map_do, bb, 64, h, tg, b);
         tma_load_4d(base + B_DZ, &map_dzr, bb, 0, h, tg, b);
         tma_load_4d(base + B_DZ + 8192, &map_dzr, bb, 64, h, tg, b);
-        tma_load_4d(base + B_Q, &map_q, bb, 0, h, tg, b);
-        tma_load_4d(base + B_Q + 8192, &map_q, bb, 64, h, tg, b);
+        tma_load_4d(base + B_DO, &map_do, bb, 64 * ch, h, tg, b);
+        tma_load_4d(base + B_Q, &map_q, bb, 64 * ch, h, tg, b);
     };
     auto issue_sx = [&](int r) {
-        mbar_arrive_expect_tx(&bar[BAR_SX], 32768);
-        bulk_load(sm + OFF_SX, ck + static_cast<size_t>(r) * kCkptChunkBytes + 32768, 32768, &bar[BAR_SX]);
+        mbar_arrive_expect_tx(&bar[BAR_SX], 16384);
+        bulk_load(sm + OFF_SX, ck + static_cast<size_t>(r) * kCkptChunkBytes + 32768 + 16384 * ch, 16384, &bar[BAR_SX]);
     };
     if (tid == 0 && NC > 0) {
         issue(NC - 1, 0);
@@ -755,61 +756,53 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
         // Diag(e^{Gc_r - Gmid_r}) dS_{r+1} = (f_r e^{Gmid_{r+1}}) X as the image and in place
         const float hs = f * em_next;
         float cs = 0.f;
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-            const int c = 2 * half + cc;
+        {
             float x[32];
-            tmem_ld32(tq + TM_X + 32 * c, x);
+            tmem_ld32(tq + TM_X + 32 * th, x);
             if (it > 0) {
-                const uint8_t *tile = sm + OFF_SX + half * 16384;
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     float sx[8];
-                    load_row_chunk(tile, row, 4 * cc + q4, sx);
+                    load_row_chunk(sm + OFF_SX, row, 4 * th + q4, sx);
 #pragma unroll
                     for (int e = 0; e < 8; ++e) cs = fmaf(x[8 * q4 + e], sx[e], cs);
                 }
             }
 #pragma unroll
             for (int e = 0; e < 32; ++e) x[e] *= hs;
-            uint8_t *tile = sm + OFF_IMG + half * 16384;
 #pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * cc + q4, x + 8 * q4);
-            tmem_st32(tq + TM_X + 32 * c, x);
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_IMG, row, 4 * th + q4, x + 8 * q4);
+            tmem_st32(tq + TM_X + 32 * th, x);
+            float y[32];
+            tmem_ld32(tq + TM_DC + 32 * th, y);
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_IMG + 16384, row, 4 * th + q4, y + 8 * q4);
         }
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-            const int c = 2 * half + cc;
-            float x[32];
-            tmem_ld32(tq + TM_DC + 32 * c, x);
-            uint8_t *tile = sm + OFF_IMG + 32768 + half * 16384;
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * cc + q4, x + 8 * q4);
-        }
-        if (it > 0) carry[half * kD + row] = cs;
+        if (it > 0) carry[th * kD + row] = cs;
         em_next = em;
         tmem_wait_st();
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
-        if (half == 0) {
-            a.state_vec[ci * 2 * kD + row] = Dm[row];
-            a.state_vec[ci * 2 * kD + kD + row] = carry[row] + carry[kD + row];
+        if (th == 0) {
+            if (ch == 0) a.state_vec[ci * 3 * kD + row] = Dm[row];
+            a.state_vec[ci * 3 * kD + (1 + ch) * kD + row] = carry[row] + carry[kD + row];
             Dm[row] += ddm;  // Dm_r
         }
         if (tid == 0 && !*abort_flag && r >= 1) issue_sx(r);  // Sx_{r+1} has been read
         mbar_wait(&bar[BAR_IN0 + buf], bpar, abort_flag, status);
         if (tid == 0 && !*abort_flag) {
-            bulk_store(a.state_img + ci * 65536, sm + OFF_IMG, 65536);
+            bulk_store(a.state_img + ci * 65536 + 16384 * ch, sm + OFF_IMG, 16384);
+            bulk_store(a.state_img + ci * 65536 + 32768 + 16384 * ch, sm + OFF_IMG + 16384, 16384);
             tma_store_commit();
             tc_fence_after();
             const uint32_t base = sb + buf * BUF_BYTES;
             const uint64_t dQGm = make_desc(base + B_QG, 8192, 1024), dDOm = make_desc(base + B_DO, 8192, 1024);
             const uint64_t dDZm = make_desc(base + B_DZ, 8192, 1024), dQm = make_desc(base + B_Q, 8192, 1024);
-            for (int k = 0; k < 4; ++k)  // X += QG^T dO  (-> e^{-Gmid_r} dS_r)
-                mma_bf16(tbase + TM_X, dQGm + k * 128, dDOm + k * 128, ID_128x128_MM, 1);
-            for (int k = 0; k < 4; ++k)  // DC += (DZ / |q|)^T q  (= DZ^T Qbar)
-                mma_bf16(tbase + TM_DC, dDZm + k * 128, dQm + k * 128, ID_128x128_MM, 1);
+            for (int k = 0; k < 4; ++k)  // X += QG^T dO  (-> e^{-Gmid_r} dS_r), this CTA's columns
+                mma_bf16(tbase + TM_X, dQGm + k * 128, dDOm + k * 128, ID_128x64_MM, 1);
+            for (int k = 0; k < 4; ++k)  // DC += (DZ / |q|)^T q  (= DZ^T Qbar), this CTA's columns
+                mma_bf16(tbase + TM_DC, dDZm + k * 128, dQm + k * 128, ID_128x64_MM, 1);
             mma_commit(&bar[BAR_MMA]);
         }
     }
@@ -821,31 +814,29 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
     {
         const size_t grow = static_cast<size_t>(bh) * kD + row;
         const float e0 = em_next;  // e^{Gmid_0}: dS_0 = e^{Gmid_0} X
-#pragma unroll
-        for (int cc = 0; cc < 2; ++cc) {
-            const int c = 2 * half + cc;
+        {
             float x[32];
-            tmem_ld32(tq + TM_X + 32 * c, x);
+            tmem_ld32(tq + TM_X + 32 * th, x);
             if (a.dS0)
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
                     reinterpret_cast<float4 *>(a.dS0 + grow * kD + 32 * c)[e] =
                         make_float4(e0 * x[4 * e], e0 * x[4 * e + 1], e0 * x[4 * e + 2], e0 * x[4 * e + 3]);
-            tmem_ld32(tq + TM_DC + 32 * c, x);
+            tmem_ld32(tq + TM_DC + 32 * th, x);
             if (a.dC0)
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
                     reinterpret_cast<float4 *>(a.dC0 + grow * kD + 32 * c)[e] =
                         make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
         }
-        if (a.dm0 && half == 0) a.dm0[grow] = Dm[row];
+        if (a.dm0 && ch == 0 && th == 0) a.dm0[grow] = Dm[row];
     }
     if (tid == 0) tma_store_wait_all();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) {
         tc_fence_after();
-        tmem_dealloc(tbase, 256);
+        tmem_dealloc(tbase, 128);
     }
 }
 
@@ -868,9 +859,9 @@ constexpr uint32_t OFF_SA = 204800;  // SA
 constexpr uint32_t OFF_DG = 131072;  // fp32 dG [64][kDgStride], over the two images once they are dead
 constexpr int kDgStride = 129;
 constexpr uint32_t OFF_MISC = 212992;
-constexpr uint32_t M_VEC = 0,        // [2][128] Dm_{r+1}, gate carry (from the state pass)
-                   M_RK = 1024, M_GQ4 = 1280, M_RED = 3328, M_BAR = 4352, M_TMEM = 4384, M_ABORT = 4388;
-constexpr uint32_t kMisc = 4480;
+constexpr uint32_t M_VEC = 0,        // [3][128] Dm_{r+1}, the gate carry's two column-half sums (state pass)
+                   M_RK = 1536, M_GQ4 = 1792, M_RED = 3840, M_BAR = 4864, M_TMEM = 4896, M_ABORT = 4900;
+constexpr uint32_t kMisc = 4992;
 constexpr uint32_t kSmem = OFF_MISC + kMisc + 1024;
 static_assert(OFF_DG + 64 * kDgStride * 4 <= OFF_P1, "dG scratch reaches P1");
 static_assert(OFF_DC == OFF_DS + 32768, "a state image record lands as one block");
@@ -917,7 +908,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         fence_barrier_init();
         uint64_t *ba = &bar[BAR_IN], *bb = &bar[BAR_INB];
         mbar_arrive_expect_tx(ba, 16384 + g_bytes);
-        mbar_arrive_expect_tx(bb, 5 * 16384 + 65536 + 1024);
+        mbar_arrive_expect_tx(bb, 5 * 16384 + 65536 + 1536);
         tma_load_4d(sm + OFF_K, &map_k, ba, 0, h, c0, b);
         tma_load_4d(sm + OFF_K + 8192, &map_k, ba, 64, h, c0, b);
         tma_load_4d(sm + OFF_KD, &map_g, ba, 0, h, c0, b);
@@ -938,7 +929,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
             tma_load_4d(sm + OFF_GQ, &map_gq, bb, 0, h, c0, b);
             tma_load_4d(sm + OFF_GQ + 8192, &map_gq, bb, 64, h, c0, b);
             bulk_load(sm + OFF_DS, a.state_img + static_cast<size_t>(blockIdx.x) * 65536, 65536, bb);
-            bulk_load(misc + M_VEC, a.state_vec + static_cast<size_t>(blockIdx.x) * 2 * kD, 1024, bb);
+            bulk_load(misc + M_VEC, a.state_vec + static_cast<size_t>(blockIdx.x) * 3 * kD, 1536, bb);
             // the chunk one wave later finds its inputs in L2
             const int nx = blockIdx.x + a.wave;
             if (a.wave > 0 && nx < static_cast<int>(gridDim.x)) {
@@ -951,7 +942,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
                 }
                 tma_prefetch_l2_4d(&map_g, 0, h2, c2, b2);
                 bulk_prefetch_l2(a.state_img + static_cast<size_t>(nx) * 65536, 65536);
-                bulk_prefetch_l2(a.state_vec + static_cast<size_t>(nx) * 2 * kD, 1024);
+                bulk_prefetch_l2(a.state_vec + static_cast<size_t>(nx) * 3 * kD, 1536);
             }
         }
         return;
@@ -1107,7 +1098,7 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         }
         red[hh * 128 + d] = tot;
         compute_sync();
-        float acc = vec[kD + d] + (hh == 0 ? red[128 + d] : 0.f);
+        float acc = vec[kD + d] + vec[2 * kD + d] + (hh == 0 ? red[128 + d] : 0.f);
         const int nvalid = min(kC, T - c0);
 #pragma unroll
         for (int u = 31; u >= 0; --u) {
@@ -1151,7 +1142,7 @@ cudaError_t launch_gla_bwd(const BwdArgs &a, const BwdMaps &m, cudaStream_t s) {
                                                           m.dzr, a);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    gla_bwd_state_kernel<<<a.B * a.H, kThreads, st::kSmem, s>>>(m.qg, m.dO, m.dzr, m.q, a);
+    gla_bwd_state_kernel<<<a.B * a.H * 2, kThreads, st::kSmem, s>>>(m.qg, m.dO, m.dzr, m.q, a);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     gla_bwd_kv_kernel<<<chunks, kThreadsLoad, kv::kSmem, s>>>(m.k, m.v, m.dO, m.g, m.qg, m.dkc, m.gq, m.dk, m.dv, a);

@@ -134,7 +134,8 @@ struct BwdArgs {
     float *chunk_vec;    // [3][128] written by the q kernel: e^{Gc-Gmid}, e^{Gmid}, Dm increment
     uint8_t *state_img;  // 64 KB written by the state pass: the bf16 tile images of
                          // Diag(e^{Gc-Gmid}) dS_{r+1} and DC_{r+1} (two T64 tiles each)
-    float *state_vec;    // [2][128] written by the state pass: Dm_{r+1}, rowsum(dS_{r+1} S_{r+1})
+    float *state_vec;    // [3][128] written by the state pass: Dm_{r+1}, rowsum(dS_{r+1} S_{r+1}) as
+                         // the sums over the two column halves
     int wave = 0;        // chunk CTAs resident at once (one per SM): each prefetches into L2 the
                          // inputs of the chunk one wave after its own
 };

@@ -129,7 +129,7 @@ def test_gla_ckpt_and_bwd_workspace_sizes(lib):
     assert n.value == 2 * (65536 + 512) + 65536  # ragged tail: two chunks
     assert lib.ccq_gla_ckpt_size(1, 64, 1, 64, 64, ctypes.byref(n)) == ccq.CCQ_ERR_UNSUPPORTED
     p = ctypes.byref(ccq.params(seq_split=1))
-    x = 4 * 4 * 4096 * 16 * 128 * 2 + 4 * 16 * 64 * (3 * 512 + 65536 + 2 * 512)  # exchange + per chunk
+    x = 4 * 4 * 4096 * 16 * 128 * 2 + 4 * 16 * 64 * (3 * 512 + 65536 + 3 * 512)  # exchange + per chunk
     assert lib.ccq_gla_bwd_workspace_size(4, 4096, 16, 128, 128, 0, 1, p, ctypes.byref(n)) == 0
     assert n.value == x
     assert lib.ccq_gla_bwd_workspace_size(4, 4096, 16, 128, 128, 0, 0, p, ctypes.byref(n)) == 0
