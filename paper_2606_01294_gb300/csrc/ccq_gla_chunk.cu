@@ -557,29 +557,23 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     slot_f(s, MS_RK)[j] = a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
                 }
             }
-            // gate cumsum over this thread's 32 tokens for dims d0, d0+1
-            float g0[32], g1[32];
+            // gate cumsum over this thread's 32 tokens for dims d0, d0+1, as fp32 pairs
+            uint64_t g2[32];
             {
-                float r0 = 0.f, r1 = 0.f;
+                uint64_t r2 = 0;  // (0.f, 0.f)
 #pragma unroll
                 for (int jj = 0; jj < 32; ++jj) {
                     const int j = 32 * th + jj;
-                    float x0, x1;
-                    if (gate_f32) {
-                        const float2 f2 = *reinterpret_cast<const float2 *>(slot + SO_KG + (j * kD + d0) * 4);
-                        x0 = f2.x; x1 = f2.y;
-                    } else {
-                        const __nv_bfloat162 b2 =
-                            *reinterpret_cast<const __nv_bfloat162 *>(slot + SO_KG + (j * kD + d0) * 2);
-                        const float2 f2 = __bfloat1622float2(b2);
-                        x0 = f2.x; x1 = f2.y;
-                    }
-                    r0 += x0; r1 += x1;
-                    g0[jj] = r0; g1[jj] = r1;
+                    const uint64_t x2 =
+                        gate_f32 ? *reinterpret_cast<const uint64_t *>(slot + SO_KG + (j * kD + d0) * 4)
+                                 : f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(slot + SO_KG + (j * kD + d0) * 2));
+                    r2 = f2_add(r2, x2);
+                    g2[jj] = r2;
                 }
                 if (th == 0) {
-                    gt0[d0] = r0;
-                    gt0[d0 + 1] = r1;
+                    const float2 rv = f2_split(r2);
+                    gt0[d0] = rv.x;
+                    gt0[d0 + 1] = rv.y;
                 }
             }
             named_bar(NB_PREP, 128);  // raw gates all read, norms and gt0 visible
@@ -587,46 +581,48 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 constexpr float kLog2e = 1.4426950408889634f;
                 const float gm0 = gt0[d0], gm1 = gt0[d0 + 1];   // Gmid
                 // exponents in log2 units relative to Gmid: x = (G - Gmid) log2(e)
-                const float o0 = ((th ? gm0 : 0.f) - gm0) * kLog2e, o1 = ((th ? gm1 : 0.f) - gm1) * kLog2e;
+                const uint64_t o2 = f2_make(((th ? gm0 : 0.f) - gm0) * kLog2e, ((th ? gm1 : 0.f) - gm1) * kLog2e);
+                const uint64_t l2e = f2_make(kLog2e, kLog2e);
                 if (th == 1) {
                     // f = e^{Gtot - Gmid} (gate sum of tokens 32..63), e^{Gmid}
-                    slot_f(s, MS_F)[d0] = fast_exp2(g0[31] * kLog2e);
-                    slot_f(s, MS_F)[d0 + 1] = fast_exp2(g1[31] * kLog2e);
+                    const float2 gt = f2_split(g2[31]);
+                    slot_f(s, MS_F)[d0] = fast_exp2(gt.x * kLog2e);
+                    slot_f(s, MS_F)[d0 + 1] = fast_exp2(gt.y * kLog2e);
                     slot_f(s, MS_EGM)[d0] = fast_exp2(gm0 * kLog2e);
                     slot_f(s, MS_EGM)[d0 + 1] = fast_exp2(gm1 * kLog2e);
                 }
                 const float *rk = slot_f(s, MS_RK);
                 const uint32_t tcol = (d0 >> 6) * 8192;
-                float dm0 = 0.f, dm1 = 0.f;
+                uint64_t dm2 = 0;
                 // four batches of eight tokens: every load of a batch is issued before its
                 // stores (the in-place kbar store may alias a later load)
 #pragma unroll
                 for (int bt = 0; bt < 4; ++bt) {
                     uint32_t kraw[8];
-                    float rkv[8];
 #pragma unroll
                     for (int u = 0; u < 8; ++u) {
                         const int j = 32 * th + 8 * bt + u;
                         kraw[u] = *reinterpret_cast<const uint32_t *>(slot + SO_K + tcol + t64_offset(j, d0 & 63));
-                        rkv[u] = rk[j];
                     }
+                    const float4 rka = *reinterpret_cast<const float4 *>(rk + 32 * th + 8 * bt);
+                    const float4 rkb = *reinterpret_cast<const float4 *>(rk + 32 * th + 8 * bt + 4);
+                    const float rkv[8] = {rka.x, rka.y, rka.z, rka.w, rkb.x, rkb.y, rkb.z, rkb.w};
 #pragma unroll
                     for (int u = 0; u < 8; ++u) {
                         const int jj = 8 * bt + u, j = 32 * th + jj;
                         const uint32_t off = tcol + t64_offset(j, d0 & 63);
-                        const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&kraw[u]));
-                        const float k0 = kr.x * rkv[u], k1 = kr.y * rkv[u];
-                        const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
-                        *reinterpret_cast<uint32_t *>(slot + SO_K + off) = pack_bf16(k0, k1);
+                        const uint64_t k2 = f2_mul(f2_from_bf16x2(kraw[u]), f2_make(rkv[u], rkv[u]));
+                        const float2 x = f2_split(f2_fma(g2[jj], l2e, o2));
+                        *reinterpret_cast<uint32_t *>(slot + SO_K + off) = bf16x2_from_f2(k2);
                         *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
-                            pack_bf16(k0 * fast_exp2(-x0), k1 * fast_exp2(-x1));
-                        *reinterpret_cast<uint32_t *>(slot + SO_EG + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
-                        dm0 += k0;
-                        dm1 += k1;
+                            bf16x2_from_f2(f2_mul(k2, f2_make(fast_exp2(-x.x), fast_exp2(-x.y))));
+                        *reinterpret_cast<uint32_t *>(slot + SO_EG + off) = pack_bf16(fast_exp2(x.x), fast_exp2(x.y));
+                        dm2 = f2_add(dm2, k2);
                     }
                 }
-                dmp[th * kD + d0] = dm0;
-                dmp[th * kD + d0 + 1] = dm1;
+                const float2 dmv = f2_split(dm2);
+                dmp[th * kD + d0] = dmv.x;
+                dmp[th * kD + d0 + 1] = dmv.y;
             }
             fence_proxy_async_smem();
             named_bar(NB_PREP, 128);
