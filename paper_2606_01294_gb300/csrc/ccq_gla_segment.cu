@@ -263,16 +263,37 @@ gla_segment_combine_kernel(const ChunkArgs a) {
         else if (e < 2 * kSS + kD) x = a.m0 ? a.m0[sq * kD + e - 2 * kSS] : 0.f;
         cur[u] = x;
     }
-    for (int s = 0; s < a.nseg; ++s) {
-        float *slot = a.seg_ws + (sq * a.nseg + s) * kSegFloats;
-        const float *D = slot + 2 * kSS + kD;
+    // segments in groups of kGroup: every load of a group is issued before its scan steps
+    // (the loads do not depend on the scan), so the group costs one memory round trip
+    constexpr int kGroup = 8;
+    for (int s0 = 0; s0 < a.nseg; s0 += kGroup) {
+        const int ns = min(kGroup, a.nseg - s0);
+        float dv[kGroup][4], Dv[kGroup][4];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int e = el[u];
-            if (e >= 2 * kSS + kD) continue;
-            const float d = slot[e];
-            slot[e] = cur[u];
-            cur[u] = (e < kSS ? D[e >> 7] * cur[u] : cur[u]) + d;
+        for (int g = 0; g < kGroup; ++g) {
+            if (g < ns) {
+                const float *slot = a.seg_ws + (sq * a.nseg + s0 + g) * kSegFloats;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int e = el[u];
+                    const bool live = e < 2 * kSS + kD;
+                    dv[g][u] = live ? slot[e] : 0.f;
+                    Dv[g][u] = (e < kSS) ? slot[2 * kSS + kD + (e >> 7)] : 1.f;
+                }
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < kGroup; ++g) {
+            if (g < ns) {
+                float *slot = a.seg_ws + (sq * a.nseg + s0 + g) * kSegFloats;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int e = el[u];
+                    if (e >= 2 * kSS + kD) continue;
+                    slot[e] = cur[u];
+                    cur[u] = Dv[g][u] * cur[u] + dv[g][u];
+                }
+            }
         }
     }
 }
