@@ -56,6 +56,19 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Non-blocking test of the phase with the given parity.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Wait for the phase with the given parity to complete, giving up after
 // kWaitLimitCycles.  On give-up (or when *abort is already set) returns false,
 // sets *abort and records kStatusTimeout in *status.  Callers keep executing
@@ -64,7 +77,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volati
                                           int *status) {
     if (*abort) return false;
     const uint32_t a = smem_addr(bar);
-    if (mbar_try_wait(a, parity)) return true;
+    if (mbar_test_wait(a, parity)) return true;  // already complete: no suspend
     const long long start = clock64();
     while (!mbar_try_wait(a, parity)) {
         if (*abort) return false;
