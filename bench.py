@@ -131,10 +131,16 @@ KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kerne
                 "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu"}
 
 
+SHARED_DEVICE_SOURCES = ("sm100_ptx.cuh", "ccq_internal.h")  # inlined into every kernel
+
+
 def source_sha(fname):
-    p = os.path.join(ROOT, "paper_2606_01294_gb300", "csrc", fname)
-    with open(p, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    """Hash of a kernel's source file and the device headers every kernel inlines."""
+    h = hashlib.sha256()
+    for f in (fname,) + SHARED_DEVICE_SOURCES:
+        with open(os.path.join(ROOT, "paper_2606_01294_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
 
 
 def kernel_sha(kind):
