@@ -454,37 +454,51 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const uint8_t *egt = sm + OFF_EG + hf * 8192;
         float dl = 0.f, mdz = 0.f;
         {
+            // fp32 pairs over consecutive columns
             const int h2 = grp;
             float zi[32], dqa[32];
             tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, zi);
             tmem_ld16x2_32<64>(tq + TM_DQ + 32 * h2, dqa);
+            const uint64_t nc1 = f2_make(-c1, -c1), itau2 = f2_make(itau, itau), nlam2 = f2_make(-lam, -lam);
+            const uint64_t sc2 = f2_make(a.scale, a.scale), nl2 = f2_make(nl, nl), rq2 = f2_make(rq, rq);
+            uint64_t dl2 = 0, mdz2 = 0;  // sum of z dqc (negated at the end), sum of m d
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) {
                 const int cc = 4 * h2 + q4;
-                float qb[8], eg[8], qg[8], dz[8], dzr[8], dqv[8], gq[8];
-                load_row_chunk(qbt, i, cc, qb);
-                load_row_chunk(egt, i, cc, eg);
+                const uint4 qraw = *reinterpret_cast<const uint4 *>(qbt + t64_chunk(i, cc));
+                const uint4 eraw = *reinterpret_cast<const uint4 *>(egt + t64_chunk(i, cc));
+                const ulonglong2 mlo = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc);
+                const ulonglong2 mhi = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc + 4);
+                const uint32_t qw[4] = {qraw.x, qraw.y, qraw.z, qraw.w};
+                const uint32_t ew[4] = {eraw.x, eraw.y, eraw.z, eraw.w};
+                const uint64_t mp[4] = {mlo.x, mlo.y, mhi.x, mhi.y};
+                uint32_t qg[4], dz[4], dzr[4], dqv[4], gq[4];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float m = Mh[8 * cc + e];
-                    const float z = (zi[8 * q4 + e] - c1 * m) * itau;
-                    const float qc = qb[e] - lam * z;
-                    const float dqc = a.scale * eg[e] * dqa[8 * q4 + e];
-                    const float d = nl * dqc;
-                    dl = fmaf(-z, dqc, dl);
-                    mdz = fmaf(m, d, mdz);
-                    qg[e] = a.scale * qc * eg[e];
-                    dz[e] = d;
-                    dzr[e] = d * rq;
-                    dqv[e] = dqc;
-                    gq[e] = qc * dqc;
+                for (int w = 0; w < 4; ++w) {
+                    const int e = 8 * q4 + 2 * w;
+                    const uint64_t eg2 = f2_from_bf16x2(ew[w]);
+                    const uint64_t z2 = f2_mul(f2_fma(nc1, mp[w], f2_make(zi[e], zi[e + 1])), itau2);
+                    const uint64_t qc2 = f2_fma(nlam2, z2, f2_from_bf16x2(qw[w]));
+                    const uint64_t dqc2 = f2_mul(f2_mul(sc2, eg2), f2_make(dqa[e], dqa[e + 1]));
+                    const uint64_t d2 = f2_mul(nl2, dqc2);
+                    dl2 = f2_fma(z2, dqc2, dl2);
+                    mdz2 = f2_fma(mp[w], d2, mdz2);
+                    qg[w] = bf16x2_from_f2(f2_mul(f2_mul(sc2, qc2), eg2));
+                    dz[w] = bf16x2_from_f2(d2);
+                    dzr[w] = bf16x2_from_f2(f2_mul(d2, rq2));
+                    dqv[w] = bf16x2_from_f2(dqc2);
+                    gq[w] = bf16x2_from_f2(f2_mul(qc2, dqc2));
                 }
-                store_row_chunk(sm + OFF_V + hf * 8192, i, cc, qg);
-                store_row_chunk(sm + OFF_DO + hf * 8192, i, cc, dz);
-                store_row_chunk(sm + OFF_KD + hf * 8192, i, cc, dzr);
-                store_row_chunk(sm + OFF_SX + hf * 8192, i, cc, dqv);
-                store_row_chunk(sm + OFF_SX + 16384 + hf * 8192, i, cc, gq);
+                const uint32_t off = t64_chunk(i, cc);
+                *reinterpret_cast<uint4 *>(sm + OFF_V + hf * 8192 + off) = make_uint4(qg[0], qg[1], qg[2], qg[3]);
+                *reinterpret_cast<uint4 *>(sm + OFF_DO + hf * 8192 + off) = make_uint4(dz[0], dz[1], dz[2], dz[3]);
+                *reinterpret_cast<uint4 *>(sm + OFF_KD + hf * 8192 + off) = make_uint4(dzr[0], dzr[1], dzr[2], dzr[3]);
+                *reinterpret_cast<uint4 *>(sm + OFF_SX + hf * 8192 + off) = make_uint4(dqv[0], dqv[1], dqv[2], dqv[3]);
+                *reinterpret_cast<uint4 *>(sm + OFF_SX + 16384 + hf * 8192 + off) = make_uint4(gq[0], gq[1], gq[2], gq[3]);
             }
+            const float2 dlv = f2_split(dl2), mdv = f2_split(mdz2);
+            dl = -(dlv.x + dlv.y);
+            mdz = mdv.x + mdv.y;
         }
         dl += __shfl_xor_sync(0xffffffffu, dl, 16);
         mdz += __shfl_xor_sync(0xffffffffu, mdz, 16);
