@@ -583,24 +583,33 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         uint8_t *qbt = sm + OFF_Q + hf * 8192;
         const uint8_t *dqt = sm + OFF_SX + hf * 8192;
         const int h2 = grp;
-        float dqb[32];
-        float dot = 0.f;
+        uint64_t dqb[16];  // fp32 pairs over consecutive columns
+        float dot;
         {
             float u[32];
             tmem_ld16x2_32<64>(tq + TM_Z + 32 * h2, u);
+            const uint64_t ncz = f2_make(-cz, -cz);
+            uint64_t dot2 = 0;
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) {
                 const int cc = 4 * h2 + q4;
-                float dqc[8], qb[8];
-                load_row_chunk(dqt, i, cc, dqc);
-                load_row_chunk(qbt, i, cc, qb);
+                const uint4 draw = *reinterpret_cast<const uint4 *>(dqt + t64_chunk(i, cc));
+                const uint4 qraw = *reinterpret_cast<const uint4 *>(qbt + t64_chunk(i, cc));
+                const ulonglong2 mlo = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc);
+                const ulonglong2 mhi = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc + 4);
+                const uint32_t dw[4] = {draw.x, draw.y, draw.z, draw.w};
+                const uint32_t qw[4] = {qraw.x, qraw.y, qraw.z, qraw.w};
+                const uint64_t mp[4] = {mlo.x, mlo.y, mhi.x, mhi.y};
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float v = dqc[e] + u[8 * q4 + e] - cz * Mh[8 * cc + e];
-                    dqb[8 * q4 + e] = v;
-                    dot = fmaf(qb[e], v, dot);
+                for (int w = 0; w < 4; ++w) {
+                    const int e = 8 * q4 + 2 * w;
+                    const uint64_t v = f2_fma(ncz, mp[w], f2_add(f2_from_bf16x2(dw[w]), f2_make(u[e], u[e + 1])));
+                    dqb[4 * q4 + w] = v;
+                    dot2 = f2_fma(f2_from_bf16x2(qw[w]), v, dot2);
                 }
             }
+            const float2 dv = f2_split(dot2);
+            dot = dv.x + dv.y;
         }
         dot += __shfl_xor_sync(0xffffffffu, dot, 16);
         if (hf == 0) red[grp * 128 + i] = dot;
@@ -614,15 +623,19 @@ gla_bwd_q_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         }
         compute_sync();
         dot = red[i] + red[128 + i];
+        const uint64_t ndot = f2_make(-dot, -dot), rq2 = f2_make(rq, rq);
 #pragma unroll
         for (int q4 = 0; q4 < 4; ++q4) {
             const int cc = 4 * h2 + q4;
-            float qb[8], out[8];
-            load_row_chunk(qbt, i, cc, qb);
+            const uint4 qraw = *reinterpret_cast<const uint4 *>(qbt + t64_chunk(i, cc));
+            const uint32_t qw[4] = {qraw.x, qraw.y, qraw.z, qraw.w};
+            uint32_t ow[4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e)
-                out[e] = a.l2norm ? rq * fmaf(-qb[e], dot, dqb[8 * q4 + e]) : dqb[8 * q4 + e];
-            store_row_chunk(qbt, i, cc, out);
+            for (int w = 0; w < 4; ++w) {
+                const uint64_t v = dqb[4 * q4 + w];
+                ow[w] = bf16x2_from_f2(a.l2norm ? f2_mul(rq2, f2_fma(ndot, f2_from_bf16x2(qw[w]), v)) : v);
+            }
+            *reinterpret_cast<uint4 *>(qbt + t64_chunk(i, cc)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
         }
     }
     fence_proxy_async_smem();
@@ -1044,29 +1057,42 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         const uint8_t *gqt = sm + OFF_GQ + hf * 8192;
         float *dgrow = dG + i * kDgStride + 64 * hf;
         const int h2 = grp;  // this group's 32-column slice of each 128-column product
-        float dkb[32];
-        float dot = 0.f;
+        uint64_t dkb[16];    // fp32 pairs over consecutive columns
+        float dot;
         {
             float x[32], y[32];
             tmem_ld16x2_32<64>(tq + TM_DK + 32 * h2, x);
             tmem_ld16x2_32<64>(tq + TM_KC + 32 * h2, y);
+            uint64_t dot2 = 0;
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) {
                 const int cc = 4 * h2 + q4;
-                float eg[8], kb[8], kc[8], gq[8];
-                load_row_chunk(egt, i, cc, eg);
-                load_row_chunk(kt, i, cc, kb);
-                load_row_chunk(dkct, i, cc, kc);
-                load_row_chunk(gqt, i, cc, gq);
+                const uint32_t off = t64_chunk(i, cc);
+                const uint4 er = *reinterpret_cast<const uint4 *>(egt + off);
+                const uint4 kr = *reinterpret_cast<const uint4 *>(kt + off);
+                const uint4 cr = *reinterpret_cast<const uint4 *>(dkct + off);
+                const uint4 gr = *reinterpret_cast<const uint4 *>(gqt + off);
+                const ulonglong2 dlo = *reinterpret_cast<const ulonglong2 *>(Dh + 8 * cc);
+                const ulonglong2 dhi = *reinterpret_cast<const ulonglong2 *>(Dh + 8 * cc + 4);
+                const uint32_t ew[4] = {er.x, er.y, er.z, er.w}, kw[4] = {kr.x, kr.y, kr.z, kr.w};
+                const uint32_t cw[4] = {cr.x, cr.y, cr.z, cr.w}, gw[4] = {gr.x, gr.y, gr.z, gr.w};
+                const uint64_t dm[4] = {dlo.x, dlo.y, dhi.x, dhi.y};
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float dkw = x[8 * q4 + e] * __frcp_rn(eg[e]);
-                    const float v = dkw + kc[e] + y[8 * q4 + e] + Dh[8 * cc + e];
-                    dkb[8 * q4 + e] = v;
-                    dot = fmaf(kb[e], v, dot);
-                    dgrow[8 * cc + e] = fmaf(-kb[e], dkw, gq[e]);
+                for (int w = 0; w < 4; ++w) {
+                    const int e = 8 * q4 + 2 * w;
+                    const float2 eg = f2_split(f2_from_bf16x2(ew[w]));
+                    const uint64_t kb2 = f2_from_bf16x2(kw[w]);
+                    const uint64_t dkw = f2_mul(f2_make(x[e], x[e + 1]), f2_make(__frcp_rn(eg.x), __frcp_rn(eg.y)));
+                    const uint64_t v = f2_add(f2_add(f2_add(dkw, f2_from_bf16x2(cw[w])), f2_make(y[e], y[e + 1])), dm[w]);
+                    dkb[4 * q4 + w] = v;
+                    dot2 = f2_fma(kb2, v, dot2);
+                    const float2 g = f2_split(f2_fma(f2_mul(kb2, f2_make(-1.f, -1.f)), dkw, f2_from_bf16x2(gw[w])));
+                    dgrow[8 * cc + 2 * w] = g.x;
+                    dgrow[8 * cc + 2 * w + 1] = g.y;
                 }
             }
+            const float2 dv = f2_split(dot2);
+            dot = dv.x + dv.y;
         }
         dot += __shfl_xor_sync(0xffffffffu, dot, 16);
         if (hf == 0) red[grp * 128 + i] = dot;
@@ -1079,15 +1105,19 @@ gla_bwd_kv_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_consta
         }
         compute_sync();
         dot = red[i] + red[128 + i];
+        const uint64_t ndot = f2_make(-dot, -dot), rk2 = f2_make(rk, rk);
 #pragma unroll
         for (int q4 = 0; q4 < 4; ++q4) {
             const int cc = 4 * h2 + q4;
-            float kb[8], out[8];
-            load_row_chunk(kt, i, cc, kb);
+            const uint4 kr = *reinterpret_cast<const uint4 *>(kt + t64_chunk(i, cc));
+            const uint32_t kw[4] = {kr.x, kr.y, kr.z, kr.w};
+            uint32_t ow[4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e)
-                out[e] = a.l2norm ? rk * fmaf(-kb[e], dot, dkb[8 * q4 + e]) : dkb[8 * q4 + e];
-            store_row_chunk(kt, i, cc, out);
+            for (int w = 0; w < 4; ++w) {
+                const uint64_t v = dkb[4 * q4 + w];
+                ow[w] = bf16x2_from_f2(a.l2norm ? f2_mul(rk2, f2_fma(ndot, f2_from_bf16x2(kw[w]), v)) : v);
+            }
+            *reinterpret_cast<uint4 *>(kt + t64_chunk(i, cc)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
         }
     }
     fence_proxy_async_smem();
