@@ -239,10 +239,11 @@ __device__ __forceinline__ void masked_row(uint8_t *tile, int i, int hf, const f
 }
 
 __device__ __forceinline__ float masked_sum(int i, int hf, const float (&sc)[32]) {
-    float part = 0.f;
+    float pa[4] = {0.f, 0.f, 0.f, 0.f};  // four chains of eight
 #pragma unroll
     for (int jj = 0; jj < 32; ++jj)
-        if (32 * hf + jj <= i) part += sc[jj];
+        if (32 * hf + jj <= i) pa[jj & 3] += sc[jj];
+    const float part = (pa[0] + pa[1]) + (pa[2] + pa[3]);
     return part + __shfl_xor_sync(0xffffffffu, part, 16);
 }
 
@@ -787,16 +788,25 @@ gla_bwd_state_kernel(const __grid_constant__ CUtensorMap map_qg, const __grid_co
             float x[32];
             tmem_ld32(tq + TM_X + 32 * th, x);
             if (it > 0) {
+                uint64_t cs2 = 0;  // fp32 pairs: two chains
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
-                    float sx[8];
-                    load_row_chunk(sm + OFF_SX, row, 4 * th + q4, sx);
+                    const uint4 sr = *reinterpret_cast<const uint4 *>(sm + OFF_SX + t64_chunk(row, 4 * th + q4));
+                    const uint32_t sw[4] = {sr.x, sr.y, sr.z, sr.w};
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) cs = fmaf(x[8 * q4 + e], sx[e], cs);
+                    for (int w = 0; w < 4; ++w)
+                        cs2 = f2_fma(f2_make(x[8 * q4 + 2 * w], x[8 * q4 + 2 * w + 1]), f2_from_bf16x2(sw[w]), cs2);
                 }
+                const float2 cv = f2_split(cs2);
+                cs = cv.x + cv.y;
             }
+            const uint64_t hs2 = f2_make(hs, hs);
 #pragma unroll
-            for (int e = 0; e < 32; ++e) x[e] *= hs;
+            for (int e = 0; e < 16; ++e) {
+                const float2 y = f2_split(f2_mul(f2_make(x[2 * e], x[2 * e + 1]), hs2));
+                x[2 * e] = y.x;
+                x[2 * e + 1] = y.y;
+            }
 #pragma unroll
             for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_IMG, row, 4 * th + q4, x + 8 * q4);
             tmem_st32(tq + TM_X + 32 * th, x);
