@@ -167,22 +167,18 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
     }
     compute_sync();
     const int p = pt & 63, qt = pt >> 6, d0 = 2 * p;
-    float g0[16], g1[16];
-    float r0 = 0.f, r1 = 0.f;
+    uint64_t g2[16];  // cumulative gates of dims d0, d0 + 1 as fp32 pairs
+    uint64_t r2 = 0;
 #pragma unroll
     for (int jj = 0; jj < 16; ++jj) {
         const int j = 16 * qt + jj;
-        float x0, x1;
-        if (gate_f32) {
-            const float2 f2 = *reinterpret_cast<const float2 *>(kd_tile + (j * kD + d0) * 4);
-            x0 = f2.x; x1 = f2.y;
-        } else {
-            const float2 f2 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(kd_tile + (j * kD + d0) * 2));
-            x0 = f2.x; x1 = f2.y;
-        }
-        r0 += x0; r1 += x1;
-        g0[jj] = r0; g1[jj] = r1;
+        const uint64_t x2 = gate_f32 ? *reinterpret_cast<const uint64_t *>(kd_tile + (j * kD + d0) * 4)
+                                     : f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(kd_tile + (j * kD + d0) * 2));
+        r2 = f2_add(r2, x2);
+        g2[jj] = r2;
     }
+    const float2 rv = f2_split(r2);
+    const float r0 = rv.x, r1 = rv.y;
     gq4[qt * kD + d0] = r0;
     gq4[qt * kD + d0 + 1] = r1;
     compute_sync();  // every raw gate read, quarter sums visible
@@ -194,7 +190,8 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
             off1 += gq4[q * kD + d0 + 1];
         }
     const float gm0 = gq4[d0] + gq4[kD + d0], gm1 = gq4[d0 + 1] + gq4[kD + d0 + 1];  // Gmid
-    const float o0 = (off0 - gm0) * kLog2e, o1 = (off1 - gm1) * kLog2e;
+    const uint64_t o2 = f2_make((off0 - gm0) * kLog2e, (off1 - gm1) * kLog2e);
+    const uint64_t l2e = f2_make(kLog2e, kLog2e);
     if (qt == 3) {
         if (f) {
             f[d0] = fast_exp2((off0 + r0 - gm0) * kLog2e);
@@ -214,10 +211,10 @@ __device__ void prep_chunk(uint8_t *q_tile, uint8_t *k_tile, uint8_t *kd_tile, u
     for (int jj = 0; jj < 16; ++jj) {
         const int j = 16 * qt + jj;
         const uint32_t off = tcol + t64_offset(j, d0 & 63);
-        const float2 kr = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&kraw[jj]));
-        const float x0 = fmaf(g0[jj], kLog2e, o0), x1 = fmaf(g1[jj], kLog2e, o1);
-        *reinterpret_cast<uint32_t *>(kd_tile + off) = pack_bf16(kr.x * fast_exp2(-x0), kr.y * fast_exp2(-x1));
-        *reinterpret_cast<uint32_t *>(eg_tile + off) = pack_bf16(fast_exp2(x0), fast_exp2(x1));
+        const float2 x = f2_split(f2_fma(g2[jj], l2e, o2));
+        *reinterpret_cast<uint32_t *>(kd_tile + off) =
+            bf16x2_from_f2(f2_mul(f2_from_bf16x2(kraw[jj]), f2_make(fast_exp2(-x.x), fast_exp2(-x.y))));
+        *reinterpret_cast<uint32_t *>(eg_tile + off) = pack_bf16(fast_exp2(x.x), fast_exp2(x.y));
     }
     fence_proxy_async_smem();
     compute_sync();
