@@ -162,17 +162,16 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     __syncthreads();
     {
         // A_ij for j < i, written over the k tile (the product has read it)
-        const float ri = epos[i];
+        const uint64_t ri2 = f2_make(epos[i], epos[i]);
 #pragma unroll
         for (int q4 = 0; q4 < 8; ++q4) {
-            const float4 cf = *reinterpret_cast<const float4 *>(eneg + 32 * hf + 4 * q4);
-            const float cfa[4] = {cf.x, cf.y, cf.z, cf.w};
+            const ulonglong2 cf = *reinterpret_cast<const ulonglong2 *>(eneg + 32 * hf + 4 * q4);
+            const float2 a01 = f2_split(f2_mul(f2_mul(ri2, cf.x), f2_make(kk[4 * q4], kk[4 * q4 + 1])));
+            const float2 a23 = f2_split(f2_mul(f2_mul(ri2, cf.y), f2_make(kk[4 * q4 + 2], kk[4 * q4 + 3])));
+            const float av[4] = {a01.x, a01.y, a23.x, a23.y};
             float w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int j = 32 * hf + 4 * q4 + e;
-                w[e] = (j < i) ? ri * cfa[e] * kk[4 * q4 + e] : 0.f;
-            }
+            for (int e = 0; e < 4; ++e) w[e] = (32 * hf + 4 * q4 + e < i) ? av[e] : 0.f;
             *reinterpret_cast<float4 *>(A + i * kAS + 32 * hf + 4 * q4) = make_float4(w[0], w[1], w[2], w[3]);
         }
     }
@@ -675,10 +674,15 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             {
                 float x[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
+                const uint64_t sc2 = f2_make(a.scale, a.scale);
 #pragma unroll
-                for (int e = 0; e < 32; ++e) x[e] *= a.scale;
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    uint32_t w[4];
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_UB + grp * 8192, i, 4 * hf + q4, x + 8 * q4);
+                    for (int u = 0; u < 4; ++u)
+                        w[u] = bf16x2_from_f2(f2_mul(f2_make(x[8 * q4 + 2 * u], x[8 * q4 + 2 * u + 1]), sc2));
+                    *reinterpret_cast<uint4 *>(sm + OFF_UB + grp * 8192 + t64_chunk(i, 4 * hf + q4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                }
                 fence_proxy_async_smem();
             }
             tc_fence_before();

@@ -437,10 +437,15 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (!a.skip_o) {
                 float x[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
+                const uint64_t sc2 = f2_make(a.scale, a.scale);
 #pragma unroll
-                for (int e = 0; e < 32; ++e) x[e] *= a.scale;
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    uint32_t w[4];
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(sm + OFF_V + grp * 8192, i, 4 * hf + q4, x + 8 * q4);
+                    for (int u = 0; u < 4; ++u)
+                        w[u] = bf16x2_from_f2(f2_mul(f2_make(x[8 * q4 + 2 * u], x[8 * q4 + 2 * u + 1]), sc2));
+                    *reinterpret_cast<uint4 *>(sm + OFF_V + grp * 8192 + t64_chunk(i, 4 * hf + q4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                }
                 fence_proxy_async_smem();
             }
             tc_fence_before();
