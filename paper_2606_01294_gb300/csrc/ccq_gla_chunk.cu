@@ -30,7 +30,7 @@
 // Kg = kbar * e^{Gmid - G}, Ssnap = e^{Gmid} S_r, and S_{r+1} = e^{Gtot - Gmid} X_{r+1}
 // (that factor is applied at the next snapshot).
 //
-// Warp specialisation (13 warps):
+// Warp specialisation (14 warps):
 //   EPI   (warps 0-7)   the epilogues of chunk r -- W, q_clean, mask of A, output --
 //                       and the bf16 operand copies of the states, placed where EPI
 //                       would otherwise wait on an MMA: S^K_{r+1} while G4 runs,
@@ -41,12 +41,14 @@
 //                       from registers straight to global memory.
 //   PREP  (warps 8-11)  prep of chunk r+1 while the chain runs chunk r: gate
 //                       cumsum, row norms, kbar, Kg, e^{G-Gmid}, M . qbar, lambda.
-//   ISSUE (warp 12)     one thread issues every tcgen05.mma and TMA load, in the
-//                       order G2 | G1 | G3 G8 | G7 | G4 G6 | G5, so that G1, G7 and G6
-//                       run under the epilogues.  An MMA instruction holds its issuing
-//                       thread for its whole execution, which is why no epilogue
-//                       thread issues.  EPI signals the issuer with named-barrier
-//                       arrives; the issuer signals EPI with MMA commits.
+//   ISSUE (warp 12)     one thread issues every tcgen05.mma (and, unless COPY does,
+//                       the per-chunk TMA copies), in the order G2 | G1 | G3 G8 | G7 |
+//                       G4 G6 | G5, so that G1, G7 and G6 run under the epilogues.  An MMA
+//                       instruction holds its issuing thread for its whole execution,
+//                       which is why no epilogue thread issues.  EPI signals the issuer
+//                       with named-barrier arrives; the issuer signals EPI with commits.
+//   COPY  (warp 13)     in the COPY instance: the loads of chunk r+2, the store of O and the
+//                       next v, plus an L2 prefetch of chunk r+2 beyond each load.
 // Per-chunk tiles are double-buffered (two slots); the loads of chunk r+2 start as
 // soon as chunk r's last MMA reader of the slot (G6) completes.  v is single-buffered
 // and reloaded once G5 of the previous chunk completes.
@@ -73,9 +75,10 @@ namespace {
 constexpr int kC = 64;         // chunk length
 constexpr int kD = 128;        // Dk = Dv
 constexpr int kEpiThreads = 256;
-constexpr int kPrepWarp0 = 8, kIssueWarp = 12;
-constexpr int kThreads = 32 * (kIssueWarp + 1);  // 416
-constexpr int kSyncCount = kEpiThreads + 32;     // EPI + the issuing warp
+constexpr int kPrepWarp0 = 8, kIssueWarp = 12, kCopyWarp = 13;
+constexpr int kThreadsNoCopy = 32 * kCopyWarp;       // 416
+constexpr int kThreadsCopy = 32 * (kCopyWarp + 1);    // 448
+constexpr int kSyncCount = kEpiThreads + 32;          // EPI + the issuing warp
 
 // ---- shared memory map (bytes from the 1024-aligned base)
 // two slots of per-chunk tiles, each [64 rows][128 cols] bf16 as two T64 tiles of 8 KB:
@@ -141,10 +144,13 @@ __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chun
     *reinterpret_cast<uint4 *>(tile + t64_chunk(row, chunk)) = u;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+template <bool COPY>
+__global__ void __launch_bounds__(COPY ? kThreadsCopy : kThreadsNoCopy, 1)
 gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                  const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_g,
                  const __grid_constant__ CUtensorMap map_o, const ChunkArgs a) {
+    // the output barrier: EPI and the issuing warp, and the copy warp when there is one
+    constexpr int kOutCount = kEpiThreads + (COPY ? 64 : 32);
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = smem_align1024(smem_raw);
     const uint32_t sb = smem_addr(sm);
@@ -196,12 +202,24 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_4d(base + SO_K, &map_k, bb, 0, h, tg, b);
         tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tg, b);
         tma_load_4d(base + SO_KG, &map_g, bb, 0, h, tg, b);
+        if (COPY && r + 2 < NC) {  // chunk r + 2 into L2, so that its loads hit there
+            const int tp = tg + 2 * kC;
+            tma_prefetch_l2_4d(&map_q, 0, h, tp, b);
+            tma_prefetch_l2_4d(&map_q, 64, h, tp, b);
+            tma_prefetch_l2_4d(&map_k, 0, h, tp, b);
+            tma_prefetch_l2_4d(&map_k, 64, h, tp, b);
+            tma_prefetch_l2_4d(&map_g, 0, h, tp, b);
+        }
     };
     auto issue_v = [&](int r) {
         const int tg = (cb + r) * kC;
         mbar_arrive_expect_tx(&bar[BAR_V], 2 * 8192);
         tma_load_4d(sm + OFF_V, &map_v, &bar[BAR_V], 0, h, tg, b);
         tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, tg, b);
+        if (COPY && r + 2 < NC) {
+            tma_prefetch_l2_4d(&map_v, 0, h, tg + 2 * kC, b);
+            tma_prefetch_l2_4d(&map_v, 64, h, tg + 2 * kC, b);
+        }
     };
 
     // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
@@ -449,7 +467,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 fence_proxy_async_smem();
             }
             tc_fence_before();
-            named_bar_arrive(NB_OUT, kSyncCount);
+            named_bar_arrive(NB_OUT, kOutCount);
             // ---- e^{Gmid_{r+1}} S_{r+1} while G2 of chunk r+1 runs (G6 and G7 of chunk r
             // have run: GD follows them)
             if (r + 1 < NC) {
@@ -639,7 +657,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const int sl = (NC - 1) & 1;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
-    } else {
+    } else if (warp == kIssueWarp) {
         // =============================================================== ISSUE
         const bool lead = lane == 0;
         // descriptor bases (start-address field advanced per K slice: +2 per 32 B)
@@ -668,10 +686,11 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
             __syncwarp();
             if (r > 0) {
-                // O of chunk r-1 is staged in the v tile: store it
+                // O of chunk r-1 has left PO (staged in the v tile): store it (unless the copy
+                // warp does)
                 mbar_wait(&bar[BAR_GD], (r - 1) & 1, abort_flag, status);
-                named_bar(NB_OUT, kSyncCount);  // O of chunk r-1 read out of PO and staged
-                if (lead && !a.skip_o) {
+                named_bar(NB_OUT, kOutCount);
+                if (lead && !COPY && !a.skip_o) {
                     const int cp = (cb + r - 1) * kC;
                     tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
                     tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
@@ -687,7 +706,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
                              dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
             // v of chunk r replaces the staged output once the store has read it
-            if (r > 0 && lead) {
+            if (r > 0 && lead && !COPY) {
                 tma_store_wait_read();
                 if (!*abort_flag) issue_v(r);
             }
@@ -737,7 +756,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
             __syncwarp();
             // the slot's last MMA reader (G6) is done: load chunk r + 2 into it
-            if (r + 2 < NC) {
+            if (!COPY && r + 2 < NC) {
                 mbar_wait(&bar[BAR_GC2], par, abort_flag, status);
                 if (lead && !*abort_flag) issue_in(r + 2);
                 __syncwarp();
@@ -745,8 +764,8 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         }
         if (NC > 0) {
             mbar_wait(&bar[BAR_GD], (NC - 1) & 1, abort_flag, status);
-            named_bar(NB_OUT, kSyncCount);
-            if (lead && !a.skip_o) {
+            named_bar(NB_OUT, kOutCount);
+            if (lead && !COPY && !a.skip_o) {
                 const int cp = (cb + NC - 1) * kC;
                 tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
                 tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
@@ -758,6 +777,39 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 mbar_drain(&bar[BAR_V], (NC - 1) & 1);
                 for (int r = (NC > 2 ? NC - 2 : 0); r < NC; ++r) mbar_drain(&bar[BAR_IN0 + (r & 1)], (r >> 1) & 1);
             }
+        }
+    } else {
+        // =============================================================== COPY
+        // The per-chunk copies, which can hold a thread for a thousand
+        // cycles while the copy engine is busy -- the loads of chunk r + 2 once G6 of chunk r
+        // has read the slot, the store of O (staged in the v tile), the next v once that
+        // store has read it (the instance without this warp has the issuer make them).
+        const bool lead = lane == 0;
+        for (int r = 0; r < NC; ++r) {
+            if (COPY && r + 2 < NC) {
+                mbar_wait(&bar[BAR_GC2], r & 1, abort_flag, status);
+                if (lead && !*abort_flag) issue_in(r + 2);
+                __syncwarp();
+            }
+            named_bar(NB_OUT, kOutCount);  // O of chunk r staged in the v tile
+            if (lead && COPY) {
+                if (!a.skip_o) {
+                    const int cp = (cb + r) * kC;
+                    tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
+                    tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
+                    tma_store_commit();
+                }
+                if (r + 1 < NC) {
+                    tma_store_wait_read();
+                    if (!*abort_flag) issue_v(r + 1);
+                }
+            }
+            __syncwarp();
+        }
+        if (lead) tma_store_wait_all();
+        if (lead && COPY && NC > 0 && *abort_flag) {
+            mbar_drain(&bar[BAR_V], (NC - 1) & 1);
+            for (int r = (NC > 2 ? NC - 2 : 0); r < NC; ++r) mbar_drain(&bar[BAR_IN0 + (r & 1)], (r >> 1) & 1);
         }
     }
 
@@ -774,12 +826,20 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s) {
     static bool attr_set = false;
     if (!attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gla_chunk_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(gla_chunk_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(kSmemBytes));
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(gla_chunk_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(kSmemBytes));
         if (e != cudaSuccess) return e;
         attr_set = true;
     }
-    gla_chunk_kernel<<<a.B * a.H * a.nseg, kThreads, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, m.o, a);
+    // The copy warp (with the L2 prefetch of chunk r + 2) measured faster for whole sequences
+    // without checkpoints (4K: 268 -> 253 us) and slower with segments or checkpoint copies.
+    if (a.nseg == 1 && a.ckpt == nullptr)
+        gla_chunk_kernel<true><<<a.B * a.H, kThreadsCopy, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, m.o, a);
+    else
+        gla_chunk_kernel<false><<<a.B * a.H * a.nseg, kThreadsNoCopy, kSmemBytes, s>>>(m.q, m.k, m.v, m.g, m.o, a);
     return cudaGetLastError();
 }
 
