@@ -37,20 +37,22 @@
 //                        the chunk-local CCQ part of dkbar (W2^T DZ + W3^T Qbar),
 //                        and the chunk's inputs to the carried sums (QG, DZ
 //                        scaled by 1/|q|, the Dm increment, the gate factors).
-//   gla_bwd_state_kernel one CTA per sequence and head, chunks last to first:
-//                        carries dS (kept as e^{-Gmid} dS, like the forward's
-//                        deferred state scaling) and DC in TMEM and Dm, and
-//                        writes, per chunk, the states carried into it (bf16
-//                        tile images of Diag(e^{Gc-Gmid}) dS_{r+1} and DC_{r+1},
-//                        Dm_{r+1}) and the gate carry rowsum(dS_{r+1} S_{r+1}).
+//   gla_bwd_state_kernel two CTAs per sequence and head (one per column half of
+//                        dS and DC), chunks last to first: carries dS (kept as
+//                        e^{-Gmid} dS, like the forward's deferred state scaling)
+//                        and DC in TMEM and Dm, and writes, per chunk, the states
+//                        carried into it (bf16 tile images of Diag(e^{Gc-Gmid})
+//                        dS_{r+1} and DC_{r+1}, Dm_{r+1}) and the gate carry
+//                        rowsum(dS_{r+1} S_{r+1}) as two column-half sums.
 //   gla_bwd_kv_kernel    one CTA per chunk (parallel): dk (write part, the
 //                        CCQ inter term K (DC + DC^T), Dm), dv, dgk.
 // 64-row products are M = 64 MMAs whose rows 16q..16q+15 sit in TMEM lanes
-// 32q..32q+15, so in the chunk-parallel kernels (256 threads, two warps per lane
-// quadrant) thread (warp w, lane l) owns row 16 (w % 4) + l % 16, column half
-// l / 16 of a 64-column load, and -- for 128-column products -- the 32-column
-// slice w / 4 of each half; 128-row products (the carried states, 128 threads)
-// give thread t row t.
+// 32q..32q+15, so in the chunk-parallel kernels (256 compute threads, two warps
+// per lane quadrant, plus a warp that issues the input copies) thread (warp w,
+// lane l) owns row 16 (w % 4) + l % 16, column half l / 16 of a 64-column load,
+// and -- for 128-column products -- the 32-column slice w / 4 of each half; in
+// the state pass (256 threads) thread t owns state row t % 128 and the 32-column
+// slice t / 128 of its CTA's column half.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
