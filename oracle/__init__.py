@@ -15,6 +15,9 @@ Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``)
                      with the recurrent form.
   gla_backward       reverse mode of the CCQ-GLA forward -- pinned by central
                      finite differences of the forward (fp64).
+  gdn_backward       reverse mode of the CCQ-Gated-DeltaNet forward -- pinned the
+                     same way (tests/test_oracle_backward_gdn.py); no GPU path
+                     consumes it yet.
   Absolute outputs on the benchmark-shaped random inputs are pinned only
   through the above: the paper prints no worked numerical example.
 """
@@ -23,6 +26,7 @@ from .ccq_oracle import (  # noqa: F401
     forward,
     decode_step,
     gla_backward,
+    gdn_backward,
     GLA,
     GDN,
 )

@@ -432,6 +432,10 @@ typedef struct {
     const double *q, *k, *v, *gk, *lam, *S0, *C0, *m0, *dout, *dST, *dCT, *dmT;
     const int64_t *t0;
     double *dq, *dk, *dv, *dgk, *dlam, *dS0, *dC0, *dm0;
+    /* Gated DeltaNet only: gk is then the scalar log decay g [B,T,H], beta [B,T,H],
+       and dgk receives dg [B,T,H] */
+    const double *beta;
+    double *dbeta;
     int next;
     pthread_mutex_t mu;
 } bjob_t;
@@ -660,6 +664,240 @@ int ccq_oracle_gla_backward(int B, int T, int H, int Dk, int Dv, const double *q
     if (nthreads > B * H) nthreads = B * H > 0 ? B * H : 1;
     pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
     for (int i = 0; i < nthreads; ++i) pthread_create(&th[i], NULL, bworker, &J);
+    for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
+    free(th);
+    pthread_mutex_destroy(&J.mu);
+    return 0;
+}
+
+/* ====================================================================== reverse mode, Gated DeltaNet
+ *
+ * Gradients of the CCQ-Gated-DeltaNet forward (recurrent form above), same scheme as the GLA
+ * backward: block checkpoints every 64 tokens, each block recomputed and walked backwards.  The
+ * write, with the state stored as Hs = S^T [Dk][Dv], a = e^{g_t}, u = Hs_{t-1}^T kbar, is
+ *   Hs_t = a (Hs_{t-1} - beta kbar u^T) + beta kbar v^T,
+ * and with G the adjoint of Hs_t its adjoints are
+ *   dv = beta G^T kbar,  du = -a beta G^T kbar,
+ *   dkbar (write) = G (beta v - a beta u) + Hs_{t-1} du,
+ *   da = sum(G * (Hs_{t-1} - beta kbar u^T)),  dg = a da,
+ *   dbeta = kbar^T G (v - a u),  dHs_{t-1} = a G + kbar du^T.
+ * The read, the cleaned query and the key statistics are as in the GLA backward.
+ */
+static void backward_pair_gdn(const bjob_t *J, int b, int h) {
+    const int Dk = J->Dk, Dv = J->Dv, T = J->T, BL = 64;
+    const int NB = (T + BL - 1) / BL;
+    const size_t bh = (size_t)b * J->H + h;
+    const size_t SS = (size_t)Dk * Dv, CC = (size_t)Dk * Dk;
+    double *ckS = malloc(sizeof(double) * SS * (NB + 1));
+    double *ckC = malloc(sizeof(double) * CC * (NB + 1));
+    double *ckm = malloc(sizeof(double) * Dk * (NB + 1));
+    double *bS = malloc(sizeof(double) * SS * (BL + 1));
+    double *bC = malloc(sizeof(double) * CC * (BL + 1));
+    double *bm = malloc(sizeof(double) * Dk * (BL + 1));
+    double *qb = malloc(sizeof(double) * Dk), *kb = malloc(sizeof(double) * Dk);
+    double *z = malloc(sizeof(double) * Dk), *qc = malloc(sizeof(double) * Dk);
+    double *dqc = malloc(sizeof(double) * Dk), *dz = malloc(sizeof(double) * Dk);
+    double *dqb = malloc(sizeof(double) * Dk), *dkb = malloc(sizeof(double) * Dk);
+    double *u = malloc(sizeof(double) * Dv), *gtk = malloc(sizeof(double) * Dv), *du = malloc(sizeof(double) * Dv);
+    double *dS = malloc(sizeof(double) * SS), *dC = malloc(sizeof(double) * CC);
+    double *dm = malloc(sizeof(double) * Dk);
+    const int64_t tstart = J->t0 ? J->t0[b] : 0;
+
+    if (J->S0) memcpy(ckS, J->S0 + bh * SS, sizeof(double) * SS); else memset(ckS, 0, sizeof(double) * SS);
+    if (J->C0) memcpy(ckC, J->C0 + bh * CC, sizeof(double) * CC); else memset(ckC, 0, sizeof(double) * CC);
+    if (J->m0) memcpy(ckm, J->m0 + bh * Dk, sizeof(double) * Dk); else memset(ckm, 0, sizeof(double) * Dk);
+
+    /* one token's write: Sn = a (Sp - beta kb u^T) + beta kb v^T, u = Sp^T kb */
+#define GDN_WRITE(Sp, Sn, r)                                                                  \
+    do {                                                                                      \
+        const double a_ = exp(J->gk[(r)]), be_ = J->beta[(r)];                                \
+        const double *vr_ = J->v + (r) * Dv;                                                  \
+        for (int e = 0; e < Dv; ++e) {                                                        \
+            double acc = 0.0;                                                                 \
+            for (int i = 0; i < Dk; ++i) acc += kb[i] * (Sp)[(size_t)i * Dv + e];             \
+            u[e] = acc;                                                                       \
+        }                                                                                     \
+        for (int i = 0; i < Dk; ++i)                                                          \
+            for (int e = 0; e < Dv; ++e)                                                      \
+                (Sn)[(size_t)i * Dv + e] =                                                    \
+                    a_ * ((Sp)[(size_t)i * Dv + e] - be_ * kb[i] * u[e]) + be_ * kb[i] * vr_[e]; \
+    } while (0)
+
+    for (int blk = 0; blk < NB; ++blk) {
+        double *S = ckS + SS * (blk + 1), *C = ckC + CC * (blk + 1), *m = ckm + (size_t)Dk * (blk + 1);
+        memcpy(bS, ckS + SS * blk, sizeof(double) * SS);
+        memcpy(C, ckC + CC * blk, sizeof(double) * CC);
+        memcpy(m, ckm + (size_t)Dk * blk, sizeof(double) * Dk);
+        for (int tl = blk * BL; tl < T && tl < (blk + 1) * BL; ++tl) {
+            const size_t r = brow(J, b, tl, h);
+            double nk;
+            normalise_with_norm(J->k + r * Dk, kb, &nk, Dk, J->l2norm);
+            for (int i = 0; i < Dk; ++i) {
+                for (int j = 0; j < Dk; ++j) C[(size_t)i * Dk + j] += kb[i] * kb[j];
+                m[i] += kb[i];
+            }
+            GDN_WRITE(bS, bS + SS, r);
+            memcpy(bS, bS + SS, sizeof(double) * SS);
+        }
+        memcpy(S, bS, sizeof(double) * SS);
+    }
+
+    if (J->dST) memcpy(dS, J->dST + bh * SS, sizeof(double) * SS); else memset(dS, 0, sizeof(double) * SS);
+    if (J->dCT) memcpy(dC, J->dCT + bh * CC, sizeof(double) * CC); else memset(dC, 0, sizeof(double) * CC);
+    if (J->dmT) memcpy(dm, J->dmT + bh * Dk, sizeof(double) * Dk); else memset(dm, 0, sizeof(double) * Dk);
+
+    for (int blk = NB - 1; blk >= 0; --blk) {
+        const int t_lo = blk * BL, t_hi = (T < (blk + 1) * BL) ? T : (blk + 1) * BL;
+        /* recompute the block's per-token states: index 0 = block start, i + 1 = after token t_lo + i */
+        memcpy(bS, ckS + SS * blk, sizeof(double) * SS);
+        memcpy(bC, ckC + CC * blk, sizeof(double) * CC);
+        memcpy(bm, ckm + (size_t)Dk * blk, sizeof(double) * Dk);
+        for (int tl = t_lo; tl < t_hi; ++tl) {
+            const int ix = tl - t_lo;
+            const size_t r = brow(J, b, tl, h);
+            double nk;
+            normalise_with_norm(J->k + r * Dk, kb, &nk, Dk, J->l2norm);
+            const double *Cp = bC + CC * ix, *mp = bm + (size_t)Dk * ix;
+            double *Cn = bC + CC * (ix + 1), *mn = bm + (size_t)Dk * (ix + 1);
+            for (int i = 0; i < Dk; ++i) {
+                for (int j = 0; j < Dk; ++j) Cn[(size_t)i * Dk + j] = Cp[(size_t)i * Dk + j] + kb[i] * kb[j];
+                mn[i] = mp[i] + kb[i];
+            }
+            GDN_WRITE(bS + SS * ix, bS + SS * (ix + 1), r);
+        }
+        for (int tl = t_hi - 1; tl >= t_lo; --tl) {
+            const int ix = tl - t_lo;
+            const size_t r = brow(J, b, tl, h);
+            const double tf = (double)(tstart + tl + 1);
+            const double *St = bS + SS * (ix + 1), *Sp = bS + SS * ix;
+            const double *Ct = bC + CC * (ix + 1), *mt = bm + (size_t)Dk * (ix + 1);
+            const double lam = J->lam[r], a = exp(J->gk[r]), be = J->beta[r];
+            const double *dor = J->dout + r * Dv, *vr = J->v + r * Dv;
+            double nq, nk;
+            normalise_with_norm(J->q + r * Dk, qb, &nq, Dk, J->l2norm);
+            normalise_with_norm(J->k + r * Dk, kb, &nk, Dk, J->l2norm);
+            /* forward quantities of token t: z, q_clean, u = Hs_{t-1}^T kbar */
+            double mq = 0.0;
+            for (int j = 0; j < Dk; ++j) mq += mt[j] * qb[j];
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int j = 0; j < Dk; ++j) acc += Ct[(size_t)i * Dk + j] * qb[j];
+                z[i] = acc / tf - (J->centered ? mt[i] * mq / (tf * tf) : 0.0);
+                qc[i] = qb[i] - lam * z[i];
+            }
+            for (int e = 0; e < Dv; ++e) {
+                double acc = 0.0;
+                for (int i = 0; i < Dk; ++i) acc += kb[i] * Sp[(size_t)i * Dv + e];
+                u[e] = acc;
+            }
+            /* read: o = scale Hs_t^T q_clean */
+            double dl = 0.0;
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int e = 0; e < Dv; ++e) {
+                    acc += St[(size_t)i * Dv + e] * dor[e];
+                    dS[(size_t)i * Dv + e] += J->scale * qc[i] * dor[e];
+                }
+                dqc[i] = J->scale * acc;
+                dz[i] = -lam * dqc[i];
+                dl -= z[i] * dqc[i];
+            }
+            J->dlam[r] = dl;
+            /* clean: dqbar = dq_clean + Sigma_t dz; statistics adjoints */
+            double mdz = 0.0;
+            for (int j = 0; j < Dk; ++j) mdz += mt[j] * dz[j];
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int j = 0; j < Dk; ++j) acc += Ct[(size_t)i * Dk + j] * dz[j];
+                dqb[i] = dqc[i] + acc / tf - (J->centered ? mt[i] * mdz / (tf * tf) : 0.0);
+            }
+            for (int i = 0; i < Dk; ++i) {
+                for (int j = 0; j < Dk; ++j) dC[(size_t)i * Dk + j] += dz[i] * qb[j] / tf;
+                if (J->centered) dm[i] -= (mq * dz[i] + mdz * qb[i]) / (tf * tf);
+            }
+            /* write: G = dS is the adjoint of Hs_t */
+            for (int e = 0; e < Dv; ++e) {
+                double acc = 0.0;
+                for (int i = 0; i < Dk; ++i) acc += dS[(size_t)i * Dv + e] * kb[i];
+                gtk[e] = acc;                       /* G^T kbar */
+                J->dv[r * Dv + e] = be * acc;
+                du[e] = -a * be * acc;
+            }
+            double da = 0.0, dbe = 0.0;
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0, hs = 0.0, gsum = 0.0;
+                for (int e = 0; e < Dv; ++e) {
+                    const double G = dS[(size_t)i * Dv + e];
+                    acc += G * (be * vr[e] - a * be * u[e]);
+                    hs += Sp[(size_t)i * Dv + e] * du[e];
+                    gsum += G * (Sp[(size_t)i * Dv + e] - be * kb[i] * u[e]);
+                    dbe += kb[i] * G * (vr[e] - a * u[e]);
+                }
+                dkb[i] = acc + hs;
+                da += gsum;
+            }
+            J->dgk[r] = a * da;
+            J->dbeta[r] = dbe;
+            for (int i = 0; i < Dk; ++i)
+                for (int e = 0; e < Dv; ++e)
+                    dS[(size_t)i * Dv + e] = a * dS[(size_t)i * Dv + e] + kb[i] * du[e];
+            /* statistics: C_t = C_{t-1} + kbar kbar^T, m_t = m_{t-1} + kbar */
+            for (int i = 0; i < Dk; ++i) {
+                double acc = 0.0;
+                for (int j = 0; j < Dk; ++j) acc += (dC[(size_t)i * Dk + j] + dC[(size_t)j * Dk + i]) * kb[j];
+                dkb[i] += acc + dm[i];
+            }
+            normalise_backward(qb, nq, dqb, J->dq + r * Dk, Dk, J->l2norm);
+            normalise_backward(kb, nk, dkb, J->dk + r * Dk, Dk, J->l2norm);
+        }
+    }
+#undef GDN_WRITE
+    if (J->dS0) memcpy(J->dS0 + bh * SS, dS, sizeof(double) * SS);
+    if (J->dC0) memcpy(J->dC0 + bh * CC, dC, sizeof(double) * CC);
+    if (J->dm0) memcpy(J->dm0 + bh * Dk, dm, sizeof(double) * Dk);
+    free(ckS); free(ckC); free(ckm); free(bS); free(bC); free(bm); free(qb); free(kb); free(z); free(qc);
+    free(dqc); free(dz); free(dqb); free(dkb); free(u); free(gtk); free(du); free(dS); free(dC); free(dm);
+}
+
+static void *bworker_gdn(void *arg) {
+    bjob_t *J = (bjob_t *)arg;
+    for (;;) {
+        pthread_mutex_lock(&J->mu);
+        const int w = J->next++;
+        pthread_mutex_unlock(&J->mu);
+        if (w >= J->B * J->H) break;
+        backward_pair_gdn(J, w / J->H, w % J->H);
+    }
+    return NULL;
+}
+
+/*
+ * CCQ-Gated-DeltaNet backward.  Inputs as ccq_oracle_forward (GDN: g the log decay and beta,
+ * both [B,T,H]) plus dout [B,T,H,Dv] and optional adjoints of the final states (NULL = 0).
+ * Outputs dq, dk [B,T,H,Dk], dv [B,T,H,Dv], dg and dbeta [B,T,H], dlam [B,T,H], dS0, dC0,
+ * dm0 (each of the last three may be NULL).  Returns 0, or -1 on a bad argument.
+ */
+int ccq_oracle_gdn_backward(int B, int T, int H, int Dk, int Dv, const double *q, const double *k,
+                            const double *v, const double *g, const double *beta, const double *lam,
+                            const double *S0, const double *C0, const double *m0, const int64_t *t0,
+                            const double *dout, const double *dST, const double *dCT, const double *dmT,
+                            double *dq, double *dk, double *dv, double *dg, double *dbeta, double *dlam,
+                            double *dS0, double *dC0, double *dm0, int l2norm, int centered, double scale,
+                            int nthreads) {
+    if (B < 0 || T < 0 || H < 0 || Dk <= 0 || Dv <= 0 || nthreads < 1) return -1;
+    if (!q || !k || !v || !g || !beta || !lam || !dout || !dq || !dk || !dv || !dg || !dbeta || !dlam) return -1;
+    bjob_t J;
+    memset(&J, 0, sizeof J);
+    J.B = B; J.T = T; J.H = H; J.Dk = Dk; J.Dv = Dv; J.l2norm = l2norm; J.centered = centered;
+    J.scale = scale;
+    J.q = q; J.k = k; J.v = v; J.gk = g; J.beta = beta; J.lam = lam; J.S0 = S0; J.C0 = C0; J.m0 = m0;
+    J.t0 = t0; J.dout = dout; J.dST = dST; J.dCT = dCT; J.dmT = dmT;
+    J.dq = dq; J.dk = dk; J.dv = dv; J.dgk = dg; J.dbeta = dbeta; J.dlam = dlam;
+    J.dS0 = dS0; J.dC0 = dC0; J.dm0 = dm0;
+    pthread_mutex_init(&J.mu, NULL);
+    if (nthreads > B * H) nthreads = B * H > 0 ? B * H : 1;
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int i = 0; i < nthreads; ++i) pthread_create(&th[i], NULL, bworker_gdn, &J);
     for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
     free(th);
     pthread_mutex_destroy(&J.mu);

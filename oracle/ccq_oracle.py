@@ -52,6 +52,10 @@ def load_library(path: str):
         [ctypes.c_int] * 5 + [dp] * 8 + [ip] + [dp] * 4 + [dp] * 8
         + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int])
     lib.ccq_oracle_gla_backward.restype = ctypes.c_int
+    lib.ccq_oracle_gdn_backward.argtypes = (
+        [ctypes.c_int] * 5 + [dp] * 9 + [ip] + [dp] * 4 + [dp] * 9
+        + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int])
+    lib.ccq_oracle_gdn_backward.restype = ctypes.c_int
     return lib
 
 
@@ -174,3 +178,34 @@ def gla_backward(q, k, v, gk, lam, dout, S0=None, C0=None, m0=None, t0=None, dST
     if rc != 0:
         raise ValueError("ccq_oracle_gla_backward rejected its arguments")
     return g
+
+
+def gdn_backward(q, k, v, g, beta, lam, dout, S0=None, C0=None, m0=None, t0=None, dST=None,
+                 dCT=None, dmT=None, *, l2norm=True, centered=True, scale=None,
+                 nthreads=None, lib=None):
+    """Reverse mode of the CCQ-Gated-DeltaNet forward: gradients of sum(dout * o)
+    + sum(dST * S_T) + sum(dCT * C_T) + sum(dmT * m_T) with respect to
+    q, k, v, g (the log decay), beta, lam, S0, C0, m0 (shapes as in :func:`forward`)."""
+    lib = lib or _load()
+    q, k, v, g, beta, lam, dout = map(_f64, (q, k, v, g, beta, lam, dout))
+    S0, C0, m0, dST, dCT, dmT = map(_f64, (S0, C0, m0, dST, dCT, dmT))
+    t0 = _i64(t0)
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    if scale is None:
+        scale = Dk ** -0.5
+    if nthreads is None:
+        nthreads = os.cpu_count() or 1
+    r = {"dq": np.zeros_like(q), "dk": np.zeros_like(k), "dv": np.zeros_like(v),
+         "dg": np.zeros_like(g), "dbeta": np.zeros_like(beta), "dlam": np.zeros_like(lam),
+         "dS0": np.zeros((B, H, Dk, Dv)), "dC0": np.zeros((B, H, Dk, Dk)),
+         "dm0": np.zeros((B, H, Dk))}
+    rc = lib.ccq_oracle_gdn_backward(
+        B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _ptr(S0),
+        _ptr(C0), _ptr(m0), _ptr(t0, ctypes.c_int64), _ptr(dout), _ptr(dST), _ptr(dCT), _ptr(dmT),
+        _ptr(r["dq"]), _ptr(r["dk"]), _ptr(r["dv"]), _ptr(r["dg"]), _ptr(r["dbeta"]), _ptr(r["dlam"]),
+        _ptr(r["dS0"]), _ptr(r["dC0"]), _ptr(r["dm0"]), int(bool(l2norm)), int(bool(centered)),
+        float(scale), int(nthreads))
+    if rc != 0:
+        raise ValueError("ccq_oracle_gdn_backward rejected its arguments")
+    return r
