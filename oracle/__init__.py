@@ -18,6 +18,11 @@ Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``)
   gdn_backward       reverse mode of the CCQ-Gated-DeltaNet forward -- pinned the
                      same way (tests/test_oracle_backward_gdn.py); no GPU path
                      consumes it yet.
+  gdn_forward_decayed  CCQ-Gated-DeltaNet with the decay-aligned covariance (a reading of
+                     the paper's future-work variant, stated in ccq_oracle.c) -- pinned
+                     by brute-force weighted covariances, the undecayed special case,
+                     the spectrum bound and resumption (tests/test_oracle_decayed.py);
+                     no GPU path consumes it yet.
   Absolute outputs on the benchmark-shaped random inputs are pinned only
   through the above: the paper prints no worked numerical example.
 """
@@ -27,6 +32,7 @@ from .ccq_oracle import (  # noqa: F401
     decode_step,
     gla_backward,
     gdn_backward,
+    gdn_forward_decayed,
     GLA,
     GDN,
 )

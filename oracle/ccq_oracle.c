@@ -407,6 +407,128 @@ int ccq_oracle_forward(int backbone, int B, int T, int H, int Dk, int Dv,
     return 0;
 }
 
+/* ====================================================================== decay-aligned covariance
+ *
+ * The variant the paper names as future work for decayed backbones (Sec. 6 and the appendix
+ * paragraph on decayed backbones): the covariance is computed from gamma-weighted running
+ * statistics, gamma_{j,t} the factor by which the backbone has decayed key j's write by
+ * token t.  The paper fixes neither gamma nor the normaliser; this oracle takes the reading
+ *   gamma_{j,t} = prod_{s=j+1..t} alpha_s      (Gated DeltaNet's scalar decay),
+ *   C_t = alpha_t C_{t-1} + kbar_t kbar_t^T,  m_t = alpha_t m_{t-1} + kbar_t,
+ *   n_t = alpha_t n_{t-1} + 1                   (the decayed count, in place of t),
+ *   Sigma_t = C_t / n_t - (m_t / n_t)(m_t / n_t)^T  (centred; C_t / n_t uncentred),
+ * which is the undecayed definition when every alpha_t = 1.  Only a backbone with one decay
+ * per key (Gated DeltaNet) has such a factor; GLA's per-dimension gates have none.
+ */
+typedef struct {
+    int B, T, H, Dk, Dv, l2norm, centered;
+    double scale;
+    const double *q, *k, *v, *g, *beta, *lam, *S0, *C0, *m0, *n0;
+    double *o, *ST, *CT, *mT, *nT, *qc_out;
+    int next;
+    pthread_mutex_t mu;
+} djob_t;
+
+static void decayed_pair(const djob_t *J, int b, int h) {
+    const int Dk = J->Dk, Dv = J->Dv;
+    const size_t bh = (size_t)b * J->H + h;
+    double *Hs = calloc((size_t)Dk * Dv, sizeof(double));
+    double *Cg = calloc((size_t)Dk * Dk, sizeof(double));
+    double *mg = calloc((size_t)Dk, sizeof(double));
+    double *qb = malloc(sizeof(double) * Dk), *kb = malloc(sizeof(double) * Dk);
+    double *sg = malloc(sizeof(double) * Dk), *qcl = malloc(sizeof(double) * Dk);
+    double *kS = malloc(sizeof(double) * Dv);
+    if (J->S0) memcpy(Hs, J->S0 + bh * Dk * Dv, sizeof(double) * Dk * Dv);
+    if (J->C0) memcpy(Cg, J->C0 + bh * Dk * Dk, sizeof(double) * Dk * Dk);
+    if (J->m0) memcpy(mg, J->m0 + bh * Dk, sizeof(double) * Dk);
+    double n = J->n0 ? J->n0[bh] : 0.0;
+    for (int tl = 0; tl < J->T; ++tl) {
+        const size_t r = ((size_t)b * J->T + tl) * J->H + h;
+        const double *vr = J->v + r * Dv;
+        l2_normalise(J->q + r * Dk, qb, Dk, J->l2norm);
+        l2_normalise(J->k + r * Dk, kb, Dk, J->l2norm);
+        const double a = exp(J->g[r]), be = J->beta[r], lam = J->lam[r];
+        /* gamma-weighted statistics including token t */
+        for (int i = 0; i < Dk; ++i) {
+            for (int j = 0; j < Dk; ++j) Cg[(size_t)i * Dk + j] = a * Cg[(size_t)i * Dk + j] + kb[i] * kb[j];
+            mg[i] = a * mg[i] + kb[i];
+        }
+        n = a * n + 1.0;
+        /* Sigma^gamma_t qbar, then the cleaned query (Eq. clean with Sigma^gamma) */
+        double mq = 0.0;
+        for (int j = 0; j < Dk; ++j) mq += mg[j] * qb[j];
+        for (int i = 0; i < Dk; ++i) {
+            double acc = 0.0;
+            for (int j = 0; j < Dk; ++j) acc += Cg[(size_t)i * Dk + j] * qb[j];
+            sg[i] = acc / n - (J->centered ? mg[i] * mq / (n * n) : 0.0);
+        }
+        for (int i = 0; i < Dk; ++i) qcl[i] = qb[i] - lam * sg[i];
+        if (J->qc_out) memcpy(J->qc_out + r * Dk, qcl, sizeof(double) * Dk);
+        /* gated delta rule, written as S_t = a S_{t-1} + kbar u^T with u = beta (v - a S_{t-1}^T kbar) */
+        for (int j = 0; j < Dv; ++j) {
+            double acc = 0.0;
+            for (int i = 0; i < Dk; ++i) acc += kb[i] * Hs[(size_t)i * Dv + j];
+            kS[j] = be * (vr[j] - a * acc);
+        }
+        for (int i = 0; i < Dk; ++i)
+            for (int j = 0; j < Dv; ++j) Hs[(size_t)i * Dv + j] = a * Hs[(size_t)i * Dv + j] + kb[i] * kS[j];
+        double *orow = J->o + r * Dv;
+        for (int j = 0; j < Dv; ++j) {
+            double acc = 0.0;
+            for (int i = 0; i < Dk; ++i) acc += Hs[(size_t)i * Dv + j] * qcl[i];
+            orow[j] = J->scale * acc;
+        }
+    }
+    if (J->ST) memcpy(J->ST + bh * Dk * Dv, Hs, sizeof(double) * Dk * Dv);
+    if (J->CT) memcpy(J->CT + bh * Dk * Dk, Cg, sizeof(double) * Dk * Dk);
+    if (J->mT) memcpy(J->mT + bh * Dk, mg, sizeof(double) * Dk);
+    if (J->nT) J->nT[bh] = n;
+    free(Hs); free(Cg); free(mg); free(qb); free(kb); free(sg); free(qcl); free(kS);
+}
+
+static void *dworker(void *arg) {
+    djob_t *J = (djob_t *)arg;
+    for (;;) {
+        pthread_mutex_lock(&J->mu);
+        const int w = J->next++;
+        pthread_mutex_unlock(&J->mu);
+        if (w >= J->B * J->H) break;
+        decayed_pair(J, w / J->H, w % J->H);
+    }
+    return NULL;
+}
+
+/*
+ * Gated DeltaNet forward with the decay-aligned covariance (reading above).  Arguments as
+ * ccq_oracle_forward for the Gated DeltaNet backbone, except that the position count is
+ * replaced by the decayed count: n0 [B,H] (NULL = 0) in, nT [B,H] out (may be NULL).
+ * Returns 0, or -1 on a bad argument.
+ */
+int ccq_oracle_gdn_forward_decayed(int B, int T, int H, int Dk, int Dv, const double *q, const double *k,
+                                   const double *v, const double *g, const double *beta,
+                                   const double *lam, const double *S0, const double *C0,
+                                   const double *m0, const double *n0, double *o, double *ST,
+                                   double *CT, double *mT, double *nT, double *qc_out, int l2norm,
+                                   int centered, double scale, int nthreads) {
+    if (B < 0 || T < 0 || H < 0 || Dk <= 0 || Dv <= 0 || nthreads < 1) return -1;
+    if (!q || !k || !v || !g || !beta || !lam || !o) return -1;
+    djob_t J;
+    memset(&J, 0, sizeof J);
+    J.B = B; J.T = T; J.H = H; J.Dk = Dk; J.Dv = Dv; J.l2norm = l2norm; J.centered = centered;
+    J.scale = scale;
+    J.q = q; J.k = k; J.v = v; J.g = g; J.beta = beta; J.lam = lam;
+    J.S0 = S0; J.C0 = C0; J.m0 = m0; J.n0 = n0;
+    J.o = o; J.ST = ST; J.CT = CT; J.mT = mT; J.nT = nT; J.qc_out = qc_out;
+    pthread_mutex_init(&J.mu, NULL);
+    if (nthreads > B * H) nthreads = B * H > 0 ? B * H : 1;
+    pthread_t *th = malloc(sizeof(pthread_t) * (size_t)nthreads);
+    for (int i = 0; i < nthreads; ++i) pthread_create(&th[i], NULL, dworker, &J);
+    for (int i = 0; i < nthreads; ++i) pthread_join(th[i], NULL);
+    free(th);
+    pthread_mutex_destroy(&J.mu);
+    return 0;
+}
+
 /* ====================================================================== reverse mode
  *
  * Gradients of the CCQ-GLA forward (recurrent form above) with respect to every

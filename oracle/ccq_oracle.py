@@ -56,6 +56,10 @@ def load_library(path: str):
         [ctypes.c_int] * 5 + [dp] * 9 + [ip] + [dp] * 4 + [dp] * 9
         + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int])
     lib.ccq_oracle_gdn_backward.restype = ctypes.c_int
+    lib.ccq_oracle_gdn_forward_decayed.argtypes = (
+        [ctypes.c_int] * 5 + [dp] * 10 + [dp] * 6
+        + [ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int])
+    lib.ccq_oracle_gdn_forward_decayed.restype = ctypes.c_int
     return lib
 
 
@@ -209,3 +213,33 @@ def gdn_backward(q, k, v, g, beta, lam, dout, S0=None, C0=None, m0=None, t0=None
     if rc != 0:
         raise ValueError("ccq_oracle_gdn_backward rejected its arguments")
     return r
+
+
+def gdn_forward_decayed(q, k, v, g, beta, lam, S0=None, C0=None, m0=None, n0=None, *, l2norm=True,
+                        centered=True, scale=None, want_qclean=False, nthreads=None, lib=None):
+    """CCQ-Gated-DeltaNet forward with the decay-aligned covariance: the running statistics
+    decay with the backbone's own scalar decay and are normalised by the decayed count n
+    (the reading stated in ccq_oracle.c).  q, k [B,T,H,Dk]; v [B,T,H,Dv]; g, beta, lam
+    [B,T,H]; S0 [B,H,Dk,Dv], C0 [B,H,Dk,Dk], m0 [B,H,Dk], n0 [B,H] (None = zero).
+    Returns dict o, S, C, m, n (and qclean when asked)."""
+    lib = lib or _load()
+    q, k, v, g, beta, lam = map(_f64, (q, k, v, g, beta, lam))
+    S0, C0, m0, n0 = map(_f64, (S0, C0, m0, n0))
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    if scale is None:
+        scale = Dk ** -0.5
+    if nthreads is None:
+        nthreads = os.cpu_count() or 1
+    out = {"o": np.zeros((B, T, H, Dv)), "S": np.zeros((B, H, Dk, Dv)), "C": np.zeros((B, H, Dk, Dk)),
+           "m": np.zeros((B, H, Dk)), "n": np.zeros((B, H))}
+    qc = np.zeros((B, T, H, Dk)) if want_qclean else None
+    rc = lib.ccq_oracle_gdn_forward_decayed(
+        B, T, H, Dk, Dv, _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _ptr(S0),
+        _ptr(C0), _ptr(m0), _ptr(n0), _ptr(out["o"]), _ptr(out["S"]), _ptr(out["C"]), _ptr(out["m"]),
+        _ptr(out["n"]), _ptr(qc), int(bool(l2norm)), int(bool(centered)), float(scale), int(nthreads))
+    if rc != 0:
+        raise ValueError("ccq_oracle_gdn_forward_decayed rejected its arguments")
+    if want_qclean:
+        out["qclean"] = qc
+    return out
