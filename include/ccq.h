@@ -232,6 +232,37 @@ CCQ_API ccq_status ccq_gla_bwd_workspace_size(int B, int T, int H, int Dk, int D
                                               int with_ckpt, const ccq_params *p, size_t *bytes);
 
 /*
+ * CCQ-Gated-DeltaNet backward: the gradients of a scalar loss L through ccq_gdn_fwd,
+ * given dL/do and (optionally) dL/d(final states).  The paper gives no backward; this is
+ * the reverse mode of Eqs. clean/read, the running sums of Sec. 3.2 and the gated delta
+ * rule, chunked like Algorithm 1 (only the state adjoint crosses chunks sequentially).
+ *   q, k, v, g, beta, lambda, in_dtype, S0/C0/m0/t0   the forward's inputs.
+ *   dout      dL/do [B,T,H,Dv] in in_dtype.
+ *   dST [B,H,Dk,Dv], dCT [B,H,Dk,Dk], dmT [B,H,Dk] fp32: dL/d(ST, CT, mT); NULL = 0.
+ *   dq, dk    [B,T,H,Dk], dv [B,T,H,Dv] in in_dtype: gradients of q, k, v (the raw,
+ *             un-normalised q and k when l2norm_qk = 1).
+ *   dg, dbeta [B,T,H] fp32: gradients of the log decay and of beta.
+ *   dlambda   [B,T,H] fp32 (may be NULL);  dS0, dC0, dm0 fp32 (each may be NULL).
+ *   workspace at least ccq_gdn_bwd_workspace_size() bytes (16-byte aligned): per
+ *             64-token chunk of every (sequence, head), the chunk's forward states,
+ *             state adjoints and intermediate tiles in fp32.
+ * Supported: Dk = Dv in {64, 128}, bf16 or fp32 inputs; the kernels compute in fp32 on
+ * the CUDA cores (seven launches; the algo parameter is ignored).  T = 0 copies the
+ * final-state gradients to the initial-state ones.
+ */
+CCQ_API ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float *g,
+                               const float *beta, const float *lambda, ccq_dtype in_dtype,
+                               const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                               const void *dout, const float *dST, const float *dCT, const float *dmT,
+                               void *dq, void *dk, void *dv, float *dg, float *dbeta, float *dlambda,
+                               float *dS0, float *dC0, float *dm0, int B, int T, int H, int Dk, int Dv,
+                               void *workspace, size_t workspace_bytes, const ccq_params *p, void *stream);
+
+/* Workspace bytes ccq_gdn_bwd needs for these sizes (0 when T = 0).  Host-only. */
+CCQ_API ccq_status ccq_gdn_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                              const ccq_params *p, size_t *bytes);
+
+/*
  * ccq_gla_fwd for callers that cannot supply any device memory of their own --
  * for instance an engine that gave all device memory to its own caches at
  * start-up, or code on a path where allocating is not allowed or would stall

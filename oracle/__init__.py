@@ -16,8 +16,8 @@ Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``)
   gla_backward       reverse mode of the CCQ-GLA forward -- pinned by central
                      finite differences of the forward (fp64).
   gdn_backward       reverse mode of the CCQ-Gated-DeltaNet forward -- pinned the
-                     same way (tests/test_oracle_backward_gdn.py); no GPU path
-                     consumes it yet.
+                     same way (tests/test_oracle_backward_gdn.py) and by a chunkwise
+                     adjoint; the reference of the ccq_gdn_bwd parity tests.
   gdn_forward_decayed  CCQ-Gated-DeltaNet with the decay-aligned covariance (a reading of
                      the paper's future-work variant, stated in ccq_oracle.c) -- pinned
                      by brute-force weighted covariances, the undecayed special case,

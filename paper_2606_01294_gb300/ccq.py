@@ -90,6 +90,14 @@ def load_library() -> ctypes.CDLL:
         lib.ccq_gla_bwd_workspace_size.argtypes = ([_I] * 7 + [ctypes.POINTER(_Params),
                                                                ctypes.POINTER(ctypes.c_size_t)])
         lib.ccq_gla_bwd_workspace_size.restype = _I
+        # q, k, v, g, beta, lambda | in_dtype | S0, C0, m0, t0, dout, dST, dCT, dmT, dq, dk, dv,
+        # dg, dbeta, dlambda, dS0, dC0, dm0 | B, T, H, Dk, Dv | workspace, bytes, params, stream
+        lib.ccq_gdn_bwd.argtypes = ([_VP] * 6 + [_I] + [_VP] * 17 + [_I] * 5
+                                    + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
+        lib.ccq_gdn_bwd.restype = _I
+        lib.ccq_gdn_bwd_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
+                                                               ctypes.POINTER(ctypes.c_size_t)])
+        lib.ccq_gdn_bwd_workspace_size.restype = _I
         _lib = lib
     return _lib
 
@@ -379,6 +387,59 @@ def gdn_fwd(q, k, v, g, beta, lam, state: Optional[CCQState] = None, *, out=None
         ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
+
+
+def gdn_bwd(q, k, v, g, beta, lam, dout, state: Optional[CCQState] = None, *, dST=None, dCT=None,
+            dmT=None, out: Optional[dict] = None, workspace=None, stream=None, **kw):
+    """CCQ-Gated-DeltaNet backward.  Returns a dict of gradients dq, dk, dv (q's dtype),
+    dg, dbeta, dlambda [B,T,H] and dS0, dC0, dm0 (fp32).  ``dST``/``dCT``/``dmT`` are the
+    gradients of the final states (None = 0).  ``out`` may hold preallocated tensors under
+    those names; ``workspace`` (a CUDA byte tensor of at least
+    ccq_gdn_bwd_workspace_size bytes) is allocated on the fly when not given."""
+    dev = q.device
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, T, H, Dv))
+    _req(g, "g", dev, torch.float32, (B, T, H))
+    _req(beta, "beta", dev, torch.float32, (B, T, H))
+    _req(lam, "lam", dev, torch.float32, (B, T, H))
+    _req(dout, "dout", dev, q.dtype, (B, T, H, Dv))
+    S0, C0, m0, t0 = _state_in(state, B, H, Dk, Dv, dev)
+    if dST is not None:
+        _req(dST, "dST", dev, torch.float32, (B, H, Dk, Dv))
+    if dCT is not None:
+        _req(dCT, "dCT", dev, torch.float32, (B, H, Dk, Dk))
+    if dmT is not None:
+        _req(dmT, "dmT", dev, torch.float32, (B, H, Dk))
+    grads = dict(out or {})
+    shapes = {"dq": ((B, T, H, Dk), q.dtype), "dk": ((B, T, H, Dk), q.dtype),
+              "dv": ((B, T, H, Dv), q.dtype), "dg": ((B, T, H), torch.float32),
+              "dbeta": ((B, T, H), torch.float32), "dlambda": ((B, T, H), torch.float32),
+              "dS0": ((B, H, Dk, Dv), torch.float32), "dC0": ((B, H, Dk, Dk), torch.float32),
+              "dm0": ((B, H, Dk), torch.float32)}
+    for name, (shape, dt) in shapes.items():
+        if grads.get(name) is None:
+            grads[name] = torch.empty(shape, dtype=dt, device=dev)
+        _req(grads[name], name, dev, dt, shape)
+    p = params(**kw)
+    lib = load_library()
+    need = ctypes.c_size_t(0)
+    _check(lib.ccq_gdn_bwd_workspace_size(B, T, H, Dk, Dv, _dtype_code(q), ctypes.byref(p),
+                                          ctypes.byref(need)))
+    if workspace is None and need.value:
+        workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_gdn_bwd(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _dtype_code(q),
+        _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(dout), _ptr(dST), _ptr(dCT), _ptr(dmT),
+        _ptr(grads["dq"]), _ptr(grads["dk"]), _ptr(grads["dv"]), _ptr(grads["dg"]),
+        _ptr(grads["dbeta"]), _ptr(grads["dlambda"]), _ptr(grads["dS0"]), _ptr(grads["dC0"]),
+        _ptr(grads["dm0"]), B, T, H, Dk, Dv, _ptr(workspace), ws_bytes, ctypes.byref(p),
+        _stream(dev, stream))
+    _check(st)
+    return grads
 
 
 def gla_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):

@@ -12,6 +12,7 @@
 #include <initializer_list>
 
 #include "../../include/ccq.h"
+#include "ccq_gdn_bwd.h"
 #include "ccq_internal.h"
 
 namespace ccq {
@@ -565,6 +566,71 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
     ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT;
     st = run_recurrent(ra, static_cast<cudaStream_t>(stream));
     return st != CCQ_OK ? st : finish_t(t0, tT, B, T, static_cast<cudaStream_t>(stream));
+}
+
+// Copies the final-state gradients to the initial-state ones (zero where a final one is NULL):
+// the backward of a call with no tokens.
+static ccq_status copy_state_grads(const float *dST, const float *dCT, const float *dmT, float *dS0, float *dC0,
+                                   float *dm0, int B, int H, int Dk, int Dv, cudaStream_t s) {
+    const size_t n[3] = {static_cast<size_t>(B) * H * Dk * Dv * 4, static_cast<size_t>(B) * H * Dk * Dk * 4,
+                         static_cast<size_t>(B) * H * Dk * 4};
+    float *dst[3] = {dS0, dC0, dm0};
+    const float *src[3] = {dST, dCT, dmT};
+    for (int i = 0; i < 3; ++i) {
+        if (!dst[i]) continue;
+        cudaError_t e = src[i] ? cudaMemcpyAsync(dst[i], src[i], n[i], cudaMemcpyDeviceToDevice, s)
+                               : cudaMemsetAsync(dst[i], 0, n[i], s);
+        if (e != cudaSuccess) return cuda_fail(e, "state gradient copy");
+    }
+    return CCQ_OK;
+}
+
+ccq_status ccq_gdn_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                      const ccq_params *p, size_t *bytes) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    *bytes = T > 0 ? gdn_bwd_workspace_bytes(B, T, H, Dk) : 0;
+    return CCQ_OK;
+}
+
+ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float *g, const float *beta,
+                       const float *lambda, ccq_dtype in_dtype, const float *S0, const float *C0,
+                       const float *m0, const int64_t *t0, const void *dout, const float *dST,
+                       const float *dCT, const float *dmT, void *dq, void *dk, void *dv, float *dg,
+                       float *dbeta, float *dlambda, float *dS0, float *dC0, float *dm0, int B, int T,
+                       int H, int Dk, int Dv, void *workspace, size_t workspace_bytes,
+                       const ccq_params *p, void *stream) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    st = check_ptrs("", {}, {S0, C0, m0, t0, dST, dCT, dmT, dlambda, dS0, dC0, dm0});
+    if (st != CCQ_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) return copy_state_grads(dST, dCT, dmT, dS0, dC0, dm0, B, H, Dk, Dv, s);
+    st = check_ptrs("q,k,v,g,beta,lambda,dout,dq,dk,dv,dg,dbeta",
+                    {q, k, v, g, beta, lambda, dout, dq, dk, dv, dg, dbeta}, {});
+    if (st != CCQ_OK) return st;
+    const size_t need = gdn_bwd_workspace_bytes(B, T, H, Dk);
+    if (!workspace || workspace_bytes < need)
+        return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
+                    workspace ? workspace_bytes : static_cast<size_t>(0));
+    if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+    GdnBwdCall a = {};
+    a.B = B; a.T = T; a.H = H; a.D = Dk; a.bf16 = in_dtype == CCQ_BF16;
+    a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
+    a.q = q; a.k = k; a.v = v; a.dout = dout;
+    a.g = g; a.beta = beta; a.lambda = lambda; a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
+    a.dST = dST; a.dCT = dCT; a.dmT = dmT;
+    a.dq = dq; a.dk = dk; a.dv = dv; a.dg = dg; a.dbeta = dbeta; a.dlambda = dlambda;
+    a.dS0 = dS0; a.dC0 = dC0; a.dm0 = dm0;
+    a.workspace = workspace;
+    cudaError_t e = launch_gdn_bwd(a, s);
+    if (e != cudaSuccess) return cuda_fail(e, "Gated DeltaNet backward launch");
+    return CCQ_OK;
 }
 
 ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,

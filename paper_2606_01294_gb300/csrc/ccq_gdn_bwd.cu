@@ -1,0 +1,78 @@
+// ccq_gdn_bwd.cu -- launches of the CUDA-core CCQ-Gated-DeltaNet backward
+// (kernels and the adjoint they evaluate: ccq_gdn_bwd_kernels.cuh).
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ccq_gdn_bwd_kernels.cuh"
+#include "ccq_gdn_bwd.h"
+
+namespace ccq {
+
+namespace {
+
+// Workspace floats per chunk (layout of gbwd::GdnBwdArgs): Tt, S^K_r, M_r, H_r, dH, DC, Dm,
+// P^T D, (diag(E) Qc)^T D, qbar, qc, U, R, W and the row vectors.
+size_t per_chunk_floats(int D) {
+    const size_t d = static_cast<size_t>(D);
+    return 64 * 64 + 5 * d * d + 2 * d + 6 * 64 * d + 4 * 64;
+}
+
+template <typename K>
+cudaError_t allow_smem(K kernel, size_t bytes) {
+    return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+}
+
+template <int D, typename Tin>
+cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
+    using namespace gbwd;
+    cudaError_t e;
+    if ((e = allow_smem(gdn_bwd_prep_kernel<D, Tin>, prep_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_fstate_kernel<D, Tin>, fstate_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_local_kernel<D, Tin>, local_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_dstate_kernel<D, Tin>, dstate_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_kv_kernel<D, Tin>, kv_smem<D>())) != cudaSuccess) return e;
+    const unsigned nch = static_cast<unsigned>(a.B * a.H * a.NC), bh = static_cast<unsigned>(a.B * a.H);
+    const long long elems = (static_cast<long long>(D) * D + D) * a.B * a.H;
+    const unsigned eblocks = static_cast<unsigned>((elems + 255) / 256);
+    gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
+    gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
+    gdn_bwd_fstate_kernel<D, Tin><<<bh, 512, fstate_smem<D>(), s>>>(a);
+    gdn_bwd_local_kernel<D, Tin><<<nch, 256, local_smem<D>(), s>>>(a);
+    gdn_bwd_dstate_kernel<D, Tin><<<bh, 512, dstate_smem<D>(), s>>>(a);
+    gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
+    gdn_bwd_kv_kernel<D, Tin><<<nch, 256, kv_smem<D>(), s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D) {
+    const size_t chunks = static_cast<size_t>(B) * H * ((T + 63) / 64);
+    return chunks * per_chunk_floats(D) * sizeof(float);
+}
+
+cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s) {
+    gbwd::GdnBwdArgs a{};
+    a.B = c.B; a.T = c.T; a.H = c.H; a.NC = (c.T + 63) / 64;
+    a.l2norm = c.l2norm; a.centered = c.centered; a.scale = c.scale;
+    a.q = c.q; a.k = c.k; a.v = c.v; a.dout = c.dout;
+    a.g = c.g; a.beta = c.beta; a.lambda = c.lambda;
+    a.S0 = c.S0; a.C0 = c.C0; a.m0 = c.m0; a.t0 = c.t0;
+    a.dST = c.dST; a.dCT = c.dCT; a.dmT = c.dmT;
+    a.dq = c.dq; a.dk = c.dk; a.dv = c.dv;
+    a.dg = c.dg; a.dbeta = c.dbeta; a.dlambda = c.dlambda;
+    a.dS0 = c.dS0; a.dC0 = c.dC0; a.dm0 = c.dm0;
+    const size_t chunks = static_cast<size_t>(c.B) * c.H * a.NC;
+    const size_t d = static_cast<size_t>(c.D);
+    float *p = static_cast<float *>(c.workspace);
+    auto take = [&](size_t per) { float *r = p; p += chunks * per; return r; };
+    a.tt = take(64 * 64); a.sk = take(d * d); a.mk = take(d); a.hs = take(d * d); a.dh = take(d * d);
+    a.dc = take(d * d); a.dm = take(d); a.x1 = take(64 * d); a.y1 = take(d * d);
+    a.qb = take(64 * d); a.qc = take(64 * d); a.u = take(64 * d); a.r = take(64 * d); a.w = take(64 * d);
+    a.vec = take(4 * 64);
+    if (c.D == 128) return c.bf16 ? run<128, __nv_bfloat16>(a, s) : run<128, float>(a, s);
+    if (c.D == 64) return c.bf16 ? run<64, __nv_bfloat16>(a, s) : run<64, float>(a, s);
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace ccq

@@ -1,0 +1,28 @@
+// ccq_gdn_bwd.h -- launch interface of the CUDA-core CCQ-Gated-DeltaNet backward
+// (ccq_gdn_bwd.cu), used by the C ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace ccq {
+
+// Arguments of the CUDA-core CCQ-Gated-DeltaNet backward (ccq_gdn_bwd.cu): the C ABI's
+// pointers as given (token tensors [B][T][H][D] in bf16 or fp32, D = Dk = Dv) and a
+// caller workspace of gdn_bwd_workspace_bytes() bytes.
+struct GdnBwdCall {
+    int B, T, H, D, bf16, l2norm, centered;
+    float scale;
+    const void *q, *k, *v, *dout;
+    const float *g, *beta, *lambda, *S0, *C0, *m0;
+    const int64_t *t0;
+    const float *dST, *dCT, *dmT;
+    void *dq, *dk, *dv;
+    float *dg, *dbeta, *dlambda, *dS0, *dC0, *dm0;
+    void *workspace;
+};
+size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D);
+cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s);
+
+}  // namespace ccq

@@ -1,0 +1,876 @@
+// ccq_gdn_bwd_kernels.cuh -- CCQ-Gated-DeltaNet backward, CUDA-core kernels (fp32 arithmetic).
+//
+// Reverse mode of the CCQ read (Eq. clean, Eq. read, the undecayed running sums of Sec. 3.2)
+// with the Gated DeltaNet write as the backbone, chunked as Algorithm 1 chunks the forward.
+// The paper gives no backward; the adjoint below is the reverse mode of the chunk map
+//
+//   A  = strict_lower(diag(beta) (Kbar Kbar^T) o Gamma),  Gamma_ij = e^{gc_i - gc_j},
+//   Tt = (I + A)^{-1},  Tb = Tt diag(beta),  R = V - diag(E) Kbar H,  U = Tb R,  E_i = e^{gc_i}
+//   O  = scale (diag(E) Qc H + P U),  P = (Qc Kbar^T) o Gamma o causal
+//   H' = e^{gc_last} H + Kd^T U,  Kd = diag(e^{gc_last - gc}) Kbar
+//
+// (gc the in-chunk cumulative log decay, H the state entering the chunk with key dims as
+// rows), with the CCQ contraction qc = qbar - lambda z, z = Sigma_t qbar.  Given the
+// adjoint dH of H' and D = scale dO, per chunk:
+//   dU  = P^T D + Kd dH,       dv = dR = Tb^T dU
+//   dP  = (D U^T) o Gamma o causal,   dqc = diag(E) D H^T + dP Kbar
+//   dH_enter = e^{gc_last} dH + (diag(E) Qc)^T D - (diag(E) Kbar)^T dR
+//   dTb = dU R^T,  dbeta_j = sum_i dTb_ij Tt_ij + sum_l dA_jl Gamma_jl KK_jl,
+//   dA  = strict_lower(-Tt^T (dTb diag(beta)) Tt^T),  dKK = diag(beta) (dA o Gamma)
+//   dkbar = dP^T Qc + diag(e^{gc_last - gc}) U dH^T - diag(E) dR H^T + (dKK + dKK^T) Kbar
+//           + the CCQ terms (as in the GLA backward)
+//   dgc = rowsum - colsum of (dA o A) and (dP o S) + E o rowsum((Qc H) o D)
+//         - rowsum(Kd o U dH^T) - E o rowsum((Kbar H) o dR),
+//         plus e^{gc_last} <dH, H> + sum_i rowsum(Kd o U dH^T)_i at the last row;
+//   dg  = the in-chunk reverse cumulative sum of dgc.
+// Only dH crosses chunks sequentially: the CCQ adjoints DC, Dm are sums of chunk-local
+// terms.  So the backward is seven launches:
+//   gdn_bwd_prep_kernel    per chunk: Tt and the chunk's key statistics (Kbar^T Kbar, sum Kbar)
+//   gdn_bwd_prefix_kernel  exclusive prefix of the key statistics over chunks (S^K_r, M_r)
+//   gdn_bwd_fstate_kernel  per sequence and head, chunks in order: the entering states H_r
+//   gdn_bwd_local_kernel   per chunk: z, qc, R, U, dqc, dq, dlambda, the CCQ increments of
+//                          DC and Dm, and P^T D, (diag(E) Qc)^T D for the state pass
+//   gdn_bwd_dstate_kernel  per sequence and head, chunks last to first: dH at every chunk end
+//   gdn_bwd_suffix_kernel  exclusive suffix of the DC, Dm increments (DC_{r+1}, Dm_{r+1})
+//   gdn_bwd_kv_kernel      per chunk: dv, dk, dbeta, dg
+//
+// Every kernel is a sequence of phases separated by __syncthreads(); inside a phase each
+// thread strides over the elements it owns and reads only what earlier phases wrote (row
+// reductions go through shared-memory atomics).  Arithmetic is fp32 on the CUDA cores.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace ccq {
+namespace gbwd {
+
+constexpr int kC = 64;  // chunk length
+
+#define GBWD_FOR(i, n) for (int i = static_cast<int>(threadIdx.x); i < (n); i += static_cast<int>(blockDim.x))
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f<__nv_bfloat16>(float x) { return __float2bfloat16_rn(x); }
+
+// Kernel arguments.  Token tensors are [B][T][H][D]; g, beta, lambda [B][T][H] fp32.
+// The workspace arrays are indexed by the chunk ch = (b*H + h)*NC + r.
+struct GdnBwdArgs {
+    int B, T, H, NC;
+    int l2norm, centered;
+    float scale;
+    const void *q, *k, *v, *dout;
+    const float *g, *beta, *lambda;
+    const float *S0, *C0, *m0;  // may be NULL (zero)
+    const int64_t *t0;          // may be NULL (zero)
+    const float *dST, *dCT, *dmT;  // may be NULL (zero)
+    void *dq, *dk, *dv;
+    float *dg, *dbeta, *dlambda;   // dlambda may be NULL
+    float *dS0, *dC0, *dm0;        // each may be NULL
+    // workspace, per chunk
+    float *tt;   // [64][64] Tt
+    float *sk;   // [D][D]   chunk's Kbar^T Kbar, then S^K_r
+    float *mk;   // [D]      chunk's sum Kbar, then M_r
+    float *hs;   // [D][D]   H_r (the state entering the chunk)
+    float *dh;   // [D][D]   adjoint of H_{r+1} (the state leaving the chunk)
+    float *dc;   // [D][D]   chunk's increment of DC, then DC_{r+1}
+    float *dm;   // [D]      chunk's increment of Dm, then Dm_{r+1}
+    float *x1;   // [64][D]  P^T D
+    float *y1;   // [D][D]   (diag(E) Qc)^T D
+    float *qb, *qc, *u, *r, *w;  // [64][D] each: qbar, qc, U, R, W = dz / t
+    float *vec;  // [4][64]  cq, cz, E o rowsum((Qc H) o D), spare
+};
+
+__device__ __forceinline__ size_t tok_row(const GdnBwdArgs &a, int b, int t, int h) {
+    return (static_cast<size_t>(b) * a.T + t) * a.H + h;
+}
+
+// Load the rows of chunk r of a [B][T][H][D] tensor into dst[64][D] (zero past T).
+template <int D, typename Tin>
+__device__ __forceinline__ void load_tile(float *dst, const void *src, const GdnBwdArgs &a, int b, int h, int r) {
+    const Tin *s = static_cast<const Tin *>(src);
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, c = idx % D, t = r * kC + i;
+        dst[idx] = t < a.T ? to_f(s[tok_row(a, b, t, h) * D + c]) : 0.f;
+    }
+}
+
+// Per-row inverse norms (phase) of a [64][D] tile: 1/max(|x|, 1e-6), 0 for an all-zero row
+// (which normalises to itself and passes no gradient), or 1 when disabled.
+template <int D>
+__device__ __forceinline__ void row_rnorm(const float *x, float *rn, int l2norm) {
+    GBWD_FOR(i, kC) {
+        float ss = 0.f;
+        for (int c = 0; c < D; ++c) ss += x[i * D + c] * x[i * D + c];
+        rn[i] = !l2norm ? 1.f : (ss > 0.f ? 1.f / sqrtf(fmaxf(ss, 1e-12f)) : 0.f);
+    }
+}
+
+// Gate scalars (phase, one thread): in-chunk cumulative log decay of the first n rows,
+// held constant past them.
+__device__ __forceinline__ void gate_prefix(const float *graw, float *gc) {
+    if (threadIdx.x == 0) {
+        float acc = 0.f;
+        for (int i = 0; i < kC; ++i) {
+            acc += graw[i];
+            gc[i] = acc;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------------
+// Per chunk: Tt = (I + A)^{-1} by forward substitution, and the chunk's key statistics.
+template <int D, typename Tin>
+__global__ void __launch_bounds__(256) gdn_bwd_prep_kernel(const GdnBwdArgs a) {
+    extern __shared__ float4 gbwd_smem4[];
+    float *sm = reinterpret_cast<float *>(gbwd_smem4);
+    float *Kb = sm;                // [64][D]
+    float *A = Kb + kC * D;        // [64][64]
+    float *Tt = A + kC * kC;       // [64][64]
+    float *graw = Tt + kC * kC;    // [64]
+    float *gc = graw + kC;
+    float *be = gc + kC;
+    float *rk = be + kC;
+
+    const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
+    load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+    GBWD_FOR(i, kC) {
+        const int t = r * kC + i;
+        const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
+        graw[i] = t < a.T ? a.g[row] : 0.f;
+        be[i] = t < a.T ? a.beta[row] : 0.f;
+    }
+    __syncthreads();
+    row_rnorm<D>(Kb, rk, a.l2norm);
+    gate_prefix(graw, gc);
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+    __syncthreads();
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float v = 0.f;
+        if (j < i) {
+            float kk = 0.f;
+            for (int c = 0; c < D; ++c) kk += Kb[i * D + c] * Kb[j * D + c];
+            v = be[i] * expf(gc[i] - gc[j]) * kk;
+        }
+        A[idx] = v;
+    }
+    __syncthreads();
+    // (I + A) Tt = I with A strictly lower: row i of Tt needs rows 0..i-1.
+    for (int i = 0; i < kC; ++i) {
+        GBWD_FOR(j, kC) {
+            float v = i == j ? 1.f : 0.f;
+            for (int l = j; l < i; ++l) v -= A[i * kC + l] * Tt[l * kC + j];
+            Tt[i * kC + j] = v;
+        }
+        __syncthreads();
+    }
+    float *tt = a.tt + static_cast<size_t>(ch) * kC * kC;
+    GBWD_FOR(idx, kC * kC) tt[idx] = Tt[idx];
+    float *sk = a.sk + static_cast<size_t>(ch) * D * D;
+    GBWD_FOR(idx, D * D) {
+        const int p = idx / D, c = idx % D;
+        float acc = 0.f;
+        for (int i = 0; i < kC; ++i) acc += Kb[i * D + p] * Kb[i * D + c];
+        sk[idx] = acc;
+    }
+    float *mk = a.mk + static_cast<size_t>(ch) * D;
+    GBWD_FOR(c, D) {
+        float acc = 0.f;
+        for (int i = 0; i < kC; ++i) acc += Kb[i * D + c];
+        mk[c] = acc;
+    }
+}
+
+// Exclusive prefix over the chunks of each sequence and head: sk[r] <- C0 + sum_{s<r} sk[s],
+// mk[r] <- m0 + sum_{s<r} mk[s].  One thread per (sequence-head, element).
+template <int D>
+__global__ void __launch_bounds__(256) gdn_bwd_prefix_kernel(const GdnBwdArgs a) {
+    const long long per = static_cast<long long>(D) * D + D;
+    const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (gid >= per * a.B * a.H) return;
+    const int bh = static_cast<int>(gid / per);
+    const int e = static_cast<int>(gid % per);
+    const bool isC = e < D * D;
+    float *base = isC ? a.sk + static_cast<size_t>(bh) * a.NC * D * D + e
+                      : a.mk + static_cast<size_t>(bh) * a.NC * D + (e - D * D);
+    const size_t stride = isC ? static_cast<size_t>(D) * D : static_cast<size_t>(D);
+    float acc = 0.f;
+    if (isC && a.C0) acc = a.C0[static_cast<size_t>(bh) * D * D + e];
+    if (!isC && a.m0) acc = a.m0[static_cast<size_t>(bh) * D + (e - D * D)];
+    for (int r = 0; r < a.NC; ++r) {
+        const float x = base[r * stride];
+        base[r * stride] = acc;
+        acc += x;
+    }
+}
+
+// Per sequence and head, chunks in order: the state entering every chunk.
+template <int D, typename Tin>
+__global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a) {
+    extern __shared__ float4 gbwd_smem4[];
+    float *sm = reinterpret_cast<float *>(gbwd_smem4);
+    float *Hs = sm;               // [D][D]
+    float *Kb = Hs + D * D;       // [64][D]
+    float *R = Kb + kC * D;       // [64][D]
+    float *U = R + kC * D;        // [64][D]
+    float *Tt = U + kC * D;       // [64][64]
+    float *graw = Tt + kC * kC;   // [64]
+    float *gc = graw + kC, *be = gc + kC, *rk = be + kC, *E = rk + kC, *ed = E + kC;
+
+    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    GBWD_FOR(idx, D * D) Hs[idx] = a.S0 ? a.S0[static_cast<size_t>(bh) * D * D + idx] : 0.f;
+    __syncthreads();
+    for (int r = 0; r < a.NC; ++r) {
+        const size_t ch = static_cast<size_t>(bh) * a.NC + r;
+        float *hs = a.hs + ch * D * D;
+        GBWD_FOR(idx, D * D) hs[idx] = Hs[idx];
+        load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+        load_tile<D, Tin>(R, a.v, a, b, h, r);
+        const float *tt = a.tt + ch * kC * kC;
+        GBWD_FOR(idx, kC * kC) Tt[idx] = tt[idx];
+        GBWD_FOR(i, kC) {
+            const int t = r * kC + i;
+            const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
+            graw[i] = t < a.T ? a.g[row] : 0.f;
+            be[i] = t < a.T ? a.beta[row] : 0.f;
+        }
+        __syncthreads();
+        row_rnorm<D>(Kb, rk, a.l2norm);
+        gate_prefix(graw, gc);
+        __syncthreads();
+        GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+        GBWD_FOR(i, kC) {
+            E[i] = expf(gc[i]);
+            ed[i] = expf(gc[kC - 1] - gc[i]);
+        }
+        __syncthreads();
+        // R = V - diag(E) Kbar H
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * Hs[l * D + j];
+            R[idx] -= E[i] * acc;
+        }
+        __syncthreads();
+        // U = Tt diag(beta) R
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * R[l * D + j];
+            U[idx] = acc;
+        }
+        __syncthreads();
+        // H <- e^{gc_last} H + Kd^T U
+        const float elast = expf(gc[kC - 1]);
+        GBWD_FOR(idx, D * D) {
+            const int l = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int i = 0; i < kC; ++i) acc += ed[i] * Kb[i * D + l] * U[i * D + j];
+            Hs[idx] = elast * Hs[idx] + acc;
+        }
+        __syncthreads();
+    }
+}
+
+// Per chunk, everything that does not need dH: z, qc, R, U, dqc, dq, dlambda, the CCQ
+// increments of DC and Dm, P^T D and (diag(E) Qc)^T D.
+template <int D, typename Tin>
+__global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) {
+    extern __shared__ float4 gbwd_smem4[];
+    float *sm = reinterpret_cast<float *>(gbwd_smem4);
+    float *Qb = sm;                // [64][D] qbar
+    float *Kb = Qb + kC * D;       // [64][D] kbar
+    float *Rq = Kb + kC * D;       // [64][D] V, then R, then qc
+    float *Zw = Rq + kC * D;       // [64][D] z, then W
+    float *Ud = Zw + kC * D;       // [64][D] U, then dqc, then dqbar
+    float *sA = Ud + kC * D;       // [64][64] (Qbar Kbar^T) o causal, then dP
+    float *sB = sA + kC * kC;      // [64][64] P, then (W Kbar^T) o causal
+    float *graw = sB + kC * kC;
+    float *gc = graw + kC, *E = gc + kC, *be = E + kC, *lam = be + kC, *tinv = lam + kC;
+    float *rq = tinv + kC, *rk = rq + kC, *cq = rk + kC, *cz = cq + kC, *gqh = cz + kC;
+    float *rdot = gqh + kC;
+
+    const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
+    const int n = min(kC, a.T - r * kC);
+    const float c = a.centered ? 1.f : 0.f;
+    const float *H = a.hs + static_cast<size_t>(ch) * D * D;
+    const float *SK = a.sk + static_cast<size_t>(ch) * D * D;
+    const float *M = a.mk + static_cast<size_t>(ch) * D;
+    const float *Tt = a.tt + static_cast<size_t>(ch) * kC * kC;
+    const Tin *dout = static_cast<const Tin *>(a.dout);
+    const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
+    auto Dsc = [&](int i, int col) -> float {
+        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + col]) : 0.f;
+    };
+
+    load_tile<D, Tin>(Qb, a.q, a, b, h, r);
+    load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+    load_tile<D, Tin>(Rq, a.v, a, b, h, r);
+    GBWD_FOR(i, kC) {
+        const int t = r * kC + i;
+        const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
+        graw[i] = i < n ? a.g[row] : 0.f;
+        be[i] = i < n ? a.beta[row] : 0.f;
+        lam[i] = i < n ? a.lambda[row] : 0.f;
+        tinv[i] = 1.f / (t_start + 1.f + static_cast<float>(i));
+        gqh[i] = 0.f;
+    }
+    __syncthreads();
+    row_rnorm<D>(Qb, rq, a.l2norm);
+    row_rnorm<D>(Kb, rk, a.l2norm);
+    gate_prefix(graw, gc);
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) {
+        Qb[idx] *= rq[idx / D];
+        Kb[idx] *= rk[idx / D];
+    }
+    GBWD_FOR(i, kC) E[i] = expf(gc[i]);
+    __syncthreads();
+    // (Qbar Kbar^T) o causal;  R = V - diag(E) Kbar H
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        if (j <= i)
+            for (int l = 0; l < D; ++l) acc += Qb[i * D + l] * Kb[j * D + l];
+        sA[idx] = acc;
+    }
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float acc = 0.f;
+        for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * H[l * D + j];
+        Rq[idx] -= E[i] * acc;
+    }
+    __syncthreads();
+    // cq_i = CumK_i . qbar_i with CumK_i = M + sum_{j<=i} kbar_j;  U = Tt diag(beta) R
+    GBWD_FOR(i, kC) {
+        float acc = 0.f;
+        for (int l = 0; l < D; ++l) acc += M[l] * Qb[i * D + l];
+        for (int j = 0; j <= i; ++j) acc += sA[i * kC + j];
+        cq[i] = acc;
+    }
+    {
+        float *Rg = a.r + static_cast<size_t>(ch) * kC * D;
+        float *Ug = a.u + static_cast<size_t>(ch) * kC * D;
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * Rq[l * D + j];
+            Ud[idx] = acc;
+            Ug[idx] = acc;
+            Rg[idx] = Rq[idx];
+        }
+    }
+    __syncthreads();
+    // z = Sigma_t qbar (App. B form): (Qbar S^K + ((Qbar Kbar^T) o causal) Kbar) / t - c CumK cq / t^2
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float acc = 0.f, cum = M[j];
+        for (int l = 0; l < D; ++l) acc += Qb[i * D + l] * SK[l * D + j];
+        for (int l = 0; l <= i; ++l) {
+            acc += sA[i * kC + l] * Kb[l * D + j];
+            cum += Kb[l * D + j];
+        }
+        Zw[idx] = acc * tinv[i] - c * cum * cq[i] * tinv[i] * tinv[i];
+    }
+    __syncthreads();
+    // qc = qbar - lambda z (Eq. clean)
+    {
+        float *Qg = a.qb + static_cast<size_t>(ch) * kC * D;
+        float *Qcg = a.qc + static_cast<size_t>(ch) * kC * D;
+        GBWD_FOR(idx, kC * D) {
+            const float v = Qb[idx] - lam[idx / D] * Zw[idx];
+            Rq[idx] = v;
+            Qcg[idx] = v;
+            Qg[idx] = Qb[idx];
+        }
+    }
+    __syncthreads();
+    // P = (Qc Kbar^T) o Gamma o causal
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        if (j <= i) {
+            for (int l = 0; l < D; ++l) acc += Rq[i * D + l] * Kb[j * D + l];
+            acc *= expf(gc[i] - gc[j]);
+        }
+        sB[idx] = acc;
+    }
+    __syncthreads();
+    // P^T D and (diag(E) Qc)^T D for the state pass;  dP = (D U^T) o Gamma o causal
+    {
+        float *X1 = a.x1 + static_cast<size_t>(ch) * kC * D;
+        float *Y1 = a.y1 + static_cast<size_t>(ch) * D * D;
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = i; l < n; ++l) acc += sB[l * kC + i] * Dsc(l, j);
+            X1[idx] = acc;
+        }
+        GBWD_FOR(idx, D * D) {
+            const int p = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int i = 0; i < n; ++i) acc += E[i] * Rq[i * D + p] * Dsc(i, j);
+            Y1[idx] = acc;
+        }
+        GBWD_FOR(idx, kC * kC) {
+            const int i = idx / kC, j = idx % kC;
+            float acc = 0.f;
+            if (j <= i && i < n) {
+                for (int l = 0; l < D; ++l) acc += Dsc(i, l) * Ud[j * D + l];
+                acc *= expf(gc[i] - gc[j]);
+            }
+            sA[idx] = acc;
+        }
+    }
+    __syncthreads();
+    // dqc = diag(E) D H^T + dP Kbar  (into Ud; U is no longer needed here);
+    // gqh_i = E_i rowsum((Qc H) o D)_i = E_i sum_j qc_ij (D H^T)_ij
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float dh = 0.f;
+        for (int l = 0; l < D; ++l) dh += Dsc(i, l) * H[j * D + l];
+        float acc = E[i] * dh;
+        for (int l = 0; l <= i; ++l) acc += sA[i * kC + l] * Kb[l * D + j];
+        Ud[idx] = acc;
+        if (i < n) atomicAdd(&gqh[i], E[i] * Rq[idx] * dh);
+    }
+    __syncthreads();
+    // dlambda_i = -z_i . dqc_i
+    GBWD_FOR(i, kC) {
+        float acc = 0.f;
+        for (int j = 0; j < D; ++j) acc += Zw[i * D + j] * Ud[i * D + j];
+        if (i < n && a.dlambda) a.dlambda[tok_row(a, b, r * kC + i, h)] = -acc;
+    }
+    __syncthreads();
+    // W = dz / t with dz = -lambda dqc
+    {
+        float *Wg = a.w + static_cast<size_t>(ch) * kC * D;
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D;
+            const float wv = -lam[i] * Ud[idx] * tinv[i];
+            Zw[idx] = wv;
+            Wg[idx] = wv;
+        }
+    }
+    __syncthreads();
+    // (W Kbar^T) o causal
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        if (j <= i)
+            for (int l = 0; l < D; ++l) acc += Zw[i * D + l] * Kb[j * D + l];
+        sB[idx] = acc;
+    }
+    __syncthreads();
+    // cz_i = CumK_i . dz_i = t_i (M . W_i + sum_{j<=i} W_i . kbar_j)
+    GBWD_FOR(i, kC) {
+        float acc = 0.f;
+        for (int l = 0; l < D; ++l) acc += M[l] * Zw[i * D + l];
+        for (int j = 0; j <= i; ++j) acc += sB[i * kC + j];
+        cz[i] = acc / tinv[i];
+    }
+    __syncthreads();
+    // dqbar = dqc + W S^K + ((W Kbar^T) o causal) Kbar - c CumK cz / t^2 (in place);
+    // the chunk's increments DC += W^T Qbar and Dm += sum_i dCum_i,
+    // dCum_i = -c (dz_i cq_i + qbar_i cz_i) / t_i^2
+    {
+        float *dC = a.dc + static_cast<size_t>(ch) * D * D;
+        float *dM = a.dm + static_cast<size_t>(ch) * D;
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f, cum = M[j];
+            for (int l = 0; l < D; ++l) acc += Zw[i * D + l] * SK[l * D + j];
+            for (int l = 0; l <= i; ++l) {
+                acc += sB[i * kC + l] * Kb[l * D + j];
+                cum += Kb[l * D + j];
+            }
+            Ud[idx] += acc - c * cum * cz[i] * tinv[i] * tinv[i];
+        }
+        GBWD_FOR(idx, D * D) {
+            const int p = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int i = 0; i < kC; ++i) acc += Zw[i * D + p] * Qb[i * D + j];
+            dC[idx] = acc;
+        }
+        GBWD_FOR(j, D) {
+            float acc = 0.f;
+            for (int i = 0; i < kC; ++i)
+                acc += (Zw[i * D + j] * cq[i] / tinv[i] + Qb[i * D + j] * cz[i]) * tinv[i] * tinv[i];
+            dM[j] = -c * acc;
+        }
+        float *vec = a.vec + static_cast<size_t>(ch) * 4 * kC;
+        GBWD_FOR(i, kC) {
+            vec[i] = cq[i];
+            vec[kC + i] = cz[i];
+            vec[2 * kC + i] = gqh[i];
+            vec[3 * kC + i] = 0.f;
+        }
+    }
+    __syncthreads();
+    GBWD_FOR(i, kC) {
+        float acc = 0.f;
+        for (int j = 0; j < D; ++j) acc += Qb[i * D + j] * Ud[i * D + j];
+        rdot[i] = a.l2norm ? acc : 0.f;
+    }
+    __syncthreads();
+    {
+        Tin *dq = static_cast<Tin *>(a.dq);
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            if (i < n) dq[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((Ud[idx] - Qb[idx] * rdot[i]) * rq[i]);
+        }
+    }
+}
+
+// Per sequence and head, chunks last to first: the adjoint dH of the state leaving every
+// chunk (stored), then carried into the chunk: dU = P^T D + Kd dH, dR = diag(beta) Tt^T dU,
+// dH <- e^{gc_last} dH + (diag(E) Qc)^T D - (diag(E) Kbar)^T dR.  Writes dS0.
+template <int D, typename Tin>
+__global__ void __launch_bounds__(512) gdn_bwd_dstate_kernel(const GdnBwdArgs a) {
+    extern __shared__ float4 gbwd_smem4[];
+    float *sm = reinterpret_cast<float *>(gbwd_smem4);
+    float *dH = sm;               // [D][D]
+    float *Kb = dH + D * D;       // [64][D]
+    float *dU = Kb + kC * D;      // [64][D]
+    float *dR = dU + kC * D;      // [64][D]
+    float *Tt = dR + kC * D;      // [64][64]
+    float *graw = Tt + kC * kC;   // [64]
+    float *gc = graw + kC, *be = gc + kC, *rk = be + kC, *E = rk + kC, *ed = E + kC;
+
+    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
+    GBWD_FOR(idx, D * D) dH[idx] = a.dST ? a.dST[static_cast<size_t>(bh) * D * D + idx] : 0.f;
+    __syncthreads();
+    for (int r = a.NC - 1; r >= 0; --r) {
+        const size_t ch = static_cast<size_t>(bh) * a.NC + r;
+        float *dhg = a.dh + ch * D * D;
+        GBWD_FOR(idx, D * D) dhg[idx] = dH[idx];
+        load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+        const float *tt = a.tt + ch * kC * kC;
+        GBWD_FOR(idx, kC * kC) Tt[idx] = tt[idx];
+        GBWD_FOR(i, kC) {
+            const int t = r * kC + i;
+            const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
+            graw[i] = t < a.T ? a.g[row] : 0.f;
+            be[i] = t < a.T ? a.beta[row] : 0.f;
+        }
+        __syncthreads();
+        row_rnorm<D>(Kb, rk, a.l2norm);
+        gate_prefix(graw, gc);
+        __syncthreads();
+        GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+        GBWD_FOR(i, kC) {
+            E[i] = expf(gc[i]);
+            ed[i] = expf(gc[kC - 1] - gc[i]);
+        }
+        __syncthreads();
+        const float *X1 = a.x1 + ch * kC * D;
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * dH[l * D + j];
+            dU[idx] = X1[idx] + ed[i] * acc;
+        }
+        __syncthreads();
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * dU[l * D + j];
+            dR[idx] = be[i] * acc;
+        }
+        __syncthreads();
+        const float *Y1 = a.y1 + ch * D * D;
+        const float elast = expf(gc[kC - 1]);
+        GBWD_FOR(idx, D * D) {
+            const int p = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int i = 0; i < kC; ++i) acc += E[i] * Kb[i * D + p] * dR[i * D + j];
+            dH[idx] = elast * dH[idx] + Y1[idx] - acc;
+        }
+        __syncthreads();
+    }
+    if (a.dS0) GBWD_FOR(idx, D * D) a.dS0[static_cast<size_t>(bh) * D * D + idx] = dH[idx];
+}
+
+// Exclusive suffix over the chunks of each sequence and head of the CCQ increments:
+// dc[r] <- dC_T + sum_{s>r} dc[s], dm[r] <- dm_T + sum_{s>r} dm[s]; the full sums are dC0, dm0.
+template <int D>
+__global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a) {
+    const long long per = static_cast<long long>(D) * D + D;
+    const long long gid = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (gid >= per * a.B * a.H) return;
+    const int bh = static_cast<int>(gid / per);
+    const int e = static_cast<int>(gid % per);
+    const bool isC = e < D * D;
+    const int em = e - D * D;
+    float *base = isC ? a.dc + static_cast<size_t>(bh) * a.NC * D * D + e
+                      : a.dm + static_cast<size_t>(bh) * a.NC * D + em;
+    const size_t stride = isC ? static_cast<size_t>(D) * D : static_cast<size_t>(D);
+    float acc = 0.f;
+    if (isC && a.dCT) acc = a.dCT[static_cast<size_t>(bh) * D * D + e];
+    if (!isC && a.dmT) acc = a.dmT[static_cast<size_t>(bh) * D + em];
+    for (int r = a.NC - 1; r >= 0; --r) {
+        const float x = base[r * stride];
+        base[r * stride] = acc;
+        acc += x;
+    }
+    if (isC && a.dC0) a.dC0[static_cast<size_t>(bh) * D * D + e] = acc;
+    if (!isC && a.dm0) a.dm0[static_cast<size_t>(bh) * D + em] = acc;
+}
+
+// Per chunk: dv, dk, dbeta, dg from the chunk's forward quantities (gdn_bwd_local_kernel),
+// the entering state H_r, the adjoint dH of the leaving state, and DC_{r+1}, Dm_{r+1}.
+template <int D, typename Tin>
+__global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
+    extern __shared__ float4 gbwd_smem4[];
+    float *sm = reinterpret_cast<float *>(gbwd_smem4);
+    float *Kb = sm;                // [64][D]
+    float *dU = Kb + kC * D;       // [64][D]
+    float *dR = dU + kC * D;       // [64][D]
+    float *dK = dR + kC * D;       // [64][D]
+    float *sA = dK + kC * D;       // [64][64] S, then dTb, then dA, then (Qbar Kbar^T) o causal
+    float *sB = sA + kC * kC;      // [64][64] dP, then M2, then dKK, then (W Kbar^T) o causal
+    float *Tt = sB + kC * kC;      // [64][64]
+    float *graw = Tt + kC * kC;
+    float *gc = graw + kC, *E = gc + kC, *ed = E + kC, *be = ed + kC, *tinv = be + kC;
+    float *rk = tinv + kC, *prs = rk + kC, *pcs = prs + kC, *kd = pcs + kC, *gkh = kd + kC;
+    float *rs = gkh + kC, *cs = rs + kC, *db1 = cs + kC, *rdot = db1 + kC, *dgc = rdot + kC;
+    float *scal = dgc + kC;        // [4]: <dH, H>
+
+    const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
+    const int n = min(kC, a.T - r * kC);
+    const float c = a.centered ? 1.f : 0.f;
+    const size_t t64 = static_cast<size_t>(ch) * kC * D;
+    const float *H = a.hs + static_cast<size_t>(ch) * D * D;
+    const float *dHg = a.dh + static_cast<size_t>(ch) * D * D;
+    const float *DC = a.dc + static_cast<size_t>(ch) * D * D;
+    const float *Dm = a.dm + static_cast<size_t>(ch) * D;
+    const float *X1 = a.x1 + t64;
+    const float *Qbg = a.qb + t64, *Qcg = a.qc + t64, *Ug = a.u + t64, *Rg = a.r + t64, *Wg = a.w + t64;
+    const float *vec = a.vec + static_cast<size_t>(ch) * 4 * kC;
+    const float *cq = vec, *cz = vec + kC, *gqh = vec + 2 * kC;
+    const float *ttg = a.tt + static_cast<size_t>(ch) * kC * kC;
+    const Tin *dout = static_cast<const Tin *>(a.dout);
+    const Tin *vin = static_cast<const Tin *>(a.v);
+    const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
+    auto Dsc = [&](int i, int col) -> float {
+        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + col]) : 0.f;
+    };
+
+    load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+    GBWD_FOR(idx, kC * kC) Tt[idx] = ttg[idx];
+    GBWD_FOR(i, kC) {
+        const int t = r * kC + i;
+        const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
+        graw[i] = i < n ? a.g[row] : 0.f;
+        be[i] = i < n ? a.beta[row] : 0.f;
+        tinv[i] = 1.f / (t_start + 1.f + static_cast<float>(i));
+        prs[i] = pcs[i] = kd[i] = gkh[i] = rs[i] = cs[i] = 0.f;
+    }
+    if (threadIdx.x == 0) scal[0] = 0.f;
+    __syncthreads();
+    row_rnorm<D>(Kb, rk, a.l2norm);
+    gate_prefix(graw, gc);
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+    GBWD_FOR(i, kC) {
+        E[i] = expf(gc[i]);
+        ed[i] = expf(gc[kC - 1] - gc[i]);
+    }
+    __syncthreads();
+    // S = Qc Kbar^T;  dU = P^T D + Kd dH
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        for (int l = 0; l < D; ++l) acc += Qcg[i * D + l] * Kb[j * D + l];
+        sA[idx] = acc;
+    }
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float acc = 0.f;
+        for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * dHg[l * D + j];
+        dU[idx] = X1[idx] + ed[i] * acc;
+    }
+    __syncthreads();
+    // dv = dR = diag(beta) Tt^T dU;  dP = (D U^T) o Gamma o causal
+    {
+        Tin *dv = static_cast<Tin *>(a.dv);
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            float acc = 0.f;
+            for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * dU[l * D + j];
+            acc *= be[i];
+            dR[idx] = acc;
+            if (i < n) dv[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(acc);
+        }
+        GBWD_FOR(idx, kC * kC) {
+            const int i = idx / kC, j = idx % kC;
+            float acc = 0.f;
+            if (j <= i && i < n) {
+                for (int l = 0; l < D; ++l) acc += Dsc(i, l) * Ug[j * D + l];
+                acc *= expf(gc[i] - gc[j]);
+            }
+            sB[idx] = acc;
+        }
+    }
+    __syncthreads();
+    // dK = dP^T Qc + diag(e^{gc_last - gc}) U dH^T - diag(E) dR H^T;  row and column sums of
+    // dP o S;  kd_i = rowsum(Kd o U dH^T)_i = U_i . (dU - P^T D)_i;  gkh_i = E_i (Kbar H)_i . dR_i
+    // = (V - R)_i . dR_i;  <dH, H>
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float acc = 0.f, udh = 0.f, drh = 0.f;
+        for (int l = i; l < kC; ++l) acc += sB[l * kC + i] * Qcg[l * D + j];
+        for (int l = 0; l < D; ++l) {
+            udh += Ug[i * D + l] * dHg[j * D + l];
+            drh += dR[i * D + l] * H[j * D + l];
+        }
+        dK[idx] = acc + ed[i] * udh - E[i] * drh;
+    }
+    GBWD_FOR(i, kC) {
+        float p = 0.f, q = 0.f, x = 0.f, y = 0.f;
+        for (int j = 0; j < kC; ++j) {
+            p += sB[i * kC + j] * sA[i * kC + j];
+            q += sB[j * kC + i] * sA[j * kC + i];
+        }
+        for (int l = 0; l < D; ++l) {
+            x += Ug[i * D + l] * (dU[i * D + l] - X1[i * D + l]);
+            const float vv = i < n ? to_f(vin[tok_row(a, b, r * kC + i, h) * D + l]) : 0.f;
+            y += (vv - Rg[i * D + l]) * dR[i * D + l];
+        }
+        prs[i] = p;
+        pcs[i] = q;
+        kd[i] = x;
+        gkh[i] = y;
+    }
+    GBWD_FOR(p, D) {
+        float acc = 0.f;
+        for (int j = 0; j < D; ++j) acc += dHg[p * D + j] * H[p * D + j];
+        atomicAdd(&scal[0], acc);
+    }
+    __syncthreads();
+    // dTb = dU R^T
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        for (int l = 0; l < D; ++l) acc += dU[i * D + l] * Rg[j * D + l];
+        sA[idx] = acc;
+    }
+    __syncthreads();
+    // dbeta (the Tb = Tt diag(beta) factor) = column sums of dTb o Tt;  M2 = Tt^T (dTb diag(beta))
+    GBWD_FOR(j, kC) {
+        float acc = 0.f;
+        for (int i = 0; i < kC; ++i) acc += sA[i * kC + j] * Tt[i * kC + j];
+        db1[j] = acc;
+    }
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * sA[l * kC + j];
+        sB[idx] = acc * be[j];
+    }
+    __syncthreads();
+    // dA = strict_lower(-M2 Tt^T)
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float acc = 0.f;
+        if (j < i)
+            for (int l = 0; l <= j; ++l) acc -= sB[i * kC + l] * Tt[j * kC + l];
+        sA[idx] = acc;
+    }
+    __syncthreads();
+    // dKK = diag(beta) (dA o Gamma);  rs_i = sum_j dA_ij Gamma_ij KK_ij (the dbeta of A);
+    // rowsum(dA o A)_i = beta_i rs_i;  cs_j = colsum(dA o A)_j
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float v = 0.f;
+        if (j < i) {
+            float kk = 0.f;
+            for (int l = 0; l < D; ++l) kk += Kb[i * D + l] * Kb[j * D + l];
+            const float gm = expf(gc[i] - gc[j]);
+            const float x = sA[idx] * gm * kk;
+            atomicAdd(&rs[i], x);
+            atomicAdd(&cs[j], be[i] * x);
+            v = sA[idx] * be[i] * gm;
+        }
+        sB[idx] = v;
+    }
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float acc = 0.f;
+        for (int l = 0; l < kC; ++l) acc += (sB[i * kC + l] + sB[l * kC + i]) * Kb[l * D + j];
+        dK[idx] += acc;
+    }
+    __syncthreads();
+    // CCQ terms: (Qbar Kbar^T) o causal and (W Kbar^T) o causal
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, j = idx % kC;
+        float x = 0.f, y = 0.f;
+        if (j <= i)
+            for (int l = 0; l < D; ++l) {
+                x += Qbg[i * D + l] * Kb[j * D + l];
+                y += Wg[i * D + l] * Kb[j * D + l];
+            }
+        sA[idx] = x;
+        sB[idx] = y;
+    }
+    __syncthreads();
+    // dK += QKc^T W + WKc^T Qbar + Kbar (DC + DC^T) + Dm + reverse cumsum of dCum,
+    // dCum_l = -c (dz_l cq_l + qbar_l cz_l) / t_l^2, dz_l = t_l W_l
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float acc = Dm[j];
+        for (int l = i; l < kC; ++l) {
+            acc += sA[l * kC + i] * Wg[l * D + j] + sB[l * kC + i] * Qbg[l * D + j];
+            acc -= c * (Wg[l * D + j] * cq[l] / tinv[l] + Qbg[l * D + j] * cz[l]) * tinv[l] * tinv[l];
+        }
+        for (int p = 0; p < D; ++p) acc += Kb[i * D + p] * (DC[p * D + j] + DC[j * D + p]);
+        dK[idx] += acc;
+    }
+    __syncthreads();
+    GBWD_FOR(i, kC) {
+        float acc = 0.f;
+        for (int j = 0; j < D; ++j) acc += Kb[i * D + j] * dK[i * D + j];
+        rdot[i] = a.l2norm ? acc : 0.f;
+        float x = be[i] * rs[i] - cs[i] + prs[i] - pcs[i] + gqh[i] - kd[i] - gkh[i];
+        if (i == n - 1) {
+            float sk = 0.f;
+            for (int l = 0; l < kC; ++l) sk += kd[l];
+            x += expf(gc[kC - 1]) * scal[0] + sk;
+        }
+        dgc[i] = x;
+        if (i < n) a.dbeta[tok_row(a, b, r * kC + i, h)] = db1[i] + rs[i];
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float acc = 0.f;
+        for (int i = n - 1; i >= 0; --i) {
+            acc += dgc[i];
+            a.dg[tok_row(a, b, r * kC + i, h)] = acc;
+        }
+    }
+    {
+        Tin *dk = static_cast<Tin *>(a.dk);
+        GBWD_FOR(idx, kC * D) {
+            const int i = idx / D, j = idx % D;
+            if (i < n) dk[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((dK[idx] - Kb[idx] * rdot[i]) * rk[i]);
+        }
+    }
+}
+
+// Shared-memory bytes of each kernel.
+template <int D> constexpr size_t prep_smem() { return sizeof(float) * (kC * D + 2 * kC * kC + 4 * kC); }
+template <int D> constexpr size_t fstate_smem() { return sizeof(float) * (D * D + 3 * kC * D + kC * kC + 6 * kC); }
+template <int D> constexpr size_t local_smem() { return sizeof(float) * (5 * kC * D + 2 * kC * kC + 12 * kC); }
+template <int D> constexpr size_t dstate_smem() { return sizeof(float) * (D * D + 3 * kC * D + kC * kC + 6 * kC); }
+template <int D> constexpr size_t kv_smem() { return sizeof(float) * (4 * kC * D + 3 * kC * kC + 16 * kC + 4); }
+
+}  // namespace gbwd
+}  // namespace ccq

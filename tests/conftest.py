@@ -17,3 +17,9 @@ def oracle_mod():
     import oracle
     oracle.build_oracle()
     return oracle
+
+
+# Parity tests of entry points whose kernels have not yet run on a GPU.  They are collected
+# (moved up into tests/) once a GPU run has passed them, so that an unverified kernel never
+# runs first inside the suite.
+collect_ignore = ["gpu_pending"]
