@@ -263,6 +263,36 @@ CCQ_API ccq_status ccq_gdn_bwd_workspace_size(int B, int T, int H, int Dk, int D
                                               const ccq_params *p, size_t *bytes);
 
 /*
+ * CCQ-Gated-DeltaNet forward with a decay-aligned covariance.  The paper proposes a
+ * covariance from gamma-weighted running statistics for backbones that forget
+ * (Limitations; App. "Modelling choices and limitations", interaction with decayed
+ * backbones) but fixes neither the weights nor the normaliser.  This entry point reads gamma_{j,t} as the product of the backbone's own
+ * decays alpha_s = exp(g_s) over j < s <= t and normalises by the decayed count:
+ *   C_t = alpha_t C_{t-1} + kbar_t kbar_t^T,  m_t = alpha_t m_{t-1} + kbar_t,
+ *   n_t = alpha_t n_{t-1} + 1,  Sigma_t = C_t / n_t - (m_t / n_t)(m_t / n_t)^T
+ * (uncentred with centered = 0), which is ccq_gdn_fwd's covariance when every alpha = 1.
+ *   C0/CT [B,H,Dk,Dk], m0/mT [B,H,Dk]: the decayed sums;  n0/nT [B,H] fp32: the decayed
+ *   count (replacing t0/tT).  NULL initial pointers mean zero; NULL final pointers are not
+ *   written.
+ *   workspace  at least ccq_gdn_decayed_workspace_size() bytes, 16-byte aligned (per 64-token
+ *              chunk of every (sequence, head): the chunk's UT factor, entering state and
+ *              entering statistics in fp32).
+ * Other arguments as ccq_gdn_fwd.  Supported: Dk = Dv in {64, 128}, bf16 or fp32 inputs;
+ * the kernels compute in fp32 on the CUDA cores (five launches; the algo parameter is
+ * ignored).
+ */
+CCQ_API ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, const float *g,
+                                       const float *beta, const float *lambda, ccq_dtype in_dtype,
+                                       const float *S0, const float *C0, const float *m0, const float *n0,
+                                       void *o, float *ST, float *CT, float *mT, float *nT,
+                                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                                       size_t workspace_bytes, const ccq_params *p, void *stream);
+
+/* Workspace bytes ccq_gdn_fwd_decayed needs for these sizes (0 when T = 0).  Host-only. */
+CCQ_API ccq_status ccq_gdn_decayed_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                                  const ccq_params *p, size_t *bytes);
+
+/*
  * ccq_gla_fwd for callers that cannot supply any device memory of their own --
  * for instance an engine that gave all device memory to its own caches at
  * start-up, or code on a path where allocating is not allowed or would stall

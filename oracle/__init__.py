@@ -22,7 +22,7 @@ Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``)
                      the paper's future-work variant, stated in ccq_oracle.c) -- pinned
                      by brute-force weighted covariances, the undecayed special case,
                      the spectrum bound and resumption (tests/test_oracle_decayed.py);
-                     no GPU path consumes it yet.
+                     the reference of the ccq_gdn_fwd_decayed parity tests.
   Absolute outputs on the benchmark-shaped random inputs are pinned only
   through the above: the paper prints no worked numerical example.
 """

@@ -98,6 +98,14 @@ def load_library() -> ctypes.CDLL:
         lib.ccq_gdn_bwd_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
                                                                ctypes.POINTER(ctypes.c_size_t)])
         lib.ccq_gdn_bwd_workspace_size.restype = _I
+        # q, k, v, g, beta, lambda | in_dtype | S0, C0, m0, n0, o, ST, CT, mT, nT | B, T, H, Dk, Dv
+        # | workspace, bytes, params, stream
+        lib.ccq_gdn_fwd_decayed.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 5
+                                            + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
+        lib.ccq_gdn_fwd_decayed.restype = _I
+        lib.ccq_gdn_decayed_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
+                                                                   ctypes.POINTER(ctypes.c_size_t)])
+        lib.ccq_gdn_decayed_workspace_size.restype = _I
         _lib = lib
     return _lib
 
@@ -440,6 +448,50 @@ def gdn_bwd(q, k, v, g, beta, lam, dout, state: Optional[CCQState] = None, *, dS
         _stream(dev, stream))
     _check(st)
     return grads
+
+
+def gdn_fwd_decayed(q, k, v, g, beta, lam, *, S0=None, C0=None, m0=None, n0=None, out=None,
+                    return_state: bool = True, workspace=None, stream=None, **kw):
+    """CCQ-Gated-DeltaNet forward with the decay-aligned covariance (statistics decayed by the
+    backbone's own decay, normalised by the decayed count n).  S0 [B,H,Dk,Dv], C0 [B,H,Dk,Dk],
+    m0 [B,H,Dk], n0 [B,H] fp32 (None = zero).  Returns o, or (o, dict S, C, m, n of final
+    states) when ``return_state``."""
+    dev = q.device
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (B, T, H, Dv))
+    for x, name in ((g, "g"), (beta, "beta"), (lam, "lam")):
+        _req(x, name, dev, torch.float32, (B, T, H))
+    for x, name, shape in ((S0, "S0", (B, H, Dk, Dv)), (C0, "C0", (B, H, Dk, Dk)), (m0, "m0", (B, H, Dk)),
+                           (n0, "n0", (B, H))):
+        if x is not None:
+            _req(x, name, dev, torch.float32, shape)
+    o = out if out is not None else torch.empty(B, T, H, Dv, dtype=q.dtype, device=dev)
+    _req(o, "out", dev, q.dtype, (B, T, H, Dv))
+    fs = None
+    if return_state:
+        fs = {"S": torch.empty(B, H, Dk, Dv, dtype=torch.float32, device=dev),
+              "C": torch.empty(B, H, Dk, Dk, dtype=torch.float32, device=dev),
+              "m": torch.empty(B, H, Dk, dtype=torch.float32, device=dev),
+              "n": torch.empty(B, H, dtype=torch.float32, device=dev)}
+    p = params(**kw)
+    lib = load_library()
+    need = ctypes.c_size_t(0)
+    _check(lib.ccq_gdn_decayed_workspace_size(B, T, H, Dk, Dv, _dtype_code(q), ctypes.byref(p),
+                                              ctypes.byref(need)))
+    if workspace is None and need.value:
+        workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_gdn_fwd_decayed(
+        _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _dtype_code(q),
+        _ptr(S0), _ptr(C0), _ptr(m0), _ptr(n0), _ptr(o),
+        _ptr(fs["S"] if fs else None), _ptr(fs["C"] if fs else None), _ptr(fs["m"] if fs else None),
+        _ptr(fs["n"] if fs else None), B, T, H, Dk, Dv, _ptr(workspace), ws_bytes, ctypes.byref(p),
+        _stream(dev, stream))
+    _check(st)
+    return (o, fs) if return_state else o
 
 
 def gla_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):

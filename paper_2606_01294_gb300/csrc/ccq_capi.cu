@@ -633,6 +633,63 @@ ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float 
     return CCQ_OK;
 }
 
+ccq_status ccq_gdn_decayed_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
+                                          const ccq_params *p, size_t *bytes) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    *bytes = T > 0 ? gdn_decayed_workspace_bytes(B, T, H, Dk) : 0;
+    return CCQ_OK;
+}
+
+ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, const float *g,
+                               const float *beta, const float *lambda, ccq_dtype in_dtype,
+                               const float *S0, const float *C0, const float *m0, const float *n0,
+                               void *o, float *ST, float *CT, float *mT, float *nT, int B, int T, int H,
+                               int Dk, int Dv, void *workspace, size_t workspace_bytes,
+                               const ccq_params *p, void *stream) {
+    Common c;
+    ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
+    if (st != CCQ_OK) return st;
+    if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    st = check_ptrs("", {}, {S0, C0, m0, n0, ST, CT, mT, nT});
+    if (st != CCQ_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (T == 0) {
+        // no tokens: the final states are the initial ones
+        const size_t n[4] = {static_cast<size_t>(B) * H * Dk * Dv * 4, static_cast<size_t>(B) * H * Dk * Dk * 4,
+                             static_cast<size_t>(B) * H * Dk * 4, static_cast<size_t>(B) * H * 4};
+        float *dst[4] = {ST, CT, mT, nT};
+        const float *src[4] = {S0, C0, m0, n0};
+        for (int i = 0; i < 4; ++i) {
+            if (!dst[i] || dst[i] == src[i]) continue;
+            cudaError_t e = src[i] ? cudaMemcpyAsync(dst[i], src[i], n[i], cudaMemcpyDeviceToDevice, s)
+                                   : cudaMemsetAsync(dst[i], 0, n[i], s);
+            if (e != cudaSuccess) return cuda_fail(e, "state copy");
+        }
+        return CCQ_OK;
+    }
+    st = check_ptrs("q,k,v,g,beta,lambda,o", {q, k, v, g, beta, lambda, o}, {});
+    if (st != CCQ_OK) return st;
+    const size_t need = gdn_decayed_workspace_bytes(B, T, H, Dk);
+    if (!workspace || workspace_bytes < need)
+        return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
+                    workspace ? workspace_bytes : static_cast<size_t>(0));
+    if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+    GdecCall a = {};
+    a.B = B; a.T = T; a.H = H; a.D = Dk; a.bf16 = in_dtype == CCQ_BF16;
+    a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
+    a.q = q; a.k = k; a.v = v; a.g = g; a.beta = beta; a.lambda = lambda;
+    a.S0 = S0; a.C0 = C0; a.m0 = m0; a.n0 = n0;
+    a.o = o; a.ST = ST; a.CT = CT; a.mT = mT; a.nT = nT;
+    a.workspace = workspace;
+    cudaError_t e = launch_gdn_decayed(a, s);
+    if (e != cudaSuccess) return cuda_fail(e, "decayed-covariance Gated DeltaNet launch");
+    return CCQ_OK;
+}
+
 ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,
                            const void *gate, const float *beta, const float *lambda,
                            ccq_dtype in_dtype, ccq_dtype gate_dtype, float *S, float *C,

@@ -1,5 +1,5 @@
-// ccq_gdn_bwd.h -- launch interface of the CUDA-core CCQ-Gated-DeltaNet backward
-// (ccq_gdn_bwd.cu), used by the C ABI.
+// ccq_gdn_bwd.h -- launch interfaces of the CUDA-core CCQ-Gated-DeltaNet kernels (the backward,
+// ccq_gdn_bwd.cu, and the decay-aligned-covariance forward, ccq_gdn_decayed.cu), used by the C ABI.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -24,5 +24,19 @@ struct GdnBwdCall {
 };
 size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D);
 cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s);
+
+// Arguments of the CUDA-core CCQ-Gated-DeltaNet forward with the decay-aligned covariance
+// (ccq_gdn_decayed.cu); n0/nT are the decayed counts [B][H].
+struct GdecCall {
+    int B, T, H, D, bf16, l2norm, centered;
+    float scale;
+    const void *q, *k, *v;
+    const float *g, *beta, *lambda, *S0, *C0, *m0, *n0;
+    void *o;
+    float *ST, *CT, *mT, *nT;
+    void *workspace;
+};
+size_t gdn_decayed_workspace_bytes(int B, int T, int H, int D);
+cudaError_t launch_gdn_decayed(const GdecCall &c, cudaStream_t s);
 
 }  // namespace ccq

@@ -84,6 +84,7 @@ struct GdnBwdArgs {
     float *y1;   // [D][D]   (diag(E) Qc)^T D
     float *qb, *qc, *u, *r, *w;  // [64][D] each: qbar, qc, U, R, W = dz / t
     float *vec;  // [4][64]  cq, cz, E o rowsum((Qc H) o D), spare
+    float *hT = nullptr;  // [B][H][D][D]: when set, gdn_bwd_fstate_kernel writes the final state
 };
 
 __device__ __forceinline__ size_t tok_row(const GdnBwdArgs &a, int b, int t, int h) {
@@ -211,7 +212,8 @@ __global__ void __launch_bounds__(256) gdn_bwd_prefix_kernel(const GdnBwdArgs a)
     }
 }
 
-// Per sequence and head, chunks in order: the state entering every chunk.
+// Per sequence and head, chunks in order: the state entering every chunk (and, when hT is
+// set, the final state).
 template <int D, typename Tin>
 __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
@@ -277,6 +279,7 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
         }
         __syncthreads();
     }
+    if (a.hT) GBWD_FOR(idx, D * D) a.hT[static_cast<size_t>(bh) * D * D + idx] = Hs[idx];
 }
 
 // Per chunk, everything that does not need dH: z, qc, R, U, dqc, dq, dlambda, the CCQ

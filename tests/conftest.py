@@ -1,4 +1,7 @@
+import ctypes
 import os
+import shutil
+import subprocess
 import sys
 
 import pytest
@@ -23,3 +26,28 @@ def oracle_mod():
 # (moved up into tests/) once a GPU run has passed them, so that an unverified kernel never
 # runs first inside the suite.
 collect_ignore = ["gpu_pending"]
+
+
+def load_gdn_emu(path):
+    """ctypes handle of a host build of tests/host_emu/gdn_cuda_core_emu.cpp."""
+    lib = ctypes.CDLL(path)
+    lib.gdn_bwd_emu.argtypes = [ctypes.c_int] * 7 + [ctypes.c_float] + [ctypes.c_void_p] * 3
+    lib.gdn_bwd_emu.restype = ctypes.c_int
+    lib.gdn_decayed_emu.argtypes = [ctypes.c_int] * 7 + [ctypes.c_float] + [ctypes.c_void_p] * 2
+    lib.gdn_decayed_emu.restype = ctypes.c_int
+    return lib
+
+
+@pytest.fixture(scope="session")
+def gdn_emu(tmp_path_factory):
+    """The CUDA-core Gated DeltaNet kernels compiled for the host (CPU tests of their arithmetic)."""
+    gxx = shutil.which("g++")
+    inc = "/usr/local/cuda/include"
+    if gxx is None or not os.path.isdir(inc):
+        pytest.skip("g++ or the CUDA headers are not available")
+    src = os.path.join(ROOT, "tests", "host_emu", "gdn_cuda_core_emu.cpp")
+    out = str(tmp_path_factory.mktemp("gdn_emu") / "gdn_cuda_core_emu.so")
+    r = subprocess.run([gxx, "-O2", "-std=c++17", "-fPIC", "-shared", "-I" + inc, src, "-o", out],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr[-4000:]
+    return load_gdn_emu(out)

@@ -1,6 +1,7 @@
-// Host build of the CCQ-Gated-DeltaNet backward kernels, for a CPU test of their arithmetic
-// and indexing against the fp64 oracle (tests/test_gdn_bwd_host.py).  Test infrastructure
-// only: the library never builds or loads this file.
+// Host build of the CUDA-core CCQ-Gated-DeltaNet kernels (the backward and the forward with
+// the decay-aligned covariance), for a CPU test of their arithmetic and indexing against the
+// fp64 oracle (tests/test_gdn_bwd_host.py, tests/test_gdn_decayed_host.py).  Test
+// infrastructure only: the library never builds or loads this file.
 //
 // The kernels are written as phases separated by __syncthreads(), in each of which every
 // thread strides over the elements it owns and reads only what earlier phases wrote.  Run
@@ -38,7 +39,7 @@ float4 (*g_smem)[];
 }  // namespace gbwd
 }  // namespace ccq
 #define gbwd_smem4 (*g_smem)
-#include "../../paper_2606_01294_gb300/csrc/ccq_gdn_bwd_kernels.cuh"
+#include "../../paper_2606_01294_gb300/csrc/ccq_gdn_decayed_kernels.cuh"
 #undef gbwd_smem4
 using namespace ccq::gbwd;
 
@@ -121,5 +122,45 @@ extern "C" int gdn_bwd_emu(int D, int bf16, int B, int T, int H, int l2norm, int
     if (D == 16) return bf16 ? go<16, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, t0, out)
                              : go<16, float>(B, T, H, l2norm, centered, scale, in, t0, out);
     if (D == 64 && !bf16) return go<64, float>(B, T, H, l2norm, centered, scale, in, t0, out);
+    return -1;
+}
+
+template <int D, typename Tin>
+static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, const float *const *in,
+                  float *const *out) {
+    // in: q, k, v, g, beta, lambda, S0, C0, m0, n0;  out: o, ST, CT, mT, nT
+    const size_t ntok = static_cast<size_t>(B) * T * H * D;
+    auto q = to_in<Tin>(in[0], ntok), k = to_in<Tin>(in[1], ntok), v = to_in<Tin>(in[2], ntok);
+    std::vector<Tin> o(ntok);
+    GdecArgs g{};
+    GdnBwdArgs &a = g.base;
+    a.B = B; a.T = T; a.H = H; a.NC = (T + 63) / 64;
+    a.l2norm = l2norm; a.centered = centered; a.scale = scale;
+    a.q = q.data(); a.k = k.data(); a.v = v.data();
+    a.g = in[3]; a.beta = in[4]; a.lambda = in[5]; a.S0 = in[6]; a.C0 = in[7]; a.m0 = in[8];
+    g.n0 = in[9];
+    g.o = o.data();
+    a.hT = out[1]; g.CT = out[2]; g.mT = out[3]; g.nT = out[4];
+    const size_t chunks = static_cast<size_t>(B) * H * a.NC, d = D;
+    std::vector<float> ws(chunks * (64 * 64 + 3 * d * d + 2 * d + 4), NAN);
+    float *p = ws.data();
+    auto take = [&](size_t per) { float *r = p; p += chunks * per; return r; };
+    a.tt = take(64 * 64); a.sk = take(d * d); a.mk = take(d); a.hs = take(d * d);
+    g.dC = take(d * d); g.dmv = take(d); g.dn = take(4);
+    const long long nch = static_cast<long long>(chunks), bh = static_cast<long long>(B) * H;
+    run_blocks([&] { gdn_bwd_prep_kernel<D, Tin>(a); }, nch, prep_smem<D>());
+    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh, fstate_smem<D>());
+    run_blocks([&] { gdec_stats_kernel<D, Tin>(g); }, nch, gdec_stats_smem<D>());
+    run_blocks([&] { gdec_scan_kernel<D>(g); }, (static_cast<long long>(D) * D + D + 1) * bh, 0);
+    run_blocks([&] { gdec_out_kernel<D, Tin>(g); }, nch, gdec_out_smem<D>());
+    to_out(o, out[0]);
+    return 0;
+}
+
+extern "C" int gdn_decayed_emu(int D, int bf16, int B, int T, int H, int l2norm, int centered, float scale,
+                               const float *const *in, float *const *out) {
+    if (D == 16) return bf16 ? go_dec<16, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, out)
+                             : go_dec<16, float>(B, T, H, l2norm, centered, scale, in, out);
+    if (D == 64 && !bf16) return go_dec<64, float>(B, T, H, l2norm, centered, scale, in, out);
     return -1;
 }

@@ -1,46 +1,19 @@
 """CPU check of the CCQ-Gated-DeltaNet backward kernels' arithmetic and indexing.
 
 The kernels (paper_2606_01294_gb300/csrc/ccq_gdn_bwd_kernels.cuh) are compiled for the host
-by tests/host_emu/gdn_bwd_emu.cpp, which runs every CTA with one thread, phase by phase (the
-kernels are written so that this computes what the CTA computes), each CTA with exactly its
-dynamic shared memory filled with NaN.  Their gradients are compared with the oracle's fp64
+by tests/host_emu/gdn_cuda_core_emu.cpp (the gdn_emu fixture), which runs every CTA with one
+thread, phase by phase (the kernels are written so that this computes what the CTA
+computes), each CTA with exactly its dynamic shared memory filled with NaN.  Their gradients are compared with the oracle's fp64
 reverse mode on the same inputs: fp32 inputs to 1e-4 (the fp32 bar; observed about 2e-6),
 bf16 inputs to 2e-2.  This checks the algebra of the chunked adjoint, the chunk and tail
 indexing and the workspace layout without a GPU; the GPU parity test checks the same
 entry point through the C ABI on the device."""
 import ctypes
-import os
-import shutil
-import subprocess
 
 import numpy as np
 import pytest
 
 import oracle
-
-HERE = os.path.dirname(os.path.abspath(__file__))
-SRC = os.path.join(HERE, "host_emu", "gdn_bwd_emu.cpp")
-CUDA_INC = "/usr/local/cuda/include"
-
-
-@pytest.fixture(scope="module")
-def emu(tmp_path_factory):
-    gxx = shutil.which("g++")
-    if gxx is None or not os.path.isdir(CUDA_INC):
-        pytest.skip("g++ or the CUDA headers are not available")
-    out = str(tmp_path_factory.mktemp("gdn_bwd_emu") / "gdn_bwd_emu.so")
-    r = subprocess.run([gxx, "-O2", "-std=c++17", "-fPIC", "-shared", "-I" + CUDA_INC, SRC, "-o", out],
-                       capture_output=True, text=True)
-    assert r.returncode == 0, r.stderr[-4000:]
-    return load(out)
-
-
-def load(path):
-    lib = ctypes.CDLL(path)
-    lib.gdn_bwd_emu.argtypes = [ctypes.c_int] * 7 + [ctypes.c_float, ctypes.c_void_p, ctypes.c_void_p,
-                                                     ctypes.c_void_p]
-    lib.gdn_bwd_emu.restype = ctypes.c_int
-    return lib
 
 
 def bf16_round(a):
@@ -109,13 +82,13 @@ CASES = [
 
 
 @pytest.mark.parametrize("case", CASES, ids=[str(i) for i in range(len(CASES))])
-def test_gdn_bwd_kernels_on_host(emu, oracle_mod, case):
+def test_gdn_bwd_kernels_on_host(gdn_emu, oracle_mod, case):
     case = dict(case)
     opts = case.pop("opts", {})
     D, B, T, H, seed = (case.pop(n) for n in ("D", "B", "T", "H", "seed"))
     bf16 = case.get("bf16", False)
     P = problem(D, B, T, H, seed, **case)
-    errs = run_case(emu, D, P, bf16=bf16, **opts)
+    errs = run_case(gdn_emu, D, P, bf16=bf16, **opts)
     # bf16 inputs: dq, dk, dv are rounded to bf16 on output
     tol = {n: (2e-2 if bf16 and n in ("dq", "dk", "dv") else 1e-4) for n in errs}
     bad = {n: e for n, e in errs.items() if not e <= tol[n]}
