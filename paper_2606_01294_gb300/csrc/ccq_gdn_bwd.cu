@@ -27,18 +27,18 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
     using namespace gbwd;
     cudaError_t e;
     if ((e = allow_smem(gdn_bwd_prep_kernel<D, Tin>, prep_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_fstate_kernel<D, Tin>, fstate_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_fstate_kernel<D, Tin>, fstate_smem<D>(a.nsplit))) != cudaSuccess) return e;
     if ((e = allow_smem(gdn_bwd_local_kernel<D, Tin>, local_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_dstate_kernel<D, Tin>, dstate_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_dstate_kernel<D, Tin>, dstate_smem<D>(a.nsplit))) != cudaSuccess) return e;
     if ((e = allow_smem(gdn_bwd_kv_kernel<D, Tin>, kv_smem<D>())) != cudaSuccess) return e;
     const unsigned nch = static_cast<unsigned>(a.B * a.H * a.NC), bh = static_cast<unsigned>(a.B * a.H);
     const long long elems = (static_cast<long long>(D) * D + D) * a.B * a.H;
     const unsigned eblocks = static_cast<unsigned>((elems + 255) / 256);
     gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
     gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
-    gdn_bwd_fstate_kernel<D, Tin><<<bh, 512, fstate_smem<D>(), s>>>(a);
+    gdn_bwd_fstate_kernel<D, Tin><<<bh * a.nsplit, 512, fstate_smem<D>(a.nsplit), s>>>(a);
     gdn_bwd_local_kernel<D, Tin><<<nch, 256, local_smem<D>(), s>>>(a);
-    gdn_bwd_dstate_kernel<D, Tin><<<bh, 512, dstate_smem<D>(), s>>>(a);
+    gdn_bwd_dstate_kernel<D, Tin><<<bh * a.nsplit, 512, dstate_smem<D>(a.nsplit), s>>>(a);
     gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
     gdn_bwd_kv_kernel<D, Tin><<<nch, 256, kv_smem<D>(), s>>>(a);
     return cudaGetLastError();
@@ -54,6 +54,7 @@ size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D) {
 cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s) {
     gbwd::GdnBwdArgs a{};
     a.B = c.B; a.T = c.T; a.H = c.H; a.NC = (c.T + 63) / 64;
+    a.nsplit = gbwd::seq_split(c.B, c.H);
     a.l2norm = c.l2norm; a.centered = c.centered; a.scale = c.scale;
     a.q = c.q; a.k = c.k; a.v = c.v; a.dout = c.dout;
     a.g = c.g; a.beta = c.beta; a.lambda = c.lambda;

@@ -85,6 +85,9 @@ struct GdnBwdArgs {
     float *qb, *qc, *u, *r, *w;  // [64][D] each: qbar, qc, U, R, W = dz / t
     float *vec;  // [4][64]  cq, cz, E o rowsum((Qc H) o D), spare
     float *hT = nullptr;  // [B][H][D][D]: when set, gdn_bwd_fstate_kernel writes the final state
+    int nsplit = 1;       // value-column blocks of the sequential passes (a divisor of D): the
+                          // delta rule acts on the columns of H independently, so each
+                          // (sequence, head) runs as nsplit CTAs of D / nsplit columns
 };
 
 __device__ __forceinline__ size_t tok_row(const GdnBwdArgs &a, int b, int t, int h) {
@@ -213,28 +216,37 @@ __global__ void __launch_bounds__(256) gdn_bwd_prefix_kernel(const GdnBwdArgs a)
 }
 
 // Per sequence and head, chunks in order: the state entering every chunk (and, when hT is
-// set, the final state).
+// set, the final state).  CTA (sequence-head, s) carries the value columns
+// [s D/nsplit, (s+1) D/nsplit) of H.
 template <int D, typename Tin>
 __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
+    const int ns = a.nsplit, DC = D / ns;
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *Hs = sm;               // [D][D]
-    float *Kb = Hs + D * D;       // [64][D]
-    float *R = Kb + kC * D;       // [64][D]
-    float *U = R + kC * D;        // [64][D]
-    float *Tt = U + kC * D;       // [64][64]
+    float *Hs = sm;               // [D][DC]
+    float *Kb = Hs + D * DC;      // [64][D]
+    float *R = Kb + kC * D;       // [64][DC]
+    float *U = R + kC * DC;       // [64][DC]
+    float *Tt = U + kC * DC;      // [64][64]
     float *graw = Tt + kC * kC;   // [64]
     float *gc = graw + kC, *be = gc + kC, *rk = be + kC, *E = rk + kC, *ed = E + kC;
 
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
-    GBWD_FOR(idx, D * D) Hs[idx] = a.S0 ? a.S0[static_cast<size_t>(bh) * D * D + idx] : 0.f;
+    const int bh = blockIdx.x / ns, c0 = (blockIdx.x % ns) * DC, b = bh / a.H, h = bh % a.H;
+    const Tin *vin = static_cast<const Tin *>(a.v);
+    GBWD_FOR(idx, D * DC) {
+        const int l = idx / DC, j = idx % DC;
+        Hs[idx] = a.S0 ? a.S0[(static_cast<size_t>(bh) * D + l) * D + c0 + j] : 0.f;
+    }
     __syncthreads();
     for (int r = 0; r < a.NC; ++r) {
         const size_t ch = static_cast<size_t>(bh) * a.NC + r;
         float *hs = a.hs + ch * D * D;
-        GBWD_FOR(idx, D * D) hs[idx] = Hs[idx];
+        GBWD_FOR(idx, D * DC) hs[(idx / DC) * D + c0 + idx % DC] = Hs[idx];
         load_tile<D, Tin>(Kb, a.k, a, b, h, r);
-        load_tile<D, Tin>(R, a.v, a, b, h, r);
+        GBWD_FOR(idx, kC * DC) {
+            const int i = idx / DC, j = idx % DC, t = r * kC + i;
+            R[idx] = t < a.T ? to_f(vin[tok_row(a, b, t, h) * D + c0 + j]) : 0.f;
+        }
         const float *tt = a.tt + ch * kC * kC;
         GBWD_FOR(idx, kC * kC) Tt[idx] = tt[idx];
         GBWD_FOR(i, kC) {
@@ -254,32 +266,33 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
         }
         __syncthreads();
         // R = V - diag(E) Kbar H
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
+        GBWD_FOR(idx, kC * DC) {
+            const int i = idx / DC, j = idx % DC;
             float acc = 0.f;
-            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * Hs[l * D + j];
+            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * Hs[l * DC + j];
             R[idx] -= E[i] * acc;
         }
         __syncthreads();
         // U = Tt diag(beta) R
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
+        GBWD_FOR(idx, kC * DC) {
+            const int i = idx / DC, j = idx % DC;
             float acc = 0.f;
-            for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * R[l * D + j];
+            for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * R[l * DC + j];
             U[idx] = acc;
         }
         __syncthreads();
         // H <- e^{gc_last} H + Kd^T U
         const float elast = expf(gc[kC - 1]);
-        GBWD_FOR(idx, D * D) {
-            const int l = idx / D, j = idx % D;
+        GBWD_FOR(idx, D * DC) {
+            const int l = idx / DC, j = idx % DC;
             float acc = 0.f;
-            for (int i = 0; i < kC; ++i) acc += ed[i] * Kb[i * D + l] * U[i * D + j];
+            for (int i = 0; i < kC; ++i) acc += ed[i] * Kb[i * D + l] * U[i * DC + j];
             Hs[idx] = elast * Hs[idx] + acc;
         }
         __syncthreads();
     }
-    if (a.hT) GBWD_FOR(idx, D * D) a.hT[static_cast<size_t>(bh) * D * D + idx] = Hs[idx];
+    if (a.hT)
+        GBWD_FOR(idx, D * DC) a.hT[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] = Hs[idx];
 }
 
 // Per chunk, everything that does not need dH: z, qc, R, U, dqc, dq, dlambda, the CCQ
@@ -534,26 +547,31 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
 
 // Per sequence and head, chunks last to first: the adjoint dH of the state leaving every
 // chunk (stored), then carried into the chunk: dU = P^T D + Kd dH, dR = diag(beta) Tt^T dU,
-// dH <- e^{gc_last} dH + (diag(E) Qc)^T D - (diag(E) Kbar)^T dR.  Writes dS0.
+// dH <- e^{gc_last} dH + (diag(E) Qc)^T D - (diag(E) Kbar)^T dR.  Writes dS0.  Like the
+// forward pass, CTA (sequence-head, s) carries the value columns [s D/nsplit, (s+1) D/nsplit).
 template <int D, typename Tin>
 __global__ void __launch_bounds__(512) gdn_bwd_dstate_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
+    const int ns = a.nsplit, DC = D / ns;
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *dH = sm;               // [D][D]
-    float *Kb = dH + D * D;       // [64][D]
-    float *dU = Kb + kC * D;      // [64][D]
-    float *dR = dU + kC * D;      // [64][D]
-    float *Tt = dR + kC * D;      // [64][64]
+    float *dH = sm;               // [D][DC]
+    float *Kb = dH + D * DC;      // [64][D]
+    float *dU = Kb + kC * D;      // [64][DC]
+    float *dR = dU + kC * DC;     // [64][DC]
+    float *Tt = dR + kC * DC;     // [64][64]
     float *graw = Tt + kC * kC;   // [64]
     float *gc = graw + kC, *be = gc + kC, *rk = be + kC, *E = rk + kC, *ed = E + kC;
 
-    const int bh = blockIdx.x, b = bh / a.H, h = bh % a.H;
-    GBWD_FOR(idx, D * D) dH[idx] = a.dST ? a.dST[static_cast<size_t>(bh) * D * D + idx] : 0.f;
+    const int bh = blockIdx.x / ns, c0 = (blockIdx.x % ns) * DC, b = bh / a.H, h = bh % a.H;
+    GBWD_FOR(idx, D * DC) {
+        const int l = idx / DC, j = idx % DC;
+        dH[idx] = a.dST ? a.dST[(static_cast<size_t>(bh) * D + l) * D + c0 + j] : 0.f;
+    }
     __syncthreads();
     for (int r = a.NC - 1; r >= 0; --r) {
         const size_t ch = static_cast<size_t>(bh) * a.NC + r;
         float *dhg = a.dh + ch * D * D;
-        GBWD_FOR(idx, D * D) dhg[idx] = dH[idx];
+        GBWD_FOR(idx, D * DC) dhg[(idx / DC) * D + c0 + idx % DC] = dH[idx];
         load_tile<D, Tin>(Kb, a.k, a, b, h, r);
         const float *tt = a.tt + ch * kC * kC;
         GBWD_FOR(idx, kC * kC) Tt[idx] = tt[idx];
@@ -574,31 +592,32 @@ __global__ void __launch_bounds__(512) gdn_bwd_dstate_kernel(const GdnBwdArgs a)
         }
         __syncthreads();
         const float *X1 = a.x1 + ch * kC * D;
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
+        GBWD_FOR(idx, kC * DC) {
+            const int i = idx / DC, j = idx % DC;
             float acc = 0.f;
-            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * dH[l * D + j];
-            dU[idx] = X1[idx] + ed[i] * acc;
+            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * dH[l * DC + j];
+            dU[idx] = X1[i * D + c0 + j] + ed[i] * acc;
         }
         __syncthreads();
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
+        GBWD_FOR(idx, kC * DC) {
+            const int i = idx / DC, j = idx % DC;
             float acc = 0.f;
-            for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * dU[l * D + j];
+            for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * dU[l * DC + j];
             dR[idx] = be[i] * acc;
         }
         __syncthreads();
         const float *Y1 = a.y1 + ch * D * D;
         const float elast = expf(gc[kC - 1]);
-        GBWD_FOR(idx, D * D) {
-            const int p = idx / D, j = idx % D;
+        GBWD_FOR(idx, D * DC) {
+            const int p = idx / DC, j = idx % DC;
             float acc = 0.f;
-            for (int i = 0; i < kC; ++i) acc += E[i] * Kb[i * D + p] * dR[i * D + j];
-            dH[idx] = elast * dH[idx] + Y1[idx] - acc;
+            for (int i = 0; i < kC; ++i) acc += E[i] * Kb[i * D + p] * dR[i * DC + j];
+            dH[idx] = elast * dH[idx] + Y1[p * D + c0 + j] - acc;
         }
         __syncthreads();
     }
-    if (a.dS0) GBWD_FOR(idx, D * D) a.dS0[static_cast<size_t>(bh) * D * D + idx] = dH[idx];
+    if (a.dS0)
+        GBWD_FOR(idx, D * DC) a.dS0[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] = dH[idx];
 }
 
 // Exclusive suffix over the chunks of each sequence and head of the CCQ increments:
@@ -870,9 +889,21 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
 
 // Shared-memory bytes of each kernel.
 template <int D> constexpr size_t prep_smem() { return sizeof(float) * (kC * D + 2 * kC * kC + 4 * kC); }
-template <int D> constexpr size_t fstate_smem() { return sizeof(float) * (D * D + 3 * kC * D + kC * kC + 6 * kC); }
+template <int D> constexpr size_t fstate_smem(int ns) {
+    return sizeof(float) * (D * (D / ns) + kC * D + 2 * kC * (D / ns) + kC * kC + 6 * kC);
+}
 template <int D> constexpr size_t local_smem() { return sizeof(float) * (5 * kC * D + 2 * kC * kC + 12 * kC); }
-template <int D> constexpr size_t dstate_smem() { return sizeof(float) * (D * D + 3 * kC * D + kC * kC + 6 * kC); }
+template <int D> constexpr size_t dstate_smem(int ns) {
+    return sizeof(float) * (D * (D / ns) + kC * D + 2 * kC * (D / ns) + kC * kC + 6 * kC);
+}
+
+// Value-column blocks of the sequential passes: the most (up to 4) that keep the CTAs within
+// about two per SM of a 152-SM GPU.
+inline int seq_split(int B, int H) {
+    int ns = 1;
+    while (ns < 4 && static_cast<long long>(B) * H * ns * 2 <= 304) ns *= 2;
+    return ns;
+}
 template <int D> constexpr size_t kv_smem() { return sizeof(float) * (4 * kC * D + 3 * kC * kC + 16 * kC + 4); }
 
 }  // namespace gbwd

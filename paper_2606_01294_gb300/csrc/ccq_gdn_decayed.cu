@@ -28,14 +28,14 @@ cudaError_t run(const gbwd::GdecArgs &g, cudaStream_t s) {
     const GdnBwdArgs &a = g.base;
     cudaError_t e;
     if ((e = allow_smem(gdn_bwd_prep_kernel<D, Tin>, prep_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_fstate_kernel<D, Tin>, fstate_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_fstate_kernel<D, Tin>, fstate_smem<D>(a.nsplit))) != cudaSuccess) return e;
     if ((e = allow_smem(gdec_stats_kernel<D, Tin>, gdec_stats_smem<D>())) != cudaSuccess) return e;
     if ((e = allow_smem(gdec_out_kernel<D, Tin>, gdec_out_smem<D>())) != cudaSuccess) return e;
     const unsigned nch = static_cast<unsigned>(a.B * a.H * a.NC), bh = static_cast<unsigned>(a.B * a.H);
     const long long elems = (static_cast<long long>(D) * D + D + 1) * a.B * a.H;
     const unsigned eblocks = static_cast<unsigned>((elems + 255) / 256);
     gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
-    gdn_bwd_fstate_kernel<D, Tin><<<bh, 512, fstate_smem<D>(), s>>>(a);
+    gdn_bwd_fstate_kernel<D, Tin><<<bh * a.nsplit, 512, fstate_smem<D>(a.nsplit), s>>>(a);
     gdec_stats_kernel<D, Tin><<<nch, 256, gdec_stats_smem<D>(), s>>>(g);
     gdec_scan_kernel<D><<<eblocks, 256, 0, s>>>(g);
     gdec_out_kernel<D, Tin><<<nch, 256, gdec_out_smem<D>(), s>>>(g);
@@ -53,6 +53,7 @@ cudaError_t launch_gdn_decayed(const GdecCall &c, cudaStream_t s) {
     gbwd::GdecArgs g{};
     gbwd::GdnBwdArgs &a = g.base;
     a.B = c.B; a.T = c.T; a.H = c.H; a.NC = (c.T + 63) / 64;
+    a.nsplit = gbwd::seq_split(c.B, c.H);
     a.l2norm = c.l2norm; a.centered = c.centered; a.scale = c.scale;
     a.q = c.q; a.k = c.k; a.v = c.v;
     a.g = c.g; a.beta = c.beta; a.lambda = c.lambda;

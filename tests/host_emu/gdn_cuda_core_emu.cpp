@@ -66,9 +66,9 @@ static void run(const GdnBwdArgs &a) {
     const long long elems = (static_cast<long long>(D) * D + D) * bh;
     run_blocks([&] { gdn_bwd_prep_kernel<D, Tin>(a); }, nch, prep_smem<D>());
     run_blocks([&] { gdn_bwd_prefix_kernel<D>(a); }, elems, 0);
-    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh, fstate_smem<D>());
+    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh * a.nsplit, fstate_smem<D>(a.nsplit));
     run_blocks([&] { gdn_bwd_local_kernel<D, Tin>(a); }, nch, local_smem<D>());
-    run_blocks([&] { gdn_bwd_dstate_kernel<D, Tin>(a); }, bh, dstate_smem<D>());
+    run_blocks([&] { gdn_bwd_dstate_kernel<D, Tin>(a); }, bh * a.nsplit, dstate_smem<D>(a.nsplit));
     run_blocks([&] { gdn_bwd_suffix_kernel<D>(a); }, elems, 0);
     run_blocks([&] { gdn_bwd_kv_kernel<D, Tin>(a); }, nch, kv_smem<D>());
 }
@@ -96,6 +96,7 @@ static int go(int B, int T, int H, int l2norm, int centered, float scale, const 
     std::vector<Tin> dq(ntok), dk(ntok), dv(ntok);
     GdnBwdArgs a{};
     a.B = B; a.T = T; a.H = H; a.NC = (T + 63) / 64;
+    a.nsplit = 1 << (T % 3);  // 1, 2 or 4 value-column blocks in the sequential passes, by T
     a.l2norm = l2norm; a.centered = centered; a.scale = scale;
     a.q = q.data(); a.k = k.data(); a.v = v.data(); a.dout = dout.data();
     a.g = in[4]; a.beta = in[5]; a.lambda = in[6]; a.S0 = in[7]; a.C0 = in[8]; a.m0 = in[9]; a.t0 = t0;
@@ -135,6 +136,7 @@ static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, co
     GdecArgs g{};
     GdnBwdArgs &a = g.base;
     a.B = B; a.T = T; a.H = H; a.NC = (T + 63) / 64;
+    a.nsplit = 1 << (T % 3);  // 1, 2 or 4 value-column blocks in the sequential passes, by T
     a.l2norm = l2norm; a.centered = centered; a.scale = scale;
     a.q = q.data(); a.k = k.data(); a.v = v.data();
     a.g = in[3]; a.beta = in[4]; a.lambda = in[5]; a.S0 = in[6]; a.C0 = in[7]; a.m0 = in[8];
@@ -149,7 +151,7 @@ static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, co
     g.dC = take(d * d); g.dmv = take(d); g.dn = take(4);
     const long long nch = static_cast<long long>(chunks), bh = static_cast<long long>(B) * H;
     run_blocks([&] { gdn_bwd_prep_kernel<D, Tin>(a); }, nch, prep_smem<D>());
-    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh, fstate_smem<D>());
+    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh * a.nsplit, fstate_smem<D>(a.nsplit));
     run_blocks([&] { gdec_stats_kernel<D, Tin>(g); }, nch, gdec_stats_smem<D>());
     run_blocks([&] { gdec_scan_kernel<D>(g); }, (static_cast<long long>(D) * D + D + 1) * bh, 0);
     run_blocks([&] { gdec_out_kernel<D, Tin>(g); }, nch, gdec_out_smem<D>());
