@@ -170,3 +170,57 @@ def test_gla_fwd_save_rejects_bad_checkpoint_buffer(lib):
     st = lib.ccq_gla_fwd_save(*([fake] * 5), 1, 1, *([None] * 4), fake, *([None] * 4), 1, 64, 1, 128, 128,
                               None, 0, fake, 1 << 20, p, None)
     assert st == ccq.CCQ_ERR_UNSUPPORTED  # fp32 inputs have no checkpointing path
+
+
+def _gdn_bwd(lib, ptrs=None, sizes=(1, 70, 2, 64, 64), ws=None, ws_bytes=0, dtype=1, opt=None):
+    fake = ctypes.c_void_p(0x10000)
+    req = ptrs if ptrs is not None else [fake] * 6
+    o = opt or {}
+    # q, k, v, g, beta, lambda, in_dtype, S0, C0, m0, t0, dout, dST, dCT, dmT, dq, dk, dv, dg, dbeta,
+    # dlambda, dS0, dC0, dm0
+    return lib.ccq_gdn_bwd(*req, dtype, o.get("S0"), None, None, None, fake, None, None, None,
+                           fake, fake, fake, fake, fake, None, None, None, None,
+                           *sizes, ws, ws_bytes, ctypes.byref(ccq.params()), None)
+
+
+def test_gdn_bwd_workspace_size_and_rejections(lib):
+    need = ctypes.c_size_t(0)
+    p = ccq.params()
+    assert lib.ccq_gdn_bwd_workspace_size(4, 4096, 16, 128, 128, 0, ctypes.byref(p), ctypes.byref(need)) == 0
+    chunks = 4 * 16 * 64
+    assert need.value == chunks * (64 * 64 + 5 * 128 * 128 + 2 * 128 + 6 * 64 * 128 + 4 * 64) * 4
+    assert lib.ccq_gdn_bwd_workspace_size(1, 0, 2, 64, 64, 1, ctypes.byref(p), ctypes.byref(need)) == 0
+    assert need.value == 0
+    assert lib.ccq_gdn_bwd_workspace_size(1, 64, 2, 96, 96, 1, ctypes.byref(p),
+                                          ctypes.byref(need)) == ccq.CCQ_ERR_UNSUPPORTED
+    fake = ctypes.c_void_p(0x10000)
+    assert _gdn_bwd(lib, [None] + [fake] * 5) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gdn_bwd(lib, sizes=(1, 70, 0, 64, 64)) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gdn_bwd(lib, dtype=5) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gdn_bwd(lib, opt={"S0": ctypes.c_void_p(0x10004)}) == ccq.CCQ_ERR_INVALID_ARG
+    # a workspace one byte short of the size is refused before any launch
+    lib.ccq_gdn_bwd_workspace_size(1, 70, 2, 64, 64, 1, ctypes.byref(p), ctypes.byref(need))
+    assert _gdn_bwd(lib, ws=fake, ws_bytes=need.value - 1) == ccq.CCQ_ERR_INVALID_ARG
+    assert b"workspace" in lib.ccq_last_error()
+
+
+def _gdn_dec(lib, ptrs=None, sizes=(1, 70, 2, 64, 64), ws=None, ws_bytes=0, dtype=1):
+    fake = ctypes.c_void_p(0x10000)
+    req = ptrs if ptrs is not None else [fake] * 6
+    # q, k, v, g, beta, lambda, in_dtype, S0, C0, m0, n0, o, ST, CT, mT, nT
+    return lib.ccq_gdn_fwd_decayed(*req, dtype, None, None, None, None, fake, None, None, None, None,
+                                   *sizes, ws, ws_bytes, ctypes.byref(ccq.params()), None)
+
+
+def test_gdn_decayed_workspace_size_and_rejections(lib):
+    need = ctypes.c_size_t(0)
+    p = ccq.params()
+    assert lib.ccq_gdn_decayed_workspace_size(8, 4096, 16, 128, 128, 0, ctypes.byref(p),
+                                              ctypes.byref(need)) == 0
+    assert need.value == 8 * 16 * 64 * (64 * 64 + 3 * 128 * 128 + 2 * 128 + 4) * 4
+    fake = ctypes.c_void_p(0x10000)
+    assert _gdn_dec(lib, [fake] * 5 + [None]) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gdn_dec(lib, sizes=(1, 70, 2, 128, 64)) == ccq.CCQ_ERR_UNSUPPORTED
+    assert _gdn_dec(lib, dtype=3) == ccq.CCQ_ERR_INVALID_ARG
+    assert _gdn_dec(lib) == ccq.CCQ_ERR_INVALID_ARG  # no workspace
+    assert b"workspace" in lib.ccq_last_error()
