@@ -23,6 +23,12 @@ Parity status of each routine (what pins it is in ``tests/test_oracle_pins.py``)
                      by brute-force weighted covariances, the undecayed special case,
                      the spectrum bound and resumption (tests/test_oracle_decayed.py);
                      the reference of the ccq_gdn_fwd_decayed parity tests.
+  gdn_forward_spectral  CCQ-Gated-DeltaNet with the read contracted by I - x, (I + x)^{-1}
+                     or exp(-x), x = lambda Sigma (the paper's operator and the two
+                     alternatives it names), undecayed or decay-aligned statistics; numpy,
+                     token by token -- pinned against the C oracle (linear case), explicit
+                     eigendecompositions, the first-order agreement in lambda and the
+                     spectrum bounds (tests/test_oracle_spectral.py).
   Absolute outputs on the benchmark-shaped random inputs are pinned only
   through the above: the paper prints no worked numerical example.
 """
@@ -33,6 +39,10 @@ from .ccq_oracle import (  # noqa: F401
     gla_backward,
     gdn_backward,
     gdn_forward_decayed,
+    gdn_forward_spectral,
     GLA,
     GDN,
+    LINEAR,
+    RESOLVENT,
+    EXPONENTIAL,
 )

@@ -243,3 +243,73 @@ def gdn_forward_decayed(q, k, v, g, beta, lam, S0=None, C0=None, m0=None, n0=Non
     if want_qclean:
         out["qclean"] = qc
     return out
+
+
+# Spectral contractions of the CCQ read (Sec. 3.2, after Eq. clean): the paper's operator
+# I - lambda Sigma is the first-order form of (I + lambda Sigma)^{-1} and exp(-lambda Sigma).
+LINEAR, RESOLVENT, EXPONENTIAL = 0, 1, 2
+
+
+def gdn_forward_spectral(q, k, v, g, beta, lam, *, contraction=LINEAR, decayed=False, S0=None, C0=None,
+                         m0=None, n0=None, l2norm=True, centered=True, scale=None, want_qclean=False):
+    """CCQ-Gated-DeltaNet forward with the query contracted by f(lambda_t Sigma_t), f one of
+    the spectral contractions I - x (the paper's), (I + x)^{-1} or exp(-x) that the paper names
+    as alternatives with the same first-order form.  Plain numpy, token by token, in fp64:
+
+      statistics (Sec. 3.2): C += kbar kbar^T, m += kbar, n += 1 -- or, with ``decayed``, the
+        decay-aligned reading (C, m, n first multiplied by the token's alpha);
+      Sigma = C/n - c (m/n)(m/n)^T  (c = 1 centred, 0 uncentred);
+      q_clean = qbar - lambda Sigma qbar | solve((I + lambda Sigma), qbar) | expm(-lambda Sigma) qbar;
+      S = alpha S (I - beta kbar kbar^T) + beta v kbar^T (the Gated DeltaNet write, stored as
+        H = S^T);  o = scale S q_clean.
+
+    q, k [B,T,H,Dk]; v [B,T,H,Dv]; g, beta, lam [B,T,H]; S0 [B,H,Dk,Dv]; C0 [B,H,Dk,Dk];
+    m0 [B,H,Dk]; n0 [B,H] (the count entering, t0 for the undecayed statistics).  Returns
+    dict o, S, C, m, n (and qclean [B,T,H,Dk] when asked)."""
+    import scipy.linalg
+
+    q, k, v, g, beta, lam = map(_f64, (q, k, v, g, beta, lam))
+    B, T, H, Dk = q.shape
+    Dv = v.shape[-1]
+    scale = Dk ** -0.5 if scale is None else scale
+    c = 1.0 if centered else 0.0
+    out = {"o": np.zeros((B, T, H, Dv)), "S": np.zeros((B, H, Dk, Dv)), "C": np.zeros((B, H, Dk, Dk)),
+           "m": np.zeros((B, H, Dk)), "n": np.zeros((B, H))}
+    if want_qclean:
+        out["qclean"] = np.zeros((B, T, H, Dk))
+
+    def unit(x):
+        nrm = np.linalg.norm(x)
+        return x / nrm if (l2norm and nrm > 0) else (x.copy() if not l2norm else np.zeros_like(x))
+
+    for b in range(B):
+        for h in range(H):
+            Hs = np.zeros((Dk, Dv)) if S0 is None else _f64(S0)[b, h].copy()
+            C = np.zeros((Dk, Dk)) if C0 is None else _f64(C0)[b, h].copy()
+            m = np.zeros(Dk) if m0 is None else _f64(m0)[b, h].copy()
+            n = 0.0 if n0 is None else float(_f64(n0)[b, h])
+            for t in range(T):
+                qb, kb = unit(q[b, t, h]), unit(k[b, t, h])
+                a = np.exp(g[b, t, h])
+                if decayed:
+                    C, m, n = a * C, a * m, a * n
+                C = C + np.outer(kb, kb)
+                m = m + kb
+                n = n + 1.0
+                Sig = C / n - c * np.outer(m / n, m / n)
+                x = lam[b, t, h] * Sig
+                if contraction == LINEAR:
+                    qc = qb - x @ qb
+                elif contraction == RESOLVENT:
+                    qc = np.linalg.solve(np.eye(Dk) + x, qb)
+                elif contraction == EXPONENTIAL:
+                    qc = scipy.linalg.expm(-x) @ qb
+                else:
+                    raise ValueError("unknown contraction")
+                if want_qclean:
+                    out["qclean"][b, t, h] = qc
+                u = beta[b, t, h] * (v[b, t, h] - a * (kb @ Hs))
+                Hs = a * Hs + np.outer(kb, u)
+                out["o"][b, t, h] = scale * (qc @ Hs)
+            out["S"][b, h], out["C"][b, h], out["m"][b, h], out["n"][b, h] = Hs, C, m, n
+    return out
