@@ -65,6 +65,14 @@ typedef enum {
 
 typedef enum { CCQ_BF16 = 0, CCQ_FP32 = 1 } ccq_dtype;
 
+/* Spectral contraction of the query (ccq_gdn_fwd_spectral): the paper's first-order operator
+   and the two alternatives it names with that first-order form (Sec. 3.2, after Eq. clean). */
+typedef enum {
+    CCQ_CONTRACT_LINEAR = 0,     /* q_clean = (I - lambda Sigma) qbar (the paper's CCQ)      */
+    CCQ_CONTRACT_RESOLVENT = 1,  /* q_clean = (I + lambda Sigma)^{-1} qbar                   */
+    CCQ_CONTRACT_EXPONENTIAL = 2 /* q_clean = exp(-lambda Sigma) qbar                        */
+} ccq_contraction;
+
 typedef enum {
     CCQ_ALGO_AUTO = 0,      /* chunkwise tensor-core kernel when supported, else recurrent */
     CCQ_ALGO_RECURRENT = 1, /* token-by-token CUDA-core kernel (fp32 arithmetic)         */
@@ -288,7 +296,31 @@ CCQ_API ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void 
                                        int B, int T, int H, int Dk, int Dv, void *workspace,
                                        size_t workspace_bytes, const ccq_params *p, void *stream);
 
-/* Workspace bytes ccq_gdn_fwd_decayed needs for these sizes (0 when T = 0).  Host-only. */
+/*
+ * CCQ-Gated-DeltaNet forward with a choice of spectral contraction and of covariance
+ * statistics, on the same CUDA-core kernels as ccq_gdn_fwd_decayed.
+ *   contraction  a ccq_contraction value.  RESOLVENT runs ten conjugate-gradient iterations
+ *                per query from the linear estimate (I + lambda Sigma has spectrum in
+ *                [1, 1 + lambda] for unit keys); EXPONENTIAL sums twelve Taylor terms
+ *                (|lambda Sigma| <= 1).  Both assume unit-norm keys (l2norm_qk = 1, or keys of
+ *                norm at most 1).
+ *   decayed      1: the decay-aligned statistics of ccq_gdn_fwd_decayed (n the decayed count);
+ *                0: the paper's undecayed sums, C_t = sum kbar kbar^T, m_t = sum kbar, with n
+ *                the token count t (n0/nT [B,H] fp32 carry it) -- with LINEAR this is the
+ *                paper's CCQ-Gated-DeltaNet, computed in fp32 on the CUDA cores.
+ * Other arguments, the workspace (ccq_gdn_decayed_workspace_size) and the supported sizes as
+ * ccq_gdn_fwd_decayed, which equals this call with LINEAR and decayed = 1.
+ */
+CCQ_API ccq_status ccq_gdn_fwd_spectral(const void *q, const void *k, const void *v, const float *g,
+                                        const float *beta, const float *lambda, ccq_dtype in_dtype,
+                                        const float *S0, const float *C0, const float *m0, const float *n0,
+                                        void *o, float *ST, float *CT, float *mT, float *nT,
+                                        int B, int T, int H, int Dk, int Dv, int contraction, int decayed,
+                                        void *workspace, size_t workspace_bytes, const ccq_params *p,
+                                        void *stream);
+
+/* Workspace bytes ccq_gdn_fwd_decayed and ccq_gdn_fwd_spectral need for these sizes (0 when
+   T = 0).  Host-only. */
 CCQ_API ccq_status ccq_gdn_decayed_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
                                                   const ccq_params *p, size_t *bytes);
 

@@ -103,6 +103,9 @@ def load_library() -> ctypes.CDLL:
         lib.ccq_gdn_fwd_decayed.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 5
                                             + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
         lib.ccq_gdn_fwd_decayed.restype = _I
+        lib.ccq_gdn_fwd_spectral.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 7
+                                             + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
+        lib.ccq_gdn_fwd_spectral.restype = _I
         lib.ccq_gdn_decayed_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
                                                                    ctypes.POINTER(ctypes.c_size_t)])
         lib.ccq_gdn_decayed_workspace_size.restype = _I
@@ -450,12 +453,19 @@ def gdn_bwd(q, k, v, g, beta, lam, dout, state: Optional[CCQState] = None, *, dS
     return grads
 
 
+CONTRACTION = {"linear": 0, "resolvent": 1, "exponential": 2}
+
+
 def gdn_fwd_decayed(q, k, v, g, beta, lam, *, S0=None, C0=None, m0=None, n0=None, out=None,
-                    return_state: bool = True, workspace=None, stream=None, **kw):
-    """CCQ-Gated-DeltaNet forward with the decay-aligned covariance (statistics decayed by the
-    backbone's own decay, normalised by the decayed count n).  S0 [B,H,Dk,Dv], C0 [B,H,Dk,Dk],
-    m0 [B,H,Dk], n0 [B,H] fp32 (None = zero).  Returns o, or (o, dict S, C, m, n of final
-    states) when ``return_state``."""
+                    return_state: bool = True, workspace=None, stream=None, contraction="linear",
+                    decayed: bool = True, **kw):
+    """CCQ-Gated-DeltaNet forward on the CUDA-core kernels with the decay-aligned covariance
+    (statistics decayed by the backbone's own decay, normalised by the decayed count n) or,
+    with ``decayed=False``, the paper's undecayed statistics (n = the token count), and the
+    query contracted by ``contraction``: "linear" (the paper's I - lambda Sigma),
+    "resolvent" ((I + lambda Sigma)^{-1}) or "exponential" (exp(-lambda Sigma)).
+    S0 [B,H,Dk,Dv], C0 [B,H,Dk,Dk], m0 [B,H,Dk], n0 [B,H] fp32 (None = zero).  Returns o, or
+    (o, dict S, C, m, n of final states) when ``return_state``."""
     dev = q.device
     B, T, H, Dk = q.shape
     Dv = v.shape[-1]
@@ -484,12 +494,12 @@ def gdn_fwd_decayed(q, k, v, g, beta, lam, *, S0=None, C0=None, m0=None, n0=None
     if workspace is None and need.value:
         workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
-    st = lib.ccq_gdn_fwd_decayed(
+    st = lib.ccq_gdn_fwd_spectral(
         _ptr(q), _ptr(k), _ptr(v), _ptr(g), _ptr(beta), _ptr(lam), _dtype_code(q),
         _ptr(S0), _ptr(C0), _ptr(m0), _ptr(n0), _ptr(o),
         _ptr(fs["S"] if fs else None), _ptr(fs["C"] if fs else None), _ptr(fs["m"] if fs else None),
-        _ptr(fs["n"] if fs else None), B, T, H, Dk, Dv, _ptr(workspace), ws_bytes, ctypes.byref(p),
-        _stream(dev, stream))
+        _ptr(fs["n"] if fs else None), B, T, H, Dk, Dv, CONTRACTION[contraction], int(bool(decayed)),
+        _ptr(workspace), ws_bytes, ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
 

@@ -644,12 +644,15 @@ ccq_status ccq_gdn_decayed_workspace_size(int B, int T, int H, int Dk, int Dv, c
     return CCQ_OK;
 }
 
-ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, const float *g,
-                               const float *beta, const float *lambda, ccq_dtype in_dtype,
-                               const float *S0, const float *C0, const float *m0, const float *n0,
-                               void *o, float *ST, float *CT, float *mT, float *nT, int B, int T, int H,
-                               int Dk, int Dv, void *workspace, size_t workspace_bytes,
-                               const ccq_params *p, void *stream) {
+ccq_status ccq_gdn_fwd_spectral(const void *q, const void *k, const void *v, const float *g,
+                                const float *beta, const float *lambda, ccq_dtype in_dtype,
+                                const float *S0, const float *C0, const float *m0, const float *n0,
+                                void *o, float *ST, float *CT, float *mT, float *nT, int B, int T, int H,
+                                int Dk, int Dv, int contraction, int decayed, void *workspace,
+                                size_t workspace_bytes, const ccq_params *p, void *stream) {
+    if (contraction < CCQ_CONTRACT_LINEAR || contraction > CCQ_CONTRACT_EXPONENTIAL)
+        return fail(CCQ_ERR_INVALID_ARG, "unknown contraction %d", contraction);
+    if (decayed != 0 && decayed != 1) return fail(CCQ_ERR_INVALID_ARG, "decayed must be 0 or 1");
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
@@ -685,9 +688,21 @@ ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, cons
     a.S0 = S0; a.C0 = C0; a.m0 = m0; a.n0 = n0;
     a.o = o; a.ST = ST; a.CT = CT; a.mT = mT; a.nT = nT;
     a.workspace = workspace;
+    a.cov_decay = decayed;
+    a.contraction = contraction;
     cudaError_t e = launch_gdn_decayed(a, s);
-    if (e != cudaSuccess) return cuda_fail(e, "decayed-covariance Gated DeltaNet launch");
+    if (e != cudaSuccess) return cuda_fail(e, "CUDA-core Gated DeltaNet launch");
     return CCQ_OK;
+}
+
+ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, const float *g,
+                               const float *beta, const float *lambda, ccq_dtype in_dtype,
+                               const float *S0, const float *C0, const float *m0, const float *n0,
+                               void *o, float *ST, float *CT, float *mT, float *nT, int B, int T, int H,
+                               int Dk, int Dv, void *workspace, size_t workspace_bytes,
+                               const ccq_params *p, void *stream) {
+    return ccq_gdn_fwd_spectral(q, k, v, g, beta, lambda, in_dtype, S0, C0, m0, n0, o, ST, CT, mT, nT, B, T, H,
+                                Dk, Dv, CCQ_CONTRACT_LINEAR, 1, workspace, workspace_bytes, p, stream);
 }
 
 ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,

@@ -35,6 +35,8 @@ struct GdecCall {
     void *o;
     float *ST, *CT, *mT, *nT;
     void *workspace;
+    int cov_decay = 1;    // 1: decay-aligned statistics; 0: the paper's undecayed ones (n = t)
+    int contraction = 0;  // 0: I - lambda Sigma; 1: (I + lambda Sigma)^{-1}; 2: exp(-lambda Sigma)
 };
 size_t gdn_decayed_workspace_bytes(int B, int T, int H, int D);
 cudaError_t launch_gdn_decayed(const GdecCall &c, cudaStream_t s);

@@ -60,6 +60,7 @@ cudaError_t launch_gdn_decayed(const GdecCall &c, cudaStream_t s) {
     a.S0 = c.S0; a.C0 = c.C0; a.m0 = c.m0;
     a.hT = c.ST;
     g.n0 = c.n0; g.o = c.o; g.CT = c.CT; g.mT = c.mT; g.nT = c.nT;
+    g.cov_decay = c.cov_decay; g.contraction = c.contraction;
     const size_t chunks = static_cast<size_t>(c.B) * c.H * a.NC;
     const size_t d = static_cast<size_t>(c.D);
     float *p = static_cast<float *>(c.workspace);

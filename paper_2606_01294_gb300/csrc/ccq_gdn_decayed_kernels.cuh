@@ -12,7 +12,13 @@
 //   C_i qbar_i = E_i C_r qbar_i + sum_{j<=i} Gamma_ij (kbar_j . qbar_i) kbar_j,
 //   m_i = E_i m_r + sum_{j<=i} Gamma_ij kbar_j,  n_i = E_i n_r + sum_{j<=i} Gamma_ij,
 // (E_i = e^{gc_i}, Gamma_ij = e^{gc_i - gc_j}, gc the in-chunk cumulative log decay), and the
-// output is the Gated DeltaNet chunk form O = scale (diag(E) Qc H_r + P U).  Launches: the
+// output is the Gated DeltaNet chunk form O = scale (diag(E) Qc H_r + P U).  With cov_decay = 0
+// the statistics are the paper's undecayed sums (E and Gamma replaced by 1 in them, n = t).
+// The contraction is the paper's q_clean = qbar - lambda Sigma qbar, or one of the two
+// alternatives it names with that first-order form: (I + lambda Sigma)^{-1} qbar by conjugate
+// gradients per row (I + lambda Sigma is symmetric with spectrum in [1, 1 + lambda], so ten
+// iterations from the linear estimate leave an error below 1e-6 relative), or
+// exp(-lambda Sigma) qbar by its Taylor series (|lambda Sigma| <= 1: twelve terms leave 1e-10).  Launches: the
 // backward's gdn_bwd_prep_kernel (Tt) and gdn_bwd_fstate_kernel (H_r, S_T), then
 //   gdec_stats_kernel  per chunk: the chunk's decayed increments of C, m, n and its decay
 //   gdec_scan_kernel   the statistics entering every chunk, and the final ones
@@ -35,7 +41,12 @@ struct GdecArgs {
     float *dC;                 // [D][D]
     float *dmv;                // [D]
     float *dn;                 // [4]: increment of n, the chunk's total decay e^{gc_last}, spare
+    int cov_decay = 1;         // 1: decay-aligned statistics; 0: the paper's undecayed ones
+    int contraction = 0;       // 0: I - lambda Sigma; 1: (I + lambda Sigma)^{-1}; 2: exp(-lambda Sigma)
 };
+
+constexpr int kCgIters = 10;   // conjugate-gradient iterations of the resolvent contraction
+constexpr int kExpTerms = 12;  // Taylor terms of the exponential contraction
 
 // Per chunk: dC = sum_j e^{gc_last - gc_j} kbar_j kbar_j^T, dm likewise, dn = sum over the
 // chunk's tokens of e^{gc_last - gc_j}, and the chunk's decay e^{gc_last}.
@@ -60,7 +71,7 @@ __global__ void __launch_bounds__(256) gdec_stats_kernel(const GdecArgs g) {
     gate_prefix(graw, gc);
     __syncthreads();
     GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
-    GBWD_FOR(i, kC) w[i] = i < n ? expf(gc[kC - 1] - gc[i]) : 0.f;
+    GBWD_FOR(i, kC) w[i] = i < n ? (g.cov_decay ? expf(gc[kC - 1] - gc[i]) : 1.f) : 0.f;
     __syncthreads();
     float *dC = g.dC + static_cast<size_t>(ch) * D * D;
     GBWD_FOR(idx, D * D) {
@@ -80,7 +91,7 @@ __global__ void __launch_bounds__(256) gdec_stats_kernel(const GdecArgs g) {
         for (int i = 0; i < kC; ++i) acc += w[i];
         float *dn = g.dn + static_cast<size_t>(ch) * 4;
         dn[0] = acc;
-        dn[1] = expf(gc[kC - 1]);
+        dn[1] = g.cov_decay ? expf(gc[kC - 1]) : 1.f;
         dn[2] = dn[3] = 0.f;
     }
 }
@@ -129,22 +140,62 @@ __global__ void __launch_bounds__(256) gdec_scan_kernel(const GdecArgs g) {
     }
 }
 
-// Per chunk: q_clean with the decayed statistics, U = Tt diag(beta)(V - diag(E) Kbar H_r),
-// o = scale (diag(E) Qc H_r + P U).
+// Row-wise Sigma_i p_i for the 64 rows of a chunk (three phases): with W the covariance
+// weights (Gamma o causal, or the causal mask for undecayed statistics) and Ec_i the weight of
+// the chunk-start statistics, Sigma_i p = (Ec_i C_r p + sum_{l<=i} W_il (kbar_l . p) kbar_l) / n_i
+// - c m_i (m_i . p) / n_i^2,  m_i = Ec_i m_r + sum_{l<=i} W_il kbar_l.  Rows past n give 0.
+template <int D>
+__device__ __forceinline__ void apply_sigma(const float *P, float *out, const float *Kb, const float *Wc,
+                                            const float *Ec, const float *ninv, const float *Cr,
+                                            const float *mr, float c, float *sS, float *mp) {
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, l = idx % kC;
+        float acc = 0.f;
+        if (l <= i)
+            for (int j = 0; j < D; ++j) acc += Kb[l * D + j] * P[i * D + j];
+        sS[idx] = acc * Wc[idx];
+    }
+    __syncthreads();
+    GBWD_FOR(i, kC) {
+        float acc = 0.f;
+        for (int j = 0; j < D; ++j) acc += mr[j] * P[i * D + j];
+        acc *= Ec[i];
+        for (int l = 0; l <= i; ++l) acc += sS[i * kC + l];
+        mp[i] = acc;
+    }
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        float cp = 0.f;
+        for (int l = 0; l < D; ++l) cp += Cr[j * D + l] * P[i * D + l];
+        cp *= Ec[i];
+        float mi = Ec[i] * mr[j];
+        for (int l = 0; l <= i; ++l) {
+            cp += sS[i * kC + l] * Kb[l * D + j];
+            mi += Wc[i * kC + l] * Kb[l * D + j];
+        }
+        out[idx] = cp * ninv[i] - c * mi * mp[i] * ninv[i] * ninv[i];
+    }
+    __syncthreads();
+}
+
+// Per chunk: q_clean with the chunk's statistics and contraction,
+// U = Tt diag(beta)(V - diag(E) Kbar H_r), o = scale (diag(E) Qc H_r + P U).
 template <int D, typename Tin>
 __global__ void __launch_bounds__(256) gdec_out_kernel(const GdecArgs g) {
     extern __shared__ float4 gbwd_smem4[];
     const GdnBwdArgs &a = g.base;
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *Qb = sm;                // [64][D] qbar, then qc
+    float *Qb = sm;                // [64][D] qbar, then q_clean
     float *Kb = Qb + kC * D;       // [64][D]
-    float *Rv = Kb + kC * D;       // [64][D] V, then R
-    float *Uu = Rv + kC * D;       // [64][D] U
-    float *Zz = Uu + kC * D;       // [64][D] Sigma^gamma qbar
-    float *sA = Zz + kC * D;       // [64][64] (Qbar Kbar^T) o Gamma o causal, then P
-    float *graw = sA + kC * kC;
-    float *gc = graw + kC, *E = gc + kC, *be = E + kC, *lam = be + kC, *rq = lam + kC, *rk = rq + kC;
-    float *nn = rk + kC, *mq = nn + kC;
+    float *B1 = Kb + kC * D;       // [64][D] scratch, then R
+    float *B2 = B1 + kC * D;       // [64][D] scratch, then U
+    float *B3 = B2 + kC * D;       // [64][D] scratch
+    float *sA = B3 + kC * D;       // [64][64] scores, then P
+    float *Wc = sA + kC * kC;      // [64][64] covariance weights
+    float *graw = Wc + kC * kC;
+    float *gc = graw + kC, *E = gc + kC, *Ec = E + kC, *be = Ec + kC, *lam = be + kC, *rq = lam + kC;
+    float *rk = rq + kC, *ninv = rk + kC, *mp = ninv + kC, *rr = mp + kC, *al = rr + kC, *bt = al + kC;
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
     const int n = min(kC, a.T - r * kC);
@@ -157,7 +208,6 @@ __global__ void __launch_bounds__(256) gdec_out_kernel(const GdecArgs g) {
 
     load_tile<D, Tin>(Qb, a.q, a, b, h, r);
     load_tile<D, Tin>(Kb, a.k, a, b, h, r);
-    load_tile<D, Tin>(Rv, a.v, a, b, h, r);
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -174,59 +224,105 @@ __global__ void __launch_bounds__(256) gdec_out_kernel(const GdecArgs g) {
         Qb[idx] *= rq[idx / D];
         Kb[idx] *= rk[idx / D];
     }
-    GBWD_FOR(i, kC) E[i] = expf(gc[i]);
-    __syncthreads();
-    // decayed causal scores (diagonal included);  R = V - diag(E) Kbar H_r
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        if (j <= i) {
-            for (int l = 0; l < D; ++l) acc += Qb[i * D + l] * Kb[j * D + l];
-            acc *= expf(gc[i] - gc[j]);
-        }
-        sA[idx] = acc;
+    GBWD_FOR(i, kC) {
+        E[i] = expf(gc[i]);
+        Ec[i] = g.cov_decay ? E[i] : 1.f;
     }
+    GBWD_FOR(idx, kC * kC) {
+        const int i = idx / kC, l = idx % kC;
+        Wc[idx] = l <= i && l < n ? (g.cov_decay ? expf(gc[i] - gc[l]) : 1.f) : 0.f;
+    }
+    __syncthreads();
+    GBWD_FOR(i, kC) {
+        float cnt = Ec[i] * nr;
+        for (int l = 0; l <= i; ++l) cnt += Wc[i * kC + l];
+        ninv[i] = i < n ? 1.f / cnt : 0.f;
+    }
+    __syncthreads();
+    // q_clean (into Qb)
+    apply_sigma<D>(Qb, B3, Kb, Wc, Ec, ninv, Cr, mr, c, sA, mp);  // B3 = Sigma qbar
+    if (g.contraction == 1) {
+        // (I + lambda Sigma) x = qbar by conjugate gradients per row, from x0 = qbar - lambda Sigma qbar
+        GBWD_FOR(idx, kC * D) B1[idx] = Qb[idx] - lam[idx / D] * B3[idx];
+        __syncthreads();
+        apply_sigma<D>(B1, B3, Kb, Wc, Ec, ninv, Cr, mr, c, sA, mp);
+        GBWD_FOR(idx, kC * D) {
+            const float res = Qb[idx] - B1[idx] - lam[idx / D] * B3[idx];
+            Qb[idx] = res;  // r (qbar is no longer needed)
+            B2[idx] = res;  // p
+        }
+        __syncthreads();
+        GBWD_FOR(i, kC) {
+            float acc = 0.f;
+            for (int j = 0; j < D; ++j) acc += Qb[i * D + j] * Qb[i * D + j];
+            rr[i] = acc;
+        }
+        __syncthreads();
+        for (int it = 0; it < kCgIters; ++it) {
+            apply_sigma<D>(B2, B3, Kb, Wc, Ec, ninv, Cr, mr, c, sA, mp);
+            GBWD_FOR(idx, kC * D) B3[idx] = B2[idx] + lam[idx / D] * B3[idx];  // A p
+            __syncthreads();
+            GBWD_FOR(i, kC) {
+                float pap = 0.f;
+                for (int j = 0; j < D; ++j) pap += B2[i * D + j] * B3[i * D + j];
+                al[i] = pap > 0.f ? rr[i] / pap : 0.f;
+            }
+            __syncthreads();
+            GBWD_FOR(idx, kC * D) {
+                const int i = idx / D;
+                B1[idx] += al[i] * B2[idx];
+                Qb[idx] -= al[i] * B3[idx];
+            }
+            __syncthreads();
+            GBWD_FOR(i, kC) {
+                float acc = 0.f;
+                for (int j = 0; j < D; ++j) acc += Qb[i * D + j] * Qb[i * D + j];
+                bt[i] = rr[i] > 0.f ? acc / rr[i] : 0.f;
+                rr[i] = acc;
+            }
+            __syncthreads();
+            GBWD_FOR(idx, kC * D) B2[idx] = Qb[idx] + bt[idx / D] * B2[idx];
+            __syncthreads();
+        }
+        GBWD_FOR(idx, kC * D) Qb[idx] = B1[idx];
+    } else if (g.contraction == 2) {
+        // exp(-lambda Sigma) qbar = sum_k (-lambda Sigma)^k qbar / k!
+        GBWD_FOR(idx, kC * D) {
+            B1[idx] = Qb[idx] - lam[idx / D] * B3[idx];  // terms 0 and 1
+            B2[idx] = -lam[idx / D] * B3[idx];           // term 1
+        }
+        __syncthreads();
+        for (int k = 2; k <= kExpTerms; ++k) {
+            apply_sigma<D>(B2, B3, Kb, Wc, Ec, ninv, Cr, mr, c, sA, mp);
+            const float inv = 1.f / static_cast<float>(k);
+            GBWD_FOR(idx, kC * D) {
+                const float tv = -lam[idx / D] * inv * B3[idx];
+                B2[idx] = tv;
+                B1[idx] += tv;
+            }
+            __syncthreads();
+        }
+        GBWD_FOR(idx, kC * D) Qb[idx] = B1[idx];
+    } else {
+        GBWD_FOR(idx, kC * D) Qb[idx] -= lam[idx / D] * B3[idx];
+    }
+    __syncthreads();
+    // the Gated DeltaNet chunk: R = V - diag(E) Kbar H_r (B1), U = Tt diag(beta) R (B2)
+    load_tile<D, Tin>(B1, a.v, a, b, h, r);
+    __syncthreads();
     GBWD_FOR(idx, kC * D) {
         const int i = idx / D, j = idx % D;
         float acc = 0.f;
         for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * H[l * D + j];
-        Rv[idx] -= E[i] * acc;
+        B1[idx] -= E[i] * acc;
     }
     __syncthreads();
-    // n_i and m_i . qbar_i;  U = Tt diag(beta) R
-    GBWD_FOR(i, kC) {
-        float cnt = E[i] * nr, dot = 0.f;
-        for (int j = 0; j <= i && j < n; ++j) cnt += expf(gc[i] - gc[j]);
-        for (int l = 0; l < D; ++l) dot += mr[l] * Qb[i * D + l];
-        dot *= E[i];
-        for (int j = 0; j <= i; ++j) dot += sA[i * kC + j];
-        nn[i] = cnt;
-        mq[i] = dot;
-    }
     GBWD_FOR(idx, kC * D) {
         const int i = idx / D, j = idx % D;
         float acc = 0.f;
-        for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * Rv[l * D + j];
-        Uu[idx] = acc;
+        for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * B1[l * D + j];
+        B2[idx] = acc;
     }
-    __syncthreads();
-    // Sigma^gamma qbar = C_i qbar_i / n_i - c m_i (m_i . qbar_i) / n_i^2
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float cq = 0.f, mi = 0.f;
-        for (int l = 0; l < D; ++l) cq += Cr[j * D + l] * Qb[i * D + l];
-        cq *= E[i];
-        mi = E[i] * mr[j];
-        for (int l = 0; l <= i; ++l) {
-            cq += sA[i * kC + l] * Kb[l * D + j];
-            mi += expf(gc[i] - gc[l]) * Kb[l * D + j];
-        }
-        const float ninv = i < n ? 1.f / nn[i] : 0.f;
-        Zz[idx] = cq * ninv - c * mi * mq[i] * ninv * ninv;
-    }
-    __syncthreads();
-    GBWD_FOR(idx, kC * D) Qb[idx] -= lam[idx / D] * Zz[idx];
-    __syncthreads();
     // P = (Qc Kbar^T) o Gamma o causal
     GBWD_FOR(idx, kC * kC) {
         const int i = idx / kC, j = idx % kC;
@@ -246,14 +342,14 @@ __global__ void __launch_bounds__(256) gdec_out_kernel(const GdecArgs g) {
             float acc = 0.f;
             for (int l = 0; l < D; ++l) acc += Qb[i * D + l] * H[l * D + j];
             acc *= E[i];
-            for (int l = 0; l <= i; ++l) acc += sA[i * kC + l] * Uu[l * D + j];
+            for (int l = 0; l <= i; ++l) acc += sA[i * kC + l] * B2[l * D + j];
             o[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(a.scale * acc);
         }
     }
 }
 
 template <int D> constexpr size_t gdec_stats_smem() { return sizeof(float) * (kC * D + 4 * kC); }
-template <int D> constexpr size_t gdec_out_smem() { return sizeof(float) * (5 * kC * D + kC * kC + 9 * kC); }
+template <int D> constexpr size_t gdec_out_smem() { return sizeof(float) * (5 * kC * D + 2 * kC * kC + 14 * kC); }
 
 }  // namespace gbwd
 }  // namespace ccq

@@ -33,8 +33,9 @@ def load_gdn_emu(path):
     lib = ctypes.CDLL(path)
     lib.gdn_bwd_emu.argtypes = [ctypes.c_int] * 7 + [ctypes.c_float] + [ctypes.c_void_p] * 3
     lib.gdn_bwd_emu.restype = ctypes.c_int
-    lib.gdn_decayed_emu.argtypes = [ctypes.c_int] * 7 + [ctypes.c_float] + [ctypes.c_void_p] * 2
-    lib.gdn_decayed_emu.restype = ctypes.c_int
+    lib.gdn_spectral_emu.argtypes = [ctypes.c_int] * 7 + [ctypes.c_float, ctypes.c_int, ctypes.c_int,
+                                                          ctypes.c_void_p, ctypes.c_void_p]
+    lib.gdn_spectral_emu.restype = ctypes.c_int
     return lib
 
 

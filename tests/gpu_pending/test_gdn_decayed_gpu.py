@@ -1,6 +1,7 @@
 """GPU parity of ccq_gdn_fwd_decayed (CCQ-Gated-DeltaNet with the decay-aligned covariance)
-against the oracle's gdn_forward_decayed (pinned by brute-force weighted covariances),
-element by element: o, S_T, C_T, m_T, n_T.  fp32 inputs to 1e-4, bf16 inputs to 2e-2."""
+and ccq_gdn_fwd_spectral (the resolvent and exponential contractions) against the oracle's
+gdn_forward_decayed and gdn_forward_spectral, element by element: o, S_T, C_T, m_T, n_T.
+fp32 inputs to 1e-4, bf16 inputs to 2e-2."""
 import numpy as np
 import pytest
 import torch
@@ -74,3 +75,22 @@ def test_decayed_zero_length():
                                 S0=d(st["S"]), C0=d(st["C"]), m0=d(st["m"]), n0=d(st["n"]))
     for n in ("S", "C", "m", "n"):
         assert torch.equal(fs[n].cpu(), st[n]), n
+
+
+@pytest.mark.parametrize("contraction", ["resolvent", "exponential", "linear"])
+@pytest.mark.parametrize("decayed", [True, False])
+def test_spectral_contractions(contraction, decayed):
+    """ccq_gdn_fwd_spectral against oracle.gdn_forward_spectral (numpy solve / expm per token);
+    undecayed linear is the paper's CCQ-Gated-DeltaNet."""
+    P = gen.make_inputs(GDN, 1, 150, 2, 64, 64, dtype=torch.float32, seed=57, lam="high", keys="structured")
+    d = lambda x: x.cuda().contiguous()  # noqa: E731
+    o, fs = ccq.gdn_fwd_decayed(d(P["q"]), d(P["k"]), d(P["v"]), d(P["gate"]), d(P["beta"]), d(P["lam"]),
+                                contraction=contraction, decayed=decayed)
+    torch.cuda.synchronize()
+    ref = oracle.gdn_forward_spectral(P["q"], P["k"], P["v"], P["gate"], P["beta"], P["lam"],
+                                      contraction={"linear": oracle.LINEAR, "resolvent": oracle.RESOLVENT,
+                                                   "exponential": oracle.EXPONENTIAL}[contraction],
+                                      decayed=decayed)
+    errs = {n: rel_err(x, ref[n]) for n, x in (("o", o), ("S", fs["S"]), ("C", fs["C"]), ("m", fs["m"]),
+                                               ("n", fs["n"]))}
+    assert max(errs.values()) <= TOL[torch.float32], errs

@@ -127,8 +127,8 @@ extern "C" int gdn_bwd_emu(int D, int bf16, int B, int T, int H, int l2norm, int
 }
 
 template <int D, typename Tin>
-static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, const float *const *in,
-                  float *const *out) {
+static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, int contraction, int decayed,
+                  const float *const *in, float *const *out) {
     // in: q, k, v, g, beta, lambda, S0, C0, m0, n0;  out: o, ST, CT, mT, nT
     const size_t ntok = static_cast<size_t>(B) * T * H * D;
     auto q = to_in<Tin>(in[0], ntok), k = to_in<Tin>(in[1], ntok), v = to_in<Tin>(in[2], ntok);
@@ -142,6 +142,8 @@ static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, co
     a.g = in[3]; a.beta = in[4]; a.lambda = in[5]; a.S0 = in[6]; a.C0 = in[7]; a.m0 = in[8];
     g.n0 = in[9];
     g.o = o.data();
+    g.contraction = contraction;
+    g.cov_decay = decayed;
     a.hT = out[1]; g.CT = out[2]; g.mT = out[3]; g.nT = out[4];
     const size_t chunks = static_cast<size_t>(B) * H * a.NC, d = D;
     std::vector<float> ws(chunks * (64 * 64 + 3 * d * d + 2 * d + 4), NAN);
@@ -159,10 +161,11 @@ static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, co
     return 0;
 }
 
-extern "C" int gdn_decayed_emu(int D, int bf16, int B, int T, int H, int l2norm, int centered, float scale,
-                               const float *const *in, float *const *out) {
-    if (D == 16) return bf16 ? go_dec<16, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, out)
-                             : go_dec<16, float>(B, T, H, l2norm, centered, scale, in, out);
-    if (D == 64 && !bf16) return go_dec<64, float>(B, T, H, l2norm, centered, scale, in, out);
+extern "C" int gdn_spectral_emu(int D, int bf16, int B, int T, int H, int l2norm, int centered, float scale,
+                                int contraction, int decayed, const float *const *in, float *const *out) {
+    if (D == 16)
+        return bf16 ? go_dec<16, __nv_bfloat16>(B, T, H, l2norm, centered, scale, contraction, decayed, in, out)
+                    : go_dec<16, float>(B, T, H, l2norm, centered, scale, contraction, decayed, in, out);
+    if (D == 64 && !bf16) return go_dec<64, float>(B, T, H, l2norm, centered, scale, contraction, decayed, in, out);
     return -1;
 }

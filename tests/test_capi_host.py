@@ -224,3 +224,18 @@ def test_gdn_decayed_workspace_size_and_rejections(lib):
     assert _gdn_dec(lib, dtype=3) == ccq.CCQ_ERR_INVALID_ARG
     assert _gdn_dec(lib) == ccq.CCQ_ERR_INVALID_ARG  # no workspace
     assert b"workspace" in lib.ccq_last_error()
+
+
+def test_gdn_spectral_rejects_unknown_contraction(lib):
+    fake = ctypes.c_void_p(0x10000)
+
+    def call(contraction, decayed):
+        return lib.ccq_gdn_fwd_spectral(*([fake] * 6), 1, None, None, None, None, fake, None, None, None, None,
+                                        1, 70, 2, 64, 64, contraction, decayed, None, 0,
+                                        ctypes.byref(ccq.params()), None)
+    assert call(3, 1) == ccq.CCQ_ERR_INVALID_ARG
+    assert b"contraction" in lib.ccq_last_error()
+    assert call(-1, 0) == ccq.CCQ_ERR_INVALID_ARG
+    assert call(1, 2) == ccq.CCQ_ERR_INVALID_ARG
+    assert call(2, 0) == ccq.CCQ_ERR_INVALID_ARG      # valid request, but no workspace
+    assert b"workspace" in lib.ccq_last_error()

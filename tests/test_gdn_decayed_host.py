@@ -39,7 +39,7 @@ def problem(D, B, T, H, seed, *, bf16=False, lam=None, states=True, g_scale=1.0)
     return P
 
 
-def run_case(lib, D, P, *, bf16=False, l2norm=True, centered=True):
+def run_case(lib, D, P, *, bf16=False, l2norm=True, centered=True, contraction=0, decayed=True):
     B, T, H, _ = P["q"].shape
     scale = D ** -0.5
     names_in = ("q", "k", "v", "g", "beta", "lam", "S0", "C0", "m0", "n0")
@@ -48,10 +48,16 @@ def run_case(lib, D, P, *, bf16=False, l2norm=True, centered=True):
     ptr = lambda x: None if x is None else x.ctypes.data  # noqa: E731
     ins = (ctypes.c_void_p * 10)(*[ptr(P[n]) for n in names_in])
     outs = (ctypes.c_void_p * 5)(*[ptr(out[n]) for n in shapes])
-    assert lib.gdn_decayed_emu(D, int(bf16), B, T, H, int(l2norm), int(centered), scale, ins, outs) == 0
-    ref = oracle.gdn_forward_decayed(P["q"], P["k"], P["v"], P["g"], P["beta"], P["lam"], S0=P["S0"],
-                                     C0=P["C0"], m0=P["m0"], n0=P["n0"], l2norm=l2norm, centered=centered,
-                                     scale=scale)
+    assert lib.gdn_spectral_emu(D, int(bf16), B, T, H, int(l2norm), int(centered), scale, contraction,
+                                int(decayed), ins, outs) == 0
+    if contraction == 0 and decayed:
+        ref = oracle.gdn_forward_decayed(P["q"], P["k"], P["v"], P["g"], P["beta"], P["lam"], S0=P["S0"],
+                                         C0=P["C0"], m0=P["m0"], n0=P["n0"], l2norm=l2norm, centered=centered,
+                                         scale=scale)
+    else:
+        ref = oracle.gdn_forward_spectral(P["q"], P["k"], P["v"], P["g"], P["beta"], P["lam"],
+                                          contraction=contraction, decayed=decayed, S0=P["S0"], C0=P["C0"],
+                                          m0=P["m0"], n0=P["n0"], l2norm=l2norm, centered=centered, scale=scale)
     errs = {}
     for n in shapes:
         x = out[n].astype(np.float64)
@@ -83,3 +89,28 @@ def test_gdn_decayed_kernels_on_host(gdn_emu, oracle_mod, case):
     tol = {n: (2e-2 if bf16 and n == "o" else 1e-4) for n in errs}
     bad = {n: e for n, e in errs.items() if not e <= tol[n]}
     assert not bad, f"{case}: {errs}"
+
+
+SPECTRAL = [
+    dict(D=16, B=1, T=130, H=2, seed=11, opts=dict(contraction=1)),
+    dict(D=16, B=1, T=130, H=2, seed=12, opts=dict(contraction=2)),
+    dict(D=16, B=1, T=100, H=1, seed=13, lam=0.9, opts=dict(contraction=1, decayed=False)),
+    dict(D=16, B=1, T=100, H=1, seed=14, lam=0.9, opts=dict(contraction=2, decayed=False)),
+    dict(D=16, B=1, T=70, H=2, seed=15, opts=dict(contraction=0, decayed=False)),
+    dict(D=16, B=1, T=65, H=1, seed=16, opts=dict(contraction=1, centered=False)),
+    dict(D=16, B=1, T=1, H=1, seed=17, opts=dict(contraction=2)),
+]
+
+
+@pytest.mark.parametrize("case", SPECTRAL, ids=[str(i) for i in range(len(SPECTRAL))])
+def test_gdn_spectral_kernels_on_host(gdn_emu, oracle_mod, case):
+    """The resolvent and exponential contractions, with decayed and undecayed statistics,
+    against oracle.gdn_forward_spectral; the undecayed linear case is the paper's CCQ-GDN."""
+    case = dict(case)
+    opts = case.pop("opts", {})
+    D, B, T, H, seed = (case.pop(n) for n in ("D", "B", "T", "H", "seed"))
+    P = problem(D, B, T, H, seed, **case)
+    if not opts.get("decayed", True):
+        P["n0"] = np.full((B, H), 9.0, dtype=np.float32)  # the entering count of the 9-key history
+    errs = run_case(gdn_emu, D, P, **opts)
+    assert max(errs.values()) <= 1e-4, f"{case} {opts}: {errs}"
