@@ -325,6 +325,35 @@ CCQ_API ccq_status ccq_gdn_decayed_workspace_size(int B, int T, int H, int Dk, i
                                                   const ccq_params *p, size_t *bytes);
 
 /*
+ * Forward of packed variable-length sequences (GLA or Gated DeltaNet backbone): sequence s is
+ * tokens [cu_seqlens[s], cu_seqlens[s+1]) of the packed tensors, and runs as one batch-1
+ * ccq_gla_fwd / ccq_gdn_fwd call on them (the calls follow each other on `stream` and share
+ * the workspace).  The paper trains on fixed-length sequences; this is for serving mixes.
+ *   backbone     0 = GLA, 1 = Gated DeltaNet.
+ *   q, k [total,H,Dk]; v, o [total,H,Dv] in in_dtype;  gate: GLA log forget gate
+ *                [total,H,Dk] in gate_dtype, or Gated DeltaNet log decay [total,H] fp32;
+ *                beta (GDN only) and lambda [total,H] fp32.
+ *   cu_seqlens   HOST array of num_seqs + 1 offsets, cu_seqlens[0] = 0, non-decreasing
+ *                (empty sequences allowed).  cu_seqlens[s] * H must be a multiple of 4 so that
+ *                every sequence's fp32 rows start 16-byte aligned (any offsets when H % 4 = 0).
+ *   S0, C0, m0, t0 / ST, CT, mT, tT  per-sequence states [num_seqs, H, ...] and [num_seqs], as
+ *                in ccq_gla_fwd (NULL allowed as there).
+ *   workspace    at least ccq_fwd_varlen_workspace_size() bytes (the largest per-sequence need).
+ */
+CCQ_API ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void *v, const void *gate,
+                                  const float *beta, const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                                  const int64_t *cu_seqlens, int num_seqs, const float *S0, const float *C0,
+                                  const float *m0, const int64_t *t0, void *o, float *ST, float *CT, float *mT,
+                                  int64_t *tT, int H, int Dk, int Dv, void *workspace, size_t workspace_bytes,
+                                  const ccq_params *p, void *stream);
+
+/* Workspace bytes ccq_fwd_varlen needs for these sequences.  Queries the device (the segment
+   split of long GLA sequences) but launches nothing. */
+CCQ_API ccq_status ccq_fwd_varlen_workspace_size(int backbone, const int64_t *cu_seqlens, int num_seqs, int H,
+                                                 int Dk, int Dv, ccq_dtype in_dtype, const ccq_params *p,
+                                                 size_t *bytes);
+
+/*
  * ccq_gla_fwd for callers that cannot supply any device memory of their own --
  * for instance an engine that gave all device memory to its own caches at
  * start-up, or code on a path where allocating is not allowed or would stall

@@ -106,6 +106,14 @@ def load_library() -> ctypes.CDLL:
         lib.ccq_gdn_fwd_spectral.argtypes = ([_VP] * 6 + [_I] + [_VP] * 9 + [_I] * 7
                                              + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
         lib.ccq_gdn_fwd_spectral.restype = _I
+        # backbone | q, k, v, gate, beta, lambda | in_dtype, gate_dtype | cu_seqlens (host), num_seqs |
+        # S0, C0, m0, t0, o, ST, CT, mT, tT | H, Dk, Dv | workspace, bytes, params, stream
+        lib.ccq_fwd_varlen.argtypes = ([_I] + [_VP] * 6 + [_I, _I] + [_VP, _I] + [_VP] * 9 + [_I] * 3
+                                       + [_VP, ctypes.c_size_t, ctypes.POINTER(_Params), _VP])
+        lib.ccq_fwd_varlen.restype = _I
+        lib.ccq_fwd_varlen_workspace_size.argtypes = ([_I, _VP] + [_I] * 5 + [ctypes.POINTER(_Params),
+                                                                               ctypes.POINTER(ctypes.c_size_t)])
+        lib.ccq_fwd_varlen_workspace_size.restype = _I
         lib.ccq_gdn_decayed_workspace_size.argtypes = ([_I] * 6 + [ctypes.POINTER(_Params),
                                                                    ctypes.POINTER(ctypes.c_size_t)])
         lib.ccq_gdn_decayed_workspace_size.restype = _I
@@ -500,6 +508,47 @@ def gdn_fwd_decayed(q, k, v, g, beta, lam, *, S0=None, C0=None, m0=None, n0=None
         _ptr(fs["S"] if fs else None), _ptr(fs["C"] if fs else None), _ptr(fs["m"] if fs else None),
         _ptr(fs["n"] if fs else None), B, T, H, Dk, Dv, CONTRACTION[contraction], int(bool(decayed)),
         _ptr(workspace), ws_bytes, ctypes.byref(p), _stream(dev, stream))
+    _check(st)
+    return (o, fs) if return_state else o
+
+
+def fwd_varlen(backbone, q, k, v, gate, lam, cu_seqlens, *, beta=None, state: Optional[CCQState] = None,
+               out=None, return_state: bool = True, workspace=None, stream=None, **kw):
+    """Forward of packed variable-length sequences (ccq_fwd_varlen).  q, k [total,H,Dk]; v
+    [total,H,Dv]; gate [total,H,Dk] (GLA) or [total,H] fp32 (GDN, with beta [total,H]); lam
+    [total,H]; ``cu_seqlens`` the num_seqs + 1 offsets (a list or CPU integer tensor; it stays on
+    the host).  ``state`` / the returned CCQState hold one row per sequence.  Returns o
+    [total,H,Dv] and (optionally) the final CCQState."""
+    dev = q.device
+    total, H, Dk = q.shape
+    Dv = v.shape[-1]
+    cu = [int(x) for x in (cu_seqlens.tolist() if hasattr(cu_seqlens, "tolist") else cu_seqlens)]
+    ns = len(cu) - 1
+    _req(q, "q", dev)
+    _req(k, "k", dev, q.dtype, q.shape)
+    _req(v, "v", dev, q.dtype, (total, H, Dv))
+    _req(gate, "gate", dev, None, (total, H, Dk) if backbone == 0 else (total, H))
+    _req(lam, "lam", dev, torch.float32, (total, H))
+    if beta is not None:
+        _req(beta, "beta", dev, torch.float32, (total, H))
+    S0, C0, m0, t0 = _state_in(state, ns, H, Dk, Dv, dev)
+    o = out if out is not None else torch.empty(total, H, Dv, dtype=q.dtype, device=dev)
+    _req(o, "out", dev, q.dtype, (total, H, Dv))
+    fs = CCQState.empty(ns, H, Dk, Dv, dev) if return_state else None
+    cu_arr = (ctypes.c_int64 * len(cu))(*cu)
+    p = params(**kw)
+    lib = load_library()
+    need = ctypes.c_size_t(0)
+    _check(lib.ccq_fwd_varlen_workspace_size(int(backbone), ctypes.cast(cu_arr, _VP), ns, H, Dk, Dv,
+                                             _dtype_code(q), ctypes.byref(p), ctypes.byref(need)))
+    if workspace is None and need.value:
+        workspace = torch.empty(need.value, dtype=torch.uint8, device=dev)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    st = lib.ccq_fwd_varlen(
+        int(backbone), _ptr(q), _ptr(k), _ptr(v), _ptr(gate), _ptr(beta), _ptr(lam), _dtype_code(q),
+        _dtype_code(gate), ctypes.cast(cu_arr, _VP), ns, _ptr(S0), _ptr(C0), _ptr(m0), _ptr(t0), _ptr(o),
+        _ptr(fs.S if fs else None), _ptr(fs.C if fs else None), _ptr(fs.m if fs else None),
+        _ptr(fs.t if fs else None), H, Dk, Dv, _ptr(workspace), ws_bytes, ctypes.byref(p), _stream(dev, stream))
     _check(st)
     return (o, fs) if return_state else o
 

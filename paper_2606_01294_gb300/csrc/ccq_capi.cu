@@ -705,6 +705,94 @@ ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, cons
                                 Dk, Dv, CCQ_CONTRACT_LINEAR, 1, workspace, workspace_bytes, p, stream);
 }
 
+// Packed variable-length sequences: validation shared by the call and its workspace query.
+static ccq_status check_varlen(int backbone, const int64_t *cu, int num_seqs, int H, long long *max_len) {
+    if (backbone != 0 && backbone != 1) return fail(CCQ_ERR_INVALID_ARG, "backbone must be 0 (GLA) or 1 (GDN)");
+    if (!cu || num_seqs < 1) return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens is NULL or num_seqs < 1");
+    if (cu[0] != 0) return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
+    long long mx = 0;
+    for (int s = 0; s < num_seqs; ++s) {
+        const long long len = cu[s + 1] - cu[s];
+        if (len < 0) return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens decreases at %d", s);
+        if (len > 0x7fffffffLL) return fail(CCQ_ERR_INVALID_ARG, "sequence %d is too long", s);
+        // per-token fp32 rows [T][H] start on 16-byte boundaries only if cu[s] * H is a multiple of 4
+        if ((cu[s] * H) % 4 != 0)
+            return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens[%d] * H must be a multiple of 4 (16-byte aligned rows)", s);
+        mx = std::max(mx, len);
+    }
+    *max_len = mx;
+    return CCQ_OK;
+}
+
+ccq_status ccq_fwd_varlen_workspace_size(int backbone, const int64_t *cu_seqlens, int num_seqs, int H, int Dk,
+                                         int Dv, ccq_dtype in_dtype, const ccq_params *p, size_t *bytes) {
+    long long mx = 0;
+    ccq_status st = check_varlen(backbone, cu_seqlens, num_seqs, H, &mx);
+    if (st != CCQ_OK) return st;
+    if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    size_t need = 0;
+    for (int s = 0; s < num_seqs; ++s) {
+        const int len = static_cast<int>(cu_seqlens[s + 1] - cu_seqlens[s]);
+        size_t b = 0;
+        st = backbone == 0 ? ccq_gla_workspace_size(1, len, H, Dk, Dv, in_dtype, p, &b)
+                           : ccq_gdn_workspace_size(1, len, H, Dk, Dv, in_dtype, p, &b);
+        if (st != CCQ_OK) return st;
+        need = std::max(need, b);
+    }
+    *bytes = need;
+    return CCQ_OK;
+}
+
+ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void *v, const void *gate,
+                          const float *beta, const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
+                          const int64_t *cu_seqlens, int num_seqs, const float *S0, const float *C0,
+                          const float *m0, const int64_t *t0, void *o, float *ST, float *CT, float *mT,
+                          int64_t *tT, int H, int Dk, int Dv, void *workspace, size_t workspace_bytes,
+                          const ccq_params *p, void *stream) {
+    long long mx = 0;
+    ccq_status st = check_varlen(backbone, cu_seqlens, num_seqs, H, &mx);
+    if (st != CCQ_OK) return st;
+    if ((in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) || (gate_dtype != CCQ_BF16 && gate_dtype != CCQ_FP32))
+        return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    size_t need = 0;
+    st = ccq_fwd_varlen_workspace_size(backbone, cu_seqlens, num_seqs, H, Dk, Dv, in_dtype, p, &need);
+    if (st != CCQ_OK) return st;
+    if (need && (!workspace || workspace_bytes < need))
+        return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
+                    workspace ? workspace_bytes : static_cast<size_t>(0));
+    const size_t esz = in_dtype == CCQ_BF16 ? 2 : 4, gsz = gate_dtype == CCQ_BF16 ? 2 : 4;
+    const size_t h = static_cast<size_t>(H);
+    // One call of the (batch-1) forward per sequence, in stream order: the calls share the
+    // workspace, and sequence s reads and writes row s of every state.
+    for (int s = 0; s < num_seqs; ++s) {
+        const size_t off = static_cast<size_t>(cu_seqlens[s]);
+        const int len = static_cast<int>(cu_seqlens[s + 1] - cu_seqlens[s]);
+        auto at = [&](const void *base, size_t bytes_per_token) -> const void * {
+            return base ? static_cast<const uint8_t *>(base) + off * bytes_per_token : nullptr;
+        };
+        auto row = [&](const float *base, size_t per) -> const float * { return base ? base + s * per : nullptr; };
+        auto rowm = [&](float *base, size_t per) -> float * { return base ? base + s * per : nullptr; };
+        const void *qs = at(q, h * Dk * esz), *ks = at(k, h * Dk * esz), *vs = at(v, h * Dv * esz);
+        void *os = const_cast<void *>(at(o, h * Dv * esz));
+        const float *ls = static_cast<const float *>(at(lambda, h * 4));
+        const size_t sS = h * Dk * Dv, sC = h * Dk * Dk, sm = h * Dk;
+        const int64_t *t0s = t0 ? t0 + s : nullptr;
+        int64_t *tTs = tT ? tT + s : nullptr;
+        if (backbone == 0) {
+            st = ccq_gla_fwd(qs, ks, vs, at(gate, h * Dk * gsz), ls, in_dtype, gate_dtype, row(S0, sS), row(C0, sC),
+                             row(m0, sm), t0s, os, rowm(ST, sS), rowm(CT, sC), rowm(mT, sm), tTs, 1, len, H, Dk, Dv,
+                             workspace, workspace_bytes, p, stream);
+        } else {
+            st = ccq_gdn_fwd(qs, ks, vs, static_cast<const float *>(at(gate, h * 4)),
+                             static_cast<const float *>(at(beta, h * 4)), ls, in_dtype, row(S0, sS), row(C0, sC),
+                             row(m0, sm), t0s, os, rowm(ST, sS), rowm(CT, sC), rowm(mT, sm), tTs, 1, len, H, Dk, Dv,
+                             workspace, workspace_bytes, p, stream);
+        }
+        if (st != CCQ_OK) return st;
+    }
+    return CCQ_OK;
+}
+
 ccq_status ccq_decode_step(int backbone, const void *q, const void *k, const void *v,
                            const void *gate, const float *beta, const float *lambda,
                            ccq_dtype in_dtype, ccq_dtype gate_dtype, float *S, float *C,

@@ -239,3 +239,23 @@ def test_gdn_spectral_rejects_unknown_contraction(lib):
     assert call(1, 2) == ccq.CCQ_ERR_INVALID_ARG
     assert call(2, 0) == ccq.CCQ_ERR_INVALID_ARG      # valid request, but no workspace
     assert b"workspace" in lib.ccq_last_error()
+
+
+def test_varlen_rejects_bad_offsets(lib):
+    fake = ctypes.c_void_p(0x10000)
+
+    def call(cu, H=16, backbone=0):
+        arr = (ctypes.c_int64 * len(cu))(*cu)
+        return lib.ccq_fwd_varlen(backbone, *([fake] * 6), 0, 0, ctypes.cast(arr, ctypes.c_void_p), len(cu) - 1,
+                                  None, None, None, None, fake, None, None, None, None, H, 128, 128, None, 0,
+                                  ctypes.byref(ccq.params()), None)
+    assert call([1, 5]) == ccq.CCQ_ERR_INVALID_ARG          # must start at 0
+    assert b"cu_seqlens[0]" in lib.ccq_last_error()
+    assert call([0, 9, 5]) == ccq.CCQ_ERR_INVALID_ARG       # decreasing
+    assert call([0, 3, 8], H=2) == ccq.CCQ_ERR_INVALID_ARG  # 3 * 2 fp32 rows: not 16-byte aligned
+    assert b"multiple of 4" in lib.ccq_last_error()
+    assert call([0, 3, 8], backbone=2) == ccq.CCQ_ERR_INVALID_ARG
+    arr = (ctypes.c_int64 * 1)(0)
+    assert lib.ccq_fwd_varlen(0, *([fake] * 6), 0, 0, ctypes.cast(arr, ctypes.c_void_p), 0, None, None, None, None,
+                              fake, None, None, None, None, 16, 128, 128, None, 0, ctypes.byref(ccq.params()),
+                              None) == ccq.CCQ_ERR_INVALID_ARG  # no sequences
