@@ -302,8 +302,10 @@ CCQ_API ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void 
  *   contraction  a ccq_contraction value.  RESOLVENT runs ten conjugate-gradient iterations
  *                per query from the linear estimate (I + lambda Sigma has spectrum in
  *                [1, 1 + lambda] for unit keys); EXPONENTIAL sums twelve Taylor terms
- *                (|lambda Sigma| <= 1).  Both assume unit-norm keys (l2norm_qk = 1, or keys of
- *                norm at most 1).
+ *                (|lambda Sigma| <= 1).  Both rely on unit-norm keys for those bounds, so they
+ *                need l2norm_qk = 1: with l2norm_qk = 0 they return CCQ_ERR_UNSUPPORTED
+ *                (arbitrary key norms would leave the fixed iteration counts without an
+ *                error bound).
  *   decayed      1: the decay-aligned statistics of ccq_gdn_fwd_decayed (n the decayed count);
  *                0: the paper's undecayed sums, C_t = sum kbar kbar^T, m_t = sum kbar, with n
  *                the token count t (n0/nT [B,H] fp32 carry it) -- with LINEAR this is the
@@ -366,6 +368,10 @@ CCQ_API ccq_status ccq_fwd_varlen_workspace_size(int backbone, const int64_t *cu
  *     CCQ_ERR_INVALID_ARG and a message naming both sizes.
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *     The address is then kept for the life of the process, which assumes the
+ *     device's primary context lives that long: after cudaDeviceReset (or any
+ *     teardown and re-creation of that context) the kept address is stale, so
+ *     do not reset a device while this library is in use on it.
  *   - All calls share the one array and it keeps the last call's contents: two
  *     calls whose work overlaps on the GPU (other streams, other host threads)
  *     race and corrupt each other's results; serialise them.

@@ -524,6 +524,14 @@ def fwd_varlen(backbone, q, k, v, gate, lam, cu_seqlens, *, beta=None, state: Op
     Dv = v.shape[-1]
     cu = [int(x) for x in (cu_seqlens.tolist() if hasattr(cu_seqlens, "tolist") else cu_seqlens)]
     ns = len(cu) - 1
+    # The C ABI cannot see the packed length: an offset past it would make the kernels read
+    # and write beyond the tensors, so the pack is checked here.
+    if ns < 1 or cu[0] != 0:
+        raise ValueError("cu_seqlens must start at 0 and hold num_seqs + 1 >= 2 offsets")
+    if any(b < a for a, b in zip(cu, cu[1:])):
+        raise ValueError("cu_seqlens must be non-decreasing")
+    if cu[-1] != total:
+        raise ValueError(f"cu_seqlens[-1] = {cu[-1]} must equal the packed length {total}")
     _req(q, "q", dev)
     _req(k, "k", dev, q.dtype, q.shape)
     _req(v, "v", dev, q.dtype, (total, H, Dv))

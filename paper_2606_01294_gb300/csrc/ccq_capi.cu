@@ -108,6 +108,17 @@ ccq_status check_ptrs(const char *names, std::initializer_list<const void *> req
     return CCQ_OK;
 }
 
+// The int64 position counters t0 / tT are read and written one element per
+// batch row, so they need only their natural 8-byte alignment (a row of a
+// larger counter array, as the packed-sequence call passes, is enough).
+ccq_status check_counts(std::initializer_list<const void *> counts) {
+    for (const void *p : counts) {
+        if (p && (reinterpret_cast<uintptr_t>(p) & 7u) != 0)
+            return fail(CCQ_ERR_INVALID_ARG, "a position-count pointer (t0 / tT) is not 8-byte aligned");
+    }
+    return CCQ_OK;
+}
+
 // Final position count, after the kernels that read t0 (tT may alias it).
 ccq_status finish_t(const int64_t *t0, int64_t *tT, int B, int T, cudaStream_t s) {
     cudaError_t e = launch_t_update(t0, tT, B, T, s);
@@ -243,17 +254,19 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
                                void *o, float *ST, float *CT, float *mT, int64_t *tT,
                                int B, int T, int H, int Dk, int Dv, void *workspace,
                                size_t workspace_bytes, uint8_t *ckpt, int skip_o, const ccq_params *p,
-                               void *stream) {
+                               void *stream, bool dry = false) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
     if ((in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) || (gate_dtype != CCQ_BF16 && gate_dtype != CCQ_FP32))
         return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
     if (T > 0) {
-        st = check_ptrs("q,k,v,gk,lambda,o", {q, k, v, gk, lambda, o}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        st = check_ptrs("q,k,v,gk,lambda,o", {q, k, v, gk, lambda, o}, {S0, C0, m0, ST, CT, mT});
+        if (st == CCQ_OK) st = check_counts({t0, tT});
         if (st != CCQ_OK) return st;
     } else {
-        st = check_ptrs("", {}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        st = check_ptrs("", {}, {S0, C0, m0, ST, CT, mT});
+        if (st == CCQ_OK) st = check_counts({t0, tT});
         if (st != CCQ_OK) return st;
     }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -280,6 +293,7 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
             !make_token_map(&maps.g, gk, geb, B, T, H, 128, 128, false) ||
             !make_token_map(&maps.o, o, 2, B, T, H, 128, 64, true))
             return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
+        if (dry) return CCQ_OK;
         ChunkArgs a = {};
         a.B = B; a.T = T; a.H = H;
         a.gate_dtype = gate_dtype == CCQ_BF16 ? 0 : 1;
@@ -304,6 +318,7 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
         if (e != cudaSuccess) return cuda_fail(e, "chunkwise GLA kernel launch");
         return finish_t(t0, tT, B, T, s);
     }
+    if (dry) return CCQ_OK;
     RecurrentArgs ra = {};
     ra.backbone = 0; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
     ra.in_dtype = in_dtype; ra.gate_dtype = gate_dtype;
@@ -398,7 +413,8 @@ ccq_status ccq_gla_bwd(const void *q, const void *k, const void *v, const void *
         return fail(CCQ_ERR_UNSUPPORTED, "the backward needs bf16 inputs and Dk = Dv = 128");
     if (c.p.algo == CCQ_ALGO_RECURRENT)
         return fail(CCQ_ERR_UNSUPPORTED, "the backward is chunkwise only (algo recurrent given)");
-    st = check_ptrs("", {}, {S0, C0, m0, t0, dST, dCT, dmT, ckpt, dlambda, dS0, dC0, dm0});
+    st = check_ptrs("", {}, {S0, C0, m0, dST, dCT, dmT, ckpt, dlambda, dS0, dC0, dm0});
+    if (st == CCQ_OK) st = check_counts({t0});
     if (st != CCQ_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (T == 0) {
@@ -498,21 +514,25 @@ ccq_status ccq_gdn_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype
     return CCQ_OK;
 }
 
-ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
-                       const float *beta, const float *lambda, ccq_dtype in_dtype,
-                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
-                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
-                       int B, int T, int H, int Dk, int Dv, void *workspace,
-                       size_t workspace_bytes, const ccq_params *p, void *stream) {
+// The Gated DeltaNet forward behind ccq_gdn_fwd; `dry` runs every argument check and
+// returns before the first CUDA call.
+static ccq_status gdn_fwd_impl(const void *q, const void *k, const void *v, const float *g,
+                               const float *beta, const float *lambda, ccq_dtype in_dtype,
+                               const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                               void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                               int B, int T, int H, int Dk, int Dv, void *workspace,
+                               size_t workspace_bytes, const ccq_params *p, void *stream, bool dry) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
     if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
     if (T > 0) {
-        st = check_ptrs("q,k,v,g,beta,lambda,o", {q, k, v, g, beta, lambda, o}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        st = check_ptrs("q,k,v,g,beta,lambda,o", {q, k, v, g, beta, lambda, o}, {S0, C0, m0, ST, CT, mT});
+        if (st == CCQ_OK) st = check_counts({t0, tT});
         if (st != CCQ_OK) return st;
     } else {
-        st = check_ptrs("", {}, {S0, C0, m0, t0, ST, CT, mT, tT});
+        st = check_ptrs("", {}, {S0, C0, m0, ST, CT, mT});
+        if (st == CCQ_OK) st = check_counts({t0, tT});
         if (st != CCQ_OK) return st;
     }
     const bool chunk_ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
@@ -533,6 +553,7 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
             !make_token_map(&maps.o, o, 2, B, T, H, 128, 64, true) ||
             !make_rows_map(&maps.tb, workspace, rows, 64))
             return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
+        if (dry) return CCQ_OK;
         ChunkArgs a = {};
         a.B = B; a.T = T; a.H = H;
         a.gate_dtype = 1;
@@ -557,6 +578,7 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
         if (e != cudaSuccess) return cuda_fail(e, "chunkwise Gated DeltaNet kernel launch");
         return finish_t(t0, tT, B, T, static_cast<cudaStream_t>(stream));
     }
+    if (dry) return CCQ_OK;
     RecurrentArgs ra = {};
     ra.backbone = 1; ra.B = B; ra.T = T; ra.H = H; ra.Dk = Dk; ra.Dv = Dv;
     ra.in_dtype = in_dtype; ra.gate_dtype = CCQ_FP32;
@@ -566,6 +588,16 @@ ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float 
     ra.o = o; ra.ST = ST; ra.CT = CT; ra.mT = mT;
     st = run_recurrent(ra, static_cast<cudaStream_t>(stream));
     return st != CCQ_OK ? st : finish_t(t0, tT, B, T, static_cast<cudaStream_t>(stream));
+}
+
+ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
+                       const float *beta, const float *lambda, ccq_dtype in_dtype,
+                       const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                       void *o, float *ST, float *CT, float *mT, int64_t *tT,
+                       int B, int T, int H, int Dk, int Dv, void *workspace,
+                       size_t workspace_bytes, const ccq_params *p, void *stream) {
+    return gdn_fwd_impl(q, k, v, g, beta, lambda, in_dtype, S0, C0, m0, t0, o, ST, CT, mT, tT, B, T, H, Dk, Dv,
+                        workspace, workspace_bytes, p, stream, false);
 }
 
 // Copies the final-state gradients to the initial-state ones (zero where a final one is NULL):
@@ -607,7 +639,8 @@ ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float 
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
     if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
-    st = check_ptrs("", {}, {S0, C0, m0, t0, dST, dCT, dmT, dlambda, dS0, dC0, dm0});
+    st = check_ptrs("", {}, {S0, C0, m0, dST, dCT, dmT, dlambda, dS0, dC0, dm0});
+    if (st == CCQ_OK) st = check_counts({t0});
     if (st != CCQ_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (T == 0) return copy_state_grads(dST, dCT, dmT, dS0, dC0, dm0, B, H, Dk, Dv, s);
@@ -657,6 +690,9 @@ ccq_status ccq_gdn_fwd_spectral(const void *q, const void *k, const void *v, con
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
     if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    // The fixed CG / Taylor iteration counts are bounded only for unit-norm keys (|lambda Sigma| <= 1).
+    if (contraction != CCQ_CONTRACT_LINEAR && !c.p.l2norm_qk)
+        return fail(CCQ_ERR_UNSUPPORTED, "the resolvent and exponential contractions need l2norm_qk = 1");
     st = check_ptrs("", {}, {S0, C0, m0, n0, ST, CT, mT, nT});
     if (st != CCQ_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -762,8 +798,15 @@ ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void
                     workspace ? workspace_bytes : static_cast<size_t>(0));
     const size_t esz = in_dtype == CCQ_BF16 ? 2 : 4, gsz = gate_dtype == CCQ_BF16 ? 2 : 4;
     const size_t h = static_cast<size_t>(H);
+    ccq_params pin;
+    if (p) pin = *p;
+    else ccq_default_params(&pin);
+    ccq_params pempty = pin;  // an empty sequence passes its state through on any path
+    pempty.algo = CCQ_ALGO_AUTO;
     // One call of the (batch-1) forward per sequence, in stream order: the calls share the
-    // workspace, and sequence s reads and writes row s of every state.
+    // workspace, and sequence s reads and writes row s of every state.  Pass 0 checks every
+    // call's arguments, pass 1 launches, so that a rejected pack enqueues nothing.
+    for (int pass = 0; pass < 2; ++pass)
     for (int s = 0; s < num_seqs; ++s) {
         const size_t off = static_cast<size_t>(cu_seqlens[s]);
         const int len = static_cast<int>(cu_seqlens[s + 1] - cu_seqlens[s]);
@@ -778,15 +821,17 @@ ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void
         const size_t sS = h * Dk * Dv, sC = h * Dk * Dk, sm = h * Dk;
         const int64_t *t0s = t0 ? t0 + s : nullptr;
         int64_t *tTs = tT ? tT + s : nullptr;
+        const ccq_params *ps = len > 0 ? &pin : &pempty;
+        const bool dry = pass == 0;
         if (backbone == 0) {
-            st = ccq_gla_fwd(qs, ks, vs, at(gate, h * Dk * gsz), ls, in_dtype, gate_dtype, row(S0, sS), row(C0, sC),
-                             row(m0, sm), t0s, os, rowm(ST, sS), rowm(CT, sC), rowm(mT, sm), tTs, 1, len, H, Dk, Dv,
-                             workspace, workspace_bytes, p, stream);
+            st = gla_fwd_impl(qs, ks, vs, at(gate, h * Dk * gsz), ls, in_dtype, gate_dtype, row(S0, sS), row(C0, sC),
+                              row(m0, sm), t0s, os, rowm(ST, sS), rowm(CT, sC), rowm(mT, sm), tTs, 1, len, H, Dk, Dv,
+                              workspace, workspace_bytes, nullptr, 0, ps, stream, dry);
         } else {
-            st = ccq_gdn_fwd(qs, ks, vs, static_cast<const float *>(at(gate, h * 4)),
-                             static_cast<const float *>(at(beta, h * 4)), ls, in_dtype, row(S0, sS), row(C0, sC),
-                             row(m0, sm), t0s, os, rowm(ST, sS), rowm(CT, sC), rowm(mT, sm), tTs, 1, len, H, Dk, Dv,
-                             workspace, workspace_bytes, p, stream);
+            st = gdn_fwd_impl(qs, ks, vs, static_cast<const float *>(at(gate, h * 4)),
+                              static_cast<const float *>(at(beta, h * 4)), ls, in_dtype, row(S0, sS), row(C0, sC),
+                              row(m0, sm), t0s, os, rowm(ST, sS), rowm(CT, sC), rowm(mT, sm), tTs, 1, len, H, Dk, Dv,
+                              workspace, workspace_bytes, ps, stream, dry);
         }
         if (st != CCQ_OK) return st;
     }

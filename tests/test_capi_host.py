@@ -239,6 +239,13 @@ def test_gdn_spectral_rejects_unknown_contraction(lib):
     assert call(1, 2) == ccq.CCQ_ERR_INVALID_ARG
     assert call(2, 0) == ccq.CCQ_ERR_INVALID_ARG      # valid request, but no workspace
     assert b"workspace" in lib.ccq_last_error()
+    # the fixed CG / Taylor counts are bounded only for unit-norm keys
+    for contraction in (1, 2):
+        st = lib.ccq_gdn_fwd_spectral(*([fake] * 6), 1, None, None, None, None, fake, None, None, None, None,
+                                      1, 70, 2, 64, 64, contraction, 0, None, 0,
+                                      ctypes.byref(ccq.params(l2norm=False)), None)
+        assert st == ccq.CCQ_ERR_UNSUPPORTED
+        assert b"l2norm_qk" in lib.ccq_last_error()
 
 
 def test_varlen_rejects_bad_offsets(lib):
@@ -259,3 +266,40 @@ def test_varlen_rejects_bad_offsets(lib):
     assert lib.ccq_fwd_varlen(0, *([fake] * 6), 0, 0, ctypes.cast(arr, ctypes.c_void_p), 0, None, None, None, None,
                               fake, None, None, None, None, 16, 128, 128, None, 0, ctypes.byref(ccq.params()),
                               None) == ccq.CCQ_ERR_INVALID_ARG  # no sequences
+
+
+def test_varlen_argument_checks_pass_for_a_pack(lib):
+    """A pack of several sequences (empty ones included) with per-sequence position counters
+    passes every argument check: without a GPU the call then fails at its first launch
+    (CCQ_ERR_CUDA), not with CCQ_ERR_INVALID_ARG.  Row s of t0 / tT sits 8 bytes after row s-1."""
+    fake = ctypes.c_void_p(0x10000)
+    cu = [0, 4, 4, 12, 16]
+    arr = (ctypes.c_int64 * len(cu))(*cu)
+
+    def call(backbone, beta, algo="auto", fp32=True):
+        p = ccq.params(algo=algo)
+        dt = 1 if fp32 else 0
+        D = 64 if fp32 else 128
+        return lib.ccq_fwd_varlen(backbone, fake, fake, fake, fake, beta, fake, dt, 1,
+                                  ctypes.cast(arr, ctypes.c_void_p), len(cu) - 1,
+                                  fake, fake, fake, fake, fake, fake, fake, fake, fake, 4, D, D, None, 0,
+                                  ctypes.byref(p), None)
+    for backbone in (0, 1):
+        st = call(backbone, fake)
+        assert st == ccq.CCQ_ERR_CUDA, (backbone, st, lib.ccq_last_error())
+    # every call is checked before the first launch: GDN without beta is rejected as an
+    # argument error although sequence 0 alone would have been launched first
+    assert call(1, None) == ccq.CCQ_ERR_INVALID_ARG
+    assert b"NULL" in lib.ccq_last_error()
+    # an empty sequence passes its state through even when the chunkwise path is forced
+    # (fp32 inputs make the non-empty ones unsupported there, which is reported, not launched)
+    assert call(0, fake, algo="chunkwise") == ccq.CCQ_ERR_UNSUPPORTED
+    assert b"chunkwise" in lib.ccq_last_error()
+
+
+def test_varlen_binding_checks_offsets_against_the_pack():
+    import torch
+    q = torch.zeros(10, 2, 64)
+    for cu, msg in (([1, 10], "start at 0"), ([0, 6, 4, 10], "non-decreasing"), ([0, 4, 12], "packed length")):
+        with pytest.raises(ValueError, match=msg):
+            ccq.fwd_varlen(0, q, q, q, q, torch.zeros(10, 2), cu)
