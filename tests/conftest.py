@@ -22,12 +22,6 @@ def oracle_mod():
     return oracle
 
 
-# Parity tests of entry points whose kernels have not yet run on a GPU.  They are collected
-# (moved up into tests/) once a GPU run has passed them, so that an unverified kernel never
-# runs first inside the suite.
-collect_ignore = ["gpu_pending"]
-
-
 def load_gdn_emu(path):
     """ctypes handle of a host build of tests/host_emu/gdn_cuda_core_emu.cpp."""
     lib = ctypes.CDLL(path)
