@@ -316,29 +316,15 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
-def run_gpu(args):
+def setup_workload(kind, B, H, T, D, dev, seed):
+    """Inputs resident in HBM plus pinned host copies for one workload.  Returns
+    (step, e2e_step, tokens_per_step, h2d_bytes, d2h_bytes): `step` runs one step on the
+    device-resident inputs, `e2e_step` copies that step's inputs from pinned host memory,
+    runs it and reads the result back."""
     import torch
-    import torch.distributed as dist
-
-    rank, local_rank, world = dist_env()
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=dev)
-    from __graft_entry__ import build
-    if rank == 0 or world == 1:
-        build()
-    if world > 1:
-        dist.barrier()
-        build()
     from paper_2606_01294_gb300 import ccq
     from paper_2606_01294_gb300 import inputs as gen
 
-    kind, B, H, T, D = WORKLOADS[args.workload]
-    seed = 1236 + rank
-    stream = torch.cuda.current_stream(dev)
-
-    # ---------------- inputs resident in HBM
     if kind == "decode":
         Dd = gen.make_decode_inputs(gen.GLA, B, H, D, D, seed=seed)
         pre = {n: (None if x is None else x.to(dev)) for n, x in Dd["prefix"].items()}
@@ -397,15 +383,43 @@ def run_gpu(args):
         tokens_per_step = B * T
         host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
 
+    def e2e_step():
+        d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
+        if kind == "decode":
+            o = ccq.decode_step(gen.GLA, d["q"], d["k"], d["v"], d["gate"], d["lam"], state, out=out)
+            return o.to("cpu", non_blocking=True)
+        if kind == "glabwd":
+            train_step(d)
+            return [grads[n].to("cpu", non_blocking=True) for n in ("dq", "dk", "dv", "dgk")]
+        if kind == "gla":
+            o, _ = ccq.gla_fwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out,
+                               final_state=fstate, workspace=ws)
+        else:
+            o, _ = ccq.gdn_fwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], out=out,
+                               final_state=fstate, workspace=ws)
+        return o.to("cpu", non_blocking=True)
+
+    h2d = sum(x.numel() * x.element_size() for x in host.values() if x is not None)
+    d2h = out.numel() * out.element_size() * (4 if kind == "glabwd" else 1)
+    return step, e2e_step, tokens_per_step, h2d, d2h
+
+
+def time_steps(step, steps, warmup, dev, local_rank, world):
+    """W untimed warm-up steps, then exactly K steps bracketed by a barrier and a
+    synchronize, each step between two CUDA events on the launching stream; clocks sampled
+    during the timed region.  Returns (total_ms max over ranks, per-step event ms, clocks)."""
+    import torch
+    import torch.distributed as dist
+    from paper_2606_01294_gb300 import ccq
+    stream = torch.cuda.current_stream(dev)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(args.steps)]
+          for _ in range(steps)]
     with ClockSampler(local_rank) as clocks:
         time.sleep(0.3)  # nvidia-smi start-up
-        for _ in range(args.warmup):
+        for _ in range(warmup):
             step()
         ccq.device_status()
         torch.cuda.synchronize()
-        # ---------------- timed region: device-resident inputs
         if world > 1:
             dist.barrier()
         torch.cuda.synchronize()
@@ -413,7 +427,7 @@ def run_gpu(args):
         t_start = torch.cuda.Event(enable_timing=True)
         t_end = torch.cuda.Event(enable_timing=True)
         t_start.record(stream)
-        for i in range(args.steps):
+        for i in range(steps):
             ev[i][0].record(stream)
             step()
             ev[i][1].record(stream)
@@ -425,31 +439,54 @@ def run_gpu(args):
         dist.barrier()
     ccq.device_status()
     total_ms = max_over_ranks(t_start.elapsed_time(t_end), dev)
-    launch_ms = [a.elapsed_time(b) for a, b in ev]
+    return total_ms, [a.elapsed_time(b) for a, b in ev], clocks.summary()
+
+
+def roofline(kind, workload, B, H, T, D, kern_ms, peaks):
+    bytes_ = algorithmic_bytes(kind, B, H, T, D)
+    achieved = bytes_ / (kern_ms / 1e3) / 1e9
+    return {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"],
+            "traffic": measured_traffic(kind, workload),
+            "kernel": {"gla_bf16_20k": "whole step: gla_segment_state_kernel + gla_segment_combine_kernel"
+                                       " + gla_chunk_kernel",
+                       "gdn_bf16_20k": "whole step: gdn_wy_kernel + gdn_segment_state_kernel"
+                                       " + gdn_segment_combine_kernel + gdn_chunk_kernel"}.get(
+                           workload, KERNEL_NAMES[kind]), "algorithmic_bytes": bytes_,
+            "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
+            "flops": algorithmic_flops(kind, B, H, T, D)}
+
+
+# Workloads the default run times beside the headline one (same steps and warm-up), each
+# reported under "also" with its own roofline: the second T = 4096 forward configuration.
+ALSO_DEFAULT = ("gdn_bf16_4k",)
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    rank, local_rank, world = dist_env()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+    from __graft_entry__ import build
+    if rank == 0 or world == 1:
+        build()
+    if world > 1:
+        dist.barrier()
+        build()
+
+    kind, B, H, T, D = WORKLOADS[args.workload]
+    seed = 1236 + rank
+    stream = torch.cuda.current_stream(dev)
+    step, e2e_step, tokens_per_step, h2d, d2h = setup_workload(kind, B, H, T, D, dev, seed)
+    total_ms, launch_ms, clock_summary = time_steps(step, args.steps, args.warmup, dev, local_rank, world)
     ms_per_step = total_ms / args.steps
     value = whole_job_rate(world, tokens_per_step, args.steps, total_ms)
 
     # ---------------- e2e: host buffers, copies inside the timed region
-    def e2e_step():
-        if kind == "decode":
-            d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
-            o = ccq.decode_step(gen.GLA, d["q"], d["k"], d["v"], d["gate"], d["lam"], state, out=out)
-            res = o.to("cpu", non_blocking=True)
-            return res
-        d = {n: (None if x is None else x.to(dev, non_blocking=True)) for n, x in host.items()}
-        if kind == "glabwd":
-            train_step(d)
-            return [grads[n].to("cpu", non_blocking=True) for n in ("dq", "dk", "dv", "dgk")]
-        if kind == "gla":
-            o, st = ccq.gla_fwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out,
-                                final_state=fstate, workspace=ws)
-        else:
-            o, st = ccq.gdn_fwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], out=out,
-                                final_state=fstate, workspace=ws)
-        return o.to("cpu", non_blocking=True)
-
-    h2d = sum(x.numel() * x.element_size() for x in host.values() if x is not None)
-    d2h = out.numel() * out.element_size() * (4 if kind == "glabwd" else 1)
     e2e_steps = max(3, min(args.steps, 10))
     e2e_step()
     torch.cuda.synchronize()
@@ -464,24 +501,34 @@ def run_gpu(args):
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dev)
     e2e_value = whole_job_rate(world, tokens_per_step, 1, e2e_ms)
+    del step, e2e_step
+
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    also = {}
+    if args.workload == "gla_bf16_4k" and not args.no_also:
+        for name in ALSO_DEFAULT:
+            k2, B2, H2, T2, D2 = WORKLOADS[name]
+            st2, _, tok2, _, _ = setup_workload(k2, B2, H2, T2, D2, dev, seed + 1)
+            tot2, lms2, clk2 = time_steps(st2, args.steps, args.warmup, dev, local_rank, world)
+            also[name] = {"ms_per_step": tot2 / args.steps,
+                          "value": whole_job_rate(world, tok2, args.steps, tot2), "unit": "tokens/s",
+                          "config": {"backbone": k2, "B": B2, "H": H2, "T": T2, "d_k": D2, "d_v": D2,
+                                     "chunk": 64},
+                          "gpu_launches": args.steps * launches_per_step(k2, B2, H2, T2, sms),
+                          "kernel_ms_mean": statistics.mean(lms2), "clocks": clk2, "lms": lms2}
+            del st2
+            torch.cuda.empty_cache()
 
     line = None
     if rank == 0:
         with open(PEAKS_FILE) as f:
             peaks = json.load(f)
         kern_ms = statistics.mean(launch_ms)
-        bytes_ = algorithmic_bytes(kind, B, H, T, D)
-        achieved = bytes_ / (kern_ms / 1e3) / 1e9
-        roof = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                "frac": achieved / peaks["hbm_gbs"],
-                "traffic": measured_traffic(kind, args.workload),
-                "kernel": {"gla_bf16_20k": "whole step: gla_segment_state_kernel + gla_segment_combine_kernel"
-                                           " + gla_chunk_kernel",
-                           "gdn_bf16_20k": "whole step: gdn_wy_kernel + gdn_segment_state_kernel"
-                                           " + gdn_segment_combine_kernel + gdn_chunk_kernel"}.get(
-                               args.workload, KERNEL_NAMES[kind]), "algorithmic_bytes": bytes_,
-                "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs)",
-                "flops": algorithmic_flops(kind, B, H, T, D)}
+        roof = roofline(kind, args.workload, B, H, T, D, kern_ms, peaks)
+        for name, a in also.items():
+            k2, B2, H2, T2, D2 = WORKLOADS[name]
+            a["roofline"] = roofline(k2, name, B2, H2, T2, D2, a["kernel_ms_mean"], peaks)
+            del a["lms"]
         cpu = None
         if not args.no_cpu_baseline and world == 1:
             import oracle
@@ -499,7 +546,6 @@ def run_gpu(args):
                    "kind": "oracle",
                    "sample": (f"{sample_b} of {B} batch rows, all {H} heads, {Tc} of {T} tokens, "
                               f"{passes} passes ({secs:.1f} s)")}
-        sms = torch.cuda.get_device_properties(dev).multi_processor_count
         line = {
             "metric": METRIC_FWDBWD if kind == "glabwd" else METRIC, "value": value,
             "unit": "tokens/s", "n_gpus": world,
@@ -515,10 +561,12 @@ def run_gpu(args):
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": args.steps * launches_per_step(kind, B, H, T, sms),
-            "clocks": clocks.summary(),
+            "clocks": clock_summary,
             "kernel_ms_mean": kern_ms,
             "kernel_ms_min": min(launch_ms),
         }
+        if also:
+            line["also"] = also
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.barrier()
@@ -533,6 +581,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="gla_bf16_4k", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-also", action="store_true",
+                    help="time only the named workload (the default run also times gdn_bf16_4k)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -2,30 +2,33 @@
 //
 // The gated delta rule S_t = alpha_t S_{t-1}(I - beta_t kbar_t kbar_t^T) + beta_t v_t kbar_t^T
 // (the Gated DeltaNet write, Sec. 2.2) is kept as H = S^T [Dk][Dv].  Inside a 64-token
-// chunk with start state H0, gc_i the in-chunk cumulative log-decay and gc_m its value at
-// the chunk midpoint (token 31), unrolling the recurrence gives (chunkwise form):
+// chunk with start state H0, gc_i the in-chunk cumulative log-decay and gC its value at the
+// chunk's end, unrolling the recurrence gives (chunkwise form):
 //   A_ij = beta_i e^{gc_i - gc_j} kbar_i . kbar_j   (j < i),   Tt = (I + A)^{-1}
-//   U    = Tt diag(beta) V - Tt diag(beta e^{gc - gc_m}) Kbar (e^{gc_m} H0)
-//        = Tb (V - Diag(e^{gc - gc_m}) Kbar Hm),   Tb = Tt diag(beta)
-//   o_i  = scale [ e^{gc_i - gc_m} q_clean_i Hm + sum_{j<=i} e^{gc_i - gc_j}(q_clean_i . kbar_j) U_j ]
-//   H_C  = e^{gc_C - gc_m} [ Hm + sum_j e^{gc_m - gc_j} kbar_j U_j^T ]
-// with Hm = e^{gc_m} H0.  Tb depends only on the chunk's own keys, gates and betas, so it
-// is computed for every chunk in parallel by gdn_wy_kernel (64 x 64 bf16 per chunk, into a
-// caller workspace); gdn_chunk_kernel then walks the chunks of each (batch, head)
-// sequentially with the same warp-specialised structure as the GLA kernel and the same CCQ
-// read (App. B):
+//   U    = Tb (V - Diag(e^{gc}) Kbar H0),   Tb = Tt diag(beta)
+//   o_i  = scale [ e^{gc_i} q_clean_i H0 + sum_{j<=i} e^{gc_i - gc_j}(q_clean_i . kbar_j) U_j ]
+//   H_C  = e^{gC} H0 + sum_j e^{gC - gc_j} kbar_j U_j^T
+// Every decay factor is e^{x} with x <= 0 (gc_i, gC - gc_j and, per score entry, gc_i - gc_j
+// for j <= i), so no factor overflows however strong the forgetting, and a decay that
+// underflows contributes an exact zero.  Tb depends only on the chunk's own keys, gates and
+// betas, so it is computed for every chunk in parallel by gdn_wy_kernel (64 x 64 bf16 per
+// chunk, into a caller workspace); gdn_chunk_kernel then walks the chunks of each (batch,
+// head) sequentially with the same warp-specialised structure as the GLA kernel and the same
+// CCQ read (App. B):
 //
-//   G2  Sc  = Q Kbar^T           D2  KH = Kbar Hm
-//   (epilogue: W' of the CCQ mean fold;  R = V - Diag(e^{gc - gc_m}) KH -> bf16 R tile)
+//   G2  Sc  = Q Kbar^T           D2  KH = Kbar H0
+//   (epilogue: W' of the CCQ mean fold;  R = V - Diag(e^{gc}) KH -> bf16 R tile)
 //   G1  P   = Q S^K              DU  U = Tb R            G3  P += W' Kbar
-//   (epilogue: U -> bf16 U tile; q_clean e^{gc - gc_m} into the Q tile)
-//   D6  X  += Kd^T U             G8  S^K += Kbar^T Kbar      (Kd = kbar e^{gc_m - gc})
-//   D4  QK  = Qc Kbar^T          D3  O  = Qc Hm
-//   (epilogue: Pm_ij = [j<=i] QK_ij e^{gc_m - gc_j})
-//   D5  O  += Pm U
-//   (epilogue: o = scale O, TMA store)
-// X = e^{gc_m - gc_C} H_{r+1} stays in TMEM; the scalar e^{gc_C - gc_m} is applied at the
-// next snapshot.
+//   (epilogue: U -> bf16 U tile; q_clean into the Q tile)
+//   D6  X  += Kd^T U             G8  S^K += Kbar^T Kbar      (Kd = kbar e^{gC - gc})
+//   D4  QK  = Qc Kbar^T          D3  O1^T = H0^T Qc^T
+//   (epilogue: Pm_ij = [j<=i] QK_ij e^{gc_i - gc_j})
+//   D5  O2^T = U^T Pm^T
+//   (epilogue: o_i = scale (e^{gc_i} O1_i + O2_i), TMA store)
+// The two output products are transposed (M = 128 = Dv, N = 64 rows) into their own TMEM
+// accumulators, so the row factor e^{gc_i} of the inter-chunk read is applied in the output
+// epilogue.  X = H stays in TMEM; the snapshot that copies H0 to bf16 for D2 and D3 also
+// scales the TMEM copy by e^{gC}, so that D6 accumulates H_C onto it.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -75,8 +78,8 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
     float *Y = reinterpret_cast<float *>(sm + WY_Y);
     float *gcs = reinterpret_cast<float *>(sm + WY_MISC);        // [64] cumulative log decay
     float *bet = gcs + 64;                                        // [64] beta
-    float *epos = gcs + 128;                                      // [64] beta e^{gc - gc_m} / |k|
-    float *eneg = gcs + 192;                                      // [64] e^{gc_m - gc} / |k|
+    float *epos = gcs + 128;                                      // [64] beta / |k|
+    float *eneg = gcs + 192;                                      // [64] gc log2(e)
     float *rk = gcs + 256;                                        // [64] 1/|k|
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + WY_MISC + 1536);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(sm + WY_MISC + 1560);
@@ -153,25 +156,26 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         rk[i] = a.l2norm ? rsqrtf(fmaxf(d, 1e-12f)) : 1.f;
     }
     __syncthreads();
-    // row and column factors of A: A_ij = (beta_i e^{gc_i - gc_m} rk_i) (e^{gc_m - gc_j} rk_j) KK_ij
+    // row and column factors of A: A_ij = (beta_i rk_i) (rk_j) KK_ij e^{gc_i - gc_j}; the decay
+    // is one exponential of gc_i - gc_j <= 0 per entry (j < i), so no factor can overflow
+    // however strong the forgetting, and a decay that underflows gives an exact zero
     if (tid < 64) {
-        const float gm = gcs[31];
-        epos[tid] = bet[tid] * fast_exp2((gcs[tid] - gm) * kLog2e) * rk[tid];
-        eneg[tid] = fast_exp2((gm - gcs[tid]) * kLog2e) * rk[tid];
+        epos[tid] = bet[tid] * rk[tid];
+        eneg[tid] = gcs[tid] * kLog2e;  // log2 of the cumulative decay
     }
     __syncthreads();
     {
         // A_ij for j < i, written over the k tile (the product has read it)
-        const uint64_t ri2 = f2_make(epos[i], epos[i]);
+        const float ri = epos[i], li = eneg[i];
 #pragma unroll
         for (int q4 = 0; q4 < 8; ++q4) {
-            const ulonglong2 cf = *reinterpret_cast<const ulonglong2 *>(eneg + 32 * hf + 4 * q4);
-            const float2 a01 = f2_split(f2_mul(f2_mul(ri2, cf.x), f2_make(kk[4 * q4], kk[4 * q4 + 1])));
-            const float2 a23 = f2_split(f2_mul(f2_mul(ri2, cf.y), f2_make(kk[4 * q4 + 2], kk[4 * q4 + 3])));
-            const float av[4] = {a01.x, a01.y, a23.x, a23.y};
+            const float4 rkj = *reinterpret_cast<const float4 *>(rk + 32 * hf + 4 * q4);
+            const float4 lj = *reinterpret_cast<const float4 *>(eneg + 32 * hf + 4 * q4);
+            const float rkv[4] = {rkj.x, rkj.y, rkj.z, rkj.w}, lv[4] = {lj.x, lj.y, lj.z, lj.w};
             float w[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) w[e] = (32 * hf + 4 * q4 + e < i) ? av[e] : 0.f;
+            for (int e = 0; e < 4; ++e)
+                w[e] = (32 * hf + 4 * q4 + e < i) ? ri * rkv[e] * kk[4 * q4 + e] * fast_exp2(li - lv[e]) : 0.f;
             *reinterpret_cast<float4 *>(A + i * kAS + 32 * hf + 4 * q4) = make_float4(w[0], w[1], w[2], w[3]);
         }
     }
@@ -304,13 +308,13 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 // ============================================================================ main kernel
 //
 // Warp specialisation (13 warps), as in the GLA kernel:
-//   EPI   (warps 0-7)   the epilogues of chunk r -- W' and U = Ut - W Hm, q_clean, Pm,
+//   EPI   (warps 0-7)   the epilogues of chunk r -- W', R and U, q_clean, Pm,
 //                       output -- and the bf16 copies of S^K_{r+1} (while D4 runs) and
-//                       Hm_{r+1} (while G2 of chunk r+1 runs).  Warps w and w+4 share
+//                       H_{r+1} (while G2 of chunk r+1 runs).  Warps w and w+4 share
 //                       TMEM lane quadrant w % 4 and split its columns.
 //   PREP  (warps 8-11)  prep of chunk r+1: row norms, cumulative decay, kbar, Kd.
 //   ISSUE (warp 12)     every tcgen05.mma and TMA copy, in the order
-//                       G2 D2 | G1 | DU G3 G8 | D4 D6 D3 | D5.  D2 (Kbar Hm) lands in the
+//                       G2 D2 | G1 | DU G3 G8 | D4 D6 D3 | D5.  D2 (Kbar H0) lands in the
 //                       P/O accumulator, so EPI reads it out first and frees the accumulator
 //                       for G1 before it builds R; U = Tb R lands in TMEM columns 384-511
 //                       (Sc has been read, QK comes later).
@@ -321,26 +325,27 @@ constexpr int kEpiThreads = 256;
 constexpr int kPrepWarp0 = 8, kIssueWarp = 12;
 constexpr int kSyncCount = kEpiThreads + 32;
 constexpr uint32_t SLOT_BYTES = 49152;
-constexpr uint32_t SO_Q = 0;        // raw q, then q_clean e^{gc - gc_m}
+constexpr uint32_t SO_Q = 0;        // raw q, then q_clean
 constexpr uint32_t SO_K = 16384;    // raw k, then kbar
-constexpr uint32_t SO_KD = 32768;   // kbar e^{gc_m - gc}
+constexpr uint32_t SO_KD = 32768;   // kbar e^{gC - gc}
 constexpr uint32_t OFF_V = 98304;   // 16K  v of the chunk
 constexpr uint32_t OFF_TB = 114688; // 8K   Tb of the chunk (workspace), [64][64]
 constexpr uint32_t OFF_UB = 122880; // 16K  R, then U (bf16, rows j), after D5 the output staging
 constexpr uint32_t OFF_WM = 139264; // 8K   W' of the CCQ fold, then Pm
 constexpr uint32_t OFF_SK = 147456; // 32K  bf16 S^K
-constexpr uint32_t OFF_HB = 180224; // 32K  bf16 Hm = e^{gc_m} H
+constexpr uint32_t OFF_HB = 180224; // 32K  bf16 H0, the state entering the chunk
 constexpr uint32_t OFF_MISC = 212992;
 constexpr uint32_t MS_BYTES = 3072;
 constexpr uint32_t MS_RQ = 0, MS_MQ = 256, MS_LT = 512, MS_RK = 768, MS_EP = 1024, MS_EN = 1280,
                    MS_SCAL = 1536, MS_MST = 2048, MS_ITI = 2560, MS_QN = 2816;
-// SCAL: [0] e^{gc_m}, [1] e^{gc_C - gc_m}, [2..65] gc;  LT = lambda / t, ITI = 1 / t, QN = |q|
+// EP: e^{gc}, EN: e^{gC - gc}, SCAL: [1] e^{gC}, [2..65] gc;  LT = lambda / t, ITI = 1 / t, QN = |q|
 constexpr uint32_t M_DMP = 6144;     // [2][128] key-sum halves of the chunk
 constexpr uint32_t M_DMPREV = 7168;  // [128]
 constexpr uint32_t M_BAR = 7680;     // mbarriers
 constexpr uint32_t M_TMEM = 7808;
 constexpr uint32_t M_ABORT = 7812;
-constexpr uint32_t kMiscBytes = 7936;
+constexpr uint32_t M_EPO = 7936;     // [2][64] e^{gc} of the chunk whose output is being written
+constexpr uint32_t kMiscBytes = 8448;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;
 static_assert(kSmemBytes <= 232448, "exceeds the 227 KB per-CTA limit");
 static_assert(MS_SCAL + 66 * 4 <= MS_MST, "scalar area overlaps");
@@ -353,10 +358,13 @@ static_assert(M_BAR + 8 * kNumBars <= M_TMEM, "barrier area");
 enum { NB_PO = 1, NB_W = 2, NB_QC = 3, NB_MASK = 4, NB_OUT = 5, NB_PREP = 6, NB_EPI = 7 };
 
 constexpr uint32_t TM_S = 0, TM_SK = 128, TM_PO = 256, TM_SA = 384, TM_U = 384, kTmemCols = 512;
+// the transposed output accumulators (M = 128 layout) inside the P/O region
+constexpr uint32_t TM_O1 = 256, TM_O2 = 320;
 constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
 constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
 constexpr uint32_t ID_64x128_KM = make_idesc(64, 128, 0, 1);
 constexpr uint32_t ID_128x128_MM = make_idesc(128, 128, 1, 1);
+constexpr uint32_t ID_128x64_MK = make_idesc(128, 64, 1, 0);
 
 __global__ void __launch_bounds__(kThreads, 1)
 gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
@@ -488,7 +496,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             named_bar(NB_EPI, kEpiThreads);
             if (tid == 0) mbar_arrive(&bar[BAR_SNAPK]);
         };
-        // Hm = e^{gc_m} H = hs X, X rescaled in TMEM
+        // bf16 copy of the state H entering the next chunk; the TMEM copy is scaled by that
+        // chunk's e^{gC} (hs), onto which D6 accumulates the chunk's write
         auto snap_s = [&](float hs) {
             tc_fence_after();
 #pragma unroll
@@ -499,10 +508,10 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 uint32_t w[16];
 #pragma unroll
                 for (int e = 0; e < 16; ++e) {
+                    w[e] = pack_bf16(x[2 * e], x[2 * e + 1]);
                     const float2 y = f2_split(f2_mul(f2_make(x[2 * e], x[2 * e + 1]), hs2));
                     x[2 * e] = y.x;
                     x[2 * e + 1] = y.y;
-                    w[e] = pack_bf16(y.x, y.y);
                 }
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4)
@@ -516,18 +525,17 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             named_bar(NB_EPI, kEpiThreads);
             if (tid == 0) mbar_arrive(&bar[BAR_SNAPS]);
         };
-        float fc = 1.f;  // e^{gc_C - gc_m} of the chunk in flight
+        float *epo = reinterpret_cast<float *>(misc + M_EPO);
         if (NC > 0) {
             mbar_wait(&bar[BAR_PREP0], 0, abort_flag, status);
             snap_sk();
-            snap_s(slot_f(0, MS_SCAL)[0]);
+            snap_s(slot_f(0, MS_SCAL)[1]);
         }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1, par = r & 1;
             uint8_t *slot = sm + s * SLOT_BYTES;
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
-            fc = slot_f(s, MS_SCAL)[1];
             const float rqi = slot_f(s, MS_RQ)[i];
             const float mqi = slot_f(s, MS_MQ)[i];
             const float iti = slot_f(s, MS_ITI)[i];
@@ -562,7 +570,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     store_row_chunk(sm + OFF_WM, i, 4 * hf + 2 * grp + q2, w);
                 }
             }
-            // ---- R = V - e^{gc - gc_m} Kbar Hm: read Kbar Hm out of the P/O accumulator
+            // ---- R = V - e^{gc} Kbar H0: read Kbar H0 out of the P/O accumulator
             // first, freeing it for G1
             mbar_wait(&bar[BAR_GA2], par, abort_flag, status);
             tc_fence_after();
@@ -590,7 +598,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar_arrive(NB_W, kSyncCount);
-            // ---- q_clean (Eq. clean) scaled by e^{gc_i - gc_m}, into the Q tile
+            // ---- q_clean (Eq. clean) into the Q tile
             {
                 uint8_t *qt = slot + SO_Q + grp * 8192;
                 const float *Mst = slot_f(s, MS_MST) + 64 * grp + 32 * hf;
@@ -610,8 +618,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 const float cm = lt * c;
                 float p[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
-                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqi, rqi), cm2 = f2_make(cm, cm),
-                               ep2 = f2_make(ep, ep);
+                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqi, rqi), cm2 = f2_make(cm, cm);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4);
@@ -623,21 +630,20 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     for (int w = 0; w < 4; ++w) {
                         const uint64_t p2 = f2_make(p[8 * q4 + 2 * w], p[8 * q4 + 2 * w + 1]);
                         const uint64_t t = f2_fma(nlt, p2, f2_from_bf16x2(qw[w]));
-                        const uint64_t u = f2_fma(rq2, t, f2_mul(cm2, mp[w]));
-                        ow[w] = bf16x2_from_f2(f2_mul(ep2, u));
+                        ow[w] = bf16x2_from_f2(f2_fma(rq2, t, f2_mul(cm2, mp[w])));
                     }
                     *reinterpret_cast<uint4 *>(qt + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
                 }
             }
-            // e^{gc_m - gc_j} of this thread's 16 key columns, read before the slot is released
+            // gc_i - gc_j (log2 units) of this thread's 16 key columns, and e^{gc} of the rows for
+            // the output epilogue, read before the slot is released
             float ev[16];
             {
-                const float4 *en4 = reinterpret_cast<const float4 *>(slot_f(s, MS_EN) + 32 * hf + 16 * grp);
+                const float *gcv = slot_f(s, MS_SCAL) + 2;
+                const float gi = gcv[i];
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float4 e4 = en4[q];
-                    ev[4 * q] = e4.x; ev[4 * q + 1] = e4.y; ev[4 * q + 2] = e4.z; ev[4 * q + 3] = e4.w;
-                }
+                for (int q = 0; q < 16; ++q) ev[q] = (gi - gcv[32 * hf + 16 * grp + q]) * kLog2e;
+                if (tid < 64) epo[(r & 1) * 64 + tid] = slot_f(s, MS_EP)[tid];
             }
             fence_proxy_async_smem();
             tc_fence_before();
@@ -647,7 +653,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 mbar_wait(&bar[BAR_GK], par, abort_flag, status);
                 snap_sk();
             }
-            // ---- Pm_ij = [j<=i] QK_ij e^{gc_m - gc_j}
+            // ---- Pm_ij = [j<=i] QK_ij e^{gc_i - gc_j} (one exponential of a non-positive argument)
             mbar_wait(&bar[BAR_GC], par, abort_flag, status);
             tc_fence_after();
             {
@@ -660,7 +666,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     for (int e = 0; e < 8; ++e) {
                         const int jj = 8 * q2 + e;
                         const float v = grp ? sc[16 + jj] : sc[jj];
-                        w[e] = (32 * hf + 16 * grp + jj <= i) ? v * ev[jj] : 0.f;
+                        w[e] = (32 * hf + 16 * grp + jj <= i) ? v * fast_exp2(ev[jj]) : 0.f;
                     }
                     store_row_chunk(sm + OFF_WM, i, 4 * hf + 2 * grp + q2, w);
                 }
@@ -668,32 +674,44 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar_arrive(NB_MASK, kSyncCount);
-            // ---- output o = scale O, staged in the U tile for the TMA store
+            // ---- output o_i = scale (e^{gc_i} O1_i + O2_i), staged in the U tile for the TMA store.
+            // O1^T, O2^T are M = 128 accumulators: this thread holds value column `row` for the
+            // chunk rows 32 grp .. 32 grp + 31.
+            named_bar(NB_EPI, kEpiThreads);  // epo of this chunk visible
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             {
-                float x[32];
-                tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
-                const uint64_t sc2 = f2_make(a.scale, a.scale);
+                __nv_bfloat16 *ot = reinterpret_cast<__nv_bfloat16 *>(sm + OFF_UB + (row >> 6) * 8192);
+#pragma unroll 1
+                for (int hh = 0; hh < 2; ++hh) {
+                    const int i0 = 32 * grp + 16 * hh;
+                    float o1[16], o2[16];
+                    tmem_ld16(tq + TM_O1 + i0, o1);
+                    tmem_ld16(tq + TM_O2 + i0, o2);
+                    const float *ep_r = epo + (r & 1) * 64 + i0;
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    uint32_t w[4];
+                    for (int q = 0; q < 4; ++q) {
+                        const float4 e4 = *reinterpret_cast<const float4 *>(ep_r + 4 * q);
+                        const float ev4[4] = {e4.x, e4.y, e4.z, e4.w};
 #pragma unroll
-                    for (int u = 0; u < 4; ++u)
-                        w[u] = bf16x2_from_f2(f2_mul(f2_make(x[8 * q4 + 2 * u], x[8 * q4 + 2 * u + 1]), sc2));
-                    *reinterpret_cast<uint4 *>(sm + OFF_UB + grp * 8192 + t64_chunk(i, 4 * hf + q4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                        for (int u = 0; u < 4; ++u) {
+                            const int e = 4 * q + u;
+                            ot[t64_offset(i0 + e, row & 63) >> 1] =
+                                __float2bfloat16_rn(a.scale * fmaf(ev4[u], o1[e], o2[e]));
+                        }
+                    }
                 }
                 fence_proxy_async_smem();
             }
             tc_fence_before();
             named_bar_arrive(NB_OUT, kSyncCount);
-            // ---- Hm_{r+1} while G2 of chunk r+1 runs (D3, D6 of chunk r have run: GD follows them)
+            // ---- H_{r+1} while G2 of chunk r+1 runs (D3, D6 of chunk r have run: GD follows them)
             if (r + 1 < NC) {
                 mbar_wait(&bar[BAR_PREP0 + (s ^ 1)], ((r + 1) >> 1) & 1, abort_flag, status);
-                snap_s(fc * slot_f(s ^ 1, MS_SCAL)[0]);
+                snap_s(slot_f(s ^ 1, MS_SCAL)[1]);
             }
         }
-        // final states: H_T = e^{gc_C - gc_m} X (last chunk), S^K
+        // final states: H_T (the TMEM state after the last chunk), S^K
         if (NC > 0 && last_seg) {
             tc_fence_after();
             const size_t bhs = static_cast<size_t>(bh);
@@ -706,7 +724,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     float4 *dst = reinterpret_cast<float4 *>(a.ST + (bhs * kD + row) * kD + 32 * cl);
 #pragma unroll
                     for (int e = 0; e < 8; ++e)
-                        dst[e] = make_float4(fc * x[4 * e], fc * x[4 * e + 1], fc * x[4 * e + 2], fc * x[4 * e + 3]);
+                        dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
                 }
                 tmem_ld32(tq + TM_SK + 32 * cl, x);
                 if (a.CT) {
@@ -802,16 +820,13 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
             named_bar(NB_PREP, 128);  // gc, rk visible
             if (wt < 64) {
-                const float gm = scal[2 + 31];
-                slot_f(s, MS_EP)[wt] = fast_exp2((scal[2 + wt] - gm) * kLog2e);
-                slot_f(s, MS_EN)[wt] = fast_exp2((gm - scal[2 + wt]) * kLog2e);
-                if (wt == 0) {
-                    scal[0] = fast_exp2(gm * kLog2e);
-                    scal[1] = fast_exp2((scal[2 + 63] - gm) * kLog2e);
-                }
+                const float gC = scal[2 + 63];
+                slot_f(s, MS_EP)[wt] = fast_exp2(scal[2 + wt] * kLog2e);           // e^{gc} <= 1
+                slot_f(s, MS_EN)[wt] = fast_exp2((gC - scal[2 + wt]) * kLog2e);    // e^{gC - gc} <= 1
+                if (wt == 0) scal[1] = fast_exp2(gC * kLog2e);
             }
-            named_bar(NB_PREP, 128);  // e^{gc_m - gc} visible
-            // kbar (in place) and Kd = kbar e^{gc_m - gc}: thread = (row, T64 tile)
+            named_bar(NB_PREP, 128);  // e^{gC - gc} visible
+            // kbar (in place) and Kd = kbar e^{gC - gc}: thread = (row, T64 tile)
             {
                 const int j = wt >> 1, hh = wt & 1;
                 const float rkj = slot_f(s, MS_RK)[j], enj = slot_f(s, MS_EN)[j];
@@ -898,7 +913,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 }
                 __syncwarp();
             }
-            // D2 KH = Kbar Hm (needs the Hm copy)
+            // D2 KH = Kbar H0 (needs the H0 copy)
             mbar_wait(&bar[BAR_SNAPS], par, abort_flag, status);
             tc_fence_after();
             if (lead && !*abort_flag)
@@ -931,7 +946,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 mma_commit(&bar[BAR_GK]);
             }
             __syncwarp();
-            // D4 QK = Qc Kbar^T, D6 X += Kd^T U, D3 O = Qc Hm
+            // D4 QK = Qc Kbar^T, D6 X += Kd^T U, D3 O1^T = H0^T Qc^T
             named_bar(NB_QC, kSyncCount);
             tc_fence_after();
             if (lead && !*abort_flag) {
@@ -942,16 +957,17 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 }
                 mma_commit(&bar[BAR_GC]);
                 for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_S, dKDm + k * 128, dUBm + k * 128, ID_128x128_MM, 1);
+                // D3 O1^T = H0^T Qc^T (A = the H0 copy, MN-major; B = Qc, K-major)
                 for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
+                    mma_bf16(tbase + TM_O1, dHB + k * 128, dQ + (k >> 2) * 512 + (k & 3) * 2, ID_128x64_MK, k != 0);
                 mma_commit(&bar[BAR_GC2]);
             }
             __syncwarp();
-            // D5 O += Pm U
+            // D5 O2^T = U^T Pm^T (A = U, MN-major; B = Pm, K-major)
             named_bar(NB_MASK, kSyncCount);
             tc_fence_after();
             if (lead && !*abort_flag) {
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dUBm + k * 128, ID_64x128_KM, 1);
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_O2, dUBm + k * 128, dWm + k * 2, ID_128x64_MK, k != 0);
                 mma_commit(&bar[BAR_GD]);
             }
             __syncwarp();

@@ -4,15 +4,16 @@
 // chunks, as for CCQ-GLA (ccq_gla_segment.cu).  The gated delta state is affine in the
 // state entering a chunk: with H = S^T [Dk][Dv], Tb = Tt diag(beta) and the chunk factors
 // of ccq_gdn_chunk.cu,
-//   H_{r+1} = A_r H_r + B_r,   A_r = e^{gc_C} (I - Kd^T Tb Ke),   Ke = Diag(e^{gc - gc_m}) Kbar,
-//   B_r = e^{gc_C - gc_m} Kd^T Tb V,
-// so a segment maps its entering state H to P H + Q, with P the product of its A_r and Q
-// the state it reaches from zero.  The covariance C and key sum m are plain sums.  Three
-// launches replace the long walk:
+//   H_{r+1} = A_r H_r + B_r,   A_r = e^{gC} I - Kd^T Tb Ke,   Ke = Diag(e^{gc}) Kbar,
+//   Kd = Diag(e^{gC - gc}) Kbar,   B_r = Kd^T Tb V,
+// every factor an exponential of a non-positive argument, so a segment maps its entering
+// state H to P H + Q, with P the product of its A_r and Q the state it reaches from zero.
+// The covariance C and key sum m are plain sums.  Three launches replace the long walk:
 //   1. gdn_segment_state_kernel: per (sequence, segment), from a zero state, Q, P, dC, dm.
-//      P = e^{sum gc_C} Pt with Pt updated exactly like the state without its V term, so one
-//      set of products serves both: with Z = [Qm | Pt] (Dk x 2Dv),
-//        Y^T = Z^T Ke^T,  R^T = [V^T - Y_Q^T | -Y_P^T],  U^T = R^T Tb^T,  [X | Pt] += Kd^T U
+//      P is updated exactly like the state without its V term, so one set of products
+//      serves both: with Z = [Q | P] (Dk x 2Dv),
+//        Y^T = Z^T Ke^T,  R^T = [V^T - Y_Q^T | -Y_P^T],  U^T = R^T Tb^T,
+//        [Q | P] = e^{gC} [Q | P] + Kd^T U
 //      (M = 128 products over the transposed operands, so everything fits 512 TMEM columns).
 //   2. gdn_segment_combine_kernel: per (sequence, 16 state columns), H_{s+1} = P_s H_s + Q_s,
 //      C and m by prefix sums, in fp32; each slot then holds its segment's entering states.
@@ -40,14 +41,14 @@ constexpr int kSS = kD * kD;
 // shared memory: two slots of {k 16K, v 16K, Tb 8K}, then Ke, Kd, Z, R/U and scratch
 constexpr uint32_t SL_BYTES = 40960;
 constexpr uint32_t SL_K = 0, SL_V = 16384, SL_TB = 32768;
-constexpr uint32_t OFF_KE = 81920;    // 16K  e^{gc - gc_m} kbar (K-major B of Y^T)
-constexpr uint32_t OFF_KD = 98304;    // 16K  e^{gc_m - gc} kbar (MN-major A of the state update)
-constexpr uint32_t OFF_Z = 114688;    // 64K  bf16 [Qm | Pt], [128 rows][256 cols] as four T64 tiles
+constexpr uint32_t OFF_KE = 81920;    // 16K  e^{gc} kbar (K-major B of Y^T)
+constexpr uint32_t OFF_KD = 98304;    // 16K  e^{gC - gc} kbar (MN-major A of the state update)
+constexpr uint32_t OFF_Z = 114688;    // 64K  bf16 [Q | P], [128 rows][256 cols] as four T64 tiles
 constexpr uint32_t OFF_RU = 180224;   // 32K  bf16 R^T, then U^T: [256 rows][64 cols] as two T64 tiles
 constexpr uint32_t OFF_MISC = 212992;
 constexpr uint32_t M_GC = 0;      // [64] cumulative log decay
-constexpr uint32_t M_EP = 256;    // [64] e^{gc - gc_m}
-constexpr uint32_t M_EN = 512;    // [64] e^{gc_m - gc}
+constexpr uint32_t M_EP = 256;    // [64] e^{gc}
+constexpr uint32_t M_EN = 512;    // [64] e^{gC - gc}
 constexpr uint32_t M_RK = 768;    // [64] 1/|k|
 constexpr uint32_t M_DMP = 1024;  // [4][128] key-sum quarters
 constexpr uint32_t M_BAR = 3072;  // in[2], mma
@@ -56,11 +57,11 @@ constexpr uint32_t kSmem = OFF_MISC + 4096 + 1024;
 static_assert(kSmem <= 232448, "smem");
 
 // TMEM columns
-constexpr uint32_t TM_X = 0, TM_PT = 128, TM_DC = 256, TM_YU = 384;
+constexpr uint32_t TM_X = 0, TM_PT = 128, TM_DC = 256, TM_YU = 384;  // Q, P, dC, Y^T / U^T
 
 constexpr uint32_t ID_Y = make_idesc(128, 64, 1, 0);     // Y^T = Z^T Ke^T
 constexpr uint32_t ID_U = make_idesc(128, 64, 0, 0);     // U^T = R^T Tb^T
-constexpr uint32_t ID_ST = make_idesc(128, 256, 1, 0);   // [X | Pt] += Kd^T U
+constexpr uint32_t ID_ST = make_idesc(128, 256, 1, 0);   // [Q | P] += Kd^T U
 constexpr uint32_t ID_DC = make_idesc(128, 128, 1, 1);   // dC += Kbar^T Kbar
 
 __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chunk, const float *w) {
@@ -127,7 +128,7 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
         tma_prefetch_desc(&map_tb);
         issue_in(0);
     }
-    // X = 0, Pt = I, dC = 0 (this thread: row `row`, the 128 columns of half hz)
+    // Q = 0, P = I, dC = 0 (this thread: row `row`, the 128 columns of half hz)
     {
         float x[32];
 #pragma unroll
@@ -147,8 +148,6 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
         g_reg = t < T ? a.g[(static_cast<size_t>(b) * T + t) * H + h] : 0.f;
     }
     float dm_acc = 0.f;      // key sum of dim tid (tid < 128)
-    float lsum = 0.f;        // sum of gc_C over the chunks done (P's scalar, natural log)
-    float f_prev = 1.f;      // e^{gc_C - gc_m} of the previous chunk (X's deferred factor)
     tc_fence_before();
     __syncthreads();
 
@@ -199,12 +198,11 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
             if (qq == 0) rkv[j] = a.l2norm ? rsqrtf(fmaxf(ss, 1e-12f)) : 1.f;
         }
         __syncthreads();  // gc, rk visible
+        const float gC = gc[63];
         if (tid < 64) {
-            const float gm = gc[31];
-            epv[tid] = fast_exp2((gc[tid] - gm) * kLog2e);
-            env[tid] = fast_exp2((gm - gc[tid]) * kLog2e);
+            epv[tid] = fast_exp2(gc[tid] * kLog2e);         // e^{gc} <= 1
+            env[tid] = fast_exp2((gC - gc[tid]) * kLog2e);  // e^{gC - gc} <= 1
         }
-        const float gm = gc[31], gC = gc[63];
         __syncthreads();  // factors visible
         {
             const float rk = rkv[j];
@@ -246,27 +244,24 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
             const uint64_t dKm = make_desc(sb + s * SL_BYTES + SL_K, 8192, 1024);
             for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_DC, dKm + k * 128, dKm + k * 128, ID_DC, 1);
         }
-        // ---- Z = [e^{gc_m} X f_prev | Pt] (X rescaled in TMEM)
+        // ---- Z = [Q | P] as bf16; the TMEM copies scaled by e^{gC}, onto which the state
+        // update of this chunk accumulates
         tc_fence_after();
         {
-            const float hs = f_prev * fast_exp2(gm * kLog2e);
+            const float hs = fast_exp2(gC * kLog2e);
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 float x[32];
                 tmem_ld32(tq + (hz ? TM_PT : TM_X) + 32 * c, x);
-                if (hz == 0) {
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) x[e] *= hs;
-                    tmem_st32(tq + TM_X + 32 * c, x);
-                }
                 uint8_t *tile = sm + OFF_Z + (2 * hz + (c >> 1)) * 16384;
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) store_row_chunk(tile, row, 4 * (c & 1) + q4, x + 8 * q4);
+#pragma unroll
+                for (int e = 0; e < 32; ++e) x[e] *= hs;
+                tmem_st32(tq + (hz ? TM_PT : TM_X) + 32 * c, x);
             }
             tmem_wait_st();
         }
-        f_prev = fast_exp2((gC - gm) * kLog2e);
-        lsum += gC;
         __syncthreads();
         if (tid < kD) dm_acc += (dmp[tid] + dmp[kD + tid]) + (dmp[2 * kD + tid] + dmp[3 * kD + tid]);
         fence_proxy_async_smem();
@@ -335,7 +330,7 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
-        // ---- [X | Pt] += Kd^T U (N = 256: U^T rows 0..255 across both tiles)
+        // ---- [Q | P] += Kd^T U (N = 256: U^T rows 0..255 across both tiles)
         if (tid == 0 && !*abort_flag) {
             tc_fence_after();
             const uint64_t dKDm = make_desc(sb + OFF_KD, 8192, 1024);
@@ -344,19 +339,18 @@ gdn_segment_state_kernel(const __grid_constant__ CUtensorMap map_k, const __grid
             mma_commit(&bar[2]);
         }
     }
-    // ---- outputs: Q = f X, P = e^{lsum} Pt, dC, dm
+    // ---- outputs: Q, P, dC, dm
     if (n > 0) mbar_wait(&bar[2], (3 * (n - 1) + 2) & 1, abort_flag, status);
     tc_fence_after();
     float *out = a.seg_ws + static_cast<size_t>(blockIdx.x) * kGdnSegFloats;
     {
-        const float sc = hz ? fast_exp2(lsum * kLog2e) : f_prev;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             float x[32];
             tmem_ld32(tq + (hz ? TM_PT : TM_X) + 32 * c, x);
             float4 *dst = reinterpret_cast<float4 *>(out + hz * kSS + row * kD + 32 * c);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) dst[e] = make_float4(sc * x[4 * e], sc * x[4 * e + 1], sc * x[4 * e + 2], sc * x[4 * e + 3]);
+            for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
             if (hz == 0) {
                 tmem_ld32(tq + TM_DC + 32 * c, x);
                 float4 *dc = reinterpret_cast<float4 *>(out + 2 * kSS + row * kD + 32 * c);

@@ -22,7 +22,17 @@ the order q, k, v, gate, beta, lambda, then cast to the requested dtype):
                  low-rank key spread with a non-zero mean, so Sigma_t is large and
                  the mean term matters; or "lowrank": k = normalise(U z + 0.1 eps)
                  with a fixed orthonormal d x 2 basis U, so Sigma_t has two
-                 eigenvalues near 1/2 and the CCQ correction is large.
+                 eigenvalues near 1/2 and the CCQ correction is large; or "rank2": the
+                 same with 0.01 eps, so that the keys lie almost in the subspace.
+  queries        "iso" (above) or "lowrank": q = U z + 0.01 eps in the same d x 2
+                 subspace as the low-rank keys (drawn after lambda, so the other
+                 draws are unchanged); with "rank2" keys and lambda near 1 the CCQ
+                 term is more than half of o.
+  gates          "default" (above); "strong": GLA logsigmoid(N(0,1)) without the
+                 1/16, GDN -8 softplus(N(0,1)) (about -6 per token, as strongly
+                 forgetting trained heads); or a float c: every GLA log-gate entry,
+                 or every GDN log decay, equal to c (c <= 0).  The normal draw of the
+                 default gate is made in every case, so the other draws are unchanged.
 """
 from __future__ import annotations
 
@@ -49,12 +59,12 @@ def _structured_keys(gen, B, T, H, Dk, rank=16):
     return m0 + z @ U.T + 0.25 * eps
 
 
-def _lowrank_keys(gen, B, T, H, Dk, rank=2):
+def _lowrank_keys(gen, B, T, H, Dk, rank=2, noise=0.1):
     basis_gen = torch.Generator().manual_seed(104729)
     U, _ = torch.linalg.qr(torch.randn(Dk, rank, generator=basis_gen))
     z = torch.randn(B, T, H, rank, generator=gen)
     eps = torch.randn(B, T, H, Dk, generator=gen)
-    return z @ U.T + 0.1 * eps
+    return z @ U.T + noise * eps
 
 
 def _lambda(gen, B, T, H, lam):
@@ -72,7 +82,7 @@ def _lambda(gen, B, T, H, lam):
 
 def make_inputs(backbone: int, B: int, T: int, H: int, Dk: int, Dv: int, *,
                 dtype=torch.bfloat16, gate_dtype=None, seed: int = 1234,
-                lam="init", keys: str = "iso") -> dict:
+                lam="init", keys: str = "iso", queries: str = "iso", gates="default") -> dict:
     """Draw one CCQ forward problem on the CPU.
 
     Returns a dict of CPU tensors: q, k [B,T,H,Dk] and v [B,T,H,Dv] in
@@ -88,6 +98,8 @@ def make_inputs(backbone: int, B: int, T: int, H: int, Dk: int, Dv: int, *,
         k = _structured_keys(gen, B, T, H, Dk)
     elif keys == "lowrank":
         k = _lowrank_keys(gen, B, T, H, Dk)
+    elif keys == "rank2":
+        k = _lowrank_keys(gen, B, T, H, Dk, noise=0.01)
     else:
         raise ValueError(f"unknown key distribution {keys!r}")
     k = _normalise_rows(k)
@@ -95,13 +107,37 @@ def make_inputs(backbone: int, B: int, T: int, H: int, Dk: int, Dv: int, *,
         q = _normalise_rows(q)
     v = torch.randn(B, T, H, Dv, generator=gen)
     if backbone == GLA:
-        gate = F.logsigmoid(torch.randn(B, T, H, Dk, generator=gen)) / 16
+        z = torch.randn(B, T, H, Dk, generator=gen)
+        if gates == "default":
+            gate = F.logsigmoid(z) / 16
+        elif gates == "strong":
+            gate = F.logsigmoid(z)
+        elif isinstance(gates, (int, float)) and gates <= 0:
+            gate = torch.full_like(z, float(gates))
+        else:
+            raise ValueError(f"unknown gate distribution {gates!r}")
         gate = gate.to(gate_dtype or dtype)
         beta = None
     else:
-        gate = -F.softplus(torch.randn(B, T, H, generator=gen))
+        z = torch.randn(B, T, H, generator=gen)
+        if gates == "default":
+            gate = -F.softplus(z)
+        elif gates == "strong":
+            gate = -8.0 * F.softplus(z)
+        elif isinstance(gates, (int, float)) and gates <= 0:
+            gate = torch.full_like(z, float(gates))
+        else:
+            raise ValueError(f"unknown gate distribution {gates!r}")
         beta = torch.sigmoid(torch.randn(B, T, H, generator=gen))
     lam_t = _lambda(gen, B, T, H, lam)
+    if queries == "lowrank":
+        basis_gen = torch.Generator().manual_seed(104729)
+        U, _ = torch.linalg.qr(torch.randn(Dk, 2, generator=basis_gen))
+        q = torch.randn(B, T, H, 2, generator=gen) @ U.T + 0.01 * torch.randn(B, T, H, Dk, generator=gen)
+        if backbone == GDN:
+            q = _normalise_rows(q)
+    elif queries != "iso":
+        raise ValueError(f"unknown query distribution {queries!r}")
     return {"q": q.to(dtype), "k": k.to(dtype), "v": v.to(dtype), "gate": gate,
             "beta": beta, "lam": lam_t.float()}
 

@@ -133,7 +133,36 @@ def test_gdn_chunkwise_correction_isolated():
     d_ref = ref1 - oracle_forward(GDN, P0)["o"]
     d = o1.double().cpu().numpy() - o0.double().cpu().numpy()
     assert np.abs(d_ref).max() > 0.1 * np.abs(ref1).max()
-    assert rel_err(d, d_ref) <= correction_bound(ref1, d_ref, torch.bfloat16)
+    bound, err = correction_bound(ref1, d_ref, torch.bfloat16), rel_err(d, d_ref)
+    assert err <= bound, f"isolated CCQ term: error {err:.3e} above its bound {bound:.3e}"
+
+
+def test_gdn_correction_dominant():
+    """Keys and queries in one two-dimensional subspace with lambda = 0.9: the CCQ term is more than
+    half of the output (rounding floor of the bound below 1 %)."""
+    P = gen.make_inputs(GDN, 1, 192, 2, 128, 128, dtype=torch.bfloat16, seed=15, lam="high", keys="rank2",
+                        queries="lowrank")
+    P0 = dict(P, lam=torch.zeros_like(P["lam"]))
+    o1, _ = gpu_forward(GDN, P)
+    o0, _ = gpu_forward(GDN, P0)
+    ref1 = oracle_forward(GDN, P)["o"]
+    d_ref = ref1 - oracle_forward(GDN, P0)["o"]
+    d = o1.double().cpu().numpy() - o0.double().cpu().numpy()
+    assert np.abs(d_ref).max() >= 0.5 * np.abs(ref1).max()
+    bound, err = correction_bound(ref1, d_ref, torch.bfloat16), rel_err(d, d_ref)
+    assert bound <= TOL[torch.bfloat16] + 0.008
+    assert err <= bound, f"isolated CCQ term: error {err:.3e} above its bound {bound:.3e}"
+
+
+@pytest.mark.parametrize("opts", [dict(l2norm=False), dict(scale=0.37), dict(l2norm=False, centered=False)])
+def test_gdn_forward_options(opts):
+    """Chunkwise Gated DeltaNet without in-kernel normalisation (the generator's unit q, k)
+    and with a read scale other than 1/sqrt(d_k)."""
+    P = gen.make_inputs(GDN, 2, 200, 2, 128, 128, dtype=torch.bfloat16, seed=16, lam="trained",
+                        keys="structured")
+    o, fs = gpu_forward(GDN, P, **opts)
+    ref = oracle_forward(GDN, P, **opts)
+    compare(o, fs, ref, TOL[torch.bfloat16], f"GDN {opts}")
 
 
 def test_gdn_chunkwise_resume_and_matches_recurrent():

@@ -50,7 +50,38 @@ def test_correction_isolated(algo, dtype):
     d_ref = ref1 - oracle_forward(GLA, P0)["o"]
     d = o1.double().cpu().numpy() - o0.double().cpu().numpy()
     assert np.abs(d_ref).max() > 0.1 * np.abs(ref1).max()
-    assert rel_err(d, d_ref) <= correction_bound(ref1, d_ref, dtype)
+    bound, err = correction_bound(ref1, d_ref, dtype), rel_err(d, d_ref)
+    assert err <= bound, f"isolated CCQ term: error {err:.3e} above its bound {bound:.3e}"
+
+
+@pytest.mark.parametrize("algo", ["chunkwise", "recurrent"])
+def test_correction_dominant(algo):
+    """Keys and queries in one two-dimensional subspace with lambda = 0.9: the CCQ term is more than
+    half of the output, so the rounding floor of the isolated-term bound stays below 1 %."""
+    P = gen.make_inputs(GLA, 1, 192, 2, 128, 128, dtype=torch.bfloat16, seed=13, lam="high", keys="rank2",
+                        queries="lowrank")
+    P0 = dict(P, lam=torch.zeros_like(P["lam"]))
+    o1, _ = gpu_forward(GLA, P, algo=algo)
+    o0, _ = gpu_forward(GLA, P0, algo=algo)
+    ref1 = oracle_forward(GLA, P)["o"]
+    d_ref = ref1 - oracle_forward(GLA, P0)["o"]
+    d = o1.double().cpu().numpy() - o0.double().cpu().numpy()
+    assert np.abs(d_ref).max() >= 0.5 * np.abs(ref1).max()
+    bound, err = correction_bound(ref1, d_ref, torch.bfloat16), rel_err(d, d_ref)
+    assert bound <= TOL[torch.bfloat16] + 0.008
+    assert err <= bound, f"isolated CCQ term: error {err:.3e} above its bound {bound:.3e}"
+
+
+@pytest.mark.parametrize("opts", [dict(l2norm=False), dict(scale=0.37), dict(l2norm=False, centered=False)])
+@pytest.mark.parametrize("algo", ["chunkwise", "recurrent"])
+def test_forward_options(opts, algo):
+    """The forward without in-kernel normalisation (unit keys from the generator, raw queries)
+    and with a read scale other than 1/sqrt(d_k)."""
+    P = gen.make_inputs(GLA, 2, 200, 2, 128, 128, dtype=torch.bfloat16, seed=14, lam="trained",
+                        keys="structured")
+    o, fs = gpu_forward(GLA, P, algo=algo, **opts)
+    ref = oracle_forward(GLA, P, **opts)
+    compare(o, fs, ref, TOL[torch.bfloat16], f"GLA {algo} {opts}")
 
 
 def test_chunkwise_matches_recurrent_gpu():
