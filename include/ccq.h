@@ -60,7 +60,8 @@ typedef enum {
     CCQ_ERR_INVALID_ARG = 1, /* NULL or misaligned pointer, negative size, ...    */
     CCQ_ERR_UNSUPPORTED = 2, /* a valid request this build does not implement     */
     CCQ_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed                 */
-    CCQ_ERR_TIMEOUT = 4      /* an in-kernel bounded wait ran out (device status) */
+    CCQ_ERR_TIMEOUT = 4,     /* an in-kernel bounded wait ran out (device status) */
+    CCQ_ERR_RANGE = 5        /* a chunk's gates left the range the kernel can factor (device status) */
 } ccq_status;
 
 typedef enum { CCQ_BF16 = 0, CCQ_FP32 = 1 } ccq_dtype;
@@ -76,7 +77,10 @@ typedef enum {
 typedef enum {
     CCQ_ALGO_AUTO = 0,      /* chunkwise tensor-core kernel when supported, else recurrent */
     CCQ_ALGO_RECURRENT = 1, /* token-by-token CUDA-core kernel (fp32 arithmetic)         */
-    CCQ_ALGO_CHUNKWISE = 2  /* chunkwise tcgen05 kernel (bf16 operands, fp32 accumulate)  */
+    CCQ_ALGO_CHUNKWISE = 2, /* chunkwise tcgen05 kernel (bf16 operands, fp32 accumulate)  */
+    CCQ_ALGO_CHUNKWISE_WIDE = 3 /* CCQ-GLA: the chunkwise kernel with two gate references per
+                                   chunk, for strongly forgetting gates (see ccq_gla_fwd); about
+                                   twice the time.  Gated DeltaNet: the same as CHUNKWISE.   */
 } ccq_algo;
 
 /* Contraction and read hyper-parameters. */
@@ -109,9 +113,18 @@ CCQ_API void ccq_default_params(ccq_params *p);
  * Supported: Dk = Dv in {64, 128}; T >= 0; B, H >= 1.  in_dtype BF16 runs the
  * chunkwise tensor-core kernel for Dk = Dv = 128 and the recurrent kernel
  * otherwise; FP32 always runs the recurrent kernel (fp32 arithmetic).
- * The chunkwise kernel scales by exp of in-chunk cumulative gates measured from
- * the chunk midpoint; per-chunk cumulative log-gates must stay above about -160
- * (more negative sums underflow to an exact-zero contribution).
+ * Gate range of the chunkwise kernels.  A chunk's decays are applied as factors
+ * measured from reference tokens inside the chunk.  The default kernel (AUTO,
+ * CHUNKWISE) has one reference, the chunk midpoint; it is exact (up to rounding)
+ * while, for every key dimension, the log gates of each 32-token half of a chunk
+ * sum to more than about -82 (e.g. per-token log gates above -2.5).  CHUNKWISE_WIDE
+ * has one reference per half, which doubles that range (each 16-token quarter
+ * above about -82, e.g. per-token log gates above -5) at about twice the time.
+ * Beyond its range a kernel records CCQ_ERR_RANGE in the device status word
+ * (ccq_device_status) and its outputs are not valid; the recurrent path
+ * (algo RECURRENT) has no range limit.  Within range, a decay that underflows
+ * contributes an exact zero.  The backward (ccq_gla_bwd) has the default
+ * kernel's range.
  *   workspace  caller-owned device scratch of at least ccq_gla_workspace_size()
  *              bytes (16-byte aligned) when that size is non-zero (long sequences
  *              split into segments); may be NULL otherwise.  Contents undefined on
@@ -142,8 +155,11 @@ CCQ_API ccq_status ccq_gla_workspace_size(int B, int T, int H, int Dk, int Dv, c
  *             when that size is 0.  Its contents on entry do not matter and are
  *             undefined on return.
  * All other arguments as ccq_gla_fwd.  bf16 inputs with Dk = Dv = 128 run the chunkwise
- * tensor-core kernels (CCQ_ALGO_AUTO / CHUNKWISE; CCQ_ERR_INVALID_ARG if the workspace is
- * missing or too small); other inputs run the recurrent kernel.
+ * tensor-core kernels (CCQ_ALGO_AUTO / CHUNKWISE / CHUNKWISE_WIDE, which are the same here;
+ * CCQ_ERR_INVALID_ARG if the workspace is missing or too small); other inputs run the
+ * recurrent kernel.  Every decay factor of the chunkwise kernels is an exponential of a
+ * non-positive argument (e^{gc_i}, e^{gC - gc_j} and, per score entry, e^{gc_i - gc_j}), so
+ * any g <= 0 is supported; a decay that underflows contributes an exact zero.
  */
 CCQ_API ccq_status ccq_gdn_fwd(const void *q, const void *k, const void *v, const float *g,
                        const float *beta, const float *lambda, ccq_dtype in_dtype,
@@ -186,7 +202,7 @@ CCQ_API ccq_status ccq_gla_ckpt_size(int B, int T, int H, int Dk, int Dv, size_t
  * ccq_gla_ckpt_size() bytes, 16-byte aligned), the chunk-start states the
  * backward needs, so that ccq_gla_bwd does not recompute them (a training
  * step's forward).  Only the chunkwise tensor-core path saves checkpoints:
- * bf16 inputs, Dk = Dv = 128, T >= 1, algo AUTO or CHUNKWISE; anything else
+ * bf16 inputs, Dk = Dv = 128, T >= 1, algo AUTO, CHUNKWISE or CHUNKWISE_WIDE; anything else
  * returns CCQ_ERR_UNSUPPORTED.  All other arguments as ccq_gla_fwd.
  */
 CCQ_API ccq_status ccq_gla_fwd_save(const void *q, const void *k, const void *v, const void *gk,
@@ -385,7 +401,8 @@ CCQ_API ccq_status ccq_gla_fwd_fixed_scratch(const void *q, const void *k, const
 
 /*
  * Synchronise `stream`, then read and clear the device status word that the
- * kernels' bounded waits write.  Returns CCQ_OK, CCQ_ERR_TIMEOUT (a kernel gave
+ * kernels write.  Returns CCQ_OK, CCQ_ERR_RANGE (a chunkwise CCQ-GLA kernel met
+ * gates stronger than its factored decays can represent: see ccq_gla_fwd), CCQ_ERR_TIMEOUT (a kernel gave
  * up waiting; its outputs are not valid) or CCQ_ERR_CUDA.
  */
 CCQ_API ccq_status ccq_device_status(void *stream);

@@ -18,9 +18,9 @@ import torch
 
 from . import _build
 
-CCQ_OK, CCQ_ERR_INVALID_ARG, CCQ_ERR_UNSUPPORTED, CCQ_ERR_CUDA, CCQ_ERR_TIMEOUT = range(5)
+CCQ_OK, CCQ_ERR_INVALID_ARG, CCQ_ERR_UNSUPPORTED, CCQ_ERR_CUDA, CCQ_ERR_TIMEOUT, CCQ_ERR_RANGE = range(6)
 BF16, FP32 = 0, 1
-ALGO = {"auto": 0, "recurrent": 1, "chunkwise": 2}
+ALGO = {"auto": 0, "recurrent": 1, "chunkwise": 2, "wide": 3}
 GLA, GDN = 0, 1
 
 

@@ -85,7 +85,7 @@ ccq_status check_common(const ccq_params *pin, int B, int T, int H, int Dk, int 
         return fail(CCQ_ERR_UNSUPPORTED, "head dims Dk=%d Dv=%d: supported Dk = Dv in {64, 128}", Dk, Dv);
     if (c->p.chunk != 0 && c->p.chunk != 64)
         return fail(CCQ_ERR_UNSUPPORTED, "chunk=%d: supported 64", c->p.chunk);
-    if (c->p.algo < CCQ_ALGO_AUTO || c->p.algo > CCQ_ALGO_CHUNKWISE)
+    if (c->p.algo < CCQ_ALGO_AUTO || c->p.algo > CCQ_ALGO_CHUNKWISE_WIDE)
         return fail(CCQ_ERR_INVALID_ARG, "unknown algo %d", c->p.algo);
     if (c->p.seq_split < 0) return fail(CCQ_ERR_INVALID_ARG, "seq_split must be >= 0");
     if ((static_cast<long long>(B) * H) > 0x7fffffffLL)
@@ -194,6 +194,7 @@ const char *ccq_status_string(ccq_status s) {
         case CCQ_ERR_UNSUPPORTED: return "unsupported configuration";
         case CCQ_ERR_CUDA: return "CUDA error";
         case CCQ_ERR_TIMEOUT: return "a kernel's bounded wait timed out";
+        case CCQ_ERR_RANGE: return "gates outside the range the chunkwise kernel can factor";
     }
     return "unknown status";
 }
@@ -271,7 +272,7 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
     }
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const bool chunk_ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
-    if ((c.p.algo == CCQ_ALGO_CHUNKWISE || ckpt) && !chunk_ok)
+    if ((c.p.algo == CCQ_ALGO_CHUNKWISE || c.p.algo == CCQ_ALGO_CHUNKWISE_WIDE || ckpt) && !chunk_ok)
         return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
     if (ckpt && c.p.algo == CCQ_ALGO_RECURRENT)
         return fail(CCQ_ERR_UNSUPPORTED, "checkpoints come from the chunkwise kernel (algo recurrent given)");
@@ -299,6 +300,8 @@ static ccq_status gla_fwd_impl(const void *q, const void *k, const void *v, cons
         a.gate_dtype = gate_dtype == CCQ_BF16 ? 0 : 1;
         a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
         a.lambda = lambda;
+        a.gk = gk;
+        a.wide = c.p.algo == CCQ_ALGO_CHUNKWISE_WIDE;
         a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
         a.o = static_cast<__nv_bfloat16 *>(o);
         a.ST = ST; a.CT = CT; a.mT = mT;
@@ -536,7 +539,7 @@ static ccq_status gdn_fwd_impl(const void *q, const void *k, const void *v, cons
         if (st != CCQ_OK) return st;
     }
     const bool chunk_ok = in_dtype == CCQ_BF16 && Dk == 128 && T > 0;
-    if (c.p.algo == CCQ_ALGO_CHUNKWISE && !chunk_ok)
+    if ((c.p.algo == CCQ_ALGO_CHUNKWISE || c.p.algo == CCQ_ALGO_CHUNKWISE_WIDE) && !chunk_ok)
         return fail(CCQ_ERR_UNSUPPORTED, "chunkwise kernel needs bf16 inputs, Dk = Dv = 128, T > 0");
     if (gdn_chunk_selected(c.p, in_dtype, Dk, T)) {
         const size_t need = gdn_total_workspace(c.p, B, T, H);
@@ -876,6 +879,9 @@ ccq_status ccq_device_status(void *stream) {
         const int zero = 0;
         e = cudaMemcpyToSymbol(ccq::g_status, &zero, sizeof(int));
         if (e != cudaSuccess) return cuda_fail(e, "clear device status");
+        if (v == static_cast<int>(CCQ_ERR_RANGE))  // the kernels write the status code itself
+            return fail(CCQ_ERR_RANGE, "device status %d: a chunk's cumulative log gates over 16 tokens fell "
+                                       "below about -87 (see ccq_gla_fwd); the outputs are not valid", v);
         return fail(CCQ_ERR_TIMEOUT, "device status %d: an in-kernel wait gave up", v);
     }
     return CCQ_OK;

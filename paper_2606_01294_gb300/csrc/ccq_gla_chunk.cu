@@ -28,7 +28,13 @@
 //   q_clean_i = qbar_i - lambda_i (rq_i P_i - c_i M) / t_i          (Eq. clean)
 // GLA gates are measured from the chunk midpoint Gmid: Qg = q_clean * e^{G - Gmid},
 // Kg = kbar * e^{Gmid - G}, Ssnap = e^{Gmid} S_r, and S_{r+1} = e^{Gtot - Gmid} X_{r+1}
-// (that factor is applied at the next snapshot).
+// (that factor is applied at the next snapshot).  A factor e^{G - Gmid} of a row before the
+// midpoint grows with the decay between that row and the midpoint, so the factoring is exact
+// (up to rounding) only while each 32-token half of a chunk sums its log gates to more than
+// about -82 per key dimension (2^118, where the state update from keys scaled that much still
+// fits fp32).  The prep warps check every factor's exponent and record CCQ_ERR_RANGE in the
+// status word when a chunk goes beyond that; the two-reference kernel (ccq_gla_chunk_wide.cu,
+// algo CCQ_ALGO_CHUNKWISE_WIDE) halves the span of every factor.
 //
 // Warp specialisation (14 warps):
 //   EPI   (warps 0-7)   the epilogues of chunk r -- W, q_clean, mask of A, output --
@@ -79,6 +85,9 @@ constexpr int kPrepWarp0 = 8, kIssueWarp = 12, kCopyWarp = 13;
 constexpr int kThreadsNoCopy = 32 * kCopyWarp;       // 416
 constexpr int kThreadsCopy = 32 * (kCopyWarp + 1);    // 448
 constexpr int kSyncCount = kEpiThreads + 32;          // EPI + the issuing warp
+// largest exponent (log2 units) a gate factor may have: a state accumulated over a chunk
+// from keys scaled by up to 2^118 stays inside the fp32 range
+constexpr float kMaxExp2 = 118.f;
 
 // ---- shared memory map (bytes from the 1024-aligned base)
 // two slots of per-chunk tiles, each [64 rows][128 cols] bf16 as two T64 tiles of 8 KB:
@@ -519,6 +528,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const int tn = cb * kC + (wt >> 1);
             lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
         }
+        float emax = 0.f;  // largest |exponent| (log2 units) of a gate factor met
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
             const uint32_t sp = (r >> 1) & 1;
@@ -636,6 +646,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                         const uint32_t off = tcol + t64_offset(j, d0 & 63);
                         const uint64_t k2 = f2_mul(f2_from_bf16x2(kraw[u]), f2_make(rkv[u], rkv[u]));
                         const float2 x = f2_split(f2_fma(g2[jj], l2e, o2));
+                        emax = fmaxf(emax, fmaxf(fabsf(x.x), fabsf(x.y)));
                         *reinterpret_cast<uint32_t *>(slot + SO_K + off) = bf16x2_from_f2(k2);
                         *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
                             bf16x2_from_f2(f2_mul(k2, f2_make(fast_exp2(-x.x), fast_exp2(-x.y))));
@@ -652,6 +663,9 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             dmprev[wt] = dmp[wt] + dmp[kD + wt];
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
         }
+        // a factor beyond 2^kMaxExp2 cannot be represented: report it rather than return
+        // silently wrong values
+        if (emax > kMaxExp2) atomicExch(status, kStatusRange);
         // final key sum
         if (NC > 0 && a.mT && last_seg) {
             const int sl = (NC - 1) & 1;
@@ -824,6 +838,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 }  // namespace
 
 cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s) {
+    if (a.wide) return launch_gla_chunk_wide(a, m, s);
     static bool attr_set = false;
     if (!attr_set) {
         cudaError_t e = cudaFuncSetAttribute(gla_chunk_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -40,6 +40,8 @@ struct ChunkArgs {
     float scale;
     const float *lambda;
     const float *g, *beta;  // Gated DeltaNet scalar log-decay and beta
+    const void *gk = nullptr;  // GLA log-forget gate [B][T][H][128] (gate_dtype), read by the wide kernel's prep warps
+    int wide = 0;              // GLA: the two-reference kernel (ccq_gla_chunk_wide.cu)
     const float *S0, *C0, *m0;
     const int64_t *t0;
     __nv_bfloat16 *o;
@@ -86,6 +88,9 @@ struct ChunkMaps {
 };
 
 cudaError_t launch_gla_chunk(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
+// The two-reference CCQ-GLA forward (ccq_gla_chunk_wide.cu); launch_gla_chunk dispatches to it
+// when a.wide is set.
+cudaError_t launch_gla_chunk_wide(const ChunkArgs &a, const ChunkMaps &m, cudaStream_t s);
 
 // Segment-parallel CCQ-GLA (ccq_gla_segment.cu): state deltas per segment, an
 // exclusive combine, then gla_chunk_kernel on every (sequence, segment).

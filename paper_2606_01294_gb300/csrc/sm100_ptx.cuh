@@ -14,6 +14,9 @@ namespace ccq {
 // Status code a kernel writes to its status word when a bounded wait runs
 // out (read back and cleared by ccq_device_status()).
 constexpr int kStatusTimeout = 4;
+// Status code a kernel writes when its inputs leave the range it can represent
+// (CCQ_ERR_RANGE); the kernel runs to completion, its outputs are not valid.
+constexpr int kStatusRange = 5;
 // A bounded wait gives up after this many SM clock cycles (about one second).
 constexpr long long kWaitLimitCycles = 2000000000LL;
 

@@ -29,7 +29,7 @@ def test_default_params(lib):
 
 
 def test_status_strings(lib):
-    for s in range(5):
+    for s in range(6):
         assert lib.ccq_status_string(s)
     assert b"unknown" in lib.ccq_status_string(99)
 

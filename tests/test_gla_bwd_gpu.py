@@ -162,3 +162,17 @@ def test_bwd_full_size_sampled():
         gs = {n: (g[n][b:b + 1, :, h:h + 1] if g[n].dim() in (3, 4) and g[n].shape[1] == T
                   else g[n][b:b + 1, h:h + 1]) for n in NAMES}
         _compare(gs, ref, f"b={b} h={h}")
+
+
+@pytest.mark.parametrize("split", [1, 2])
+def test_bwd_from_wide_forward_checkpoints(split):
+    """Checkpoints written by the two-reference forward (algo "wide") carry the same tile
+    images as the default kernel's, so the backward reads either."""
+    P, G = _problem(1, 300, 2, seed=29)
+    d = lambda x: x.cuda().contiguous()  # noqa: E731
+    st = state_to_dev(G["state"])
+    o1, _ = ccq.gla_fwd(d(P["q"]), d(P["k"]), d(P["v"]), d(P["gate"]), d(P["lam"]), st, seq_split=split)
+    o2, _, ck = ccq.gla_fwd_save(d(P["q"]), d(P["k"]), d(P["v"]), d(P["gate"]), d(P["lam"]), st,
+                                 seq_split=split, algo="wide")
+    assert rel_err(o2, o1.double().cpu().numpy()) <= TOLB
+    _compare(_gpu(P, G, ckpt=ck, seq_split=split), _ref(P, G), f"wide checkpoints, split {split}")

@@ -1,10 +1,13 @@
-"""GPU parity under strong forgetting.  The chunk kernels factor every decay so that no
-intermediate leaves the fp32 / bf16 range: where a true factor underflows, its
-contribution is exactly zero, and no inf * 0 is formed.  These cases push the per-token
-log decay far beyond the workload's (GLA logsigmoid(N(0,1)) without the 1/16 and a
-constant -3 per key dimension; Gated DeltaNet -8 softplus(N(0,1)) and a constant -5), on
-the whole-sequence and the segment-parallel paths, and compare element by element with
-the oracle (Sec. 2.2, the backbone write rules)."""
+"""GPU parity under strong forgetting (Sec. 2.2, the backbone write rules), element by element
+against the oracle, on the whole-sequence and the segment-parallel paths.
+
+Gated DeltaNet: every decay factor of the chunk kernels is an exponential of a non-positive
+argument, so any decay is exact (where a factor underflows its contribution is exactly zero);
+cases: -8 softplus(N(0,1)) and a constant -5 per token.
+GLA (per key dimension gates): the factors are measured from reference tokens, one per chunk
+in the default kernel and one per half chunk in the "wide" kernel; cases inside both ranges
+(logsigmoid(N(0,1)) without the 1/16), inside only the wide kernel's (a constant -3 and -4.5,
+where the default kernel must report CCQ_ERR_RANGE), and beyond both (-6, reported)."""
 import numpy as np
 import pytest
 import torch
@@ -27,14 +30,42 @@ def _finite(o, fs):
         assert torch.isfinite(x.float()).all()
 
 
-@pytest.mark.parametrize("gates", ["strong", -3.0])
+@pytest.mark.parametrize("algo", ["chunkwise", "wide"])
 @pytest.mark.parametrize("split", [1, 2])
-def test_gla_strong_gates(gates, split):
+def test_gla_strong_gates(algo, split):
+    """logsigmoid(N(0,1)) per token and key dimension, without the 1/16: inside both kernels'
+    range."""
+    P = gen.make_inputs(GLA, 1, 300, 2, 128, 128, dtype=torch.bfloat16, seed=71, lam="trained",
+                        keys="structured", gates="strong")
+    o, fs = gpu_forward(GLA, P, algo=algo, seq_split=split)
+    _finite(o, fs)
+    compare(o, fs, oracle_forward(GLA, P), TOL[torch.bfloat16], f"GLA {algo} strong split={split}")
+
+
+@pytest.mark.parametrize("gates", [-3.0, -4.5])
+@pytest.mark.parametrize("split", [1, 2])
+def test_gla_wide_range(gates, split):
+    """A constant log gate of -3 or -4.5 per token and key dimension: beyond the midpoint
+    kernel's range (a 32-token half sums to -93 or worse), which reports CCQ_ERR_RANGE, and
+    inside the two-reference kernel's, which matches the oracle."""
     P = gen.make_inputs(GLA, 1, 300, 2, 128, 128, dtype=torch.bfloat16, seed=71, lam="trained",
                         keys="structured", gates=gates)
-    o, fs = gpu_forward(GLA, P, algo="chunkwise", seq_split=split)
+    gpu_forward(GLA, P, algo="chunkwise", seq_split=split)
+    with pytest.raises(ccq.CCQError) as ex:
+        ccq.device_status()
+    assert ex.value.status == ccq.CCQ_ERR_RANGE
+    o, fs = gpu_forward(GLA, P, algo="wide", seq_split=split)
     _finite(o, fs)
-    compare(o, fs, oracle_forward(GLA, P), TOL[torch.bfloat16], f"GLA gates={gates} split={split}")
+    compare(o, fs, oracle_forward(GLA, P), TOL[torch.bfloat16], f"GLA wide gates={gates} split={split}")
+
+
+def test_gla_beyond_wide_range_is_reported():
+    """-6 per token: a 16-token quarter sums to -96, beyond the two-reference kernel too."""
+    P = gen.make_inputs(GLA, 1, 130, 1, 128, 128, dtype=torch.bfloat16, seed=74, gates=-6.0)
+    gpu_forward(GLA, P, algo="wide")
+    with pytest.raises(ccq.CCQError) as ex:
+        ccq.device_status()
+    assert ex.value.status == ccq.CCQ_ERR_RANGE
 
 
 @pytest.mark.parametrize("gates", ["strong", -5.0])
