@@ -307,22 +307,24 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 
 // ============================================================================ main kernel
 //
-// Warp specialisation (13 warps), as in the GLA kernel:
+// Warp specialisation (14 warps), as in the GLA kernel:
 //   EPI   (warps 0-7)   the epilogues of chunk r -- W', R and U, q_clean, Pm,
 //                       output -- and the bf16 copies of S^K_{r+1} (while D4 runs) and
 //                       H_{r+1} (while G2 of chunk r+1 runs).  Warps w and w+4 share
 //                       TMEM lane quadrant w % 4 and split its columns.
 //   PREP  (warps 8-11)  prep of chunk r+1: row norms, cumulative decay, kbar, Kd.
-//   ISSUE (warp 12)     every tcgen05.mma and TMA copy, in the order
+//   COPY  (warp 13)     every per-chunk TMA copy and the L2 prefetch of chunk r + 2; the
+//                       output is staged in the slot's Kd tile, so R and U never wait on it.
+//   ISSUE (warp 12)     every tcgen05.mma, in the order
 //                       G2 D2 | G1 | DU G3 G8 | D4 D6 D3 | D5.  D2 (Kbar H0) lands in the
 //                       P/O accumulator, so EPI reads it out first and frees the accumulator
 //                       for G1 before it builds R; U = Tb R lands in TMEM columns 384-511
 //                       (Sc has been read, QK comes later).
-// R, then U, then the output staging share one 16 KB tile.
+// R, then U share one 16 KB tile; the output is staged in the Kd tile of the chunk's slot.
 
-constexpr int kThreads = 416;
+constexpr int kThreads = 448;
 constexpr int kEpiThreads = 256;
-constexpr int kPrepWarp0 = 8, kIssueWarp = 12;
+constexpr int kPrepWarp0 = 8, kIssueWarp = 12, kCopyWarp = 13;
 constexpr int kSyncCount = kEpiThreads + 32;
 constexpr uint32_t SLOT_BYTES = 49152;
 constexpr uint32_t SO_Q = 0;        // raw q, then q_clean
@@ -330,7 +332,7 @@ constexpr uint32_t SO_K = 16384;    // raw k, then kbar
 constexpr uint32_t SO_KD = 32768;   // kbar e^{gC - gc}
 constexpr uint32_t OFF_V = 98304;   // 16K  v of the chunk
 constexpr uint32_t OFF_TB = 114688; // 8K   Tb of the chunk (workspace), [64][64]
-constexpr uint32_t OFF_UB = 122880; // 16K  R, then U (bf16, rows j), after D5 the output staging
+constexpr uint32_t OFF_UB = 122880; // 16K  R, then U (bf16, rows j)
 constexpr uint32_t OFF_WM = 139264; // 8K   W' of the CCQ fold, then Pm
 constexpr uint32_t OFF_SK = 147456; // 32K  bf16 S^K
 constexpr uint32_t OFF_HB = 180224; // 32K  bf16 H0, the state entering the chunk
@@ -352,7 +354,8 @@ static_assert(MS_SCAL + 66 * 4 <= MS_MST, "scalar area overlaps");
 
 enum {
     BAR_IN0 = 0, BAR_IN1 = 1, BAR_WU = 2, BAR_GA1 = 3, BAR_GA2 = 4, BAR_GB = 5, BAR_GK = 6, BAR_GC = 7,
-    BAR_GC2 = 8, BAR_GD = 9, BAR_PREP0 = 10, BAR_PREP1 = 11, BAR_SNAPK = 12, BAR_SNAPS = 13, kNumBars = 14
+    BAR_GC2 = 8, BAR_GD = 9, BAR_PREP0 = 10, BAR_PREP1 = 11, BAR_SNAPK = 12, BAR_SNAPS = 13,
+    BAR_OST0 = 14, BAR_OST1 = 15, kNumBars = 16
 };
 static_assert(M_BAR + 8 * kNumBars <= M_TMEM, "barrier area");
 enum { NB_PO = 1, NB_W = 2, NB_QC = 3, NB_MASK = 4, NB_OUT = 5, NB_PREP = 6, NB_EPI = 7 };
@@ -420,6 +423,12 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tg, b);
         tma_load_4d(base + SO_K, &map_k, bb, 0, h, tg, b);
         tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tg, b);
+        if (r + 2 < NC) {  // chunk r + 2 into L2, so that its loads hit there
+            tma_prefetch_l2_4d(&map_q, 0, h, tg + 2 * kC, b);
+            tma_prefetch_l2_4d(&map_q, 64, h, tg + 2 * kC, b);
+            tma_prefetch_l2_4d(&map_k, 0, h, tg + 2 * kC, b);
+            tma_prefetch_l2_4d(&map_k, 64, h, tg + 2 * kC, b);
+        }
     };
     auto issue_wu = [&](int r) {  // v and Tb of chunk r
         uint64_t *bb = &bar[BAR_WU];
@@ -427,6 +436,14 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, (cb + r) * kC, b);
         tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, (cb + r) * kC, b);
         tma_load_2d(sm + OFF_TB, &map_tb, bb, 0, wrow0 + r * kC);
+        if (r + 2 < NC) {
+            tma_prefetch_l2_4d(&map_v, 0, h, (cb + r + 2) * kC, b);
+            tma_prefetch_l2_4d(&map_v, 64, h, (cb + r + 2) * kC, b);
+            asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                             reinterpret_cast<uint64_t>(&map_tb)),
+                         "r"(0), "r"(wrow0 + (r + 2) * kC)
+                         : "memory");
+        }
     };
 
     // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
@@ -460,7 +477,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const int wt = tid - 32 * kPrepWarp0;
         slot_f(0, MS_MST)[wt] = m0 ? m0[(segst ? 0 : static_cast<size_t>(bh) * kD) + wt] : 0.f;
         dmprev[wt] = 0.f;
-    } else if (lane == 0) {
+    } else if (warp == kIssueWarp && lane == 0) {
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_k);
         tma_prefetch_desc(&map_v);
@@ -674,14 +691,15 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar_arrive(NB_MASK, kSyncCount);
-            // ---- output o_i = scale (e^{gc_i} O1_i + O2_i), staged in the U tile for the TMA store.
+            // ---- output o_i = scale (e^{gc_i} O1_i + O2_i), staged for the copy warp's TMA store
+            // in the slot's Kd tile (its last reader, D6, completed before GD).
             // O1^T, O2^T are M = 128 accumulators: this thread holds value column `row` for the
             // chunk rows 32 grp .. 32 grp + 31.
             named_bar(NB_EPI, kEpiThreads);  // epo of this chunk visible
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             {
-                __nv_bfloat16 *ot = reinterpret_cast<__nv_bfloat16 *>(sm + OFF_UB + (row >> 6) * 8192);
+                __nv_bfloat16 *ot = reinterpret_cast<__nv_bfloat16 *>(slot + SO_KD + (row >> 6) * 8192);
 #pragma unroll 1
                 for (int hh = 0; hh < 2; ++hh) {
                     const int i0 = 32 * grp + 16 * hh;
@@ -826,7 +844,9 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 if (wt == 0) scal[1] = fast_exp2(gC * kLog2e);
             }
             named_bar(NB_PREP, 128);  // e^{gC - gc} visible
-            // kbar (in place) and Kd = kbar e^{gC - gc}: thread = (row, T64 tile)
+            // kbar (in place) and Kd = kbar e^{gC - gc}: thread = (row, T64 tile); the Kd tile
+            // held the output of chunk r - 2 until the copy warp's store read it
+            if (r >= 2) mbar_wait(&bar[BAR_OST0 + s], ((r >> 1) - 1) & 1, abort_flag, status);
             {
                 const int j = wt >> 1, hh = wt & 1;
                 const float rkj = slot_f(s, MS_RK)[j], enj = slot_f(s, MS_EN)[j];
@@ -875,7 +895,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const int sl = (NC - 1) & 1;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
-    } else {
+    } else if (warp == kIssueWarp) {
         // =============================================================== ISSUE
         const bool lead = lane == 0;
         const uint64_t dWm = make_desc(sb + OFF_WM, 16, 1024);
@@ -902,28 +922,13 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 mma_commit(&bar[BAR_GA1]);
             }
             __syncwarp();
-            if (r > 0) {
-                // O of chunk r-1 is staged in the U tile: store it
-                mbar_wait(&bar[BAR_GD], (r - 1) & 1, abort_flag, status);
-                named_bar(NB_OUT, kSyncCount);
-                if (lead) {
-                    tma_store_4d(&map_o, sm + OFF_UB, 0, h, (cb + r - 1) * kC, b);
-                    tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (cb + r - 1) * kC, b);
-                    tma_store_commit();
-                }
-                __syncwarp();
-            }
             // D2 KH = Kbar H0 (needs the H0 copy)
             mbar_wait(&bar[BAR_SNAPS], par, abort_flag, status);
             tc_fence_after();
             if (lead && !*abort_flag)
                 for (int k = 0; k < 8; ++k)
                     mma_bf16(tbase + TM_PO, dK + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
-            // the R/U tile is rewritten once GA2 lets EPI in: the output store must have read it
-            if (lead) {
-                tma_store_wait_read();
-                if (!*abort_flag) mma_commit(&bar[BAR_GA2]);
-            }
+            if (lead && !*abort_flag) mma_commit(&bar[BAR_GA2]);
             __syncwarp();
             // G1 P = Q S^K once WH is out of the accumulator
             named_bar(NB_PO, kSyncCount);
@@ -950,7 +955,6 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             named_bar(NB_QC, kSyncCount);
             tc_fence_after();
             if (lead && !*abort_flag) {
-                if (r + 1 < NC) issue_wu(r + 1);  // v and Tb of this chunk are consumed
                 for (int k = 0; k < 8; ++k) {
                     const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
                     mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
@@ -971,26 +975,44 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 mma_commit(&bar[BAR_GD]);
             }
             __syncwarp();
-            // the slot's last MMA reader (D3) is done: load chunk r + 2 into it
+        }
+    } else {
+        // =============================================================== COPY
+        // Every per-chunk copy, off the issuing thread (a copy can hold its thread while the
+        // copy engine is busy): v and Tb of chunk r + 1 once DU of chunk r has read them (GB);
+        // q and k of chunk r + 2 into the slot once D3 and D4 of chunk r have read it (GC2);
+        // the store of O (staged in the slot's Kd tile), whose read releases that tile to the
+        // prep of chunk r + 2 (OST).
+        const bool lead = lane == 0;
+        for (int r = 0; r < NC; ++r) {
+            const int s = r & 1;
+            if (r + 1 < NC) {
+                mbar_wait(&bar[BAR_GB], r & 1, abort_flag, status);
+                if (lead && !*abort_flag) issue_wu(r + 1);
+                __syncwarp();
+            }
             if (r + 2 < NC) {
-                mbar_wait(&bar[BAR_GC2], par, abort_flag, status);
+                mbar_wait(&bar[BAR_GC2], r & 1, abort_flag, status);
                 if (lead && !*abort_flag) issue_in(r + 2);
                 __syncwarp();
             }
-        }
-        if (NC > 0) {
-            mbar_wait(&bar[BAR_GD], (NC - 1) & 1, abort_flag, status);
-            named_bar(NB_OUT, kSyncCount);
+            named_bar(NB_OUT, kSyncCount);  // O of chunk r staged
             if (lead) {
-                tma_store_4d(&map_o, sm + OFF_UB, 0, h, (cb + NC - 1) * kC, b);
-                tma_store_4d(&map_o, sm + OFF_UB + 8192, 64, h, (cb + NC - 1) * kC, b);
+                uint8_t *st = sm + s * SLOT_BYTES + SO_KD;
+                tma_store_4d(&map_o, st, 0, h, (cb + r) * kC, b);
+                tma_store_4d(&map_o, st + 8192, 64, h, (cb + r) * kC, b);
                 tma_store_commit();
-                tma_store_wait_all();
-                if (*abort_flag) {
-                    // after a give-up, wait (bounded) for the copies still in flight
-                    mbar_drain(&bar[BAR_WU], (NC - 1) & 1);
-                    for (int r = (NC > 2 ? NC - 2 : 0); r < NC; ++r) mbar_drain(&bar[BAR_IN0 + (r & 1)], (r >> 1) & 1);
-                }
+                tma_store_wait_read();
+                mbar_arrive(&bar[BAR_OST0 + s]);
+            }
+            __syncwarp();
+        }
+        if (lead) {
+            tma_store_wait_all();
+            if (NC > 0 && *abort_flag) {
+                // after a give-up, wait (bounded) for the copies still in flight
+                mbar_drain(&bar[BAR_WU], (NC - 1) & 1);
+                for (int r = (NC > 2 ? NC - 2 : 0); r < NC; ++r) mbar_drain(&bar[BAR_IN0 + (r & 1)], (r >> 1) & 1);
             }
         }
     }
