@@ -7,6 +7,8 @@
 #include <stdarg.h>
 #include <stdint.h>
 #include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
 
 #include <algorithm>
 #include <initializer_list>
@@ -745,7 +747,9 @@ ccq_status ccq_gdn_fwd_decayed(const void *q, const void *k, const void *v, cons
 }
 
 // Packed variable-length sequences: validation shared by the call and its workspace query.
-static ccq_status check_varlen(int backbone, const int64_t *cu, int num_seqs, int H, long long *max_len) {
+// The per-sequence path offsets the fp32 [T][H] row pointers, which must stay 16-byte aligned.
+static ccq_status check_varlen(int backbone, const int64_t *cu, int num_seqs, int H, bool per_sequence,
+                               long long *max_len) {
     if (backbone != 0 && backbone != 1) return fail(CCQ_ERR_INVALID_ARG, "backbone must be 0 (GLA) or 1 (GDN)");
     if (!cu || num_seqs < 1) return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens is NULL or num_seqs < 1");
     if (cu[0] != 0) return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens[0] must be 0");
@@ -754,21 +758,57 @@ static ccq_status check_varlen(int backbone, const int64_t *cu, int num_seqs, in
         const long long len = cu[s + 1] - cu[s];
         if (len < 0) return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens decreases at %d", s);
         if (len > 0x7fffffffLL) return fail(CCQ_ERR_INVALID_ARG, "sequence %d is too long", s);
-        // per-token fp32 rows [T][H] start on 16-byte boundaries only if cu[s] * H is a multiple of 4
-        if ((cu[s] * H) % 4 != 0)
+        if (per_sequence && (cu[s] * H) % 4 != 0)
             return fail(CCQ_ERR_INVALID_ARG, "cu_seqlens[%d] * H must be a multiple of 4 (16-byte aligned rows)", s);
         mx = std::max(mx, len);
     }
+    if (cu[num_seqs] > 0x7fffffffLL) return fail(CCQ_ERR_INVALID_ARG, "packed length too large");
     *max_len = mx;
     return CCQ_OK;
+}
+
+// Whether a pack runs as one launch of the chunkwise kernels (bf16, Dk = Dv = 128, a chunkwise
+// algo whose kernel reads packed sequences, a non-empty pack); else one call per sequence.
+static bool varlen_single_launch(int backbone, ccq_dtype in_dtype, int Dk, int Dv, const ccq_params *p,
+                                 long long total) {
+    ccq_params c;
+    if (p) c = *p;
+    else ccq_default_params(&c);
+    const bool algo_ok = c.algo == CCQ_ALGO_AUTO || c.algo == CCQ_ALGO_CHUNKWISE ||
+                         (backbone == 1 && c.algo == CCQ_ALGO_CHUNKWISE_WIDE);
+    return in_dtype == CCQ_BF16 && Dk == 128 && Dv == 128 && algo_ok && total > 0;
+}
+
+// Workspace of the single launch: the device copy of cu_seqlens (int64), the first packed chunk
+// of every sequence (int32, num_seqs + 1) and the sequence of every packed chunk (int32), then
+// (Gated DeltaNet) the UT factor of every packed chunk of every head.
+struct VarlenLayout {
+    size_t cbase_off, cseq_off, meta_bytes, bytes;
+    int chunks;
+};
+
+static VarlenLayout varlen_layout(int backbone, const int64_t *cu, int num_seqs, int H) {
+    VarlenLayout L{};
+    long long nct = 0;
+    for (int s = 0; s < num_seqs; ++s) nct += (cu[s + 1] - cu[s] + 63) / 64;
+    L.chunks = static_cast<int>(nct);
+    L.cbase_off = (8 * static_cast<size_t>(num_seqs + 1) + 15) & ~static_cast<size_t>(15);
+    L.cseq_off = L.cbase_off + ((4 * static_cast<size_t>(num_seqs + 1) + 15) & ~static_cast<size_t>(15));
+    L.meta_bytes = (L.cseq_off + 4 * static_cast<size_t>(nct) + 255) & ~static_cast<size_t>(255);
+    L.bytes = L.meta_bytes + (backbone == 1 ? static_cast<size_t>(nct) * H * 64 * 64 * 2 : 0);
+    return L;
 }
 
 ccq_status ccq_fwd_varlen_workspace_size(int backbone, const int64_t *cu_seqlens, int num_seqs, int H, int Dk,
                                          int Dv, ccq_dtype in_dtype, const ccq_params *p, size_t *bytes) {
     long long mx = 0;
-    ccq_status st = check_varlen(backbone, cu_seqlens, num_seqs, H, &mx);
+    ccq_status st = check_varlen(backbone, cu_seqlens, num_seqs, H, false, &mx);
     if (st != CCQ_OK) return st;
     if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
+    if (varlen_single_launch(backbone, in_dtype, Dk, Dv, p, cu_seqlens[num_seqs])) {
+        *bytes = varlen_layout(backbone, cu_seqlens, num_seqs, H).bytes;
+        return CCQ_OK;
+    }
     size_t need = 0;
     for (int s = 0; s < num_seqs; ++s) {
         const int len = static_cast<int>(cu_seqlens[s + 1] - cu_seqlens[s]);
@@ -782,6 +822,82 @@ ccq_status ccq_fwd_varlen_workspace_size(int backbone, const int64_t *cu_seqlens
     return CCQ_OK;
 }
 
+// One launch over the whole pack (chunkwise kernels with packed-sequence indexing).
+static ccq_status varlen_launch(int backbone, const void *q, const void *k, const void *v, const void *gate,
+                                const float *beta, const float *lambda, ccq_dtype gate_dtype, const int64_t *cu,
+                                int ns, const float *S0, const float *C0, const float *m0, const int64_t *t0,
+                                void *o, float *ST, float *CT, float *mT, int64_t *tT, int H, void *workspace,
+                                size_t workspace_bytes, const ccq_params *p, cudaStream_t s) {
+    Common c;
+    const int total = static_cast<int>(cu[ns]);
+    ccq_status st = check_common(p, ns, total, H, 128, 128, &c);
+    if (st != CCQ_OK) return st;
+    if (backbone == 1) st = check_ptrs("q,k,v,g,beta,lambda,o", {q, k, v, gate, beta, lambda, o}, {S0, C0, m0, ST, CT, mT});
+    else st = check_ptrs("q,k,v,gk,lambda,o", {q, k, v, gate, lambda, o}, {S0, C0, m0, ST, CT, mT});
+    if (st == CCQ_OK) st = check_counts({t0, tT});
+    if (st != CCQ_OK) return st;
+    const VarlenLayout L = varlen_layout(backbone, cu, ns, H);
+    if (!workspace || workspace_bytes < L.bytes)
+        return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", L.bytes,
+                    workspace ? workspace_bytes : static_cast<size_t>(0));
+    if (!aligned16(workspace)) return fail(CCQ_ERR_INVALID_ARG, "workspace is not 16-byte aligned");
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    ChunkArgs a = {};
+    ChunkMaps gm;
+    GdnMaps dm;
+    const int geb = gate_dtype == CCQ_BF16 ? 2 : 4;
+    bool ok = make_token_map(&gm.q, q, 2, 1, total, H, 128, 64, true) &&
+              make_token_map(&gm.k, k, 2, 1, total, H, 128, 64, true) &&
+              make_token_map(&gm.v, v, 2, 1, total, H, 128, 64, true) &&
+              make_token_map(&gm.o, o, 2, 1, total, H, 128, 64, true);
+    if (ok && backbone == 0) ok = make_token_map(&gm.g, gate, geb, 1, total, H, 128, 128, false);
+    if (ok && backbone == 1) {
+        dm.q = gm.q; dm.k = gm.k; dm.v = gm.v; dm.o = gm.o;
+        ok = make_rows_map(&dm.tb, ws + L.meta_bytes, static_cast<long long>(L.chunks) * H * 64, 64);
+    }
+    if (!ok) return fail(CCQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (driver entry point missing or map rejected)");
+    a.status = device_status_word();
+    if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
+    // the pack's offsets, chunk bases and chunk -> sequence map, staged on the host and copied in
+    // one transfer (from pageable memory: the copy is staged before this call returns)
+    {
+        uint8_t *meta = static_cast<uint8_t *>(malloc(L.meta_bytes));
+        if (!meta) return fail(CCQ_ERR_INVALID_ARG, "out of host memory for %zu bytes", L.meta_bytes);
+        memcpy(meta, cu, 8 * static_cast<size_t>(ns + 1));
+        int *cbase = reinterpret_cast<int *>(meta + L.cbase_off);
+        int *cseq = reinterpret_cast<int *>(meta + L.cseq_off);
+        int acc = 0;
+        for (int sq = 0; sq < ns; ++sq) {
+            cbase[sq] = acc;
+            const int nc = static_cast<int>((cu[sq + 1] - cu[sq] + 63) / 64);
+            for (int r = 0; r < nc; ++r) cseq[acc + r] = sq;
+            acc += nc;
+        }
+        cbase[ns] = acc;
+        cudaError_t e = cudaMemcpyAsync(ws, meta, L.meta_bytes, cudaMemcpyHostToDevice, s);
+        free(meta);
+        if (e != cudaSuccess) return cuda_fail(e, "packed-sequence offsets copy");
+    }
+    a.B = ns; a.T = total; a.H = H;
+    a.gate_dtype = gate_dtype == CCQ_BF16 ? 0 : 1;
+    a.l2norm = c.p.l2norm_qk; a.centered = c.p.centered; a.scale = c.scale;
+    a.lambda = lambda; a.gk = gate;
+    a.g = static_cast<const float *>(gate); a.beta = beta;
+    a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
+    a.o = static_cast<__nv_bfloat16 *>(o);
+    a.ST = ST; a.CT = CT; a.mT = mT;
+    a.nseg = 1;
+    a.cu = reinterpret_cast<const int64_t *>(ws);
+    a.cbase = reinterpret_cast<const int *>(ws + L.cbase_off);
+    a.chunk_seq = reinterpret_cast<const int *>(ws + L.cseq_off);
+    a.vl_chunks = L.chunks;
+    cudaError_t e = backbone == 0 ? launch_gla_chunk(a, gm, s) : launch_gdn_chunk(a, dm, s);
+    if (e != cudaSuccess) return cuda_fail(e, "packed-sequence chunkwise launch");
+    e = launch_t_update_varlen(t0, tT, a.cu, ns, s);
+    if (e != cudaSuccess) return cuda_fail(e, "position update launch");
+    return CCQ_OK;
+}
+
 ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void *v, const void *gate,
                           const float *beta, const float *lambda, ccq_dtype in_dtype, ccq_dtype gate_dtype,
                           const int64_t *cu_seqlens, int num_seqs, const float *S0, const float *C0,
@@ -789,10 +905,17 @@ ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void
                           int64_t *tT, int H, int Dk, int Dv, void *workspace, size_t workspace_bytes,
                           const ccq_params *p, void *stream) {
     long long mx = 0;
-    ccq_status st = check_varlen(backbone, cu_seqlens, num_seqs, H, &mx);
+    ccq_status st = check_varlen(backbone, cu_seqlens, num_seqs, H, false, &mx);
     if (st != CCQ_OK) return st;
     if ((in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) || (gate_dtype != CCQ_BF16 && gate_dtype != CCQ_FP32))
         return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
+    if (backbone == 1 && gate_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "Gated DeltaNet decay must be fp32");
+    if (varlen_single_launch(backbone, in_dtype, Dk, Dv, p, cu_seqlens[num_seqs]))
+        return varlen_launch(backbone, q, k, v, gate, beta, lambda, gate_dtype, cu_seqlens, num_seqs, S0, C0, m0,
+                             t0, o, ST, CT, mT, tT, H, workspace, workspace_bytes, p,
+                             static_cast<cudaStream_t>(stream));
+    st = check_varlen(backbone, cu_seqlens, num_seqs, H, true, &mx);
+    if (st != CCQ_OK) return st;
     size_t need = 0;
     st = ccq_fwd_varlen_workspace_size(backbone, cu_seqlens, num_seqs, H, Dk, Dv, in_dtype, p, &need);
     if (st != CCQ_OK) return st;
@@ -806,8 +929,8 @@ ccq_status ccq_fwd_varlen(int backbone, const void *q, const void *k, const void
     else ccq_default_params(&pin);
     ccq_params pempty = pin;  // an empty sequence passes its state through on any path
     pempty.algo = CCQ_ALGO_AUTO;
-    // One call of the (batch-1) forward per sequence, in stream order: the calls share the
-    // workspace, and sequence s reads and writes row s of every state.  Pass 0 checks every
+    // Otherwise one call of the (batch-1) forward per sequence, in stream order: the calls share
+    // the workspace, and sequence s reads and writes row s of every state.  Pass 0 checks every
     // call's arguments, pass 1 launches, so that a rejected pack enqueues nothing.
     for (int pass = 0; pass < 2; ++pass)
     for (int s = 0; s < num_seqs; ++s) {

@@ -87,8 +87,27 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int item = blockIdx.x;
-    const int r = item % NC, bh = item / NC, b = bh / a.H, h = bh % a.H;
-    const int T = a.T, H = a.H;
+    const int H = a.H;
+    // packed sequences: item = (packed chunk) * H + head; otherwise item = (b H + h) NC + r
+    const bool vl = a.cu != nullptr;
+    int b, h, r, nc_b;
+    if (vl) {
+        const int gci = item / H;
+        h = item % H;
+        b = a.chunk_seq[gci];
+        r = gci - a.cbase[b];
+        nc_b = a.cbase[b + 1] - a.cbase[b];
+    } else {
+        r = item % NC;
+        b = item / NC / H;
+        h = item / NC % H;
+        nc_b = NC;
+    }
+    const int tok0 = vl ? static_cast<int>(a.cu[b]) : 0;
+    const int T = vl ? static_cast<int>(a.cu[b + 1] - a.cu[b]) : a.T;
+    const int bt = vl ? 0 : b;
+    const size_t rowbase = vl ? static_cast<size_t>(tok0) : static_cast<size_t>(b) * a.T;
+    const int tbrow = ((vl ? a.cbase[b] : b * NC) * H + h * nc_b + r) * kC;  // first Tb row of the chunk
     const int c0 = r * kC;
     int *status = a.status;
 
@@ -97,13 +116,15 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         *abort_flag = 0;
         fence_barrier_init();
         mbar_arrive_expect_tx(&bar[0], 2 * 8192);
-        tma_load_4d(sm + WY_K, &map_k, &bar[0], 0, h, c0, b);
-        tma_load_4d(sm + WY_K + 8192, &map_k, &bar[0], 64, h, c0, b);
+        tma_load_4d(sm + WY_K, &map_k, &bar[0], 0, h, tok0 + c0, bt);
+        tma_load_4d(sm + WY_K + 8192, &map_k, &bar[0], 64, h, tok0 + c0, bt);
     }
     if (warp == 0) tmem_alloc(tslot, 64);
     if (tid < 64) {
+        // past the end of a packed sequence: beta = 0 and no decay, so the rows of the next
+        // sequence's keys in the tile add nothing
         const int t = c0 + tid;
-        const size_t row = (static_cast<size_t>(b) * T + t) * H + h;
+        const size_t row = (rowbase + t) * H + h;
         gcs[tid] = t < T ? a.g[row] : 0.f;
         bet[tid] = t < T ? a.beta[row] : 0.f;
     }
@@ -291,7 +312,7 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         asm volatile(
             "cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
                 reinterpret_cast<uint64_t>(&map_tb)),
-            "r"(smem_addr(sm + WY_A)), "r"(0), "r"(item * kC)
+            "r"(smem_addr(sm + WY_A)), "r"(0), "r"(tbrow)
             : "memory");
         tma_store_commit();
         tma_store_wait_read();  // shared memory must outlive the store's read
@@ -388,7 +409,13 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int bh = blockIdx.x / a.nseg, seg = blockIdx.x % a.nseg, b = bh / a.H, h = bh % a.H;
-    const int T = a.T, H = a.H;
+    const int H = a.H;
+    // packed sequences: sequence b is rows tok0 .. tok0 + T of a [1][a.T][H][D] tensor
+    const bool vl = a.cu != nullptr;
+    const int tok0 = vl ? static_cast<int>(a.cu[b]) : 0;
+    const int T = vl ? static_cast<int>(a.cu[b + 1] - a.cu[b]) : a.T;
+    const int bt = vl ? 0 : b;
+    const size_t rowbase = vl ? static_cast<size_t>(tok0) : static_cast<size_t>(b) * a.T;
     const int NCt = (T + kC - 1) / kC;
     const int cb = a.nseg > 1 ? seg * a.seg_chunks : 0;  // first chunk of this CTA
     const int NC = a.nseg > 1 ? min(NCt, cb + a.seg_chunks) - cb : NCt;
@@ -400,7 +427,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     const float *m0 = segst ? segst + 3 * kD * kD : a.m0;
     const int64_t t0 = (a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(cb) * kC;  // position before the CTA's first token
     int *status = a.status;
-    const int wrow0 = (bh * NCt + cb) * kC;  // first workspace row of this CTA's chunks
+    const int wrow0 = ((vl ? a.cbase[b] * H + h * NCt : bh * NCt) + cb) * kC;  // first Tb row of this CTA's chunks
 
     if (tid == 0) {
         for (int i = 0; i < kNumBars; ++i) mbar_init(&bar[i], 1);
@@ -419,32 +446,36 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         uint64_t *bb = &bar[BAR_IN0 + s];
         mbar_arrive_expect_tx(bb, 4 * 8192);
         const int tg = (cb + r) * kC;
-        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tg, b);
-        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tg, b);
-        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tg, b);
-        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tg, b);
+        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tok0 + tg, bt);
         if (r + 2 < NC) {  // chunk r + 2 into L2, so that its loads hit there
-            tma_prefetch_l2_4d(&map_q, 0, h, tg + 2 * kC, b);
-            tma_prefetch_l2_4d(&map_q, 64, h, tg + 2 * kC, b);
-            tma_prefetch_l2_4d(&map_k, 0, h, tg + 2 * kC, b);
-            tma_prefetch_l2_4d(&map_k, 64, h, tg + 2 * kC, b);
+            tma_prefetch_l2_4d(&map_q, 0, h, tok0 + tg + 2 * kC, bt);
+            tma_prefetch_l2_4d(&map_q, 64, h, tok0 + tg + 2 * kC, bt);
+            tma_prefetch_l2_4d(&map_k, 0, h, tok0 + tg + 2 * kC, bt);
+            tma_prefetch_l2_4d(&map_k, 64, h, tok0 + tg + 2 * kC, bt);
         }
     };
     auto issue_wu = [&](int r) {  // v and Tb of chunk r
         uint64_t *bb = &bar[BAR_WU];
         mbar_arrive_expect_tx(bb, 3 * 8192);
-        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, (cb + r) * kC, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, (cb + r) * kC, b);
+        tma_load_4d(sm + OFF_V, &map_v, bb, 0, h, tok0 + (cb + r) * kC, bt);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, bb, 64, h, tok0 + (cb + r) * kC, bt);
         tma_load_2d(sm + OFF_TB, &map_tb, bb, 0, wrow0 + r * kC);
         if (r + 2 < NC) {
-            tma_prefetch_l2_4d(&map_v, 0, h, (cb + r + 2) * kC, b);
-            tma_prefetch_l2_4d(&map_v, 64, h, (cb + r + 2) * kC, b);
+            tma_prefetch_l2_4d(&map_v, 0, h, tok0 + (cb + r + 2) * kC, bt);
+            tma_prefetch_l2_4d(&map_v, 64, h, tok0 + (cb + r + 2) * kC, bt);
             asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
                              reinterpret_cast<uint64_t>(&map_tb)),
                          "r"(0), "r"(wrow0 + (r + 2) * kC)
                          : "memory");
         }
     };
+
+    // the last chunk of a packed sequence ends inside the tile: its rows past the end belong to
+    // the next sequence, so its output is written row by row (not by a TMA store of the tile)
+    auto partial = [&](int r) { return vl && T - (cb + r) * kC < kC; };
 
     // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
     if (warp < kPrepWarp0) {
@@ -700,6 +731,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tc_fence_after();
             {
                 __nv_bfloat16 *ot = reinterpret_cast<__nv_bfloat16 *>(slot + SO_KD + (row >> 6) * 8192);
+                const bool direct = partial(r);
 #pragma unroll 1
                 for (int hh = 0; hh < 2; ++hh) {
                     const int i0 = 32 * grp + 16 * hh;
@@ -714,8 +746,10 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 #pragma unroll
                         for (int u = 0; u < 4; ++u) {
                             const int e = 4 * q + u;
-                            ot[t64_offset(i0 + e, row & 63) >> 1] =
-                                __float2bfloat16_rn(a.scale * fmaf(ev4[u], o1[e], o2[e]));
+                            const __nv_bfloat16 ov = __float2bfloat16_rn(a.scale * fmaf(ev4[u], o1[e], o2[e]));
+                            const int tpos = (cb + r) * kC + i0 + e;  // position in the sequence
+                            if (!direct) ot[t64_offset(i0 + e, row & 63) >> 1] = ov;
+                            else if (tpos < T) a.o[((rowbase + tpos) * H + h) * kD + row] = ov;
                         }
                     }
                 }
@@ -730,7 +764,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
         }
         // final states: H_T (the TMEM state after the last chunk), S^K
-        if (NC > 0 && last_seg) {
+        if ((NC > 0 || vl) && last_seg) {  // (an empty packed sequence: the initial states)
             tc_fence_after();
             const size_t bhs = static_cast<size_t>(bh);
 #pragma unroll
@@ -758,8 +792,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         float lam_reg, g_reg;
         {
             const int tn = cb * kC + (wt >> 1), tg = cb * kC + wt;
-            lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
-            g_reg = (wt < 64 && tg < T) ? a.g[(static_cast<size_t>(b) * T + tg) * H + h] : 0.f;
+            lam_reg = (tn < T) ? a.lambda[(rowbase + tn) * H + h] : 0.f;
+            g_reg = (wt < 64 && tg < T) ? a.g[(rowbase + tg) * H + h] : 0.f;
         }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
@@ -773,9 +807,9 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (wt < 64) scal[2 + wt] = g_reg;
             {
                 const int tn = (cb + r + 1) * kC + (wt >> 1);
-                lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+                lam_reg = (tn < T) ? a.lambda[(rowbase + tn) * H + h] : 0.f;
                 const int tg = (cb + r + 1) * kC + wt;
-                g_reg = (wt < 64 && tg < T) ? a.g[(static_cast<size_t>(b) * T + tg) * H + h] : 0.f;
+                g_reg = (wt < 64 && tg < T) ? a.g[(rowbase + tg) * H + h] : 0.f;
             }
             named_bar(NB_PREP, 128);  // key sum and raw decays visible
             // in-chunk cumulative log decay gc: one warp, a shuffle scan over two tokens a lane
@@ -833,7 +867,9 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(ssq, 1e-12f) * rq : 1.f;
                     slot_f(s, MS_LT)[j] = lam_cur * iti;
                 } else {
-                    slot_f(s, MS_RK)[j] = a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
+                    // rows past the end of a packed sequence hold the next one's keys: zero them
+                    const bool in_seq = (cb + r) * kC + j < T;
+                    slot_f(s, MS_RK)[j] = !in_seq ? 0.f : a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
                 }
             }
             named_bar(NB_PREP, 128);  // gc, rk visible
@@ -891,8 +927,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             dmprev[wt] = dmp[wt] + dmp[kD + wt];
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
         }
-        if (NC > 0 && a.mT && last_seg) {
-            const int sl = (NC - 1) & 1;
+        if ((NC > 0 || vl) && a.mT && last_seg) {
+            const int sl = NC > 0 ? (NC - 1) & 1 : 0;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
     } else if (warp == kIssueWarp) {
@@ -999,9 +1035,11 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             named_bar(NB_OUT, kSyncCount);  // O of chunk r staged
             if (lead) {
                 uint8_t *st = sm + s * SLOT_BYTES + SO_KD;
-                tma_store_4d(&map_o, st, 0, h, (cb + r) * kC, b);
-                tma_store_4d(&map_o, st + 8192, 64, h, (cb + r) * kC, b);
-                tma_store_commit();
+                if (!partial(r)) {
+                    tma_store_4d(&map_o, st, 0, h, tok0 + (cb + r) * kC, bt);
+                    tma_store_4d(&map_o, st + 8192, 64, h, tok0 + (cb + r) * kC, bt);
+                    tma_store_commit();
+                }
                 tma_store_wait_read();
                 mbar_arrive(&bar[BAR_OST0 + s]);
             }
@@ -1036,7 +1074,9 @@ cudaError_t launch_gdn_wy(const ChunkArgs &a, const GdnMaps &m, cudaStream_t s) 
         attr_set = true;
     }
     const int NC = (a.T + kC - 1) / kC;
-    gdn_wy_kernel<<<a.B * a.H * NC, 128, WY_SMEM, s>>>(m.k, m.tb, a, NC);
+    const int items = a.cu ? a.vl_chunks * a.H : a.B * a.H * NC;
+    if (items == 0) return cudaSuccess;
+    gdn_wy_kernel<<<items, 128, WY_SMEM, s>>>(m.k, m.tb, a, NC);
     return cudaGetLastError();
 }
 

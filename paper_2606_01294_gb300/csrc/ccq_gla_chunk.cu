@@ -176,7 +176,13 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int bh = blockIdx.x / a.nseg, seg = blockIdx.x % a.nseg, b = bh / a.H, h = bh % a.H;
-    const int T = a.T, H = a.H;
+    const int H = a.H;
+    // packed sequences: sequence b is rows tok0 .. tok0 + T of a [1][a.T][H][D] tensor
+    const bool vl = a.cu != nullptr;
+    const int tok0 = vl ? static_cast<int>(a.cu[b]) : 0;                  // token coordinate offset
+    const int T = vl ? static_cast<int>(a.cu[b + 1] - a.cu[b]) : a.T;     // this sequence's length
+    const int bt = vl ? 0 : b;                                            // batch coordinate
+    const size_t rowbase = vl ? static_cast<size_t>(tok0) : static_cast<size_t>(b) * a.T;  // its first [., H] row
     const int NCt = (T + kC - 1) / kC;
     const int cb = a.nseg > 1 ? seg * a.seg_chunks : 0;  // first chunk of this CTA
     const int NC = a.nseg > 1 ? min(NCt, cb + a.seg_chunks) - cb : NCt;
@@ -206,29 +212,39 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         uint8_t *base = sm + s * SLOT_BYTES;
         uint64_t *bb = &bar[BAR_IN0 + s];
         mbar_arrive_expect_tx(bb, 4 * 8192 + g_bytes);
-        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tg, b);
-        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tg, b);
-        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tg, b);
-        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tg, b);
-        tma_load_4d(base + SO_KG, &map_g, bb, 0, h, tg, b);
+        tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tok0 + tg, bt);
+        tma_load_4d(base + SO_KG, &map_g, bb, 0, h, tok0 + tg, bt);
         if (COPY && r + 2 < NC) {  // chunk r + 2 into L2, so that its loads hit there
-            const int tp = tg + 2 * kC;
-            tma_prefetch_l2_4d(&map_q, 0, h, tp, b);
-            tma_prefetch_l2_4d(&map_q, 64, h, tp, b);
-            tma_prefetch_l2_4d(&map_k, 0, h, tp, b);
-            tma_prefetch_l2_4d(&map_k, 64, h, tp, b);
-            tma_prefetch_l2_4d(&map_g, 0, h, tp, b);
+            const int tp = tok0 + tg + 2 * kC;
+            tma_prefetch_l2_4d(&map_q, 0, h, tp, bt);
+            tma_prefetch_l2_4d(&map_q, 64, h, tp, bt);
+            tma_prefetch_l2_4d(&map_k, 0, h, tp, bt);
+            tma_prefetch_l2_4d(&map_k, 64, h, tp, bt);
+            tma_prefetch_l2_4d(&map_g, 0, h, tp, bt);
         }
     };
     auto issue_v = [&](int r) {
         const int tg = (cb + r) * kC;
         mbar_arrive_expect_tx(&bar[BAR_V], 2 * 8192);
-        tma_load_4d(sm + OFF_V, &map_v, &bar[BAR_V], 0, h, tg, b);
-        tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, tg, b);
+        tma_load_4d(sm + OFF_V, &map_v, &bar[BAR_V], 0, h, tok0 + tg, bt);
+        tma_load_4d(sm + OFF_V + 8192, &map_v, &bar[BAR_V], 64, h, tok0 + tg, bt);
         if (COPY && r + 2 < NC) {
-            tma_prefetch_l2_4d(&map_v, 0, h, tg + 2 * kC, b);
-            tma_prefetch_l2_4d(&map_v, 64, h, tg + 2 * kC, b);
+            tma_prefetch_l2_4d(&map_v, 0, h, tok0 + tg + 2 * kC, bt);
+            tma_prefetch_l2_4d(&map_v, 64, h, tok0 + tg + 2 * kC, bt);
         }
+    };
+    // the last chunk of a packed sequence ends inside the tile: its rows past the end belong to
+    // the next sequence, so its output is written row by row (not by a TMA store of the tile)
+    auto partial = [&](int r) { return vl && T - (cb + r) * kC < kC; };
+    auto store_o = [&](int r) {  // TMA store of the output of local chunk r staged in the v tile
+        if (a.skip_o || partial(r)) return;
+        const int cp = (cb + r) * kC;
+        tma_store_4d(&map_o, sm + OFF_V, 0, h, tok0 + cp, bt);
+        tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, tok0 + cp, bt);
+        tma_store_commit();
     };
 
     // ---- set-up: initial states into TMEM (EPI), key sum (PREP), first loads (ISSUE)
@@ -465,13 +481,19 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 float x[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
                 const uint64_t sc2 = f2_make(a.scale, a.scale);
+                const int tpos = (cb + r) * kC + i;  // position of row i in the sequence
+                const bool direct = partial(r);
+                uint4 *dst = reinterpret_cast<uint4 *>(a.o + ((rowbase + tpos) * H + h) * kD + 64 * grp + 32 * hf);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     uint32_t w[4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
                         w[u] = bf16x2_from_f2(f2_mul(f2_make(x[8 * q4 + 2 * u], x[8 * q4 + 2 * u + 1]), sc2));
-                    *reinterpret_cast<uint4 *>(sm + OFF_V + grp * 8192 + t64_chunk(i, 4 * hf + q4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                    if (!direct)
+                        *reinterpret_cast<uint4 *>(sm + OFF_V + grp * 8192 + t64_chunk(i, 4 * hf + q4)) = make_uint4(w[0], w[1], w[2], w[3]);
+                    else if (tpos < T)
+                        dst[q4] = make_uint4(w[0], w[1], w[2], w[3]);
                 }
                 fence_proxy_async_smem();
             }
@@ -485,8 +507,9 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
         }
         if (ck_head && tid == 0) tma_store_wait_all();
-        // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K
-        if (NC > 0 && last_seg) {
+        // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K (an empty packed sequence:
+        // the initial states, still in TMEM as set up)
+        if ((NC > 0 || vl) && last_seg) {
             tc_fence_after();
             const float fs = f_cur;
             const size_t bhs = static_cast<size_t>(bh);
@@ -526,7 +549,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         float lam_reg = 0.f;  // lambda of row wt >> 1
         {
             const int tn = cb * kC + (wt >> 1);
-            lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+            lam_reg = (tn < T) ? a.lambda[(rowbase + tn) * H + h] : 0.f;
         }
         float emax = 0.f;  // largest |exponent| (log2 units) of a gate factor met
         for (int r = 0; r < NC; ++r) {
@@ -540,7 +563,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const float lam_cur = lam_reg;
             {
                 const int tn = (cb + r + 1) * kC + (wt >> 1);
-                lam_reg = (tn < T) ? a.lambda[(static_cast<size_t>(b) * T + tn) * H + h] : 0.f;
+                lam_reg = (tn < T) ? a.lambda[(rowbase + tn) * H + h] : 0.f;
             }
             named_bar(NB_PREP, 128);
             // row norms of q and k and M . q: thread pair (2j, 2j+1) takes row j, each
@@ -587,19 +610,23 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(ssq, 1e-12f) * rq : 1.f;
                     slot_f(s, MS_LT)[j] = lam_cur * iti;
                 } else {
-                    slot_f(s, MS_RK)[j] = a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
+                    // rows past the end of a packed sequence hold the next one's keys: zero them
+                    const bool in_seq = (cb + r) * kC + j < T;
+                    slot_f(s, MS_RK)[j] = !in_seq ? 0.f : a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
                 }
             }
             // gate cumsum over this thread's 32 tokens for dims d0, d0+1, as fp32 pairs
             uint64_t g2[32];
             {
                 uint64_t r2 = 0;  // (0.f, 0.f)
+                const int rem = T - (cb + r) * kC;  // tokens of the sequence in this chunk
 #pragma unroll
                 for (int jj = 0; jj < 32; ++jj) {
                     const int j = 32 * th + jj;
                     const uint64_t x2 =
-                        gate_f32 ? *reinterpret_cast<const uint64_t *>(slot + SO_KG + (j * kD + d0) * 4)
-                                 : f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(slot + SO_KG + (j * kD + d0) * 2));
+                        j >= rem ? 0
+                        : gate_f32 ? *reinterpret_cast<const uint64_t *>(slot + SO_KG + (j * kD + d0) * 4)
+                                   : f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(slot + SO_KG + (j * kD + d0) * 2));
                     r2 = f2_add(r2, x2);
                     g2[jj] = r2;
                 }
@@ -667,8 +694,8 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         // silently wrong values
         if (emax > kMaxExp2) atomicExch(status, kStatusRange);
         // final key sum
-        if (NC > 0 && a.mT && last_seg) {
-            const int sl = (NC - 1) & 1;
+        if ((NC > 0 || vl) && a.mT && last_seg) {
+            const int sl = NC > 0 ? (NC - 1) & 1 : 0;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
     } else if (warp == kIssueWarp) {
@@ -704,12 +731,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 // warp does)
                 mbar_wait(&bar[BAR_GD], (r - 1) & 1, abort_flag, status);
                 named_bar(NB_OUT, kOutCount);
-                if (lead && !COPY && !a.skip_o) {
-                    const int cp = (cb + r - 1) * kC;
-                    tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
-                    tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
-                    tma_store_commit();
-                }
+                if (lead && !COPY) store_o(r - 1);
                 __syncwarp();
             }
             // G1 P = Q S^K
@@ -779,12 +801,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         if (NC > 0) {
             mbar_wait(&bar[BAR_GD], (NC - 1) & 1, abort_flag, status);
             named_bar(NB_OUT, kOutCount);
-            if (lead && !COPY && !a.skip_o) {
-                const int cp = (cb + NC - 1) * kC;
-                tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
-                tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
-                tma_store_commit();
-            }
+            if (lead && !COPY) store_o(NC - 1);
             if (lead) tma_store_wait_all();
             // after a give-up, wait (bounded) for the copies still in flight
             if (lead && *abort_flag) {
@@ -807,12 +824,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
             named_bar(NB_OUT, kOutCount);  // O of chunk r staged in the v tile
             if (lead && COPY) {
-                if (!a.skip_o) {
-                    const int cp = (cb + r) * kC;
-                    tma_store_4d(&map_o, sm + OFF_V, 0, h, cp, b);
-                    tma_store_4d(&map_o, sm + OFF_V + 8192, 64, h, cp, b);
-                    tma_store_commit();
-                }
+                store_o(r);
                 if (r + 1 < NC) {
                     tma_store_wait_read();
                     if (!*abort_flag) issue_v(r + 1);

@@ -30,6 +30,9 @@ cudaError_t launch_recurrent(const RecurrentArgs &a, cudaStream_t s);
 // the final count to this launch, enqueued after them: tT may alias t0, and
 // every (batch, head) CTA reads t0[b] while it runs.
 cudaError_t launch_t_update(const int64_t *t0, int64_t *tT, int B, int T, cudaStream_t s);
+// tT[s] = t0[s] + (cu[s+1] - cu[s]) (t0 NULL: 0 +) for packed sequences (device cu).
+cudaError_t launch_t_update_varlen(const int64_t *t0, int64_t *tT, const int64_t *cu, int num_seqs,
+                                   cudaStream_t s);
 
 // Arguments of the chunkwise tensor-core kernels (Dk = Dv = 128, chunk 64,
 // bf16 q/k/v/o).
@@ -57,6 +60,17 @@ struct ChunkArgs {
     // backward (layout below); skip_o suppresses the output write.
     uint8_t *ckpt = nullptr;
     int skip_o = 0;
+    // Packed variable-length sequences (cu != NULL): the batch index b is the sequence, B the
+    // number of sequences, T the packed length; rows cu[b] .. cu[b+1] of the [1][T][H][D]
+    // token tensors (and of lambda, the gates, beta) are sequence b, its states are row b.
+    // Gated DeltaNet: cbase[b] is the first chunk of sequence b in the packed chunk order
+    // (cbase[B] the total), chunk_seq[c] the sequence of packed chunk c; the UT factor of
+    // chunk r of (b, h) is at rows (cbase[b] * H + h * NC_b + r) * 64 of the workspace.
+    // Device arrays; only with nseg = 1 and no checkpoints.
+    const int64_t *cu = nullptr;
+    const int *cbase = nullptr;
+    const int *chunk_seq = nullptr;
+    int vl_chunks = 0;  // cbase[B]: the packed chunk count
 };
 
 // Per (sequence, segment) workspace: S [128][128], C [128][128], m [128], D [128].

@@ -520,11 +520,23 @@ __global__ void t_update_kernel(const int64_t *t0, int64_t *tT, int B, int T) {
     if (i < B) tT[i] = (t0 ? t0[i] : 0) + T;
 }
 
+__global__ void t_update_varlen_kernel(const int64_t *t0, int64_t *tT, const int64_t *cu, int n) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) tT[i] = (t0 ? t0[i] : 0) + (cu[i + 1] - cu[i]);
+}
+
 }  // namespace
 
 cudaError_t launch_t_update(const int64_t *t0, int64_t *tT, int B, int T, cudaStream_t s) {
     if (!tT || B == 0) return cudaSuccess;
     t_update_kernel<<<(B + 255) / 256, 256, 0, s>>>(t0, tT, B, T);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_t_update_varlen(const int64_t *t0, int64_t *tT, const int64_t *cu, int num_seqs,
+                                   cudaStream_t s) {
+    if (!tT || num_seqs == 0) return cudaSuccess;
+    t_update_varlen_kernel<<<(num_seqs + 255) / 256, 256, 0, s>>>(t0, tT, cu, num_seqs);
     return cudaGetLastError();
 }
 

@@ -251,16 +251,22 @@ def test_gdn_spectral_rejects_unknown_contraction(lib):
 def test_varlen_rejects_bad_offsets(lib):
     fake = ctypes.c_void_p(0x10000)
 
-    def call(cu, H=16, backbone=0):
+    def call(cu, H=16, backbone=0, fp32=False):
         arr = (ctypes.c_int64 * len(cu))(*cu)
-        return lib.ccq_fwd_varlen(backbone, *([fake] * 6), 0, 0, ctypes.cast(arr, ctypes.c_void_p), len(cu) - 1,
-                                  None, None, None, None, fake, None, None, None, None, H, 128, 128, None, 0,
+        dt, D = (1, 64) if fp32 else (0, 128)
+        return lib.ccq_fwd_varlen(backbone, *([fake] * 6), dt, 1 if backbone else dt,
+                                  ctypes.cast(arr, ctypes.c_void_p), len(cu) - 1,
+                                  None, None, None, None, fake, None, None, None, None, H, D, D, None, 0,
                                   ctypes.byref(ccq.params()), None)
     assert call([1, 5]) == ccq.CCQ_ERR_INVALID_ARG          # must start at 0
     assert b"cu_seqlens[0]" in lib.ccq_last_error()
     assert call([0, 9, 5]) == ccq.CCQ_ERR_INVALID_ARG       # decreasing
-    assert call([0, 3, 8], H=2) == ccq.CCQ_ERR_INVALID_ARG  # 3 * 2 fp32 rows: not 16-byte aligned
+    # the per-sequence path (fp32, d = 64) offsets fp32 [T][H] row pointers: 3 * 2 rows are not
+    # 16-byte aligned; the single launch (bf16, d = 128) indexes rows itself and needs no alignment
+    assert call([0, 3, 8], H=2, fp32=True) == ccq.CCQ_ERR_INVALID_ARG
     assert b"multiple of 4" in lib.ccq_last_error()
+    assert call([0, 3, 8], H=2) == ccq.CCQ_ERR_INVALID_ARG  # single launch: no workspace given
+    assert b"workspace" in lib.ccq_last_error()
     assert call([0, 3, 8], backbone=2) == ccq.CCQ_ERR_INVALID_ARG
     arr = (ctypes.c_int64 * 1)(0)
     assert lib.ccq_fwd_varlen(0, *([fake] * 6), 0, 0, ctypes.cast(arr, ctypes.c_void_p), 0, None, None, None, None,
