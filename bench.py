@@ -42,10 +42,22 @@ WORKLOADS = {
     "gdn_bf16_20k": ("gdn", 1, 16, 20480, 128),
     "decode_b256": ("decode", 256, 16, 1, 128),
     "gla_bf16_4k_fwdbwd": ("glabwd", 4, 16, 4096, 128),
+    # packed variable-length sequences: B sequences of 100-4000 tokens (VARLEN_SEED), one launch
+    "gla_bf16_varlen64": ("glavl", 64, 16, 0, 128),
+    "gdn_bf16_varlen64": ("gdnvl", 64, 16, 0, 128),
 }
+VARLEN_SEED = 77
+
+
+def varlen_lengths(n):
+    """The sequence lengths of a packed workload: n draws from 100..4000 tokens."""
+    import numpy as np
+    return np.random.default_rng(VARLEN_SEED).integers(100, 4001, size=n).tolist()
 KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode": "ccq_recurrent.cu",
+                  "glavl": "ccq_gla_chunk.cu", "gdnvl": "ccq_gdn_chunk.cu",
                   "glabwd": "ccq_gla_bwd.cu"}
 KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_kernel",
+                "glavl": "gla_chunk_kernel (packed sequences)", "gdnvl": "gdn_wy_kernel + gdn_chunk_kernel (packed sequences)",
                 "decode": "decode_kernel",
                 "glabwd": "whole step: forward (saving checkpoints) + gla_bwd_q_kernel + gla_bwd_state_kernel"
                           " + gla_bwd_kv_kernel"}
@@ -65,6 +77,8 @@ def launches_per_step(kind, B, H, T, sms):
     Gated DeltaNet forward two (WY, chunk) or four when segmented, the backward three,
     and every call that returns the position count adds the one-thread-per-row count
     update."""
+    if kind in ("glavl", "gdnvl"):  # one launch (two for GDN: WY, chunk) plus the count update
+        return 2 if kind == "glavl" else 3
     split = gla_segments(B, H, T, sms) > 1
     fwd = 3 if split else 1
     gdn = 4 if split else 2
@@ -75,6 +89,9 @@ def algorithmic_bytes(kind, B, H, T, D):
     """Bytes one launch must move at minimum: every input read once, o written
     once, final fp32 states written once (initial states are zero / absent
     except for decode, whose cache is read and written)."""
+    if kind in ("glavl", "gdnvl"):  # B sequences, T = the packed length
+        per = algorithmic_bytes(kind[:3], 1, H, T, D) - H * (2 * D * D + D) * 4 - 8
+        return per + B * (H * (2 * D * D + D) * 4 + 8)
     tok = B * T * H
     if kind == "glabwd":
         # forward: q, k, v, gk, lambda in, o out, final states out; backward:
@@ -93,6 +110,8 @@ def algorithmic_bytes(kind, B, H, T, D):
 
 def algorithmic_flops(kind, B, H, T, D, C=64):
     """Dense tile FLOPs of the chunkwise algorithm (Algorithm 1 products)."""
+    if kind in ("glavl", "gdnvl"):
+        return sum(algorithmic_flops(kind[:3], 1, H, n, D, C) for n in varlen_lengths(B))
     nc = (T + C - 1) // C
     # GLA: four C x D x D products (Qbar S^K, Qg S, Ku^T V, Kbar^T Kbar) and four
     # C x C x D products (Qbar Kbar^T, W' Kbar, Qg Kg^T, A V), 2 FLOP per MAC.
@@ -255,6 +274,8 @@ def whole_job_rate(world, units_per_step, steps, max_ms):
 def cpu_oracle_run(kind, B, H, T, D, sample_b, seed):
     """Time the fp64 oracle on host cores over `sample_b` batch rows of T tokens."""
     import torch
+    if kind in ("glavl", "gdnvl"):  # a sample sequence of the pack
+        kind = kind[:3]
     import oracle
     from paper_2606_01294_gb300 import inputs as gen
     if kind == "decode":
@@ -290,6 +311,8 @@ def run_reference(args):
     # over the first Ts tokens, so that warm-up + steps stay within minutes
     sample_b = 1 if kind != "decode" else 16
     Ts = min(T, 1024) if kind != "decode" else 1
+    if kind in ("glavl", "gdnvl"):
+        Ts = 1024
     cores = os.cpu_count() or 1
     for _ in range(args.warmup):
         cpu_oracle_run(kind, B, H, Ts, D, sample_b, seed=99)
@@ -365,6 +388,30 @@ def setup_workload(kind, B, H, T, D, dev, seed):
             train_step(Dv)
         tokens_per_step = B * T
         host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
+    elif kind in ("glavl", "gdnvl"):
+        bb = gen.GLA if kind == "glavl" else gen.GDN
+        lens = varlen_lengths(B)
+        total = sum(lens)
+        cu = [0]
+        for n in lens:
+            cu.append(cu[-1] + n)
+        P = {n: (None if x is None else x[0])
+             for n, x in gen.make_inputs(bb, 1, total, H, D, D, dtype=torch.bfloat16, seed=seed).items()}
+        Dv = {n: (None if x is None else x.to(dev)) for n, x in P.items()}
+        out = torch.empty(total, H, D, dtype=torch.bfloat16, device=dev)
+        fstate = ccq.CCQState.empty(B, H, D, D, dev)
+        need = ccq.varlen_workspace_size(bb, cu, H, D, D)
+        ws = torch.empty(max(need, 1), dtype=torch.uint8, device=dev)
+
+        def run(d):
+            o, _ = ccq.fwd_varlen(bb, d["q"], d["k"], d["v"], d["gate"], d["lam"], cu, beta=d["beta"], out=out,
+                                  workspace=ws, final_state=fstate)
+            return o
+
+        def step():
+            run(Dv)
+        tokens_per_step = total
+        host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
     else:
         bb = gen.GLA if kind == "gla" else gen.GDN
         P = gen.make_inputs(bb, B, T, H, D, D, dtype=torch.bfloat16, seed=seed)
@@ -391,6 +438,8 @@ def setup_workload(kind, B, H, T, D, dev, seed):
         if kind == "glabwd":
             train_step(d)
             return [grads[n].to("cpu", non_blocking=True) for n in ("dq", "dk", "dv", "dgk")]
+        if kind in ("glavl", "gdnvl"):
+            return run(d).to("cpu", non_blocking=True)
         if kind == "gla":
             o, _ = ccq.gla_fwd(d["q"], d["k"], d["v"], d["gate"], d["lam"], out=out,
                                final_state=fstate, workspace=ws)
@@ -479,6 +528,8 @@ def run_gpu(args):
         build()
 
     kind, B, H, T, D = WORKLOADS[args.workload]
+    if kind in ("glavl", "gdnvl"):
+        T = sum(varlen_lengths(B))  # the packed length
     seed = 1236 + rank
     stream = torch.cuda.current_stream(dev)
     step, e2e_step, tokens_per_step, h2d, d2h = setup_workload(kind, B, H, T, D, dev, seed)
@@ -534,8 +585,8 @@ def run_gpu(args):
             import oracle
             oracle.build_oracle()
             # repeat passes over a bounded sample until about 10 s of CPU work
-            sample_b = {"decode": 32, "glabwd": 1}.get(kind, B)
-            Tc = min(T, 1024) if kind == "glabwd" else T
+            sample_b = {"decode": 32, "glabwd": 1, "glavl": 1, "gdnvl": 1}.get(kind, B)
+            Tc = min(T, 1024) if kind == "glabwd" else (1024 if kind in ("glavl", "gdnvl") else T)
             toks, secs, passes = 0.0, 0.0, 0
             while secs < 10.0 and passes < 20:
                 rate, dt = cpu_oracle_run(kind, B, H, Tc, D, sample_b, seed=seed)
@@ -565,6 +616,11 @@ def run_gpu(args):
             "kernel_ms_mean": kern_ms,
             "kernel_ms_min": min(launch_ms),
         }
+        if kind in ("glavl", "gdnvl"):
+            lens = varlen_lengths(B)
+            line["config"]["seq_len"] = None
+            line["config"]["packing"] = (f"{B} sequences of {min(lens)}-{max(lens)} tokens (seeded draw from "
+                                         f"100-4000), packed [T, H, D], one launch")
         if also:
             line["also"] = also
         print(json.dumps(line), flush=True)

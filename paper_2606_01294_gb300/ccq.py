@@ -512,8 +512,21 @@ def gdn_fwd_decayed(q, k, v, g, beta, lam, *, S0=None, C0=None, m0=None, n0=None
     return (o, fs) if return_state else o
 
 
+def varlen_workspace_size(backbone, cu_seqlens, H, Dk, Dv, dtype=torch.bfloat16, **kw) -> int:
+    """Bytes of device workspace ccq_fwd_varlen needs for this pack (ccq_fwd_varlen_workspace_size)."""
+    cu = [int(x) for x in (cu_seqlens.tolist() if hasattr(cu_seqlens, "tolist") else cu_seqlens)]
+    cu_arr = (ctypes.c_int64 * len(cu))(*cu)
+    p = params(**kw)
+    need = ctypes.c_size_t(0)
+    code = BF16 if dtype == torch.bfloat16 else FP32
+    _check(load_library().ccq_fwd_varlen_workspace_size(int(backbone), ctypes.cast(cu_arr, _VP), len(cu) - 1, H,
+                                                        Dk, Dv, code, ctypes.byref(p), ctypes.byref(need)))
+    return need.value
+
+
 def fwd_varlen(backbone, q, k, v, gate, lam, cu_seqlens, *, beta=None, state: Optional[CCQState] = None,
-               out=None, return_state: bool = True, workspace=None, stream=None, **kw):
+               out=None, final_state: Optional[CCQState] = None, return_state: bool = True, workspace=None,
+               stream=None, **kw):
     """Forward of packed variable-length sequences (ccq_fwd_varlen).  q, k [total,H,Dk]; v
     [total,H,Dv]; gate [total,H,Dk] (GLA) or [total,H] fp32 (GDN, with beta [total,H]); lam
     [total,H]; ``cu_seqlens`` the num_seqs + 1 offsets (a list or CPU integer tensor; it stays on
@@ -542,7 +555,9 @@ def fwd_varlen(backbone, q, k, v, gate, lam, cu_seqlens, *, beta=None, state: Op
     S0, C0, m0, t0 = _state_in(state, ns, H, Dk, Dv, dev)
     o = out if out is not None else torch.empty(total, H, Dv, dtype=q.dtype, device=dev)
     _req(o, "out", dev, q.dtype, (total, H, Dv))
-    fs = CCQState.empty(ns, H, Dk, Dv, dev) if return_state else None
+    fs = (final_state or CCQState.empty(ns, H, Dk, Dv, dev)) if return_state else None
+    if fs is not None:
+        _state_in(fs, ns, H, Dk, Dv, dev)
     cu_arr = (ctypes.c_int64 * len(cu))(*cu)
     p = params(**kw)
     lib = load_library()
