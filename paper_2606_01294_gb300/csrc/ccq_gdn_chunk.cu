@@ -365,8 +365,8 @@ constexpr uint32_t MS_RQ = 0, MS_MQ = 256, MS_LT = 512, MS_RK = 768, MS_EP = 102
 constexpr uint32_t M_DMP = 6144;     // [2][128] key-sum halves of the chunk
 constexpr uint32_t M_DMPREV = 7168;  // [128]
 constexpr uint32_t M_BAR = 7680;     // mbarriers
-constexpr uint32_t M_TMEM = 7808;
-constexpr uint32_t M_ABORT = 7812;
+constexpr uint32_t M_TMEM = 7824;
+constexpr uint32_t M_ABORT = 7828;
 constexpr uint32_t M_EPO = 7936;     // [2][64] e^{gc} of the chunk whose output is being written
 constexpr uint32_t kMiscBytes = 8448;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;
@@ -376,7 +376,7 @@ static_assert(MS_SCAL + 66 * 4 <= MS_MST, "scalar area overlaps");
 enum {
     BAR_IN0 = 0, BAR_IN1 = 1, BAR_WU = 2, BAR_GA1 = 3, BAR_GA2 = 4, BAR_GB = 5, BAR_GK = 6, BAR_GC = 7,
     BAR_GC2 = 8, BAR_GD = 9, BAR_PREP0 = 10, BAR_PREP1 = 11, BAR_SNAPK = 12, BAR_SNAPS = 13,
-    BAR_OST0 = 14, BAR_OST1 = 15, kNumBars = 16
+    BAR_OST0 = 14, BAR_OST1 = 15, BAR_GP = 16, kNumBars = 17
 };
 static_assert(M_BAR + 8 * kNumBars <= M_TMEM, "barrier area");
 enum { NB_PO = 1, NB_W = 2, NB_QC = 3, NB_MASK = 4, NB_OUT = 5, NB_PREP = 6, NB_EPI = 7 };
@@ -618,6 +618,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     store_row_chunk(sm + OFF_WM, i, 4 * hf + 2 * grp + q2, w);
                 }
             }
+            fence_proxy_async_smem();  // W' is read by G3, issued with G1 after NB_PO
             // ---- R = V - e^{gc} Kbar H0: read Kbar H0 out of the P/O accumulator
             // first, freeing it for G1
             mbar_wait(&bar[BAR_GA2], par, abort_flag, status);
@@ -653,16 +654,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 uint4 qraw[4];
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) qraw[q4] = *reinterpret_cast<const uint4 *>(qt + t64_chunk(i, 4 * hf + q4));
-                mbar_wait(&bar[BAR_GB], par, abort_flag, status);
+                mbar_wait(&bar[BAR_GP], par, abort_flag, status);
                 tc_fence_after();
-                {
-                    // U = Tb R (the MMA has read R) -> bf16 U tile in R's place
-                    float u[32];
-                    tmem_ld16x2_32<32>(tq + TM_U + 64 * grp, u);
-#pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4)
-                        store_row_chunk(sm + OFF_UB + grp * 8192, i, 4 * hf + q4, u + 8 * q4);
-                }
                 const float cm = lt * c;
                 float p[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
@@ -682,6 +675,17 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     }
                     *reinterpret_cast<uint4 *>(qt + t64_chunk(i, 4 * hf + q4)) = make_uint4(ow[0], ow[1], ow[2], ow[3]);
                 }
+            }
+            // U = Tb R (the MMA has read R; it ran while q_clean was formed) -> bf16 U tile in
+            // R's place
+            mbar_wait(&bar[BAR_GB], par, abort_flag, status);
+            tc_fence_after();
+            {
+                float u[32];
+                tmem_ld16x2_32<32>(tq + TM_U + 64 * grp, u);
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4)
+                    store_row_chunk(sm + OFF_UB + grp * 8192, i, 4 * hf + q4, u + 8 * q4);
             }
             // gc_i - gc_j (log2 units) of this thread's 16 key columns, and e^{gc} of the rows for
             // the output epilogue, read before the slot is released
@@ -725,13 +729,16 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             // ---- output o_i = scale (e^{gc_i} O1_i + O2_i), staged for the copy warp's TMA store
             // in the slot's Kd tile (its last reader, D6, completed before GD).
             // O1^T, O2^T are M = 128 accumulators: this thread holds value column `row` for the
-            // chunk rows 32 grp .. 32 grp + 31.
+            // chunk rows 32 grp .. 32 grp + 31.  A lane pair swaps one value per two rows so that
+            // each lane writes a bf16 pair of adjacent columns: the even lane row e, the odd lane
+            // row e + 1 (half the shared-memory stores of one column per thread).
             named_bar(NB_EPI, kEpiThreads);  // epo of this chunk visible
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             {
-                __nv_bfloat16 *ot = reinterpret_cast<__nv_bfloat16 *>(slot + SO_KD + (row >> 6) * 8192);
-                const bool direct = partial(r);
+                uint8_t *ot = slot + SO_KD + (row >> 6) * 8192;
+                const bool direct = partial(r), odd = lane & 1;
+                const int c2 = row & ~1;  // first column of this lane's pair
 #pragma unroll 1
                 for (int hh = 0; hh < 2; ++hh) {
                     const int i0 = 32 * grp + 16 * hh;
@@ -743,13 +750,19 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     for (int q = 0; q < 4; ++q) {
                         const float4 e4 = *reinterpret_cast<const float4 *>(ep_r + 4 * q);
                         const float ev4[4] = {e4.x, e4.y, e4.z, e4.w};
+                        float ov[4];
 #pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const int e = 4 * q + u;
-                            const __nv_bfloat16 ov = __float2bfloat16_rn(a.scale * fmaf(ev4[u], o1[e], o2[e]));
-                            const int tpos = (cb + r) * kC + i0 + e;  // position in the sequence
-                            if (!direct) ot[t64_offset(i0 + e, row & 63) >> 1] = ov;
-                            else if (tpos < T) a.o[((rowbase + tpos) * H + h) * kD + row] = ov;
+                        for (int u = 0; u < 4; ++u) ov[u] = a.scale * fmaf(ev4[u], o1[4 * q + u], o2[4 * q + u]);
+#pragma unroll
+                        for (int u = 0; u < 4; u += 2) {
+                            const float y = __shfl_xor_sync(0xffffffffu, odd ? ov[u] : ov[u + 1], 1);
+                            const int e = i0 + 4 * q + u + (odd ? 1 : 0);  // chunk row of the pair
+                            const uint32_t pr = odd ? pack_bf16(y, ov[u + 1]) : pack_bf16(ov[u], y);
+                            const int tpos = (cb + r) * kC + e;  // position in the sequence
+                            if (!direct)
+                                *reinterpret_cast<uint32_t *>(ot + t64_offset(e, c2 & 63)) = pr;
+                            else if (tpos < T)
+                                *reinterpret_cast<uint32_t *>(a.o + ((rowbase + tpos) * H + h) * kD + c2) = pr;
                         }
                     }
                 }
@@ -966,22 +979,25 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     mma_bf16(tbase + TM_PO, dK + (k >> 2) * 512 + (k & 3) * 2, dHB + k * 128, ID_64x128_KM, k != 0);
             if (lead && !*abort_flag) mma_commit(&bar[BAR_GA2]);
             __syncwarp();
-            // G1 P = Q S^K once WH is out of the accumulator
+            // G1 P = Q S^K once Kbar H0 is out of the accumulator, G3 P += W' Kbar (W' is
+            // written before NB_PO)
             named_bar(NB_PO, kSyncCount);
             mbar_wait(&bar[BAR_SNAPK], par, abort_flag, status);
             tc_fence_after();
-            if (lead && !*abort_flag)
+            if (lead && !*abort_flag) {
                 for (int k = 0; k < 8; ++k)
                     mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
                              dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
+                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+                mma_commit(&bar[BAR_GP]);
+            }
             __syncwarp();
-            // DU U = Tb R, G3 P += W' Kbar, G8 S^K += Kbar^T Kbar
+            // DU U = Tb R, G8 S^K += Kbar^T Kbar
             mbar_wait(&bar[BAR_WU], par, abort_flag, status);  // Tb of the chunk
             named_bar(NB_W, kSyncCount);
             tc_fence_after();
             if (lead && !*abort_flag) {
                 for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_U, dTB + k * 2, dUBm + k * 128, ID_64x128_KM, k != 0);
-                for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_PO, dWm + k * 2, dKm + k * 128, ID_64x128_KM, 1);
                 mma_commit(&bar[BAR_GB]);
                 for (int k = 0; k < 4; ++k) mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
                 mma_commit(&bar[BAR_GK]);
