@@ -140,6 +140,8 @@ STEP_KERNELS = {
     "decode_b256": ["decode_kernel"],
     "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
                            "gla_bwd_q_kernel", "gla_bwd_state_kernel", "gla_bwd_kv_kernel"],
+    "gla_bf16_varlen64": ["gla_chunk_kernel"],
+    "gdn_bf16_varlen64": ["gdn_wy_kernel", "gdn_chunk_kernel"],
 }
 # (each step also runs the one-thread-per-row position update: 8 bytes per batch row, not counted)
 KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kernel": "ccq_gla_segment.cu",

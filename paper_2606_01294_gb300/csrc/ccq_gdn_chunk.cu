@@ -41,6 +41,10 @@ namespace ccq {
 
 namespace {
 
+__device__ __forceinline__ void st_shared_b32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared.b32 [%0], %1;" ::"r"(addr), "r"(v));
+}
+
 constexpr int kC = 64;
 constexpr int kD = 128;
 constexpr float kLog2e = 1.4426950408889634f;
@@ -659,7 +663,9 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 const float cm = lt * c;
                 float p[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
-                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqi, rqi), cm2 = f2_make(cm, cm);
+                // the read scale is applied here: both output products are linear in q_clean
+                const float rqs = rqi * a.scale, cms = cm * a.scale;
+                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqs, rqs), cm2 = f2_make(cms, cms);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4);
@@ -726,19 +732,26 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar_arrive(NB_MASK, kSyncCount);
-            // ---- output o_i = scale (e^{gc_i} O1_i + O2_i), staged for the copy warp's TMA store
-            // in the slot's Kd tile (its last reader, D6, completed before GD).
-            // O1^T, O2^T are M = 128 accumulators: this thread holds value column `row` for the
-            // chunk rows 32 grp .. 32 grp + 31.  A lane pair swaps one value per two rows so that
-            // each lane writes a bf16 pair of adjacent columns: the even lane row e, the odd lane
-            // row e + 1 (half the shared-memory stores of one column per thread).
+            // ---- output o_i = e^{gc_i} O1_i + O2_i (q_clean carries the read scale), staged for
+            // the copy warp's TMA store in the slot's Kd tile (its last reader, D6, completed
+            // before GD).  O1^T, O2^T are M = 128 accumulators: this thread holds value column
+            // `row` for the chunk rows 32 grp .. 32 grp + 31.  A lane pair swaps one value per two
+            // rows so that each lane writes a bf16 pair of adjacent columns: the even lane row e,
+            // the odd lane row e + 1 (half the shared-memory stores of one column per thread).
             named_bar(NB_EPI, kEpiThreads);  // epo of this chunk visible
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             {
-                uint8_t *ot = slot + SO_KD + (row >> 6) * 8192;
                 const bool direct = partial(r), odd = lane & 1;
                 const int c2 = row & ~1;  // first column of this lane's pair
+                // Shared addresses of the pair in tile row 0 + odd for the four swizzle classes of
+                // the even rows (row & 7 = 0, 2, 4, 6); a row adds 128 bytes.
+                const uint32_t ob = smem_addr(slot + SO_KD + (row >> 6) * 8192) + (odd ? 128u : 0u) +
+                                    (static_cast<uint32_t>(c2 & 7) << 1);
+                const uint32_t cx = (static_cast<uint32_t>(c2 & 63) >> 3) ^ (odd ? 1u : 0u);
+                uint32_t bk[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) bk[k] = ob + ((cx ^ (2u * k)) << 4);
 #pragma unroll 1
                 for (int hh = 0; hh < 2; ++hh) {
                     const int i0 = 32 * grp + 16 * hh;
@@ -746,23 +759,25 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     tmem_ld16(tq + TM_O1 + i0, o1);
                     tmem_ld16(tq + TM_O2 + i0, o2);
                     const float *ep_r = epo + (r & 1) * 64 + i0;
+                    const uint32_t rb = static_cast<uint32_t>(i0) * 128u;
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
                         const float4 e4 = *reinterpret_cast<const float4 *>(ep_r + 4 * q);
                         const float ev4[4] = {e4.x, e4.y, e4.z, e4.w};
                         float ov[4];
 #pragma unroll
-                        for (int u = 0; u < 4; ++u) ov[u] = a.scale * fmaf(ev4[u], o1[4 * q + u], o2[4 * q + u]);
+                        for (int u = 0; u < 4; ++u) ov[u] = fmaf(ev4[u], o1[4 * q + u], o2[4 * q + u]);
 #pragma unroll
                         for (int u = 0; u < 4; u += 2) {
                             const float y = __shfl_xor_sync(0xffffffffu, odd ? ov[u] : ov[u + 1], 1);
-                            const int e = i0 + 4 * q + u + (odd ? 1 : 0);  // chunk row of the pair
                             const uint32_t pr = odd ? pack_bf16(y, ov[u + 1]) : pack_bf16(ov[u], y);
-                            const int tpos = (cb + r) * kC + e;  // position in the sequence
-                            if (!direct)
-                                *reinterpret_cast<uint32_t *>(ot + t64_offset(e, c2 & 63)) = pr;
-                            else if (tpos < T)
-                                *reinterpret_cast<uint32_t *>(a.o + ((rowbase + tpos) * H + h) * kD + c2) = pr;
+                            if (!direct) {
+                                st_shared_b32(bk[(2 * q + u / 2) & 3] + rb + (4 * q + u) * 128, pr);
+                            } else {
+                                const int tpos = (cb + r) * kC + i0 + 4 * q + u + (odd ? 1 : 0);
+                                if (tpos < T)
+                                    *reinterpret_cast<uint32_t *>(a.o + ((rowbase + tpos) * H + h) * kD + c2) = pr;
+                            }
                         }
                     }
                 }
