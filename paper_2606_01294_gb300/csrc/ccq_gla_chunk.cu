@@ -26,7 +26,7 @@
 //   + sum_{j<=i} (qbar_i . kbar_j - c_i) kbar_j and
 //   D (P^prev + P^intra) - MeanCorr = (rq_i P_i - c_i M) / t_i     (App. B, re-associated)
 //   q_clean_i = qbar_i - lambda_i (rq_i P_i - c_i M) / t_i          (Eq. clean)
-// GLA gates are measured from the chunk midpoint Gmid: Qg = q_clean * e^{G - Gmid},
+// GLA gates are measured from the chunk midpoint Gmid: Qg = scale q_clean e^{G - Gmid},
 // Kg = kbar * e^{Gmid - G}, Ssnap = e^{Gmid} S_r, and S_{r+1} = e^{Gtot - Gmid} X_{r+1}
 // (that factor is applied at the next snapshot).  A factor e^{G - Gmid} of a row before the
 // midpoint grows with the decay between that row and the midpoint, so the factoring is exact
@@ -424,7 +424,9 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 const float cm = lt * c;  // lambda_i c_i / t_i
                 float p[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, p);
-                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqi, rqi), cm2 = f2_make(cm, cm);
+                // the read scale is applied here: O is linear in the scaled q_clean
+                const float rqs = rqi * a.scale, cms = cm * a.scale;
+                const uint64_t nlt = f2_make(-lt, -lt), rq2 = f2_make(rqs, rqs), cm2 = f2_make(cms, cms);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4) {
                     const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mst + 8 * q4);
@@ -472,15 +474,14 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar_arrive(NB_MASK, kSyncCount);
-            // ---- output: o = scale O staged (bf16, swizzled) in the v tile, which G5 has
-            // finished reading; the issuing thread stores it with one TMA copy (rows past T
-            // fall outside the tensor and are not written)
+            // ---- output: o = O (q_clean carries the read scale) staged (bf16, swizzled) in the
+            // v tile, which G5 has finished reading; the copy warp stores it with one TMA copy
+            // (rows past T fall outside the tensor and are not written)
             mbar_wait(&bar[BAR_GD], par, abort_flag, status);
             tc_fence_after();
             if (!a.skip_o) {
                 float x[32];
                 tmem_ld16x2_32<32>(tq + TM_PO + 64 * grp, x);
-                const uint64_t sc2 = f2_make(a.scale, a.scale);
                 const int tpos = (cb + r) * kC + i;  // position of row i in the sequence
                 const bool direct = partial(r);
                 uint4 *dst = reinterpret_cast<uint4 *>(a.o + ((rowbase + tpos) * H + h) * kD + 64 * grp + 32 * hf);
@@ -489,7 +490,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     uint32_t w[4];
 #pragma unroll
                     for (int u = 0; u < 4; ++u)
-                        w[u] = bf16x2_from_f2(f2_mul(f2_make(x[8 * q4 + 2 * u], x[8 * q4 + 2 * u + 1]), sc2));
+                        w[u] = pack_bf16(x[8 * q4 + 2 * u], x[8 * q4 + 2 * u + 1]);
                     if (!direct)
                         *reinterpret_cast<uint4 *>(sm + OFF_V + grp * 8192 + t64_chunk(i, 4 * hf + q4)) = make_uint4(w[0], w[1], w[2], w[3]);
                     else if (tpos < T)
@@ -651,6 +652,12 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     slot_f(s, MS_EGM)[d0] = fast_exp2(gm0 * kLog2e);
                     slot_f(s, MS_EGM)[d0 + 1] = fast_exp2(gm1 * kLog2e);
                 }
+                {
+                    // log gates are <= 0, so G falls monotonically and the factors' exponents are
+                    // largest in magnitude at the chunk's first and last tokens
+                    const float2 xe = f2_split(f2_fma(th ? g2[31] : g2[0], l2e, o2));
+                    emax = fmaxf(emax, fmaxf(fabsf(xe.x), fabsf(xe.y)));
+                }
                 const float *rk = slot_f(s, MS_RK);
                 const uint32_t tcol = (d0 >> 6) * 8192;
                 uint64_t dm2 = 0;
@@ -673,7 +680,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                         const uint32_t off = tcol + t64_offset(j, d0 & 63);
                         const uint64_t k2 = f2_mul(f2_from_bf16x2(kraw[u]), f2_make(rkv[u], rkv[u]));
                         const float2 x = f2_split(f2_fma(g2[jj], l2e, o2));
-                        emax = fmaxf(emax, fmaxf(fabsf(x.x), fabsf(x.y)));
                         *reinterpret_cast<uint32_t *>(slot + SO_K + off) = bf16x2_from_f2(k2);
                         *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
                             bf16x2_from_f2(f2_mul(k2, f2_make(fast_exp2(-x.x), fast_exp2(-x.y))));
