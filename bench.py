@@ -31,6 +31,8 @@ sys.path.insert(0, ROOT)
 
 METRIC = "CCQ chunked fwd tokens/s at T=4K,d=128 bf16; % of roofline (tensor/HBM)"
 METRIC_FWDBWD = "CCQ-GLA chunked fwd+bwd tokens/s at T=4K,d=128 bf16; % of roofline (HBM)"
+METRIC_GDN_FWDBWD = "CCQ-GDN chunked fwd+bwd tokens/s at T=4K,d=128 bf16; % of roofline (HBM)"
+METRICS = {"glabwd": METRIC_FWDBWD, "gdnbwd": METRIC_GDN_FWDBWD}
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic.json")
 
@@ -42,6 +44,7 @@ WORKLOADS = {
     "gdn_bf16_20k": ("gdn", 1, 16, 20480, 128),
     "decode_b256": ("decode", 256, 16, 1, 128),
     "gla_bf16_4k_fwdbwd": ("glabwd", 4, 16, 4096, 128),
+    "gdn_bf16_4k_fwdbwd": ("gdnbwd", 4, 16, 4096, 128),
     # packed variable-length sequences: B sequences of 100-4000 tokens (VARLEN_SEED), one launch
     "gla_bf16_varlen64": ("glavl", 64, 16, 0, 128),
     "gdn_bf16_varlen64": ("gdnvl", 64, 16, 0, 128),
@@ -55,12 +58,13 @@ def varlen_lengths(n):
     return np.random.default_rng(VARLEN_SEED).integers(100, 4001, size=n).tolist()
 KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode": "ccq_recurrent.cu",
                   "glavl": "ccq_gla_chunk.cu", "gdnvl": "ccq_gdn_chunk.cu",
-                  "glabwd": "ccq_gla_bwd.cu"}
+                  "glabwd": "ccq_gla_bwd.cu", "gdnbwd": "ccq_gdn_bwd_kernels.cuh"}
 KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_kernel",
                 "glavl": "gla_chunk_kernel (packed sequences)", "gdnvl": "gdn_wy_kernel + gdn_chunk_kernel (packed sequences)",
                 "decode": "decode_kernel",
                 "glabwd": "whole step: forward (saving checkpoints) + gla_bwd_q_kernel + gla_bwd_state_kernel"
-                          " + gla_bwd_kv_kernel"}
+                          " + gla_bwd_kv_kernel",
+                "gdnbwd": "whole step: forward (gdn_wy_kernel + gdn_chunk_kernel) + the seven gdn_bwd_* kernels"}
 
 
 def gla_segments(B, H, T, sms):
@@ -82,7 +86,7 @@ def launches_per_step(kind, B, H, T, sms):
     split = gla_segments(B, H, T, sms) > 1
     fwd = 3 if split else 1
     gdn = 4 if split else 2
-    return {"gla": fwd + 1, "gdn": gdn + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3}[kind]
+    return {"gla": fwd + 1, "gdn": gdn + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3, "gdnbwd": gdn + 1 + 7}[kind]
 
 
 def algorithmic_bytes(kind, B, H, T, D):
@@ -99,6 +103,12 @@ def algorithmic_bytes(kind, B, H, T, D):
         # initial-state gradients out (each pass reads its own inputs once)
         fwd = algorithmic_bytes("gla", B, H, T, D)
         bwd = tok * D * 2 * 5 + tok * 4 + tok * D * 2 * 4 + tok * 4 + B * H * (2 * D * D + D) * 4
+        return fwd + bwd
+    if kind == "gdnbwd":
+        # forward as gdn; backward: q, k, v, dout (bf16) and g, beta, lambda (fp32) in, dq, dk, dv
+        # (bf16) and dg, dbeta, dlambda (fp32) out, the three initial-state gradients out
+        fwd = algorithmic_bytes("gdn", B, H, T, D)
+        bwd = tok * D * 2 * 4 + tok * 4 * 3 + tok * D * 2 * 3 + tok * 4 * 3 + B * H * (2 * D * D + D) * 4
         return fwd + bwd
     if kind == "gla":
         return tok * D * 2 * 4 + tok * D * 2 + tok * 4 + B * H * (2 * D * D + D) * 4 + B * 8
@@ -122,9 +132,13 @@ def algorithmic_flops(kind, B, H, T, D, C=64):
     # D x D x C (dS), C x D x C (P1^T QG, SA dO).
     bwd = 2 * (3 * C * C * D + 5 * C * D * D + 5 * C * D * C + D * D * C + 2 * D * C * C
                + 2 * C * C * D + 2 * C * D * D + D * D * C + 2 * C * D * C)
+    # Gated DeltaNet backward (ccq_gdn_bwd_kernels.cuh), its products per chunk summed over the
+    # prep, state, local and kv passes: fifteen C x D x D, twenty-two C x C x D, two C x C x C.
+    gbwd = 2 * (15 * C * D * D + 22 * C * C * D + 2 * C * C * C)
     per_chunk = {"gla": 8 * C * D * D + 8 * C * C * D,
                  "gdn": 10 * C * D * D + 12 * C * C * D,
-                 "glabwd": 8 * C * D * D + 8 * C * C * D + bwd}.get(kind)
+                 "glabwd": 8 * C * D * D + 8 * C * C * D + bwd,
+                 "gdnbwd": 10 * C * D * D + 12 * C * C * D + gbwd}.get(kind)
     if per_chunk is None:
         return B * H * 8 * D * D
     return B * H * nc * per_chunk
@@ -140,6 +154,9 @@ STEP_KERNELS = {
     "decode_b256": ["decode_kernel"],
     "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
                            "gla_bwd_q_kernel", "gla_bwd_state_kernel", "gla_bwd_kv_kernel"],
+    "gdn_bf16_4k_fwdbwd": ["gdn_wy_kernel", "gdn_chunk_kernel", "gdn_bwd_prep_kernel", "gdn_bwd_prefix_kernel",
+                           "gdn_bwd_fstate_kernel", "gdn_bwd_local_kernel", "gdn_bwd_dstate_kernel",
+                           "gdn_bwd_suffix_kernel", "gdn_bwd_kv_kernel"],
     "gla_bf16_varlen64": ["gla_chunk_kernel"],
     "gdn_bf16_varlen64": ["gdn_wy_kernel", "gdn_chunk_kernel"],
 }
@@ -149,7 +166,9 @@ KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kerne
                 "gdn_chunk_kernel": "ccq_gdn_chunk.cu",
                 "gdn_segment_state_kernel": "ccq_gdn_segment.cu", "gdn_segment_combine_kernel": "ccq_gdn_segment.cu", "recurrent": "ccq_recurrent.cu",
                 "decode_kernel": "ccq_recurrent.cu", "gla_bwd_state_kernel": "ccq_gla_bwd.cu",
-                "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu"}
+                "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu",
+                **{f"gdn_bwd_{n}_kernel": "ccq_gdn_bwd_kernels.cuh"
+                   for n in ("prep", "prefix", "fstate", "local", "dstate", "suffix", "kv")}}
 
 
 SHARED_DEVICE_SOURCES = ("sm100_ptx.cuh", "ccq_internal.h")  # inlined into every kernel
@@ -293,11 +312,13 @@ def cpu_oracle_run(kind, B, H, T, D, sample_b, seed):
     bb = gen.GDN if kind == "gdn" else gen.GLA
     P = gen.make_inputs(bb, sample_b, T, H, D, D, dtype=torch.bfloat16, seed=seed)
     G = gen.make_backward_inputs(sample_b, T, H, D, D, seed=seed + 1, state_grads=False) \
-        if kind == "glabwd" else None
+        if kind in ("glabwd", "gdnbwd") else None
     t0 = time.perf_counter()
     oracle.forward(bb, P["q"], P["k"], P["v"], P["gate"], P["lam"], beta=P["beta"])
     if kind == "glabwd":
         oracle.gla_backward(P["q"], P["k"], P["v"], P["gate"], P["lam"], G["dout"])
+    if kind == "gdnbwd":
+        oracle.gdn_backward(P["q"], P["k"], P["v"], P["gate"], P["beta"], P["lam"], G["dout"])
     dt = time.perf_counter() - t0
     return sample_b * T / dt, dt
 
@@ -326,7 +347,7 @@ def run_reference(args):
     sample = (f"batch row 0 of {B}, all {H} heads, first {Ts} of {T} tokens, per step"
               if kind != "decode" else f"{sample_b} of {B} batch rows, all {H} heads, one token")
     line = {
-        "impl": "reference", "metric": METRIC_FWDBWD if kind == "glabwd" else METRIC,
+        "impl": "reference", "metric": METRICS.get(kind, METRIC),
         "value": rate, "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
@@ -390,6 +411,32 @@ def setup_workload(kind, B, H, T, D, dev, seed):
             train_step(Dv)
         tokens_per_step = B * T
         host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
+    elif kind == "gdnbwd":
+        P = gen.make_inputs(gen.GDN, B, T, H, D, D, dtype=torch.bfloat16, seed=seed, lam="trained")
+        P["dout"] = gen.make_backward_inputs(B, T, H, D, D, seed=seed + 1, state_grads=False)["dout"]
+        Dv = {n: (None if x is None else x.to(dev)) for n, x in P.items()}
+        out = torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev)
+        fstate = ccq.CCQState.empty(B, H, D, D, dev)
+        ws = ccq.gdn_workspace(B, T, H, D, D, dev)
+        bws = ccq.gdn_bwd_workspace(B, T, H, D, D, dev)
+        grads = {"dq": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dk": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dv": torch.empty(B, T, H, D, dtype=torch.bfloat16, device=dev),
+                 "dg": torch.empty(B, T, H, device=dev), "dbeta": torch.empty(B, T, H, device=dev),
+                 "dlambda": torch.empty(B, T, H, device=dev),
+                 "dS0": torch.empty(B, H, D, D, device=dev), "dC0": torch.empty(B, H, D, D, device=dev),
+                 "dm0": torch.empty(B, H, D, device=dev)}
+
+        def train_step(d):
+            ccq.gdn_fwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], out=out, final_state=fstate,
+                        workspace=ws)
+            ccq.gdn_bwd(d["q"], d["k"], d["v"], d["gate"], d["beta"], d["lam"], d["dout"], out=grads,
+                        workspace=bws)
+
+        def step():
+            train_step(Dv)
+        tokens_per_step = B * T
+        host = {n: (None if x is None else x.pin_memory()) for n, x in P.items()}
     elif kind in ("glavl", "gdnvl"):
         bb = gen.GLA if kind == "glavl" else gen.GDN
         lens = varlen_lengths(B)
@@ -440,6 +487,9 @@ def setup_workload(kind, B, H, T, D, dev, seed):
         if kind == "glabwd":
             train_step(d)
             return [grads[n].to("cpu", non_blocking=True) for n in ("dq", "dk", "dv", "dgk")]
+        if kind == "gdnbwd":
+            train_step(d)
+            return [grads[n].to("cpu", non_blocking=True) for n in ("dq", "dk", "dv", "dg")]
         if kind in ("glavl", "gdnvl"):
             return run(d).to("cpu", non_blocking=True)
         if kind == "gla":
@@ -452,6 +502,8 @@ def setup_workload(kind, B, H, T, D, dev, seed):
 
     h2d = sum(x.numel() * x.element_size() for x in host.values() if x is not None)
     d2h = out.numel() * out.element_size() * (4 if kind == "glabwd" else 1)
+    if kind == "gdnbwd":
+        d2h = sum(grads[n].numel() * grads[n].element_size() for n in ("dq", "dk", "dv", "dg"))
     return step, e2e_step, tokens_per_step, h2d, d2h
 
 
@@ -587,8 +639,8 @@ def run_gpu(args):
             import oracle
             oracle.build_oracle()
             # repeat passes over a bounded sample until about 10 s of CPU work
-            sample_b = {"decode": 32, "glabwd": 1, "glavl": 1, "gdnvl": 1}.get(kind, B)
-            Tc = min(T, 1024) if kind == "glabwd" else (1024 if kind in ("glavl", "gdnvl") else T)
+            sample_b = {"decode": 32, "glabwd": 1, "gdnbwd": 1, "glavl": 1, "gdnvl": 1}.get(kind, B)
+            Tc = min(T, 1024) if kind in ("glabwd", "gdnbwd") else (1024 if kind in ("glavl", "gdnvl") else T)
             toks, secs, passes = 0.0, 0.0, 0
             while secs < 10.0 and passes < 20:
                 rate, dt = cpu_oracle_run(kind, B, H, Tc, D, sample_b, seed=seed)
@@ -600,7 +652,7 @@ def run_gpu(args):
                    "sample": (f"{sample_b} of {B} batch rows, all {H} heads, {Tc} of {T} tokens, "
                               f"{passes} passes ({secs:.1f} s)")}
         line = {
-            "metric": METRIC_FWDBWD if kind == "glabwd" else METRIC, "value": value,
+            "metric": METRICS.get(kind, METRIC), "value": value,
             "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",

@@ -596,6 +596,16 @@ def gdn_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):
     return torch.empty(need.value, dtype=torch.uint8, device=device) if need.value else None
 
 
+def gdn_bwd_workspace(B, T, H, Dk, Dv, device, dtype=torch.bfloat16, **kw):
+    """Allocate the workspace ccq_gdn_bwd needs for these sizes (None if none)."""
+    p = params(**kw)
+    need = ctypes.c_size_t(0)
+    code = BF16 if dtype == torch.bfloat16 else FP32
+    _check(load_library().ccq_gdn_bwd_workspace_size(B, T, H, Dk, Dv, code, ctypes.byref(p),
+                                                      ctypes.byref(need)))
+    return torch.empty(need.value, dtype=torch.uint8, device=device) if need.value else None
+
+
 def decode_step(backbone: int, q, k, v, gate, lam, state: CCQState, beta=None, *,
                 out=None, stream=None, **kw):
     """One recurrent token (Algorithm 2): q, k [B,H,Dk], v [B,H,Dv]; gate

@@ -127,6 +127,72 @@ __device__ __forceinline__ void gate_prefix(const float *graw, float *gc) {
     }
 }
 
+// Load the rows of chunk r of a [B][T][H][D] tensor into dst[64][ld] (zero past T).
+template <int D, typename Tin>
+__device__ __forceinline__ void load_tile_ld(float *dst, int ld, const void *src, const GdnBwdArgs &a, int b, int h,
+                                             int r) {
+    const Tin *s = static_cast<const Tin *>(src);
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, c = idx % D, t = r * kC + i;
+        dst[i * ld + c] = t < a.T ? to_f(s[tok_row(a, b, t, h) * D + c]) : 0.f;
+    }
+}
+
+// dst[rows][ld] <- src[rows][sld] (fp32, e.g. a workspace tile into shared memory).
+__device__ __forceinline__ void copy_rows(float *dst, int ld, const float *src, int sld, int rows, int cols) {
+    GBWD_FOR(idx, rows * cols) {
+        const int i = idx / cols, c = idx % cols;
+        dst[i * ld + c] = src[i * sld + c];
+    }
+}
+
+// row_rnorm over a [64][ld] tile.
+template <int D>
+__device__ __forceinline__ void row_rnorm_ld(const float *x, int ld, float *rn, int l2norm) {
+    GBWD_FOR(i, kC) {
+        float ss = 0.f;
+        for (int c = 0; c < D; ++c) ss += x[i * ld + c] * x[i * ld + c];
+        rn[i] = !l2norm ? 1.f : (ss > 0.f ? 1.f / sqrtf(fmaxf(ss, 1e-12f)) : 0.f);
+    }
+}
+
+// Register-tiled product of two operands in shared memory, computed by 256 virtual threads
+// (the CTA's threads stride over them) of TM x TN outputs each:
+//   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   m < 16 TM, n < 16 TN,
+// virtual thread (tm, tn) holding rows tm + 16 i and columns tn + 16 j, so that a warp's loads
+// of B for one j are 16 consecutive columns and its loads of A two rows (broadcasts); a B
+// column stride bcs and an A row stride ars that are odd (or 1) keep them free of bank
+// conflicts.  ep(m, n, value) consumes every output once, in the thread that computed it.
+template <int TM, int TN, typename Ep>
+__device__ __forceinline__ void tile_mm(const float *A, int ars, int acs, const float *B, int brs, int bcs, int K,
+                                        Ep ep) {
+    for (int vt = static_cast<int>(threadIdx.x); vt < 256; vt += static_cast<int>(blockDim.x)) {
+        const int tm = vt >> 4, tn = vt & 15;
+        float acc[TM][TN];
+#pragma unroll
+        for (int i = 0; i < TM; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) acc[i][j] = 0.f;
+        const float *a0 = A + tm * ars, *b0 = B + tn * bcs;
+#pragma unroll 2
+        for (int k = 0; k < K; ++k) {
+            float av[TM], bv[TN];
+#pragma unroll
+            for (int i = 0; i < TM; ++i) av[i] = a0[16 * i * ars + k * acs];
+#pragma unroll
+            for (int j = 0; j < TN; ++j) bv[j] = b0[k * brs + 16 * j * bcs];
+#pragma unroll
+            for (int i = 0; i < TM; ++i)
+#pragma unroll
+                for (int j = 0; j < TN; ++j) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+        }
+#pragma unroll
+        for (int i = 0; i < TM; ++i)
+#pragma unroll
+            for (int j = 0; j < TN; ++j) ep(tm + 16 * i, tn + 16 * j, acc[i][j]);
+    }
+}
+
 // ---------------------------------------------------------------------------------------------
 // Per chunk: Tt = (I + A)^{-1} by forward substitution, and the chunk's key statistics.
 template <int D, typename Tin>
@@ -648,18 +714,25 @@ __global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a)
 
 // Per chunk: dv, dk, dbeta, dg from the chunk's forward quantities (gdn_bwd_local_kernel),
 // the entering state H_r, the adjoint dH of the leaving state, and DC_{r+1}, Dm_{r+1}.
+// Every product runs as a register-tiled tile_mm over shared-memory operands; the [64][D]
+// tiles have the odd row stride D + 1 and the [64][64] ones 65, and the workspace operands
+// are staged through BF (and, for the D x D ones, 64 rows at a time through the S/dP pair).
 template <int D, typename Tin>
 __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
+    constexpr int LD = D + 1, LC = kC + 1, TD = D / 16;
+    constexpr int RB = D < 64 ? D : 64, NH = D / RB, TR = RB / 16;  // row blocks of the D x D operands
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *Kb = sm;                // [64][D]
-    float *dU = Kb + kC * D;       // [64][D]
-    float *dR = dU + kC * D;       // [64][D]
-    float *dK = dR + kC * D;       // [64][D]
-    float *sA = dK + kC * D;       // [64][64] S, then dTb, then dA, then (Qbar Kbar^T) o causal
-    float *sB = sA + kC * kC;      // [64][64] dP, then M2, then dKK, then (W Kbar^T) o causal
-    float *Tt = sB + kC * kC;      // [64][64]
-    float *graw = Tt + kC * kC;
+    float *Kb = sm;                // [64][LD] kbar
+    float *dU = Kb + kC * LD;      // [64][LD] dU, then the reverse sums of dCum
+    float *dR = dU + kC * LD;      // [64][LD] dR, then W
+    float *dK = dR + kC * LD;      // [64][LD] dkbar (accumulated)
+    float *BF = dK + kC * LD;      // [64][LD] staging: Qc, D, U, R, Qbar, DC + DC^T
+    float *sA = BF + kC * LD;      // [64][LC] S, then dTb, then dA, then (Qbar Kbar^T) o causal
+    float *sB = sA + kC * LC;      // [64][LC] dP, then M2, then dKK, then (W Kbar^T) o causal
+    float *B2 = sA;                // sA and sB together: [64][LD] staging of 64 rows of dH or H
+    float *Tt = sB + kC * LC;      // [64][LC]
+    float *graw = Tt + kC * LC;
     float *gc = graw + kC, *E = gc + kC, *ed = E + kC, *be = ed + kC, *tinv = be + kC;
     float *rk = tinv + kC, *prs = rk + kC, *pcs = prs + kC, *kd = pcs + kC, *gkh = kd + kC;
     float *rs = gkh + kC, *cs = rs + kC, *db1 = cs + kC, *rdot = db1 + kC, *dgc = rdot + kC;
@@ -681,12 +754,9 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     const Tin *dout = static_cast<const Tin *>(a.dout);
     const Tin *vin = static_cast<const Tin *>(a.v);
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
-    auto Dsc = [&](int i, int col) -> float {
-        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + col]) : 0.f;
-    };
 
-    load_tile<D, Tin>(Kb, a.k, a, b, h, r);
-    GBWD_FOR(idx, kC * kC) Tt[idx] = ttg[idx];
+    load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
+    GBWD_FOR(idx, kC * kC) Tt[(idx / kC) * LC + idx % kC] = ttg[idx];
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -696,75 +766,66 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         prs[i] = pcs[i] = kd[i] = gkh[i] = rs[i] = cs[i] = 0.f;
     }
     if (threadIdx.x == 0) scal[0] = 0.f;
+    copy_rows(BF, LD, Qcg, D, kC, D);
     __syncthreads();
-    row_rnorm<D>(Kb, rk, a.l2norm);
+    row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
     gate_prefix(graw, gc);
     __syncthreads();
-    GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+    GBWD_FOR(idx, kC * D) Kb[(idx / D) * LD + idx % D] *= rk[idx / D];
     GBWD_FOR(i, kC) {
         E[i] = expf(gc[i]);
         ed[i] = expf(gc[kC - 1] - gc[i]);
     }
     __syncthreads();
-    // S = Qc Kbar^T;  dU = P^T D + Kd dH
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += Qcg[i * D + l] * Kb[j * D + l];
-        sA[idx] = acc;
+    // dU = P^T D + Kd dH = X1 + diag(ed) Kbar dH, over the row blocks of dH
+    for (int hf = 0; hf < NH; ++hf) {
+        __syncthreads();
+        copy_rows(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, D, RB, D);
+        __syncthreads();
+        tile_mm<4, TD>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) {
+            dU[i * LD + j] = (hf ? dU[i * LD + j] : 0.f) + v;
+        });
     }
+    __syncthreads();
+    // S = Qc Kbar^T (Qc in BF; S in the S/dP pair, free once the staging of dH is read)
+    tile_mm<4, 4>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     GBWD_FOR(idx, kC * D) {
         const int i = idx / D, j = idx % D;
-        float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * dHg[l * D + j];
-        dU[idx] = X1[idx] + ed[i] * acc;
+        dU[i * LD + j] = X1[idx] + ed[i] * dU[i * LD + j];
+    }
+    __syncthreads();
+    // D (scaled output adjoint) and U for dP
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        BF[i * LD + j] = i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + j]) : 0.f;
+        dK[i * LD + j] = Ug[idx];
     }
     __syncthreads();
     // dv = dR = diag(beta) Tt^T dU;  dP = (D U^T) o Gamma o causal
     {
         Tin *dv = static_cast<Tin *>(a.dv);
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
-            float acc = 0.f;
-            for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * dU[l * D + j];
-            acc *= be[i];
-            dR[idx] = acc;
-            if (i < n) dv[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(acc);
-        }
-        GBWD_FOR(idx, kC * kC) {
-            const int i = idx / kC, j = idx % kC;
-            float acc = 0.f;
-            if (j <= i && i < n) {
-                for (int l = 0; l < D; ++l) acc += Dsc(i, l) * Ug[j * D + l];
-                acc *= expf(gc[i] - gc[j]);
-            }
-            sB[idx] = acc;
-        }
+        tile_mm<4, TD>(Tt, 1, LC, dU, LD, 1, kC, [&](int i, int j, float v) {
+            const float x = be[i] * v;
+            dR[i * LD + j] = x;
+            if (i < n) dv[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(x);
+        });
+        tile_mm<4, 4>(BF, LD, 1, dK, 1, LD, D, [&](int i, int j, float v) {
+            sB[i * LC + j] = (j <= i && i < n) ? v * expf(gc[i] - gc[j]) : 0.f;
+        });
     }
     __syncthreads();
-    // dK = dP^T Qc + diag(e^{gc_last - gc}) U dH^T - diag(E) dR H^T;  row and column sums of
-    // dP o S;  kd_i = rowsum(Kd o U dH^T)_i = U_i . (dU - P^T D)_i;  gkh_i = E_i (Kbar H)_i . dR_i
-    // = (V - R)_i . dR_i;  <dH, H>
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float acc = 0.f, udh = 0.f, drh = 0.f;
-        for (int l = i; l < kC; ++l) acc += sB[l * kC + i] * Qcg[l * D + j];
-        for (int l = 0; l < D; ++l) {
-            udh += Ug[i * D + l] * dHg[j * D + l];
-            drh += dR[i * D + l] * H[j * D + l];
-        }
-        dK[idx] = acc + ed[i] * udh - E[i] * drh;
-    }
+    // row and column sums of dP o S;  kd_i = U_i . (dU - P^T D)_i;  gkh_i = (V - R)_i . dR_i;
+    // <dH, H>;  Qc staged for dP^T Qc
     GBWD_FOR(i, kC) {
         float p = 0.f, q = 0.f, x = 0.f, y = 0.f;
         for (int j = 0; j < kC; ++j) {
-            p += sB[i * kC + j] * sA[i * kC + j];
-            q += sB[j * kC + i] * sA[j * kC + i];
+            p += sB[i * LC + j] * sA[i * LC + j];
+            q += sB[j * LC + i] * sA[j * LC + i];
         }
         for (int l = 0; l < D; ++l) {
-            x += Ug[i * D + l] * (dU[i * D + l] - X1[i * D + l]);
+            x += dK[i * LD + l] * (dU[i * LD + l] - X1[i * D + l]);
             const float vv = i < n ? to_f(vin[tok_row(a, b, r * kC + i, h) * D + l]) : 0.f;
-            y += (vv - Rg[i * D + l]) * dR[i * D + l];
+            y += (vv - Rg[i * D + l]) * dR[i * LD + l];
         }
         prs[i] = p;
         pcs[i] = q;
@@ -777,89 +838,96 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         atomicAdd(&scal[0], acc);
     }
     __syncthreads();
-    // dTb = dU R^T
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += dU[i * D + l] * Rg[j * D + l];
-        sA[idx] = acc;
+    // dK = dP^T Qc + diag(ed) U dH^T - diag(E) dR H^T (the last two over row blocks of dH, H)
+    copy_rows(BF, LD, Qcg, D, kC, D);
+    __syncthreads();
+    tile_mm<4, TD>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] = v; });
+    __syncthreads();
+    copy_rows(BF, LD, Ug, D, kC, D);
+    for (int hf = 0; hf < NH; ++hf) {
+        __syncthreads();
+        copy_rows(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, D, RB, D);
+        __syncthreads();
+        tile_mm<4, TR>(BF, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
+        __syncthreads();
+        copy_rows(B2, LD, H + static_cast<size_t>(RB * hf) * D, D, RB, D);
+        __syncthreads();
+        tile_mm<4, TR>(dR, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
     }
+    __syncthreads();
+    copy_rows(BF, LD, Rg, D, kC, D);
+    __syncthreads();
+    // dTb = dU R^T
+    tile_mm<4, 4>(dU, LD, 1, BF, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     __syncthreads();
     // dbeta (the Tb = Tt diag(beta) factor) = column sums of dTb o Tt;  M2 = Tt^T (dTb diag(beta))
     GBWD_FOR(j, kC) {
         float acc = 0.f;
-        for (int i = 0; i < kC; ++i) acc += sA[i * kC + j] * Tt[i * kC + j];
+        for (int i = 0; i < kC; ++i) acc += sA[i * LC + j] * Tt[i * LC + j];
         db1[j] = acc;
     }
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * sA[l * kC + j];
-        sB[idx] = acc * be[j];
-    }
+    tile_mm<4, 4>(Tt, 1, LC, sA, LC, 1, kC, [&](int i, int j, float v) { sB[i * LC + j] = v * be[j]; });
     __syncthreads();
     // dA = strict_lower(-M2 Tt^T)
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        if (j < i)
-            for (int l = 0; l <= j; ++l) acc -= sB[i * kC + l] * Tt[j * kC + l];
-        sA[idx] = acc;
-    }
+    tile_mm<4, 4>(sB, LC, 1, Tt, 1, LC, kC, [&](int i, int j, float v) { sA[i * LC + j] = j < i ? -v : 0.f; });
     __syncthreads();
     // dKK = diag(beta) (dA o Gamma);  rs_i = sum_j dA_ij Gamma_ij KK_ij (the dbeta of A);
     // rowsum(dA o A)_i = beta_i rs_i;  cs_j = colsum(dA o A)_j
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
+    tile_mm<4, 4>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float kk) {
         float v = 0.f;
         if (j < i) {
-            float kk = 0.f;
-            for (int l = 0; l < D; ++l) kk += Kb[i * D + l] * Kb[j * D + l];
             const float gm = expf(gc[i] - gc[j]);
-            const float x = sA[idx] * gm * kk;
+            const float x = sA[i * LC + j] * gm * kk;
             atomicAdd(&rs[i], x);
             atomicAdd(&cs[j], be[i] * x);
-            v = sA[idx] * be[i] * gm;
+            v = sA[i * LC + j] * be[i] * gm;
         }
-        sB[idx] = v;
-    }
+        sB[i * LC + j] = v;
+    });
     __syncthreads();
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float acc = 0.f;
-        for (int l = 0; l < kC; ++l) acc += (sB[i * kC + l] + sB[l * kC + i]) * Kb[l * D + j];
-        dK[idx] += acc;
-    }
-    __syncthreads();
-    // CCQ terms: (Qbar Kbar^T) o causal and (W Kbar^T) o causal
     GBWD_FOR(idx, kC * kC) {
         const int i = idx / kC, j = idx % kC;
-        float x = 0.f, y = 0.f;
-        if (j <= i)
-            for (int l = 0; l < D; ++l) {
-                x += Qbg[i * D + l] * Kb[j * D + l];
-                y += Wg[i * D + l] * Kb[j * D + l];
-            }
-        sA[idx] = x;
-        sB[idx] = y;
+        sA[i * LC + j] = sB[i * LC + j] + sB[j * LC + i];
     }
     __syncthreads();
-    // dK += QKc^T W + WKc^T Qbar + Kbar (DC + DC^T) + Dm + reverse cumsum of dCum,
-    // dCum_l = -c (dz_l cq_l + qbar_l cz_l) / t_l^2, dz_l = t_l W_l
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float acc = Dm[j];
-        for (int l = i; l < kC; ++l) {
-            acc += sA[l * kC + i] * Wg[l * D + j] + sB[l * kC + i] * Qbg[l * D + j];
-            acc -= c * (Wg[l * D + j] * cq[l] / tinv[l] + Qbg[l * D + j] * cz[l]) * tinv[l] * tinv[l];
+    // dK += (dKK + dKK^T) Kbar
+    tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+    __syncthreads();
+    // CCQ terms: (Qbar Kbar^T) o causal and (W Kbar^T) o causal
+    copy_rows(BF, LD, Qbg, D, kC, D);
+    copy_rows(dR, LD, Wg, D, kC, D);
+    __syncthreads();
+    tile_mm<4, 4>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
+    tile_mm<4, 4>(dR, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
+    // reverse cumulative sums G_ij = sum_{l>=i} dCum_lj / (-c), dCum_l = -c (dz_l cq_l + qbar_l cz_l) / t_l^2,
+    // dz_l = t_l W_l
+    GBWD_FOR(j, D) {
+        float acc = 0.f;
+        for (int l = kC - 1; l >= 0; --l) {
+            acc += (dR[l * LD + j] * cq[l] / tinv[l] + BF[l * LD + j] * cz[l]) * tinv[l] * tinv[l];
+            dU[l * LD + j] = acc;
         }
-        for (int p = 0; p < D; ++p) acc += Kb[i * D + p] * (DC[p * D + j] + DC[j * D + p]);
-        dK[idx] += acc;
+    }
+    __syncthreads();
+    // dK += QKc^T W + WKc^T Qbar + Dm - c G
+    tile_mm<4, TD>(sA, 1, LC, dR, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+    tile_mm<4, TD>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) {
+        dK[i * LD + j] += v + Dm[j] - c * dU[i * LD + j];
+    });
+    // dK += Kbar (DC + DC^T), over the row blocks p of DC
+    for (int hf = 0; hf < NH; ++hf) {
+        __syncthreads();
+        GBWD_FOR(idx, RB * D) {
+            const int p = idx / D, j = idx % D, pg = RB * hf + p;
+            B2[p * LD + j] = DC[pg * D + j] + DC[j * D + pg];
+        }
+        __syncthreads();
+        tile_mm<4, TD>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     }
     __syncthreads();
     GBWD_FOR(i, kC) {
         float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += Kb[i * D + j] * dK[i * D + j];
+        for (int j = 0; j < D; ++j) acc += Kb[i * LD + j] * dK[i * LD + j];
         rdot[i] = a.l2norm ? acc : 0.f;
         float x = be[i] * rs[i] - cs[i] + prs[i] - pcs[i] + gqh[i] - kd[i] - gkh[i];
         if (i == n - 1) {
@@ -882,7 +950,8 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         Tin *dk = static_cast<Tin *>(a.dk);
         GBWD_FOR(idx, kC * D) {
             const int i = idx / D, j = idx % D;
-            if (i < n) dk[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((dK[idx] - Kb[idx] * rdot[i]) * rk[i]);
+            if (i < n)
+                dk[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((dK[i * LD + j] - Kb[i * LD + j] * rdot[i]) * rk[i]);
         }
     }
 }
@@ -904,7 +973,9 @@ inline int seq_split(int B, int H) {
     while (ns < 4 && static_cast<long long>(B) * H * ns * 2 <= 304) ns *= 2;
     return ns;
 }
-template <int D> constexpr size_t kv_smem() { return sizeof(float) * (4 * kC * D + 3 * kC * kC + 16 * kC + 4); }
+template <int D> constexpr size_t kv_smem() {
+    return sizeof(float) * (5 * kC * (D + 1) + 3 * kC * (kC + 1) + 16 * kC + 4);
+}
 
 }  // namespace gbwd
 }  // namespace ccq
