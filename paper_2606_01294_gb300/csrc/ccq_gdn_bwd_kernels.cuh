@@ -127,23 +127,39 @@ __device__ __forceinline__ void gate_prefix(const float *graw, float *gc) {
     }
 }
 
+// An element-wise pass over total elements whose loads come from global memory: the thread's
+// elements go eight at a time, all eight loads issued before the first store, so that a thread
+// keeps eight loads in flight instead of one.  ld(e) loads element e, st(e, x) stores it.
+template <typename L, typename S>
+__device__ __forceinline__ void stream8(int total, L ld, S st) {
+    const int stride = static_cast<int>(blockDim.x);
+    int idx = static_cast<int>(threadIdx.x);
+    for (; idx + 7 * stride < total; idx += 8 * stride) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = ld(idx + u * stride);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) st(idx + u * stride, x[u]);
+    }
+    for (; idx < total; idx += stride) st(idx, ld(idx));
+}
+
 // Load the rows of chunk r of a [B][T][H][D] tensor into dst[64][ld] (zero past T).
 template <int D, typename Tin>
 __device__ __forceinline__ void load_tile_ld(float *dst, int ld, const void *src, const GdnBwdArgs &a, int b, int h,
                                              int r) {
     const Tin *s = static_cast<const Tin *>(src);
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, c = idx % D, t = r * kC + i;
-        dst[i * ld + c] = t < a.T ? to_f(s[tok_row(a, b, t, h) * D + c]) : 0.f;
-    }
+    stream8(kC * D, [&](int idx) {
+        const int t = r * kC + idx / D;
+        return t < a.T ? to_f(s[tok_row(a, b, t, h) * D + idx % D]) : 0.f;
+    }, [&](int idx, float x) { dst[(idx / D) * ld + idx % D] = x; });
 }
 
-// dst[rows][ld] <- src[rows][sld] (fp32, e.g. a workspace tile into shared memory).
-__device__ __forceinline__ void copy_rows(float *dst, int ld, const float *src, int sld, int rows, int cols) {
-    GBWD_FOR(idx, rows * cols) {
-        const int i = idx / cols, c = idx % cols;
-        dst[i * ld + c] = src[i * sld + c];
-    }
+// dst[rows][ld] <- src[rows][COLS] (fp32, e.g. a workspace tile into shared memory).
+template <int COLS>
+__device__ __forceinline__ void copy_rows(float *dst, int ld, const float *src, int rows) {
+    stream8(rows * COLS, [&](int idx) { return src[idx]; },
+            [&](int idx, float x) { dst[(idx / COLS) * ld + idx % COLS] = x; });
 }
 
 // row_rnorm over a [64][ld] tile.
@@ -274,7 +290,19 @@ __global__ void __launch_bounds__(256) gdn_bwd_prefix_kernel(const GdnBwdArgs a)
     float acc = 0.f;
     if (isC && a.C0) acc = a.C0[static_cast<size_t>(bh) * D * D + e];
     if (!isC && a.m0) acc = a.m0[static_cast<size_t>(bh) * D + (e - D * D)];
-    for (int r = 0; r < a.NC; ++r) {
+    // eight chunks' loads in flight before their stores
+    int r = 0;
+    for (; r + 8 <= a.NC; r += 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = base[(r + u) * stride];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            base[(r + u) * stride] = acc;
+            acc += x[u];
+        }
+    }
+    for (; r < a.NC; ++r) {
         const float x = base[r * stride];
         base[r * stride] = acc;
         acc += x;
@@ -362,39 +390,45 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
 }
 
 // Per chunk, everything that does not need dH: z, qc, R, U, dqc, dq, dlambda, the CCQ
-// increments of DC and Dm, P^T D and (diag(E) Qc)^T D.
+// increments of DC and Dm, P^T D and (diag(E) Qc)^T D.  Products as in gdn_bwd_kv_kernel
+// (tile_mm over [64][D + 1] and [64][65] tiles); the D x D operands H and S^K are staged a row
+// block at a time through a tile that is free at that point, and z waits in the W slot of the
+// workspace while its tile holds D.
 template <int D, typename Tin>
 __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
+    constexpr int LD = D + 1, LC = kC + 1, TD = D / 16;
+    constexpr int RB = D < 64 ? D : 64, NH = D / RB;      // row blocks of 64 (k-blocks)
+    constexpr int RN = D < 32 ? D : 32, NN = D / RN;      // row blocks of 32 (n-blocks, in sB)
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *Qb = sm;                // [64][D] qbar
-    float *Kb = Qb + kC * D;       // [64][D] kbar
-    float *Rq = Kb + kC * D;       // [64][D] V, then R, then qc
-    float *Zw = Rq + kC * D;       // [64][D] z, then W
-    float *Ud = Zw + kC * D;       // [64][D] U, then dqc, then dqbar
-    float *sA = Ud + kC * D;       // [64][64] (Qbar Kbar^T) o causal, then dP
-    float *sB = sA + kC * kC;      // [64][64] P, then (W Kbar^T) o causal
-    float *graw = sB + kC * kC;
+    float *Qb = sm;                // [64][LD] qbar
+    float *Kb = Qb + kC * LD;      // [64][LD] kbar
+    float *Rq = Kb + kC * LD;      // [64][LD] V, then R, then S^K blocks, then qc, then S^K blocks
+    float *Zw = Rq + kC * LD;      // [64][LD] H blocks, then z, then D (scaled by E), then W
+    float *Ud = Zw + kC * LD;      // [64][LD] U, then dqc, then dqbar
+    float *sA = Ud + kC * LD;      // [64][LC] (Qbar Kbar^T) o causal, then dP
+    float *sB = sA + kC * LC;      // [64][LC] Tt diag(beta), then P, then H blocks, then (W Kbar^T) o causal
+    float *graw = sB + kC * LC;
     float *gc = graw + kC, *E = gc + kC, *be = E + kC, *lam = be + kC, *tinv = lam + kC;
     float *rq = tinv + kC, *rk = rq + kC, *cq = rk + kC, *cz = cq + kC, *gqh = cz + kC;
     float *rdot = gqh + kC;
+    float *M = rdot + kC;          // [D] the key sum M_r entering the chunk
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
     const int n = min(kC, a.T - r * kC);
     const float c = a.centered ? 1.f : 0.f;
     const float *H = a.hs + static_cast<size_t>(ch) * D * D;
     const float *SK = a.sk + static_cast<size_t>(ch) * D * D;
-    const float *M = a.mk + static_cast<size_t>(ch) * D;
+    const float *Mg = a.mk + static_cast<size_t>(ch) * D;
     const float *Tt = a.tt + static_cast<size_t>(ch) * kC * kC;
+    const size_t t64 = static_cast<size_t>(ch) * kC * D;
+    float *Wg = a.w + t64;
     const Tin *dout = static_cast<const Tin *>(a.dout);
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
-    auto Dsc = [&](int i, int col) -> float {
-        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + col]) : 0.f;
-    };
 
-    load_tile<D, Tin>(Qb, a.q, a, b, h, r);
-    load_tile<D, Tin>(Kb, a.k, a, b, h, r);
-    load_tile<D, Tin>(Rq, a.v, a, b, h, r);
+    load_tile_ld<D, Tin>(Qb, LD, a.q, a, b, h, r);
+    load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
+    load_tile_ld<D, Tin>(Rq, LD, a.v, a, b, h, r);
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -404,189 +438,169 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
         tinv[i] = 1.f / (t_start + 1.f + static_cast<float>(i));
         gqh[i] = 0.f;
     }
+    GBWD_FOR(j, D) M[j] = Mg[j];
     __syncthreads();
-    row_rnorm<D>(Qb, rq, a.l2norm);
-    row_rnorm<D>(Kb, rk, a.l2norm);
+    row_rnorm_ld<D>(Qb, LD, rq, a.l2norm);
+    row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
     gate_prefix(graw, gc);
     __syncthreads();
     GBWD_FOR(idx, kC * D) {
-        Qb[idx] *= rq[idx / D];
-        Kb[idx] *= rk[idx / D];
+        const int i = idx / D, j = idx % D;
+        Qb[i * LD + j] *= rq[i];
+        Kb[i * LD + j] *= rk[i];
     }
     GBWD_FOR(i, kC) E[i] = expf(gc[i]);
+    // Tt diag(beta) for U (be is visible after the barrier above)
+    stream8(kC * kC, [&](int idx) { return Tt[idx]; },
+            [&](int idx, float x) { sB[(idx / kC) * LC + idx % kC] = x * be[idx % kC]; });
     __syncthreads();
-    // (Qbar Kbar^T) o causal;  R = V - diag(E) Kbar H
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        if (j <= i)
-            for (int l = 0; l < D; ++l) acc += Qb[i * D + l] * Kb[j * D + l];
-        sA[idx] = acc;
-    }
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * H[l * D + j];
-        Rq[idx] -= E[i] * acc;
+    // (Qbar Kbar^T) o causal;  R = V - diag(E) Kbar H over the row blocks of H
+    tile_mm<4, 4>(Qb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
+    for (int hf = 0; hf < NH; ++hf) {
+        __syncthreads();
+        copy_rows<D>(Zw, LD, H + static_cast<size_t>(RB * hf) * D, RB);
+        __syncthreads();
+        tile_mm<4, TD>(Kb + RB * hf, LD, 1, Zw, LD, 1, RB, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
     }
     __syncthreads();
     // cq_i = CumK_i . qbar_i with CumK_i = M + sum_{j<=i} kbar_j;  U = Tt diag(beta) R
     GBWD_FOR(i, kC) {
         float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += M[l] * Qb[i * D + l];
-        for (int j = 0; j <= i; ++j) acc += sA[i * kC + j];
+        for (int l = 0; l < D; ++l) acc += M[l] * Qb[i * LD + l];
+        for (int j = 0; j <= i; ++j) acc += sA[i * LC + j];
         cq[i] = acc;
     }
     {
-        float *Rg = a.r + static_cast<size_t>(ch) * kC * D;
-        float *Ug = a.u + static_cast<size_t>(ch) * kC * D;
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
-            float acc = 0.f;
-            for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * Rq[l * D + j];
-            Ud[idx] = acc;
-            Ug[idx] = acc;
-            Rg[idx] = Rq[idx];
-        }
+        float *Rg = a.r + t64;
+        float *Ug = a.u + t64;
+        tile_mm<4, TD>(sB, LC, 1, Rq, LD, 1, kC, [&](int i, int j, float v) {
+            Ud[i * LD + j] = v;
+            Ug[i * D + j] = v;
+        });
+        GBWD_FOR(idx, kC * D) Rg[idx] = Rq[(idx / D) * LD + idx % D];
+    }
+    // z = Sigma_t qbar (App. B form): (Qbar S^K + ((Qbar Kbar^T) o causal) Kbar) / t - c CumK cq / t^2
+    __syncthreads();
+    tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
+    for (int hf = 0; hf < NH; ++hf) {
+        __syncthreads();
+        copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
+        __syncthreads();
+        tile_mm<4, TD>(Qb + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
     }
     __syncthreads();
-    // z = Sigma_t qbar (App. B form): (Qbar S^K + ((Qbar Kbar^T) o causal) Kbar) / t - c CumK cq / t^2
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float acc = 0.f, cum = M[j];
-        for (int l = 0; l < D; ++l) acc += Qb[i * D + l] * SK[l * D + j];
-        for (int l = 0; l <= i; ++l) {
-            acc += sA[i * kC + l] * Kb[l * D + j];
-            cum += Kb[l * D + j];
+    GBWD_FOR(j, D) {
+        float cum = M[j];
+        for (int i = 0; i < kC; ++i) {
+            cum += Kb[i * LD + j];
+            const float z = Zw[i * LD + j] * tinv[i] - c * cum * cq[i] * tinv[i] * tinv[i];
+            Zw[i * LD + j] = z;
+            Wg[i * D + j] = z;  // z waits in the W slot until dlambda
         }
-        Zw[idx] = acc * tinv[i] - c * cum * cq[i] * tinv[i] * tinv[i];
     }
     __syncthreads();
     // qc = qbar - lambda z (Eq. clean)
     {
-        float *Qg = a.qb + static_cast<size_t>(ch) * kC * D;
-        float *Qcg = a.qc + static_cast<size_t>(ch) * kC * D;
-        GBWD_FOR(idx, kC * D) {
-            const float v = Qb[idx] - lam[idx / D] * Zw[idx];
-            Rq[idx] = v;
-            Qcg[idx] = v;
-            Qg[idx] = Qb[idx];
-        }
-    }
-    __syncthreads();
-    // P = (Qc Kbar^T) o Gamma o causal
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        if (j <= i) {
-            for (int l = 0; l < D; ++l) acc += Rq[i * D + l] * Kb[j * D + l];
-            acc *= expf(gc[i] - gc[j]);
-        }
-        sB[idx] = acc;
-    }
-    __syncthreads();
-    // P^T D and (diag(E) Qc)^T D for the state pass;  dP = (D U^T) o Gamma o causal
-    {
-        float *X1 = a.x1 + static_cast<size_t>(ch) * kC * D;
-        float *Y1 = a.y1 + static_cast<size_t>(ch) * D * D;
+        float *Qg = a.qb + t64;
+        float *Qcg = a.qc + t64;
         GBWD_FOR(idx, kC * D) {
             const int i = idx / D, j = idx % D;
-            float acc = 0.f;
-            for (int l = i; l < n; ++l) acc += sB[l * kC + i] * Dsc(l, j);
-            X1[idx] = acc;
-        }
-        GBWD_FOR(idx, D * D) {
-            const int p = idx / D, j = idx % D;
-            float acc = 0.f;
-            for (int i = 0; i < n; ++i) acc += E[i] * Rq[i * D + p] * Dsc(i, j);
-            Y1[idx] = acc;
-        }
-        GBWD_FOR(idx, kC * kC) {
-            const int i = idx / kC, j = idx % kC;
-            float acc = 0.f;
-            if (j <= i && i < n) {
-                for (int l = 0; l < D; ++l) acc += Dsc(i, l) * Ud[j * D + l];
-                acc *= expf(gc[i] - gc[j]);
-            }
-            sA[idx] = acc;
+            const float v = Qb[i * LD + j] - lam[i] * Zw[i * LD + j];
+            Rq[i * LD + j] = v;
+            Qcg[idx] = v;
+            Qg[idx] = Qb[i * LD + j];
         }
     }
     __syncthreads();
-    // dqc = diag(E) D H^T + dP Kbar  (into Ud; U is no longer needed here);
-    // gqh_i = E_i rowsum((Qc H) o D)_i = E_i sum_j qc_ij (D H^T)_ij
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        float dh = 0.f;
-        for (int l = 0; l < D; ++l) dh += Dsc(i, l) * H[j * D + l];
-        float acc = E[i] * dh;
-        for (int l = 0; l <= i; ++l) acc += sA[i * kC + l] * Kb[l * D + j];
-        Ud[idx] = acc;
-        if (i < n) atomicAdd(&gqh[i], E[i] * Rq[idx] * dh);
+    // P = (Qc Kbar^T) o Gamma o causal;  D (the scaled output adjoint) into z's tile
+    tile_mm<4, 4>(Rq, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) {
+        sB[i * LC + j] = j <= i ? v * expf(gc[i] - gc[j]) : 0.f;
+    });
+    stream8(kC * D, [&](int idx) {
+        const int i = idx / D;
+        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + idx % D]) : 0.f;
+    }, [&](int idx, float x) { Zw[(idx / D) * LD + idx % D] = x; });
+    __syncthreads();
+    // P^T D for the state pass;  dP = (D U^T) o Gamma o causal
+    {
+        float *X1 = a.x1 + t64;
+        tile_mm<4, TD>(sB, 1, LC, Zw, LD, 1, kC, [&](int i, int j, float v) { X1[i * D + j] = v; });
+        tile_mm<4, 4>(Zw, LD, 1, Ud, 1, LD, D, [&](int i, int j, float v) {
+            sA[i * LC + j] = (j <= i && i < n) ? v * expf(gc[i] - gc[j]) : 0.f;
+        });
     }
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) Zw[(idx / D) * LD + idx % D] *= E[idx / D];  // diag(E) D
+    __syncthreads();
+    // (diag(E) Qc)^T D = Qc^T (diag(E) D) for the state pass;  dqc = dP Kbar + (diag(E) D) H^T
+    // (over row blocks of H in sB);  gqh_i = E_i rowsum((Qc H) o D)_i = sum_j qc_ij ((E D) H^T)_ij
+    {
+        float *Y1 = a.y1 + static_cast<size_t>(ch) * D * D;
+        tile_mm<TD, TD>(Rq, 1, LD, Zw, LD, 1, kC, [&](int p, int j, float v) { Y1[p * D + j] = v; });
+        tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] = v; });
+    }
+    for (int nb = 0; nb < NN; ++nb) {
+        __syncthreads();
+        copy_rows<D>(sB, LD, H + static_cast<size_t>(RN * nb) * D, RN);
+        __syncthreads();
+        tile_mm<4, RN / 16>(Zw, LD, 1, sB, 1, LD, D, [&](int i, int j, float v) {
+            const int jg = RN * nb + j;
+            Ud[i * LD + jg] += v;
+            if (i < n) atomicAdd(&gqh[i], Rq[i * LD + jg] * v);
+        });
+    }
+    __syncthreads();
+    copy_rows<D>(Zw, LD, Wg, kC);  // z back from the W slot
     __syncthreads();
     // dlambda_i = -z_i . dqc_i
     GBWD_FOR(i, kC) {
         float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += Zw[i * D + j] * Ud[i * D + j];
+        for (int j = 0; j < D; ++j) acc += Zw[i * LD + j] * Ud[i * LD + j];
         if (i < n && a.dlambda) a.dlambda[tok_row(a, b, r * kC + i, h)] = -acc;
     }
     __syncthreads();
     // W = dz / t with dz = -lambda dqc
-    {
-        float *Wg = a.w + static_cast<size_t>(ch) * kC * D;
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D;
-            const float wv = -lam[i] * Ud[idx] * tinv[i];
-            Zw[idx] = wv;
-            Wg[idx] = wv;
-        }
+    GBWD_FOR(idx, kC * D) {
+        const int i = idx / D, j = idx % D;
+        const float wv = -lam[i] * Ud[i * LD + j] * tinv[i];
+        Zw[i * LD + j] = wv;
+        Wg[idx] = wv;
     }
     __syncthreads();
     // (W Kbar^T) o causal
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float acc = 0.f;
-        if (j <= i)
-            for (int l = 0; l < D; ++l) acc += Zw[i * D + l] * Kb[j * D + l];
-        sB[idx] = acc;
-    }
+    tile_mm<4, 4>(Zw, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     __syncthreads();
     // cz_i = CumK_i . dz_i = t_i (M . W_i + sum_{j<=i} W_i . kbar_j)
     GBWD_FOR(i, kC) {
         float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += M[l] * Zw[i * D + l];
-        for (int j = 0; j <= i; ++j) acc += sB[i * kC + j];
+        for (int l = 0; l < D; ++l) acc += M[l] * Zw[i * LD + l];
+        for (int j = 0; j <= i; ++j) acc += sB[i * LC + j];
         cz[i] = acc / tinv[i];
     }
-    __syncthreads();
     // dqbar = dqc + W S^K + ((W Kbar^T) o causal) Kbar - c CumK cz / t^2 (in place);
     // the chunk's increments DC += W^T Qbar and Dm += sum_i dCum_i,
     // dCum_i = -c (dz_i cq_i + qbar_i cz_i) / t_i^2
+    tile_mm<4, TD>(sB, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+    for (int hf = 0; hf < NH; ++hf) {
+        __syncthreads();
+        copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
+        __syncthreads();
+        tile_mm<4, TD>(Zw + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+    }
+    __syncthreads();
     {
         float *dC = a.dc + static_cast<size_t>(ch) * D * D;
         float *dM = a.dm + static_cast<size_t>(ch) * D;
-        GBWD_FOR(idx, kC * D) {
-            const int i = idx / D, j = idx % D;
-            float acc = 0.f, cum = M[j];
-            for (int l = 0; l < D; ++l) acc += Zw[i * D + l] * SK[l * D + j];
-            for (int l = 0; l <= i; ++l) {
-                acc += sB[i * kC + l] * Kb[l * D + j];
-                cum += Kb[l * D + j];
-            }
-            Ud[idx] += acc - c * cum * cz[i] * tinv[i] * tinv[i];
-        }
-        GBWD_FOR(idx, D * D) {
-            const int p = idx / D, j = idx % D;
-            float acc = 0.f;
-            for (int i = 0; i < kC; ++i) acc += Zw[i * D + p] * Qb[i * D + j];
-            dC[idx] = acc;
-        }
         GBWD_FOR(j, D) {
-            float acc = 0.f;
-            for (int i = 0; i < kC; ++i)
-                acc += (Zw[i * D + j] * cq[i] / tinv[i] + Qb[i * D + j] * cz[i]) * tinv[i] * tinv[i];
+            float cum = M[j], acc = 0.f;
+            for (int i = 0; i < kC; ++i) {
+                cum += Kb[i * LD + j];
+                Ud[i * LD + j] -= c * cum * cz[i] * tinv[i] * tinv[i];
+                acc += (Zw[i * LD + j] * cq[i] / tinv[i] + Qb[i * LD + j] * cz[i]) * tinv[i] * tinv[i];
+            }
             dM[j] = -c * acc;
         }
+        tile_mm<TD, TD>(Zw, 1, LD, Qb, LD, 1, kC, [&](int p, int j, float v) { dC[p * D + j] = v; });
         float *vec = a.vec + static_cast<size_t>(ch) * 4 * kC;
         GBWD_FOR(i, kC) {
             vec[i] = cq[i];
@@ -598,7 +612,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     __syncthreads();
     GBWD_FOR(i, kC) {
         float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += Qb[i * D + j] * Ud[i * D + j];
+        for (int j = 0; j < D; ++j) acc += Qb[i * LD + j] * Ud[i * LD + j];
         rdot[i] = a.l2norm ? acc : 0.f;
     }
     __syncthreads();
@@ -606,7 +620,8 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
         Tin *dq = static_cast<Tin *>(a.dq);
         GBWD_FOR(idx, kC * D) {
             const int i = idx / D, j = idx % D;
-            if (i < n) dq[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((Ud[idx] - Qb[idx] * rdot[i]) * rq[i]);
+            if (i < n)
+                dq[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((Ud[i * LD + j] - Qb[i * LD + j] * rdot[i]) * rq[i]);
         }
     }
 }
@@ -703,7 +718,19 @@ __global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a)
     float acc = 0.f;
     if (isC && a.dCT) acc = a.dCT[static_cast<size_t>(bh) * D * D + e];
     if (!isC && a.dmT) acc = a.dmT[static_cast<size_t>(bh) * D + em];
-    for (int r = a.NC - 1; r >= 0; --r) {
+    // eight chunks' loads in flight before their stores
+    int r = a.NC - 1;
+    for (; r - 7 >= 0; r -= 8) {
+        float x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) x[u] = base[(r - u) * stride];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            base[(r - u) * stride] = acc;
+            acc += x[u];
+        }
+    }
+    for (; r >= 0; --r) {
         const float x = base[r * stride];
         base[r * stride] = acc;
         acc += x;
@@ -756,7 +783,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
 
     load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
-    GBWD_FOR(idx, kC * kC) Tt[(idx / kC) * LC + idx % kC] = ttg[idx];
+    stream8(kC * kC, [&](int idx) { return ttg[idx]; }, [&](int idx, float x) { Tt[(idx / kC) * LC + idx % kC] = x; });
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -766,7 +793,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         prs[i] = pcs[i] = kd[i] = gkh[i] = rs[i] = cs[i] = 0.f;
     }
     if (threadIdx.x == 0) scal[0] = 0.f;
-    copy_rows(BF, LD, Qcg, D, kC, D);
+    copy_rows<D>(BF, LD, Qcg, kC);
     __syncthreads();
     row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
     gate_prefix(graw, gc);
@@ -780,7 +807,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     // dU = P^T D + Kd dH = X1 + diag(ed) Kbar dH, over the row blocks of dH
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
-        copy_rows(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, D, RB, D);
+        copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
         tile_mm<4, TD>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) {
             dU[i * LD + j] = (hf ? dU[i * LD + j] : 0.f) + v;
@@ -789,16 +816,26 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     __syncthreads();
     // S = Qc Kbar^T (Qc in BF; S in the S/dP pair, free once the staging of dH is read)
     tile_mm<4, 4>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
-    GBWD_FOR(idx, kC * D) {
+    // dU = X1 + diag(ed) t with t = Kbar dH, which also waits in dR for kd
+    stream8(kC * D, [&](int idx) { return X1[idx]; }, [&](int idx, float x) {
         const int i = idx / D, j = idx % D;
-        dU[i * LD + j] = X1[idx] + ed[i] * dU[i * LD + j];
-    }
+        const float t = dU[i * LD + j];
+        dR[i * LD + j] = t;
+        dU[i * LD + j] = x + ed[i] * t;
+    });
     __syncthreads();
     // D (scaled output adjoint) and U for dP
-    GBWD_FOR(idx, kC * D) {
-        const int i = idx / D, j = idx % D;
-        BF[i * LD + j] = i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + j]) : 0.f;
-        dK[i * LD + j] = Ug[idx];
+    stream8(kC * D, [&](int idx) {
+        const int i = idx / D;
+        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + idx % D]) : 0.f;
+    }, [&](int idx, float x) { BF[(idx / D) * LD + idx % D] = x; });
+    copy_rows<D>(dK, LD, Ug, kC);
+    __syncthreads();
+    // kd_i = rowsum(Kd o U dH^T)_i = U_i . (dU - P^T D)_i = ed_i U_i . t_i
+    GBWD_FOR(i, kC) {
+        float x = 0.f;
+        for (int l = 0; l < D; ++l) x += dK[i * LD + l] * dR[i * LD + l];
+        kd[i] = ed[i] * x;
     }
     __syncthreads();
     // dv = dR = diag(beta) Tt^T dU;  dP = (D U^T) o Gamma o causal
@@ -814,48 +851,49 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         });
     }
     __syncthreads();
-    // row and column sums of dP o S;  kd_i = U_i . (dU - P^T D)_i;  gkh_i = (V - R)_i . dR_i;
-    // <dH, H>;  Qc staged for dP^T Qc
+    // V - R (= diag(E) Kbar H) into BF for gkh;  <dH, H>
+    stream8(kC * D, [&](int idx) {
+        const int i = idx / D;
+        const float vv = i < n ? to_f(vin[tok_row(a, b, r * kC + i, h) * D + idx % D]) : 0.f;
+        return vv - Rg[idx];
+    }, [&](int idx, float x) { BF[(idx / D) * LD + idx % D] = x; });
+    {
+        float part = 0.f;
+        stream8(D * D, [&](int idx) { return dHg[idx] * H[idx]; }, [&](int, float x) { part += x; });
+        atomicAdd(&scal[0], part);
+    }
+    __syncthreads();
+    // row and column sums of dP o S;  gkh_i = (V - R)_i . dR_i
     GBWD_FOR(i, kC) {
-        float p = 0.f, q = 0.f, x = 0.f, y = 0.f;
+        float p = 0.f, q = 0.f, y = 0.f;
         for (int j = 0; j < kC; ++j) {
             p += sB[i * LC + j] * sA[i * LC + j];
             q += sB[j * LC + i] * sA[j * LC + i];
         }
-        for (int l = 0; l < D; ++l) {
-            x += dK[i * LD + l] * (dU[i * LD + l] - X1[i * D + l]);
-            const float vv = i < n ? to_f(vin[tok_row(a, b, r * kC + i, h) * D + l]) : 0.f;
-            y += (vv - Rg[i * D + l]) * dR[i * LD + l];
-        }
+        for (int l = 0; l < D; ++l) y += BF[i * LD + l] * dR[i * LD + l];
         prs[i] = p;
         pcs[i] = q;
-        kd[i] = x;
         gkh[i] = y;
-    }
-    GBWD_FOR(p, D) {
-        float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += dHg[p * D + j] * H[p * D + j];
-        atomicAdd(&scal[0], acc);
     }
     __syncthreads();
     // dK = dP^T Qc + diag(ed) U dH^T - diag(E) dR H^T (the last two over row blocks of dH, H)
-    copy_rows(BF, LD, Qcg, D, kC, D);
+    copy_rows<D>(BF, LD, Qcg, kC);
     __syncthreads();
     tile_mm<4, TD>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] = v; });
     __syncthreads();
-    copy_rows(BF, LD, Ug, D, kC, D);
+    copy_rows<D>(BF, LD, Ug, kC);
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
-        copy_rows(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, D, RB, D);
+        copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
         tile_mm<4, TR>(BF, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
         __syncthreads();
-        copy_rows(B2, LD, H + static_cast<size_t>(RB * hf) * D, D, RB, D);
+        copy_rows<D>(B2, LD, H + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
         tile_mm<4, TR>(dR, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
     }
     __syncthreads();
-    copy_rows(BF, LD, Rg, D, kC, D);
+    copy_rows<D>(BF, LD, Rg, kC);
     __syncthreads();
     // dTb = dU R^T
     tile_mm<4, 4>(dU, LD, 1, BF, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
@@ -894,8 +932,8 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     __syncthreads();
     // CCQ terms: (Qbar Kbar^T) o causal and (W Kbar^T) o causal
-    copy_rows(BF, LD, Qbg, D, kC, D);
-    copy_rows(dR, LD, Wg, D, kC, D);
+    copy_rows<D>(BF, LD, Qbg, kC);
+    copy_rows<D>(dR, LD, Wg, kC);
     __syncthreads();
     tile_mm<4, 4>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
     tile_mm<4, 4>(dR, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
@@ -961,7 +999,9 @@ template <int D> constexpr size_t prep_smem() { return sizeof(float) * (kC * D +
 template <int D> constexpr size_t fstate_smem(int ns) {
     return sizeof(float) * (D * (D / ns) + kC * D + 2 * kC * (D / ns) + kC * kC + 6 * kC);
 }
-template <int D> constexpr size_t local_smem() { return sizeof(float) * (5 * kC * D + 2 * kC * kC + 12 * kC); }
+template <int D> constexpr size_t local_smem() {
+    return sizeof(float) * (5 * kC * (D + 1) + 2 * kC * (kC + 1) + 12 * kC + D);
+}
 template <int D> constexpr size_t dstate_smem(int ns) {
     return sizeof(float) * (D * (D / ns) + kC * D + 2 * kC * (D / ns) + kC * kC + 6 * kC);
 }
