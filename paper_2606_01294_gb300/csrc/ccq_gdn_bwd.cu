@@ -22,23 +22,49 @@ cudaError_t allow_smem(K kernel, size_t bytes) {
     return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
 }
 
+// The sequential passes, instantiated per count of value-column blocks.
+template <int D, typename Tin, int NS>
+cudaError_t launch_fstate_ns(const gbwd::GdnBwdArgs &a, unsigned bh, cudaStream_t s) {
+    using namespace gbwd;
+    cudaError_t e = allow_smem(gdn_bwd_fstate_kernel<D, Tin, NS>, fstate_smem<D, NS>());
+    if (e != cudaSuccess) return e;
+    gdn_bwd_fstate_kernel<D, Tin, NS><<<bh * NS, 512, fstate_smem<D, NS>(), s>>>(a);
+    return cudaSuccess;
+}
+template <int D, typename Tin, int NS>
+cudaError_t launch_dstate_ns(const gbwd::GdnBwdArgs &a, unsigned bh, cudaStream_t s) {
+    using namespace gbwd;
+    cudaError_t e = allow_smem(gdn_bwd_dstate_kernel<D, Tin, NS>, dstate_smem<D, NS>());
+    if (e != cudaSuccess) return e;
+    gdn_bwd_dstate_kernel<D, Tin, NS><<<bh * NS, 512, dstate_smem<D, NS>(), s>>>(a);
+    return cudaSuccess;
+}
+template <int D, typename Tin>
+cudaError_t launch_fstate(const gbwd::GdnBwdArgs &a, unsigned bh, cudaStream_t s) {
+    return a.nsplit == 4 ? launch_fstate_ns<D, Tin, 4>(a, bh, s)
+         : a.nsplit == 2 ? launch_fstate_ns<D, Tin, 2>(a, bh, s) : launch_fstate_ns<D, Tin, 1>(a, bh, s);
+}
+template <int D, typename Tin>
+cudaError_t launch_dstate(const gbwd::GdnBwdArgs &a, unsigned bh, cudaStream_t s) {
+    return a.nsplit == 4 ? launch_dstate_ns<D, Tin, 4>(a, bh, s)
+         : a.nsplit == 2 ? launch_dstate_ns<D, Tin, 2>(a, bh, s) : launch_dstate_ns<D, Tin, 1>(a, bh, s);
+}
+
 template <int D, typename Tin>
 cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
     using namespace gbwd;
     cudaError_t e;
     if ((e = allow_smem(gdn_bwd_prep_kernel<D, Tin>, prep_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_fstate_kernel<D, Tin>, fstate_smem<D>(a.nsplit))) != cudaSuccess) return e;
     if ((e = allow_smem(gdn_bwd_local_kernel<D, Tin>, local_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_dstate_kernel<D, Tin>, dstate_smem<D>(a.nsplit))) != cudaSuccess) return e;
     if ((e = allow_smem(gdn_bwd_kv_kernel<D, Tin>, kv_smem<D>())) != cudaSuccess) return e;
     const unsigned nch = static_cast<unsigned>(a.B * a.H * a.NC), bh = static_cast<unsigned>(a.B * a.H);
     const long long elems = (static_cast<long long>(D) * D + D) * a.B * a.H;
     const unsigned eblocks = static_cast<unsigned>((elems + 255) / 256);
     gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
     gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
-    gdn_bwd_fstate_kernel<D, Tin><<<bh * a.nsplit, 512, fstate_smem<D>(a.nsplit), s>>>(a);
+    if ((e = launch_fstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
     gdn_bwd_local_kernel<D, Tin><<<nch, 256, local_smem<D>(), s>>>(a);
-    gdn_bwd_dstate_kernel<D, Tin><<<bh * a.nsplit, 512, dstate_smem<D>(a.nsplit), s>>>(a);
+    if ((e = launch_dstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
     gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
     gdn_bwd_kv_kernel<D, Tin><<<nch, 256, kv_smem<D>(), s>>>(a);
     return cudaGetLastError();

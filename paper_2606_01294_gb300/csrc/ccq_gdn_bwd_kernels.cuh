@@ -173,17 +173,20 @@ __device__ __forceinline__ void row_rnorm_ld(const float *x, int ld, float *rn, 
 }
 
 // Register-tiled product of two operands in shared memory, computed by 256 virtual threads
-// (the CTA's threads stride over them) of TM x TN outputs each:
-//   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   m < 16 TM, n < 16 TN,
-// virtual thread (tm, tn) holding rows tm + 16 i and columns tn + 16 j, so that a warp's loads
-// of B for one j are 16 consecutive columns and its loads of A two rows (broadcasts); a B
-// column stride bcs and an A row stride ars that are odd (or 1) keep them free of bank
+// (the CTA's threads stride over them) of TM x TN outputs each, on a (256 / GN) x GN grid:
+//   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   m < (256 / GN) TM, n < GN TN,
+// virtual thread (tm, tn) holding rows tm + (256 / GN) i and columns tn + GN j, so that a warp's
+// loads of B for one j are GN consecutive columns and its loads of A 32 / GN rows (broadcasts);
+// a B column stride bcs and an A row stride ars that are odd (or 1) keep them free of bank
 // conflicts.  ep(m, n, value) consumes every output once, in the thread that computed it.
-template <int TM, int TN, typename Ep>
+// (Rows at or past mlim are skipped: a product with fewer rows than the grid, TM = 1.)
+template <int TM, int TN, int GN = 16, typename Ep>
 __device__ __forceinline__ void tile_mm(const float *A, int ars, int acs, const float *B, int brs, int bcs, int K,
-                                        Ep ep) {
+                                        Ep ep, int mlim = 1 << 30) {
+    constexpr int GM = 256 / GN;
     for (int vt = static_cast<int>(threadIdx.x); vt < 256; vt += static_cast<int>(blockDim.x)) {
-        const int tm = vt >> 4, tn = vt & 15;
+        const int tm = vt / GN, tn = vt % GN;
+        if (tm >= mlim) continue;
         float acc[TM][TN];
 #pragma unroll
         for (int i = 0; i < TM; ++i)
@@ -194,9 +197,9 @@ __device__ __forceinline__ void tile_mm(const float *A, int ars, int acs, const 
         for (int k = 0; k < K; ++k) {
             float av[TM], bv[TN];
 #pragma unroll
-            for (int i = 0; i < TM; ++i) av[i] = a0[16 * i * ars + k * acs];
+            for (int i = 0; i < TM; ++i) av[i] = a0[GM * i * ars + k * acs];
 #pragma unroll
-            for (int j = 0; j < TN; ++j) bv[j] = b0[k * brs + 16 * j * bcs];
+            for (int j = 0; j < TN; ++j) bv[j] = b0[k * brs + GN * j * bcs];
 #pragma unroll
             for (int i = 0; i < TM; ++i)
 #pragma unroll
@@ -205,26 +208,28 @@ __device__ __forceinline__ void tile_mm(const float *A, int ars, int acs, const 
 #pragma unroll
         for (int i = 0; i < TM; ++i)
 #pragma unroll
-            for (int j = 0; j < TN; ++j) ep(tm + 16 * i, tn + 16 * j, acc[i][j]);
+            for (int j = 0; j < TN; ++j) ep(tm + GM * i, tn + GN * j, acc[i][j]);
     }
 }
 
 // ---------------------------------------------------------------------------------------------
-// Per chunk: Tt = (I + A)^{-1} by forward substitution, and the chunk's key statistics.
+// Per chunk: Tt = (I + A)^{-1} by forward substitution, and the chunk's key statistics (the
+// products KK and Kbar^T Kbar as tile_mm over padded tiles).
 template <int D, typename Tin>
 __global__ void __launch_bounds__(256) gdn_bwd_prep_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
+    constexpr int LD = D + 1, LC = kC + 1, TD = D / 16;
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *Kb = sm;                // [64][D]
-    float *A = Kb + kC * D;        // [64][64]
-    float *Tt = A + kC * kC;       // [64][64]
-    float *graw = Tt + kC * kC;    // [64]
+    float *Kb = sm;                // [64][LD]
+    float *A = Kb + kC * LD;       // [64][LC]
+    float *Tt = A + kC * LC;       // [64][LC]
+    float *graw = Tt + kC * LC;    // [64]
     float *gc = graw + kC;
     float *be = gc + kC;
     float *rk = be + kC;
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
-    load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+    load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -232,44 +237,33 @@ __global__ void __launch_bounds__(256) gdn_bwd_prep_kernel(const GdnBwdArgs a) {
         be[i] = t < a.T ? a.beta[row] : 0.f;
     }
     __syncthreads();
-    row_rnorm<D>(Kb, rk, a.l2norm);
+    row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
     gate_prefix(graw, gc);
     __syncthreads();
-    GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+    GBWD_FOR(idx, kC * D) Kb[(idx / D) * LD + idx % D] *= rk[idx / D];
     __syncthreads();
-    GBWD_FOR(idx, kC * kC) {
-        const int i = idx / kC, j = idx % kC;
-        float v = 0.f;
-        if (j < i) {
-            float kk = 0.f;
-            for (int c = 0; c < D; ++c) kk += Kb[i * D + c] * Kb[j * D + c];
-            v = be[i] * expf(gc[i] - gc[j]) * kk;
-        }
-        A[idx] = v;
-    }
+    // A_ij = beta_i e^{gc_i - gc_j} kbar_i . kbar_j for j < i
+    tile_mm<4, 4>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) {
+        A[i * LC + j] = j < i ? be[i] * expf(gc[i] - gc[j]) * v : 0.f;
+    });
     __syncthreads();
     // (I + A) Tt = I with A strictly lower: row i of Tt needs rows 0..i-1.
     for (int i = 0; i < kC; ++i) {
         GBWD_FOR(j, kC) {
             float v = i == j ? 1.f : 0.f;
-            for (int l = j; l < i; ++l) v -= A[i * kC + l] * Tt[l * kC + j];
-            Tt[i * kC + j] = v;
+            for (int l = j; l < i; ++l) v -= A[i * LC + l] * Tt[l * LC + j];
+            Tt[i * LC + j] = v;
         }
         __syncthreads();
     }
     float *tt = a.tt + static_cast<size_t>(ch) * kC * kC;
-    GBWD_FOR(idx, kC * kC) tt[idx] = Tt[idx];
+    GBWD_FOR(idx, kC * kC) tt[idx] = Tt[(idx / kC) * LC + idx % kC];
     float *sk = a.sk + static_cast<size_t>(ch) * D * D;
-    GBWD_FOR(idx, D * D) {
-        const int p = idx / D, c = idx % D;
-        float acc = 0.f;
-        for (int i = 0; i < kC; ++i) acc += Kb[i * D + p] * Kb[i * D + c];
-        sk[idx] = acc;
-    }
+    tile_mm<TD, TD>(Kb, 1, LD, Kb, LD, 1, kC, [&](int p, int c, float v) { sk[p * D + c] = v; });
     float *mk = a.mk + static_cast<size_t>(ch) * D;
     GBWD_FOR(c, D) {
         float acc = 0.f;
-        for (int i = 0; i < kC; ++i) acc += Kb[i * D + c];
+        for (int i = 0; i < kC; ++i) acc += Kb[i * LD + c];
         mk[c] = acc;
     }
 }
@@ -310,39 +304,39 @@ __global__ void __launch_bounds__(256) gdn_bwd_prefix_kernel(const GdnBwdArgs a)
 }
 
 // Per sequence and head, chunks in order: the state entering every chunk (and, when hT is
-// set, the final state).  CTA (sequence-head, s) carries the value columns
-// [s D/nsplit, (s+1) D/nsplit) of H.
-template <int D, typename Tin>
+// set, the final state).  CTA (sequence-head, s) carries the value columns [s DC, (s+1) DC),
+// DC = D / NS, of H; a chunk's three products run as tile_mm over padded tiles.
+template <int D, typename Tin, int NS>
 __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
-    const int ns = a.nsplit, DC = D / ns;
+    constexpr int DC = D / NS, LD = D + 1, LDC = DC + 1, LC = kC + 1;
+    constexpr int GN = DC < 16 ? DC : 16, GM = 256 / GN, TMD = D / GM > 0 ? D / GM : 1;
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *Hs = sm;               // [D][DC]
-    float *Kb = Hs + D * DC;      // [64][D]
-    float *R = Kb + kC * D;       // [64][DC]
-    float *U = R + kC * DC;       // [64][DC]
-    float *Tt = U + kC * DC;      // [64][64]
-    float *graw = Tt + kC * kC;   // [64]
+    float *Hs = sm;                // [D][LDC]
+    float *Kb = Hs + D * LDC;      // [64][LD]
+    float *R = Kb + kC * LD;       // [64][LDC]
+    float *U = R + kC * LDC;       // [64][LDC] diag(ed) U
+    float *Tt = U + kC * LDC;      // [64][LC] Tt diag(beta)
+    float *graw = Tt + kC * LC;    // [64]
     float *gc = graw + kC, *be = gc + kC, *rk = be + kC, *E = rk + kC, *ed = E + kC;
 
-    const int bh = blockIdx.x / ns, c0 = (blockIdx.x % ns) * DC, b = bh / a.H, h = bh % a.H;
+    const int bh = blockIdx.x / NS, c0 = (blockIdx.x % NS) * DC, b = bh / a.H, h = bh % a.H;
     const Tin *vin = static_cast<const Tin *>(a.v);
-    GBWD_FOR(idx, D * DC) {
-        const int l = idx / DC, j = idx % DC;
-        Hs[idx] = a.S0 ? a.S0[(static_cast<size_t>(bh) * D + l) * D + c0 + j] : 0.f;
-    }
+    stream8(D * DC, [&](int idx) {
+        return a.S0 ? a.S0[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] : 0.f;
+    }, [&](int idx, float x) { Hs[(idx / DC) * LDC + idx % DC] = x; });
     __syncthreads();
     for (int r = 0; r < a.NC; ++r) {
         const size_t ch = static_cast<size_t>(bh) * a.NC + r;
         float *hs = a.hs + ch * D * D;
-        GBWD_FOR(idx, D * DC) hs[(idx / DC) * D + c0 + idx % DC] = Hs[idx];
-        load_tile<D, Tin>(Kb, a.k, a, b, h, r);
-        GBWD_FOR(idx, kC * DC) {
-            const int i = idx / DC, j = idx % DC, t = r * kC + i;
-            R[idx] = t < a.T ? to_f(vin[tok_row(a, b, t, h) * D + c0 + j]) : 0.f;
-        }
+        GBWD_FOR(idx, D * DC) hs[(idx / DC) * D + c0 + idx % DC] = Hs[(idx / DC) * LDC + idx % DC];
+        load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
+        stream8(kC * DC, [&](int idx) {
+            const int t = r * kC + idx / DC;
+            return t < a.T ? to_f(vin[tok_row(a, b, t, h) * D + c0 + idx % DC]) : 0.f;
+        }, [&](int idx, float x) { R[(idx / DC) * LDC + idx % DC] = x; });
         const float *tt = a.tt + ch * kC * kC;
-        GBWD_FOR(idx, kC * kC) Tt[idx] = tt[idx];
+        stream8(kC * kC, [&](int idx) { return tt[idx]; }, [&](int idx, float x) { Tt[(idx / kC) * LC + idx % kC] = x; });
         GBWD_FOR(i, kC) {
             const int t = r * kC + i;
             const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -350,43 +344,32 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
             be[i] = t < a.T ? a.beta[row] : 0.f;
         }
         __syncthreads();
-        row_rnorm<D>(Kb, rk, a.l2norm);
+        row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
         gate_prefix(graw, gc);
         __syncthreads();
-        GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+        GBWD_FOR(idx, kC * D) Kb[(idx / D) * LD + idx % D] *= rk[idx / D];
+        GBWD_FOR(idx, kC * kC) Tt[(idx / kC) * LC + idx % kC] *= be[idx % kC];
         GBWD_FOR(i, kC) {
             E[i] = expf(gc[i]);
             ed[i] = expf(gc[kC - 1] - gc[i]);
         }
         __syncthreads();
         // R = V - diag(E) Kbar H
-        GBWD_FOR(idx, kC * DC) {
-            const int i = idx / DC, j = idx % DC;
-            float acc = 0.f;
-            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * Hs[l * DC + j];
-            R[idx] -= E[i] * acc;
-        }
+        tile_mm<kC / GM, DC / GN, GN>(Kb, LD, 1, Hs, LDC, 1, D, [&](int i, int j, float v) { R[i * LDC + j] -= E[i] * v; });
         __syncthreads();
-        // U = Tt diag(beta) R
-        GBWD_FOR(idx, kC * DC) {
-            const int i = idx / DC, j = idx % DC;
-            float acc = 0.f;
-            for (int l = 0; l <= i; ++l) acc += Tt[i * kC + l] * be[l] * R[l * DC + j];
-            U[idx] = acc;
-        }
+        // diag(ed) U = diag(ed) Tt diag(beta) R
+        tile_mm<kC / GM, DC / GN, GN>(Tt, LC, 1, R, LDC, 1, kC, [&](int i, int j, float v) { U[i * LDC + j] = ed[i] * v; });
         __syncthreads();
-        // H <- e^{gc_last} H + Kd^T U
+        // H <- e^{gc_last} H + Kd^T U = e^{gc_last} H + Kbar^T diag(ed) U
         const float elast = expf(gc[kC - 1]);
-        GBWD_FOR(idx, D * DC) {
-            const int l = idx / DC, j = idx % DC;
-            float acc = 0.f;
-            for (int i = 0; i < kC; ++i) acc += ed[i] * Kb[i * D + l] * U[i * DC + j];
-            Hs[idx] = elast * Hs[idx] + acc;
-        }
+        tile_mm<TMD, DC / GN, GN>(Kb, 1, LD, U, LDC, 1, kC, [&](int l, int j, float v) {
+            Hs[l * LDC + j] = elast * Hs[l * LDC + j] + v;
+        }, D);
         __syncthreads();
     }
     if (a.hT)
-        GBWD_FOR(idx, D * DC) a.hT[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] = Hs[idx];
+        GBWD_FOR(idx, D * DC)
+            a.hT[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] = Hs[(idx / DC) * LDC + idx % DC];
 }
 
 // Per chunk, everything that does not need dH: z, qc, R, U, dqc, dq, dlambda, the CCQ
@@ -629,33 +612,40 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
 // Per sequence and head, chunks last to first: the adjoint dH of the state leaving every
 // chunk (stored), then carried into the chunk: dU = P^T D + Kd dH, dR = diag(beta) Tt^T dU,
 // dH <- e^{gc_last} dH + (diag(E) Qc)^T D - (diag(E) Kbar)^T dR.  Writes dS0.  Like the
-// forward pass, CTA (sequence-head, s) carries the value columns [s D/nsplit, (s+1) D/nsplit).
-template <int D, typename Tin>
+// forward pass, CTA (sequence-head, s) carries the value columns [s DC, (s+1) DC), DC = D / NS.
+template <int D, typename Tin, int NS>
 __global__ void __launch_bounds__(512) gdn_bwd_dstate_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
-    const int ns = a.nsplit, DC = D / ns;
+    constexpr int DC = D / NS, LD = D + 1, LDC = DC + 1, LC = kC + 1;
+    constexpr int GN = DC < 16 ? DC : 16, GM = 256 / GN, TMD = D / GM > 0 ? D / GM : 1;
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
-    float *dH = sm;               // [D][DC]
-    float *Kb = dH + D * DC;      // [64][D]
-    float *dU = Kb + kC * D;      // [64][DC]
-    float *dR = dU + kC * DC;     // [64][DC]
-    float *Tt = dR + kC * DC;     // [64][64]
-    float *graw = Tt + kC * kC;   // [64]
+    float *dH = sm;                // [D][LDC]
+    float *Yb = dH + D * LDC;      // [D][LDC] the chunk's (diag(E) Qc)^T D columns
+    float *Kb = Yb + D * LDC;      // [64][LD]
+    float *dU = Kb + kC * LD;      // [64][LDC]
+    float *dR = dU + kC * LDC;     // [64][LDC] diag(E) dR
+    float *Tt = dR + kC * LDC;     // [64][LC]
+    float *graw = Tt + kC * LC;    // [64]
     float *gc = graw + kC, *be = gc + kC, *rk = be + kC, *E = rk + kC, *ed = E + kC;
 
-    const int bh = blockIdx.x / ns, c0 = (blockIdx.x % ns) * DC, b = bh / a.H, h = bh % a.H;
-    GBWD_FOR(idx, D * DC) {
-        const int l = idx / DC, j = idx % DC;
-        dH[idx] = a.dST ? a.dST[(static_cast<size_t>(bh) * D + l) * D + c0 + j] : 0.f;
-    }
+    const int bh = blockIdx.x / NS, c0 = (blockIdx.x % NS) * DC, b = bh / a.H, h = bh % a.H;
+    stream8(D * DC, [&](int idx) {
+        return a.dST ? a.dST[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] : 0.f;
+    }, [&](int idx, float x) { dH[(idx / DC) * LDC + idx % DC] = x; });
     __syncthreads();
     for (int r = a.NC - 1; r >= 0; --r) {
         const size_t ch = static_cast<size_t>(bh) * a.NC + r;
         float *dhg = a.dh + ch * D * D;
-        GBWD_FOR(idx, D * DC) dhg[(idx / DC) * D + c0 + idx % DC] = dH[idx];
-        load_tile<D, Tin>(Kb, a.k, a, b, h, r);
+        GBWD_FOR(idx, D * DC) dhg[(idx / DC) * D + c0 + idx % DC] = dH[(idx / DC) * LDC + idx % DC];
+        load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
         const float *tt = a.tt + ch * kC * kC;
-        GBWD_FOR(idx, kC * kC) Tt[idx] = tt[idx];
+        stream8(kC * kC, [&](int idx) { return tt[idx]; }, [&](int idx, float x) { Tt[(idx / kC) * LC + idx % kC] = x; });
+        const float *X1 = a.x1 + ch * kC * D;
+        stream8(kC * DC, [&](int idx) { return X1[(idx / DC) * D + c0 + idx % DC]; },
+                [&](int idx, float x) { dU[(idx / DC) * LDC + idx % DC] = x; });
+        const float *Y1 = a.y1 + ch * D * D;
+        stream8(D * DC, [&](int idx) { return Y1[(idx / DC) * D + c0 + idx % DC]; },
+                [&](int idx, float x) { Yb[(idx / DC) * LDC + idx % DC] = x; });
         GBWD_FOR(i, kC) {
             const int t = r * kC + i;
             const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -663,42 +653,33 @@ __global__ void __launch_bounds__(512) gdn_bwd_dstate_kernel(const GdnBwdArgs a)
             be[i] = t < a.T ? a.beta[row] : 0.f;
         }
         __syncthreads();
-        row_rnorm<D>(Kb, rk, a.l2norm);
+        row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
         gate_prefix(graw, gc);
         __syncthreads();
-        GBWD_FOR(idx, kC * D) Kb[idx] *= rk[idx / D];
+        GBWD_FOR(idx, kC * D) Kb[(idx / D) * LD + idx % D] *= rk[idx / D];
         GBWD_FOR(i, kC) {
             E[i] = expf(gc[i]);
             ed[i] = expf(gc[kC - 1] - gc[i]);
         }
         __syncthreads();
-        const float *X1 = a.x1 + ch * kC * D;
-        GBWD_FOR(idx, kC * DC) {
-            const int i = idx / DC, j = idx % DC;
-            float acc = 0.f;
-            for (int l = 0; l < D; ++l) acc += Kb[i * D + l] * dH[l * DC + j];
-            dU[idx] = X1[i * D + c0 + j] + ed[i] * acc;
-        }
+        // dU = P^T D + diag(ed) Kbar dH
+        tile_mm<kC / GM, DC / GN, GN>(Kb, LD, 1, dH, LDC, 1, D, [&](int i, int j, float v) { dU[i * LDC + j] += ed[i] * v; });
         __syncthreads();
-        GBWD_FOR(idx, kC * DC) {
-            const int i = idx / DC, j = idx % DC;
-            float acc = 0.f;
-            for (int l = i; l < kC; ++l) acc += Tt[l * kC + i] * dU[l * DC + j];
-            dR[idx] = be[i] * acc;
-        }
+        // diag(E) dR = diag(E beta) Tt^T dU
+        tile_mm<kC / GM, DC / GN, GN>(Tt, 1, LC, dU, LDC, 1, kC, [&](int i, int j, float v) {
+            dR[i * LDC + j] = E[i] * be[i] * v;
+        });
         __syncthreads();
-        const float *Y1 = a.y1 + ch * D * D;
+        // dH <- e^{gc_last} dH + (diag(E) Qc)^T D - Kbar^T diag(E) dR
         const float elast = expf(gc[kC - 1]);
-        GBWD_FOR(idx, D * DC) {
-            const int p = idx / DC, j = idx % DC;
-            float acc = 0.f;
-            for (int i = 0; i < kC; ++i) acc += E[i] * Kb[i * D + p] * dR[i * DC + j];
-            dH[idx] = elast * dH[idx] + Y1[p * D + c0 + j] - acc;
-        }
+        tile_mm<TMD, DC / GN, GN>(Kb, 1, LD, dR, LDC, 1, kC, [&](int p, int j, float v) {
+            dH[p * LDC + j] = elast * dH[p * LDC + j] + Yb[p * LDC + j] - v;
+        }, D);
         __syncthreads();
     }
     if (a.dS0)
-        GBWD_FOR(idx, D * DC) a.dS0[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] = dH[idx];
+        GBWD_FOR(idx, D * DC)
+            a.dS0[(static_cast<size_t>(bh) * D + idx / DC) * D + c0 + idx % DC] = dH[(idx / DC) * LDC + idx % DC];
 }
 
 // Exclusive suffix over the chunks of each sequence and head of the CCQ increments:
@@ -995,15 +976,15 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
 }
 
 // Shared-memory bytes of each kernel.
-template <int D> constexpr size_t prep_smem() { return sizeof(float) * (kC * D + 2 * kC * kC + 4 * kC); }
-template <int D> constexpr size_t fstate_smem(int ns) {
-    return sizeof(float) * (D * (D / ns) + kC * D + 2 * kC * (D / ns) + kC * kC + 6 * kC);
+template <int D> constexpr size_t prep_smem() { return sizeof(float) * (kC * (D + 1) + 2 * kC * (kC + 1) + 4 * kC); }
+template <int D, int NS> constexpr size_t fstate_smem() {
+    return sizeof(float) * (D * (D / NS + 1) + kC * (D + 1) + 2 * kC * (D / NS + 1) + kC * (kC + 1) + 6 * kC);
 }
 template <int D> constexpr size_t local_smem() {
     return sizeof(float) * (5 * kC * (D + 1) + 2 * kC * (kC + 1) + 12 * kC + D);
 }
-template <int D> constexpr size_t dstate_smem(int ns) {
-    return sizeof(float) * (D * (D / ns) + kC * D + 2 * kC * (D / ns) + kC * kC + 6 * kC);
+template <int D, int NS> constexpr size_t dstate_smem() {
+    return sizeof(float) * (2 * D * (D / NS + 1) + kC * (D + 1) + 2 * kC * (D / NS + 1) + kC * (kC + 1) + 6 * kC);
 }
 
 // Value-column blocks of the sequential passes: the most (up to 4) that keep the CTAs within

@@ -60,15 +60,29 @@ static void run_blocks(F f, long long grid, size_t smem_bytes) {
     }
 }
 
+// The sequential passes are instantiated per count of value-column blocks (1, 2 or 4).
+template <int D, typename Tin>
+static void run_fstate(const GdnBwdArgs &a, long long bh) {
+    if (a.nsplit == 4) run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin, 4>(a); }, bh * 4, fstate_smem<D, 4>());
+    else if (a.nsplit == 2) run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin, 2>(a); }, bh * 2, fstate_smem<D, 2>());
+    else run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin, 1>(a); }, bh, fstate_smem<D, 1>());
+}
+template <int D, typename Tin>
+static void run_dstate(const GdnBwdArgs &a, long long bh) {
+    if (a.nsplit == 4) run_blocks([&] { gdn_bwd_dstate_kernel<D, Tin, 4>(a); }, bh * 4, dstate_smem<D, 4>());
+    else if (a.nsplit == 2) run_blocks([&] { gdn_bwd_dstate_kernel<D, Tin, 2>(a); }, bh * 2, dstate_smem<D, 2>());
+    else run_blocks([&] { gdn_bwd_dstate_kernel<D, Tin, 1>(a); }, bh, dstate_smem<D, 1>());
+}
+
 template <int D, typename Tin>
 static void run(const GdnBwdArgs &a) {
     const long long nch = static_cast<long long>(a.B) * a.H * a.NC, bh = static_cast<long long>(a.B) * a.H;
     const long long elems = (static_cast<long long>(D) * D + D) * bh;
     run_blocks([&] { gdn_bwd_prep_kernel<D, Tin>(a); }, nch, prep_smem<D>());
     run_blocks([&] { gdn_bwd_prefix_kernel<D>(a); }, elems, 0);
-    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh * a.nsplit, fstate_smem<D>(a.nsplit));
+    run_fstate<D, Tin>(a, bh);
     run_blocks([&] { gdn_bwd_local_kernel<D, Tin>(a); }, nch, local_smem<D>());
-    run_blocks([&] { gdn_bwd_dstate_kernel<D, Tin>(a); }, bh * a.nsplit, dstate_smem<D>(a.nsplit));
+    run_dstate<D, Tin>(a, bh);
     run_blocks([&] { gdn_bwd_suffix_kernel<D>(a); }, elems, 0);
     run_blocks([&] { gdn_bwd_kv_kernel<D, Tin>(a); }, nch, kv_smem<D>());
 }
@@ -153,7 +167,7 @@ static int go_dec(int B, int T, int H, int l2norm, int centered, float scale, in
     g.dC = take(d * d); g.dmv = take(d); g.dn = take(4);
     const long long nch = static_cast<long long>(chunks), bh = static_cast<long long>(B) * H;
     run_blocks([&] { gdn_bwd_prep_kernel<D, Tin>(a); }, nch, prep_smem<D>());
-    run_blocks([&] { gdn_bwd_fstate_kernel<D, Tin>(a); }, bh * a.nsplit, fstate_smem<D>(a.nsplit));
+    run_fstate<D, Tin>(a, bh);
     run_blocks([&] { gdec_stats_kernel<D, Tin>(g); }, nch, gdec_stats_smem<D>());
     run_blocks([&] { gdec_scan_kernel<D>(g); }, (static_cast<long long>(D) * D + D + 1) * bh, 0);
     run_blocks([&] { gdec_out_kernel<D, Tin>(g); }, nch, gdec_out_smem<D>());
