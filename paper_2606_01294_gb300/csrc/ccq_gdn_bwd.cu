@@ -63,10 +63,10 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
     gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
     gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
     if ((e = launch_fstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
-    gdn_bwd_local_kernel<D, Tin><<<nch, 256, local_smem<D>(), s>>>(a);
+    gdn_bwd_local_kernel<D, Tin><<<nch, kBwdThreads, local_smem<D>(), s>>>(a);
     if ((e = launch_dstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
     gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
-    gdn_bwd_kv_kernel<D, Tin><<<nch, 256, kv_smem<D>(), s>>>(a);
+    gdn_bwd_kv_kernel<D, Tin><<<nch, kBwdThreads, kv_smem<D>(), s>>>(a);
     return cudaGetLastError();
 }
 

@@ -49,6 +49,7 @@ namespace ccq {
 namespace gbwd {
 
 constexpr int kC = 64;  // chunk length
+constexpr int kBwdThreads = 512;  // threads of the per-chunk local and kv kernels
 
 #define GBWD_FOR(i, n) for (int i = static_cast<int>(threadIdx.x); i < (n); i += static_cast<int>(blockDim.x))
 
@@ -172,19 +173,19 @@ __device__ __forceinline__ void row_rnorm_ld(const float *x, int ld, float *rn, 
     }
 }
 
-// Register-tiled product of two operands in shared memory, computed by 256 virtual threads
-// (the CTA's threads stride over them) of TM x TN outputs each, on a (256 / GN) x GN grid:
-//   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   m < (256 / GN) TM, n < GN TN,
-// virtual thread (tm, tn) holding rows tm + (256 / GN) i and columns tn + GN j, so that a warp's
+// Register-tiled product of two operands in shared memory, computed by VT virtual threads
+// (the CTA's threads stride over them) of TM x TN outputs each, on a (VT / GN) x GN grid:
+//   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   m < (VT / GN) TM, n < GN TN,
+// virtual thread (tm, tn) holding rows tm + (VT / GN) i and columns tn + GN j, so that a warp's
 // loads of B for one j are GN consecutive columns and its loads of A 32 / GN rows (broadcasts);
 // a B column stride bcs and an A row stride ars that are odd (or 1) keep them free of bank
 // conflicts.  ep(m, n, value) consumes every output once, in the thread that computed it.
 // (Rows at or past mlim are skipped: a product with fewer rows than the grid, TM = 1.)
-template <int TM, int TN, int GN = 16, typename Ep>
+template <int TM, int TN, int GN = 16, int VT = 256, typename Ep>
 __device__ __forceinline__ void tile_mm(const float *A, int ars, int acs, const float *B, int brs, int bcs, int K,
                                         Ep ep, int mlim = 1 << 30) {
-    constexpr int GM = 256 / GN;
-    for (int vt = static_cast<int>(threadIdx.x); vt < 256; vt += static_cast<int>(blockDim.x)) {
+    constexpr int GM = VT / GN;
+    for (int vt = static_cast<int>(threadIdx.x); vt < VT; vt += static_cast<int>(blockDim.x)) {
         const int tm = vt / GN, tn = vt % GN;
         if (tm >= mlim) continue;
         float acc[TM][TN];
@@ -210,6 +211,19 @@ __device__ __forceinline__ void tile_mm(const float *A, int ars, int acs, const 
 #pragma unroll
             for (int j = 0; j < TN; ++j) ep(tm + GM * i, tn + GN * j, acc[i][j]);
     }
+}
+
+// The grid of an M x N product for VT virtual threads: 32 columns a row of the grid for N >= 128
+// with 512 threads, 16 otherwise (N itself below 16).
+template <int M, int N, int VT>
+struct MmShape {
+    static constexpr int GN = (N >= 128 && VT >= 512) ? 32 : (N >= 16 ? 16 : N);
+    static constexpr int TN = N / GN, GM = VT / GN, TM = M / GM > 0 ? M / GM : 1;
+};
+template <int M, int N, int VT, typename Ep>
+__device__ __forceinline__ void mm(const float *A, int ars, int acs, const float *B, int brs, int bcs, int K, Ep ep) {
+    using S = MmShape<M, N, VT>;
+    tile_mm<S::TM, S::TN, S::GN, VT>(A, ars, acs, B, brs, bcs, K, ep, M);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -378,9 +392,9 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
 // block at a time through a tile that is free at that point, and z waits in the W slot of the
 // workspace while its tile holds D.
 template <int D, typename Tin>
-__global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) {
+__global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
-    constexpr int LD = D + 1, LC = kC + 1, TD = D / 16;
+    constexpr int LD = D + 1, LC = kC + 1, VT = kBwdThreads;
     constexpr int RB = D < 64 ? D : 64, NH = D / RB;      // row blocks of 64 (k-blocks)
     constexpr int RN = D < 32 ? D : 32, NN = D / RN;      // row blocks of 32 (n-blocks, in sB)
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
@@ -438,12 +452,12 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
             [&](int idx, float x) { sB[(idx / kC) * LC + idx % kC] = x * be[idx % kC]; });
     __syncthreads();
     // (Qbar Kbar^T) o causal;  R = V - diag(E) Kbar H over the row blocks of H
-    tile_mm<4, 4>(Qb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
+    mm<kC, kC, VT>(Qb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Zw, LD, H + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        tile_mm<4, TD>(Kb + RB * hf, LD, 1, Zw, LD, 1, RB, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
+        mm<kC, D, VT>(Kb + RB * hf, LD, 1, Zw, LD, 1, RB, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
     }
     __syncthreads();
     // cq_i = CumK_i . qbar_i with CumK_i = M + sum_{j<=i} kbar_j;  U = Tt diag(beta) R
@@ -456,7 +470,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     {
         float *Rg = a.r + t64;
         float *Ug = a.u + t64;
-        tile_mm<4, TD>(sB, LC, 1, Rq, LD, 1, kC, [&](int i, int j, float v) {
+        mm<kC, D, VT>(sB, LC, 1, Rq, LD, 1, kC, [&](int i, int j, float v) {
             Ud[i * LD + j] = v;
             Ug[i * D + j] = v;
         });
@@ -464,12 +478,12 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     }
     // z = Sigma_t qbar (App. B form): (Qbar S^K + ((Qbar Kbar^T) o causal) Kbar) / t - c CumK cq / t^2
     __syncthreads();
-    tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
+    mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        tile_mm<4, TD>(Qb + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
+        mm<kC, D, VT>(Qb + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
     }
     __syncthreads();
     GBWD_FOR(j, D) {
@@ -496,7 +510,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     }
     __syncthreads();
     // P = (Qc Kbar^T) o Gamma o causal;  D (the scaled output adjoint) into z's tile
-    tile_mm<4, 4>(Rq, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) {
+    mm<kC, kC, VT>(Rq, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) {
         sB[i * LC + j] = j <= i ? v * expf(gc[i] - gc[j]) : 0.f;
     });
     stream8(kC * D, [&](int idx) {
@@ -507,8 +521,8 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     // P^T D for the state pass;  dP = (D U^T) o Gamma o causal
     {
         float *X1 = a.x1 + t64;
-        tile_mm<4, TD>(sB, 1, LC, Zw, LD, 1, kC, [&](int i, int j, float v) { X1[i * D + j] = v; });
-        tile_mm<4, 4>(Zw, LD, 1, Ud, 1, LD, D, [&](int i, int j, float v) {
+        mm<kC, D, VT>(sB, 1, LC, Zw, LD, 1, kC, [&](int i, int j, float v) { X1[i * D + j] = v; });
+        mm<kC, kC, VT>(Zw, LD, 1, Ud, 1, LD, D, [&](int i, int j, float v) {
             sA[i * LC + j] = (j <= i && i < n) ? v * expf(gc[i] - gc[j]) : 0.f;
         });
     }
@@ -519,14 +533,14 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     // (over row blocks of H in sB);  gqh_i = E_i rowsum((Qc H) o D)_i = sum_j qc_ij ((E D) H^T)_ij
     {
         float *Y1 = a.y1 + static_cast<size_t>(ch) * D * D;
-        tile_mm<TD, TD>(Rq, 1, LD, Zw, LD, 1, kC, [&](int p, int j, float v) { Y1[p * D + j] = v; });
-        tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] = v; });
+        mm<D, D, VT>(Rq, 1, LD, Zw, LD, 1, kC, [&](int p, int j, float v) { Y1[p * D + j] = v; });
+        mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] = v; });
     }
     for (int nb = 0; nb < NN; ++nb) {
         __syncthreads();
         copy_rows<D>(sB, LD, H + static_cast<size_t>(RN * nb) * D, RN);
         __syncthreads();
-        tile_mm<4, RN / 16>(Zw, LD, 1, sB, 1, LD, D, [&](int i, int j, float v) {
+        mm<kC, RN, VT>(Zw, LD, 1, sB, 1, LD, D, [&](int i, int j, float v) {
             const int jg = RN * nb + j;
             Ud[i * LD + jg] += v;
             if (i < n) atomicAdd(&gqh[i], Rq[i * LD + jg] * v);
@@ -551,7 +565,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     }
     __syncthreads();
     // (W Kbar^T) o causal
-    tile_mm<4, 4>(Zw, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
+    mm<kC, kC, VT>(Zw, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     __syncthreads();
     // cz_i = CumK_i . dz_i = t_i (M . W_i + sum_{j<=i} W_i . kbar_j)
     GBWD_FOR(i, kC) {
@@ -563,12 +577,12 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
     // dqbar = dqc + W S^K + ((W Kbar^T) o causal) Kbar - c CumK cz / t^2 (in place);
     // the chunk's increments DC += W^T Qbar and Dm += sum_i dCum_i,
     // dCum_i = -c (dz_i cq_i + qbar_i cz_i) / t_i^2
-    tile_mm<4, TD>(sB, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+    mm<kC, D, VT>(sB, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        tile_mm<4, TD>(Zw + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+        mm<kC, D, VT>(Zw + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     }
     __syncthreads();
     {
@@ -583,7 +597,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_local_kernel(const GdnBwdArgs a) 
             }
             dM[j] = -c * acc;
         }
-        tile_mm<TD, TD>(Zw, 1, LD, Qb, LD, 1, kC, [&](int p, int j, float v) { dC[p * D + j] = v; });
+        mm<D, D, VT>(Zw, 1, LD, Qb, LD, 1, kC, [&](int p, int j, float v) { dC[p * D + j] = v; });
         float *vec = a.vec + static_cast<size_t>(ch) * 4 * kC;
         GBWD_FOR(i, kC) {
             vec[i] = cq[i];
@@ -726,10 +740,10 @@ __global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a)
 // tiles have the odd row stride D + 1 and the [64][64] ones 65, and the workspace operands
 // are staged through BF (and, for the D x D ones, 64 rows at a time through the S/dP pair).
 template <int D, typename Tin>
-__global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
+__global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
-    constexpr int LD = D + 1, LC = kC + 1, TD = D / 16;
-    constexpr int RB = D < 64 ? D : 64, NH = D / RB, TR = RB / 16;  // row blocks of the D x D operands
+    constexpr int LD = D + 1, LC = kC + 1, VT = kBwdThreads;
+    constexpr int RB = D < 64 ? D : 64, NH = D / RB;  // row blocks of the D x D operands
     float *sm = reinterpret_cast<float *>(gbwd_smem4);
     float *Kb = sm;                // [64][LD] kbar
     float *dU = Kb + kC * LD;      // [64][LD] dU, then the reverse sums of dCum
@@ -790,13 +804,13 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         __syncthreads();
         copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        tile_mm<4, TD>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) {
+        mm<kC, D, VT>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) {
             dU[i * LD + j] = (hf ? dU[i * LD + j] : 0.f) + v;
         });
     }
     __syncthreads();
     // S = Qc Kbar^T (Qc in BF; S in the S/dP pair, free once the staging of dH is read)
-    tile_mm<4, 4>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
+    mm<kC, kC, VT>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     // dU = X1 + diag(ed) t with t = Kbar dH, which also waits in dR for kd
     stream8(kC * D, [&](int idx) { return X1[idx]; }, [&](int idx, float x) {
         const int i = idx / D, j = idx % D;
@@ -822,12 +836,12 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     // dv = dR = diag(beta) Tt^T dU;  dP = (D U^T) o Gamma o causal
     {
         Tin *dv = static_cast<Tin *>(a.dv);
-        tile_mm<4, TD>(Tt, 1, LC, dU, LD, 1, kC, [&](int i, int j, float v) {
+        mm<kC, D, VT>(Tt, 1, LC, dU, LD, 1, kC, [&](int i, int j, float v) {
             const float x = be[i] * v;
             dR[i * LD + j] = x;
             if (i < n) dv[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(x);
         });
-        tile_mm<4, 4>(BF, LD, 1, dK, 1, LD, D, [&](int i, int j, float v) {
+        mm<kC, kC, VT>(BF, LD, 1, dK, 1, LD, D, [&](int i, int j, float v) {
             sB[i * LC + j] = (j <= i && i < n) ? v * expf(gc[i] - gc[j]) : 0.f;
         });
     }
@@ -860,24 +874,24 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     // dK = dP^T Qc + diag(ed) U dH^T - diag(E) dR H^T (the last two over row blocks of dH, H)
     copy_rows<D>(BF, LD, Qcg, kC);
     __syncthreads();
-    tile_mm<4, TD>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] = v; });
+    mm<kC, D, VT>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] = v; });
     __syncthreads();
     copy_rows<D>(BF, LD, Ug, kC);
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        tile_mm<4, TR>(BF, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
+        mm<kC, RB, VT>(BF, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
         __syncthreads();
         copy_rows<D>(B2, LD, H + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        tile_mm<4, TR>(dR, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
+        mm<kC, RB, VT>(dR, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
     }
     __syncthreads();
     copy_rows<D>(BF, LD, Rg, kC);
     __syncthreads();
     // dTb = dU R^T
-    tile_mm<4, 4>(dU, LD, 1, BF, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
+    mm<kC, kC, VT>(dU, LD, 1, BF, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     __syncthreads();
     // dbeta (the Tb = Tt diag(beta) factor) = column sums of dTb o Tt;  M2 = Tt^T (dTb diag(beta))
     GBWD_FOR(j, kC) {
@@ -885,14 +899,14 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
         for (int i = 0; i < kC; ++i) acc += sA[i * LC + j] * Tt[i * LC + j];
         db1[j] = acc;
     }
-    tile_mm<4, 4>(Tt, 1, LC, sA, LC, 1, kC, [&](int i, int j, float v) { sB[i * LC + j] = v * be[j]; });
+    mm<kC, kC, VT>(Tt, 1, LC, sA, LC, 1, kC, [&](int i, int j, float v) { sB[i * LC + j] = v * be[j]; });
     __syncthreads();
     // dA = strict_lower(-M2 Tt^T)
-    tile_mm<4, 4>(sB, LC, 1, Tt, 1, LC, kC, [&](int i, int j, float v) { sA[i * LC + j] = j < i ? -v : 0.f; });
+    mm<kC, kC, VT>(sB, LC, 1, Tt, 1, LC, kC, [&](int i, int j, float v) { sA[i * LC + j] = j < i ? -v : 0.f; });
     __syncthreads();
     // dKK = diag(beta) (dA o Gamma);  rs_i = sum_j dA_ij Gamma_ij KK_ij (the dbeta of A);
     // rowsum(dA o A)_i = beta_i rs_i;  cs_j = colsum(dA o A)_j
-    tile_mm<4, 4>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float kk) {
+    mm<kC, kC, VT>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float kk) {
         float v = 0.f;
         if (j < i) {
             const float gm = expf(gc[i] - gc[j]);
@@ -910,14 +924,14 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     }
     __syncthreads();
     // dK += (dKK + dKK^T) Kbar
-    tile_mm<4, TD>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+    mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     __syncthreads();
     // CCQ terms: (Qbar Kbar^T) o causal and (W Kbar^T) o causal
     copy_rows<D>(BF, LD, Qbg, kC);
     copy_rows<D>(dR, LD, Wg, kC);
     __syncthreads();
-    tile_mm<4, 4>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
-    tile_mm<4, 4>(dR, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
+    mm<kC, kC, VT>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
+    mm<kC, kC, VT>(dR, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     // reverse cumulative sums G_ij = sum_{l>=i} dCum_lj / (-c), dCum_l = -c (dz_l cq_l + qbar_l cz_l) / t_l^2,
     // dz_l = t_l W_l
     GBWD_FOR(j, D) {
@@ -929,19 +943,19 @@ __global__ void __launch_bounds__(256) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     }
     __syncthreads();
     // dK += QKc^T W + WKc^T Qbar + Dm - c G
-    tile_mm<4, TD>(sA, 1, LC, dR, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
-    tile_mm<4, TD>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) {
+    mm<kC, D, VT>(sA, 1, LC, dR, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+    mm<kC, D, VT>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) {
         dK[i * LD + j] += v + Dm[j] - c * dU[i * LD + j];
     });
     // dK += Kbar (DC + DC^T), over the row blocks p of DC
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
-        GBWD_FOR(idx, RB * D) {
+        stream8(RB * D, [&](int idx) {
             const int p = idx / D, j = idx % D, pg = RB * hf + p;
-            B2[p * LD + j] = DC[pg * D + j] + DC[j * D + pg];
-        }
+            return DC[pg * D + j] + DC[j * D + pg];
+        }, [&](int idx, float x) { B2[(idx / D) * LD + idx % D] = x; });
         __syncthreads();
-        tile_mm<4, TD>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+        mm<kC, D, VT>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     }
     __syncthreads();
     GBWD_FOR(i, kC) {
