@@ -36,24 +36,24 @@
 // status word when a chunk goes beyond that; the two-reference kernel (ccq_gla_chunk_wide.cu,
 // algo CCQ_ALGO_CHUNKWISE_WIDE) halves the span of every factor.
 //
-// Warp specialisation (14 warps):
+// Warp specialisation (18 warps, 96 registers a thread):
 //   EPI   (warps 0-7)   the epilogues of chunk r -- W, q_clean, mask of A, output --
 //                       and the bf16 operand copies of the states, placed where EPI
-//                       would otherwise wait on an MMA: S^K_{r+1} while G4 runs,
-//                       e^{Gmid} S_{r+1} (rescaling X in TMEM) while G2 of chunk r+1
-//                       runs.  The 64-row products are M = 64 MMAs (rows 16q..16q+15
-//                       in TMEM lanes 32q..32q+15); warps w and w+4 share lane
-//                       quadrant q = w % 4 and split its columns.  The output goes
-//                       from registers straight to global memory.
-//   PREP  (warps 8-11)  prep of chunk r+1 while the chain runs chunk r: gate
-//                       cumsum, row norms, kbar, Kg, e^{G-Gmid}, M . qbar, lambda.
-//   ISSUE (warp 12)     one thread issues every tcgen05.mma (and, unless COPY does,
+//                       would otherwise wait on an MMA: e^{Gmid} S_r (rescaling X in
+//                       TMEM) while G3 runs, S^K_{r+1} while G4 runs.  The 64-row
+//                       products are M = 64 MMAs (rows 16q..16q+15 in TMEM lanes
+//                       32q..32q+15); warps w and w+4 share lane quadrant q = w % 4
+//                       and split its columns.
+//   PREP  (warps 8-15)  prep of chunk r+1 while the chain runs chunk r: row norms
+//                       (q and M . qbar on warps 8-11, k on 12-15), gate cumsum in
+//                       four token quarters, kbar, Kg, e^{G-Gmid}, lambda.
+//   ISSUE (warp 16)     one thread issues every tcgen05.mma (and, unless COPY does,
 //                       the per-chunk TMA copies), in the order G2 | G1 | G3 G8 | G7 |
 //                       G4 G6 | G5, so that G1, G7 and G6 run under the epilogues.  An MMA
 //                       instruction holds its issuing thread for its whole execution,
 //                       which is why no epilogue thread issues.  EPI signals the issuer
 //                       with named-barrier arrives; the issuer signals EPI with commits.
-//   COPY  (warp 13)     in the COPY instance: the loads of chunk r+2, the store of O and the
+//   COPY  (warp 17)     in the COPY instance: the loads of chunk r+2, the store of O and the
 //                       next v, plus an L2 prefetch of chunk r+2 beyond each load.
 // Per-chunk tiles are double-buffered (two slots); the loads of chunk r+2 start as
 // soon as chunk r's last MMA reader of the slot (G6) completes.  v is single-buffered
@@ -61,7 +61,7 @@
 // Rows past T load as zeros: zero keys add nothing to any sum, zero gates keep
 // the cumulative gate, so the ragged tail needs no special arithmetic.
 // With a.ckpt set, EPI also copies each chunk's two state tiles and key sum to
-// the checkpoint buffer (one bulk copy per chunk) and the last segment writes
+// the checkpoint buffer (bulk copies) and the last segment writes
 // S_T there; the backward (ccq_gla_bwd.cu) reads them.
 // With a.nseg > 1 every CTA walks one segment (a range of whole chunks) of one
 // sequence, starting from the segment's initial states in a.seg_ws
@@ -81,9 +81,10 @@ namespace {
 constexpr int kC = 64;         // chunk length
 constexpr int kD = 128;        // Dk = Dv
 constexpr int kEpiThreads = 256;
-constexpr int kPrepWarp0 = 8, kIssueWarp = 12, kCopyWarp = 13;
-constexpr int kThreadsNoCopy = 32 * kCopyWarp;       // 416
-constexpr int kThreadsCopy = 32 * (kCopyWarp + 1);    // 448
+constexpr int kPrepWarp0 = 8, kIssueWarp = 16, kCopyWarp = 17;
+constexpr int kPrepThreads = 32 * (kIssueWarp - kPrepWarp0);  // 256
+constexpr int kThreadsNoCopy = 32 * kCopyWarp;       // 544
+constexpr int kThreadsCopy = 32 * (kCopyWarp + 1);    // 576
 constexpr int kSyncCount = kEpiThreads + 32;          // EPI + the issuing warp
 // largest exponent (log2 units) a gate factor may have: a state accumulated over a chunk
 // from keys scaled by up to 2^118 stays inside the fp32 range
@@ -91,16 +92,26 @@ constexpr float kMaxExp2 = 118.f;
 
 // ---- shared memory map (bytes from the 1024-aligned base)
 // two slots of per-chunk tiles, each [64 rows][128 cols] bf16 as two T64 tiles of 8 KB:
-constexpr uint32_t SLOT_BYTES = 65536;
+constexpr uint32_t SLOT_BYTES = 49152;
 constexpr uint32_t SO_Q = 0;       // raw q, then q_clean * e^{G - Gmid}
-constexpr uint32_t SO_K = 16384;   // raw k, then kbar
-constexpr uint32_t SO_KG = 32768;  // raw gates land here (bf16: 16 KB, fp32: KG+EG 32 KB); then Kg
-constexpr uint32_t SO_EG = 49152;  // e^{G - Gmid}
-constexpr uint32_t OFF_V = 131072;   // 16K  v; after G5 the output staging of the TMA store
-constexpr uint32_t OFF_W = 147456;   // 8K   W, then the masked A ([64][64], one T64 tile)
-constexpr uint32_t OFF_SK = 155648;  // 32K  bf16 S^K ([128][128], two T64 tiles of 16 KB)
+constexpr uint32_t SO_KG = 16384;  // raw gates land here (bf16: 16 KB, fp32: KG+EG 32 KB); then Kg
+constexpr uint32_t SO_EG = 32768;  // e^{G - Gmid}
+// The keys of both slots and the bf16 S^K share one region per 64-column half h of the
+// key dimension: [kbar of slot 0 (64 rows)][S^K (128 rows)][kbar of slot 1 (64 rows)],
+// 128 B per row (T64 tiles, K-major for G2 and G1, MN-major for G3 and G8).
+constexpr uint32_t OFF_KS = 98304;   // 2 x 32K
+constexpr uint32_t KS_HALF = 32768;  // distance between the two halves
+constexpr uint32_t KS_SK = 8192;     // S^K rows within a half
+constexpr uint32_t KS_K1 = 24576;    // kbar of slot 1 within a half
+constexpr uint32_t OFF_V = 163840;   // 16K  v; after G5 the output staging of the TMA store
+constexpr uint32_t OFF_W = 180224;   // 8K   W, then the masked A ([64][64], one T64 tile)
 constexpr uint32_t OFF_S = 188416;   // 32K  bf16 e^{Gmid} S ([128][128], two T64 tiles of 16 KB)
 constexpr uint32_t OFF_MISC = 221184;
+static_assert(2 * SLOT_BYTES == OFF_KS && OFF_KS + 2 * KS_HALF == OFF_V, "shared memory map");
+// the kbar tile of slot s, key columns 64 h .. 64 h + 63
+__host__ __device__ constexpr uint32_t kbar_off(int s, int h) {
+    return OFF_KS + static_cast<uint32_t>(h) * KS_HALF + (s ? KS_K1 : 0u);
+}
 // misc: per-slot arrays (3072 B per slot)
 constexpr uint32_t MS_BYTES = 3072;
 constexpr uint32_t MS_RQ = 0;      // [64] 1/|q_i|
@@ -112,16 +123,14 @@ constexpr uint32_t MS_F = 1536;    // [128] e^{Gtot - Gmid}
 constexpr uint32_t MS_MST = 2048;  // [128] key sum M at the chunk start
 constexpr uint32_t MS_ITI = 2560;  // [64] 1 / t_i
 constexpr uint32_t MS_QN = 2816;   // [64] |q_i| (1 without the l2 norm)
-constexpr uint32_t M_DMP = 6144;   // [2][128] partial key sums of the chunk (prep)
-constexpr uint32_t M_DMPREV = 7168;  // [128] key sum of the previous chunk
-constexpr uint32_t M_GT0 = 7680;   // [128] gate sum over tokens 0..31
-constexpr uint32_t M_BAR = 8192;   // mbarriers
-constexpr uint32_t M_TMEM = 8304;
-constexpr uint32_t M_ABORT = 8308;
-constexpr uint32_t kMiscBytes = 8320;
+constexpr uint32_t M_DMP = 6144;   // [4][128] per token quarter: gate sums, then key sums (prep)
+constexpr uint32_t M_DMPREV = 8192;  // [128] key sum of the previous chunk
+constexpr uint32_t M_BAR = 8704;   // mbarriers
+constexpr uint32_t M_TMEM = 8816;
+constexpr uint32_t M_ABORT = 8820;
+constexpr uint32_t kMiscBytes = 8832;
 constexpr uint32_t kSmemBytes = OFF_MISC + kMiscBytes + 1024;  // + alignment slack
 static_assert(kSmemBytes <= 232448, "exceeds the 227 KB per-CTA limit");
-static_assert(OFF_S == OFF_SK + 32768, "a checkpoint copies the S^K and S tiles as one block");
 
 enum {
     BAR_IN0 = 0, BAR_IN1 = 1, BAR_V = 2, BAR_GA = 3, BAR_GB = 4, BAR_GK = 5, BAR_GC = 6,
@@ -140,8 +149,8 @@ constexpr uint32_t TM_SA = 384;  // 64 cols: Sc, then A (M = 64 layout)
 constexpr uint32_t kTmemCols = 512;
 
 constexpr uint32_t ID_64x64_KK = make_idesc(64, 64, 0, 0);
-constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
 constexpr uint32_t ID_64x128_KM = make_idesc(64, 128, 0, 1);
+constexpr uint32_t ID_64x128_KK = make_idesc(64, 128, 0, 0);
 constexpr uint32_t ID_128x128_MM = make_idesc(128, 128, 1, 1);
 
 __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chunk, const float *w) {
@@ -154,7 +163,7 @@ __device__ __forceinline__ void store_row_chunk(uint8_t *tile, int row, int chun
 }
 
 template <bool COPY>
-__global__ void __launch_bounds__(COPY ? kThreadsCopy : kThreadsNoCopy, 1)
+__global__ void __maxnreg__(96)
 gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constant__ CUtensorMap map_k,
                  const __grid_constant__ CUtensorMap map_v, const __grid_constant__ CUtensorMap map_g,
                  const __grid_constant__ CUtensorMap map_o, const ChunkArgs a) {
@@ -166,7 +175,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
     uint8_t *misc = sm + OFF_MISC;
     float *dmp = reinterpret_cast<float *>(misc + M_DMP);
     float *dmprev = reinterpret_cast<float *>(misc + M_DMPREV);
-    float *gt0 = reinterpret_cast<float *>(misc + M_GT0);
     uint64_t *bar = reinterpret_cast<uint64_t *>(misc + M_BAR);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(misc + M_TMEM);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(misc + M_ABORT);
@@ -214,8 +222,8 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         mbar_arrive_expect_tx(bb, 4 * 8192 + g_bytes);
         tma_load_4d(base + SO_Q, &map_q, bb, 0, h, tok0 + tg, bt);
         tma_load_4d(base + SO_Q + 8192, &map_q, bb, 64, h, tok0 + tg, bt);
-        tma_load_4d(base + SO_K, &map_k, bb, 0, h, tok0 + tg, bt);
-        tma_load_4d(base + SO_K + 8192, &map_k, bb, 64, h, tok0 + tg, bt);
+        tma_load_4d(sm + kbar_off(s, 0), &map_k, bb, 0, h, tok0 + tg, bt);
+        tma_load_4d(sm + kbar_off(s, 1), &map_k, bb, 64, h, tok0 + tg, bt);
         tma_load_4d(base + SO_KG, &map_g, bb, 0, h, tok0 + tg, bt);
         if (COPY && r + 2 < NC) {  // chunk r + 2 into L2, so that its loads hit there
             const int tp = tok0 + tg + 2 * kC;
@@ -276,8 +284,10 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         tmem_wait_st();
     } else if (warp < kIssueWarp) {
         const int wt = tid - 32 * kPrepWarp0;
-        slot_f(0, MS_MST)[wt] = m0 ? m0[(segst ? 0 : static_cast<size_t>(bh) * kD) + wt] : 0.f;
-        dmprev[wt] = 0.f;
+        if (wt < kD) {
+            slot_f(0, MS_MST)[wt] = m0 ? m0[(segst ? 0 : static_cast<size_t>(bh) * kD) + wt] : 0.f;
+            dmprev[wt] = 0.f;
+        }
     } else if (warp == kIssueWarp && lane == 0) {
         tma_prefetch_desc(&map_q);
         tma_prefetch_desc(&map_k);
@@ -314,7 +324,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 tmem_ld32(tq + TM_SK + 64 * grp + 32 * cc, x);
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4)
-                    store_row_chunk(sm + OFF_SK + grp * 16384, row, 4 * cc + q4, x + 8 * q4);
+                    store_row_chunk(sm + OFF_KS + grp * KS_HALF + KS_SK, row, 4 * cc + q4, x + 8 * q4);
             }
             fence_proxy_async_smem();
             tc_fence_before();
@@ -353,7 +363,9 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                 uint8_t *rec = ck_head + static_cast<size_t>(cb + r) * kCkptChunkBytes;
                 if (grp == 0) reinterpret_cast<float *>(rec + 65536)[row] = slot_f(r & 1, MS_MST)[row];
                 if (tid == 0) {
-                    bulk_store(rec, sm + OFF_SK, 65536);
+                    bulk_store(rec, sm + OFF_KS + KS_SK, 16384);
+                    bulk_store(rec + 16384, sm + OFF_KS + KS_HALF + KS_SK, 16384);
+                    bulk_store(rec + 32768, sm + OFF_S, 32768);
                     tma_store_commit();
                 }
             }
@@ -369,6 +381,8 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const uint32_t sp = (r >> 1) & 1, par = r & 1;
             uint8_t *slot = sm + s * SLOT_BYTES;
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
+            const float f_prev = f_cur;  // e^{Gtot - Gmid} of chunk r - 1
+            const float egm = slot_f(s, MS_EGM)[row];
             f_cur = slot_f(s, MS_F)[row];
             const float rqi = slot_f(s, MS_RQ)[i];
             const float mqi = slot_f(s, MS_MQ)[i];
@@ -406,6 +420,9 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             fence_proxy_async_smem();
             tc_fence_before();
             named_bar_arrive(NB_W, kSyncCount);
+            // ---- e^{Gmid_r} S_r while G3 runs (G6 and G7 of chunk r-1 have run: the output
+            // epilogue of chunk r-1 waited for GD, which follows them)
+            if (r > 0) snap_s(r, f_prev * egm);
             // ---- q_clean epilogue (Eq. clean), scaled by e^{G - Gmid}, into the Q tile.
             // q_clean e^{G-Gmid} = e^{G-Gmid} (rq (q - (lambda/t) P) + (lambda c / t) M);
             // this thread: row i, columns 64 grp + 32 hf .. +31 (T64 tile grp, chunks 4 hf ..)
@@ -500,12 +517,6 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
             tc_fence_before();
             named_bar_arrive(NB_OUT, kOutCount);
-            // ---- e^{Gmid_{r+1}} S_{r+1} while G2 of chunk r+1 runs (G6 and G7 of chunk r
-            // have run: GD follows them)
-            if (r + 1 < NC) {
-                mbar_wait(&bar[BAR_PREP0 + (s ^ 1)], ((r + 1) >> 1) & 1, abort_flag, status);
-                snap_s(r + 1, f_cur * slot_f(s ^ 1, MS_EGM)[row]);
-            }
         }
         if (ck_head && tid == 0) tma_store_wait_all();
         // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K (an empty packed sequence:
@@ -544,12 +555,20 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         }
     } else if (warp < kIssueWarp) {
         // =============================================================== PREP
+        // Eight warps.  Row norms: warps 0-3 take the rows of q (and M . q), warps 4-7 those
+        // of k; lanes l and l + 16 of a warp share row j, each one 64-column half (one T64
+        // tile), so eight consecutive lanes read eight different rows (no bank conflicts).
+        // Gates: thread (p, tq) takes key dims 2p, 2p+1 over the sixteen tokens of quarter tq.
         const int wt = tid - 32 * kPrepWarp0;
-        const int p = wt & 63, th = wt >> 6;  // key-dim pair (2p, 2p+1), token half
+        const int pw = wt >> 5;
+        const bool nq = pw < 4;
+        const int j = 16 * (pw & 3) + (lane & 15), hh = lane >> 4;
+        const int p = wt & 63, tq = wt >> 6;
         const int d0 = 2 * p;
-        float lam_reg = 0.f;  // lambda of row wt >> 1
-        {
-            const int tn = cb * kC + (wt >> 1);
+        constexpr float kLog2e = 1.4426950408889634f;
+        float lam_reg = 0.f;  // lambda of row j of the next chunk (q warps)
+        if (nq) {
+            const int tn = cb * kC + j;
             lam_reg = (tn < T) ? a.lambda[(rowbase + tn) * H + h] : 0.f;
         }
         float emax = 0.f;  // largest |exponent| (log2 units) of a gate factor met
@@ -560,48 +579,41 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             float *Mst = slot_f(s, MS_MST);
             mbar_wait(&bar[BAR_IN0 + s], sp, abort_flag, status);
             // key sum at the chunk start and lambda of the chunk
-            if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
+            if (r > 0 && wt < kD) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
             const float lam_cur = lam_reg;
-            {
-                const int tn = (cb + r + 1) * kC + (wt >> 1);
+            if (nq) {
+                const int tn = (cb + r + 1) * kC + j;
                 lam_reg = (tn < T) ? a.lambda[(rowbase + tn) * H + h] : 0.f;
             }
-            named_bar(NB_PREP, 128);
-            // row norms of q and k and M . q: thread pair (2j, 2j+1) takes row j, each
-            // thread one 64-column half (one T64 tile) of both q and k, in fp32 pairs
-            {
-                const int j = wt >> 1, hh = wt & 1;
-                uint4 qv[8], kv[8];
+            named_bar(NB_PREP, kPrepThreads);
+            if (nq) {
+                // |q_j|^2 and M . q_j in fp32 pairs
+                uint4 qv[8];
 #pragma unroll
-                for (int cc = 0; cc < 8; ++cc) {
+                for (int cc = 0; cc < 8; ++cc)
                     qv[cc] = *reinterpret_cast<const uint4 *>(slot + SO_Q + hh * 8192 + t64_chunk(j, cc));
-                    kv[cc] = *reinterpret_cast<const uint4 *>(slot + SO_K + hh * 8192 + t64_chunk(j, cc));
-                }
                 const float *Mh = Mst + 64 * hh;
-                uint64_t sq0 = 0, sq1 = 0, sk0 = 0, sk1 = 0, md0 = 0, md1 = 0;
+                uint64_t sq0 = 0, sq1 = 0, md0 = 0, md1 = 0;
 #pragma unroll
                 for (int cc = 0; cc < 8; ++cc) {
                     const ulonglong2 m01 = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc);
                     const ulonglong2 m23 = *reinterpret_cast<const ulonglong2 *>(Mh + 8 * cc + 4);
                     const uint32_t qw[4] = {qv[cc].x, qv[cc].y, qv[cc].z, qv[cc].w};
-                    const uint32_t kw[4] = {kv[cc].x, kv[cc].y, kv[cc].z, kv[cc].w};
                     const uint64_t mp[4] = {m01.x, m01.y, m23.x, m23.y};
 #pragma unroll
                     for (int w = 0; w < 4; ++w) {
-                        const uint64_t q2 = f2_from_bf16x2(qw[w]), k2 = f2_from_bf16x2(kw[w]);
+                        const uint64_t q2 = f2_from_bf16x2(qw[w]);
                         if (w & 1) {
-                            sq1 = f2_fma(q2, q2, sq1); sk1 = f2_fma(k2, k2, sk1); md1 = f2_fma(q2, mp[w], md1);
+                            sq1 = f2_fma(q2, q2, sq1); md1 = f2_fma(q2, mp[w], md1);
                         } else {
-                            sq0 = f2_fma(q2, q2, sq0); sk0 = f2_fma(k2, k2, sk0); md0 = f2_fma(q2, mp[w], md0);
+                            sq0 = f2_fma(q2, q2, sq0); md0 = f2_fma(q2, mp[w], md0);
                         }
                     }
                 }
-                const float2 a0 = f2_split(f2_add(sq0, sq1)), b0 = f2_split(f2_add(sk0, sk1)),
-                             c0v = f2_split(f2_add(md0, md1));
-                float ssq = a0.x + a0.y, ssk = b0.x + b0.y, mdt = c0v.x + c0v.y;
-                ssq += __shfl_xor_sync(0xffffffffu, ssq, 1);
-                ssk += __shfl_xor_sync(0xffffffffu, ssk, 1);
-                mdt += __shfl_xor_sync(0xffffffffu, mdt, 1);
+                const float2 a0 = f2_split(f2_add(sq0, sq1)), c0v = f2_split(f2_add(md0, md1));
+                float ssq = a0.x + a0.y, mdt = c0v.x + c0v.y;
+                ssq += __shfl_xor_sync(0xffffffffu, ssq, 16);
+                mdt += __shfl_xor_sync(0xffffffffu, mdt, 16);
                 if (hh == 0) {
                     const float rq = a.l2norm ? rsqrtf(fmaxf(ssq, 1e-12f)) : 1.f;
                     const float iti = 1.f / static_cast<float>(tseq0 + (cb + r) * kC + j + 1);
@@ -610,97 +622,122 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                     slot_f(s, MS_ITI)[j] = iti;
                     slot_f(s, MS_QN)[j] = a.l2norm ? fmaxf(ssq, 1e-12f) * rq : 1.f;
                     slot_f(s, MS_LT)[j] = lam_cur * iti;
-                } else {
+                }
+            } else {
+                // |k_j|^2
+                uint4 kv[8];
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc)
+                    kv[cc] = *reinterpret_cast<const uint4 *>(sm + kbar_off(s, hh) + t64_chunk(j, cc));
+                uint64_t sk0 = 0, sk1 = 0;
+#pragma unroll
+                for (int cc = 0; cc < 8; ++cc) {
+                    const uint32_t kw[4] = {kv[cc].x, kv[cc].y, kv[cc].z, kv[cc].w};
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) {
+                        const uint64_t k2 = f2_from_bf16x2(kw[w]);
+                        if (w & 1) sk1 = f2_fma(k2, k2, sk1);
+                        else sk0 = f2_fma(k2, k2, sk0);
+                    }
+                }
+                const float2 b0 = f2_split(f2_add(sk0, sk1));
+                float ssk = b0.x + b0.y;
+                ssk += __shfl_xor_sync(0xffffffffu, ssk, 16);
+                if (hh == 0) {
                     // rows past the end of a packed sequence hold the next one's keys: zero them
                     const bool in_seq = (cb + r) * kC + j < T;
                     slot_f(s, MS_RK)[j] = !in_seq ? 0.f : a.l2norm ? rsqrtf(fmaxf(ssk, 1e-12f)) : 1.f;
                 }
             }
-            // gate cumsum over this thread's 32 tokens for dims d0, d0+1, as fp32 pairs
-            uint64_t g2[32];
+            // gate cumsum over this thread's sixteen tokens for dims d0, d0+1, as fp32 pairs
+            uint64_t g2[16];
             {
                 uint64_t r2 = 0;  // (0.f, 0.f)
                 const int rem = T - (cb + r) * kC;  // tokens of the sequence in this chunk
 #pragma unroll
-                for (int jj = 0; jj < 32; ++jj) {
-                    const int j = 32 * th + jj;
+                for (int u = 0; u < 16; ++u) {
+                    const int jt = 16 * tq + u;
                     const uint64_t x2 =
-                        j >= rem ? 0
-                        : gate_f32 ? *reinterpret_cast<const uint64_t *>(slot + SO_KG + (j * kD + d0) * 4)
-                                   : f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(slot + SO_KG + (j * kD + d0) * 2));
+                        jt >= rem ? 0
+                        : gate_f32 ? *reinterpret_cast<const uint64_t *>(slot + SO_KG + (jt * kD + d0) * 4)
+                                   : f2_from_bf16x2(*reinterpret_cast<const uint32_t *>(slot + SO_KG + (jt * kD + d0) * 2));
                     r2 = f2_add(r2, x2);
-                    g2[jj] = r2;
+                    g2[u] = r2;
                 }
-                if (th == 0) {
-                    const float2 rv = f2_split(r2);
-                    gt0[d0] = rv.x;
-                    gt0[d0 + 1] = rv.y;
-                }
+                *reinterpret_cast<uint64_t *>(dmp + tq * kD + d0) = r2;  // the quarter's gate sums
             }
-            named_bar(NB_PREP, 128);  // raw gates all read, norms and gt0 visible
+            named_bar(NB_PREP, kPrepThreads);  // raw gates all read, norms and quarter sums visible
+            uint64_t dm2 = 0;
             {
-                constexpr float kLog2e = 1.4426950408889634f;
-                const float gm0 = gt0[d0], gm1 = gt0[d0 + 1];   // Gmid
+                // G at this quarter's start (sum of the earlier quarters) and Gmid = G at token 31
+                uint64_t q2[4];
+#pragma unroll
+                for (int qq = 0; qq < 4; ++qq) q2[qq] = *reinterpret_cast<const uint64_t *>(dmp + qq * kD + d0);
+                uint64_t gs = 0;
+#pragma unroll
+                for (int qq = 0; qq < 3; ++qq)
+                    if (qq < tq) gs = f2_add(gs, q2[qq]);
+                const float2 gm = f2_split(f2_add(q2[0], q2[1]));
+                const float2 gsv = f2_split(gs);
                 // exponents in log2 units relative to Gmid: x = (G - Gmid) log2(e)
-                const uint64_t o2 = f2_make(((th ? gm0 : 0.f) - gm0) * kLog2e, ((th ? gm1 : 0.f) - gm1) * kLog2e);
+                const uint64_t o2 = f2_make((gsv.x - gm.x) * kLog2e, (gsv.y - gm.y) * kLog2e);
                 const uint64_t l2e = f2_make(kLog2e, kLog2e);
-                if (th == 1) {
-                    // f = e^{Gtot - Gmid} (gate sum of tokens 32..63), e^{Gmid}
-                    const float2 gt = f2_split(g2[31]);
-                    slot_f(s, MS_F)[d0] = fast_exp2(gt.x * kLog2e);
-                    slot_f(s, MS_F)[d0 + 1] = fast_exp2(gt.y * kLog2e);
-                    slot_f(s, MS_EGM)[d0] = fast_exp2(gm0 * kLog2e);
-                    slot_f(s, MS_EGM)[d0 + 1] = fast_exp2(gm1 * kLog2e);
+                if (tq == 3) {
+                    // f = e^{Gtot - Gmid} (the last token's factor), e^{Gmid}
+                    const float2 xl = f2_split(f2_fma(g2[15], l2e, o2));
+                    slot_f(s, MS_F)[d0] = fast_exp2(xl.x);
+                    slot_f(s, MS_F)[d0 + 1] = fast_exp2(xl.y);
+                    slot_f(s, MS_EGM)[d0] = fast_exp2(gm.x * kLog2e);
+                    slot_f(s, MS_EGM)[d0 + 1] = fast_exp2(gm.y * kLog2e);
                 }
-                {
+                if (tq == 0 || tq == 3) {
                     // log gates are <= 0, so G falls monotonically and the factors' exponents are
                     // largest in magnitude at the chunk's first and last tokens
-                    const float2 xe = f2_split(f2_fma(th ? g2[31] : g2[0], l2e, o2));
+                    const float2 xe = f2_split(f2_fma(tq ? g2[15] : g2[0], l2e, o2));
                     emax = fmaxf(emax, fmaxf(fabsf(xe.x), fabsf(xe.y)));
                 }
                 const float *rk = slot_f(s, MS_RK);
-                const uint32_t tcol = (d0 >> 6) * 8192;
-                uint64_t dm2 = 0;
-                // four batches of eight tokens: every load of a batch is issued before its
+                uint8_t *kt = sm + kbar_off(s, d0 >> 6);  // kbar tile of these key columns
+                // two batches of eight tokens: every load of a batch is issued before its
                 // stores (the in-place kbar store may alias a later load)
 #pragma unroll
-                for (int bt = 0; bt < 4; ++bt) {
+                for (int bt = 0; bt < 2; ++bt) {
                     uint32_t kraw[8];
 #pragma unroll
                     for (int u = 0; u < 8; ++u) {
-                        const int j = 32 * th + 8 * bt + u;
-                        kraw[u] = *reinterpret_cast<const uint32_t *>(slot + SO_K + tcol + t64_offset(j, d0 & 63));
+                        const int jt = 16 * tq + 8 * bt + u;
+                        kraw[u] = *reinterpret_cast<const uint32_t *>(kt + t64_offset(jt, d0 & 63));
                     }
-                    const float4 rka = *reinterpret_cast<const float4 *>(rk + 32 * th + 8 * bt);
-                    const float4 rkb = *reinterpret_cast<const float4 *>(rk + 32 * th + 8 * bt + 4);
+                    const float4 rka = *reinterpret_cast<const float4 *>(rk + 16 * tq + 8 * bt);
+                    const float4 rkb = *reinterpret_cast<const float4 *>(rk + 16 * tq + 8 * bt + 4);
                     const float rkv[8] = {rka.x, rka.y, rka.z, rka.w, rkb.x, rkb.y, rkb.z, rkb.w};
 #pragma unroll
                     for (int u = 0; u < 8; ++u) {
-                        const int jj = 8 * bt + u, j = 32 * th + jj;
-                        const uint32_t off = tcol + t64_offset(j, d0 & 63);
+                        const int ju = 8 * bt + u, jt = 16 * tq + ju;
+                        const uint32_t off = t64_offset(jt, d0 & 63);
+                        const uint32_t toff = (d0 >> 6) * 8192 + off;  // in the slot's Kg / EG tiles
                         const uint64_t k2 = f2_mul(f2_from_bf16x2(kraw[u]), f2_make(rkv[u], rkv[u]));
-                        const float2 x = f2_split(f2_fma(g2[jj], l2e, o2));
-                        *reinterpret_cast<uint32_t *>(slot + SO_K + off) = bf16x2_from_f2(k2);
-                        *reinterpret_cast<uint32_t *>(slot + SO_KG + off) =
+                        const float2 x = f2_split(f2_fma(g2[ju], l2e, o2));
+                        *reinterpret_cast<uint32_t *>(kt + off) = bf16x2_from_f2(k2);
+                        *reinterpret_cast<uint32_t *>(slot + SO_KG + toff) =
                             bf16x2_from_f2(f2_mul(k2, f2_make(fast_exp2(-x.x), fast_exp2(-x.y))));
-                        *reinterpret_cast<uint32_t *>(slot + SO_EG + off) = pack_bf16(fast_exp2(x.x), fast_exp2(x.y));
+                        *reinterpret_cast<uint32_t *>(slot + SO_EG + toff) = pack_bf16(fast_exp2(x.x), fast_exp2(x.y));
                         dm2 = f2_add(dm2, k2);
                     }
                 }
-                const float2 dmv = f2_split(dm2);
-                dmp[th * kD + d0] = dmv.x;
-                dmp[th * kD + d0 + 1] = dmv.y;
             }
             fence_proxy_async_smem();
-            named_bar(NB_PREP, 128);
-            dmprev[wt] = dmp[wt] + dmp[kD + wt];
+            named_bar(NB_PREP, kPrepThreads);  // tiles and scalars written, quarter sums read
             if (wt == 0) mbar_arrive(&bar[BAR_PREP0 + s]);
+            *reinterpret_cast<uint64_t *>(dmp + tq * kD + d0) = dm2;  // the quarter's key sums
+            named_bar(NB_PREP, kPrepThreads);
+            if (wt < kD) dmprev[wt] = (dmp[wt] + dmp[kD + wt]) + (dmp[2 * kD + wt] + dmp[3 * kD + wt]);
         }
         // a factor beyond 2^kMaxExp2 cannot be represented: report it rather than return
         // silently wrong values
         if (emax > kMaxExp2) atomicExch(status, kStatusRange);
         // final key sum
-        if ((NC > 0 || vl) && a.mT && last_seg) {
+        if ((NC > 0 || vl) && a.mT && last_seg && wt < kD) {
             const int sl = NC > 0 ? (NC - 1) & 1 : 0;
             a.mT[static_cast<size_t>(bh) * kD + wt] = slot_f(sl, MS_MST)[wt] + dmprev[wt];
         }
@@ -709,7 +746,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const bool lead = lane == 0;
         // descriptor bases (start-address field advanced per K slice: +2 per 32 B)
         const uint64_t dW = make_desc(sb + OFF_W, 16, 1024);
-        const uint64_t dSK = make_desc(sb + OFF_SK, 16, 1024);
+        const uint64_t dSK = make_desc(sb + OFF_KS + KS_SK, 16, 1024);
         const uint64_t dS = make_desc(sb + OFF_S, 16384, 1024);
         const uint64_t dV = make_desc(sb + OFF_V, 8192, 1024);
         for (int r = 0; r < NC; ++r) {
@@ -717,18 +754,18 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             const uint32_t sp = (r >> 1) & 1, par = r & 1;
             const uint32_t ss = sb + s * SLOT_BYTES;
             const uint64_t dQ = make_desc(ss + SO_Q, 16, 1024);
-            const uint64_t dK = make_desc(ss + SO_K, 16, 1024);
-            const uint64_t dKm = make_desc(ss + SO_K, 8192, 1024);
+            const uint64_t dK = make_desc(sb + kbar_off(s, 0), 16, 1024);
+            const uint64_t dKm = make_desc(sb + kbar_off(s, 0), KS_HALF, 1024);
             const uint64_t dKG = make_desc(ss + SO_KG, 16, 1024);
             const uint64_t dKGm = make_desc(ss + SO_KG, 8192, 1024);
+            const uint32_t tp = tbase + TM_PO, tsa = tbase + TM_SA;
             mbar_wait(&bar[BAR_PREP0 + s], sp, abort_flag, status);
             tc_fence_after();
             // G2 Sc = Q Kbar^T (SA is free: the mask epilogue of chunk r-1 has read A)
             if (lead && !*abort_flag) {
-                for (int k = 0; k < 8; ++k) {
-                    const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                    mma_bf16(tbase + TM_SA, dQ + ko, dK + ko, ID_64x64_KK, k != 0);
-                }
+                for (int k = 0; k < 8; ++k)
+                    mma_bf16(tsa, dQ + (k >> 2) * 512 + (k & 3) * 2, dK + (k >> 2) * (KS_HALF >> 4) + (k & 3) * 2,
+                             ID_64x64_KK, k != 0);
                 mma_commit(&bar[BAR_GA]);
             }
             __syncwarp();
@@ -745,8 +782,8 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tc_fence_after();
             if (lead && !*abort_flag)
                 for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2,
-                             dSK + (k >> 2) * 1024 + (k & 3) * 2, ID_64x128_KK, k != 0);
+                    mma_bf16(tp, dQ + (k >> 2) * 512 + (k & 3) * 2, dSK + (k >> 2) * (KS_HALF >> 4) + (k & 3) * 2,
+                             ID_64x128_KK, k != 0);
             // v of chunk r replaces the staged output once the store has read it
             if (r > 0 && lead && !COPY) {
                 tma_store_wait_read();
@@ -758,7 +795,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tc_fence_after();
             if (lead && !*abort_flag) {
                 for (int k = 0; k < 4; ++k)
-                    mma_bf16(tbase + TM_PO, dW + k * 2, dKm + k * 128, ID_64x128_KM, 1);
+                    mma_bf16(tp, dW + k * 2, dKm + k * 128, ID_64x128_KM, 1);
                 mma_commit(&bar[BAR_GB]);
                 for (int k = 0; k < 4; ++k)
                     mma_bf16(tbase + TM_SK, dKm + k * 128, dKm + k * 128, ID_128x128_MM, 1);
@@ -779,12 +816,11 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             if (lead && !*abort_flag) {
                 for (int k = 0; k < 8; ++k) {
                     const uint64_t ko = (k >> 2) * 512 + (k & 3) * 2;
-                    mma_bf16(tbase + TM_SA, dQ + ko, dKG + ko, ID_64x64_KK, k != 0);
+                    mma_bf16(tsa, dQ + ko, dKG + ko, ID_64x64_KK, k != 0);
                 }
                 mma_commit(&bar[BAR_GC]);
                 for (int k = 0; k < 8; ++k)
-                    mma_bf16(tbase + TM_PO, dQ + (k >> 2) * 512 + (k & 3) * 2, dS + k * 128, ID_64x128_KM,
-                             k != 0);
+                    mma_bf16(tp, dQ + (k >> 2) * 512 + (k & 3) * 2, dS + k * 128, ID_64x128_KM, k != 0);
                 mma_commit(&bar[BAR_GC2]);
             }
             __syncwarp();
@@ -793,7 +829,7 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tc_fence_after();
             if (lead && !*abort_flag) {
                 for (int k = 0; k < 4; ++k)
-                    mma_bf16(tbase + TM_PO, dW + k * 2, dV + k * 128, ID_64x128_KM, 1);
+                    mma_bf16(tp, dW + k * 2, dV + k * 128, ID_64x128_KM, 1);
                 mma_commit(&bar[BAR_GD]);
             }
             __syncwarp();
