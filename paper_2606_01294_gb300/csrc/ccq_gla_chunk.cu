@@ -421,8 +421,11 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             tc_fence_before();
             named_bar_arrive(NB_W, kSyncCount);
             // ---- e^{Gmid_r} S_r while G3 runs (G6 and G7 of chunk r-1 have run: the output
-            // epilogue of chunk r-1 waited for GD, which follows them)
-            if (r > 0) snap_s(r, f_prev * egm);
+            // epilogue of chunk r-1 waited for GD, which follows them).  The instance without
+            // the copy warp (segments, checkpoints) writes it at the end of chunk r-1 instead, so
+            // that the checkpoint copy issued with it has read the tiles before S^K_{r+1} is
+            // written over them.
+            if (COPY && r > 0) snap_s(r, f_prev * egm);
             // ---- q_clean epilogue (Eq. clean), scaled by e^{G - Gmid}, into the Q tile.
             // q_clean e^{G-Gmid} = e^{G-Gmid} (rq (q - (lambda/t) P) + (lambda c / t) M);
             // this thread: row i, columns 64 grp + 32 hf .. +31 (T64 tile grp, chunks 4 hf ..)
@@ -517,6 +520,10 @@ gla_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             }
             tc_fence_before();
             named_bar_arrive(NB_OUT, kOutCount);
+            if (!COPY && r + 1 < NC) {
+                mbar_wait(&bar[BAR_PREP0 + (s ^ 1)], ((r + 1) >> 1) & 1, abort_flag, status);
+                snap_s(r + 1, f_cur * slot_f(s ^ 1, MS_EGM)[row]);
+            }
         }
         if (ck_head && tid == 0) tma_store_wait_all();
         // final states: S_T = e^{Gtot - Gmid} X (last chunk), S^K (an empty packed sequence:
