@@ -519,6 +519,12 @@ ccq_status ccq_gdn_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype
     return CCQ_OK;
 }
 
+// Per-chunk fp32 arrays of the CCQ-Gated-DeltaNet backward that the tensor-core forward can
+// fill (ChunkArgs::tt_out and the rest); with them the forward writes no output.
+struct GdnDumps {
+    float *tt, *sk, *mk, *hs;
+};
+
 // The Gated DeltaNet forward behind ccq_gdn_fwd; `dry` runs every argument check and
 // returns before the first CUDA call.
 static ccq_status gdn_fwd_impl(const void *q, const void *k, const void *v, const float *g,
@@ -526,7 +532,8 @@ static ccq_status gdn_fwd_impl(const void *q, const void *k, const void *v, cons
                                const float *S0, const float *C0, const float *m0, const int64_t *t0,
                                void *o, float *ST, float *CT, float *mT, int64_t *tT,
                                int B, int T, int H, int Dk, int Dv, void *workspace,
-                               size_t workspace_bytes, const ccq_params *p, void *stream, bool dry) {
+                               size_t workspace_bytes, const ccq_params *p, void *stream, bool dry,
+                               const GdnDumps *dumps = nullptr) {
     Common c;
     ccq_status st = check_common(p, B, T, H, Dk, Dv, &c);
     if (st != CCQ_OK) return st;
@@ -567,6 +574,10 @@ static ccq_status gdn_fwd_impl(const void *q, const void *k, const void *v, cons
         a.S0 = S0; a.C0 = C0; a.m0 = m0; a.t0 = t0;
         a.o = static_cast<__nv_bfloat16 *>(o);
         a.ST = ST; a.CT = CT; a.mT = mT;
+        if (dumps) {
+            a.tt_out = dumps->tt; a.sk_out = dumps->sk; a.mk_out = dumps->mk; a.hs_out = dumps->hs;
+            a.skip_o = 1;
+        }
         a.status = device_status_word();
         if (!a.status) return fail(CCQ_ERR_CUDA, "cannot resolve the device status word");
         int nseg = 1, seg_chunks = 0;
@@ -622,6 +633,23 @@ static ccq_status copy_state_grads(const float *dST, const float *dCT, const flo
     return CCQ_OK;
 }
 
+// bf16 inputs with Dk = 128 recompute the forward's per-chunk quantities with the tensor-core
+// forward kernels (gdn_wy_kernel, gdn_chunk_kernel), whose own workspace follows the
+// backward's arrays (at a 1 KB boundary); other inputs compute them on the CUDA cores.
+static bool gdn_bwd_tc_forward(ccq_dtype in_dtype, int Dk) { return in_dtype == CCQ_BF16 && Dk == 128; }
+static ccq_params gdn_bwd_forward_params(const ccq_params &p) {
+    ccq_params f = p;
+    f.algo = CCQ_ALGO_CHUNKWISE;
+    return f;
+}
+static size_t gdn_bwd_forward_offset(int B, int T, int H, int Dk) {
+    return (gdn_bwd_workspace_bytes(B, T, H, Dk) + 1023) & ~static_cast<size_t>(1023);
+}
+static size_t gdn_bwd_total_workspace(const ccq_params &p, ccq_dtype in_dtype, int B, int T, int H, int Dk) {
+    if (!gdn_bwd_tc_forward(in_dtype, Dk)) return gdn_bwd_workspace_bytes(B, T, H, Dk);
+    return gdn_bwd_forward_offset(B, T, H, Dk) + gdn_total_workspace(gdn_bwd_forward_params(p), B, T, H);
+}
+
 ccq_status ccq_gdn_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
                                       const ccq_params *p, size_t *bytes) {
     Common c;
@@ -629,7 +657,7 @@ ccq_status ccq_gdn_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_d
     if (st != CCQ_OK) return st;
     if (!bytes) return fail(CCQ_ERR_INVALID_ARG, "bytes is NULL");
     if (in_dtype != CCQ_BF16 && in_dtype != CCQ_FP32) return fail(CCQ_ERR_INVALID_ARG, "unknown dtype");
-    *bytes = T > 0 ? gdn_bwd_workspace_bytes(B, T, H, Dk) : 0;
+    *bytes = T > 0 ? gdn_bwd_total_workspace(c.p, in_dtype, B, T, H, Dk) : 0;
     return CCQ_OK;
 }
 
@@ -652,7 +680,7 @@ ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float 
     st = check_ptrs("q,k,v,g,beta,lambda,dout,dq,dk,dv,dg,dbeta",
                     {q, k, v, g, beta, lambda, dout, dq, dk, dv, dg, dbeta}, {});
     if (st != CCQ_OK) return st;
-    const size_t need = gdn_bwd_workspace_bytes(B, T, H, Dk);
+    const size_t need = gdn_bwd_total_workspace(c.p, in_dtype, B, T, H, Dk);
     if (!workspace || workspace_bytes < need)
         return fail(CCQ_ERR_INVALID_ARG, "workspace of %zu bytes required (got %zu)", need,
                     workspace ? workspace_bytes : static_cast<size_t>(0));
@@ -666,6 +694,19 @@ ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float 
     a.dq = dq; a.dk = dk; a.dv = dv; a.dg = dg; a.dbeta = dbeta; a.dlambda = dlambda;
     a.dS0 = dS0; a.dC0 = dC0; a.dm0 = dm0;
     a.workspace = workspace;
+    if (gdn_bwd_tc_forward(in_dtype, Dk)) {
+        // Tt, S^K_r, M_r and H_r of every chunk from the tensor-core forward (no output written:
+        // dq stands in for the output tensor, which the forward must be given)
+        GdnDumps d;
+        gdn_bwd_state_arrays(a, &d.tt, &d.sk, &d.mk, &d.hs);
+        const ccq_params fp = gdn_bwd_forward_params(c.p);
+        const size_t off = gdn_bwd_forward_offset(B, T, H, Dk);
+        st = gdn_fwd_impl(q, k, v, g, beta, lambda, in_dtype, S0, C0, m0, t0, dq, nullptr, nullptr, nullptr,
+                          nullptr, B, T, H, Dk, Dv, static_cast<uint8_t *>(workspace) + off, workspace_bytes - off,
+                          &fp, stream, false, &d);
+        if (st != CCQ_OK) return st;
+        a.states_ready = 1;
+    }
     cudaError_t e = launch_gdn_bwd(a, s);
     if (e != cudaSuccess) return cuda_fail(e, "Gated DeltaNet backward launch");
     return CCQ_OK;

@@ -60,9 +60,11 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
     const unsigned nch = static_cast<unsigned>(a.B * a.H * a.NC), bh = static_cast<unsigned>(a.B * a.H);
     const long long elems = (static_cast<long long>(D) * D + D) * a.B * a.H;
     const unsigned eblocks = static_cast<unsigned>((elems + 255) / 256);
-    gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
-    gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
-    if ((e = launch_fstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
+    if (!a.states_ready) {
+        gdn_bwd_prep_kernel<D, Tin><<<nch, 256, prep_smem<D>(), s>>>(a);
+        gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
+        if ((e = launch_fstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
+    }
     gdn_bwd_local_kernel<D, Tin><<<nch, kBwdThreads, local_smem<D>(), s>>>(a);
     if ((e = launch_dstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
     gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
@@ -71,6 +73,16 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
 }
 
 }  // namespace
+
+void gdn_bwd_state_arrays(const GdnBwdCall &c, float **tt, float **sk, float **mk, float **hs) {
+    const size_t chunks = static_cast<size_t>(c.B) * c.H * ((c.T + 63) / 64);
+    const size_t d = static_cast<size_t>(c.D);
+    float *p = static_cast<float *>(c.workspace);
+    *tt = p;
+    *sk = p + chunks * 64 * 64;
+    *mk = *sk + chunks * d * d;
+    *hs = *mk + chunks * d;
+}
 
 size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D) {
     const size_t chunks = static_cast<size_t>(B) * H * ((T + 63) / 64);
@@ -81,6 +93,7 @@ cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s) {
     gbwd::GdnBwdArgs a{};
     a.B = c.B; a.T = c.T; a.H = c.H; a.NC = (c.T + 63) / 64;
     a.nsplit = gbwd::seq_split(c.B, c.H);
+    a.states_ready = c.states_ready;
     a.l2norm = c.l2norm; a.centered = c.centered; a.scale = c.scale;
     a.q = c.q; a.k = c.k; a.v = c.v; a.dout = c.dout;
     a.g = c.g; a.beta = c.beta; a.lambda = c.lambda;

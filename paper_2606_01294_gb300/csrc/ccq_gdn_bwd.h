@@ -21,8 +21,14 @@ struct GdnBwdCall {
     void *dq, *dk, *dv;
     float *dg, *dbeta, *dlambda, *dS0, *dC0, *dm0;
     void *workspace;
+    // 1: the forward's per-chunk quantities (Tt, S^K_r, M_r, H_r) are already in the workspace
+    // arrays that gdn_bwd_state_arrays() names (written by the tensor-core forward); the three
+    // launches that would compute them are skipped.
+    int states_ready = 0;
 };
 size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D);
+// The workspace arrays of the forward's per-chunk quantities (layout: ChunkArgs::tt_out etc.).
+void gdn_bwd_state_arrays(const GdnBwdCall &c, float **tt, float **sk, float **mk, float **hs);
 cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s);
 
 // Arguments of the CUDA-core CCQ-Gated-DeltaNet forward with the decay-aligned covariance

@@ -89,6 +89,7 @@ struct GdnBwdArgs {
     int nsplit = 1;       // value-column blocks of the sequential passes (a divisor of D): the
                           // delta rule acts on the columns of H independently, so each
                           // (sequence, head) runs as nsplit CTAs of D / nsplit columns
+    int states_ready = 0; // tt, sk, mk, hs already hold Tt, S^K_r, M_r, H_r (from the forward)
 };
 
 __device__ __forceinline__ size_t tok_row(const GdnBwdArgs &a, int b, int t, int h) {

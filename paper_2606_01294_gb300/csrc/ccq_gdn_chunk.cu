@@ -289,6 +289,19 @@ gdn_wy_kernel(const __grid_constant__ CUtensorMap map_k, const __grid_constant__
         }
         __syncthreads();
     }
+    // ---- the fp32 Tt itself for the backward (one row half per thread, as float4 stores;
+    // the blocks above the diagonal were never written: zeros)
+    if (a.tt_out) {
+        const int i2 = tid >> 1, hf2 = tid & 1;
+        float4 *dst = reinterpret_cast<float4 *>(a.tt_out + (static_cast<size_t>(item) * kC + i2) * kC + 32 * hf2);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int j0 = 32 * hf2 + 4 * q;
+            const float4 t = *reinterpret_cast<const float4 *>(Tt + i2 * kAS + j0);
+            dst[q] = make_float4(j0 <= i2 ? t.x : 0.f, j0 + 1 <= i2 ? t.y : 0.f, j0 + 2 <= i2 ? t.z : 0.f,
+                                 j0 + 3 <= i2 ? t.w : 0.f);
+        }
+    }
     // ---- Tb = Tt diag(beta) (zero above the diagonal) as the bf16 T64 tile in A's place
     {
         const int i = tid >> 1, hf = tid & 1;
@@ -533,12 +546,20 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         const int i = 16 * (warp & 3) + (lane & 15);
         const int hf = lane >> 4;
         const int row = 32 * (warp & 3) + lane;  // state row of the M = 128 layout
-        auto snap_sk = [&]() {
+        // (with a.sk_out / a.hs_out the snapshots of chunk ch of this sequence also write the
+        // fp32 states to the backward's arrays)
+        auto snap_sk = [&](int ch) {
             tc_fence_after();
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 float x[32];
                 tmem_ld32(tq + TM_SK + 64 * grp + 32 * cc, x);
+                if (a.sk_out) {
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        a.sk_out + ((static_cast<size_t>(bh) * NCt + ch) * kD + row) * kD + 64 * grp + 32 * cc);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+                }
 #pragma unroll
                 for (int q4 = 0; q4 < 4; ++q4)
                     store_row_chunk(sm + OFF_SK + grp * 16384, row, 4 * cc + q4, x + 8 * q4);
@@ -550,12 +571,18 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         };
         // bf16 copy of the state H entering the next chunk; the TMEM copy is scaled by that
         // chunk's e^{gC} (hs), onto which D6 accumulates the chunk's write
-        auto snap_s = [&](float hs) {
+        auto snap_s = [&](float hs, int ch) {
             tc_fence_after();
 #pragma unroll
             for (int cc = 0; cc < 2; ++cc) {
                 float x[32];
                 tmem_ld32(tq + TM_S + 64 * grp + 32 * cc, x);
+                if (a.hs_out) {
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        a.hs_out + ((static_cast<size_t>(bh) * NCt + ch) * kD + row) * kD + 64 * grp + 32 * cc);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) dst[e] = make_float4(x[4 * e], x[4 * e + 1], x[4 * e + 2], x[4 * e + 3]);
+                }
                 const uint64_t hs2 = f2_make(hs, hs);
                 uint32_t w[16];
 #pragma unroll
@@ -580,8 +607,8 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
         float *epo = reinterpret_cast<float *>(misc + M_EPO);
         if (NC > 0) {
             mbar_wait(&bar[BAR_PREP0], 0, abort_flag, status);
-            snap_sk();
-            snap_s(slot_f(0, MS_SCAL)[1]);
+            snap_sk(cb);
+            snap_s(slot_f(0, MS_SCAL)[1], cb);
         }
         for (int r = 0; r < NC; ++r) {
             const int s = r & 1;
@@ -709,7 +736,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             // ---- S^K_{r+1} while D4 runs
             if (r + 1 < NC) {
                 mbar_wait(&bar[BAR_GK], par, abort_flag, status);
-                snap_sk();
+                snap_sk(cb + r + 1);
             }
             // ---- Pm_ij = [j<=i] QK_ij e^{gc_i - gc_j} (one exponential of a non-positive argument)
             mbar_wait(&bar[BAR_GC], par, abort_flag, status);
@@ -775,7 +802,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
                                 st_shared_b32(bk[(2 * q + u / 2) & 3] + rb + (4 * q + u) * 128, pr);
                             } else {
                                 const int tpos = (cb + r) * kC + i0 + 4 * q + u + (odd ? 1 : 0);
-                                if (tpos < T)
+                                if (tpos < T && !a.skip_o)
                                     *reinterpret_cast<uint32_t *>(a.o + ((rowbase + tpos) * H + h) * kD + c2) = pr;
                             }
                         }
@@ -788,7 +815,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             // ---- H_{r+1} while G2 of chunk r+1 runs (D3, D6 of chunk r have run: GD follows them)
             if (r + 1 < NC) {
                 mbar_wait(&bar[BAR_PREP0 + (s ^ 1)], ((r + 1) >> 1) & 1, abort_flag, status);
-                snap_s(slot_f(s ^ 1, MS_SCAL)[1]);
+                snap_s(slot_f(s ^ 1, MS_SCAL)[1], cb + r + 1);
             }
         }
         // final states: H_T (the TMEM state after the last chunk), S^K
@@ -831,6 +858,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             float *scal = slot_f(s, MS_SCAL);
             mbar_wait(&bar[BAR_IN0 + s], sp, abort_flag, status);
             if (r > 0) Mst[wt] = slot_f(s ^ 1, MS_MST)[wt] + dmprev[wt];
+            if (a.mk_out) a.mk_out[(static_cast<size_t>(bh) * NCt + cb + r) * kD + wt] = Mst[wt];
             const float lam_cur = lam_reg;
             if (wt < 64) scal[2 + wt] = g_reg;
             {
@@ -1066,7 +1094,7 @@ gdn_chunk_kernel(const __grid_constant__ CUtensorMap map_q, const __grid_constan
             named_bar(NB_OUT, kSyncCount);  // O of chunk r staged
             if (lead) {
                 uint8_t *st = sm + s * SLOT_BYTES + SO_KD;
-                if (!partial(r)) {
+                if (!partial(r) && !a.skip_o) {
                     tma_store_4d(&map_o, st, 0, h, tok0 + (cb + r) * kC, bt);
                     tma_store_4d(&map_o, st + 8192, 64, h, tok0 + (cb + r) * kC, bt);
                     tma_store_commit();

@@ -57,7 +57,7 @@ struct ChunkArgs {
     int seg_chunks = 0;
     float *seg_ws = nullptr;
     // GLA only: when set, the chunk-start states of every chunk are saved for the
-    // backward (layout below); skip_o suppresses the output write.
+    // backward (layout below).  skip_o suppresses the output write (both backbones).
     uint8_t *ckpt = nullptr;
     int skip_o = 0;
     // Packed variable-length sequences (cu != NULL): the batch index b is the sequence, B the
@@ -71,6 +71,11 @@ struct ChunkArgs {
     const int *cbase = nullptr;
     const int *chunk_seq = nullptr;
     int vl_chunks = 0;  // cbase[B]: the packed chunk count
+    // Gated DeltaNet, for the backward (no packed sequences): when set, the forward writes per
+    // chunk ch = (b H + h) NC + r of every (sequence, head), in fp32, what the backward reads:
+    // tt_out[ch][64][64] = Tt = (I + A)^{-1} (the WY kernel), and the states entering the chunk
+    // hs_out[ch][Dk][Dv] = H_r, sk_out[ch][Dk][Dk] = S^K_r, mk_out[ch][Dk] = M_r (the chunk kernel).
+    float *tt_out = nullptr, *hs_out = nullptr, *sk_out = nullptr, *mk_out = nullptr;
 };
 
 // Per (sequence, segment) workspace: S [128][128], C [128][128], m [128], D [128].

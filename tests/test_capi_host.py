@@ -186,9 +186,18 @@ def _gdn_bwd(lib, ptrs=None, sizes=(1, 70, 2, 64, 64), ws=None, ws_bytes=0, dtyp
 def test_gdn_bwd_workspace_size_and_rejections(lib):
     need = ctypes.c_size_t(0)
     p = ccq.params()
-    assert lib.ccq_gdn_bwd_workspace_size(4, 4096, 16, 128, 128, 0, ctypes.byref(p), ctypes.byref(need)) == 0
     chunks = 4 * 16 * 64
-    assert need.value == chunks * (64 * 64 + 5 * 128 * 128 + 2 * 128 + 6 * 64 * 128 + 4 * 64) * 4
+    arrays = chunks * (64 * 64 + 5 * 128 * 128 + 2 * 128 + 6 * 64 * 128 + 4 * 64) * 4
+    # fp32 inputs: the backward's per-chunk arrays only
+    assert lib.ccq_gdn_bwd_workspace_size(4, 4096, 16, 128, 128, 1, ctypes.byref(p), ctypes.byref(need)) == 0
+    assert need.value == arrays
+    # bf16 inputs with d = 128 also hold the tensor-core forward's workspace (from a 1 KB boundary),
+    # which recomputes the forward's per-chunk quantities
+    fwd = ctypes.c_size_t(0)
+    pf = ccq.params(algo="chunkwise")
+    assert lib.ccq_gdn_workspace_size(4, 4096, 16, 128, 128, 0, ctypes.byref(pf), ctypes.byref(fwd)) == 0
+    assert lib.ccq_gdn_bwd_workspace_size(4, 4096, 16, 128, 128, 0, ctypes.byref(p), ctypes.byref(need)) == 0
+    assert need.value == (arrays + 1023) // 1024 * 1024 + fwd.value
     assert lib.ccq_gdn_bwd_workspace_size(1, 0, 2, 64, 64, 1, ctypes.byref(p), ctypes.byref(need)) == 0
     assert need.value == 0
     assert lib.ccq_gdn_bwd_workspace_size(1, 64, 2, 96, 96, 1, ctypes.byref(p),
