@@ -269,10 +269,15 @@ CCQ_API ccq_status ccq_gla_bwd_workspace_size(int B, int T, int H, int Dk, int D
  *   dlambda   [B,T,H] fp32 (may be NULL);  dS0, dC0, dm0 fp32 (each may be NULL).
  *   workspace at least ccq_gdn_bwd_workspace_size() bytes (16-byte aligned): per
  *             64-token chunk of every (sequence, head), the chunk's forward states,
- *             state adjoints and intermediate tiles in fp32.
- * Supported: Dk = Dv in {64, 128}, bf16 or fp32 inputs; the kernels compute in fp32 on
- * the CUDA cores (seven launches; the algo parameter is ignored).  T = 0 copies the
- * final-state gradients to the initial-state ones.
+ *             state adjoints and intermediate tiles in fp32 (for bf16 inputs with
+ *             Dk = 128, followed by the chunkwise forward's own workspace).
+ * Supported: Dk = Dv in {64, 128}, bf16 or fp32 inputs.  The per-chunk forward quantities
+ * the adjoint needs (the UT factor (I + A)^{-1}, the entering S^K, M and H of every chunk)
+ * come, for bf16 inputs with Dk = 128, from the chunkwise tensor-core forward kernels of
+ * ccq_gdn_fwd (which write them in fp32 and no output; their segment split follows
+ * p->seq_split), and otherwise from three CUDA-core passes; the adjoint itself runs on the
+ * CUDA cores in fp32 (the algo parameter is ignored).  T = 0 copies the final-state
+ * gradients to the initial-state ones.
  */
 CCQ_API ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float *g,
                                const float *beta, const float *lambda, ccq_dtype in_dtype,
@@ -282,7 +287,8 @@ CCQ_API ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, cons
                                float *dS0, float *dC0, float *dm0, int B, int T, int H, int Dk, int Dv,
                                void *workspace, size_t workspace_bytes, const ccq_params *p, void *stream);
 
-/* Workspace bytes ccq_gdn_bwd needs for these sizes (0 when T = 0).  Host-only. */
+/* Workspace bytes ccq_gdn_bwd needs for these sizes (0 when T = 0).  Queries the device
+ * (the forward's segment split, bf16 with Dk = 128) but launches nothing. */
 CCQ_API ccq_status ccq_gdn_bwd_workspace_size(int B, int T, int H, int Dk, int Dv, ccq_dtype in_dtype,
                                               const ccq_params *p, size_t *bytes);
 
