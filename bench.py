@@ -86,7 +86,9 @@ def launches_per_step(kind, B, H, T, sms):
     split = gla_segments(B, H, T, sms) > 1
     fwd = 3 if split else 1
     gdn = 4 if split else 2
-    return {"gla": fwd + 1, "gdn": gdn + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3, "gdnbwd": gdn + 1 + 7}[kind]
+    # the Gated DeltaNet training step runs the forward twice (the step's forward, then the
+    # backward's recompute of the forward's per-chunk quantities) and four backward kernels
+    return {"gla": fwd + 1, "gdn": gdn + 1, "decode": 1 + 1, "glabwd": fwd + 1 + 3, "gdnbwd": 2 * gdn + 1 + 4}[kind]
 
 
 def algorithmic_bytes(kind, B, H, T, D):
@@ -154,8 +156,10 @@ STEP_KERNELS = {
     "decode_b256": ["decode_kernel"],
     "gla_bf16_4k_fwdbwd": ["gla_segment_state_kernel", "gla_segment_combine_kernel", "gla_chunk_kernel",
                            "gla_bwd_q_kernel", "gla_bwd_state_kernel", "gla_bwd_kv_kernel"],
-    "gdn_bf16_4k_fwdbwd": ["gdn_wy_kernel", "gdn_chunk_kernel", "gdn_bwd_prep_kernel", "gdn_bwd_prefix_kernel",
-                           "gdn_bwd_fstate_kernel", "gdn_bwd_local_kernel", "gdn_bwd_dstate_kernel",
+    # (the forward kernels run twice: the forward itself, then the backward's recompute of the
+    # forward's per-chunk quantities; segment-parallel at B = 4, H = 16)
+    "gdn_bf16_4k_fwdbwd": ["gdn_segment_state_kernel", "gdn_segment_combine_kernel", "gdn_wy_kernel",
+                           "gdn_chunk_kernel", "gdn_bwd_local_kernel", "gdn_bwd_dstate_kernel",
                            "gdn_bwd_suffix_kernel", "gdn_bwd_kv_kernel"],
     "gla_bf16_varlen64": ["gla_chunk_kernel"],
     "gdn_bf16_varlen64": ["gdn_wy_kernel", "gdn_chunk_kernel"],
@@ -199,7 +203,7 @@ def measured_traffic(kind, workload):
             e = t.get(k)
             if not e or e.get("source_sha") != source_sha(KERNEL_FILES[k]):
                 return None
-            total += e["dram_bytes_per_launch"]
+            total += e["dram_bytes_per_launch"] * e.get("launches_per_step", 1)
         return total
     except (OSError, ValueError, KeyError):
         return None
