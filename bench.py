@@ -64,7 +64,8 @@ KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_ker
                 "decode": "decode_kernel",
                 "glabwd": "whole step: forward (saving checkpoints) + gla_bwd_q_kernel + gla_bwd_state_kernel"
                           " + gla_bwd_kv_kernel",
-                "gdnbwd": "whole step: forward (gdn_wy_kernel + gdn_chunk_kernel) + the seven gdn_bwd_* kernels"}
+                "gdnbwd": "whole step: forward (gdn_wy_kernel + gdn_chunk_kernel), the backward's forward recompute,"
+                          " gdn_bwd_local_kernel + gdn_bwd_state_tc_kernel + gdn_bwd_suffix_kernel + gdn_bwd_kv_kernel"}
 
 
 def gla_segments(B, H, T, sms):
@@ -159,7 +160,7 @@ STEP_KERNELS = {
     # (the forward kernels run twice: the forward itself, then the backward's recompute of the
     # forward's per-chunk quantities; segment-parallel at B = 4, H = 16)
     "gdn_bf16_4k_fwdbwd": ["gdn_segment_state_kernel", "gdn_segment_combine_kernel", "gdn_wy_kernel",
-                           "gdn_chunk_kernel", "gdn_bwd_local_kernel", "gdn_bwd_dstate_kernel",
+                           "gdn_chunk_kernel", "gdn_bwd_local_kernel", "gdn_bwd_state_tc_kernel",
                            "gdn_bwd_suffix_kernel", "gdn_bwd_kv_kernel"],
     "gla_bf16_varlen64": ["gla_chunk_kernel"],
     "gdn_bf16_varlen64": ["gdn_wy_kernel", "gdn_chunk_kernel"],
@@ -171,6 +172,7 @@ KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kerne
                 "gdn_segment_state_kernel": "ccq_gdn_segment.cu", "gdn_segment_combine_kernel": "ccq_gdn_segment.cu", "recurrent": "ccq_recurrent.cu",
                 "decode_kernel": "ccq_recurrent.cu", "gla_bwd_state_kernel": "ccq_gla_bwd.cu",
                 "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu",
+                "gdn_bwd_state_tc_kernel": "ccq_gdn_bwd_state_tc.cu",
                 **{f"gdn_bwd_{n}_kernel": "ccq_gdn_bwd_kernels.cuh"
                    for n in ("prep", "prefix", "fstate", "local", "dstate", "suffix", "kv")}}
 

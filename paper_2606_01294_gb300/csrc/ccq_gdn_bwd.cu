@@ -3,6 +3,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "ccq_gdn_bwd_kernels.cuh"
 #include "ccq_gdn_bwd.h"
 
@@ -66,7 +68,12 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
         if ((e = launch_fstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
     }
     gdn_bwd_local_kernel<D, Tin><<<nch, kBwdThreads, local_smem<D>(), s>>>(a);
-    if ((e = launch_dstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
+    if (D == 128 && std::is_same<Tin, __nv_bfloat16>::value && a.states_ready) {
+        // bf16, Dk = 128: the reverse state pass on tensor cores
+        if ((e = launch_gdn_dstate_tc(a, a.k, s)) != cudaSuccess) return e;
+    } else if ((e = launch_dstate<D, Tin>(a, bh, s)) != cudaSuccess) {
+        return e;
+    }
     gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
     gdn_bwd_kv_kernel<D, Tin><<<nch, kBwdThreads, kv_smem<D>(), s>>>(a);
     return cudaGetLastError();

@@ -2,11 +2,16 @@
 // ccq_gdn_bwd.cu, and the decay-aligned-covariance forward, ccq_gdn_decayed.cu), used by the C ABI.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
 
 namespace ccq {
+
+namespace gbwd {
+struct GdnBwdArgs;
+}
 
 // Arguments of the CUDA-core CCQ-Gated-DeltaNet backward (ccq_gdn_bwd.cu): the C ABI's
 // pointers as given (token tensors [B][T][H][D] in bf16 or fp32, D = Dk = Dv) and a
@@ -30,6 +35,11 @@ size_t gdn_bwd_workspace_bytes(int B, int T, int H, int D);
 // The workspace arrays of the forward's per-chunk quantities (layout: ChunkArgs::tt_out etc.).
 void gdn_bwd_state_arrays(const GdnBwdCall &c, float **tt, float **sk, float **mk, float **hs);
 cudaError_t launch_gdn_bwd(const GdnBwdCall &c, cudaStream_t s);
+// The reverse state pass on tensor cores (ccq_gdn_bwd_state_tc.cu): Dk = Dv = 128, bf16 keys k.
+cudaError_t launch_gdn_dstate_tc(const gbwd::GdnBwdArgs &a, const void *k, cudaStream_t s);
+// A 2-D tensor map over an fp32 [rows][cols] array with (box_cols x box_rows) boxes, 128-byte
+// swizzled (box_cols * 4 = 128).
+bool make_f32_rows_map(CUtensorMap *map, const void *base, long long rows, int cols, int box_cols, int box_rows);
 
 // Arguments of the CUDA-core CCQ-Gated-DeltaNet forward with the decay-aligned covariance
 // (ccq_gdn_decayed.cu); n0/nT are the decayed counts [B][H].
