@@ -7,6 +7,7 @@
 
 #include "ccq_gdn_bwd_kernels.cuh"
 #include "ccq_gdn_bwd.h"
+#include "ccq_internal.h"
 
 namespace ccq {
 
@@ -53,12 +54,16 @@ cudaError_t launch_dstate(const gbwd::GdnBwdArgs &a, unsigned bh, cudaStream_t s
 }
 
 template <int D, typename Tin>
-cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
+cudaError_t run(gbwd::GdnBwdArgs a, cudaStream_t s) {
     using namespace gbwd;
+    // bf16 inputs: the per-chunk kernels' products on the tensor cores (bf16 operands, the
+    // forward's precision); fp32 inputs keep fp32 products on the CUDA cores
+    constexpr bool kTc = std::is_same<Tin, __nv_bfloat16>::value;
     cudaError_t e;
+    if (kTc && !(a.status = device_status_word())) return cudaErrorInvalidValue;
     if ((e = allow_smem(gdn_bwd_prep_kernel<D, Tin>, prep_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_local_kernel<D, Tin>, local_smem<D>())) != cudaSuccess) return e;
-    if ((e = allow_smem(gdn_bwd_kv_kernel<D, Tin>, kv_smem<D>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_local_kernel<D, Tin, kTc>, local_smem<D, kTc>())) != cudaSuccess) return e;
+    if ((e = allow_smem(gdn_bwd_kv_kernel<D, Tin, kTc>, kv_smem<D, kTc>())) != cudaSuccess) return e;
     const unsigned nch = static_cast<unsigned>(a.B * a.H * a.NC), bh = static_cast<unsigned>(a.B * a.H);
     const long long elems = (static_cast<long long>(D) * D + D) * a.B * a.H;
     const unsigned eblocks = static_cast<unsigned>((elems + 255) / 256);
@@ -67,7 +72,7 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
         gdn_bwd_prefix_kernel<D><<<eblocks, 256, 0, s>>>(a);
         if ((e = launch_fstate<D, Tin>(a, bh, s)) != cudaSuccess) return e;
     }
-    gdn_bwd_local_kernel<D, Tin><<<nch, kBwdThreads, local_smem<D>(), s>>>(a);
+    gdn_bwd_local_kernel<D, Tin, kTc><<<nch, kBwdThreads, local_smem<D, kTc>(), s>>>(a);
     if (D == 128 && std::is_same<Tin, __nv_bfloat16>::value && a.states_ready) {
         // bf16, Dk = 128: the reverse state pass on tensor cores
         if ((e = launch_gdn_dstate_tc(a, a.k, s)) != cudaSuccess) return e;
@@ -75,7 +80,7 @@ cudaError_t run(const gbwd::GdnBwdArgs &a, cudaStream_t s) {
         return e;
     }
     gdn_bwd_suffix_kernel<D><<<eblocks, 256, 0, s>>>(a);
-    gdn_bwd_kv_kernel<D, Tin><<<nch, kBwdThreads, kv_smem<D>(), s>>>(a);
+    gdn_bwd_kv_kernel<D, Tin, kTc><<<nch, kBwdThreads, kv_smem<D, kTc>(), s>>>(a);
     return cudaGetLastError();
 }
 

@@ -45,6 +45,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "ccq_gdn_bwd_tc.cuh"
+
 namespace ccq {
 namespace gbwd {
 
@@ -90,6 +92,7 @@ struct GdnBwdArgs {
                           // delta rule acts on the columns of H independently, so each
                           // (sequence, head) runs as nsplit CTAs of D / nsplit columns
     int states_ready = 0; // tt, sk, mk, hs already hold Tt, S^K_r, M_r, H_r (from the forward)
+    int *status = nullptr; // status word of the tensor-core products' bounded waits (TC kernels)
 };
 
 __device__ __forceinline__ size_t tok_row(const GdnBwdArgs &a, int b, int t, int h) {
@@ -225,6 +228,27 @@ template <int M, int N, int VT, typename Ep>
 __device__ __forceinline__ void mm(const float *A, int ars, int acs, const float *B, int brs, int bcs, int K, Ep ep) {
     using S = MmShape<M, N, VT>;
     tile_mm<S::TM, S::TN, S::GN, VT>(A, ars, acs, B, brs, bcs, K, ep, M);
+}
+
+// An M x N x K product of the per-chunk kernels: on the tensor core (tc_mm, bf16 operands) in
+// their TC instantiation, else tile_mm on the CUDA cores.
+template <bool TC, int M, int N, int K, typename Ep>
+__device__ __forceinline__ void gmm(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs,
+                                    Ep ep) {
+    if constexpr (TC) {
+        tc_mm<M, N, K>(e, A, ars, acs, B, brs, bcs, ep);
+    } else {
+        (void)e;
+        mm<M, N, kBwdThreads>(A, ars, acs, B, brs, bcs, K, ep);
+    }
+}
+
+// v[0..NV) to dst[0..NV) as 16-byte stores (dst 16-byte aligned, NV a multiple of 4).
+template <int NV>
+__device__ __forceinline__ void st_row(float *dst, const float (&v)[NV]) {
+    float4 *d4 = reinterpret_cast<float4 *>(dst);
+#pragma unroll
+    for (int q = 0; q < NV / 4; ++q) d4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
 }
 
 // ---------------------------------------------------------------------------------------------
@@ -392,7 +416,7 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
 // (tile_mm over [64][D + 1] and [64][65] tiles); the D x D operands H and S^K are staged a row
 // block at a time through a tile that is free at that point, and z waits in the W slot of the
 // workspace while its tile holds D.
-template <int D, typename Tin>
+template <int D, typename Tin, bool TC = false>
 __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
     constexpr int LD = D + 1, LC = kC + 1, VT = kBwdThreads;
@@ -411,6 +435,8 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     float *rq = tinv + kC, *rk = rq + kC, *cq = rk + kC, *cz = cq + kC, *gqh = cz + kC;
     float *rdot = gqh + kC;
     float *M = rdot + kC;          // [D] the key sum M_r entering the chunk
+    TcEng eng{};                   // TC: the tensor-core products' state, behind M
+    if constexpr (TC) tc_setup(eng, reinterpret_cast<uint8_t *>(M + D), tc_stage_bytes(D, D), a.status);
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
     const int n = min(kC, a.T - r * kC);
@@ -453,12 +479,12 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
             [&](int idx, float x) { sB[(idx / kC) * LC + idx % kC] = x * be[idx % kC]; });
     __syncthreads();
     // (Qbar Kbar^T) o causal;  R = V - diag(E) Kbar H over the row blocks of H
-    mm<kC, kC, VT>(Qb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
+    gmm<TC, kC, kC, D>(eng, Qb, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Zw, LD, H + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        mm<kC, D, VT>(Kb + RB * hf, LD, 1, Zw, LD, 1, RB, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
+        gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, Zw, LD, 1, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
     }
     __syncthreads();
     // cq_i = CumK_i . qbar_i with CumK_i = M + sum_{j<=i} kbar_j;  U = Tt diag(beta) R
@@ -471,20 +497,28 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     {
         float *Rg = a.r + t64;
         float *Ug = a.u + t64;
-        mm<kC, D, VT>(sB, LC, 1, Rq, LD, 1, kC, [&](int i, int j, float v) {
-            Ud[i * LD + j] = v;
-            Ug[i * D + j] = v;
-        });
+        if constexpr (TC) {
+            tc_mm_rows<kC, D, kC>(eng, sB, LC, 1, Rq, LD, 1, [&](int i, int j0, const auto &v) {
+#pragma unroll
+                for (int c = 0; c < static_cast<int>(sizeof(v) / sizeof(float)); ++c) Ud[i * LD + j0 + c] = v[c];
+                st_row(Ug + i * D + j0, v);
+            });
+        } else {
+            mm<kC, D, VT>(sB, LC, 1, Rq, LD, 1, kC, [&](int i, int j, float v) {
+                Ud[i * LD + j] = v;
+                Ug[i * D + j] = v;
+            });
+        }
         GBWD_FOR(idx, kC * D) Rg[idx] = Rq[(idx / D) * LD + idx % D];
     }
     // z = Sigma_t qbar (App. B form): (Qbar S^K + ((Qbar Kbar^T) o causal) Kbar) / t - c CumK cq / t^2
     __syncthreads();
-    mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
+    gmm<TC, kC, D, kC>(eng, sA, LC, 1, Kb, LD, 1, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        mm<kC, D, VT>(Qb + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
+        gmm<TC, kC, D, RB>(eng, Qb + RB * hf, LD, 1, Rq, LD, 1, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
     }
     __syncthreads();
     GBWD_FOR(j, D) {
@@ -511,7 +545,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     }
     __syncthreads();
     // P = (Qc Kbar^T) o Gamma o causal;  D (the scaled output adjoint) into z's tile
-    mm<kC, kC, VT>(Rq, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) {
+    gmm<TC, kC, kC, D>(eng, Rq, LD, 1, Kb, 1, LD, [&](int i, int j, float v) {
         sB[i * LC + j] = j <= i ? v * expf(gc[i] - gc[j]) : 0.f;
     });
     stream8(kC * D, [&](int idx) {
@@ -522,8 +556,11 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     // P^T D for the state pass;  dP = (D U^T) o Gamma o causal
     {
         float *X1 = a.x1 + t64;
-        mm<kC, D, VT>(sB, 1, LC, Zw, LD, 1, kC, [&](int i, int j, float v) { X1[i * D + j] = v; });
-        mm<kC, kC, VT>(Zw, LD, 1, Ud, 1, LD, D, [&](int i, int j, float v) {
+        if constexpr (TC)
+            tc_mm_rows<kC, D, kC>(eng, sB, 1, LC, Zw, LD, 1, [&](int i, int j0, const auto &v) { st_row(X1 + i * D + j0, v); });
+        else
+            mm<kC, D, VT>(sB, 1, LC, Zw, LD, 1, kC, [&](int i, int j, float v) { X1[i * D + j] = v; });
+        gmm<TC, kC, kC, D>(eng, Zw, LD, 1, Ud, 1, LD, [&](int i, int j, float v) {
             sA[i * LC + j] = (j <= i && i < n) ? v * expf(gc[i] - gc[j]) : 0.f;
         });
     }
@@ -534,18 +571,40 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     // (over row blocks of H in sB);  gqh_i = E_i rowsum((Qc H) o D)_i = sum_j qc_ij ((E D) H^T)_ij
     {
         float *Y1 = a.y1 + static_cast<size_t>(ch) * D * D;
-        mm<D, D, VT>(Rq, 1, LD, Zw, LD, 1, kC, [&](int p, int j, float v) { Y1[p * D + j] = v; });
-        mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] = v; });
+        if constexpr (TC)
+            tc_mm_rows<D, D, kC>(eng, Rq, 1, LD, Zw, LD, 1, [&](int p, int j0, const auto &v) { st_row(Y1 + p * D + j0, v); });
+        else
+            mm<D, D, VT>(Rq, 1, LD, Zw, LD, 1, kC, [&](int p, int j, float v) { Y1[p * D + j] = v; });
+        gmm<TC, kC, D, kC>(eng, sA, LC, 1, Kb, LD, 1, [&](int i, int j, float v) { Ud[i * LD + j] = v; });
     }
-    for (int nb = 0; nb < NN; ++nb) {
-        __syncthreads();
-        copy_rows<D>(sB, LD, H + static_cast<size_t>(RN * nb) * D, RN);
-        __syncthreads();
-        mm<kC, RN, VT>(Zw, LD, 1, sB, 1, LD, D, [&](int i, int j, float v) {
-            const int jg = RN * nb + j;
-            Ud[i * LD + jg] += v;
-            if (i < n) atomicAdd(&gqh[i], Rq[i * LD + jg] * v);
-        });
+    if constexpr (TC) {
+        // 64 rows of H at a time through the S/dP pair (free now), one N = 64 product each
+        for (int nb = 0; nb < D / 64; ++nb) {
+            __syncthreads();
+            copy_rows<D>(sA, LD, H + static_cast<size_t>(64 * nb) * D, 64);
+            __syncthreads();
+            tc_mm_rows<kC, 64, D>(eng, Zw, LD, 1, sA, 1, LD, [&](int i, int j0, const auto &v) {
+                float acc = 0.f;
+#pragma unroll
+                for (int c = 0; c < static_cast<int>(sizeof(v) / sizeof(float)); ++c) {
+                    const int jg = 64 * nb + j0 + c;
+                    Ud[i * LD + jg] += v[c];
+                    acc += Rq[i * LD + jg] * v[c];
+                }
+                if (i < n) atomicAdd(&gqh[i], acc);
+            });
+        }
+    } else {
+        for (int nb = 0; nb < NN; ++nb) {
+            __syncthreads();
+            copy_rows<D>(sB, LD, H + static_cast<size_t>(RN * nb) * D, RN);
+            __syncthreads();
+            mm<kC, RN, VT>(Zw, LD, 1, sB, 1, LD, D, [&](int i, int j, float v) {
+                const int jg = RN * nb + j;
+                Ud[i * LD + jg] += v;
+                if (i < n) atomicAdd(&gqh[i], Rq[i * LD + jg] * v);
+            });
+        }
     }
     __syncthreads();
     copy_rows<D>(Zw, LD, Wg, kC);  // z back from the W slot
@@ -566,7 +625,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     }
     __syncthreads();
     // (W Kbar^T) o causal
-    mm<kC, kC, VT>(Zw, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
+    gmm<TC, kC, kC, D>(eng, Zw, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     __syncthreads();
     // cz_i = CumK_i . dz_i = t_i (M . W_i + sum_{j<=i} W_i . kbar_j)
     GBWD_FOR(i, kC) {
@@ -578,12 +637,12 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     // dqbar = dqc + W S^K + ((W Kbar^T) o causal) Kbar - c CumK cz / t^2 (in place);
     // the chunk's increments DC += W^T Qbar and Dm += sum_i dCum_i,
     // dCum_i = -c (dz_i cq_i + qbar_i cz_i) / t_i^2
-    mm<kC, D, VT>(sB, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+    gmm<TC, kC, D, kC>(eng, sB, LC, 1, Kb, LD, 1, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        mm<kC, D, VT>(Zw + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+        gmm<TC, kC, D, RB>(eng, Zw + RB * hf, LD, 1, Rq, LD, 1, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     }
     __syncthreads();
     {
@@ -598,7 +657,10 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
             }
             dM[j] = -c * acc;
         }
-        mm<D, D, VT>(Zw, 1, LD, Qb, LD, 1, kC, [&](int p, int j, float v) { dC[p * D + j] = v; });
+        if constexpr (TC)
+            tc_mm_rows<D, D, kC>(eng, Zw, 1, LD, Qb, LD, 1, [&](int p, int j0, const auto &v) { st_row(dC + p * D + j0, v); });
+        else
+            mm<D, D, VT>(Zw, 1, LD, Qb, LD, 1, kC, [&](int p, int j, float v) { dC[p * D + j] = v; });
         float *vec = a.vec + static_cast<size_t>(ch) * 4 * kC;
         GBWD_FOR(i, kC) {
             vec[i] = cq[i];
@@ -622,6 +684,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
                 dq[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((Ud[i * LD + j] - Qb[i * LD + j] * rdot[i]) * rq[i]);
         }
     }
+    if constexpr (TC) tc_teardown(eng);
 }
 
 // Per sequence and head, chunks last to first: the adjoint dH of the state leaving every
@@ -740,7 +803,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a)
 // Every product runs as a register-tiled tile_mm over shared-memory operands; the [64][D]
 // tiles have the odd row stride D + 1 and the [64][64] ones 65, and the workspace operands
 // are staged through BF (and, for the D x D ones, 64 rows at a time through the S/dP pair).
-template <int D, typename Tin>
+template <int D, typename Tin, bool TC = false>
 __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
     constexpr int LD = D + 1, LC = kC + 1, VT = kBwdThreads;
@@ -754,12 +817,15 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     float *sA = BF + kC * LD;      // [64][LC] S, then dTb, then dA, then (Qbar Kbar^T) o causal
     float *sB = sA + kC * LC;      // [64][LC] dP, then M2, then dKK, then (W Kbar^T) o causal
     float *B2 = sA;                // sA and sB together: [64][LD] staging of 64 rows of dH or H
-    float *Tt = sB + kC * LC;      // [64][LC]
-    float *graw = Tt + kC * LC;
+    // [64][LC] Tt (TC: read from the workspace instead, which leaves room for the engine)
+    float *Tt = TC ? nullptr : sB + kC * LC;
+    float *graw = sB + (TC ? 1 : 2) * kC * LC;
     float *gc = graw + kC, *E = gc + kC, *ed = E + kC, *be = ed + kC, *tinv = be + kC;
     float *rk = tinv + kC, *prs = rk + kC, *pcs = prs + kC, *kd = pcs + kC, *gkh = kd + kC;
     float *rs = gkh + kC, *cs = rs + kC, *db1 = cs + kC, *rdot = db1 + kC, *dgc = rdot + kC;
     float *scal = dgc + kC;        // [4]: <dH, H>
+    TcEng eng{};                   // TC: the tensor-core products' state, behind scal
+    if constexpr (TC) tc_setup(eng, reinterpret_cast<uint8_t *>(scal + 4), tc_stage_bytes(kC, D), a.status);
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
     const int n = min(kC, a.T - r * kC);
@@ -774,12 +840,15 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     const float *vec = a.vec + static_cast<size_t>(ch) * 4 * kC;
     const float *cq = vec, *cz = vec + kC, *gqh = vec + 2 * kC;
     const float *ttg = a.tt + static_cast<size_t>(ch) * kC * kC;
+    const float *TtS = TC ? ttg : Tt;  // Tt as the products and the dbeta sums read it
+    constexpr int tld = TC ? kC : LC;
     const Tin *dout = static_cast<const Tin *>(a.dout);
     const Tin *vin = static_cast<const Tin *>(a.v);
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
 
     load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
-    stream8(kC * kC, [&](int idx) { return ttg[idx]; }, [&](int idx, float x) { Tt[(idx / kC) * LC + idx % kC] = x; });
+    if constexpr (!TC)
+        stream8(kC * kC, [&](int idx) { return ttg[idx]; }, [&](int idx, float x) { Tt[(idx / kC) * LC + idx % kC] = x; });
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -805,13 +874,13 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
         __syncthreads();
         copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        mm<kC, D, VT>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) {
+        gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, [&](int i, int j, float v) {
             dU[i * LD + j] = (hf ? dU[i * LD + j] : 0.f) + v;
         });
     }
     __syncthreads();
     // S = Qc Kbar^T (Qc in BF; S in the S/dP pair, free once the staging of dH is read)
-    mm<kC, kC, VT>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
+    gmm<TC, kC, kC, D>(eng, BF, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     // dU = X1 + diag(ed) t with t = Kbar dH, which also waits in dR for kd
     stream8(kC * D, [&](int idx) { return X1[idx]; }, [&](int idx, float x) {
         const int i = idx / D, j = idx % D;
@@ -837,12 +906,29 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     // dv = dR = diag(beta) Tt^T dU;  dP = (D U^T) o Gamma o causal
     {
         Tin *dv = static_cast<Tin *>(a.dv);
-        mm<kC, D, VT>(Tt, 1, LC, dU, LD, 1, kC, [&](int i, int j, float v) {
-            const float x = be[i] * v;
-            dR[i * LD + j] = x;
-            if (i < n) dv[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(x);
-        });
-        mm<kC, kC, VT>(BF, LD, 1, dK, 1, LD, D, [&](int i, int j, float v) {
+        if constexpr (TC) {
+            tc_mm_rows<kC, D, kC>(eng, TtS, 1, tld, dU, LD, 1, [&](int i, int j0, const auto &v) {
+                constexpr int nv = static_cast<int>(sizeof(v) / sizeof(float));
+                float x[nv];
+#pragma unroll
+                for (int c = 0; c < nv; ++c) {
+                    x[c] = be[i] * v[c];
+                    dR[i * LD + j0 + c] = x[c];
+                }
+                if (i < n) {
+                    Tin *dst = dv + tok_row(a, b, r * kC + i, h) * D + j0;
+#pragma unroll
+                    for (int c = 0; c < nv; ++c) dst[c] = from_f<Tin>(x[c]);
+                }
+            });
+        } else {
+            mm<kC, D, VT>(Tt, 1, LC, dU, LD, 1, kC, [&](int i, int j, float v) {
+                const float x = be[i] * v;
+                dR[i * LD + j] = x;
+                if (i < n) dv[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>(x);
+            });
+        }
+        gmm<TC, kC, kC, D>(eng, BF, LD, 1, dK, 1, LD, [&](int i, int j, float v) {
             sB[i * LC + j] = (j <= i && i < n) ? v * expf(gc[i] - gc[j]) : 0.f;
         });
     }
@@ -875,49 +961,74 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     // dK = dP^T Qc + diag(ed) U dH^T - diag(E) dR H^T (the last two over row blocks of dH, H)
     copy_rows<D>(BF, LD, Qcg, kC);
     __syncthreads();
-    mm<kC, D, VT>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] = v; });
+    gmm<TC, kC, D, kC>(eng, sB, 1, LC, BF, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] = v; });
     __syncthreads();
     copy_rows<D>(BF, LD, Ug, kC);
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        mm<kC, RB, VT>(BF, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
+        gmm<TC, kC, RB, D>(eng, BF, LD, 1, B2, 1, LD, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
         __syncthreads();
         copy_rows<D>(B2, LD, H + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        mm<kC, RB, VT>(dR, LD, 1, B2, 1, LD, D, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
+        gmm<TC, kC, RB, D>(eng, dR, LD, 1, B2, 1, LD, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
     }
     __syncthreads();
     copy_rows<D>(BF, LD, Rg, kC);
     __syncthreads();
     // dTb = dU R^T
-    mm<kC, kC, VT>(dU, LD, 1, BF, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = v; });
+    gmm<TC, kC, kC, D>(eng, dU, LD, 1, BF, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     __syncthreads();
     // dbeta (the Tb = Tt diag(beta) factor) = column sums of dTb o Tt;  M2 = Tt^T (dTb diag(beta))
     GBWD_FOR(j, kC) {
         float acc = 0.f;
-        for (int i = 0; i < kC; ++i) acc += sA[i * LC + j] * Tt[i * LC + j];
+        for (int i = 0; i < kC; ++i) acc += sA[i * LC + j] * TtS[i * tld + j];
         db1[j] = acc;
     }
-    mm<kC, kC, VT>(Tt, 1, LC, sA, LC, 1, kC, [&](int i, int j, float v) { sB[i * LC + j] = v * be[j]; });
+    gmm<TC, kC, kC, kC>(eng, TtS, 1, tld, sA, LC, 1, [&](int i, int j, float v) { sB[i * LC + j] = v * be[j]; });
     __syncthreads();
     // dA = strict_lower(-M2 Tt^T)
-    mm<kC, kC, VT>(sB, LC, 1, Tt, 1, LC, kC, [&](int i, int j, float v) { sA[i * LC + j] = j < i ? -v : 0.f; });
+    gmm<TC, kC, kC, kC>(eng, sB, LC, 1, TtS, 1, tld, [&](int i, int j, float v) { sA[i * LC + j] = j < i ? -v : 0.f; });
     __syncthreads();
     // dKK = diag(beta) (dA o Gamma);  rs_i = sum_j dA_ij Gamma_ij KK_ij (the dbeta of A);
     // rowsum(dA o A)_i = beta_i rs_i;  cs_j = colsum(dA o A)_j
-    mm<kC, kC, VT>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float kk) {
-        float v = 0.f;
-        if (j < i) {
-            const float gm = expf(gc[i] - gc[j]);
-            const float x = sA[i * LC + j] * gm * kk;
-            atomicAdd(&rs[i], x);
-            atomicAdd(&cs[j], be[i] * x);
-            v = sA[i * LC + j] * be[i] * gm;
+    if constexpr (TC) {
+        // the terms x of rs and cs wait in dU (free between dTb and the reverse sums below)
+        tc_mm<kC, kC, D>(eng, Kb, LD, 1, Kb, 1, LD, [&](int i, int j, float kk) {
+            float v = 0.f, x = 0.f;
+            if (j < i) {
+                const float gm = expf(gc[i] - gc[j]);
+                x = sA[i * LC + j] * gm * kk;
+                v = sA[i * LC + j] * be[i] * gm;
+            }
+            sB[i * LC + j] = v;
+            dU[i * LD + j] = x;
+        });
+        GBWD_FOR(t, 2 * kC) {
+            float acc = 0.f;
+            if (t < kC) {
+                for (int j = 0; j < t; ++j) acc += dU[t * LD + j];
+                rs[t] = acc;
+            } else {
+                const int j = t - kC;
+                for (int i = j + 1; i < kC; ++i) acc += be[i] * dU[i * LD + j];
+                cs[j] = acc;
+            }
         }
-        sB[i * LC + j] = v;
-    });
+    } else {
+        mm<kC, kC, VT>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float kk) {
+            float v = 0.f;
+            if (j < i) {
+                const float gm = expf(gc[i] - gc[j]);
+                const float x = sA[i * LC + j] * gm * kk;
+                atomicAdd(&rs[i], x);
+                atomicAdd(&cs[j], be[i] * x);
+                v = sA[i * LC + j] * be[i] * gm;
+            }
+            sB[i * LC + j] = v;
+        });
+    }
     __syncthreads();
     GBWD_FOR(idx, kC * kC) {
         const int i = idx / kC, j = idx % kC;
@@ -925,14 +1036,14 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     }
     __syncthreads();
     // dK += (dKK + dKK^T) Kbar
-    mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+    gmm<TC, kC, D, kC>(eng, sA, LC, 1, Kb, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     __syncthreads();
     // CCQ terms: (Qbar Kbar^T) o causal and (W Kbar^T) o causal
     copy_rows<D>(BF, LD, Qbg, kC);
     copy_rows<D>(dR, LD, Wg, kC);
     __syncthreads();
-    mm<kC, kC, VT>(BF, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
-    mm<kC, kC, VT>(dR, LD, 1, Kb, 1, LD, D, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
+    gmm<TC, kC, kC, D>(eng, BF, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
+    gmm<TC, kC, kC, D>(eng, dR, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     // reverse cumulative sums G_ij = sum_{l>=i} dCum_lj / (-c), dCum_l = -c (dz_l cq_l + qbar_l cz_l) / t_l^2,
     // dz_l = t_l W_l
     GBWD_FOR(j, D) {
@@ -944,8 +1055,8 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     }
     __syncthreads();
     // dK += QKc^T W + WKc^T Qbar + Dm - c G
-    mm<kC, D, VT>(sA, 1, LC, dR, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
-    mm<kC, D, VT>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) {
+    gmm<TC, kC, D, kC>(eng, sA, 1, LC, dR, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+    gmm<TC, kC, D, kC>(eng, sB, 1, LC, BF, LD, 1, [&](int i, int j, float v) {
         dK[i * LD + j] += v + Dm[j] - c * dU[i * LD + j];
     });
     // dK += Kbar (DC + DC^T), over the row blocks p of DC
@@ -956,7 +1067,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
             return DC[pg * D + j] + DC[j * D + pg];
         }, [&](int idx, float x) { B2[(idx / D) * LD + idx % D] = x; });
         __syncthreads();
-        mm<kC, D, VT>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+        gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     }
     __syncthreads();
     GBWD_FOR(i, kC) {
@@ -988,6 +1099,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
                 dk[tok_row(a, b, r * kC + i, h) * D + j] = from_f<Tin>((dK[i * LD + j] - Kb[i * LD + j] * rdot[i]) * rk[i]);
         }
     }
+    if constexpr (TC) tc_teardown(eng);
 }
 
 // Shared-memory bytes of each kernel.
@@ -995,8 +1107,8 @@ template <int D> constexpr size_t prep_smem() { return sizeof(float) * (kC * (D 
 template <int D, int NS> constexpr size_t fstate_smem() {
     return sizeof(float) * (D * (D / NS + 1) + kC * (D + 1) + 2 * kC * (D / NS + 1) + kC * (kC + 1) + 6 * kC);
 }
-template <int D> constexpr size_t local_smem() {
-    return sizeof(float) * (5 * kC * (D + 1) + 2 * kC * (kC + 1) + 12 * kC + D);
+template <int D, bool TC = false> constexpr size_t local_smem() {
+    return sizeof(float) * (5 * kC * (D + 1) + 2 * kC * (kC + 1) + 12 * kC + D) + (TC ? tc_smem_bytes(D, D) : 0);
 }
 template <int D, int NS> constexpr size_t dstate_smem() {
     return sizeof(float) * (2 * D * (D / NS + 1) + kC * (D + 1) + 2 * kC * (D / NS + 1) + kC * (kC + 1) + 6 * kC);
@@ -1009,8 +1121,9 @@ inline int seq_split(int B, int H) {
     while (ns < 4 && static_cast<long long>(B) * H * ns * 2 <= 304) ns *= 2;
     return ns;
 }
-template <int D> constexpr size_t kv_smem() {
-    return sizeof(float) * (5 * kC * (D + 1) + 3 * kC * (kC + 1) + 16 * kC + 4);
+template <int D, bool TC = false> constexpr size_t kv_smem() {
+    return sizeof(float) * (5 * kC * (D + 1) + (TC ? 2 : 3) * kC * (kC + 1) + 16 * kC + 4) +
+           (TC ? tc_smem_bytes(kC, D) : 0);
 }
 
 }  // namespace gbwd

@@ -1,0 +1,227 @@
+// ccq_gdn_bwd_tc.cuh -- the tensor-core product of the CCQ-Gated-DeltaNet backward's per-chunk
+// kernels (gdn_bwd_local_kernel and gdn_bwd_kv_kernel, instantiated with TC = true for bf16
+// inputs).
+//
+// Those kernels keep their operands as fp32 tiles in shared memory (row strides D + 1 and 65) and
+// evaluate some thirty small products a chunk,
+//   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   M in {64, 128}, N in {64, 128},
+// the same contract as tile_mm.  tc_mm runs one on the tensor core: the CTA's 512 threads convert
+// the operands sixteen reduction steps at a time into bf16 MN-major T64 slices (16 K-rows of 64
+// M- or N-columns, 128-byte swizzled; one 16-byte chunk of eight consecutive M or N a thread),
+// one thread issues a K = 16 tcgen05.mma of the slice into an fp32 TMEM accumulator, and the next
+// slice is converted into the second buffer while it runs.  Then every thread reads its share of
+// the accumulator (one row, N/8 or N/4 consecutive columns) and hands it to the epilogue.  The
+// operand strides are odd in shared memory, so the lanes of a warp (sixteen K-rows of two 8-row
+// groups 16 apart) convert without bank conflicts.  Operands may also be in global memory.
+//
+// Rounding: operands to bf16 (round to nearest even), accumulation in fp32 -- the precision of the
+// forward's tensor-core products.
+#pragma once
+
+#include <stdint.h>
+
+#ifdef __CUDACC__
+#include "sm100_ptx.cuh"
+#endif
+
+namespace ccq {
+namespace gbwd {
+
+// Per-CTA state of the tensor-core products: two staging buffers and their commit barriers, the
+// TMEM accumulator (128 columns), the give-up flag of the bounded waits and the status word.
+struct TcEng {
+    uint8_t *stage;
+    int stride;  // bytes between the two staging buffers
+    uint64_t *bar;
+    uint32_t *tmem_slot;
+    volatile int *abort;
+    int *status;
+    uint32_t tmem;
+    uint32_t commits0, commits1;  // products committed to bar[0], bar[1]
+    uint32_t slices;
+};
+
+// Bytes of one staging buffer for products up to M x N: one 16 x 64 bf16 slice per 64 rows or
+// columns.
+constexpr int tc_stage_bytes(int M, int N) { return (M / 64 + N / 64) * 2048; }
+// Shared memory the engine adds behind a kernel's own: 1024-byte alignment, two staging buffers,
+// two barriers, the TMEM address and the give-up flag.
+constexpr int tc_smem_bytes(int M, int N) { return 1024 + 2 * tc_stage_bytes(M, N) + 64; }
+constexpr int kTcCols = 128;
+
+#ifdef __CUDACC__
+
+// Set up (all threads): `region` is the first byte behind the kernel's own shared memory.
+__device__ __forceinline__ void tc_setup(TcEng &e, uint8_t *region, int stage_bytes, int *status) {
+    e.stage = smem_align1024(region);
+    e.stride = stage_bytes;
+    uint8_t *misc = e.stage + 2 * stage_bytes;
+    e.bar = reinterpret_cast<uint64_t *>(misc);
+    e.tmem_slot = reinterpret_cast<uint32_t *>(misc + 16);
+    e.abort = reinterpret_cast<volatile int *>(misc + 20);
+    e.status = status;
+    e.commits0 = e.commits1 = 0;
+    e.slices = 0;
+    if (threadIdx.x == 0) {
+        mbar_init(&e.bar[0], 1);
+        mbar_init(&e.bar[1], 1);
+        *e.abort = 0;
+        fence_barrier_init();
+    }
+    if (threadIdx.x < 32) tmem_alloc(e.tmem_slot, kTcCols);
+    __syncthreads();
+    tc_fence_after();
+    e.tmem = *e.tmem_slot;
+}
+
+// Tear down (all threads, uniform control flow): after a give-up, wait (bounded) for the
+// products still in flight, then free the TMEM.
+__device__ __forceinline__ void tc_teardown(TcEng &e) {
+    if (threadIdx.x == 0 && *e.abort) {
+        if (e.commits0) mbar_drain(&e.bar[0], (e.commits0 - 1) & 1);
+        if (e.commits1) mbar_drain(&e.bar[1], (e.commits1 - 1) & 1);
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        tc_fence_after();
+        tmem_dealloc(e.tmem, kTcCols);
+    }
+}
+
+// Wait until the last product issued from buffer b has completed.
+__device__ __forceinline__ void tc_wait_buf(TcEng &e, int b) {
+    const uint32_t c = b ? e.commits1 : e.commits0;
+    if (c) mbar_wait(&e.bar[b], (c - 1) & 1, e.abort, e.status);
+}
+
+// 16 fp32 columns of the thread's TMEM lane quadrant as two half-warps: threads 0-15 lanes 0-15 at
+// columns [c, c + NR), threads 16-31 the same lanes at [c + NR, c + 2 NR).
+template <int NR>
+__device__ __forceinline__ void tmem_ld16x2(uint32_t taddr, float (&v)[NR]);
+template <>
+__device__ __forceinline__ void tmem_ld16x2<8>(uint32_t taddr, float (&v)[8]) {
+    uint32_t r[8];
+    asm volatile("tcgen05.ld.sync.aligned.16x32bx2.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8], 8;"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+                   "=r"(r[7])
+                 : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+template <>
+__device__ __forceinline__ void tmem_ld16x2<16>(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.16x32bx2.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16], 16;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Convert reduction steps [k0, k0 + 16) of A (M x K) and B (N x K) into the MN-major slices of
+// buffer buf: A's M/64 slices first, then B's N/64.  Item it (one 16-byte chunk) is K-row
+// it % 16 of the 8-row group mc of its operand; a warp's two halves take groups 16 rows apart.
+template <int M, int N>
+__device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, int acs, const float *B, int brs,
+                                         int bcs, int k0) {
+    constexpr int kA = 2 * M, kItems = 2 * (M + N);
+    for (int it = static_cast<int>(threadIdx.x); it < kItems; it += static_cast<int>(blockDim.x)) {
+        const bool isA = it < kA;
+        const int j = isA ? it : it - kA;
+        const int k = j & 15, p = j >> 5;
+        const int mc = (p & 1) + ((p >> 1) << 2) + 2 * ((j >> 4) & 1);
+        const float *src = isA ? A + static_cast<long long>(k0 + k) * acs + static_cast<long long>(8 * mc) * ars
+                               : B + static_cast<long long>(k0 + k) * brs + static_cast<long long>(8 * mc) * bcs;
+        const int st = isA ? ars : bcs;
+        float f[8];
+#pragma unroll
+        for (int x = 0; x < 8; ++x) f[x] = src[static_cast<long long>(x) * st];
+        uint4 u;
+        u.x = pack_bf16(f[0], f[1]);
+        u.y = pack_bf16(f[2], f[3]);
+        u.z = pack_bf16(f[4], f[5]);
+        u.w = pack_bf16(f[6], f[7]);
+        uint8_t *dst = buf + (isA ? 0 : (M / 64) * 2048) + (mc >> 3) * 2048 + t64_chunk(k, mc & 7);
+        *reinterpret_cast<uint4 *>(dst) = u;
+    }
+}
+
+// The product (every thread of the 512-thread CTA calls it, operands complete and visible).
+// ep(i, j0, v) receives row i, columns [j0, j0 + NV) of the result in v[NV], NV = M N / 512; each
+// output is handed over once.  Returns after every thread's epilogue (a block barrier).
+template <int M, int N, int K, typename Ep>
+__device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, int acs, const float *B, int brs,
+                                           int bcs, Ep ep) {
+    static_assert((M == 64 || M == 128) && (N == 64 || N == 128) && K % 16 == 0 && K > 0, "tc_mm shape");
+    constexpr uint32_t kIdesc = make_idesc(M, N, 1, 1);
+    constexpr int kNV = M * N / 512;
+#pragma unroll 1
+    for (int ks = 0; ks < K / 16; ++ks) {
+        const int b = static_cast<int>(e.slices & 1u);
+        uint8_t *buf = e.stage + b * e.stride;  // e.stride >= tc_stage_bytes(M, N)
+        tc_wait_buf(e, b);
+        tc_stage<M, N>(buf, A, ars, acs, B, brs, bcs, 16 * ks);
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (threadIdx.x == 0 && !*e.abort) {
+            tc_fence_after();
+            const uint32_t sa = smem_addr(buf);
+            mma_bf16(e.tmem, make_desc(sa, 2048, 1024), make_desc(sa + (M / 64) * 2048, 2048, 1024), kIdesc,
+                     ks > 0 ? 1u : 0u);
+            mma_commit(&e.bar[b]);
+        }
+        if (b) ++e.commits1;
+        else ++e.commits0;
+        ++e.slices;
+    }
+    tc_wait_buf(e, static_cast<int>((e.slices - 1) & 1u));
+    tc_fence_after();
+    {
+        const int warp = static_cast<int>(threadIdx.x >> 5), lane = static_cast<int>(threadIdx.x & 31);
+        const int q = warp & 3, cg = warp >> 2;
+        const uint32_t tq = e.tmem + (static_cast<uint32_t>(32 * q) << 16) + static_cast<uint32_t>(cg * (N / 4));
+        float v[kNV];
+        if constexpr (M == 64) {
+            // rows 16q..16q+15 sit in TMEM lanes 32q..32q+15
+            tmem_ld16x2<kNV>(tq, v);
+            ep(16 * q + (lane & 15), cg * (N / 4) + (lane >> 4) * kNV, v);
+        } else {
+            if constexpr (kNV == 32) tmem_ld32(tq, v);
+            else tmem_ld16(tq, v);
+            ep(32 * q + lane, cg * (N / 4), v);
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+}
+
+// The same with an element-wise epilogue ep(i, j, value), as tile_mm calls it.
+template <int M, int N, int K, typename Ep>
+__device__ __forceinline__ void tc_mm(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs,
+                                      Ep ep) {
+    constexpr int kNV = M * N / 512;
+    tc_mm_rows<M, N, K>(e, A, ars, acs, B, brs, bcs, [&](int i, int j0, const float (&v)[kNV]) {
+#pragma unroll
+        for (int c = 0; c < kNV; ++c) ep(i, j0 + c, v[c]);
+    });
+}
+
+#else  // host builds of the kernels instantiate only TC = false: declarations for the parser
+
+template <typename X> void tc_setup(TcEng &, uint8_t *, int, X *);
+template <typename X> void tc_teardown(X &);
+template <int M, int N, int K, typename Ep>
+void tc_mm_rows(TcEng &, const float *, int, int, const float *, int, int, Ep);
+template <int M, int N, int K, typename Ep>
+void tc_mm(TcEng &, const float *, int, int, const float *, int, int, Ep);
+
+#endif
+
+}  // namespace gbwd
+}  // namespace ccq

@@ -2,10 +2,11 @@
 (itself pinned by finite differences and by an independent chunkwise adjoint), element by
 element.
 
-The kernels compute in fp32 on the CUDA cores, so fp32 inputs are held to the fp32 bar
-(max|g - ref| / max|ref| <= 1e-4) and bf16 inputs to the bf16 bar (2e-2, the outputs dq,
-dk, dv being rounded to bf16), for every gradient: dq, dk, dv, dg, dbeta, dlambda, dS0,
-dC0, dm0."""
+With fp32 inputs every product runs in fp32 on the CUDA cores, held to the fp32 bar
+(max|g - ref| / max|ref| <= 1e-4); with bf16 inputs the per-chunk products run on the tensor
+cores with bf16 operands (the forward's precision), held to the bf16 bar (2e-2, the outputs dq,
+dk, dv being rounded to bf16).  Every gradient is compared: dq, dk, dv, dg, dbeta, dlambda,
+dS0, dC0, dm0."""
 import numpy as np
 import pytest
 import torch
@@ -70,6 +71,29 @@ def test_bwd_bf16(keys):
     """bf16 inputs, D = 128, T = 130, from the zero state."""
     P, G = _problem(2, 130, 2, 128, dtype=torch.bfloat16, seed=32, keys=keys, prefix=0)
     _compare(_gpu(P, G), _ref(P, G), TOL[torch.bfloat16], keys)
+
+
+@pytest.mark.parametrize("D", [64, 128])
+@pytest.mark.parametrize("lam", ["init", "high"])
+def test_bwd_bf16_ragged_resumed(D, lam):
+    """bf16 inputs (tensor-core products), T = 200 (three chunks and an 8-token tail), resumed
+    from a 40-token state, with final-state gradients."""
+    P, G = _problem(2, 200, 3, D, dtype=torch.bfloat16, seed=51, lam=lam)
+    _compare(_gpu(P, G), _ref(P, G), TOL[torch.bfloat16], f"bf16 D={D} {lam}")
+
+
+@pytest.mark.parametrize("T", [1, 63, 65])
+def test_bwd_bf16_lengths(T):
+    """bf16 inputs: a single token, one short chunk, and a chunk plus one token."""
+    P, G = _problem(1, T, 2, 128, dtype=torch.bfloat16, seed=52 + T, prefix=40 if T == 1 else 0)
+    _compare(_gpu(P, G), _ref(P, G), TOL[torch.bfloat16], f"bf16 T={T}")
+
+
+@pytest.mark.parametrize("opts", [dict(centered=False), dict(l2norm=False)])
+def test_bwd_bf16_variants(opts):
+    """bf16 inputs with the uncentred covariance (App. D) and with un-normalised q, k."""
+    P, G = _problem(1, 150, 2, 128, dtype=torch.bfloat16, seed=56)
+    _compare(_gpu(P, G, **opts), _ref(P, G, **opts), TOL[torch.bfloat16], f"bf16 {opts}")
 
 
 @pytest.mark.parametrize("T", [1, 63, 64, 65])
