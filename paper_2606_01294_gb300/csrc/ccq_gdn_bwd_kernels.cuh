@@ -44,6 +44,7 @@
 #include <math.h>
 #include <stddef.h>
 #include <stdint.h>
+#include <string.h>
 
 #include "ccq_gdn_bwd_tc.cuh"
 
@@ -132,39 +133,113 @@ __device__ __forceinline__ void gate_prefix(const float *graw, float *gc) {
     }
 }
 
-// An element-wise pass over total elements whose loads come from global memory: the thread's
-// elements go eight at a time, all eight loads issued before the first store, so that a thread
-// keeps eight loads in flight instead of one.  ld(e) loads element e, st(e, x) stores it.
-template <typename L, typename S>
-__device__ __forceinline__ void stream8(int total, L ld, S st) {
+// An element-wise pass over total items whose loads come from global memory: the thread's
+// items go U at a time, all U loads issued before the first store (the last, fewer than U, the
+// same way), so that a thread keeps U loads in flight instead of one.  ld(e) loads item e,
+// st(e, x) stores it.
+template <int U, typename L, typename S>
+__device__ __forceinline__ void stream_u(int total, L ld, S st) {
+    using X = decltype(ld(0));
     const int stride = static_cast<int>(blockDim.x);
     int idx = static_cast<int>(threadIdx.x);
-    for (; idx + 7 * stride < total; idx += 8 * stride) {
-        float x[8];
+    for (; idx + (U - 1) * stride < total; idx += U * stride) {
+        X x[U];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) x[u] = ld(idx + u * stride);
+        for (int u = 0; u < U; ++u) x[u] = ld(idx + u * stride);
 #pragma unroll
-        for (int u = 0; u < 8; ++u) st(idx + u * stride, x[u]);
+        for (int u = 0; u < U; ++u) st(idx + u * stride, x[u]);
     }
-    for (; idx < total; idx += stride) st(idx, ld(idx));
+    X x[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+        if (idx + u * stride < total) x[u] = ld(idx + u * stride);
+#pragma unroll
+    for (int u = 0; u < U; ++u)
+        if (idx + u * stride < total) st(idx + u * stride, x[u]);
+}
+template <typename L, typename S>
+__device__ __forceinline__ void stream8(int total, L ld, S st) {
+    stream_u<8>(total, ld, st);
 }
 
-// Load the rows of chunk r of a [B][T][H][D] tensor into dst[64][ld] (zero past T).
+// 16-byte chunks of a [rows][CPR chunks] row-major array: chunk c is (row, column chunk).  With
+// CPR a multiple of 8 (rows a multiple of 4) the eight lanes of a warp quarter take consecutive
+// chunks of one row (128 contiguous bytes) and the four quarters four consecutive rows, so that
+// stores into a tile of odd row stride hit 32 different banks; narrower rows go in row order.
+template <int CPR>
+__device__ __forceinline__ void chunk_rc(int c, int &row, int &col_chunk) {
+    if constexpr (CPR % 8 == 0) {
+        const int w = c >> 5;
+        row = 4 * (w / (CPR / 8)) + ((c >> 3) & 3);
+        col_chunk = 8 * (w % (CPR / 8)) + (c & 7);
+    } else {
+        row = c / CPR;
+        col_chunk = c % CPR;
+    }
+}
+
+// Unpack 16 bytes holding 16 / sizeof(T) values of type T into floats.
+template <typename T>
+__device__ __forceinline__ void unpack16(const uint4 &u, float (&f)[16 / sizeof(T)]) {
+    T e[16 / sizeof(T)];
+    memcpy(e, &u, 16);
+#pragma unroll
+    for (int x = 0; x < static_cast<int>(16 / sizeof(T)); ++x) f[x] = to_f(e[x]);
+}
+
+// Load the rows of chunk r of a [B][T][H][D] tensor, times scale, into dst[64][ld] (zero past T):
+// 16-byte loads, all of a thread's issued before its stores.
 template <int D, typename Tin>
 __device__ __forceinline__ void load_tile_ld(float *dst, int ld, const void *src, const GdnBwdArgs &a, int b, int h,
-                                             int r) {
+                                             int r, float scale = 1.f) {
+    constexpr int V = 16 / sizeof(Tin), CPR = D / V;
     const Tin *s = static_cast<const Tin *>(src);
-    stream8(kC * D, [&](int idx) {
-        const int t = r * kC + idx / D;
-        return t < a.T ? to_f(s[tok_row(a, b, t, h) * D + idx % D]) : 0.f;
-    }, [&](int idx, float x) { dst[(idx / D) * ld + idx % D] = x; });
+    stream_u<4>(kC * CPR, [&](int c) {
+        int i, cc;
+        chunk_rc<CPR>(c, i, cc);
+        const int t = r * kC + i;
+        uint4 u = make_uint4(0u, 0u, 0u, 0u);
+        if (t < a.T) u = *reinterpret_cast<const uint4 *>(s + tok_row(a, b, t, h) * D + cc * V);
+        return u;
+    }, [&](int c, uint4 u) {
+        int i, cc;
+        chunk_rc<CPR>(c, i, cc);
+        float f[V];
+        unpack16<Tin>(u, f);
+        float *d = dst + i * ld + cc * V;
+#pragma unroll
+        for (int x = 0; x < V; ++x) d[x] = scale * f[x];
+    });
 }
 
-// dst[rows][ld] <- src[rows][COLS] (fp32, e.g. a workspace tile into shared memory).
+// A pass over rows [0, rows) and columns [0, COLS) of an fp32 array in global memory with row
+// stride sld (floats), 16 bytes at a time (src and sld 16-byte aligned, rows a multiple of 4), all
+// of a thread's loads issued before its stores: f(i, j0, x) gets row i, columns [j0, j0 + 4).
+template <int COLS, typename F>
+__device__ __forceinline__ void rows4(const float *src, int sld, int rows, F f) {
+    constexpr int CPR = COLS / 4;
+    stream_u<8>(rows * CPR, [&](int c) {
+        int i, cc;
+        chunk_rc<CPR>(c, i, cc);
+        return *reinterpret_cast<const float4 *>(src + static_cast<size_t>(i) * sld + 4 * cc);
+    }, [&](int c, float4 x) {
+        int i, cc;
+        chunk_rc<CPR>(c, i, cc);
+        f(i, 4 * cc, x);
+    });
+}
+
+// dst[rows][ld] <- src[rows][COLS] (fp32, e.g. a workspace tile into shared memory; src 16-byte
+// aligned, rows a multiple of 4).
 template <int COLS>
 __device__ __forceinline__ void copy_rows(float *dst, int ld, const float *src, int rows) {
-    stream8(rows * COLS, [&](int idx) { return src[idx]; },
-            [&](int idx, float x) { dst[(idx / COLS) * ld + idx % COLS] = x; });
+    rows4<COLS>(src, COLS, rows, [&](int i, int j0, float4 x) {
+        float *d = dst + i * ld + j0;
+        d[0] = x.x;
+        d[1] = x.y;
+        d[2] = x.z;
+        d[3] = x.w;
+    });
 }
 
 // row_rnorm over a [64][ld] tile.
@@ -175,6 +250,30 @@ __device__ __forceinline__ void row_rnorm_ld(const float *x, int ld, float *rn, 
         for (int c = 0; c < D; ++c) ss += x[i * ld + c] * x[i * ld + c];
         rn[i] = !l2norm ? 1.f : (ss > 0.f ? 1.f / sqrtf(fmaxf(ss, 1e-12f)) : 0.f);
     }
+}
+
+struct Pair4 {
+    float4 a, b;
+};
+
+// Row sums over the 64 rows of a chunk: out[i] += sum_{c < ncols} f(i, c), as eight work items a
+// row (a warp's items on 32 consecutive rows, so reads of a tile with odd row stride are free of
+// bank conflicts) combined by shared-memory atomics.  out must be zero before the preceding
+// barrier; the sums are complete after the next one.
+template <typename F>
+__device__ __forceinline__ void row_sums(float *out, int ncols, F f) {
+    GBWD_FOR(w, 8 * kC) {
+        const int i = w & (kC - 1), part = w / kC;
+        float acc = 0.f;
+        for (int c2 = part; c2 < ncols; c2 += 8) acc += f(i, c2);
+        atomicAdd(&out[i], acc);
+    }
+}
+
+// The l2 normalisation factor of a row from its sum of squares: 1/max(|x|, 1e-6), 0 for an
+// all-zero row (which normalises to itself and passes no gradient), or 1 when disabled.
+__device__ __forceinline__ float rnorm_of(float ss, int l2norm) {
+    return !l2norm ? 1.f : (ss > 0.f ? 1.f / sqrtf(fmaxf(ss, 1e-12f)) : 0.f);
 }
 
 // Register-tiled product of two operands in shared memory, computed by VT virtual threads
@@ -240,6 +339,30 @@ __device__ __forceinline__ void gmm(TcEng &e, const float *A, int ars, int acs, 
     } else {
         (void)e;
         mm<M, N, kBwdThreads>(A, ars, acs, B, brs, bcs, K, ep);
+    }
+}
+
+// Staging-buffer bytes of the two per-chunk kernels' tensor-core products (the local kernel's
+// D x D products, M = 128 when D = 128, stage 16 reduction steps at a time).
+template <int D> constexpr int local_tc_stage() {
+    return tc_stage_bytes(kC, D, kTcSliceK) > tc_stage_bytes(D, D, D == 128 ? 16 : kTcSliceK)
+               ? tc_stage_bytes(kC, D, kTcSliceK) : tc_stage_bytes(D, D, D == 128 ? 16 : kTcSliceK);
+}
+template <int D> constexpr int kv_tc_stage() { return tc_stage_bytes(kC, D, kTcSliceK); }
+
+// v[0..NV) to dst[0..NV) in the tensor's type as 16-byte stores (dst 16-byte aligned, NV a
+// multiple of 8).
+template <typename T, int NV>
+__device__ __forceinline__ void st_row_t(T *dst, const float (&v)[NV]) {
+    constexpr int E = 16 / sizeof(T);
+#pragma unroll
+    for (int q = 0; q < NV / E; ++q) {
+        T e[E];
+#pragma unroll
+        for (int x = 0; x < E; ++x) e[x] = from_f<T>(v[E * q + x]);
+        uint4 u;
+        memcpy(&u, e, 16);
+        reinterpret_cast<uint4 *>(dst)[q] = u;
     }
 }
 
@@ -417,7 +540,7 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
 // block at a time through a tile that is free at that point, and z waits in the W slot of the
 // workspace while its tile holds D.
 template <int D, typename Tin, bool TC = false>
-__global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwdArgs a) {
+__global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_local_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
     constexpr int LD = D + 1, LC = kC + 1, VT = kBwdThreads;
     constexpr int RB = D < 64 ? D : 64, NH = D / RB;      // row blocks of 64 (k-blocks)
@@ -435,8 +558,11 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     float *rq = tinv + kC, *rk = rq + kC, *cq = rk + kC, *cz = cq + kC, *gqh = cz + kC;
     float *rdot = gqh + kC;
     float *M = rdot + kC;          // [D] the key sum M_r entering the chunk
-    TcEng eng{};                   // TC: the tensor-core products' state, behind M
-    if constexpr (TC) tc_setup(eng, reinterpret_cast<uint8_t *>(M + D), tc_stage_bytes(D, D), a.status);
+    float *ssq = M + D, *ssk = ssq + kC, *dls = ssk + kC;  // row sums of squares, -dlambda
+    float *segs = dls + kC;        // [4][D] sums of kbar over the four 16-row segments
+    float *dMs = segs + 4 * D;     // [D] the Dm increment, accumulated
+    TcEng eng{};                   // TC: the tensor-core products' state, behind dMs
+    if constexpr (TC) tc_setup(eng, reinterpret_cast<uint8_t *>(dMs + D), local_tc_stage<D>(), kTcBufLocal, a.status);
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
     const int n = min(kC, a.T - r * kC);
@@ -447,7 +573,6 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     const float *Tt = a.tt + static_cast<size_t>(ch) * kC * kC;
     const size_t t64 = static_cast<size_t>(ch) * kC * D;
     float *Wg = a.w + t64;
-    const Tin *dout = static_cast<const Tin *>(a.dout);
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
 
     load_tile_ld<D, Tin>(Qb, LD, a.q, a, b, h, r);
@@ -460,24 +585,39 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
         be[i] = i < n ? a.beta[row] : 0.f;
         lam[i] = i < n ? a.lambda[row] : 0.f;
         tinv[i] = 1.f / (t_start + 1.f + static_cast<float>(i));
-        gqh[i] = 0.f;
+        gqh[i] = cq[i] = cz[i] = rdot[i] = ssq[i] = ssk[i] = dls[i] = 0.f;
     }
-    GBWD_FOR(j, D) M[j] = Mg[j];
+    GBWD_FOR(j, D) {
+        M[j] = Mg[j];
+        dMs[j] = 0.f;
+    }
     __syncthreads();
-    row_rnorm_ld<D>(Qb, LD, rq, a.l2norm);
-    row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
+    row_sums(ssq, D, [&](int i, int l) { return Qb[i * LD + l] * Qb[i * LD + l]; });
+    row_sums(ssk, D, [&](int i, int l) { return Kb[i * LD + l] * Kb[i * LD + l]; });
     gate_prefix(graw, gc);
+    __syncthreads();
+    GBWD_FOR(i, kC) {
+        E[i] = expf(gc[i]);
+        rq[i] = rnorm_of(ssq[i], a.l2norm);
+        rk[i] = rnorm_of(ssk[i], a.l2norm);
+    }
     __syncthreads();
     GBWD_FOR(idx, kC * D) {
         const int i = idx / D, j = idx % D;
         Qb[i * LD + j] *= rq[i];
         Kb[i * LD + j] *= rk[i];
     }
-    GBWD_FOR(i, kC) E[i] = expf(gc[i]);
     // Tt diag(beta) for U (be is visible after the barrier above)
     stream8(kC * kC, [&](int idx) { return Tt[idx]; },
             [&](int idx, float x) { sB[(idx / kC) * LC + idx % kC] = x * be[idx % kC]; });
     __syncthreads();
+    // the segment sums of kbar, for CumK_i = M + sum_{j<=i} kbar_j
+    GBWD_FOR(w, 4 * D) {
+        const int j = w % D, sg = w / D;
+        float acc = 0.f;
+        for (int i = 16 * sg; i < 16 * sg + 16; ++i) acc += Kb[i * LD + j];
+        segs[sg * D + j] = acc;
+    }
     // (Qbar Kbar^T) o causal;  R = V - diag(E) Kbar H over the row blocks of H
     gmm<TC, kC, kC, D>(eng, Qb, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = j <= i ? v : 0.f; });
     for (int hf = 0; hf < NH; ++hf) {
@@ -488,12 +628,9 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     }
     __syncthreads();
     // cq_i = CumK_i . qbar_i with CumK_i = M + sum_{j<=i} kbar_j;  U = Tt diag(beta) R
-    GBWD_FOR(i, kC) {
-        float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += M[l] * Qb[i * LD + l];
-        for (int j = 0; j <= i; ++j) acc += sA[i * LC + j];
-        cq[i] = acc;
-    }
+    row_sums(cq, D + kC, [&](int i, int l) {
+        return l < D ? M[l] * Qb[i * LD + l] : (l - D <= i ? sA[i * LC + l - D] : 0.f);
+    });
     {
         float *Rg = a.r + t64;
         float *Ug = a.u + t64;
@@ -521,9 +658,11 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
         gmm<TC, kC, D, RB>(eng, Qb + RB * hf, LD, 1, Rq, LD, 1, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
     }
     __syncthreads();
-    GBWD_FOR(j, D) {
+    GBWD_FOR(w, 4 * D) {
+        const int j = w % D, sg = w / D;
         float cum = M[j];
-        for (int i = 0; i < kC; ++i) {
+        for (int s2 = 0; s2 < sg; ++s2) cum += segs[s2 * D + j];
+        for (int i = 16 * sg; i < 16 * sg + 16; ++i) {
             cum += Kb[i * LD + j];
             const float z = Zw[i * LD + j] * tinv[i] - c * cum * cq[i] * tinv[i] * tinv[i];
             Zw[i * LD + j] = z;
@@ -548,10 +687,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     gmm<TC, kC, kC, D>(eng, Rq, LD, 1, Kb, 1, LD, [&](int i, int j, float v) {
         sB[i * LC + j] = j <= i ? v * expf(gc[i] - gc[j]) : 0.f;
     });
-    stream8(kC * D, [&](int idx) {
-        const int i = idx / D;
-        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + idx % D]) : 0.f;
-    }, [&](int idx, float x) { Zw[(idx / D) * LD + idx % D] = x; });
+    load_tile_ld<D, Tin>(Zw, LD, a.dout, a, b, h, r, a.scale);
     __syncthreads();
     // P^T D for the state pass;  dP = (D U^T) o Gamma o causal
     {
@@ -610,12 +746,10 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     copy_rows<D>(Zw, LD, Wg, kC);  // z back from the W slot
     __syncthreads();
     // dlambda_i = -z_i . dqc_i
-    GBWD_FOR(i, kC) {
-        float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += Zw[i * LD + j] * Ud[i * LD + j];
-        if (i < n && a.dlambda) a.dlambda[tok_row(a, b, r * kC + i, h)] = -acc;
-    }
+    row_sums(dls, D, [&](int i, int j) { return Zw[i * LD + j] * Ud[i * LD + j]; });
     __syncthreads();
+    GBWD_FOR(i, kC)
+        if (i < n && a.dlambda) a.dlambda[tok_row(a, b, r * kC + i, h)] = -dls[i];
     // W = dz / t with dz = -lambda dqc
     GBWD_FOR(idx, kC * D) {
         const int i = idx / D, j = idx % D;
@@ -628,12 +762,9 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     gmm<TC, kC, kC, D>(eng, Zw, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     __syncthreads();
     // cz_i = CumK_i . dz_i = t_i (M . W_i + sum_{j<=i} W_i . kbar_j)
-    GBWD_FOR(i, kC) {
-        float acc = 0.f;
-        for (int l = 0; l < D; ++l) acc += M[l] * Zw[i * LD + l];
-        for (int j = 0; j <= i; ++j) acc += sB[i * LC + j];
-        cz[i] = acc / tinv[i];
-    }
+    row_sums(cz, D + kC, [&](int i, int l) {
+        return (l < D ? M[l] * Zw[i * LD + l] : (l - D <= i ? sB[i * LC + l - D] : 0.f)) / tinv[i];
+    });
     // dqbar = dqc + W S^K + ((W Kbar^T) o causal) Kbar - c CumK cz / t^2 (in place);
     // the chunk's increments DC += W^T Qbar and Dm += sum_i dCum_i,
     // dCum_i = -c (dz_i cq_i + qbar_i cz_i) / t_i^2
@@ -647,15 +778,16 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
     __syncthreads();
     {
         float *dC = a.dc + static_cast<size_t>(ch) * D * D;
-        float *dM = a.dm + static_cast<size_t>(ch) * D;
-        GBWD_FOR(j, D) {
+        GBWD_FOR(w, 4 * D) {
+            const int j = w % D, sg = w / D;
             float cum = M[j], acc = 0.f;
-            for (int i = 0; i < kC; ++i) {
+            for (int s2 = 0; s2 < sg; ++s2) cum += segs[s2 * D + j];
+            for (int i = 16 * sg; i < 16 * sg + 16; ++i) {
                 cum += Kb[i * LD + j];
                 Ud[i * LD + j] -= c * cum * cz[i] * tinv[i] * tinv[i];
                 acc += (Zw[i * LD + j] * cq[i] / tinv[i] + Qb[i * LD + j] * cz[i]) * tinv[i] * tinv[i];
             }
-            dM[j] = -c * acc;
+            atomicAdd(&dMs[j], acc);
         }
         if constexpr (TC)
             tc_mm_rows<D, D, kC>(eng, Zw, 1, LD, Qb, LD, 1, [&](int p, int j0, const auto &v) { st_row(dC + p * D + j0, v); });
@@ -670,11 +802,8 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_local_kernel(const GdnBwd
         }
     }
     __syncthreads();
-    GBWD_FOR(i, kC) {
-        float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += Qb[i * LD + j] * Ud[i * LD + j];
-        rdot[i] = a.l2norm ? acc : 0.f;
-    }
+    row_sums(rdot, D, [&](int i, int j) { return a.l2norm ? Qb[i * LD + j] * Ud[i * LD + j] : 0.f; });
+    GBWD_FOR(j, D) a.dm[static_cast<size_t>(ch) * D + j] = -c * dMs[j];
     __syncthreads();
     {
         Tin *dq = static_cast<Tin *>(a.dq);
@@ -804,7 +933,7 @@ __global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a)
 // tiles have the odd row stride D + 1 and the [64][64] ones 65, and the workspace operands
 // are staged through BF (and, for the D x D ones, 64 rows at a time through the S/dP pair).
 template <int D, typename Tin, bool TC = false>
-__global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
+__global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
     constexpr int LD = D + 1, LC = kC + 1, VT = kBwdThreads;
     constexpr int RB = D < 64 ? D : 64, NH = D / RB;  // row blocks of the D x D operands
@@ -824,8 +953,10 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     float *rk = tinv + kC, *prs = rk + kC, *pcs = prs + kC, *kd = pcs + kC, *gkh = kd + kC;
     float *rs = gkh + kC, *cs = rs + kC, *db1 = cs + kC, *rdot = db1 + kC, *dgc = rdot + kC;
     float *scal = dgc + kC;        // [4]: <dH, H>
-    TcEng eng{};                   // TC: the tensor-core products' state, behind scal
-    if constexpr (TC) tc_setup(eng, reinterpret_cast<uint8_t *>(scal + 4), tc_stage_bytes(kC, D), a.status);
+    float *ssk = scal + 4;         // row sums of squares of k
+    float *segs = ssk + kC;        // [4][D] segment sums of the reverse cumulative sums below
+    TcEng eng{};                   // TC: the tensor-core products' state, behind segs
+    if constexpr (TC) tc_setup(eng, reinterpret_cast<uint8_t *>(segs + 4 * D), kv_tc_stage<D>(), kTcBufKv, a.status);
 
     const int ch = blockIdx.x, r = ch % a.NC, bh = ch / a.NC, b = bh / a.H, h = bh % a.H;
     const int n = min(kC, a.T - r * kC);
@@ -842,8 +973,6 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     const float *ttg = a.tt + static_cast<size_t>(ch) * kC * kC;
     const float *TtS = TC ? ttg : Tt;  // Tt as the products and the dbeta sums read it
     constexpr int tld = TC ? kC : LC;
-    const Tin *dout = static_cast<const Tin *>(a.dout);
-    const Tin *vin = static_cast<const Tin *>(a.v);
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
 
     load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
@@ -855,19 +984,21 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
         graw[i] = i < n ? a.g[row] : 0.f;
         be[i] = i < n ? a.beta[row] : 0.f;
         tinv[i] = 1.f / (t_start + 1.f + static_cast<float>(i));
-        prs[i] = pcs[i] = kd[i] = gkh[i] = rs[i] = cs[i] = 0.f;
+        prs[i] = pcs[i] = kd[i] = gkh[i] = rs[i] = cs[i] = db1[i] = rdot[i] = ssk[i] = 0.f;
     }
     if (threadIdx.x == 0) scal[0] = 0.f;
     copy_rows<D>(BF, LD, Qcg, kC);
     __syncthreads();
-    row_rnorm_ld<D>(Kb, LD, rk, a.l2norm);
+    row_sums(ssk, D, [&](int i, int l) { return Kb[i * LD + l] * Kb[i * LD + l]; });
     gate_prefix(graw, gc);
     __syncthreads();
-    GBWD_FOR(idx, kC * D) Kb[(idx / D) * LD + idx % D] *= rk[idx / D];
     GBWD_FOR(i, kC) {
         E[i] = expf(gc[i]);
         ed[i] = expf(gc[kC - 1] - gc[i]);
+        rk[i] = rnorm_of(ssk[i], a.l2norm);
     }
+    __syncthreads();
+    GBWD_FOR(idx, kC * D) Kb[(idx / D) * LD + idx % D] *= rk[idx / D];
     __syncthreads();
     // dU = P^T D + Kd dH = X1 + diag(ed) Kbar dH, over the row blocks of dH
     for (int hf = 0; hf < NH; ++hf) {
@@ -882,26 +1013,22 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     // S = Qc Kbar^T (Qc in BF; S in the S/dP pair, free once the staging of dH is read)
     gmm<TC, kC, kC, D>(eng, BF, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     // dU = X1 + diag(ed) t with t = Kbar dH, which also waits in dR for kd
-    stream8(kC * D, [&](int idx) { return X1[idx]; }, [&](int idx, float x) {
-        const int i = idx / D, j = idx % D;
-        const float t = dU[i * LD + j];
-        dR[i * LD + j] = t;
-        dU[i * LD + j] = x + ed[i] * t;
+    rows4<D>(X1, D, kC, [&](int i, int j0, float4 x4) {
+        const float xs[4] = {x4.x, x4.y, x4.z, x4.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float t = dU[i * LD + j0 + e];
+            dR[i * LD + j0 + e] = t;
+            dU[i * LD + j0 + e] = xs[e] + ed[i] * t;
+        }
     });
     __syncthreads();
     // D (scaled output adjoint) and U for dP
-    stream8(kC * D, [&](int idx) {
-        const int i = idx / D;
-        return i < n ? a.scale * to_f(dout[tok_row(a, b, r * kC + i, h) * D + idx % D]) : 0.f;
-    }, [&](int idx, float x) { BF[(idx / D) * LD + idx % D] = x; });
+    load_tile_ld<D, Tin>(BF, LD, a.dout, a, b, h, r, a.scale);
     copy_rows<D>(dK, LD, Ug, kC);
     __syncthreads();
     // kd_i = rowsum(Kd o U dH^T)_i = U_i . (dU - P^T D)_i = ed_i U_i . t_i
-    GBWD_FOR(i, kC) {
-        float x = 0.f;
-        for (int l = 0; l < D; ++l) x += dK[i * LD + l] * dR[i * LD + l];
-        kd[i] = ed[i] * x;
-    }
+    row_sums(kd, D, [&](int i, int l) { return ed[i] * dK[i * LD + l] * dR[i * LD + l]; });
     __syncthreads();
     // dv = dR = diag(beta) Tt^T dU;  dP = (D U^T) o Gamma o causal
     {
@@ -915,11 +1042,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
                     x[c] = be[i] * v[c];
                     dR[i * LD + j0 + c] = x[c];
                 }
-                if (i < n) {
-                    Tin *dst = dv + tok_row(a, b, r * kC + i, h) * D + j0;
-#pragma unroll
-                    for (int c = 0; c < nv; ++c) dst[c] = from_f<Tin>(x[c]);
-                }
+                if (i < n) st_row_t<Tin>(dv + tok_row(a, b, r * kC + i, h) * D + j0, x);
             });
         } else {
             mm<kC, D, VT>(Tt, 1, LC, dU, LD, 1, kC, [&](int i, int j, float v) {
@@ -934,29 +1057,20 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     }
     __syncthreads();
     // V - R (= diag(E) Kbar H) into BF for gkh;  <dH, H>
-    stream8(kC * D, [&](int idx) {
-        const int i = idx / D;
-        const float vv = i < n ? to_f(vin[tok_row(a, b, r * kC + i, h) * D + idx % D]) : 0.f;
-        return vv - Rg[idx];
-    }, [&](int idx, float x) { BF[(idx / D) * LD + idx % D] = x; });
-    {
-        float part = 0.f;
-        stream8(D * D, [&](int idx) { return dHg[idx] * H[idx]; }, [&](int, float x) { part += x; });
-        atomicAdd(&scal[0], part);
-    }
+    load_tile_ld<D, Tin>(BF, LD, a.v, a, b, h, r);
+    __syncthreads();
+    rows4<D>(Rg, D, kC, [&](int i, int j0, float4 x4) {
+        float *d = BF + i * LD + j0;
+        d[0] -= x4.x;
+        d[1] -= x4.y;
+        d[2] -= x4.z;
+        d[3] -= x4.w;
+    });
     __syncthreads();
     // row and column sums of dP o S;  gkh_i = (V - R)_i . dR_i
-    GBWD_FOR(i, kC) {
-        float p = 0.f, q = 0.f, y = 0.f;
-        for (int j = 0; j < kC; ++j) {
-            p += sB[i * LC + j] * sA[i * LC + j];
-            q += sB[j * LC + i] * sA[j * LC + i];
-        }
-        for (int l = 0; l < D; ++l) y += BF[i * LD + l] * dR[i * LD + l];
-        prs[i] = p;
-        pcs[i] = q;
-        gkh[i] = y;
-    }
+    row_sums(prs, kC, [&](int i, int j) { return sB[i * LC + j] * sA[i * LC + j]; });
+    row_sums(pcs, kC, [&](int i, int j) { return sB[j * LC + i] * sA[j * LC + i]; });
+    row_sums(gkh, D, [&](int i, int l) { return BF[i * LD + l] * dR[i * LD + l]; });
     __syncthreads();
     // dK = dP^T Qc + diag(ed) U dH^T - diag(E) dR H^T (the last two over row blocks of dH, H)
     copy_rows<D>(BF, LD, Qcg, kC);
@@ -970,7 +1084,30 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
         __syncthreads();
         gmm<TC, kC, RB, D>(eng, BF, LD, 1, B2, 1, LD, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] += ed[i] * v; });
         __syncthreads();
-        copy_rows<D>(B2, LD, H + static_cast<size_t>(RB * hf) * D, RB);
+        {
+            // these rows of H, and their part of <dH, H> (the rows of dH again, from L2)
+            constexpr int CPR = D / 4;
+            const float *Hb = H + static_cast<size_t>(RB * hf) * D, *dHb = dHg + static_cast<size_t>(RB * hf) * D;
+            float part = 0.f;
+            stream_u<4>(RB * CPR, [&](int c) {
+                int i, cc;
+                chunk_rc<CPR>(c, i, cc);
+                float4 x[2];
+                x[0] = *reinterpret_cast<const float4 *>(Hb + i * D + 4 * cc);
+                x[1] = *reinterpret_cast<const float4 *>(dHb + i * D + 4 * cc);
+                return Pair4{x[0], x[1]};
+            }, [&](int c, Pair4 p) {
+                int i, cc;
+                chunk_rc<CPR>(c, i, cc);
+                float *d = B2 + i * LD + 4 * cc;
+                d[0] = p.a.x;
+                d[1] = p.a.y;
+                d[2] = p.a.z;
+                d[3] = p.a.w;
+                part += p.a.x * p.b.x + p.a.y * p.b.y + p.a.z * p.b.z + p.a.w * p.b.w;
+            });
+            atomicAdd(&scal[0], part);
+        }
         __syncthreads();
         gmm<TC, kC, RB, D>(eng, dR, LD, 1, B2, 1, LD, [&](int i, int j, float v) { dK[i * LD + RB * hf + j] -= E[i] * v; });
     }
@@ -981,11 +1118,7 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     gmm<TC, kC, kC, D>(eng, dU, LD, 1, BF, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = v; });
     __syncthreads();
     // dbeta (the Tb = Tt diag(beta) factor) = column sums of dTb o Tt;  M2 = Tt^T (dTb diag(beta))
-    GBWD_FOR(j, kC) {
-        float acc = 0.f;
-        for (int i = 0; i < kC; ++i) acc += sA[i * LC + j] * TtS[i * tld + j];
-        db1[j] = acc;
-    }
+    row_sums(db1, kC, [&](int j, int i) { return sA[i * LC + j] * TtS[i * tld + j]; });
     gmm<TC, kC, kC, kC>(eng, TtS, 1, tld, sA, LC, 1, [&](int i, int j, float v) { sB[i * LC + j] = v * be[j]; });
     __syncthreads();
     // dA = strict_lower(-M2 Tt^T)
@@ -1005,17 +1138,8 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
             sB[i * LC + j] = v;
             dU[i * LD + j] = x;
         });
-        GBWD_FOR(t, 2 * kC) {
-            float acc = 0.f;
-            if (t < kC) {
-                for (int j = 0; j < t; ++j) acc += dU[t * LD + j];
-                rs[t] = acc;
-            } else {
-                const int j = t - kC;
-                for (int i = j + 1; i < kC; ++i) acc += be[i] * dU[i * LD + j];
-                cs[j] = acc;
-            }
-        }
+        row_sums(rs, kC, [&](int i, int j) { return dU[i * LD + j]; });
+        row_sums(cs, kC, [&](int j, int i) { return be[i] * dU[i * LD + j]; });
     } else {
         mm<kC, kC, VT>(Kb, LD, 1, Kb, 1, LD, D, [&](int i, int j, float kk) {
             float v = 0.f;
@@ -1046,10 +1170,22 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     gmm<TC, kC, kC, D>(eng, dR, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sB[i * LC + j] = j <= i ? v : 0.f; });
     // reverse cumulative sums G_ij = sum_{l>=i} dCum_lj / (-c), dCum_l = -c (dz_l cq_l + qbar_l cz_l) / t_l^2,
     // dz_l = t_l W_l
-    GBWD_FOR(j, D) {
+    auto dcum = [&](int l, int j) {
+        return (dR[l * LD + j] * cq[l] / tinv[l] + BF[l * LD + j] * cz[l]) * tinv[l] * tinv[l];
+    };
+    GBWD_FOR(w, 4 * D) {  // four 16-row segments: their sums, then the suffix sums within them
+        const int j = w % D, sg = w / D;
         float acc = 0.f;
-        for (int l = kC - 1; l >= 0; --l) {
-            acc += (dR[l * LD + j] * cq[l] / tinv[l] + BF[l * LD + j] * cz[l]) * tinv[l] * tinv[l];
+        for (int l = 16 * sg; l < 16 * sg + 16; ++l) acc += dcum(l, j);
+        segs[sg * D + j] = acc;
+    }
+    __syncthreads();
+    GBWD_FOR(w, 4 * D) {
+        const int j = w % D, sg = w / D;
+        float acc = 0.f;
+        for (int s2 = sg + 1; s2 < 4; ++s2) acc += segs[s2 * D + j];
+        for (int l = 16 * sg + 15; l >= 16 * sg; --l) {
+            acc += dcum(l, j);
             dU[l * LD + j] = acc;
         }
     }
@@ -1062,18 +1198,20 @@ __global__ void __launch_bounds__(kBwdThreads) gdn_bwd_kv_kernel(const GdnBwdArg
     // dK += Kbar (DC + DC^T), over the row blocks p of DC
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
-        stream8(RB * D, [&](int idx) {
-            const int p = idx / D, j = idx % D, pg = RB * hf + p;
-            return DC[pg * D + j] + DC[j * D + pg];
-        }, [&](int idx, float x) { B2[(idx / D) * LD + idx % D] = x; });
+        copy_rows<D>(B2, LD, DC + static_cast<size_t>(RB * hf) * D, RB);
+        __syncthreads();
+        rows4<RB>(DC + RB * hf, D, D, [&](int j, int p0, float4 x4) {
+            B2[p0 * LD + j] += x4.x;
+            B2[(p0 + 1) * LD + j] += x4.y;
+            B2[(p0 + 2) * LD + j] += x4.z;
+            B2[(p0 + 3) * LD + j] += x4.w;
+        });
         __syncthreads();
         gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     }
     __syncthreads();
+    row_sums(rdot, D, [&](int i, int j) { return a.l2norm ? Kb[i * LD + j] * dK[i * LD + j] : 0.f; });
     GBWD_FOR(i, kC) {
-        float acc = 0.f;
-        for (int j = 0; j < D; ++j) acc += Kb[i * LD + j] * dK[i * LD + j];
-        rdot[i] = a.l2norm ? acc : 0.f;
         float x = be[i] * rs[i] - cs[i] + prs[i] - pcs[i] + gqh[i] - kd[i] - gkh[i];
         if (i == n - 1) {
             float sk = 0.f;
@@ -1108,8 +1246,10 @@ template <int D, int NS> constexpr size_t fstate_smem() {
     return sizeof(float) * (D * (D / NS + 1) + kC * (D + 1) + 2 * kC * (D / NS + 1) + kC * (kC + 1) + 6 * kC);
 }
 template <int D, bool TC = false> constexpr size_t local_smem() {
-    return sizeof(float) * (5 * kC * (D + 1) + 2 * kC * (kC + 1) + 12 * kC + D) + (TC ? tc_smem_bytes(D, D) : 0);
+    return sizeof(float) * (5 * kC * (D + 1) + 2 * kC * (kC + 1) + 15 * kC + 6 * D) +
+           (TC ? tc_smem_bytes(local_tc_stage<D>(), kTcBufLocal) : 0);
 }
+static_assert(local_smem<128, true>() <= 232448, "local kernel shared memory");
 template <int D, int NS> constexpr size_t dstate_smem() {
     return sizeof(float) * (2 * D * (D / NS + 1) + kC * (D + 1) + 2 * kC * (D / NS + 1) + kC * (kC + 1) + 6 * kC);
 }
@@ -1122,9 +1262,10 @@ inline int seq_split(int B, int H) {
     return ns;
 }
 template <int D, bool TC = false> constexpr size_t kv_smem() {
-    return sizeof(float) * (5 * kC * (D + 1) + (TC ? 2 : 3) * kC * (kC + 1) + 16 * kC + 4) +
-           (TC ? tc_smem_bytes(kC, D) : 0);
+    return sizeof(float) * (5 * kC * (D + 1) + (TC ? 2 : 3) * kC * (kC + 1) + 17 * kC + 4 + 4 * D) +
+           (TC ? tc_smem_bytes(kv_tc_stage<D>(), kTcBufKv) : 0);
 }
+static_assert(kv_smem<128, true>() <= 232448, "kv kernel shared memory");
 
 }  // namespace gbwd
 }  // namespace ccq

@@ -6,10 +6,10 @@
 // evaluate some thirty small products a chunk,
 //   out(m, n) = sum_{k<K} A[m ars + k acs] B[k brs + n bcs],   M in {64, 128}, N in {64, 128},
 // the same contract as tile_mm.  tc_mm runs one on the tensor core: the CTA's 512 threads convert
-// the operands sixteen reduction steps at a time into bf16 MN-major T64 slices (16 K-rows of 64
-// M- or N-columns, 128-byte swizzled; one 16-byte chunk of eight consecutive M or N a thread),
-// one thread issues a K = 16 tcgen05.mma of the slice into an fp32 TMEM accumulator, and the next
-// slice is converted into the second buffer while it runs.  Then every thread reads its share of
+// the operands kTcSliceK reduction steps at a time into bf16 MN-major slices (SK K-rows of 64 M-
+// or N-columns, 128-byte swizzled; one 16-byte chunk of eight consecutive M or N a thread), one
+// thread issues the slice's K = 16 tcgen05.mma into an fp32 TMEM accumulator, and the next slices
+// are converted into the other staging buffers while it runs.  Then every thread reads its share of
 // the accumulator (one row, N/8 or N/4 consecutive columns) and hands it to the epilogue.  The
 // operand strides are odd in shared memory, so the lanes of a warp (sixteen K-rows of two 8-row
 // groups 16 apart) convert without bank conflicts.  Operands may also be in global memory.
@@ -31,40 +31,45 @@ namespace gbwd {
 // TMEM accumulator (128 columns), the give-up flag of the bounded waits and the status word.
 struct TcEng {
     uint8_t *stage;
-    int stride;  // bytes between the two staging buffers
-    uint64_t *bar;
+    int stride;  // bytes of one staging buffer
+    int nbuf;    // staging buffers (2 to 4), used in turn
+    uint64_t *bar;  // [nbuf] commit barriers
     uint32_t *tmem_slot;
     volatile int *abort;
     int *status;
     uint32_t tmem;
-    uint32_t commits0, commits1;  // products committed to bar[0], bar[1]
-    uint32_t slices;
+    uint32_t used, par;  // bit b: buffer b has a commit; the parity of its last commit
+    int next;            // the buffer the next slice goes to
 };
 
-// Bytes of one staging buffer for products up to M x N: one 16 x 64 bf16 slice per 64 rows or
-// columns.
-constexpr int tc_stage_bytes(int M, int N) { return (M / 64 + N / 64) * 2048; }
-// Shared memory the engine adds behind a kernel's own: 1024-byte alignment, two staging buffers,
-// two barriers, the TMEM address and the give-up flag.
-constexpr int tc_smem_bytes(int M, int N) { return 1024 + 2 * tc_stage_bytes(M, N) + 64; }
+// Reduction steps per staged slice (16 or 32; M = 128 products take 16).
+constexpr int kTcSliceK = 32;
+// Staging buffers of the local and the kv kernel.
+constexpr int kTcBufLocal = 2, kTcBufKv = 2;
+
+// Bytes of one staging slice of an M x N product: an SK x 64 bf16 tile per 64 rows or columns.
+constexpr int tc_stage_bytes(int M, int N, int SK) { return (M / 64 + N / 64) * SK * 128; }
+// Shared memory the engine adds behind a kernel's own: 1024-byte alignment, the staging buffers,
+// the barriers, the TMEM address and the give-up flag.
+constexpr int tc_smem_bytes(int stage, int nbuf) { return 1024 + nbuf * stage + 64; }
 constexpr int kTcCols = 128;
 
 #ifdef __CUDACC__
 
 // Set up (all threads): `region` is the first byte behind the kernel's own shared memory.
-__device__ __forceinline__ void tc_setup(TcEng &e, uint8_t *region, int stage_bytes, int *status) {
+__device__ __forceinline__ void tc_setup(TcEng &e, uint8_t *region, int stage_bytes, int nbuf, int *status) {
     e.stage = smem_align1024(region);
     e.stride = stage_bytes;
-    uint8_t *misc = e.stage + 2 * stage_bytes;
+    e.nbuf = nbuf;
+    uint8_t *misc = e.stage + nbuf * stage_bytes;
     e.bar = reinterpret_cast<uint64_t *>(misc);
-    e.tmem_slot = reinterpret_cast<uint32_t *>(misc + 16);
-    e.abort = reinterpret_cast<volatile int *>(misc + 20);
+    e.tmem_slot = reinterpret_cast<uint32_t *>(misc + 32);
+    e.abort = reinterpret_cast<volatile int *>(misc + 36);
     e.status = status;
-    e.commits0 = e.commits1 = 0;
-    e.slices = 0;
+    e.used = e.par = 0;
+    e.next = 0;
     if (threadIdx.x == 0) {
-        mbar_init(&e.bar[0], 1);
-        mbar_init(&e.bar[1], 1);
+        for (int b = 0; b < nbuf; ++b) mbar_init(&e.bar[b], 1);
         *e.abort = 0;
         fence_barrier_init();
     }
@@ -78,8 +83,8 @@ __device__ __forceinline__ void tc_setup(TcEng &e, uint8_t *region, int stage_by
 // products still in flight, then free the TMEM.
 __device__ __forceinline__ void tc_teardown(TcEng &e) {
     if (threadIdx.x == 0 && *e.abort) {
-        if (e.commits0) mbar_drain(&e.bar[0], (e.commits0 - 1) & 1);
-        if (e.commits1) mbar_drain(&e.bar[1], (e.commits1 - 1) & 1);
+        for (int b = 0; b < e.nbuf; ++b)
+            if ((e.used >> b) & 1u) mbar_drain(&e.bar[b], (e.par >> b) & 1u);
     }
     tc_fence_before();
     __syncthreads();
@@ -91,8 +96,7 @@ __device__ __forceinline__ void tc_teardown(TcEng &e) {
 
 // Wait until the last product issued from buffer b has completed.
 __device__ __forceinline__ void tc_wait_buf(TcEng &e, int b) {
-    const uint32_t c = b ? e.commits1 : e.commits0;
-    if (c) mbar_wait(&e.bar[b], (c - 1) & 1, e.abort, e.status);
+    if ((e.used >> b) & 1u) mbar_wait(&e.bar[b], (e.par >> b) & 1u, e.abort, e.status);
 }
 
 // 16 fp32 columns of the thread's TMEM lane quadrant as two half-warps: threads 0-15 lanes 0-15 at
@@ -124,18 +128,26 @@ __device__ __forceinline__ void tmem_ld16x2<16>(uint32_t taddr, float (&v)[16]) 
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
-// Convert reduction steps [k0, k0 + 16) of A (M x K) and B (N x K) into the MN-major slices of
-// buffer buf: A's M/64 slices first, then B's N/64.  Item it (one 16-byte chunk) is K-row
-// it % 16 of the 8-row group mc of its operand; a warp's two halves take groups 16 rows apart.
-template <int M, int N>
+// Convert reduction steps [k0, k0 + SK) of A (M x K) and B (N x K) into the MN-major SK x 64
+// tiles of buffer buf: A's M/64 tiles first, then B's N/64.  Item it (one 16-byte chunk) is K-row
+// k of the 8-row group mc of its operand: for SK = 32 a warp takes the 32 K-rows of one group,
+// for SK = 16 its two halves take groups 16 rows apart.
+template <int M, int N, int SK>
 __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, int acs, const float *B, int brs,
                                          int bcs, int k0) {
-    constexpr int kA = 2 * M, kItems = 2 * (M + N);
+    constexpr int kA = M / 8 * SK, kItems = (M + N) / 8 * SK, kTile = SK * 128;
     for (int it = static_cast<int>(threadIdx.x); it < kItems; it += static_cast<int>(blockDim.x)) {
         const bool isA = it < kA;
         const int j = isA ? it : it - kA;
-        const int k = j & 15, p = j >> 5;
-        const int mc = (p & 1) + ((p >> 1) << 2) + 2 * ((j >> 4) & 1);
+        int k, mc;
+        if constexpr (SK == 32) {
+            k = j & 31;
+            mc = j >> 5;
+        } else {
+            const int p = j >> 5;
+            k = j & 15;
+            mc = (p & 1) + ((p >> 1) << 2) + 2 * ((j >> 4) & 1);
+        }
         const float *src = isA ? A + static_cast<long long>(k0 + k) * acs + static_cast<long long>(8 * mc) * ars
                                : B + static_cast<long long>(k0 + k) * brs + static_cast<long long>(8 * mc) * bcs;
         const int st = isA ? ars : bcs;
@@ -147,7 +159,7 @@ __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, 
         u.y = pack_bf16(f[2], f[3]);
         u.z = pack_bf16(f[4], f[5]);
         u.w = pack_bf16(f[6], f[7]);
-        uint8_t *dst = buf + (isA ? 0 : (M / 64) * 2048) + (mc >> 3) * 2048 + t64_chunk(k, mc & 7);
+        uint8_t *dst = buf + (isA ? 0 : (M / 64) * kTile) + (mc >> 3) * kTile + t64_chunk(k, mc & 7);
         *reinterpret_cast<uint4 *>(dst) = u;
     }
 }
@@ -158,29 +170,35 @@ __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, 
 template <int M, int N, int K, typename Ep>
 __device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, int acs, const float *B, int brs,
                                            int bcs, Ep ep) {
-    static_assert((M == 64 || M == 128) && (N == 64 || N == 128) && K % 16 == 0 && K > 0, "tc_mm shape");
+    static_assert((M == 64 || M == 128) && (N == 64 || N == 128) && K % 32 == 0 && K > 0, "tc_mm shape");
+    constexpr int SK = M == 128 ? 16 : kTcSliceK;  // e.stride >= tc_stage_bytes(M, N, SK)
+    constexpr int kTile = SK * 128;
     constexpr uint32_t kIdesc = make_idesc(M, N, 1, 1);
     constexpr int kNV = M * N / 512;
+    int b = e.next;
 #pragma unroll 1
-    for (int ks = 0; ks < K / 16; ++ks) {
-        const int b = static_cast<int>(e.slices & 1u);
-        uint8_t *buf = e.stage + b * e.stride;  // e.stride >= tc_stage_bytes(M, N)
+    for (int ks = 0; ks < K / SK; ++ks) {
+        b = e.next;
+        e.next = e.next + 1 == e.nbuf ? 0 : e.next + 1;
+        uint8_t *buf = e.stage + b * e.stride;
         tc_wait_buf(e, b);
-        tc_stage<M, N>(buf, A, ars, acs, B, brs, bcs, 16 * ks);
+        tc_stage<M, N, SK>(buf, A, ars, acs, B, brs, bcs, SK * ks);
         fence_proxy_async_smem();
         __syncthreads();
         if (threadIdx.x == 0 && !*e.abort) {
             tc_fence_after();
             const uint32_t sa = smem_addr(buf);
-            mma_bf16(e.tmem, make_desc(sa, 2048, 1024), make_desc(sa + (M / 64) * 2048, 2048, 1024), kIdesc,
-                     ks > 0 ? 1u : 0u);
+#pragma unroll
+            for (int k16 = 0; k16 < SK / 16; ++k16)
+                mma_bf16(e.tmem, make_desc(sa + 2048 * k16, kTile, 1024),
+                         make_desc(sa + (M / 64) * kTile + 2048 * k16, kTile, 1024), kIdesc,
+                         (ks > 0 || k16 > 0) ? 1u : 0u);
             mma_commit(&e.bar[b]);
         }
-        if (b) ++e.commits1;
-        else ++e.commits0;
-        ++e.slices;
+        e.par = ((e.used >> b) & 1u) ? (e.par ^ (1u << b)) : (e.par & ~(1u << b));
+        e.used |= 1u << b;
     }
-    tc_wait_buf(e, static_cast<int>((e.slices - 1) & 1u));
+    tc_wait_buf(e, b);
     tc_fence_after();
     {
         const int warp = static_cast<int>(threadIdx.x >> 5), lane = static_cast<int>(threadIdx.x & 31);
@@ -214,7 +232,7 @@ __device__ __forceinline__ void tc_mm(TcEng &e, const float *A, int ars, int acs
 
 #else  // host builds of the kernels instantiate only TC = false: declarations for the parser
 
-template <typename X> void tc_setup(TcEng &, uint8_t *, int, X *);
+template <typename X> void tc_setup(TcEng &, uint8_t *, int, int, X *);
 template <typename X> void tc_teardown(X &);
 template <int M, int N, int K, typename Ep>
 void tc_mm_rows(TcEng &, const float *, int, int, const float *, int, int, Ep);
