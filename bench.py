@@ -58,7 +58,7 @@ def varlen_lengths(n):
     return np.random.default_rng(VARLEN_SEED).integers(100, 4001, size=n).tolist()
 KERNEL_SOURCES = {"gla": "ccq_gla_chunk.cu", "gdn": "ccq_gdn_chunk.cu", "decode": "ccq_recurrent.cu",
                   "glavl": "ccq_gla_chunk.cu", "gdnvl": "ccq_gdn_chunk.cu",
-                  "glabwd": "ccq_gla_bwd.cu", "gdnbwd": "ccq_gdn_bwd_kernels.cuh"}
+                  "glabwd": "ccq_gla_bwd.cu", "gdnbwd": ("ccq_gdn_bwd_kernels.cuh", "ccq_gdn_bwd_tc.cuh")}
 KERNEL_NAMES = {"gla": "gla_chunk_kernel", "gdn": "gdn_wy_kernel + gdn_chunk_kernel",
                 "glavl": "gla_chunk_kernel (packed sequences)", "gdnvl": "gdn_wy_kernel + gdn_chunk_kernel (packed sequences)",
                 "decode": "decode_kernel",
@@ -174,16 +174,17 @@ KERNEL_FILES = {"gla_chunk_kernel": "ccq_gla_chunk.cu", "gla_segment_state_kerne
                 "gla_bwd_q_kernel": "ccq_gla_bwd.cu", "gla_bwd_kv_kernel": "ccq_gla_bwd.cu",
                 "gdn_bwd_state_tc_kernel": "ccq_gdn_bwd_state_tc.cu",
                 **{f"gdn_bwd_{n}_kernel": "ccq_gdn_bwd_kernels.cuh"
-                   for n in ("prep", "prefix", "fstate", "local", "dstate", "suffix", "kv")}}
+                   for n in ("prep", "prefix", "fstate", "dstate", "suffix")},
+                **{f"gdn_bwd_{n}_kernel": ("ccq_gdn_bwd_kernels.cuh", "ccq_gdn_bwd_tc.cuh") for n in ("local", "kv")}}
 
 
 SHARED_DEVICE_SOURCES = ("sm100_ptx.cuh", "ccq_internal.h")  # inlined into every kernel
 
 
 def source_sha(fname):
-    """Hash of a kernel's source file and the device headers every kernel inlines."""
+    """Hash of a kernel's source file (or files) and the device headers every kernel inlines."""
     h = hashlib.sha256()
-    for f in (fname,) + SHARED_DEVICE_SOURCES:
+    for f in (fname if isinstance(fname, tuple) else (fname,)) + SHARED_DEVICE_SOURCES:
         with open(os.path.join(ROOT, "paper_2606_01294_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
