@@ -275,11 +275,13 @@ CCQ_API ccq_status ccq_gla_bwd_workspace_size(int B, int T, int H, int Dk, int D
  * the adjoint needs (the UT factor (I + A)^{-1}, the entering S^K, M and H of every chunk)
  * come, for bf16 inputs with Dk = 128, from the chunkwise tensor-core forward kernels of
  * ccq_gdn_fwd (which write them in fp32 and no output; their segment split follows
- * p->seq_split), and otherwise from three CUDA-core passes.  The adjoint's per-chunk kernels run
- * on the CUDA cores in fp32; its reverse pass over the state adjoint runs, for bf16 inputs with
- * Dk = 128, on the tensor cores (bf16 operands, fp32 accumulation), and otherwise on the CUDA
- * cores (the algo parameter is ignored).  T = 0 copies the final-state gradients to the
- * initial-state ones.
+ * p->seq_split), and otherwise from three CUDA-core passes.  The products of the adjoint's
+ * per-chunk kernels run, for bf16 inputs, on the tensor cores (bf16 operands, fp32 accumulation;
+ * their element-wise parts stay fp32) and, for fp32 inputs, on the CUDA cores in fp32; its reverse
+ * pass over the state adjoint runs, for bf16 inputs with Dk = 128, on the tensor cores, and
+ * otherwise on the CUDA cores (the algo parameter is ignored).  A bounded wait of the tensor-core
+ * kernels that gives up leaves the gradients invalid and CCQ_ERR_TIMEOUT for
+ * ccq_device_status().  T = 0 copies the final-state gradients to the initial-state ones.
  */
 CCQ_API ccq_status ccq_gdn_bwd(const void *q, const void *k, const void *v, const float *g,
                                const float *beta, const float *lambda, ccq_dtype in_dtype,

@@ -1,4 +1,5 @@
-// ccq_gdn_bwd_kernels.cuh -- CCQ-Gated-DeltaNet backward, CUDA-core kernels (fp32 arithmetic).
+// ccq_gdn_bwd_kernels.cuh -- CCQ-Gated-DeltaNet backward kernels (fp32 tiles; the per-chunk kernels'
+// products on the tensor cores for bf16 inputs).
 //
 // Reverse mode of the CCQ read (Eq. clean, Eq. read, the undecayed running sums of Sec. 3.2)
 // with the Gated DeltaNet write as the backbone, chunked as Algorithm 1 chunks the forward.
@@ -36,7 +37,9 @@
 //
 // Every kernel is a sequence of phases separated by __syncthreads(); inside a phase each
 // thread strides over the elements it owns and reads only what earlier phases wrote (row
-// reductions go through shared-memory atomics).  Arithmetic is fp32 on the CUDA cores.
+// reductions go through shared-memory atomics).  Arithmetic is fp32 on the CUDA cores, except
+// that the local and kv kernels instantiated with TC = true (bf16 inputs) run their products on
+// the tensor cores with bf16 operands and fp32 accumulation (tc_mm, ccq_gdn_bwd_tc.cuh).
 #pragma once
 
 #include <cuda_bf16.h>
@@ -536,7 +539,7 @@ __global__ void __launch_bounds__(512) gdn_bwd_fstate_kernel(const GdnBwdArgs a)
 
 // Per chunk, everything that does not need dH: z, qc, R, U, dqc, dq, dlambda, the CCQ
 // increments of DC and Dm, P^T D and (diag(E) Qc)^T D.  Products as in gdn_bwd_kv_kernel
-// (tile_mm over [64][D + 1] and [64][65] tiles); the D x D operands H and S^K are staged a row
+// (gmm over [64][D + 1] and [64][65] tiles); the D x D operands H and S^K are staged a row
 // block at a time through a tile that is free at that point, and z waits in the W slot of the
 // workspace while its tile holds D.
 template <int D, typename Tin, bool TC = false>
@@ -929,9 +932,10 @@ __global__ void __launch_bounds__(256) gdn_bwd_suffix_kernel(const GdnBwdArgs a)
 
 // Per chunk: dv, dk, dbeta, dg from the chunk's forward quantities (gdn_bwd_local_kernel),
 // the entering state H_r, the adjoint dH of the leaving state, and DC_{r+1}, Dm_{r+1}.
-// Every product runs as a register-tiled tile_mm over shared-memory operands; the [64][D]
-// tiles have the odd row stride D + 1 and the [64][64] ones 65, and the workspace operands
-// are staged through BF (and, for the D x D ones, 64 rows at a time through the S/dP pair).
+// Every product runs through gmm (tile_mm on the CUDA cores, or tc_mm on the tensor cores when
+// TC) over shared-memory operands; the [64][D] tiles have the odd row stride D + 1 and the
+// [64][64] ones 65, and the workspace operands are staged through BF (and, for the D x D ones,
+// 64 rows at a time through the S/dP pair).  With TC the kernel reads Tt from the workspace.
 template <int D, typename Tin, bool TC = false>
 __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_kv_kernel(const GdnBwdArgs a) {
     extern __shared__ float4 gbwd_smem4[];
