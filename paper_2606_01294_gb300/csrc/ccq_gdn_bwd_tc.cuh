@@ -8,11 +8,11 @@
 // the same contract as tile_mm.  tc_mm runs one on the tensor core: the CTA's 512 threads convert
 // the operands kTcSliceK reduction steps at a time into bf16 MN-major slices (SK K-rows of 64 M-
 // or N-columns, 128-byte swizzled; one 16-byte chunk of eight consecutive M or N a thread), one
-// thread issues the slice's K = 16 tcgen05.mma into an fp32 TMEM accumulator, and the next slices
-// are converted into the other staging buffers while it runs.  Then every thread reads its share of
+// thread issues the slice's K = 16 tcgen05.mma into an fp32 TMEM accumulator, and (with more than
+// one staging buffer) the next slice is converted while they run.  Then every thread reads its share of
 // the accumulator (one row, N/8 or N/4 consecutive columns) and hands it to the epilogue.  The
-// operand strides are odd in shared memory, so the lanes of a warp (sixteen K-rows of two 8-row
-// groups 16 apart) convert without bank conflicts.  Operands may also be in global memory.
+// operand strides are odd in shared memory, so the lanes of a warp (32 consecutive K-rows of one
+// 8-row group) convert without bank conflicts.  Operands may also be in global memory.
 //
 // Rounding: operands to bf16 (round to nearest even), accumulation in fp32 -- the precision of the
 // forward's tensor-core products.
@@ -32,7 +32,7 @@ namespace gbwd {
 struct TcEng {
     uint8_t *stage;
     int stride;  // bytes of one staging buffer
-    int nbuf;    // staging buffers (2 to 4), used in turn
+    int nbuf;    // staging buffers (1 to 4), used in turn
     uint64_t *bar;  // [nbuf] commit barriers
     uint32_t *tmem_slot;
     volatile int *abort;
@@ -42,10 +42,13 @@ struct TcEng {
     int next;            // the buffer the next slice goes to
 };
 
-// Reduction steps per staged slice (16 or 32; M = 128 products take 16).
-constexpr int kTcSliceK = 32;
-// Staging buffers of the local and the kv kernel.
-constexpr int kTcBufLocal = 2, kTcBufKv = 2;
+// Reduction steps per staged slice (16, 32 or 64; M = 128 products take 16), and the staging
+// buffers of the local and the kv kernel.  Measured on the backward (B=4, H=16, T=4096):
+// 16-deep slices in two buffers 7.82 ms, in three or four 7.83 ms, 32-deep in two 7.45 ms, and
+// (after the non-product phases were reworked) 32-deep in two 6.89 ms, 64-deep in one 6.33 ms:
+// each slice costs a conversion pass and a block barrier, the MMA round trip hardly shows.
+constexpr int kTcSliceK = 64;
+constexpr int kTcBufLocal = 1, kTcBufKv = 1;
 
 // Bytes of one staging slice of an M x N product: an SK x 64 bf16 tile per 64 rows or columns.
 constexpr int tc_stage_bytes(int M, int N, int SK) { return (M / 64 + N / 64) * SK * 128; }
@@ -130,8 +133,8 @@ __device__ __forceinline__ void tmem_ld16x2<16>(uint32_t taddr, float (&v)[16]) 
 
 // Convert reduction steps [k0, k0 + SK) of A (M x K) and B (N x K) into the MN-major SK x 64
 // tiles of buffer buf: A's M/64 tiles first, then B's N/64.  Item it (one 16-byte chunk) is K-row
-// k of the 8-row group mc of its operand: for SK = 32 a warp takes the 32 K-rows of one group,
-// for SK = 16 its two halves take groups 16 rows apart.
+// k of the 8-row group mc of its operand: for SK >= 32 a warp takes 32 consecutive K-rows of one
+// group, for SK = 16 its two halves take groups 16 rows apart.
 template <int M, int N, int SK>
 __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, int acs, const float *B, int brs,
                                          int bcs, int k0) {
@@ -140,9 +143,9 @@ __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, 
         const bool isA = it < kA;
         const int j = isA ? it : it - kA;
         int k, mc;
-        if constexpr (SK == 32) {
-            k = j & 31;
-            mc = j >> 5;
+        if constexpr (SK >= 32) {
+            k = j & (SK - 1);
+            mc = j / SK;
         } else {
             const int p = j >> 5;
             k = j & 15;
@@ -170,8 +173,8 @@ __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, 
 template <int M, int N, int K, typename Ep>
 __device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, int acs, const float *B, int brs,
                                            int bcs, Ep ep) {
-    static_assert((M == 64 || M == 128) && (N == 64 || N == 128) && K % 32 == 0 && K > 0, "tc_mm shape");
     constexpr int SK = M == 128 ? 16 : kTcSliceK;  // e.stride >= tc_stage_bytes(M, N, SK)
+    static_assert((M == 64 || M == 128) && (N == 64 || N == 128) && K % SK == 0 && K > 0, "tc_mm shape");
     constexpr int kTile = SK * 128;
     constexpr uint32_t kIdesc = make_idesc(M, N, 1, 1);
     constexpr int kNV = M * N / 512;
