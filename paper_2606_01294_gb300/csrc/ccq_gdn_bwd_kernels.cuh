@@ -215,6 +215,35 @@ __device__ __forceinline__ void load_tile_ld(float *dst, int ld, const void *src
     });
 }
 
+// load_tile_ld for three tensors at once (all of a thread's loads of the three issued before its
+// stores): the rows of chunk r of s0, s1, s2 into d0, d1, d2.
+template <int D, typename Tin>
+__device__ __forceinline__ void load_tiles3_ld(float *d0, float *d1, float *d2, int ld, const void *s0,
+                                               const void *s1, const void *s2, const GdnBwdArgs &a, int b, int h,
+                                               int r) {
+    constexpr int V = 16 / sizeof(Tin), CPR = D / V, PER = kC * CPR;
+    constexpr int U = 3 * ((PER + kBwdThreads - 1) / kBwdThreads);
+    stream_u<U>(3 * PER, [&](int c) {
+        const int tix = c / PER;
+        int i, cc;
+        chunk_rc<CPR>(c - tix * PER, i, cc);
+        const Tin *sp = static_cast<const Tin *>(tix == 0 ? s0 : (tix == 1 ? s1 : s2));
+        const int t = r * kC + i;
+        uint4 u = make_uint4(0u, 0u, 0u, 0u);
+        if (t < a.T) u = *reinterpret_cast<const uint4 *>(sp + tok_row(a, b, t, h) * D + cc * V);
+        return u;
+    }, [&](int c, uint4 u) {
+        const int tix = c / PER;
+        int i, cc;
+        chunk_rc<CPR>(c - tix * PER, i, cc);
+        float f[V];
+        unpack16<Tin>(u, f);
+        float *d = (tix == 0 ? d0 : (tix == 1 ? d1 : d2)) + i * ld + cc * V;
+#pragma unroll
+        for (int x = 0; x < V; ++x) d[x] = f[x];
+    });
+}
+
 // A pass over rows [0, rows) and columns [0, COLS) of an fp32 array in global memory with row
 // stride sld (floats), 16 bytes at a time (src and sld 16-byte aligned, rows a multiple of 4), all
 // of a thread's loads issued before its stores: f(i, j0, x) gets row i, columns [j0, j0 + 4).
@@ -578,9 +607,7 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_local_kernel(const Gdn
     float *Wg = a.w + t64;
     const float t_start = static_cast<float>((a.t0 ? a.t0[b] : 0) + static_cast<int64_t>(r) * kC);
 
-    load_tile_ld<D, Tin>(Qb, LD, a.q, a, b, h, r);
-    load_tile_ld<D, Tin>(Kb, LD, a.k, a, b, h, r);
-    load_tile_ld<D, Tin>(Rq, LD, a.v, a, b, h, r);
+    load_tiles3_ld<D, Tin>(Qb, Kb, Rq, LD, a.q, a.k, a.v, a, b, h, r);
     GBWD_FOR(i, kC) {
         const int t = r * kC + i;
         const size_t row = tok_row(a, b, t < a.T ? t : 0, h);
@@ -627,8 +654,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_local_kernel(const Gdn
         __syncthreads();
         copy_rows<D>(Zw, LD, H + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, Zw, LD, 1, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
+        if constexpr (TC)  // the row blocks' products sum in TMEM, read back once
+            tc_mma<kC, D, RB>(eng, Kb + RB * hf, LD, 1, Zw, LD, 1, hf > 0);
+        else
+            mm<kC, D, VT>(Kb + RB * hf, LD, 1, Zw, LD, 1, RB, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
     }
+    if constexpr (TC) tc_read_elem<kC, D>(eng, [&](int i, int j, float v) { Rq[i * LD + j] -= E[i] * v; });
     __syncthreads();
     // cq_i = CumK_i . qbar_i with CumK_i = M + sum_{j<=i} kbar_j;  U = Tt diag(beta) R
     row_sums(cq, D + kC, [&](int i, int l) {
@@ -653,13 +684,20 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_local_kernel(const Gdn
     }
     // z = Sigma_t qbar (App. B form): (Qbar S^K + ((Qbar Kbar^T) o causal) Kbar) / t - c CumK cq / t^2
     __syncthreads();
-    gmm<TC, kC, D, kC>(eng, sA, LC, 1, Kb, LD, 1, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
+    if constexpr (TC)
+        tc_mma<kC, D, kC>(eng, sA, LC, 1, Kb, LD, 1, false);
+    else
+        mm<kC, D, VT>(sA, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        gmm<TC, kC, D, RB>(eng, Qb + RB * hf, LD, 1, Rq, LD, 1, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
+        if constexpr (TC)
+            tc_mma<kC, D, RB>(eng, Qb + RB * hf, LD, 1, Rq, LD, 1, true);
+        else
+            mm<kC, D, VT>(Qb + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Zw[i * LD + j] += v; });
     }
+    if constexpr (TC) tc_read_elem<kC, D>(eng, [&](int i, int j, float v) { Zw[i * LD + j] = v; });
     __syncthreads();
     GBWD_FOR(w, 4 * D) {
         const int j = w % D, sg = w / D;
@@ -771,13 +809,20 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_local_kernel(const Gdn
     // dqbar = dqc + W S^K + ((W Kbar^T) o causal) Kbar - c CumK cz / t^2 (in place);
     // the chunk's increments DC += W^T Qbar and Dm += sum_i dCum_i,
     // dCum_i = -c (dz_i cq_i + qbar_i cz_i) / t_i^2
-    gmm<TC, kC, D, kC>(eng, sB, LC, 1, Kb, LD, 1, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+    if constexpr (TC)
+        tc_mma<kC, D, kC>(eng, sB, LC, 1, Kb, LD, 1, false);
+    else
+        mm<kC, D, VT>(sB, LC, 1, Kb, LD, 1, kC, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
         copy_rows<D>(Rq, LD, SK + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        gmm<TC, kC, D, RB>(eng, Zw + RB * hf, LD, 1, Rq, LD, 1, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
+        if constexpr (TC)
+            tc_mma<kC, D, RB>(eng, Zw + RB * hf, LD, 1, Rq, LD, 1, true);
+        else
+            mm<kC, D, VT>(Zw + RB * hf, LD, 1, Rq, LD, 1, RB, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     }
+    if constexpr (TC) tc_read_elem<kC, D>(eng, [&](int i, int j, float v) { Ud[i * LD + j] += v; });
     __syncthreads();
     {
         float *dC = a.dc + static_cast<size_t>(ch) * D * D;
@@ -1009,10 +1054,14 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_kv_kernel(const GdnBwd
         __syncthreads();
         copy_rows<D>(B2, LD, dHg + static_cast<size_t>(RB * hf) * D, RB);
         __syncthreads();
-        gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, [&](int i, int j, float v) {
-            dU[i * LD + j] = (hf ? dU[i * LD + j] : 0.f) + v;
-        });
+        if constexpr (TC)
+            tc_mma<kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, hf > 0);
+        else
+            mm<kC, D, VT>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) {
+                dU[i * LD + j] = (hf ? dU[i * LD + j] : 0.f) + v;
+            });
     }
+    if constexpr (TC) tc_read_elem<kC, D>(eng, [&](int i, int j, float v) { dU[i * LD + j] = v; });
     __syncthreads();
     // S = Qc Kbar^T (Qc in BF; S in the S/dP pair, free once the staging of dH is read)
     gmm<TC, kC, kC, D>(eng, BF, LD, 1, Kb, 1, LD, [&](int i, int j, float v) { sA[i * LC + j] = v; });
@@ -1195,10 +1244,16 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_kv_kernel(const GdnBwd
     }
     __syncthreads();
     // dK += QKc^T W + WKc^T Qbar + Dm - c G
-    gmm<TC, kC, D, kC>(eng, sA, 1, LC, dR, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] += v; });
-    gmm<TC, kC, D, kC>(eng, sB, 1, LC, BF, LD, 1, [&](int i, int j, float v) {
-        dK[i * LD + j] += v + Dm[j] - c * dU[i * LD + j];
-    });
+    if constexpr (TC) {
+        tc_mma<kC, D, kC>(eng, sA, 1, LC, dR, LD, 1, false);
+        tc_mma<kC, D, kC>(eng, sB, 1, LC, BF, LD, 1, true);
+        tc_read_elem<kC, D>(eng, [&](int i, int j, float v) { dK[i * LD + j] += v + Dm[j] - c * dU[i * LD + j]; });
+    } else {
+        mm<kC, D, VT>(sA, 1, LC, dR, LD, 1, kC, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+        mm<kC, D, VT>(sB, 1, LC, BF, LD, 1, kC, [&](int i, int j, float v) {
+            dK[i * LD + j] += v + Dm[j] - c * dU[i * LD + j];
+        });
+    }
     // dK += Kbar (DC + DC^T), over the row blocks p of DC
     for (int hf = 0; hf < NH; ++hf) {
         __syncthreads();
@@ -1211,8 +1266,12 @@ __global__ void __launch_bounds__(kBwdThreads, 1) gdn_bwd_kv_kernel(const GdnBwd
             B2[(p0 + 3) * LD + j] += x4.w;
         });
         __syncthreads();
-        gmm<TC, kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, [&](int i, int j, float v) { dK[i * LD + j] += v; });
+        if constexpr (TC)
+            tc_mma<kC, D, RB>(eng, Kb + RB * hf, LD, 1, B2, LD, 1, hf > 0);
+        else
+            mm<kC, D, VT>(Kb + RB * hf, LD, 1, B2, LD, 1, RB, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     }
+    if constexpr (TC) tc_read_elem<kC, D>(eng, [&](int i, int j, float v) { dK[i * LD + j] += v; });
     __syncthreads();
     row_sums(rdot, D, [&](int i, int j) { return a.l2norm ? Kb[i * LD + j] * dK[i * LD + j] : 0.f; });
     GBWD_FOR(i, kC) {

@@ -167,21 +167,20 @@ __device__ __forceinline__ void tc_stage(uint8_t *buf, const float *A, int ars, 
     }
 }
 
-// The product (every thread of the 512-thread CTA calls it, operands complete and visible).
-// ep(i, j0, v) receives row i, columns [j0, j0 + NV) of the result in v[NV], NV = M N / 512; each
-// output is handed over once.  Returns after every thread's epilogue (a block barrier).
-template <int M, int N, int K, typename Ep>
-__device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, int acs, const float *B, int brs,
-                                           int bcs, Ep ep) {
+// Stage and issue an M x N x K product into the TMEM accumulator (every thread of the 512-thread
+// CTA calls it, operands complete and visible): on top of what the accumulator holds when acc
+// (products chained this way sum), else in its place.  Nothing is read back; the operand tiles may
+// be overwritten as soon as it returns.
+template <int M, int N, int K>
+__device__ __forceinline__ void tc_mma(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs,
+                                       bool acc) {
     constexpr int SK = M == 128 ? 16 : kTcSliceK;  // e.stride >= tc_stage_bytes(M, N, SK)
     static_assert((M == 64 || M == 128) && (N == 64 || N == 128) && K % SK == 0 && K > 0, "tc_mm shape");
     constexpr int kTile = SK * 128;
     constexpr uint32_t kIdesc = make_idesc(M, N, 1, 1);
-    constexpr int kNV = M * N / 512;
-    int b = e.next;
 #pragma unroll 1
     for (int ks = 0; ks < K / SK; ++ks) {
-        b = e.next;
+        const int b = e.next;
         e.next = e.next + 1 == e.nbuf ? 0 : e.next + 1;
         uint8_t *buf = e.stage + b * e.stride;
         tc_wait_buf(e, b);
@@ -195,13 +194,21 @@ __device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, in
             for (int k16 = 0; k16 < SK / 16; ++k16)
                 mma_bf16(e.tmem, make_desc(sa + 2048 * k16, kTile, 1024),
                          make_desc(sa + (M / 64) * kTile + 2048 * k16, kTile, 1024), kIdesc,
-                         (ks > 0 || k16 > 0) ? 1u : 0u);
+                         (acc || ks > 0 || k16 > 0) ? 1u : 0u);
             mma_commit(&e.bar[b]);
         }
         e.par = ((e.used >> b) & 1u) ? (e.par ^ (1u << b)) : (e.par & ~(1u << b));
         e.used |= 1u << b;
     }
-    tc_wait_buf(e, b);
+}
+
+// Wait for the products issued so far and hand the M x N accumulator to the epilogue:
+// ep(i, j0, v) receives row i, columns [j0, j0 + NV) in v[NV], NV = M N / 512; each output is
+// handed over once.  Returns after every thread's epilogue (a block barrier).
+template <int M, int N, typename Ep>
+__device__ __forceinline__ void tc_read(TcEng &e, Ep ep) {
+    constexpr int kNV = M * N / 512;
+    for (int b = 0; b < e.nbuf; ++b) tc_wait_buf(e, b);
     tc_fence_after();
     {
         const int warp = static_cast<int>(threadIdx.x >> 5), lane = static_cast<int>(threadIdx.x & 31);
@@ -222,6 +229,24 @@ __device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, in
     __syncthreads();
 }
 
+// The element-wise form of tc_read: ep(i, j, value), as tile_mm calls it.
+template <int M, int N, typename Ep>
+__device__ __forceinline__ void tc_read_elem(TcEng &e, Ep ep) {
+    constexpr int kNV = M * N / 512;
+    tc_read<M, N>(e, [&](int i, int j0, const float (&v)[kNV]) {
+#pragma unroll
+        for (int c = 0; c < kNV; ++c) ep(i, j0 + c, v[c]);
+    });
+}
+
+// One product read back at once: ep as for tc_read.
+template <int M, int N, int K, typename Ep>
+__device__ __forceinline__ void tc_mm_rows(TcEng &e, const float *A, int ars, int acs, const float *B, int brs,
+                                           int bcs, Ep ep) {
+    tc_mma<M, N, K>(e, A, ars, acs, B, brs, bcs, false);
+    tc_read<M, N>(e, ep);
+}
+
 // The same with an element-wise epilogue ep(i, j, value), as tile_mm calls it.
 template <int M, int N, int K, typename Ep>
 __device__ __forceinline__ void tc_mm(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs,
@@ -239,6 +264,10 @@ template <typename X> void tc_setup(TcEng &, uint8_t *, int, int, X *);
 template <typename X> void tc_teardown(X &);
 template <int M, int N, int K, typename Ep>
 void tc_mm_rows(TcEng &, const float *, int, int, const float *, int, int, Ep);
+template <int M, int N, int K>
+void tc_mma(TcEng &, const float *, int, int, const float *, int, int, bool);
+template <int M, int N, typename Ep>
+void tc_read_elem(TcEng &, Ep);
 template <int M, int N, int K, typename Ep>
 void tc_mm(TcEng &, const float *, int, int, const float *, int, int, Ep);
 
