@@ -18,6 +18,7 @@
 // forward's tensor-core products.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <stdint.h>
 
 #ifdef __CUDACC__
@@ -40,6 +41,7 @@ struct TcEng {
     uint32_t tmem;
     uint32_t used, par;  // bit b: buffer b has a commit; the parity of its last commit
     int next;            // the buffer the next slice goes to
+    float *host_acc;     // host builds: the accumulator ([128][128] fp32)
 };
 
 // Reduction steps per staged slice (16, 32 or 64; M = 128 products take 16), and the staging
@@ -258,18 +260,55 @@ __device__ __forceinline__ void tc_mm(TcEng &e, const float *A, int ars, int acs
     });
 }
 
-#else  // host builds of the kernels instantiate only TC = false: declarations for the parser
+#else  // host builds (the CPU check of the kernels): the same contract, computed in place
 
-template <typename X> void tc_setup(TcEng &, uint8_t *, int, int, X *);
-template <typename X> void tc_teardown(X &);
-template <int M, int N, int K, typename Ep>
-void tc_mm_rows(TcEng &, const float *, int, int, const float *, int, int, Ep);
+// A product on the host: operands rounded to bf16 (nearest even) as the staging rounds them,
+// sums in fp32 in order of increasing k (the tensor core's order within a slice is not
+// specified; either is a valid fp32 sum of the same bf16 products).
+inline float tc_host_bf16(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+template <typename X>
+void tc_setup(TcEng &e, uint8_t *, int, int, X *) {
+    static thread_local float acc[128 * 128];
+    e.host_acc = acc;
+}
+template <typename X>
+void tc_teardown(X &) {}
 template <int M, int N, int K>
-void tc_mma(TcEng &, const float *, int, int, const float *, int, int, bool);
+void tc_mma(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs, bool acc) {
+    for (int m = 0; m < M; ++m)
+        for (int n = 0; n < N; ++n) {
+            float s = acc ? e.host_acc[m * N + n] : 0.f;
+            for (int k = 0; k < K; ++k)
+                s += tc_host_bf16(A[m * ars + k * acs]) * tc_host_bf16(B[k * brs + n * bcs]);
+            e.host_acc[m * N + n] = s;
+        }
+}
 template <int M, int N, typename Ep>
-void tc_read_elem(TcEng &, Ep);
+void tc_read(TcEng &e, Ep ep) {
+    constexpr int kNV = M * N / 512;
+    for (int i = 0; i < M; ++i)
+        for (int j0 = 0; j0 < N; j0 += kNV) {
+            float v[kNV];
+            for (int c = 0; c < kNV; ++c) v[c] = e.host_acc[i * N + j0 + c];
+            ep(i, j0, v);
+        }
+}
+template <int M, int N, typename Ep>
+void tc_read_elem(TcEng &e, Ep ep) {
+    for (int i = 0; i < M; ++i)
+        for (int j = 0; j < N; ++j) ep(i, j, e.host_acc[i * N + j]);
+}
 template <int M, int N, int K, typename Ep>
-void tc_mm(TcEng &, const float *, int, int, const float *, int, int, Ep);
+void tc_mm_rows(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs, Ep ep) {
+    tc_mma<M, N, K>(e, A, ars, acs, B, brs, bcs, false);
+    tc_read<M, N>(e, ep);
+}
+template <int M, int N, int K, typename Ep>
+void tc_mm(TcEng &e, const float *A, int ars, int acs, const float *B, int brs, int bcs, Ep ep) {
+    tc_mma<M, N, K>(e, A, ars, acs, B, brs, bcs, false);
+    tc_read_elem<M, N>(e, ep);
+}
 
 #endif
 

@@ -18,6 +18,7 @@
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
+#include <type_traits>
 #include <vector>
 
 static uint3 threadIdx, blockIdx;
@@ -81,10 +82,13 @@ static void run(const GdnBwdArgs &a) {
     run_blocks([&] { gdn_bwd_prep_kernel<D, Tin>(a); }, nch, prep_smem<D>());
     run_blocks([&] { gdn_bwd_prefix_kernel<D>(a); }, elems, 0);
     run_fstate<D, Tin>(a, bh);
-    run_blocks([&] { gdn_bwd_local_kernel<D, Tin>(a); }, nch, local_smem<D>());
+    // bf16 inputs with D >= 64 take the kernels' tensor-core instantiation, as the library does; on
+    // the host its products are computed in place on bf16-rounded operands (ccq_gdn_bwd_tc.cuh)
+    constexpr bool kTc = std::is_same<Tin, __nv_bfloat16>::value && D >= 64;
+    run_blocks([&] { gdn_bwd_local_kernel<D, Tin, kTc>(a); }, nch, local_smem<D, kTc>());
     run_dstate<D, Tin>(a, bh);
     run_blocks([&] { gdn_bwd_suffix_kernel<D>(a); }, elems, 0);
-    run_blocks([&] { gdn_bwd_kv_kernel<D, Tin>(a); }, nch, kv_smem<D>());
+    run_blocks([&] { gdn_bwd_kv_kernel<D, Tin, kTc>(a); }, nch, kv_smem<D, kTc>());
 }
 
 template <typename Tin>
@@ -136,7 +140,8 @@ extern "C" int gdn_bwd_emu(int D, int bf16, int B, int T, int H, int l2norm, int
                            const float *const *in, const int64_t *t0, float *const *out) {
     if (D == 16) return bf16 ? go<16, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, t0, out)
                              : go<16, float>(B, T, H, l2norm, centered, scale, in, t0, out);
-    if (D == 64 && !bf16) return go<64, float>(B, T, H, l2norm, centered, scale, in, t0, out);
+    if (D == 64) return bf16 ? go<64, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, t0, out)
+                             : go<64, float>(B, T, H, l2norm, centered, scale, in, t0, out);
     return -1;
 }
 
