@@ -142,6 +142,7 @@ extern "C" int gdn_bwd_emu(int D, int bf16, int B, int T, int H, int l2norm, int
                              : go<16, float>(B, T, H, l2norm, centered, scale, in, t0, out);
     if (D == 64) return bf16 ? go<64, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, t0, out)
                              : go<64, float>(B, T, H, l2norm, centered, scale, in, t0, out);
+    if (D == 128 && bf16) return go<128, __nv_bfloat16>(B, T, H, l2norm, centered, scale, in, t0, out);
     return -1;
 }
 

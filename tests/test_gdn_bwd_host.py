@@ -84,6 +84,8 @@ CASES = [
     dict(D=64, B=1, T=65, H=1, seed=10, bf16=True, lam=0.9, states=False),
     dict(D=64, B=1, T=100, H=1, seed=11, bf16=True, opts=dict(centered=False)),
     dict(D=64, B=1, T=70, H=1, seed=12, bf16=True, opts=dict(l2norm=False)),
+    # D = 128: the two-block chains and the M = 128 products
+    dict(D=128, B=1, T=80, H=1, seed=13, bf16=True),
 ]
 
 
